@@ -1,0 +1,256 @@
+/*
+ * CPU oracle for the sparse contact operators of "ECO: Efficient Human-Contact
+ * Representation for Human-Scene Interaction".
+ *
+ * TEST INFRASTRUCTURE ONLY. This file is the plain, slow reference that the
+ * CUDA path is checked against. Only the tests, the smoke check and the
+ * benchmark's CPU-baseline leg may load it; the product path never does.
+ * It shares no code, header, table or helper with the CUDA library.
+ *
+ * Arithmetic: every sum is accumulated in fp64 in the order the definition
+ * reads (spiral slot, then input channel). bf16 inputs are widened exactly;
+ * outputs are rounded once, from fp64, to the storage type (fp32, or bf16
+ * round-to-nearest-even). The fp64 value before that rounding is also
+ * returned so tests can apply tolerances against it.
+ *
+ * Functions (each cites the passage it follows):
+ *   hco_mask_compact        decomposition into (C', S') coordinates, Eq. 2,
+ *                           plus the inverse map idx() of Eq. 4
+ *   hco_sparse_spiral_conv  sparse convolution, Eqs. 4-5, with the spiral
+ *                           neighbourhood of the POSA spiral blocks (Fig. 2)
+ *                           and the activation of Eq. 10
+ *   hco_dense_spiral_conv   the same layer on every vertex, no mask (the dense
+ *                           operator the sparse one replaces, Sec. 3.2)
+ *   hco_sparse_linear       linear layer on compact rows, Eq. 6
+ *   hco_scatter_dense       inverse of the decomposition: compact rows back
+ *                           into a dense [B, V, C] tensor
+ *   hco_bf16_round          fp64 -> bf16 rounding (storage format)
+ *
+ * Parity status: compaction, conv, dense conv, linear and scatter are pinned
+ * by tests against library routines (numpy.nonzero, numpy matmul), closed
+ * forms, hand-worked cases and brute force (tests/test_oracle_pins.py). The
+ * paper prints no numeric worked example for any operator.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#define HCO_F32 0
+#define HCO_BF16 1
+#define HCO_ACT_NONE 0
+#define HCO_ACT_ELU 1
+#define HCO_ACT_RELU 2
+#define HCO_LAYOUT_DENSE 0
+#define HCO_LAYOUT_COMPACT 1
+
+/* ---------------------------------------------------------------- dtypes */
+
+/* bf16 is the upper half of an IEEE binary32 pattern: widening is exact. */
+static double bf16_to_double(uint16_t h) {
+    uint32_t u = (uint32_t)h << 16;
+    float f;
+    memcpy(&f, &u, sizeof f);
+    return (double)f;
+}
+
+/* fp64 -> bf16, round to nearest, ties to even, from the format's
+ * definition: bf16 has 8 significant bits for normal numbers (exponent
+ * range of binary32) and a fixed quantum of 2^-133 below 2^-126. The value
+ * is scaled by its quantum (exact: a power of two), rounded to an integer
+ * with nearbyint (default mode: nearest-even), and scaled back; the result
+ * is a bf16 number, so converting it to binary32 is exact and its upper
+ * 16 bits are the answer. Overflow gives infinity; NaN stays NaN. */
+uint16_t hco_bf16_round(double x) {
+    float f;
+    uint32_t u;
+    if (isnan(x)) return (uint16_t)0x7FC0;
+    if (x == 0.0 || isinf(x)) {
+        f = (float)x;
+        memcpy(&u, &f, sizeof u);
+        return (uint16_t)(u >> 16);
+    }
+    int e;
+    frexp(x, &e); /* |x| in [2^(e-1), 2^e) */
+    int qexp = e - 8;       /* quantum for 8 significant bits */
+    if (qexp < -133) qexp = -133; /* subnormal range: fixed quantum */
+    double n = nearbyint(ldexp(x, -qexp));
+    double r = ldexp(n, qexp);
+    f = (float)r; /* exact, or +-inf past the largest bf16 */
+    memcpy(&u, &f, sizeof u);
+    return (uint16_t)(u >> 16);
+}
+
+static double load_elem(const void* p, int dtype, int64_t i) {
+    if (dtype == HCO_F32) return (double)((const float*)p)[i];
+    return bf16_to_double(((const uint16_t*)p)[i]);
+}
+
+static void store_elem(void* p, int dtype, int64_t i, double v) {
+    if (dtype == HCO_F32)
+        ((float*)p)[i] = (float)v;
+    else
+        ((uint16_t*)p)[i] = hco_bf16_round(v);
+}
+
+/* Activation of Eq. 10; ELU with alpha = 1. */
+static double activate(double z, int act) {
+    if (act == HCO_ACT_ELU) return z > 0.0 ? z : expm1(z);
+    if (act == HCO_ACT_RELU) return z > 0.0 ? z : 0.0;
+    return z;
+}
+
+/* ----------------------------------------------------------- compaction */
+
+/* Eq. 2: drop the zero rows of the masked tensor. Row (b, v) is kept iff
+ * mask[b, v] != 0; kept rows are listed in ascending (b, v) order as the
+ * coordinate matrix C' (frame index b, vertex index v). row_of[b, v] is the
+ * position of (b, v) in C' or -1: this is idx() of Eq. 4. offsets[b] counts
+ * the kept rows of frames before b, so rows of frame b are
+ * [offsets[b], offsets[b+1]) (the "i : C[i][0] = b" ranges of Eqs. 7-8).
+ * Returns N', the number of kept rows. */
+int64_t hco_mask_compact(const uint8_t* mask, int64_t B, int64_t V,
+                         int32_t* coords, int32_t* row_of, int32_t* offsets) {
+    int64_t n = 0;
+    for (int64_t b = 0; b < B; ++b) {
+        offsets[b] = (int32_t)n;
+        for (int64_t v = 0; v < V; ++v) {
+            if (mask[b * V + v] != 0) {
+                coords[2 * n + 0] = (int32_t)b;
+                coords[2 * n + 1] = (int32_t)v;
+                row_of[b * V + v] = (int32_t)n;
+                ++n;
+            } else {
+                row_of[b * V + v] = -1;
+            }
+        }
+    }
+    offsets[B] = (int32_t)n;
+    return n;
+}
+
+/* --------------------------------------------------- sparse spiral conv */
+
+/* Eqs. 4-5 on the spiral neighbourhood. For the output row at coordinate
+ * (b, v) = C'[r]:
+ *     acc[o] = sum_{l < L} sum_{c < C_in} S[idx(b, spiral[v][l])][c] * W[l*C_in + c][o]
+ * where a term is present only if spiral[v][l] >= 0 and the neighbour
+ * (b, spiral[v][l]) is an active row (Eq. 4 keeps only kernel taps whose
+ * coordinate is found in C). Slot 0 of the spiral is the vertex itself, the
+ * centre tap of Eq. 4. Then y = act(acc + bias) (Eqs. 6 and 10), and the
+ * output coordinate is the centre coordinate (Eq. 5, first line).
+ *
+ * x_layout DENSE: S row of (b, u) is x[(b*V + u)*C_in ...] (read only when
+ * (b, u) is active); COMPACT: it is x[row_of[b*V + u]*C_in ...].
+ * rows: the output rows to compute (indices into coords), or NULL for
+ * 0..n_rows-1. Output i goes to y_pre[i*C_out ...] (fp64, before rounding)
+ * and y[i*C_out ...] (storage dtype); either may be NULL. */
+void hco_sparse_spiral_conv(const void* x, int x_layout, int dtype,
+                            const int32_t* coords, const int32_t* row_of,
+                            const int64_t* rows, int64_t n_rows,
+                            const int32_t* spiral, int64_t B, int64_t V, int L,
+                            int C_in, int C_out, const void* W, const float* bias,
+                            int act, double* y_pre, void* y, int n_threads) {
+    (void)B;
+#pragma omp parallel for schedule(dynamic, 8) num_threads(n_threads > 0 ? n_threads : 1)
+    for (int64_t i = 0; i < n_rows; ++i) {
+        int64_t r = rows ? rows[i] : i;
+        int64_t b = coords[2 * r + 0];
+        int64_t v = coords[2 * r + 1];
+        double* acc = (double*)calloc((size_t)C_out, sizeof(double));
+        for (int l = 0; l < L; ++l) {
+            int64_t u = spiral[v * L + l];
+            if (u < 0) continue; /* no neighbour in this slot */
+            int64_t j = row_of[b * V + u];
+            if (j < 0) continue; /* neighbour not in C: tap absent */
+            int64_t src = (x_layout == HCO_LAYOUT_DENSE) ? (b * V + u) : j;
+            for (int c = 0; c < C_in; ++c) {
+                double xv = load_elem(x, dtype, src * C_in + c);
+                for (int o = 0; o < C_out; ++o)
+                    acc[o] += xv * load_elem(W, dtype, ((int64_t)l * C_in + c) * C_out + o);
+            }
+        }
+        for (int o = 0; o < C_out; ++o) {
+            double z = acc[o] + (bias ? (double)bias[o] : 0.0);
+            double a = activate(z, act);
+            if (y_pre) y_pre[i * C_out + o] = a;
+            if (y) store_elem(y, dtype, i * C_out + o, a);
+        }
+        free(acc);
+    }
+}
+
+/* ---------------------------------------------------- dense spiral conv */
+
+/* The dense layer the sparse one replaces: every (b, v) of the [B, V] grid
+ * is an output row (row index r = b*V + v), every neighbour slot with
+ * spiral[v][l] >= 0 contributes, no mask is consulted.
+ *     acc[o] = sum_{l < L} sum_{c < C_in} x[b, spiral[v][l], c] * W[l*C_in + c][o]
+ * Written as its own loop so that "sparse == dense on the masked input"
+ * compares two independent codings of the definition. */
+void hco_dense_spiral_conv(const void* x, int dtype, const int64_t* rows, int64_t n_rows,
+                           const int32_t* spiral, int64_t B, int64_t V, int L, int C_in,
+                           int C_out, const void* W, const float* bias, int act,
+                           double* y_pre, void* y, int n_threads) {
+    (void)B;
+#pragma omp parallel for schedule(dynamic, 8) num_threads(n_threads > 0 ? n_threads : 1)
+    for (int64_t i = 0; i < n_rows; ++i) {
+        int64_t r = rows ? rows[i] : i;
+        int64_t b = r / V, v = r % V;
+        double* acc = (double*)calloc((size_t)C_out, sizeof(double));
+        for (int l = 0; l < L; ++l) {
+            int64_t u = spiral[v * L + l];
+            if (u < 0) continue;
+            for (int c = 0; c < C_in; ++c) {
+                double xv = load_elem(x, dtype, (b * V + u) * C_in + c);
+                for (int o = 0; o < C_out; ++o)
+                    acc[o] += xv * load_elem(W, dtype, ((int64_t)l * C_in + c) * C_out + o);
+            }
+        }
+        for (int o = 0; o < C_out; ++o) {
+            double a = activate(acc[o] + (bias ? (double)bias[o] : 0.0), act);
+            if (y_pre) y_pre[i * C_out + o] = a;
+            if (y) store_elem(y, dtype, i * C_out + o, a);
+        }
+        free(acc);
+    }
+}
+
+/* -------------------------------------------------------- sparse linear */
+
+/* Eq. 6, row-wise: y_i = act(s_i^T W_l + b) for every compact row i; the
+ * coordinates are unchanged. W_l is [C_in, C_out] row-major. */
+void hco_sparse_linear(const void* x, int dtype, const int64_t* rows, int64_t n_rows,
+                       int C_in, int C_out, const void* W, const float* bias, int act,
+                       double* y_pre, void* y, int n_threads) {
+#pragma omp parallel for schedule(dynamic, 8) num_threads(n_threads > 0 ? n_threads : 1)
+    for (int64_t i = 0; i < n_rows; ++i) {
+        int64_t r = rows ? rows[i] : i;
+        for (int o = 0; o < C_out; ++o) {
+            double acc = 0.0;
+            for (int c = 0; c < C_in; ++c)
+                acc += load_elem(x, dtype, r * C_in + c) * load_elem(W, dtype, (int64_t)c * C_out + o);
+            double a = activate(acc + (bias ? (double)bias[o] : 0.0), act);
+            if (y_pre) y_pre[i * C_out + o] = a;
+            if (y) store_elem(y, dtype, i * C_out + o, a);
+        }
+    }
+}
+
+/* ------------------------------------------------------------- scatter */
+
+/* Inverse of the decomposition (Eq. 2): compact row n goes back to dense
+ * position coords[n] = (b, v). With zero_fill, every dense row first
+ * becomes zero, so inactive rows read 0 (the masked tensor of Eq. 1);
+ * without it they are left as they were. Elements are copied bit for bit. */
+void hco_scatter_dense(const void* y, int elem_bytes, const int32_t* coords, int64_t count,
+                       int64_t B, int64_t V, int C, int zero_fill, void* out) {
+    const unsigned char* src = (const unsigned char*)y;
+    unsigned char* dst = (unsigned char*)out;
+    int64_t row_bytes = (int64_t)C * elem_bytes;
+    if (zero_fill) memset(dst, 0, (size_t)(B * V * row_bytes));
+    for (int64_t n = 0; n < count; ++n) {
+        int64_t b = coords[2 * n + 0], v = coords[2 * n + 1];
+        memcpy(dst + (b * V + v) * row_bytes, src + n * row_bytes, (size_t)row_bytes);
+    }
+}

@@ -1,0 +1,369 @@
+"""Pins for the CPU oracle: each check ties the oracle to something other than
+itself (a library routine, a closed form, a hand-worked case, brute force or an
+invariant the paper's definitions fix), chosen so that a plausible mistake
+(a dropped term, a wrong index, a transposed operand, a wrong sign) fails at
+least one of them. Planted-mistake tests at the end show that it does."""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2608_09388_gb300 import inputs
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "octahedron.json")
+ACT = {"none": oracle.ACT_NONE, "elu": oracle.ACT_ELU, "relu": oracle.ACT_RELU}
+
+
+# --------------------------------------------------------------- compaction
+
+def check_compact_vs_nonzero(mask):
+    """Decomposition (Eq. 2) against numpy's row-major nonzero listing."""
+    coords, row_of, offsets, n = oracle.mask_compact(mask)
+    nz = np.argwhere(mask != 0).astype(np.int32)
+    assert n == nz.shape[0]
+    np.testing.assert_array_equal(coords, nz)
+    ref_row = np.full(mask.shape, -1, dtype=np.int32)
+    ref_row[nz[:, 0], nz[:, 1]] = np.arange(n, dtype=np.int32)
+    np.testing.assert_array_equal(row_of, ref_row)
+    ref_off = np.concatenate([[0], np.cumsum((mask != 0).sum(axis=1))]).astype(np.int32)
+    np.testing.assert_array_equal(offsets, ref_off)
+
+
+@pytest.mark.parametrize("B", [1, 7, 64])
+@pytest.mark.parametrize("V", [1, 31, 32, 33, 655])
+@pytest.mark.parametrize("density", [0.0, 0.01, 0.1, 0.5, 1.0])
+def test_compact_matches_numpy_nonzero(B, V, density):
+    rng = np.random.default_rng(B * 1000 + V)
+    check_compact_vs_nonzero(inputs.uniform_mask(rng, B, V, density))
+
+
+def test_compact_nonbinary_bytes_are_active():
+    mask = np.array([[0, 2, 255, 0, 1]], dtype=np.uint8)
+    coords, row_of, offsets, n = oracle.mask_compact(mask)
+    assert n == 3
+    np.testing.assert_array_equal(coords, [[0, 1], [0, 2], [0, 4]])
+
+
+def test_compact_empty_and_full():
+    z = np.zeros((3, 10), np.uint8)
+    coords, row_of, offsets, n = oracle.mask_compact(z)
+    assert n == 0 and (row_of == -1).all() and (offsets == 0).all()
+    o = np.ones((3, 10), np.uint8)
+    coords, row_of, offsets, n = oracle.mask_compact(o)
+    assert n == 30
+    np.testing.assert_array_equal(row_of.ravel(), np.arange(30))
+    np.testing.assert_array_equal(offsets, [0, 10, 20, 30])
+
+
+# ------------------------------------------------------------ golden cases
+
+def _golden():
+    with open(GOLDEN) as f:
+        return json.load(f)
+
+
+def _golden_case_inputs(g, case):
+    sp = np.array(g["spiral_L3"], dtype=np.int32)[:, : case.get("spiral_cols", 3)].copy()
+    for k, row in case.get("spiral_override", {}).items():
+        sp[int(k)] = row
+    x = np.array(case["x"], dtype=np.float32)
+    mask = np.array(case["mask"], dtype=np.uint8)
+    W = np.array(case["W"], dtype=np.float32)
+    b = np.array(case["bias"], dtype=np.float32)
+    return sp, x, mask, W, b
+
+
+def check_golden_cases():
+    g = _golden()
+    for case in g["cases"]:
+        sp, x, mask, W, b = _golden_case_inputs(g, case)
+        coords, row_of, offsets, n = oracle.mask_compact(mask)
+        if "coords" in case:
+            np.testing.assert_array_equal(coords, case["coords"])
+            np.testing.assert_array_equal(row_of, case["row_of"])
+            np.testing.assert_array_equal(offsets, case["offsets"])
+        y_pre, y = oracle.sparse_spiral_conv(x, oracle.LAYOUT_DENSE, coords, row_of, sp, W, b,
+                                             ACT[case["act"]])
+        if "y" in case:
+            np.testing.assert_array_equal(y_pre, np.array(case["y"], dtype=np.float64))
+        if "y_expm1_of" in case:
+            ref = np.vectorize(math.expm1)(np.array(case["y_expm1_of"], dtype=np.float64))
+            np.testing.assert_allclose(y_pre, ref, rtol=1e-15, atol=0)
+        if "y_rows" in case:
+            for k, v in case["y_rows"].items():
+                np.testing.assert_array_equal(y_pre[int(k)], np.array(v, dtype=np.float64))
+    d = g["dense_full_input"]
+    sp = np.array(g["spiral_L3"], dtype=np.int32)
+    y_pre, _ = oracle.dense_spiral_conv(np.array(d["x"], np.float32), sp,
+                                        np.array(d["W"], np.float32), None, oracle.ACT_NONE)
+    np.testing.assert_array_equal(y_pre, np.array(d["y"], dtype=np.float64))
+
+
+def test_golden_octahedron():
+    check_golden_cases()
+
+
+# ------------------------------------------------- conv against library GEMM
+
+def check_conv_vs_gather_matmul(seed=3, B=3, V=40, L=5, C_in=6, C_out=7, density=0.4):
+    """The sparse conv written as an explicit gather (numpy fancy indexing,
+    zero rows for absent taps) followed by numpy's matmul in fp64: the
+    layout [L*C_in, C_out] with row l*C_in + c must agree with the loop."""
+    sp, m, x, W, b = inputs.random_case(seed, B, V, L, C_in, C_out, "f32", density, neg_frac=0.2)
+    coords, row_of, offsets, n = oracle.mask_compact(m)
+    y_pre, _ = oracle.sparse_spiral_conv(x, oracle.LAYOUT_DENSE, coords, row_of, sp, W, b,
+                                         oracle.ACT_NONE)
+    xs = np.concatenate([x.astype(np.float64).reshape(B * V, C_in), np.zeros((1, C_in))])
+    bb, vv = coords[:, 0].astype(np.int64), coords[:, 1].astype(np.int64)
+    u = sp[vv]  # [n, L]
+    act_nb = (u >= 0) & (m[bb[:, None], np.where(u >= 0, u, 0)] != 0)
+    src = np.where(act_nb, bb[:, None] * V + np.where(u >= 0, u, 0), B * V)
+    G = xs[src].reshape(n, L * C_in)  # [n, L*C_in], slot-major
+    ref = np.matmul(G, W.astype(np.float64)) + b.astype(np.float64)
+    np.testing.assert_allclose(y_pre, ref, rtol=1e-12, atol=1e-12)
+
+
+def test_conv_vs_gather_matmul():
+    check_conv_vs_gather_matmul()
+
+
+def test_conv_L1_is_matmul():
+    """L = 1 (only the centre tap): the sparse conv is a plain matmul of the
+    active rows (Eq. 6 special case) -- numpy matmul in fp64."""
+    sp, m, x, W, b = inputs.random_case(5, 4, 50, 1, 9, 11, "f32", 0.3)
+    coords, row_of, offsets, n = oracle.mask_compact(m)
+    y_pre, _ = oracle.sparse_spiral_conv(x, oracle.LAYOUT_DENSE, coords, row_of, sp, W, b,
+                                         oracle.ACT_NONE)
+    xa = x[coords[:, 0], coords[:, 1]].astype(np.float64)
+    np.testing.assert_allclose(y_pre, xa @ W.astype(np.float64) + b, rtol=1e-12, atol=1e-12)
+
+
+def test_linear_is_matmul():
+    rng = np.random.default_rng(11)
+    x = rng.standard_normal((37, 13)).astype(np.float32)
+    W = rng.standard_normal((13, 5)).astype(np.float32)
+    b = rng.standard_normal(5).astype(np.float32)
+    y_pre, _ = oracle.sparse_linear(x, W, b, oracle.ACT_NONE)
+    np.testing.assert_allclose(y_pre, x.astype(np.float64) @ W.astype(np.float64) + b,
+                               rtol=1e-12, atol=1e-12)
+    y_pre, _ = oracle.sparse_linear(x, W, b, oracle.ACT_RELU)
+    np.testing.assert_allclose(y_pre, np.maximum(x.astype(np.float64) @ W.astype(np.float64) + b, 0),
+                               rtol=1e-12, atol=1e-12)
+
+
+# ------------------------------------------------------------- invariants
+
+def check_sparse_equals_dense_on_masked_input(seed=7, B=4, V=60, L=7, C_in=5, C_out=6,
+                                              density=0.3, act=oracle.ACT_ELU):
+    """Eq. 1 + Eq. 5: the sparse layer equals the dense layer applied to the
+    masked input M o X, restricted to active rows (bit-identical in fp64:
+    the dense sum only adds exact zeros)."""
+    sp, m, x, W, b = inputs.random_case(seed, B, V, L, C_in, C_out, "f32", density, neg_frac=0.1)
+    coords, row_of, offsets, n = oracle.mask_compact(m)
+    y_sp, _ = oracle.sparse_spiral_conv(x, oracle.LAYOUT_DENSE, coords, row_of, sp, W, b, act)
+    xm = x * m[:, :, None].astype(np.float32)
+    rows = coords[:, 0].astype(np.int64) * V + coords[:, 1]
+    y_de, _ = oracle.dense_spiral_conv(xm, sp, W, b, act, rows=rows)
+    np.testing.assert_array_equal(y_sp, y_de)
+
+
+def test_sparse_equals_dense_on_masked_input():
+    check_sparse_equals_dense_on_masked_input()
+
+
+def test_all_ones_mask_reproduces_dense():
+    sp, m, x, W, b = inputs.random_case(8, 3, 45, 9, 4, 8, "f32", 1.0)
+    coords, row_of, offsets, n = oracle.mask_compact(m)
+    assert n == 3 * 45
+    y_sp, _ = oracle.sparse_spiral_conv(x, oracle.LAYOUT_DENSE, coords, row_of, sp, W, b,
+                                        oracle.ACT_ELU)
+    y_de, _ = oracle.dense_spiral_conv(x, sp, W, b, oracle.ACT_ELU)
+    np.testing.assert_array_equal(y_sp, y_de)
+
+
+def test_empty_mask_has_no_rows():
+    sp, m, x, W, b = inputs.random_case(9, 2, 30, 4, 3, 3, "f32", 0.0)
+    coords, row_of, offsets, n = oracle.mask_compact(m)
+    assert n == 0
+    y_pre, y = oracle.sparse_spiral_conv(x, oracle.LAYOUT_DENSE, coords, row_of, sp, W, b,
+                                         oracle.ACT_ELU)
+    assert y_pre.shape == (0, 3)
+
+
+def test_compact_input_layout_equals_dense_layout():
+    sp, m, x, W, b = inputs.random_case(10, 3, 50, 6, 4, 5, "f32", 0.35)
+    coords, row_of, offsets, n = oracle.mask_compact(m)
+    xc = x[coords[:, 0], coords[:, 1]]
+    a, _ = oracle.sparse_spiral_conv(x, oracle.LAYOUT_DENSE, coords, row_of, sp, W, b, oracle.ACT_ELU)
+    c, _ = oracle.sparse_spiral_conv(xc, oracle.LAYOUT_COMPACT, coords, row_of, sp, W, b,
+                                     oracle.ACT_ELU)
+    np.testing.assert_array_equal(a, c)
+
+
+def test_brute_force_all_masks_tiny_mesh():
+    """Every one of the 2^8 masks on an 8-vertex mesh: compaction against
+    numpy, sparse conv against the dense layer on the masked input."""
+    V, L = 8, 4
+    sp, _, x, W, b = inputs.random_case(12, 1, V, L, 3, 2, "f32", 0.5, neg_frac=0.15)
+    for bits in range(1 << V):
+        m = np.array([[(bits >> v) & 1 for v in range(V)]], dtype=np.uint8)
+        check_compact_vs_nonzero(m)
+        coords, row_of, offsets, n = oracle.mask_compact(m)
+        y_sp, _ = oracle.sparse_spiral_conv(x, oracle.LAYOUT_DENSE, coords, row_of, sp, W, b,
+                                            oracle.ACT_ELU)
+        y_de, _ = oracle.dense_spiral_conv(x * m[:, :, None], sp, W, b, oracle.ACT_ELU,
+                                           rows=coords[:, 1].astype(np.int64))
+        np.testing.assert_array_equal(y_sp, y_de)
+
+
+def test_stack_equals_dense_stack_remasked():
+    """A 4-layer sparse stack on one mask equals the dense stack with the
+    input re-masked before every layer (fp32 storage, so each layer's stored
+    values agree exactly)."""
+    B, V, L = 3, 64, 9
+    sp, m, x, _, _ = inputs.random_case(13, B, V, L, 16, 1, "f32", 0.2)
+    rng = np.random.default_rng(99)
+    chans = [16, 12, 12, 8, 8]
+    layers = [inputs.Layer("conv", ci, co, oracle.ACT_ELU,
+                           inputs.weights(rng, L * ci, co, "f32"), inputs.bias(co))
+              for ci, co in zip(chans[:-1], chans[1:])]
+    coords, row_of, offsets, n, outs = oracle.encoder(x, m, sp, layers)
+    h = x
+    for ly in layers:
+        _, hy = oracle.dense_spiral_conv(h * m[:, :, None], sp, ly.W, ly.b, ly.act)
+        h = hy.reshape(B, V, -1)
+    act_rows = h[coords[:, 0], coords[:, 1]]
+    np.testing.assert_array_equal(outs[-1][1], act_rows)
+
+
+def test_scatter_matches_numpy_assignment():
+    rng = np.random.default_rng(14)
+    m = inputs.uniform_mask(rng, 3, 20, 0.3)
+    coords, row_of, offsets, n = oracle.mask_compact(m)
+    y = rng.standard_normal((n, 4)).astype(np.float32)
+    prev = rng.standard_normal((3, 20, 4)).astype(np.float32)
+    out = oracle.scatter_dense(y, coords, 3, 20, zero_fill=False, out=prev)
+    ref = prev.copy()
+    ref[coords[:, 0], coords[:, 1]] = y
+    np.testing.assert_array_equal(out, ref)
+    out0 = oracle.scatter_dense(y, coords, 3, 20, zero_fill=True, out=prev)
+    ref0 = np.zeros_like(prev)
+    ref0[coords[:, 0], coords[:, 1]] = y
+    np.testing.assert_array_equal(out0, ref0)
+
+
+# ----------------------------------------------------------- bf16 storage
+
+def check_bf16_round():
+    """fp64 -> bf16 rounding against torch's float32 -> bf16 routine on values
+    exactly representable in float32, and against closed-form cases that a
+    round-through-float32 implementation gets wrong."""
+    import torch
+    rng = np.random.default_rng(15)
+    vals = np.concatenate([
+        rng.standard_normal(4000).astype(np.float32),
+        (rng.standard_normal(1000) * 1e-39).astype(np.float32),  # subnormal range
+        (rng.standard_normal(1000) * 1e38).astype(np.float32),
+        np.array([0.0, -0.0, 1.0, -1.0, 3.0e38, 3.3961776e38, 1e-45], dtype=np.float32),
+        # exact ties: lower 16 bits 0x8000
+        (np.arange(1, 2000, dtype=np.uint32) << 16 | 0x8000).view(np.float32),
+    ])
+    ref = torch.from_numpy(vals).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    got = np.array([oracle.bf16_round(float(v)) for v in vals], dtype=np.uint16)
+    finite = np.isfinite(vals)
+    np.testing.assert_array_equal(got[finite], ref[finite])
+    # 1 + 2^-8 is a tie -> even (1.0); a hair above must round up to 1 + 2^-7.
+    assert oracle.bf16_round(1.0 + 2.0 ** -8) == 0x3F80
+    assert oracle.bf16_round(1.0 + 2.0 ** -8 + 2.0 ** -30) == 0x3F81
+    assert oracle.bf16_round(-(1.0 + 2.0 ** -8 + 2.0 ** -30)) == 0xBF81
+    assert oracle.bf16_round(1.0 + 3 * 2.0 ** -8) == 0x3F82  # tie, odd -> up to even
+
+
+def test_bf16_round():
+    check_bf16_round()
+
+
+def test_bf16_conv_rounds_once_from_fp64():
+    sp, m, x, W, b = inputs.random_case(16, 2, 40, 5, 8, 8, "bf16", 0.5)
+    coords, row_of, offsets, n = oracle.mask_compact(m)
+    y_pre, y = oracle.sparse_spiral_conv(x, oracle.LAYOUT_DENSE, coords, row_of, sp, W, b,
+                                         oracle.ACT_ELU)
+    want = np.array([oracle.bf16_round(v) for v in y_pre.ravel()], np.uint16).reshape(y.shape)
+    np.testing.assert_array_equal(y, want)
+    # bf16 inputs are widened exactly: same as the f32 oracle on widened data
+    xf = inputs.bf16_bits_to_f32(x)
+    Wf = inputs.bf16_bits_to_f32(W)
+    y32, _ = oracle.sparse_spiral_conv(xf, oracle.LAYOUT_DENSE, coords, row_of, sp, Wf, b,
+                                       oracle.ACT_ELU)
+    np.testing.assert_array_equal(y_pre, y32)
+
+
+# ------------------------------------------------------ workload statistics
+
+def test_workload_statistics():
+    """The synthetic workloads reproduce the paper's statistics: 655 vertices,
+    about 10% active at a 90% sparsity ratio (Table 4: 66 of 655)."""
+    w = inputs.make_workload("encoder655_bf16")
+    d = w.masks[0].mean()
+    assert w.V == 655 and abs(d - 0.1) < 0.01
+    sp = w.spiral
+    assert (sp[:, 0] == np.arange(655)).all()
+    assert ((sp >= 0) & (sp < 655)).all()
+    # neighbours are distinct from the vertex and ordered by distance
+    p = w.points
+    d2 = ((p[sp[:, 1:]] - p[:, None, :]) ** 2).sum(-1)
+    assert (np.diff(d2, axis=1) >= 0).all()
+    assert (sp[:, 1:] != np.arange(655)[:, None]).all()
+
+
+# ----------------------------------------------------- planted mistakes
+
+MUTANTS = {
+    "transposed weight index": ("acc[o] += xv * load_elem(W, dtype, ((int64_t)l * C_in + c) * C_out + o);",
+                                "acc[o] += xv * load_elem(W, dtype, ((int64_t)c * L + l) * C_out + o);"),
+    "inactive neighbour not skipped": ("if (j < 0) continue; /* neighbour not in C: tap absent */",
+                                       "/* dropped */"),
+    "ELU sign": ("return z > 0.0 ? z : expm1(z);", "return z > 0.0 ? z : expm1(-z);"),
+    "compaction order": ("for (int64_t b = 0; b < B; ++b) {\n        offsets[b] = (int32_t)n;\n        for (int64_t v = 0; v < V; ++v) {",
+                         "for (int64_t b = B - 1; b >= 0; --b) {\n        offsets[b] = (int32_t)n;\n        for (int64_t v = 0; v < V; ++v) {"),
+    "bf16 rounded through float32": ("double n = nearbyint(ldexp(x, -qexp));",
+                                     "double n = nearbyint(ldexp((double)(float)x, -qexp));"),
+    "centre tap dropped": ("for (int l = 0; l < L; ++l) {\n            int64_t u = spiral[v * L + l];\n            if (u < 0) continue; /* no neighbour in this slot */",
+                           "for (int l = 1; l < L; ++l) {\n            int64_t u = spiral[v * L + l];\n            if (u < 0) continue; /* no neighbour in this slot */"),
+}
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_planted_mistake_is_caught(name, tmp_path, monkeypatch):
+    """Compile a copy of the oracle with one plausible mistake planted and
+    check that the pins above reject it."""
+    import ctypes
+    import subprocess
+    src = open(oracle._SRC).read()
+    old, new = MUTANTS[name]
+    assert src.count(old) >= 1, name
+    mut = tmp_path / "mut.c"
+    mut.write_text(src.replace(old, new, 1))  # first occurrence: the sparse operator
+    so = tmp_path / "libmut.so"
+    subprocess.run(["gcc", "-O1", "-std=c11", "-fPIC", "-shared", "-fopenmp", str(mut), "-o",
+                    str(so), "-lm"], check=True)
+    good = oracle._load()
+    lib = ctypes.CDLL(str(so))
+    for fn in ("hco_mask_compact", "hco_sparse_spiral_conv", "hco_dense_spiral_conv",
+               "hco_sparse_linear", "hco_scatter_dense", "hco_bf16_round"):
+        getattr(lib, fn).argtypes = getattr(good, fn).argtypes
+        getattr(lib, fn).restype = getattr(good, fn).restype
+    monkeypatch.setattr(oracle, "_lib", lib)
+    checks = [check_golden_cases, check_conv_vs_gather_matmul,
+              lambda: check_compact_vs_nonzero(inputs.uniform_mask(np.random.default_rng(1), 5, 20, 0.3)),
+              check_bf16_round]
+    caught = 0
+    for chk in checks:
+        try:
+            chk()
+        except AssertionError:
+            caught += 1
+    assert caught >= 1, f"planted mistake '{name}' passed every pin"
