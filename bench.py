@@ -1,0 +1,657 @@
+#!/usr/bin/env python3
+"""Benchmark of the sparse spiral-conv hot path on one GB300 (or N replicas).
+
+One step = one pass of the hot path over one batch of the 10475-vertex
+workload (B = 32 frames, spiral length L = 12, 64 -> 128 channels, bf16,
+clustered contact masks at ~5% density):
+    hc_mask_compact           mask -> coords, row_of, offsets, count
+    hc_sparse_spiral_conv_fwd gather + tcgen05 contraction + bias + ELU
+    hc_scatter_dense          compact rows -> dense [B, V, 128]
+Inputs are resident in HBM; every step reads its own input set (mask and
+features) from a rotation whose total size is more than twice the L2, so
+consecutive steps do not hit in L2. The timed steps are replayed from CUDA
+graphs captured on the bench stream.
+
+Printed (one JSON line, rank 0): active rows/s over all ranks, the roofline
+of the dominant kernel (the tensor-core conv, timed alone with CUDA events),
+the CPU oracle as a reported baseline, an end-to-end number through the
+C-ABI with host buffers, the dense operator and the speed-up over it, the
+density sweep, and the SM clocks sampled around the timed region.
+
+--impl reference times the CPU oracle (test infrastructure, plain C, fp64)
+on bounded samples of the same workload; it is the only other place this
+script runs the oracle.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+METRIC = "active vertex-rows/s & % roofline, sparse spiral-conv layer; speed-up vs dense"
+WORKLOAD = "layer10475_bf16"
+
+
+def parse_args():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=400)
+    p.add_argument("--warmup", type=int, default=10)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--no-extras", action="store_true", help="skip the density sweep")
+    p.add_argument("--clocks-csv", default=None, help="also write the raw clock samples here")
+    p.add_argument("--e2e-steps", type=int, default=30)
+    return p.parse_args()
+
+
+# ----------------------------------------------------------------- helpers
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        d = json.load(open(path))
+        return {"hbm_gbs": d["hbm_gbs"], "bf16_tflops": d["bf16_tflops"],
+                "bf16_tflops_sustained": d.get("bf16_tflops_sustained"), "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+            "source": "fallback"}
+
+
+def kernel_source_hash():
+    h = hashlib.sha256()
+    for f in ("conv_tc.cu", "hc_internal.cuh"):
+        h.update(open(os.path.join(ROOT, "paper_2608_09388_gb300", "csrc", f), "rb").read())
+    return h.hexdigest()[:16]
+
+
+def ncu_traffic():
+    """DRAM bytes per launch of the conv kernel from the committed ncu summary,
+    or None if the summary is missing or the kernel source changed since."""
+    path = os.path.join(ROOT, "profiles", "conv_tc_layer10475_bf16.json")
+    if not os.path.exists(path):
+        return None, None
+    d = json.load(open(path))
+    if d.get("kernel_source_hash") != kernel_source_hash():
+        return None, d.get("kernel_source_hash")
+    return d.get("dram_bytes_per_launch"), d.get("kernel_source_hash")
+
+
+class ClockSampler:
+    """nvidia-smi samples (every 200 ms) while the load runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index, csv_path=None):
+        self.proc = None
+        self.out = None
+        self.csv_path = csv_path
+        sel = []
+        try:
+            import torch
+            u = str(torch.cuda.get_device_properties(device_index).uuid)
+            sel = ["-i", u if u.startswith("GPU-") else "GPU-" + u]
+        except Exception:
+            vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+            if vis:
+                sel = ["-i", vis.split(",")[device_index]]
+        self.cmd = ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                    "-lms", "200", *sel]
+
+    def start(self):
+        import tempfile
+        self.out = tempfile.TemporaryFile(mode="w+")
+        try:
+            self.proc = subprocess.Popen(self.cmd, stdout=self.out, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.out.seek(0)
+        text = self.out.read()
+        if self.csv_path:
+            with open(self.csv_path, "w") as f:
+                f.write(self.FIELDS + "\n" + text)
+        sm, mx, power, reasons = [], [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in text.strip().splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+                power.append(float(parts[3]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
+                "power_w_max": max(power) if power else None, "reasons": sorted(reasons)}
+
+
+# ----------------------------------------------------------------- our arm
+
+class LayerSet:
+    """One rotation entry: a batch's mask and features plus its outputs."""
+
+
+def build_sets(torch, w, R, seed_base, dev):
+    """Input set 0 is the seeded workload itself; sets 1..R-1 use the same
+    recipe with their own seeds (masks from numpy, features drawn on the
+    device from a seeded torch generator)."""
+    from paper_2608_09388_gb300 import inputs
+    ly = w.layers[0]
+    B, V = w.B, w.V
+    sets = []
+    for i in range(R):
+        s = LayerSet()
+        if i == 0:
+            mask = w.masks[0]
+            x = torch.from_numpy(w.x.view(np.int16)).view(torch.bfloat16).to(dev)
+        else:
+            rng = np.random.default_rng(seed_base + 7919 * i)
+            mask = inputs.clustered_mask(rng, w.points, B, 8, 0.05)
+            g = torch.Generator(device=dev)
+            g.manual_seed(seed_base + 104729 * i)
+            x = torch.randn((B, V, ly.C_in), generator=g, device=dev,
+                            dtype=torch.float32).to(torch.bfloat16)
+        s.mask_np = mask
+        s.rows = int(np.count_nonzero(mask))
+        s.mask = torch.from_numpy(mask).to(dev)
+        s.x = x
+        s.coords = torch.empty((B * V, 2), dtype=torch.int32, device=dev)
+        s.row_of = torch.empty((B, V), dtype=torch.int32, device=dev)
+        s.offs = torch.empty((B + 1,), dtype=torch.int32, device=dev)
+        s.count = torch.empty((1,), dtype=torch.int32, device=dev)
+        s.y = torch.empty((B * V, ly.C_out), dtype=torch.bfloat16, device=dev)
+        s.out = torch.zeros((B, V, ly.C_out), dtype=torch.bfloat16, device=dev)
+        sets.append(s)
+    return sets
+
+
+def run_ours(args, rank, world, local_rank):
+    import torch
+
+    from paper_2608_09388_gb300 import build as hc_build
+    from paper_2608_09388_gb300 import hc, inputs
+
+    if rank == 0 or not os.path.exists(os.path.join(ROOT, "paper_2608_09388_gb300", "_build",
+                                                    "libhc.so")):
+        hc_build.build()
+    if world > 1:
+        torch.distributed.barrier()
+    hc.load_library()
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    props = torch.cuda.get_device_properties(dev)
+    l2 = int(getattr(props, "L2_cache_size", 0) or 0) or 126 * 2 ** 20
+
+    w = inputs.make_workload(WORKLOAD)
+    ly = w.layers[0]
+    B, V, L = w.B, w.V, w.L
+    set_bytes = B * V * (1 + 2 * ly.C_in)
+    R = max(4, math.ceil(2.5 * l2 / set_bytes))
+    sets = build_sets(torch, w, R, inputs.SEEDS[WORKLOAD] + 1000 * rank, dev)
+    spiral = torch.from_numpy(w.spiral).to(dev)
+    Wt = torch.from_numpy(ly.W.view(np.int16)).view(torch.bfloat16).to(dev)
+    bias = torch.from_numpy(ly.b).to(dev)
+    stream = torch.cuda.Stream(device=dev)
+
+    def step(s):
+        hc.hc_mask_compact(s.mask, s.coords, s.row_of, s.offs, s.count, stream)
+        hc.hc_sparse_spiral_conv_fwd(s.x, hc.HC_LAYOUT_DENSE, s.coords, s.row_of, s.count, spiral,
+                                     B, V, Wt, bias, ly.act, s.y, stream)
+        hc.hc_scatter_dense(s.y, s.coords, s.row_of, s.count, B, V, 0, s.out, stream)
+
+    def conv_only(s):
+        hc.hc_sparse_spiral_conv_fwd(s.x, hc.HC_LAYOUT_DENSE, s.coords, s.row_of, s.count, spiral,
+                                     B, V, Wt, bias, ly.act, s.y, stream)
+
+    def dense_only(s):
+        hc.hc_spiral_conv_fwd(s.x, spiral, Wt, bias, ly.act, s.dense, stream)
+
+    kernels_per_step = 2 + (1 if (B * V + 4095) // 4096 > 1024 else 0) + 1 + 1
+
+    # W warm-up steps, then one priming pass over every input set (both
+    # eager, untimed; they also set up the library's per-stream workspace).
+    with torch.cuda.stream(stream):
+        for i in range(args.warmup):
+            step(sets[i % R])
+        for s in sets:
+            step(s)
+    torch.cuda.synchronize(dev)
+    st = hc.hc_get_device_status(stream)
+    if st != hc.HC_OK:
+        raise RuntimeError(f"device status {hc.STATUS_NAMES.get(st)} after warm-up")
+    for s in sets:
+        assert int(s.count.item()) == s.rows, "active-row count differs from the mask"
+
+    def capture(fn, idx):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for i in idx:
+                fn(sets[i])
+        return g
+
+    K = args.steps
+    g_full = capture(step, range(R))
+    g_rem = capture(step, range(K % R)) if K % R else None
+
+    rows_per_round = sum(s.rows for s in sets)
+    rows_timed = (K // R) * rows_per_round + sum(sets[i].rows for i in range(K % R))
+
+    def timed_region():
+        """Exactly K steps, bracketed by a barrier and a synchronize."""
+        if world > 1:
+            torch.distributed.barrier()
+        torch.cuda.synchronize(dev)
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            for _ in range(K // R):
+                g_full.replay()
+            if g_rem is not None:
+                g_rem.replay()
+            e1.record(stream)
+        torch.cuda.synchronize(dev)
+        if world > 1:
+            torch.distributed.barrier()
+        return e0.elapsed_time(e1)
+
+    # The timed region is repeated (at least 3 times, and until a second has
+    # passed) while nvidia-smi samples the clocks; ms is the median repeat.
+    sampler = ClockSampler(local_rank, args.clocks_csv if rank == 0 else None)
+    sampler.start()
+    reps_ms = []
+    t_start = time.perf_counter()
+    while len(reps_ms) < 3 or time.perf_counter() - t_start < 1.0:
+        reps_ms.append(timed_region())
+        if world > 1:
+            # every rank must agree on whether to run another repeat
+            flag = torch.tensor([1 if time.perf_counter() - t_start < 1.0 else 0],
+                                device=dev)
+            torch.distributed.all_reduce(flag, op=torch.distributed.ReduceOp.MAX)
+            if len(reps_ms) >= 3 and int(flag.item()) == 0:
+                break
+    clocks = sampler.stop()
+    ms = statistics.median(reps_ms)
+
+    # Dominant kernel alone: the tensor-core conv over the same rotation.
+    g_conv = capture(conv_only, range(R))
+    reps = max(1, 200 // R)
+    with torch.cuda.stream(stream):
+        g_conv.replay()
+        c0 = torch.cuda.Event(enable_timing=True)
+        c1 = torch.cuda.Event(enable_timing=True)
+        c0.record(stream)
+        for _ in range(reps):
+            g_conv.replay()
+        c1.record(stream)
+    torch.cuda.synchronize(dev)
+    conv_ms = c0.elapsed_time(c1) / (reps * R)
+    mean_rows = rows_per_round / R
+    flops_per_launch = 2.0 * L * ly.C_in * ly.C_out * mean_rows
+    pk = peaks()
+    achieved = flops_per_launch / (conv_ms * 1e-3) / 1e12
+    traffic, khash = ncu_traffic()
+
+    # Dense operator (the speed-up denominator): our dense kernel and torch's
+    # gather + matmul, the faster of the two.
+    for s in sets:
+        s.dense = torch.empty((B, V, ly.C_out), dtype=torch.bfloat16, device=dev)
+    g_dense = capture(dense_only, range(R))
+    with torch.cuda.stream(stream):
+        g_dense.replay()
+        d0 = torch.cuda.Event(enable_timing=True)
+        d1 = torch.cuda.Event(enable_timing=True)
+        d0.record(stream)
+        for _ in range(3):
+            g_dense.replay()
+        d1.record(stream)
+    torch.cuda.synchronize(dev)
+    dense_ms = d0.elapsed_time(d1) / (3 * R)
+    torch_dense_ms = time_torch_dense(torch, sets, w, Wt, bias, stream, dev)
+    best_dense = min(dense_ms, torch_dense_ms)
+    for s in sets:
+        del s.dense
+    torch.cuda.empty_cache()
+
+    e2e = measure_e2e(torch, hc, sets, w, spiral, Wt, bias, stream, dev, args.e2e_steps)
+
+    sweep = None
+    if not args.no_extras and rank == 0:
+        sweep = run_sweep(torch, hc, dev, stream)
+
+    # Aggregate over ranks: rows summed, time = max over ranks.
+    tot_rows, max_ms = float(rows_timed), ms
+    if world > 1:
+        t = torch.tensor([tot_rows, ms], dtype=torch.float64, device=dev)
+        r_sum = t.clone()
+        torch.distributed.all_reduce(r_sum, op=torch.distributed.ReduceOp.SUM)
+        r_max = t.clone()
+        torch.distributed.all_reduce(r_max, op=torch.distributed.ReduceOp.MAX)
+        tot_rows, max_ms = float(r_sum[0].item()), float(r_max[1].item())
+    if rank != 0:
+        return None
+
+    cpu = cpu_baseline(w)
+    value = tot_rows / (max_ms * 1e-3)
+    line = {
+        "metric": METRIC,
+        "value": value,
+        "unit": "rows/s",
+        "n_gpus": world,
+        "steps": K,
+        "warmup": args.warmup,
+        "ms_per_step": max_ms / K,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic",
+        "impl": "ours",
+        "config": {
+            "workload": WORKLOAD,
+            "B": B, "V": V, "L": L, "C_in": ly.C_in, "C_out": ly.C_out, "act": "elu",
+            "mask": "clustered, 8 caps per frame, ~5% active",
+            "active_rows_per_step": mean_rows,
+            "rotation_sets": R,
+            "launches_before_timed": (args.warmup + R) * kernels_per_step,
+            "step": "hc_mask_compact + hc_sparse_spiral_conv_fwd + hc_scatter_dense",
+            "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+            "l2": f"{R} rotating input sets of {set_bytes / 2**20:.1f} MiB "
+                  f"({R * set_bytes / 2**20:.0f} MiB > 2x L2 {l2 / 2**20:.0f} MiB)",
+            "timing": f"CUDA events around CUDA-graph replays on the bench stream; median of "
+                      f"{len(reps_ms)} repeats of exactly {K} steps",
+        },
+        "roofline": {
+            "kernel": "conv_tc_kernel<128> (sparse spiral conv, tcgen05)",
+            "bound": "tensor",
+            "achieved": achieved,
+            "peak": pk["bf16_tflops"],
+            "unit": "TFLOP/s",
+            "frac": achieved / pk["bf16_tflops"],
+            "peak_source": f"{pk['source']} bf16 burst",
+            "traffic": traffic,
+            "flops_per_launch": flops_per_launch,
+            "launch_us": conv_ms * 1e3,
+            "kernel_source_hash": khash if traffic is not None else kernel_source_hash(),
+        },
+        "dense": {
+            "hc_spiral_conv_fwd_us": dense_ms * 1e3,
+            "torch_gather_matmul_us": torch_dense_ms * 1e3,
+            "sparse_conv_us": conv_ms * 1e3,
+            "sparse_step_us": max_ms / K * 1e3,
+            "speedup_conv_vs_dense": best_dense / conv_ms,
+            "speedup_step_vs_dense": best_dense / (max_ms / K),
+            "dense_tflops": 2.0 * L * ly.C_in * ly.C_out * B * V / (dense_ms * 1e-3) / 1e12,
+        },
+        "cpu_baseline": cpu,
+        "e2e": e2e,
+        "gpu_launches": K * kernels_per_step,
+        "clocks": clocks,
+    }
+    if sweep is not None:
+        line["sweep"] = sweep
+    return line
+
+
+def time_torch_dense(torch, sets, w, Wt, bias, stream, dev):
+    """torch reference of the dense layer: gather the spiral rows
+    (index_select), one bf16 matmul, bias, ELU."""
+    ly = w.layers[0]
+    B, V, L = w.B, w.V, w.L
+    idx = torch.from_numpy(w.spiral.astype(np.int64).ravel()).to(dev)
+
+    def run(s):
+        g = s.x.index_select(1, idx).view(B * V, L * ly.C_in)
+        return torch.nn.functional.elu(torch.addmm(bias.to(torch.bfloat16), g, Wt))
+
+    with torch.cuda.stream(stream):
+        for s in sets[:2]:
+            run(s)
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        t0.record(stream)
+        for s in sets:
+            run(s)
+        t1.record(stream)
+    torch.cuda.synchronize(dev)
+    return t0.elapsed_time(t1) / len(sets)
+
+
+def measure_e2e(torch, hc, sets, w, spiral, Wt, bias, stream, dev, steps):
+    """Same metric through the C-ABI with host buffers: every step copies its
+    mask and features from pinned host memory, runs the hot path, and reads
+    back the count, the coordinates and the compact output rows."""
+    ly = w.layers[0]
+    B, V = w.B, w.V
+    host = []
+    for s in sets:
+        host.append((s.mask.cpu().pin_memory(), s.x.cpu().pin_memory()))
+    mask_d = torch.empty_like(sets[0].mask)
+    x_d = torch.empty_like(sets[0].x)
+    s0 = sets[0]
+    cnt_h = torch.empty((1,), dtype=torch.int32).pin_memory()
+    y_h = torch.empty((B * V, ly.C_out), dtype=torch.bfloat16).pin_memory()
+    c_h = torch.empty((B * V, 2), dtype=torch.int32).pin_memory()
+    h2d = d2h = 0
+    rows = 0
+
+    def one(i):
+        nonlocal h2d, d2h, rows
+        mh, xh = host[i % len(host)]
+        mask_d.copy_(mh, non_blocking=True)
+        x_d.copy_(xh, non_blocking=True)
+        hc.hc_mask_compact(mask_d, s0.coords, s0.row_of, s0.offs, s0.count, stream)
+        hc.hc_sparse_spiral_conv_fwd(x_d, hc.HC_LAYOUT_DENSE, s0.coords, s0.row_of, s0.count,
+                                     spiral, B, V, Wt, bias, ly.act, s0.y, stream)
+        hc.hc_scatter_dense(s0.y, s0.coords, s0.row_of, s0.count, B, V, 0, s0.out, stream)
+        cnt_h.copy_(s0.count, non_blocking=True)
+        stream.synchronize()
+        n = int(cnt_h[0])
+        y_h[:n].copy_(s0.y[:n], non_blocking=True)
+        c_h[:n].copy_(s0.coords[:n], non_blocking=True)
+        stream.synchronize()
+        h2d += mh.numel() + xh.numel() * 2
+        d2h += 4 + n * 8 + n * ly.C_out * 2
+        rows += n
+
+    with torch.cuda.stream(stream):
+        for i in range(2):
+            one(i)
+        h2d = d2h = rows = 0
+        torch.cuda.synchronize(dev)
+        t0 = time.perf_counter()
+        for i in range(steps):
+            one(i)
+        torch.cuda.synchronize(dev)
+        dt = time.perf_counter() - t0
+    return {"value": rows / dt, "unit": "rows/s", "steps": steps,
+            "h2d_bytes_per_step": h2d // steps, "d2h_bytes_per_step": d2h // steps,
+            "ms_per_step": dt / steps * 1e3,
+            "path": "pinned host mask + features -> C-ABI calls -> count, coords, rows to host"}
+
+
+def run_sweep(torch, hc, dev, stream):
+    """Mask-density sweep at V = 10475, L = 9, B = 64, 128 -> 128 channels:
+    sparse conv (compaction done beforehand) against the dense layer."""
+    from paper_2608_09388_gb300 import inputs
+    w = inputs.make_workload("sweep10475_bf16")
+    ly = w.layers[0]
+    B, V, L = w.B, w.V, w.L
+    x = torch.from_numpy(w.x.view(np.int16)).view(torch.bfloat16).to(dev)
+    spiral = torch.from_numpy(w.spiral).to(dev)
+    Wt = torch.from_numpy(ly.W.view(np.int16)).view(torch.bfloat16).to(dev)
+    bias = torch.from_numpy(ly.b).to(dev)
+    y = torch.empty((B * V, ly.C_out), dtype=torch.bfloat16, device=dev)
+    coords = torch.empty((B * V, 2), dtype=torch.int32, device=dev)
+    row_of = torch.empty((B, V), dtype=torch.int32, device=dev)
+    offs = torch.empty((B + 1,), dtype=torch.int32, device=dev)
+    count = torch.empty((1,), dtype=torch.int32, device=dev)
+    pk = peaks()
+
+    def timeit(fn, reps=20):
+        with torch.cuda.stream(stream):
+            fn()
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                for _ in range(reps):
+                    fn()
+            g.replay()
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            g.replay()
+            b.record(stream)
+        torch.cuda.synchronize(dev)
+        return a.elapsed_time(b) / reps
+
+    yd = torch.empty((B, V, ly.C_out), dtype=torch.bfloat16, device=dev)
+    dense_ms = timeit(lambda: hc.hc_spiral_conv_fwd(x, spiral, Wt, bias, ly.act, yd, stream), 5)
+    out = []
+    for d, m in zip(w.densities, w.masks):
+        mt = torch.from_numpy(m).to(dev)
+        with torch.cuda.stream(stream):
+            hc.hc_mask_compact(mt, coords, row_of, offs, count, stream)
+        n = int(np.count_nonzero(m))
+        ms = timeit(lambda: hc.hc_sparse_spiral_conv_fwd(
+            x, hc.HC_LAYOUT_DENSE, coords, row_of, count, spiral, B, V, Wt, bias, ly.act, y,
+            stream))
+        fl = 2.0 * L * ly.C_in * ly.C_out * n
+        out.append({"density": d, "active_rows": n, "sparse_us": ms * 1e3,
+                    "dense_us": dense_ms * 1e3, "speedup": dense_ms / ms,
+                    "rows_per_s": n / (ms * 1e-3),
+                    "tensor_frac": fl / (ms * 1e-3) / 1e12 / pk["bf16_tflops"]})
+    st = hc.hc_get_device_status(stream)
+    if st != hc.HC_OK:
+        raise RuntimeError(f"device status {hc.STATUS_NAMES.get(st)} in the sweep")
+    return out
+
+
+def cpu_baseline(w, budget_s=20.0):
+    """The CPU oracle as it stands on this host's cores: compaction, sparse
+    conv and scatter of batch 0 of the workload (all of its active rows when
+    that fits the time budget, else a prefix of them, scaled to rows/s)."""
+    import oracle
+    ly = w.layers[0]
+    cores = len(os.sched_getaffinity(0))
+    t0 = time.perf_counter()
+    coords, row_of, offs, n = oracle.mask_compact(w.masks[0])
+    t_compact = time.perf_counter() - t0
+    probe = np.arange(min(n, 256), dtype=np.int64)
+    t0 = time.perf_counter()
+    oracle.sparse_spiral_conv(w.x, oracle.LAYOUT_DENSE, coords, row_of, w.spiral, ly.W, ly.b,
+                              ly.act, rows=probe, n_threads=cores)
+    per_row = (time.perf_counter() - t0) / max(1, len(probe))
+    k = n if per_row * n <= budget_s else max(256, int(budget_s / per_row))
+    rows = np.arange(k, dtype=np.int64)
+    t0 = time.perf_counter()
+    _, y = oracle.sparse_spiral_conv(w.x, oracle.LAYOUT_DENSE, coords, row_of, w.spiral, ly.W,
+                                     ly.b, ly.act, rows=rows, n_threads=cores)
+    t_conv = time.perf_counter() - t0
+    t0 = time.perf_counter()
+    oracle.scatter_dense(y, coords[:k], w.B, w.V, False)
+    t_scatter = time.perf_counter() - t0
+    secs = t_compact * k / max(n, 1) + t_conv + t_scatter
+    return {"value": k / secs, "unit": "rows/s", "cores": cores, "kind": "oracle",
+            "sample": f"batch 0 of {WORKLOAD}: compaction, sparse conv and scatter of "
+                      f"{k} of its {n} active rows (fp64 C oracle, OpenMP over rows)"}
+
+
+# ----------------------------------------------------------------- reference arm
+
+def run_reference(args, rank):
+    """The CPU oracle, as it stands, timed on this host's cores on bounded
+    samples of the same workload: each step computes 512 consecutive active
+    rows (compaction pro rata, conv, scatter)."""
+    if rank != 0:
+        return None
+    import oracle
+    from paper_2608_09388_gb300 import inputs
+    w = inputs.make_workload(WORKLOAD)
+    ly = w.layers[0]
+    cores = len(os.sched_getaffinity(0))
+    t0 = time.perf_counter()
+    coords, row_of, offs, n = oracle.mask_compact(w.masks[0])
+    t_compact_row = (time.perf_counter() - t0) / max(n, 1)
+    per = 512
+
+    def step(i):
+        s = (i * per) % max(1, n - per)
+        rows = np.arange(s, min(n, s + per), dtype=np.int64)
+        _, y = oracle.sparse_spiral_conv(w.x, oracle.LAYOUT_DENSE, coords, row_of, w.spiral, ly.W,
+                                         ly.b, ly.act, rows=rows, n_threads=cores)
+        oracle.scatter_dense(y, coords[rows], w.B, w.V, False)
+        return len(rows)
+
+    for i in range(args.warmup):
+        step(i)
+    t0 = time.perf_counter()
+    done = 0
+    for i in range(args.steps):
+        done += step(i)
+    secs = time.perf_counter() - t0 + t_compact_row * done
+    value = done / secs
+    return {
+        "metric": METRIC, "value": value, "unit": "rows/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": secs / args.steps * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "impl": "reference",
+        "config": {"workload": WORKLOAD, "B": w.B, "V": w.V, "L": w.L, "C_in": ly.C_in,
+                   "C_out": ly.C_out, "rows_per_step": per},
+        "cpu_baseline": {"value": value, "unit": "rows/s", "cores": cores, "kind": "oracle",
+                         "sample": f"{per} consecutive active rows of batch 0 per step"},
+        "e2e": {"value": value, "unit": "rows/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+
+
+def main():
+    args = parse_args()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        line = run_reference(args, rank)
+        if line is not None:
+            print(json.dumps(line), flush=True)
+        return
+    import torch
+    if world > 1:
+        torch.cuda.set_device(local_rank)
+        torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    try:
+        line = run_ours(args, rank, world, local_rank)
+    finally:
+        if world > 1:
+            torch.distributed.destroy_process_group()
+    if line is not None:
+        print(json.dumps(line), flush=True)
+
+
+if __name__ == "__main__":
+    main()

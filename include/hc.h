@@ -1,0 +1,176 @@
+/*
+ * hc.h -- C ABI of libhc, the GB300 (sm_103a) sparse contact operators of
+ * "ECO: Efficient Human-Contact Representation for Human-Scene Interaction".
+ *
+ * A sparse contact mask over body-mesh vertices selects the rows of a dense
+ * human-scene tensor (Eq. 1); the selected rows are decomposed into a
+ * coordinate list C' and compact features S' (Eq. 2); sparse layers then run
+ * on the compact rows only (Sec. 3.2): convolution over each vertex's spiral
+ * neighbourhood (Eqs. 4-5), linear (Eq. 6) and activation (Eq. 10).
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ *  - Every pointer argument is a DEVICE pointer on the current CUDA device,
+ *    except where a comment says otherwise. The caller owns every buffer;
+ *    nothing is retained after the call returns.
+ *  - Work is enqueued on `stream` (NULL = the legacy default stream) and is
+ *    asynchronous: the return status reports argument checks and launch
+ *    errors only. Problems found on the device (an out-of-range index, a
+ *    count above capacity, a bounded wait that ran out) set a sticky device
+ *    status word, read and cleared by hc_get_device_status().
+ *  - The active-row count N' stays on the device (`count`, one int32), so a
+ *    chain of calls needs no host synchronisation and can be captured into a
+ *    CUDA graph once the library has set itself up on the device (see
+ *    hc_mask_compact).
+ *  - Layouts are row-major. dtype HC_F32 means IEEE binary32; HC_BF16 means
+ *    bfloat16 storage with fp32 accumulation (tensor cores) and a
+ *    round-to-nearest-even store. Bias is always fp32. The input, weight and
+ *    output of one call share one dtype.
+ *  - Neighbours outside the active set contribute nothing (Eq. 4 keeps only
+ *    kernel taps whose coordinate is present in C), which equals the dense
+ *    layer on the masked input (Eq. 1) restricted to active rows.
+ *  - Sizes are int; B*V and every row count must stay below 2^31.
+ */
+#ifndef HC_H
+#define HC_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* hc_stream_t; /* same type as cudaStream_t */
+
+typedef enum {
+    HC_OK = 0,
+    HC_ERR_INVALID_ARG = 1,   /* null pointer, bad size, bad enum, misaligned pointer */
+    HC_ERR_UNSUPPORTED = 2,   /* valid but not supported (e.g. L > HC_MAX_SPIRAL) */
+    HC_ERR_CAPACITY = 3,      /* device: count exceeded the stated capacity */
+    HC_ERR_INVALID_INDEX = 4, /* device: spiral/row_of/coords entry out of range */
+    HC_ERR_TIMEOUT = 5,       /* device: a bounded wait inside a kernel ran out */
+    HC_ERR_CUDA = 6           /* CUDA runtime error; see hc_last_error_string() */
+} hc_status;
+
+typedef enum { HC_F32 = 0, HC_BF16 = 1 } hc_dtype;
+typedef enum { HC_ACT_NONE = 0, HC_ACT_ELU = 1, HC_ACT_RELU = 2 } hc_act;
+typedef enum {
+    HC_LAYOUT_DENSE = 0,  /* [B, V, C]: row (b, v) at (b*V + v)*C */
+    HC_LAYOUT_COMPACT = 1 /* [N', C]: row n is the n-th entry of coords */
+} hc_layout;
+
+#define HC_MAX_SPIRAL 32 /* largest spiral length L */
+
+/*
+ * hc_mask_compact -- decomposition of a masked tensor into coordinates (Eq. 2)
+ * and the inverse index map idx() used by the sparse convolution (Eq. 4).
+ *
+ *   mask     [B, V] uint8. Row (b, v) is active iff mask[b*V + v] != 0
+ *            (the paper's mask holds 0/1, Eq. 1; any nonzero byte counts).
+ *   coords   [B*V, 2] int32 capacity. Receives the active rows as (b, v)
+ *            pairs in ascending (b, v) order: the coordinate matrix C'.
+ *   row_of   [B, V] int32, or NULL. Receives the position of (b, v) in
+ *            coords, or -1 if inactive.
+ *   batch_offsets [B+1] int32, or NULL. Receives the number of active rows
+ *            in frames before b; batch_offsets[B] = N'. Rows of frame b are
+ *            [batch_offsets[b], batch_offsets[b+1]).
+ *   count    one int32: receives N'.
+ * B >= 0, V >= 0; B*V == 0 gives N' = 0. Results are bit-exact and unique.
+ *
+ * Scratch: a small per-(device, stream) workspace (one int32 per 4096 mask
+ * bytes) is allocated by the library on the first call that needs it and
+ * kept until process exit. Make the first call on each device and stream
+ * outside stream capture; later calls allocate nothing unless a larger mask
+ * is seen. Calls on one stream are ordered; calls on different streams use
+ * different workspaces.
+ */
+hc_status hc_mask_compact(const uint8_t* mask, int B, int V, int32_t* coords,
+                          int32_t* row_of, int32_t* batch_offsets, int32_t* count,
+                          hc_stream_t stream);
+
+/*
+ * hc_sparse_spiral_conv_fwd -- sparse convolution on the spiral
+ * neighbourhood (Eqs. 4-5) with fused bias (Eq. 6) and activation (Eq. 10).
+ *
+ * For each active row n < N' with coordinate (b, v) = coords[n]:
+ *   y[n, o] = act( bias[o] + sum_{l<L} sum_{c<C_in}
+ *                  S(b, spiral[v*L + l])[c] * W[(l*C_in + c)*C_out + o] )
+ * where S(b, u) is the input row of (b, u) when u >= 0 and row_of[b*V+u] >= 0,
+ * and the term is absent otherwise. Slot 0 of the spiral is the vertex
+ * itself (the centre tap); -1 entries mean "no neighbour".
+ *
+ *   x        x_layout DENSE: [B, V, C_in]; COMPACT: [N', C_in] in coords order
+ *   coords, row_of, count   as written by hc_mask_compact (row_of required)
+ *   spiral   [V, L] int32, entries in [-1, V)
+ *   W        [L*C_in, C_out] of dtype dt, row index l*C_in + c
+ *   bias     [C_out] fp32, or NULL for zero
+ *   y        [B*V, C_out] capacity of dtype dt; rows 0..N'-1 are written,
+ *            in coords order (the conv outputs the centre coordinates, Eq. 5).
+ * 1 <= L <= HC_MAX_SPIRAL, C_in >= 1, C_out >= 1.
+ * Out-of-range spiral/row_of/coords entries contribute nothing and set
+ * HC_ERR_INVALID_INDEX; a count above B*V is clamped and sets HC_ERR_CAPACITY.
+ * bf16 with C_in % 8 == 0, C_out % 8 == 0 and 16-byte aligned x, W, y runs
+ * on the tensor cores (tcgen05); other shapes run on CUDA cores.
+ */
+hc_status hc_sparse_spiral_conv_fwd(const void* x, hc_layout x_layout, hc_dtype dt,
+                                    const int32_t* coords, const int32_t* row_of,
+                                    const int32_t* count, const int32_t* spiral, int B, int V,
+                                    int L, int C_in, int C_out, const void* W, const float* bias,
+                                    hc_act act, void* y, hc_stream_t stream);
+
+/*
+ * hc_sparse_linear_fwd -- linear layer on compact rows (Eq. 6), row-wise
+ *   y[n, o] = act( bias[o] + sum_{c<C_in} x[n, c] * W[c*C_out + o] ),  n < N'
+ * The coordinates are unchanged (C' = C).
+ *   x [capacity, C_in], y [capacity, C_out], W [C_in, C_out] of dtype dt;
+ *   count: one int32 on the device (N'), must not exceed `capacity`
+ *   (clamped, HC_ERR_CAPACITY).
+ */
+hc_status hc_sparse_linear_fwd(const void* x, hc_dtype dt, const int32_t* count, int capacity,
+                               int C_in, int C_out, const void* W, const float* bias, hc_act act,
+                               void* y, hc_stream_t stream);
+
+/*
+ * hc_scatter_dense -- inverse of the decomposition (Eq. 2): compact rows back
+ * into a dense [B, V, C] tensor.
+ *   zero_fill == 0: out[coords[n]] = y[n] for n < N'; other rows untouched.
+ *   zero_fill != 0: every row of out is written: y[row_of[b,v]] where active,
+ *                   zeros elsewhere (the masked tensor of Eq. 1); needs row_of.
+ *   y [N', C] of dtype dt (elements are copied bit for bit), coords/row_of/
+ *   count as written by hc_mask_compact, out [B, V, C].
+ */
+hc_status hc_scatter_dense(const void* y, hc_dtype dt, const int32_t* coords,
+                           const int32_t* row_of, const int32_t* count, int B, int V, int C,
+                           int zero_fill, void* out, hc_stream_t stream);
+
+/*
+ * hc_spiral_conv_fwd -- the dense spiral-conv layer the sparse one replaces
+ * (Sec. 3.2), used as the speed-up denominator: every (b, v) is an output row,
+ *   y[(b*V+v), o] = act( bias[o] + sum_l sum_c x[b, spiral[v*L+l], c] *
+ *                                            W[(l*C_in + c)*C_out + o] )
+ * with -1 spiral entries skipped. x [B, V, C_in], y [B, V, C_out].
+ */
+hc_status hc_spiral_conv_fwd(const void* x, hc_dtype dt, const int32_t* spiral, int B, int V,
+                             int L, int C_in, int C_out, const void* W, const float* bias,
+                             hc_act act, void* y, hc_stream_t stream);
+
+/*
+ * hc_get_device_status -- synchronises `stream`, then reads and clears the
+ * current device's sticky status word. Returns HC_OK if no kernel reported a
+ * problem since the last read, else the lowest-numbered device error seen
+ * (HC_ERR_CAPACITY, HC_ERR_INVALID_INDEX or HC_ERR_TIMEOUT), or HC_ERR_CUDA
+ * if the synchronisation itself failed.
+ */
+hc_status hc_get_device_status(hc_stream_t stream);
+
+/* Text of the last host-side error on the calling thread ("" if none). */
+const char* hc_last_error_string(void);
+
+/* Library version, "major.minor.patch". */
+const char* hc_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* HC_H */

@@ -1,0 +1,141 @@
+// Spiral convolution / linear layer on CUDA cores (FFMA, fp32 accumulate).
+//
+// Used for fp32 (genuine IEEE fp32 multiply-adds: no TF32) and for bf16
+// shapes the tensor-core kernel does not take (channel counts that are not a
+// multiple of 8, e.g. a 45-channel input or a 42- or 1-wide output head).
+//
+// Each CTA owns a 64-row x 64-column output tile and walks K = L*C_in in
+// steps of 16: the A tile is gathered through the per-tile table of source
+// rows (idx() of Eq. 4: -1 when the tap is absent), the W tile is read
+// directly, and each thread accumulates a 4x4 block. The grid is persistent
+// over row tiles because the row count N' is only known on the device.
+#include <cuda_bf16.h>
+
+#include "hc_internal.cuh"
+
+namespace hc {
+namespace {
+
+constexpr int kBM = 64;
+constexpr int kBN = 64;
+constexpr int kBK = 16;
+constexpr int kThreads = 256;
+
+template <typename T>
+__device__ __forceinline__ float to_float(T v);
+template <>
+__device__ __forceinline__ float to_float<float>(float v) {
+    return v;
+}
+template <>
+__device__ __forceinline__ float to_float<__nv_bfloat16>(__nv_bfloat16 v) {
+    return __bfloat162float(v);
+}
+template <typename T>
+__device__ __forceinline__ T from_float(float v);
+template <>
+__device__ __forceinline__ float from_float<float>(float v) {
+    return v;
+}
+template <>
+__device__ __forceinline__ __nv_bfloat16 from_float<__nv_bfloat16>(float v) {
+    return __float2bfloat16_rn(v);
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kThreads) conv_simt_kernel(const ConvArgs a) {
+    __shared__ __align__(16) float As[kBK][kBM + 4];
+    __shared__ __align__(16) float Bs[kBK][kBN];
+    extern __shared__ int src_tab[];  // [kBM][L]
+
+    const T* __restrict__ x = static_cast<const T*>(a.x);
+    const T* __restrict__ W = static_cast<const T*>(a.W);
+    T* __restrict__ y = static_cast<T*>(a.y);
+    const long long rows = active_rows(a);
+    const long long m_tiles = (rows + kBM - 1) / kBM;
+    const int n0 = blockIdx.y * kBN;
+    const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+    const int L = a.L, C_in = a.C_in, C_out = a.C_out, K = a.K;
+
+    for (long long mt = blockIdx.x; mt < m_tiles; mt += gridDim.x) {
+        const long long m0 = mt * kBM;
+        __syncthreads();  // the previous tile is done with src_tab
+        for (int e = tid; e < kBM * L; e += kThreads) {
+            const int r = e / L, l = e - r * L;
+            const long long n = m0 + r;
+            long long src = -1;
+            int b, v;
+            if (n < rows && row_coord(a, n, b, v)) src = tap_row(a, n, b, v, l, rows);
+            src_tab[e] = (int)src;
+        }
+        __syncthreads();
+
+        float acc[4][4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+#pragma unroll
+            for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
+
+        for (int k0 = 0; k0 < K; k0 += kBK) {
+            for (int e = tid; e < kBM * kBK; e += kThreads) {
+                const int r = e / kBK, kk = e - r * kBK;
+                const int k = k0 + kk;
+                float val = 0.f;
+                if (k < K) {
+                    const int l = k / C_in, c = k - l * C_in;
+                    const int s = src_tab[r * L + l];
+                    if (s >= 0) val = to_float(x[(long long)s * C_in + c]);
+                }
+                As[kk][r] = val;
+            }
+            for (int e = tid; e < kBK * kBN; e += kThreads) {
+                const int kk = e / kBN, o = e - kk * kBN;
+                const int k = k0 + kk, col = n0 + o;
+                Bs[kk][o] = (k < K && col < C_out) ? to_float(W[(long long)k * C_out + col]) : 0.f;
+            }
+            __syncthreads();
+#pragma unroll
+            for (int kk = 0; kk < kBK; ++kk) {
+                const float4 av = *reinterpret_cast<const float4*>(&As[kk][ty * 4]);
+                const float4 bv = *reinterpret_cast<const float4*>(&Bs[kk][tx * 4]);
+                const float ar[4] = {av.x, av.y, av.z, av.w};
+                const float br[4] = {bv.x, bv.y, bv.z, bv.w};
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(ar[i], br[j], acc[i][j]);
+            }
+            __syncthreads();
+        }
+
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const long long n = m0 + ty * 4 + i;
+            if (n >= rows) continue;
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const int col = n0 + tx * 4 + j;
+                if (col >= C_out) continue;
+                const float z = acc[i][j] + (a.bias ? __ldg(a.bias + col) : 0.f);
+                y[n * C_out + col] = from_float<T>(act_apply(z, a.act));
+            }
+        }
+    }
+}
+
+}  // namespace
+
+hc_status launch_conv_simt(const DeviceCtx* ctx, const ConvArgs& a, hc_dtype dt, cudaStream_t s) {
+    long long cap_tiles = (a.capacity + kBM - 1) / kBM;
+    long long gx = cap_tiles < (long long)ctx->num_sms * 8 ? cap_tiles : (long long)ctx->num_sms * 8;
+    if (gx < 1) gx = 1;
+    dim3 grid((unsigned)gx, (unsigned)((a.C_out + kBN - 1) / kBN));
+    size_t smem = sizeof(int) * (size_t)kBM * a.L;
+    if (dt == HC_F32)
+        conv_simt_kernel<float><<<grid, kThreads, smem, s>>>(a);
+    else
+        conv_simt_kernel<__nv_bfloat16><<<grid, kThreads, smem, s>>>(a);
+    return check_cuda(cudaGetLastError(), "conv_simt_kernel");
+}
+
+}  // namespace hc

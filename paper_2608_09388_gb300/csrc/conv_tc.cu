@@ -1,0 +1,332 @@
+// Sparse / dense spiral convolution and linear layer on the sm_103a tensor
+// cores: gather -> tcgen05.mma (bf16 x bf16 -> fp32 in TMEM) -> fused
+// bias + activation epilogue -> bf16 compact rows.
+//
+// The gathered operand A is the implicit [rows, L*C_in] matrix whose row n
+// is the concatenation over spiral slots l of the input row idx(b, spiral[v][l])
+// (zeros for absent taps, Eq. 4); the layer computes A * W + bias (Eq. 5 with
+// the bias of Eq. 6) and the activation of Eq. 10.
+//
+// One persistent CTA per SM, 288 threads in three roles:
+//   warps 0-3  producers: gather 128 rows x 64 bf16 of A and the 64 x BN
+//              slice of W per k-block into a 128-byte-swizzled stage with
+//              16-byte cp.async (zero-fill for absent taps and ragged edges),
+//              then publish the stage on its "full" mbarrier;
+//   warp 8     MMA issuer (one thread): 4 x tcgen05.mma (K = 16 each) per
+//              stage into a TMEM accumulator, tcgen05.commit frees the stage;
+//   warps 4-7  epilogue: tcgen05.ld the 128 x BN fp32 accumulator (warp w
+//              reads TMEM lanes 32*(w%4)..+32), add bias, activation, round
+//              to bf16 and store. Two accumulators (2*BN TMEM columns) let
+//              the epilogue of one tile overlap the main loop of the next.
+// Shared-memory operand layouts (canonical tcgen05 forms, 128-byte swizzle):
+//   A: K-major, row r of the 128-row tile at r*128 bytes, 16-byte chunk q
+//      stored at chunk q ^ (r % 8); 8-row groups 1024 bytes apart (SBO).
+//   B: MN-major (W is [K, C_out] row-major, C_out contiguous), per 64-column
+//      block a [64 K-rows x 128 bytes] slab, K-row kr at kr*128 with chunk
+//      q stored at q ^ (kr % 8); 8-row groups 1024 bytes apart (SBO), the
+//      64-column blocks BK*128 bytes apart (LBO).
+// Every mbarrier wait is bounded (hc::kWaitLimitNs); on timeout the CTA
+// records HC_ERR_TIMEOUT, unwinds, waits for its own copies and MMAs and
+// frees its TMEM.
+#include <cuda_bf16.h>
+
+#include "hc_internal.cuh"
+
+namespace hc {
+namespace {
+
+constexpr int kBM = 128;  // rows per tile = TMEM lanes
+constexpr int kBK = 64;   // bf16 per 128-byte smem row
+constexpr int kAStageBytes = kBM * kBK * 2;
+constexpr int kProducerWarps = 4;
+constexpr int kEpilogueWarps = 4;
+constexpr int kMmaWarp = kProducerWarps + kEpilogueWarps;
+constexpr int kThreads = (kMmaWarp + 1) * 32;
+
+template <int BN>
+struct Cfg {
+    static constexpr int kBStageBytes = kBK * BN * 2;
+    static constexpr int kStages = BN == 64 ? 8 : 6;
+    static constexpr int kLag = kStages - 1;  // cp.async groups a producer keeps in flight
+    static constexpr int kTmemCols = 2 * BN;  // two accumulators
+    // Instruction descriptor, kind::f16: D fp32 (bit 4), A bf16 (bits 7-9 = 1),
+    // B bf16 (bits 10-12 = 1), A K-major (bit 15 = 0), B MN-major (bit 16 = 1),
+    // N >> 3 at bits 17-22, M >> 4 at bits 24-28.
+    static constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | (1u << 16) |
+                                       ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(kBM >> 4) << 24);
+    static constexpr int kBarBytes = 8 * (2 * kStages + 5);
+    static size_t smem_bytes(int L) {
+        return 1024 + (size_t)kStages * (kAStageBytes + kBStageBytes) + kBarBytes + 16 +
+               sizeof(int) * (size_t)kBM * L;
+    }
+};
+
+// Shared-memory matrix descriptor: start address, leading and stride byte
+// offsets (>> 4), fixed version bits 46-48 = 0b001, 128-byte swizzle (2 at
+// bits 61-63), base offset 0 (stage buffers are 1024-byte aligned).
+__device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+    return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)(lbo >> 4) << 16) |
+           ((uint64_t)(sbo >> 4) << 32) | (1ull << 46) | (2ull << 61);
+}
+
+template <int BN>
+__global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const ConvArgs a) {
+    using C = Cfg<BN>;
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t raw = smem_u32(smem_raw);
+    const uint32_t base = (raw + 1023u) & ~1023u;
+    uint8_t* const base_ptr = smem_raw + (base - raw);
+    const uint32_t sA = base;
+    const uint32_t sB = sA + C::kStages * kAStageBytes;
+    const uint32_t sBar = sB + C::kStages * C::kBStageBytes;
+    uint8_t* const misc = base_ptr + (sBar - base) + C::kBarBytes;
+    volatile uint32_t* const tmem_holder = reinterpret_cast<volatile uint32_t*>(misc);
+    volatile int* const abort_flag = reinterpret_cast<volatile int*>(misc + 4);
+    int* const src_tab = reinterpret_cast<int*>(misc + 16);  // [kBM][L]
+
+    auto full_bar = [&](int s) { return sBar + 8u * s; };
+    auto empty_bar = [&](int s) { return sBar + 8u * (C::kStages + s); };
+    auto tfull_bar = [&](int i) { return sBar + 8u * (2 * C::kStages + i); };
+    auto tempty_bar = [&](int i) { return sBar + 8u * (2 * C::kStages + 2 + i); };
+    const uint32_t fin_bar = sBar + 8u * (2 * C::kStages + 4);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < C::kStages; ++s) {
+            mbar_init(full_bar(s), kProducerWarps * 32);
+            mbar_init(empty_bar(s), 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(tfull_bar(i), 1);
+            mbar_init(tempty_bar(i), kEpilogueWarps * 32);
+        }
+        mbar_init(fin_bar, 1);
+        *abort_flag = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
+    }
+    if (warp == kMmaWarp) {
+        tmem_alloc(smem_u32((const void*)tmem_holder), C::kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_holder;
+
+    const long long rows = active_rows(a);
+    const long long m_tiles = (rows + kBM - 1) / kBM;
+    const int n_tiles = (a.C_out + BN - 1) / BN;
+    const long long work_total = m_tiles * n_tiles;
+    const int num_kb = (a.K + kBK - 1) / kBK;
+    const int L = a.L, C_in = a.C_in, C_out = a.C_out, K = a.K;
+
+    if (warp < kProducerWarps) {
+        // ------------------------------------------------------------ producers
+        const __nv_bfloat16* __restrict__ x = static_cast<const __nv_bfloat16*>(a.x);
+        const __nv_bfloat16* __restrict__ W = static_cast<const __nv_bfloat16*>(a.W);
+        const int t = threadIdx.x;  // 0..127
+        const int q = t & 7;        // A: 16-byte chunk of the 128-byte row
+        // This warp gathers rows r with r % 16 in [4*warp, 4*warp+4); lane
+        // fills the source table of one of them, so the table is warp-private.
+        const int tab_row = 4 * warp + (lane & 3) + 16 * (lane >> 2);
+        long long it = 0;
+        bool ok = true;
+        for (long long w = blockIdx.x; w < work_total && ok; w += gridDim.x) {
+            const long long m0 = (w / n_tiles) * kBM;
+            const int n0 = (int)(w % n_tiles) * BN;
+            __syncwarp();
+            {
+                const long long n = m0 + tab_row;
+                int b = 0, v = 0;
+                const bool valid = n < rows && row_coord(a, n, b, v);
+                for (int l = 0; l < L; ++l)
+                    src_tab[tab_row * L + l] = valid ? (int)tap_row(a, n, b, v, l, rows) : -1;
+            }
+            __syncwarp();
+            int l = (q * 8) / C_in;  // slot and channel of this thread's chunk at k-block 0
+            int c = q * 8 - l * C_in;
+            for (int kb = 0; kb < num_kb; ++kb) {
+                const int s = (int)(it % C::kStages);
+                const uint32_t ph = (uint32_t)((it / C::kStages) & 1);
+                if (!mbar_wait(empty_bar(s), ph ^ 1u, abort_flag, a.status)) {
+                    ok = false;
+                    break;
+                }
+                const uint32_t a_st = sA + s * kAStageBytes;
+                const bool kval = kb * kBK + q * 8 < K;
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const int r = (t >> 3) + 16 * i;
+                    const int src = kval ? src_tab[r * L + l] : -1;
+                    const __nv_bfloat16* gp = x + (src >= 0 ? (long long)src * C_in + c : 0);
+                    cp_async_16(a_st + r * 128 + ((q ^ (r & 7)) << 4), gp, src >= 0);
+                }
+                const uint32_t b_st = sB + s * C::kBStageBytes;
+                constexpr int kCpr = BN / 8;  // 16-byte chunks per W row slice
+#pragma unroll
+                for (int i = 0; i < (kBK * kCpr) / 128; ++i) {
+                    const int e = t + 128 * i;
+                    const int kr = e / kCpr, nq = e % kCpr;
+                    const int kk = kb * kBK + kr, col = n0 + nq * 8;
+                    const bool valid = kk < K && col < C_out;
+                    const __nv_bfloat16* gp = W + (valid ? (long long)kk * C_out + col : 0);
+                    cp_async_16(b_st + (nq >> 3) * (kBK * 128) + kr * 128 +
+                                    (((nq & 7) ^ (kr & 7)) << 4),
+                                gp, valid);
+                }
+                cp_async_commit();
+                if (it >= C::kLag) {
+                    cp_async_wait<C::kLag>();
+                    fence_proxy_async_smem();
+                    mbar_arrive(full_bar((int)((it - C::kLag) % C::kStages)));
+                }
+                ++it;
+                c += kBK;
+                while (c >= C_in) {
+                    c -= C_in;
+                    ++l;
+                }
+            }
+        }
+        cp_async_wait_all();
+        fence_proxy_async_smem();
+        if (ok)
+            for (long long j = it > C::kLag ? it - C::kLag : 0; j < it; ++j)
+                mbar_arrive(full_bar((int)(j % C::kStages)));
+    } else if (warp == kMmaWarp) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            long long it = 0;
+            int lt = 0;
+            bool ok = true;
+            for (long long w = blockIdx.x; w < work_total && ok; w += gridDim.x, ++lt) {
+                const int acc = lt & 1;
+                const uint32_t acc_ph = (uint32_t)((lt >> 1) & 1);
+                if (!mbar_wait(tempty_bar(acc), acc_ph ^ 1u, abort_flag, a.status)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
+                for (int kb = 0; kb < num_kb; ++kb) {
+                    const int s = (int)(it % C::kStages);
+                    const uint32_t ph = (uint32_t)((it / C::kStages) & 1);
+                    if (!mbar_wait(full_bar(s), ph, abort_flag, a.status)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    fence_proxy_async_smem();
+                    const uint32_t a_st = sA + s * kAStageBytes;
+                    const uint32_t b_st = sB + s * C::kBStageBytes;
+#pragma unroll
+                    for (int k = 0; k < kBK / 16; ++k) {
+                        const uint64_t ad = smem_desc_sw128(a_st + k * 32, 16, 1024);
+                        const uint64_t bd = smem_desc_sw128(b_st + k * 16 * 128, kBK * 128, 1024);
+                        tc_mma_bf16(d_tmem, ad, bd, C::kIdesc, (kb | k) != 0 ? 1u : 0u);
+                    }
+                    tc_commit(empty_bar(s));
+                    ++it;
+                }
+                if (!ok) break;
+                tc_commit(tfull_bar(acc));
+            }
+            // Every MMA issued by this thread has completed once fin_bar fires.
+            tc_commit(fin_bar);
+            int no_abort = 0;
+            mbar_wait(fin_bar, 0, &no_abort, a.status);
+        }
+        __syncwarp();
+    } else {
+        // ------------------------------------------------------------ epilogue
+        const int ew = warp - kProducerWarps;  // == warp % 4: TMEM lanes 32*ew..+32
+        __nv_bfloat16* __restrict__ y = static_cast<__nv_bfloat16*>(a.y);
+        int lt = 0;
+        for (long long w = blockIdx.x; w < work_total; w += gridDim.x, ++lt) {
+            const long long m0 = (w / n_tiles) * kBM;
+            const int n0 = (int)(w % n_tiles) * BN;
+            const int acc = lt & 1;
+            const uint32_t ph = (uint32_t)((lt >> 1) & 1);
+            if (!mbar_wait(tfull_bar(acc), ph, abort_flag, a.status)) break;
+            tc_fence_after();
+            const long long row = m0 + ew * 32 + lane;
+            const bool rvalid = row < rows;
+#pragma unroll 1
+            for (int cb = 0; cb < BN / 32; ++cb) {
+                uint32_t r[32];
+                tmem_ld_32x32b_x32(tmem_base + ((uint32_t)(ew * 32) << 16) + (uint32_t)(acc * BN + cb * 32),
+                                   r);
+                tmem_ld_wait();
+                const int col0 = n0 + cb * 32;
+                if (rvalid) {
+                    __nv_bfloat16* yp = y + row * C_out + col0;
+#pragma unroll
+                    for (int j8 = 0; j8 < 4; ++j8) {
+                        if (col0 + j8 * 8 < C_out) {
+                            uint32_t packed[4];
+#pragma unroll
+                            for (int h = 0; h < 4; ++h) {
+                                const int j = j8 * 8 + 2 * h;
+                                float z0 = __uint_as_float(r[j]);
+                                float z1 = __uint_as_float(r[j + 1]);
+                                if (a.bias) {
+                                    z0 += __ldg(a.bias + col0 + j);
+                                    z1 += __ldg(a.bias + col0 + j + 1);
+                                }
+                                const __nv_bfloat162 p =
+                                    __floats2bfloat162_rn(act_apply(z0, a.act), act_apply(z1, a.act));
+                                packed[h] = *reinterpret_cast<const uint32_t*>(&p);
+                            }
+                            *reinterpret_cast<uint4*>(yp + j8 * 8) =
+                                make_uint4(packed[0], packed[1], packed[2], packed[3]);
+                        }
+                    }
+                }
+            }
+            tc_fence_before();
+            mbar_arrive(tempty_bar(acc));
+        }
+    }
+
+    __syncthreads();
+    if (warp == kMmaWarp) {
+        tc_fence_after();
+        tmem_dealloc(tmem_base, C::kTmemCols);
+    }
+}
+
+template <int BN>
+hc_status launch_bn(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s) {
+    using C = Cfg<BN>;
+    static bool attr_set[64] = {};
+    if (!attr_set[ctx->device]) {
+        hc_status st = check_cuda(
+            cudaFuncSetAttribute(conv_tc_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)C::smem_bytes(HC_MAX_SPIRAL)),
+            "cudaFuncSetAttribute(conv_tc_kernel)");
+        if (st != HC_OK) return st;
+        attr_set[ctx->device] = true;
+    }
+    const long long n_tiles = (a.C_out + BN - 1) / BN;
+    const long long cap_work = (a.capacity + kBM - 1) / kBM * n_tiles;
+    long long grid = cap_work < ctx->num_sms ? cap_work : ctx->num_sms;
+    if (grid < 1) grid = 1;
+    conv_tc_kernel<BN><<<(unsigned)grid, kThreads, C::smem_bytes(a.L), s>>>(a);
+    return check_cuda(cudaGetLastError(), "conv_tc_kernel");
+}
+
+}  // namespace
+
+bool conv_tc_supported(const ConvArgs& a, hc_dtype dt) {
+    const uintptr_t al = (uintptr_t)a.x | (uintptr_t)a.W | (uintptr_t)a.y;
+    return dt == HC_BF16 && a.C_in % 8 == 0 && a.C_out % 8 == 0 && al % 16 == 0 &&
+           a.L <= HC_MAX_SPIRAL;
+}
+
+hc_status launch_conv_tc(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s) {
+    if (a.C_out <= 64) return launch_bn<64>(ctx, a, s);
+    return launch_bn<128>(ctx, a, s);
+}
+
+}  // namespace hc

@@ -1,0 +1,306 @@
+// C ABI of libhc (include/hc.h): host-side argument checks, the per-device
+// context and status word, the per-stream workspace, and dispatch to the
+// kernels. Every entry point validates before it launches anything.
+#include <cuda_runtime.h>
+#include <stdarg.h>
+#include <stdio.h>
+#include <stdlib.h>
+#include <string.h>
+
+#include <map>
+#include <mutex>
+#include <utility>
+
+#include "hc_internal.cuh"
+
+namespace hc {
+
+// Sticky per-device status word; kernels OR kErr* bits into it.
+__device__ unsigned g_device_status;
+
+static thread_local char t_last_error[512];
+
+void set_error(const char* fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(t_last_error, sizeof t_last_error, fmt, ap);
+    va_end(ap);
+}
+
+hc_status check_cuda(cudaError_t e, const char* what) {
+    if (e == cudaSuccess) return HC_OK;
+    set_error("%s: %s", what, cudaGetErrorString(e));
+    return HC_ERR_CUDA;
+}
+
+static constexpr int kMaxDevices = 64;
+static DeviceCtx g_ctx[kMaxDevices];
+static bool g_ctx_ready[kMaxDevices];
+static std::mutex g_ctx_mutex;
+
+const DeviceCtx* device_ctx() {
+    int dev = -1;
+    if (check_cuda(cudaGetDevice(&dev), "cudaGetDevice") != HC_OK) return nullptr;
+    if (dev < 0 || dev >= kMaxDevices) {
+        set_error("device ordinal %d out of range", dev);
+        return nullptr;
+    }
+    std::lock_guard<std::mutex> lock(g_ctx_mutex);
+    if (!g_ctx_ready[dev]) {
+        DeviceCtx c;
+        c.device = dev;
+        if (check_cuda(cudaDeviceGetAttribute(&c.num_sms, cudaDevAttrMultiProcessorCount, dev),
+                       "cudaDeviceGetAttribute") != HC_OK)
+            return nullptr;
+        void* p = nullptr;
+        if (check_cuda(cudaGetSymbolAddress(&p, g_device_status), "cudaGetSymbolAddress") != HC_OK)
+            return nullptr;
+        c.status = (unsigned*)p;
+        g_ctx[dev] = c;
+        g_ctx_ready[dev] = true;
+    }
+    return &g_ctx[dev];
+}
+
+struct Workspace {
+    void* ptr = nullptr;
+    size_t bytes = 0;
+};
+static std::map<std::pair<int, cudaStream_t>, Workspace> g_ws;
+static std::mutex g_ws_mutex;
+
+void* stream_workspace(cudaStream_t s, size_t bytes) {
+    int dev = -1;
+    if (check_cuda(cudaGetDevice(&dev), "cudaGetDevice") != HC_OK) return nullptr;
+    std::lock_guard<std::mutex> lock(g_ws_mutex);
+    Workspace& w = g_ws[std::make_pair(dev, s)];
+    if (w.bytes >= bytes) return w.ptr;
+    size_t want = bytes < 4096 ? 4096 : bytes;
+    if (w.ptr) {
+        // The old buffer may still be read by work queued on this stream.
+        if (check_cuda(cudaStreamSynchronize(s), "cudaStreamSynchronize") != HC_OK) return nullptr;
+        cudaFree(w.ptr);
+        w.ptr = nullptr;
+        w.bytes = 0;
+    }
+    void* p = nullptr;
+    if (check_cuda(cudaMalloc(&p, want), "cudaMalloc(workspace)") != HC_OK) return nullptr;
+    w.ptr = p;
+    w.bytes = want;
+    return p;
+}
+
+static bool misaligned(const void* p, size_t a) {
+    return ((uintptr_t)p) % a != 0;
+}
+
+}  // namespace hc
+
+using namespace hc;
+
+#define HC_REQUIRE(cond, ...)             \
+    do {                                  \
+        if (!(cond)) {                    \
+            set_error(__VA_ARGS__);       \
+            return HC_ERR_INVALID_ARG;    \
+        }                                 \
+    } while (0)
+
+extern "C" {
+
+const char* hc_last_error_string(void) {
+    return t_last_error;
+}
+
+const char* hc_version(void) {
+    return "0.1.0";
+}
+
+hc_status hc_mask_compact(const uint8_t* mask, int B, int V, int32_t* coords, int32_t* row_of,
+                          int32_t* batch_offsets, int32_t* count, hc_stream_t stream) {
+    t_last_error[0] = 0;
+    HC_REQUIRE(B >= 0 && V >= 0, "hc_mask_compact: B=%d V=%d must be >= 0", B, V);
+    HC_REQUIRE((long long)B * V < (1ll << 31), "hc_mask_compact: B*V must be < 2^31");
+    HC_REQUIRE(count != nullptr, "hc_mask_compact: count is NULL");
+    HC_REQUIRE((long long)B * V == 0 || (mask && coords),
+               "hc_mask_compact: mask and coords are required");
+    const DeviceCtx* ctx = device_ctx();
+    if (!ctx) return HC_ERR_CUDA;
+    return launch_compact(ctx, mask, B, V, coords, row_of, batch_offsets, count,
+                          (cudaStream_t)stream);
+}
+
+static hc_status check_conv_common(const char* fn, hc_dtype dt, int L, int C_in, int C_out,
+                                   hc_act act, const void* x, const void* W, void* y) {
+    HC_REQUIRE(dt == HC_F32 || dt == HC_BF16, "%s: unknown dtype %d", fn, (int)dt);
+    HC_REQUIRE(act == HC_ACT_NONE || act == HC_ACT_ELU || act == HC_ACT_RELU,
+               "%s: unknown activation %d", fn, (int)act);
+    HC_REQUIRE(C_in >= 1 && C_out >= 1, "%s: C_in=%d C_out=%d must be >= 1", fn, C_in, C_out);
+    HC_REQUIRE(L >= 1, "%s: L=%d must be >= 1", fn, L);
+    if (L > HC_MAX_SPIRAL) {
+        set_error("%s: L=%d exceeds HC_MAX_SPIRAL=%d", fn, L, HC_MAX_SPIRAL);
+        return HC_ERR_UNSUPPORTED;
+    }
+    HC_REQUIRE((long long)L * C_in < (1ll << 31), "%s: L*C_in too large", fn);
+    HC_REQUIRE(x && W && y, "%s: x, W and y are required", fn);
+    size_t eb = dt == HC_F32 ? 4 : 2;
+    HC_REQUIRE(!misaligned(x, eb) && !misaligned(W, eb) && !misaligned(y, eb),
+               "%s: x, W, y must be aligned to the element size", fn);
+    return HC_OK;
+}
+
+static hc_status dispatch_conv(const DeviceCtx* ctx, ConvArgs& a, hc_dtype dt, cudaStream_t s) {
+    static int force_simt = -1;
+    if (force_simt < 0) {
+        const char* e = getenv("HC_FORCE_SIMT");
+        force_simt = (e && e[0] == '1') ? 1 : 0;
+    }
+    a.status = ctx->status;
+    if (!force_simt && conv_tc_supported(a, dt)) return launch_conv_tc(ctx, a, s);
+    return launch_conv_simt(ctx, a, dt, s);
+}
+
+hc_status hc_sparse_spiral_conv_fwd(const void* x, hc_layout x_layout, hc_dtype dt,
+                                    const int32_t* coords, const int32_t* row_of,
+                                    const int32_t* count, const int32_t* spiral, int B, int V,
+                                    int L, int C_in, int C_out, const void* W, const float* bias,
+                                    hc_act act, void* y, hc_stream_t stream) {
+    const char* fn = "hc_sparse_spiral_conv_fwd";
+    t_last_error[0] = 0;
+    hc_status st = check_conv_common(fn, dt, L, C_in, C_out, act, x, W, y);
+    if (st != HC_OK) return st;
+    HC_REQUIRE(x_layout == HC_LAYOUT_DENSE || x_layout == HC_LAYOUT_COMPACT,
+               "%s: unknown layout %d", fn, (int)x_layout);
+    HC_REQUIRE(B >= 0 && V >= 0, "%s: B=%d V=%d must be >= 0", fn, B, V);
+    HC_REQUIRE((long long)B * V < (1ll << 31), "%s: B*V must be < 2^31", fn);
+    HC_REQUIRE(coords && row_of && count && spiral, "%s: coords, row_of, count, spiral required",
+               fn);
+    if ((long long)B * V == 0) return HC_OK;
+    const DeviceCtx* ctx = device_ctx();
+    if (!ctx) return HC_ERR_CUDA;
+    ConvArgs a{};
+    a.x = x;
+    a.coords = coords;
+    a.row_of = row_of;
+    a.count = count;
+    a.spiral = spiral;
+    a.W = W;
+    a.bias = bias;
+    a.y = y;
+    a.capacity = (long long)B * V;
+    a.B = B;
+    a.V = V;
+    a.L = L;
+    a.C_in = C_in;
+    a.C_out = C_out;
+    a.K = L * C_in;
+    a.mode = x_layout == HC_LAYOUT_DENSE ? kSparseDenseX : kSparseCompactX;
+    a.act = act;
+    return dispatch_conv(ctx, a, dt, (cudaStream_t)stream);
+}
+
+hc_status hc_sparse_linear_fwd(const void* x, hc_dtype dt, const int32_t* count, int capacity,
+                               int C_in, int C_out, const void* W, const float* bias, hc_act act,
+                               void* y, hc_stream_t stream) {
+    const char* fn = "hc_sparse_linear_fwd";
+    t_last_error[0] = 0;
+    hc_status st = check_conv_common(fn, dt, 1, C_in, C_out, act, x, W, y);
+    if (st != HC_OK) return st;
+    HC_REQUIRE(capacity >= 0, "%s: capacity=%d must be >= 0", fn, capacity);
+    HC_REQUIRE(count != nullptr, "%s: count is NULL", fn);
+    if (capacity == 0) return HC_OK;
+    const DeviceCtx* ctx = device_ctx();
+    if (!ctx) return HC_ERR_CUDA;
+    ConvArgs a{};
+    a.x = x;
+    a.count = count;
+    a.W = W;
+    a.bias = bias;
+    a.y = y;
+    a.capacity = capacity;
+    a.B = 1;
+    a.V = capacity;
+    a.L = 1;
+    a.C_in = C_in;
+    a.C_out = C_out;
+    a.K = C_in;
+    a.mode = kLinear;
+    a.act = act;
+    return dispatch_conv(ctx, a, dt, (cudaStream_t)stream);
+}
+
+hc_status hc_spiral_conv_fwd(const void* x, hc_dtype dt, const int32_t* spiral, int B, int V,
+                             int L, int C_in, int C_out, const void* W, const float* bias,
+                             hc_act act, void* y, hc_stream_t stream) {
+    const char* fn = "hc_spiral_conv_fwd";
+    t_last_error[0] = 0;
+    hc_status st = check_conv_common(fn, dt, L, C_in, C_out, act, x, W, y);
+    if (st != HC_OK) return st;
+    HC_REQUIRE(B >= 0 && V >= 0, "%s: B=%d V=%d must be >= 0", fn, B, V);
+    HC_REQUIRE((long long)B * V < (1ll << 31), "%s: B*V must be < 2^31", fn);
+    HC_REQUIRE(spiral != nullptr, "%s: spiral is NULL", fn);
+    if ((long long)B * V == 0) return HC_OK;
+    const DeviceCtx* ctx = device_ctx();
+    if (!ctx) return HC_ERR_CUDA;
+    ConvArgs a{};
+    a.x = x;
+    a.spiral = spiral;
+    a.W = W;
+    a.bias = bias;
+    a.y = y;
+    a.capacity = (long long)B * V;
+    a.B = B;
+    a.V = V;
+    a.L = L;
+    a.C_in = C_in;
+    a.C_out = C_out;
+    a.K = L * C_in;
+    a.mode = kDense;
+    a.act = act;
+    return dispatch_conv(ctx, a, dt, (cudaStream_t)stream);
+}
+
+hc_status hc_scatter_dense(const void* y, hc_dtype dt, const int32_t* coords,
+                           const int32_t* row_of, const int32_t* count, int B, int V, int C,
+                           int zero_fill, void* out, hc_stream_t stream) {
+    const char* fn = "hc_scatter_dense";
+    t_last_error[0] = 0;
+    HC_REQUIRE(dt == HC_F32 || dt == HC_BF16, "%s: unknown dtype %d", fn, (int)dt);
+    HC_REQUIRE(B >= 0 && V >= 0 && C >= 1, "%s: B=%d V=%d C=%d", fn, B, V, C);
+    HC_REQUIRE((long long)B * V < (1ll << 31), "%s: B*V must be < 2^31", fn);
+    HC_REQUIRE(y && count && out, "%s: y, count and out are required", fn);
+    HC_REQUIRE(zero_fill ? row_of != nullptr : coords != nullptr,
+               "%s: zero_fill needs row_of; scatter without it needs coords", fn);
+    int eb = dt == HC_F32 ? 4 : 2;
+    HC_REQUIRE(!misaligned(y, eb) && !misaligned(out, eb), "%s: misaligned y/out", fn);
+    if ((long long)B * V == 0) return HC_OK;
+    const DeviceCtx* ctx = device_ctx();
+    if (!ctx) return HC_ERR_CUDA;
+    return launch_scatter(ctx, y, eb, coords, row_of, count, B, V, C, zero_fill, out,
+                          (cudaStream_t)stream);
+}
+
+hc_status hc_get_device_status(hc_stream_t stream) {
+    t_last_error[0] = 0;
+    const DeviceCtx* ctx = device_ctx();
+    if (!ctx) return HC_ERR_CUDA;
+    if (check_cuda(cudaStreamSynchronize((cudaStream_t)stream), "cudaStreamSynchronize") != HC_OK)
+        return HC_ERR_CUDA;
+    unsigned word = 0, zero = 0;
+    if (check_cuda(cudaMemcpy(&word, ctx->status, sizeof word, cudaMemcpyDeviceToHost),
+                   "read device status") != HC_OK)
+        return HC_ERR_CUDA;
+    if (word == 0) return HC_OK;
+    if (check_cuda(cudaMemcpy(ctx->status, &zero, sizeof zero, cudaMemcpyHostToDevice),
+                   "clear device status") != HC_OK)
+        return HC_ERR_CUDA;
+    for (int code = HC_ERR_CAPACITY; code <= HC_ERR_TIMEOUT; ++code)
+        if (word & (1u << code)) {
+            set_error("device reported status word 0x%x", word);
+            return (hc_status)code;
+        }
+    set_error("device reported unknown status word 0x%x", word);
+    return HC_ERR_CUDA;
+}
+
+}  // extern "C"

@@ -1,0 +1,280 @@
+// Internal declarations shared by the libhc translation units: the device
+// status word, the per-device context, the row/neighbour index logic of the
+// sparse operators, and thin inline-PTX wrappers for sm_103a (cp.async,
+// mbarrier, tcgen05). Nothing here is part of the public ABI (include/hc.h).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "hc.h"
+
+namespace hc {
+
+// ------------------------------------------------------------ status bits
+// Device kernels OR one of these into the per-device status word.
+enum : unsigned {
+    kErrCapacity = 1u << HC_ERR_CAPACITY,
+    kErrIndex = 1u << HC_ERR_INVALID_INDEX,
+    kErrTimeout = 1u << HC_ERR_TIMEOUT,
+};
+
+// Longest a kernel waits on any one barrier before it gives up, records
+// HC_ERR_TIMEOUT and unwinds (nanoseconds of %globaltimer).
+constexpr unsigned long long kWaitLimitNs = 2000000000ull;
+
+// ------------------------------------------------------------ host context
+struct DeviceCtx {
+    int device;
+    int num_sms;
+    unsigned* status;  // device address of the sticky status word
+};
+
+// Context of the current device (cached); nullptr after recording an error.
+const DeviceCtx* device_ctx();
+void set_error(const char* fmt, ...);
+hc_status check_cuda(cudaError_t e, const char* what);
+// Per-(device, stream) scratch of at least `bytes`, grown on demand and kept
+// until exit. nullptr after recording an error.
+void* stream_workspace(cudaStream_t s, size_t bytes);
+
+// ------------------------------------------------------------ operator modes
+enum RowMode : int {
+    kSparseDenseX = 0,    // rows = coords[0..count); input rows at b*V+u
+    kSparseCompactX = 1,  // rows = coords[0..count); input rows at row_of[b*V+u]
+    kDense = 2,           // rows = all b*V+v; input rows at b*V+u
+    kLinear = 3,          // rows = 0..count; input row = output row; L = 1
+};
+
+struct ConvArgs {
+    const void* x;
+    const int32_t* coords;
+    const int32_t* row_of;
+    const int32_t* count;  // device N' (sparse/linear), unused for dense
+    const int32_t* spiral;
+    const void* W;
+    const float* bias;
+    void* y;
+    unsigned* status;
+    long long capacity;  // upper bound on rows (B*V, or the linear capacity)
+    int B, V, L, C_in, C_out, K;  // K = L*C_in
+    int mode;
+    int act;
+};
+
+// Launchers (each in its own translation unit). All return HC_OK or an
+// error already recorded with set_error().
+hc_status launch_compact(const DeviceCtx* ctx, const uint8_t* mask, int B, int V, int32_t* coords,
+                         int32_t* row_of, int32_t* offsets, int32_t* count, cudaStream_t s);
+hc_status launch_conv_simt(const DeviceCtx* ctx, const ConvArgs& a, hc_dtype dt, cudaStream_t s);
+hc_status launch_conv_tc(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s);
+bool conv_tc_supported(const ConvArgs& a, hc_dtype dt);
+hc_status launch_scatter(const DeviceCtx* ctx, const void* y, int elem_bytes, const int32_t* coords,
+                         const int32_t* row_of, const int32_t* count, int B, int V, int C,
+                         int zero_fill, void* out, cudaStream_t s);
+
+// ------------------------------------------------------------ device helpers
+#if defined(__CUDACC__)
+
+__device__ __forceinline__ void report(unsigned* status, unsigned bit) {
+    atomicOr(status, bit);
+}
+
+// Number of output rows of this call: N' from the device count (clamped to
+// the capacity, which is reported), or every grid row for the dense layer.
+__device__ __forceinline__ long long active_rows(const ConvArgs& a) {
+    if (a.mode == kDense) return (long long)a.B * a.V;
+    long long n = *a.count;
+    if (n < 0) {
+        report(a.status, kErrIndex);
+        return 0;
+    }
+    if (n > a.capacity) {
+        report(a.status, kErrCapacity);
+        n = a.capacity;
+    }
+    return n;
+}
+
+// Output row n -> coordinate (b, v). Returns false (and reports) for an
+// out-of-range coordinate; linear rows have no coordinate (b = v = 0).
+__device__ __forceinline__ bool row_coord(const ConvArgs& a, long long n, int& b, int& v) {
+    if (a.mode == kDense) {
+        b = (int)(n / a.V);
+        v = (int)(n - (long long)b * a.V);
+        return true;
+    }
+    if (a.mode == kLinear) {
+        b = 0;
+        v = 0;
+        return true;
+    }
+    b = __ldg(a.coords + 2 * n);
+    v = __ldg(a.coords + 2 * n + 1);
+    if (b < 0 || b >= a.B || v < 0 || v >= a.V) {
+        report(a.status, kErrIndex);
+        return false;
+    }
+    return true;
+}
+
+// Input row that feeds spiral slot l of output row n at (b, v), or -1 when
+// the tap is absent (no neighbour, or the neighbour is not an active row).
+// This is idx() of Eq. 4 for the sparse modes.
+__device__ __forceinline__ long long tap_row(const ConvArgs& a, long long n, int b, int v, int l,
+                                             long long n_rows) {
+    if (a.mode == kLinear) return n;
+    int u = __ldg(a.spiral + (long long)v * a.L + l);
+    if (u == -1) return -1;
+    if (u < -1 || u >= a.V) {
+        report(a.status, kErrIndex);
+        return -1;
+    }
+    long long dense_row = (long long)b * a.V + u;
+    if (a.mode == kDense) return dense_row;
+    int j = __ldg(a.row_of + dense_row);
+    if (j < 0) {
+        if (j != -1) report(a.status, kErrIndex);
+        return -1;
+    }
+    if (j >= n_rows) {
+        report(a.status, kErrIndex);
+        return -1;
+    }
+    return a.mode == kSparseDenseX ? dense_row : (long long)j;
+}
+
+__device__ __forceinline__ float act_apply(float z, int act) {
+    if (act == HC_ACT_ELU) return z > 0.f ? z : expm1f(z);
+    if (act == HC_ACT_RELU) return z > 0.f ? z : 0.f;
+    return z;
+}
+
+__device__ __forceinline__ unsigned long long globaltimer_ns() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+// ---- cp.async (16 bytes, zero-filled when !valid)
+__device__ __forceinline__ void cp_async_16(uint32_t dst, const void* src, bool valid) {
+    uint32_t n = valid ? 16u : 0u;
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(dst), "l"(src), "r"(n)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+    asm volatile("cp.async.commit_group;\n" ::: "memory");
+}
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+    asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+    asm volatile("cp.async.wait_all;\n" ::: "memory");
+}
+
+// Make this thread's generic-proxy shared-memory writes visible to the
+// async proxy (tcgen05.mma operand reads).
+__device__ __forceinline__ void fence_proxy_async_smem() {
+    asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
+}
+
+// ---- mbarrier
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;\n" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];\n" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n"
+        " mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+        " selp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// Wait for the phase with the given parity, for at most kWaitLimitNs. On
+// timeout (or when another role already gave up) it records HC_ERR_TIMEOUT,
+// raises the CTA's abort flag and returns false.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                          unsigned* status) {
+    if (mbar_try_wait(bar, parity)) return true;
+    unsigned long long t0 = globaltimer_ns();
+    for (uint32_t i = 1;; ++i) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if ((i & 63u) == 0) {
+            if (*abort_flag) return false;
+            if (globaltimer_ns() - t0 > kWaitLimitNs) {
+                *abort_flag = 1;
+                report(status, kErrTimeout);
+                return false;
+            }
+        }
+    }
+}
+
+// ---- tcgen05 (5th-generation tensor cores, accumulators in TMEM)
+__device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(dst_smem),
+                 "r"(ncols)
+                 : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;\n" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(taddr), "r"(ncols)
+                 : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+    asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+    asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory");
+}
+// D[tmem] (+)= A[smem] * B[smem], kind::f16 (bf16 inputs, fp32 accumulate).
+__device__ __forceinline__ void tc_mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                            uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+        " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+// Arrive once on `bar` when every tcgen05 op issued so far by this thread
+// has completed.
+__device__ __forceinline__ void tc_commit(uint32_t bar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n" ::"r"(bar)
+        : "memory");
+}
+// 32 lanes x 32 consecutive fp32 columns: thread i of the warp receives
+// lane (base lane + i), columns [col, col+32).
+__device__ __forceinline__ void tmem_ld_32x32b_x32(uint32_t taddr, uint32_t (&r)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+          "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
+          "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
+          "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr)
+        : "memory");
+}
+__device__ __forceinline__ void tmem_ld_wait() {
+    asm volatile("tcgen05.wait::ld.sync.aligned;\n" ::: "memory");
+}
+
+#endif  // __CUDACC__
+
+}  // namespace hc

@@ -1,0 +1,164 @@
+"""Python binding of libhc (include/hc.h): argument marshalling only.
+
+Each function has the name of the C entry point it calls and takes torch CUDA
+tensors (device memory) plus an optional stream (default: torch's current
+stream). Every step of the computation runs in libhc's CUDA kernels; there is
+no host or CPU fallback. If the library has not been built, or no GPU is
+present, the calls raise instead of computing anything.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(PKG, "_build", "libhc.so")
+
+HC_OK, HC_ERR_INVALID_ARG, HC_ERR_UNSUPPORTED, HC_ERR_CAPACITY = 0, 1, 2, 3
+HC_ERR_INVALID_INDEX, HC_ERR_TIMEOUT, HC_ERR_CUDA = 4, 5, 6
+HC_F32, HC_BF16 = 0, 1
+HC_ACT_NONE, HC_ACT_ELU, HC_ACT_RELU = 0, 1, 2
+HC_LAYOUT_DENSE, HC_LAYOUT_COMPACT = 0, 1
+HC_MAX_SPIRAL = 32
+
+STATUS_NAMES = {0: "HC_OK", 1: "HC_ERR_INVALID_ARG", 2: "HC_ERR_UNSUPPORTED",
+                3: "HC_ERR_CAPACITY", 4: "HC_ERR_INVALID_INDEX", 5: "HC_ERR_TIMEOUT",
+                6: "HC_ERR_CUDA"}
+
+# Exported symbols, as declared in include/hc.h.
+EXPORTS = ("hc_mask_compact", "hc_sparse_spiral_conv_fwd", "hc_sparse_linear_fwd",
+           "hc_scatter_dense", "hc_spiral_conv_fwd", "hc_get_device_status",
+           "hc_last_error_string", "hc_version")
+
+
+class HcError(RuntimeError):
+    def __init__(self, status: int, where: str, msg: str):
+        super().__init__(f"{where}: {STATUS_NAMES.get(status, status)}: {msg}")
+        self.status = status
+
+
+_lib = None
+_lock = threading.Lock()
+
+
+def load_library(path: str | None = None):
+    """Load libhc.so (built by paper_2608_09388_gb300.build). Raises if absent."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        p = path or LIB_PATH
+        if not os.path.exists(p):
+            raise RuntimeError(f"libhc is not built ({p} missing): run __graft_entry__.build()")
+        lib = ctypes.CDLL(p)
+        P, I = ctypes.c_void_p, ctypes.c_int
+        sig = {
+            "hc_mask_compact": [P, I, I, P, P, P, P, P],
+            "hc_sparse_spiral_conv_fwd": [P, I, I, P, P, P, P, I, I, I, I, I, P, P, I, P, P],
+            "hc_sparse_linear_fwd": [P, I, P, I, I, I, P, P, I, P, P],
+            "hc_scatter_dense": [P, I, P, P, P, I, I, I, I, P, P],
+            "hc_spiral_conv_fwd": [P, I, P, I, I, I, I, I, P, P, I, P, P],
+            "hc_get_device_status": [P],
+            "hc_last_error_string": [],
+            "hc_version": [],
+        }
+        for name, args in sig.items():
+            fn = getattr(lib, name)
+            fn.argtypes = args
+            fn.restype = ctypes.c_char_p if name in ("hc_last_error_string", "hc_version") else I
+        _lib = lib
+        return lib
+
+
+def _p(t):
+    if t is None:
+        return None
+    if not t.is_cuda:
+        raise ValueError("libhc takes device tensors")
+    if not t.is_contiguous():
+        raise ValueError("libhc takes contiguous tensors")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _s(stream):
+    import torch
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream))
+
+
+def _dt(t):
+    import torch
+    if t.dtype == torch.float32:
+        return HC_F32
+    if t.dtype == torch.bfloat16:
+        return HC_BF16
+    raise TypeError(f"unsupported dtype {t.dtype}")
+
+
+def _check(status: int, where: str):
+    if status != HC_OK:
+        msg = load_library().hc_last_error_string().decode()
+        raise HcError(status, where, msg)
+
+
+def hc_mask_compact(mask, coords, row_of, batch_offsets, count, stream=None):
+    """mask uint8 [B, V] -> coords int32 [B*V, 2], row_of int32 [B, V] (or None),
+    batch_offsets int32 [B+1] (or None), count int32 [1]."""
+    B, V = mask.shape
+    _check(load_library().hc_mask_compact(_p(mask), B, V, _p(coords), _p(row_of),
+                                          _p(batch_offsets), _p(count), _s(stream)),
+           "hc_mask_compact")
+
+
+def hc_sparse_spiral_conv_fwd(x, x_layout, coords, row_of, count, spiral, B, V, W, bias, act, y,
+                              stream=None):
+    """Sparse spiral conv; x dense [B, V, C_in] or compact [., C_in]; W [L*C_in, C_out];
+    y [B*V, C_out] capacity (rows 0..N'-1 written)."""
+    L = spiral.shape[1]
+    C_in = x.shape[-1]
+    C_out = W.shape[1]
+    _check(load_library().hc_sparse_spiral_conv_fwd(
+        _p(x), x_layout, _dt(x), _p(coords), _p(row_of), _p(count), _p(spiral), B, V, L, C_in,
+        C_out, _p(W), _p(bias), act, _p(y), _s(stream)), "hc_sparse_spiral_conv_fwd")
+
+
+def hc_sparse_linear_fwd(x, count, W, bias, act, y, stream=None):
+    """Linear layer on compact rows: x [capacity, C_in], W [C_in, C_out], y [capacity, C_out]."""
+    capacity, C_in = x.shape
+    C_out = W.shape[1]
+    _check(load_library().hc_sparse_linear_fwd(
+        _p(x), _dt(x), _p(count), capacity, C_in, C_out, _p(W), _p(bias), act, _p(y),
+        _s(stream)), "hc_sparse_linear_fwd")
+
+
+def hc_scatter_dense(y, coords, row_of, count, B, V, zero_fill, out, stream=None):
+    """Compact rows y [., C] -> dense out [B, V, C]."""
+    C = y.shape[-1]
+    _check(load_library().hc_scatter_dense(
+        _p(y), _dt(y), _p(coords), _p(row_of), _p(count), B, V, C, int(zero_fill), _p(out),
+        _s(stream)), "hc_scatter_dense")
+
+
+def hc_spiral_conv_fwd(x, spiral, W, bias, act, y, stream=None):
+    """Dense spiral conv over every (b, v): x [B, V, C_in] -> y [B, V, C_out]."""
+    B, V, C_in = x.shape
+    L = spiral.shape[1]
+    C_out = W.shape[1]
+    _check(load_library().hc_spiral_conv_fwd(
+        _p(x), _dt(x), _p(spiral), B, V, L, C_in, C_out, _p(W), _p(bias), act, _p(y),
+        _s(stream)), "hc_spiral_conv_fwd")
+
+
+def hc_get_device_status(stream=None) -> int:
+    """Synchronise the stream, read and clear the device status word."""
+    return int(load_library().hc_get_device_status(_s(stream)))
+
+
+def hc_last_error_string() -> str:
+    return load_library().hc_last_error_string().decode()
+
+
+def hc_version() -> str:
+    return load_library().hc_version().decode()

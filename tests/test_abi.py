@@ -1,0 +1,78 @@
+"""The C-ABI library builds, loads and exports every entry point that
+include/hc.h declares; host-side argument checks reject bad calls before
+anything reaches a GPU. No compute call is made here (no GPU needed)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2608_09388_gb300 import build, hc
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(__file__)), "include", "hc.h")
+
+
+def _declared():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(hc_[a-z_0-9]+)\s*\(", src)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build()
+    return hc.load_library()
+
+
+def test_header_declares_the_boundary():
+    d = _declared()
+    for name in ("hc_mask_compact", "hc_sparse_spiral_conv_fwd", "hc_sparse_linear_fwd",
+                 "hc_scatter_dense", "hc_spiral_conv_fwd", "hc_get_device_status",
+                 "hc_last_error_string"):
+        assert name in d
+    assert set(hc.EXPORTS) <= set(d)
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in _declared():
+        assert hasattr(lib, name), f"libhc.so does not export {name}"
+
+
+def test_version(lib):
+    assert re.match(r"^\d+\.\d+\.\d+$", hc.hc_version())
+
+
+# Host-side validation returns before any CUDA call, so it runs without a GPU.
+def test_invalid_arguments_rejected_on_host(lib):
+    P = ctypes.c_void_p
+    fake = P(0x1000)
+    assert lib.hc_mask_compact(fake, -1, 5, fake, None, None, fake, None) == hc.HC_ERR_INVALID_ARG
+    assert lib.hc_mask_compact(fake, 2, 5, fake, None, None, None, None) == hc.HC_ERR_INVALID_ARG
+    assert "count" in hc.hc_last_error_string()
+    # unknown dtype
+    assert lib.hc_sparse_spiral_conv_fwd(fake, 0, 7, fake, fake, fake, fake, 1, 4, 3, 8, 8, fake,
+                                         None, 1, fake, None) == hc.HC_ERR_INVALID_ARG
+    # spiral longer than supported
+    assert lib.hc_sparse_spiral_conv_fwd(fake, 0, 1, fake, fake, fake, fake, 1, 40, 33, 8, 8, fake,
+                                         None, 1, fake, None) == hc.HC_ERR_UNSUPPORTED
+    # unknown activation
+    assert lib.hc_spiral_conv_fwd(fake, 1, fake, 1, 4, 3, 8, 8, fake, None, 9, fake,
+                                  None) == hc.HC_ERR_INVALID_ARG
+    # misaligned pointer for the element size
+    assert lib.hc_spiral_conv_fwd(P(0x1001), 1, fake, 1, 4, 3, 8, 8, fake, None, 1, fake,
+                                  None) == hc.HC_ERR_INVALID_ARG
+    # zero_fill without row_of
+    assert lib.hc_scatter_dense(fake, 1, fake, None, fake, 2, 3, 8, 1, fake,
+                                None) == hc.HC_ERR_INVALID_ARG
+    # negative capacity
+    assert lib.hc_sparse_linear_fwd(fake, 1, fake, -1, 8, 8, fake, None, 0, fake,
+                                    None) == hc.HC_ERR_INVALID_ARG
+    # C_in < 1
+    assert lib.hc_sparse_linear_fwd(fake, 1, fake, 4, 0, 8, fake, None, 0, fake,
+                                    None) == hc.HC_ERR_INVALID_ARG
+
+
+def test_missing_library_fails_loudly(tmp_path, monkeypatch):
+    monkeypatch.setattr(hc, "_lib", None)
+    with pytest.raises(RuntimeError, match="not built"):
+        hc.load_library(str(tmp_path / "nope.so"))

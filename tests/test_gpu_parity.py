@@ -1,0 +1,379 @@
+"""Parity of the CUDA path (through the C-ABI) with the CPU oracle.
+
+Indices (coords, row_of, offsets, count) must match bit for bit; fp32 outputs
+within 1e-4 absolute of the oracle's fp64 value; bf16 outputs within
+2e-2 * max(|r|, 1) of the oracle's fp64 value r before rounding. Small cases
+are compared element by element; full-size workloads on sampled rows that
+the oracle computes one by one."""
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2608_09388_gb300 import hc, inputs
+
+from _util import check_close, sample_rows, to_numpy, to_torch
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+NCPU = len(os.sched_getaffinity(0))
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2608_09388_gb300 import build
+    build.build()
+    hc.load_library()
+    assert hc.hc_get_device_status() == hc.HC_OK
+
+
+def gpu_compact(mask_np, offset=0):
+    """Run hc_mask_compact; returns torch (coords, row_of, offsets, count).
+    `offset` > 0 places the mask at a misaligned address."""
+    B, V = mask_np.shape
+    if offset:
+        buf = torch.zeros(B * V + offset, dtype=torch.uint8, device="cuda")
+        buf[offset:] = torch.from_numpy(mask_np.ravel()).cuda()
+        mask = buf[offset:].view(B, V)
+    else:
+        mask = to_torch(mask_np)
+    coords = torch.full((max(B * V, 1), 2), -7, dtype=torch.int32, device="cuda")
+    row_of = torch.full((B, V), -7, dtype=torch.int32, device="cuda")
+    offs = torch.full((B + 1,), -7, dtype=torch.int32, device="cuda")
+    count = torch.full((1,), -7, dtype=torch.int32, device="cuda")
+    hc.hc_mask_compact(mask, coords, row_of, offs, count)
+    return coords, row_of, offs, count
+
+
+def assert_compact_equal(mask_np, got):
+    coords, row_of, offs, count = got
+    c_ref, r_ref, o_ref, n = oracle.mask_compact(mask_np)
+    assert int(count.item()) == n
+    np.testing.assert_array_equal(to_numpy(coords)[:n], c_ref)
+    np.testing.assert_array_equal(to_numpy(row_of), r_ref)
+    np.testing.assert_array_equal(to_numpy(offs), o_ref)
+
+
+def run_sparse_conv(x_np, x_layout, mask_np, sp_np, W_np, b_np, act, coords=None, row_of=None,
+                    count=None, y_fill=None):
+    B, V = mask_np.shape
+    if coords is None:
+        coords, row_of, _, count = gpu_compact(mask_np)
+    C_out = W_np.shape[1]
+    x = to_torch(x_np)
+    dt = torch.float32 if x_np.dtype == np.float32 else torch.bfloat16
+    y = torch.full((B * V, C_out), float("nan") if y_fill is None else y_fill, dtype=dt,
+                   device="cuda")
+    hc.hc_sparse_spiral_conv_fwd(x, x_layout, coords, row_of, count, to_torch(sp_np), B, V,
+                                 to_torch(W_np), None if b_np is None else to_torch(b_np), act, y)
+    assert hc.hc_get_device_status() == hc.HC_OK
+    return to_numpy(y), int(count.item())
+
+
+# ------------------------------------------------------------------ compaction
+
+@pytest.mark.parametrize("B,V", [(1, 1), (1, 31), (7, 32), (7, 33), (64, 655), (256, 655),
+                                 (3, 10475), (32, 10475)])
+@pytest.mark.parametrize("density", [0.0, 0.01, 0.1, 0.5, 1.0])
+def test_compact_bit_exact(B, V, density):
+    m = inputs.uniform_mask(np.random.default_rng(B * 7919 + V), B, V, density)
+    assert_compact_equal(m, gpu_compact(m))
+
+
+@pytest.mark.parametrize("offset", [1, 3, 8])
+def test_compact_misaligned_mask(offset):
+    m = inputs.uniform_mask(np.random.default_rng(offset), 9, 777, 0.3)
+    assert_compact_equal(m, gpu_compact(m, offset))
+
+
+def test_compact_nonbinary_and_many_tiles():
+    rng = np.random.default_rng(4)
+    m = (rng.integers(0, 4, size=(520, 10475)) * (rng.random((520, 10475)) < 0.1)).astype(np.uint8)
+    assert_compact_equal(m, gpu_compact(m))  # > 1024 tiles: pre-scanned offsets
+
+
+def test_compact_empty_sizes():
+    for B, V in [(0, 5), (3, 0), (0, 0)]:
+        m = np.zeros((B, V), np.uint8)
+        coords = torch.zeros((1, 2), dtype=torch.int32, device="cuda")
+        offs = torch.full((B + 1,), -7, dtype=torch.int32, device="cuda")
+        count = torch.full((1,), -7, dtype=torch.int32, device="cuda")
+        hc.hc_mask_compact(torch.zeros((B, V), dtype=torch.uint8, device="cuda"), coords, None,
+                           offs, count)
+        assert int(count.item()) == 0 and (to_numpy(offs) == 0).all()
+
+
+def test_compact_workload_masks():
+    for name in ("layer655_f32", "encoder655_bf16", "motion655_bf16", "layer10475_bf16"):
+        w = inputs.make_workload(name)
+        for m in w.masks:
+            assert_compact_equal(m, gpu_compact(m))
+
+
+# ------------------------------------------------------------------ sparse conv
+
+def test_golden_octahedron_on_gpu():
+    """The hand-worked octahedron cases (fp32 path)."""
+    import json
+    g = json.load(open(os.path.join(os.path.dirname(__file__), "golden", "octahedron.json")))
+    acts = {"none": hc.HC_ACT_NONE, "elu": hc.HC_ACT_ELU}
+    for case in g["cases"]:
+        sp = np.array(g["spiral_L3"], dtype=np.int32)[:, : case.get("spiral_cols", 3)].copy()
+        for k, row in case.get("spiral_override", {}).items():
+            sp[int(k)] = row
+        x = np.array(case["x"], dtype=np.float32)
+        m = np.array(case["mask"], dtype=np.uint8)
+        W = np.array(case["W"], dtype=np.float32)
+        b = np.array(case["bias"], dtype=np.float32)
+        y, n = run_sparse_conv(x, hc.HC_LAYOUT_DENSE, m, sp, W, b, acts[case["act"]])
+        c_ref, r_ref, _, n_ref = oracle.mask_compact(m)
+        y_pre, _ = oracle.sparse_spiral_conv(x, oracle.LAYOUT_DENSE, c_ref, r_ref, sp, W, b,
+                                             acts[case["act"]])
+        check_close(y[:n], y_pre, case["name"])
+
+
+def test_layer655_f32_full():
+    w = inputs.make_workload("layer655_f32")
+    ly = w.layers[0]
+    y, n = run_sparse_conv(w.x, hc.HC_LAYOUT_DENSE, w.masks[0], w.spiral, ly.W, ly.b, ly.act)
+    c, r, _, n_ref = oracle.mask_compact(w.masks[0])
+    assert n == n_ref
+    y_pre, _ = oracle.sparse_spiral_conv(w.x, oracle.LAYOUT_DENSE, c, r, w.spiral, ly.W, ly.b,
+                                         ly.act)
+    check_close(y[:n], y_pre, "layer655_f32")
+
+
+# (B, V, L, C_in, C_out, density, neg_frac): ragged N', several tiles, -1 entries
+SHAPES = [
+    (1, 40, 1, 8, 8, 0.5, 0.0),
+    (3, 200, 9, 16, 64, 0.3, 0.1),
+    (5, 300, 12, 64, 128, 0.4, 0.05),
+    (2, 500, 9, 128, 128, 0.6, 0.0),
+    (4, 333, 7, 24, 40, 0.5, 0.2),
+    (2, 257, 5, 8, 136, 0.9, 0.0),
+    (2, 400, 9, 64, 256, 0.5, 0.0),
+    (1, 700, 12, 32, 72, 0.35, 0.1),
+]
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("layout", [hc.HC_LAYOUT_DENSE, hc.HC_LAYOUT_COMPACT])
+@pytest.mark.parametrize("shape", SHAPES)
+def test_sparse_conv_shapes(shape, layout, dtype):
+    B, V, L, C_in, C_out, dens, neg = shape
+    sp, m, x, W, b = inputs.random_case(B * 1000 + V + L + C_in + C_out, B, V, L, C_in, C_out,
+                                        dtype, dens, neg)
+    c, r, _, n = oracle.mask_compact(m)
+    xin = x if layout == hc.HC_LAYOUT_DENSE else np.ascontiguousarray(x[c[:, 0], c[:, 1]])
+    y, n_gpu = run_sparse_conv(xin, layout, m, sp, W, b, hc.HC_ACT_ELU)
+    assert n_gpu == n
+    y_pre, _ = oracle.sparse_spiral_conv(xin, layout, c, r, sp, W, b, oracle.ACT_ELU)
+    check_close(y[:n], y_pre, f"{shape} layout={layout} {dtype}")
+
+
+@pytest.mark.parametrize("C_in,C_out", [(45, 64), (16, 42), (10, 3), (64, 1)])
+def test_sparse_conv_odd_channels_bf16(C_in, C_out):
+    sp, m, x, W, b = inputs.random_case(C_in * 100 + C_out, 3, 300, 9, C_in, C_out, "bf16", 0.3)
+    c, r, _, n = oracle.mask_compact(m)
+    y, _ = run_sparse_conv(x, hc.HC_LAYOUT_DENSE, m, sp, W, b, hc.HC_ACT_ELU)
+    y_pre, _ = oracle.sparse_spiral_conv(x, oracle.LAYOUT_DENSE, c, r, sp, W, b, oracle.ACT_ELU)
+    check_close(y[:n], y_pre, f"odd channels {C_in}->{C_out}")
+
+
+@pytest.mark.parametrize("act", [hc.HC_ACT_NONE, hc.HC_ACT_RELU])
+def test_sparse_conv_activations(act):
+    sp, m, x, W, b = inputs.random_case(31, 2, 300, 9, 64, 64, "bf16", 0.4)
+    c, r, _, n = oracle.mask_compact(m)
+    y, _ = run_sparse_conv(x, hc.HC_LAYOUT_DENSE, m, sp, W, None, act)
+    y_pre, _ = oracle.sparse_spiral_conv(x, oracle.LAYOUT_DENSE, c, r, sp, W, None, act)
+    check_close(y[:n], y_pre, f"act {act}")
+
+
+def test_empty_mask_leaves_output_untouched():
+    sp, m, x, W, b = inputs.random_case(32, 2, 300, 9, 64, 128, "bf16", 0.0)
+    y, n = run_sparse_conv(x, hc.HC_LAYOUT_DENSE, m, sp, W, b, hc.HC_ACT_ELU, y_fill=3.0)
+    assert n == 0
+    assert (y == to_numpy(torch.tensor([3.0], dtype=torch.bfloat16))[0]).all()
+
+
+def test_all_ones_mask_equals_dense_operator():
+    sp, m, x, W, b = inputs.random_case(33, 3, 300, 9, 64, 128, "bf16", 1.0)
+    y, n = run_sparse_conv(x, hc.HC_LAYOUT_DENSE, m, sp, W, b, hc.HC_ACT_ELU)
+    yd = torch.empty((3, 300, 128), dtype=torch.bfloat16, device="cuda")
+    hc.hc_spiral_conv_fwd(to_torch(x), to_torch(sp), to_torch(W), to_torch(b), hc.HC_ACT_ELU, yd)
+    np.testing.assert_array_equal(y[:n], to_numpy(yd).reshape(-1, 128))
+
+
+def test_deterministic_and_stream_ordered():
+    sp, m, x, W, b = inputs.random_case(34, 4, 500, 12, 64, 128, "bf16", 0.3)
+    s = torch.cuda.Stream()
+    with torch.cuda.stream(s):
+        y1, _ = run_sparse_conv(x, hc.HC_LAYOUT_DENSE, m, sp, W, b, hc.HC_ACT_ELU)
+        y2, _ = run_sparse_conv(x, hc.HC_LAYOUT_DENSE, m, sp, W, b, hc.HC_ACT_ELU)
+    np.testing.assert_array_equal(y1, y2)
+
+
+# ------------------------------------------------------------------ dense conv
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("shape", [(2, 300, 9, 64, 128), (3, 257, 12, 16, 64), (1, 100, 5, 40, 24)])
+def test_dense_conv(shape, dtype):
+    B, V, L, C_in, C_out = shape
+    sp, m, x, W, b = inputs.random_case(sum(shape), B, V, L, C_in, C_out, dtype, 1.0, 0.1)
+    xt = to_torch(x)
+    y = torch.empty((B, V, C_out), dtype=xt.dtype, device="cuda")
+    hc.hc_spiral_conv_fwd(xt, to_torch(sp), to_torch(W), to_torch(b), hc.HC_ACT_ELU, y)
+    assert hc.hc_get_device_status() == hc.HC_OK
+    y_pre, _ = oracle.dense_spiral_conv(x, sp, W, b, oracle.ACT_ELU)
+    check_close(to_numpy(y).reshape(B * V, C_out), y_pre, f"dense {shape} {dtype}")
+
+
+# ------------------------------------------------------------------ linear
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("C_in,C_out", [(64, 42), (64, 1), (64, 128), (128, 64), (45, 7)])
+def test_sparse_linear(C_in, C_out, dtype):
+    rng = np.random.default_rng(C_in * 1000 + C_out)
+    cap, n = 1000, 777
+    x = inputs.features(rng, (cap, C_in), dtype)
+    W = inputs.weights(rng, C_in, C_out, dtype)
+    b = inputs.bias(C_out)
+    count = torch.tensor([n], dtype=torch.int32, device="cuda")
+    xt = to_torch(x)
+    y = torch.full((cap, C_out), float("nan"), dtype=xt.dtype, device="cuda")
+    hc.hc_sparse_linear_fwd(xt, count, to_torch(W), to_torch(b), hc.HC_ACT_NONE, y)
+    assert hc.hc_get_device_status() == hc.HC_OK
+    y_pre, _ = oracle.sparse_linear(x[:n], W, b, oracle.ACT_NONE)
+    got = to_numpy(y)
+    check_close(got[:n], y_pre, f"linear {C_in}->{C_out} {dtype}")
+    assert np.isnan(got[n:].astype(np.float64) if dtype == "f32" else
+                    (got[n:].astype(np.uint32) << 16).view(np.float32)).all()
+
+
+# ------------------------------------------------------------------ scatter
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("C", [1, 3, 8, 42, 128])
+@pytest.mark.parametrize("zero_fill", [0, 1])
+def test_scatter_dense(C, zero_fill, dtype):
+    rng = np.random.default_rng(C * 10 + zero_fill)
+    B, V = 5, 333
+    m = inputs.uniform_mask(rng, B, V, 0.25)
+    coords, row_of, offs, count = gpu_compact(m)
+    c, r, _, n = oracle.mask_compact(m)
+    y = inputs.features(rng, (n, C), dtype)
+    prev = inputs.features(rng, (B, V, C), dtype)
+    out = to_torch(prev)
+    hc.hc_scatter_dense(to_torch(y), coords, row_of, count, B, V, zero_fill, out)
+    assert hc.hc_get_device_status() == hc.HC_OK
+    ref = oracle.scatter_dense(y, c, B, V, zero_fill, out=prev)
+    np.testing.assert_array_equal(to_numpy(out), ref)
+
+
+# ------------------------------------------------------------------ encoders
+
+def run_encoder_gpu(w):
+    """The stacked sparse layers of a workload through the C-ABI: compact
+    once, first conv on the dense input, later layers on compact rows, then
+    the linear head."""
+    m = w.masks[0]
+    B, V = m.shape
+    coords, row_of, offs, count = gpu_compact(m)
+    h = to_torch(w.x)
+    layout = hc.HC_LAYOUT_DENSE
+    sp = to_torch(w.spiral)
+    for ly in w.layers:
+        y = torch.empty((B * V, ly.C_out), dtype=h.dtype, device="cuda")
+        if ly.kind == "conv":
+            hc.hc_sparse_spiral_conv_fwd(h, layout, coords, row_of, count, sp, B, V,
+                                         to_torch(ly.W), to_torch(ly.b), ly.act, y)
+        else:
+            hc.hc_sparse_linear_fwd(h, count, to_torch(ly.W), to_torch(ly.b), ly.act, y)
+        h, layout = y, hc.HC_LAYOUT_COMPACT
+    assert hc.hc_get_device_status() == hc.HC_OK
+    return to_numpy(h), int(count.item())
+
+
+@pytest.mark.parametrize("name", ["encoder655_bf16", "motion655_bf16"])
+def test_encoder_end_to_end(name):
+    """Whole stack against the oracle's own stack (each layer stored in bf16
+    on both sides). The final layer is compared under the bf16 tolerance."""
+    w = inputs.make_workload(name)
+    got, n = run_encoder_gpu(w)
+    c, r, o, n_ref, outs = oracle.encoder(w.x, w.masks[0], w.spiral, w.layers, n_threads=NCPU)
+    assert n == n_ref
+    check_close(got[:n], outs[-1][0], name)
+
+
+# ------------------------------------------------------------------ full size, sampled
+
+def test_layer10475_full_size_sampled():
+    w = inputs.make_workload("layer10475_bf16")
+    ly = w.layers[0]
+    y, n = run_sparse_conv(w.x, hc.HC_LAYOUT_DENSE, w.masks[0], w.spiral, ly.W, ly.b, ly.act)
+    c, r, _, n_ref = oracle.mask_compact(w.masks[0])
+    assert n == n_ref
+    rows = sample_rows(n, 3000, seed=1)
+    y_pre, _ = oracle.sparse_spiral_conv(w.x, oracle.LAYOUT_DENSE, c, r, w.spiral, ly.W, ly.b,
+                                         ly.act, rows=rows, n_threads=NCPU)
+    check_close(y[rows], y_pre, "layer10475 sampled")
+
+
+def test_sweep10475_full_size_sampled():
+    w = inputs.make_workload("sweep10475_bf16")
+    ly = w.layers[0]
+    B, V = w.B, w.V
+    xt = to_torch(w.x)
+    for d, m in zip(w.densities, w.masks):
+        y, n = run_sparse_conv(w.x, hc.HC_LAYOUT_DENSE, m, w.spiral, ly.W, ly.b, ly.act)
+        c, r, _, n_ref = oracle.mask_compact(m)
+        assert n == n_ref
+        rows = sample_rows(n, 600, seed=2)
+        y_pre, _ = oracle.sparse_spiral_conv(w.x, oracle.LAYOUT_DENSE, c, r, w.spiral, ly.W, ly.b,
+                                             ly.act, rows=rows, n_threads=NCPU)
+        check_close(y[rows], y_pre, f"sweep density {d}")
+    yd = torch.empty((B, V, ly.C_out), dtype=torch.bfloat16, device="cuda")
+    hc.hc_spiral_conv_fwd(xt, to_torch(w.spiral), to_torch(ly.W), to_torch(ly.b), ly.act, yd)
+    assert hc.hc_get_device_status() == hc.HC_OK
+    rows = sample_rows(B * V, 1500, seed=3)
+    y_pre, _ = oracle.dense_spiral_conv(w.x, w.spiral, ly.W, ly.b, ly.act, rows=rows,
+                                        n_threads=NCPU)
+    check_close(to_numpy(yd).reshape(B * V, -1)[rows], y_pre, "dense full size")
+
+
+# ------------------------------------------------------------------ device status
+
+def test_out_of_range_spiral_entry_is_reported():
+    """A spiral entry outside [-1, V) is caught by the kernel's own bounds
+    check: the tap contributes nothing and HC_ERR_INVALID_INDEX is raised."""
+    for C_out in (64, 42):  # tensor-core path and CUDA-core path
+        sp, m, x, W, b = inputs.random_case(40 + C_out, 2, 100, 5, 16, C_out, "bf16", 1.0)
+        sp[3, 2] = 100  # == V: out of range
+        sp[7, 1] = -5
+        coords, row_of, _, count = gpu_compact(m)
+        out = torch.empty((200, C_out), dtype=torch.bfloat16, device="cuda")
+        hc.hc_sparse_spiral_conv_fwd(to_torch(x), hc.HC_LAYOUT_DENSE, coords, row_of, count,
+                                     to_torch(sp), 2, 100, to_torch(W), to_torch(b),
+                                     hc.HC_ACT_ELU, out)
+        assert hc.hc_get_device_status() == hc.HC_ERR_INVALID_INDEX
+        assert hc.hc_get_device_status() == hc.HC_OK  # reading clears it
+
+
+def test_count_above_capacity_is_reported():
+    x = torch.zeros((10, 16), dtype=torch.bfloat16, device="cuda")
+    W = torch.zeros((16, 16), dtype=torch.bfloat16, device="cuda")
+    y = torch.zeros((10, 16), dtype=torch.bfloat16, device="cuda")
+    count = torch.tensor([11], dtype=torch.int32, device="cuda")
+    hc.hc_sparse_linear_fwd(x, count, W, None, hc.HC_ACT_NONE, y)
+    assert hc.hc_get_device_status() == hc.HC_ERR_CAPACITY
+
+
+def test_host_rejects_bad_arguments():
+    x = torch.zeros((4, 16), dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(hc.HcError) as e:
+        hc.hc_sparse_linear_fwd(x, None, x, None, hc.HC_ACT_NONE, x)
+    assert e.value.status == hc.HC_ERR_INVALID_ARG
