@@ -60,13 +60,59 @@ __global__ void __launch_bounds__(kThreads) conv_simt_kernel(const ConvArgs a) {
     for (long long mt = blockIdx.x; mt < m_tiles; mt += gridDim.x) {
         const long long m0 = mt * kBM;
         __syncthreads();  // the previous tile is done with src_tab
-        for (int e = tid; e < kBM * L; e += kThreads) {
-            const int r = e / L, l = e - r * L;
+        {
+            // Four threads per row, slots l = part + 4*j: the coordinate, the
+            // spiral entries and the row_of lookups are each issued together
+            // (three dependent round trips per tile).
+            const int r = tid >> 2, part = tid & 3;
             const long long n = m0 + r;
-            long long src = -1;
-            int b, v;
-            if (n < rows && row_coord(a, n, b, v)) src = tap_row(a, n, b, v, l, rows);
-            src_tab[e] = (int)src;
+            const bool in = n < rows;
+            const long long nn = in ? n : 0;
+            unsigned err = 0;
+            int b = 0, v = 0;
+            if (a.mode == kSparseDenseX || a.mode == kSparseCompactX) {
+                b = __ldg(a.coords + 2 * nn);
+                v = __ldg(a.coords + 2 * nn + 1);
+            } else if (a.mode == kDense) {
+                b = (int)(nn / a.V);
+                v = (int)(nn - (long long)b * a.V);
+            }
+            const bool in_range = b >= 0 && b < a.B && v >= 0 && v < a.V;
+            if (in && !in_range) err |= kErrIndex;
+            const bool ok = in && in_range;
+            if (!ok) b = v = 0;
+            const bool linear = a.mode == kLinear;
+            // Loads from clamped, always-valid addresses first; checks after.
+            int u[HC_MAX_SPIRAL / 4];
+#pragma unroll
+            for (int j = 0; j < HC_MAX_SPIRAL / 4; ++j) {
+                const int l = part + 4 * j < L ? part + 4 * j : L - 1;
+                u[j] = linear ? 0 : __ldg(a.spiral + (long long)v * L + l);
+            }
+#pragma unroll
+            for (int j = 0; j < HC_MAX_SPIRAL / 4; ++j) {
+                const int l = part + 4 * j;
+                if (l >= L) continue;
+                int src = -1;
+                if (ok && linear) {
+                    src = (int)n;
+                } else if (ok) {
+                    const int uu = u[j];
+                    if (uu < -1 || uu >= a.V) err |= kErrIndex;
+                    if (uu >= 0 && uu < a.V) {
+                        const long long dr = (long long)b * a.V + uu;
+                        if (a.mode == kDense) {
+                            src = (int)dr;
+                        } else {
+                            const int jj = __ldg(a.row_of + dr);
+                            if (jj < -1 || jj >= rows) err |= kErrIndex;
+                            if (jj >= 0 && jj < rows) src = a.mode == kSparseDenseX ? (int)dr : jj;
+                        }
+                    }
+                }
+                src_tab[r * L + l] = src;
+            }
+            if (err) report(a.status, err);
         }
         __syncthreads();
 

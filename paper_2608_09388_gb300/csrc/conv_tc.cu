@@ -7,11 +7,15 @@
 // (zeros for absent taps, Eq. 4); the layer computes A * W + bias (Eq. 5 with
 // the bias of Eq. 6) and the activation of Eq. 10.
 //
-// One persistent CTA per SM, 288 threads in three roles:
-//   warps 0-3  producers: gather 128 rows x 64 bf16 of A and the 64 x BN
-//              slice of W per k-block into a 128-byte-swizzled stage with
-//              16-byte cp.async (zero-fill for absent taps and ragged edges),
-//              then publish the stage on its "full" mbarrier;
+// One persistent CTA per SM, 320 threads in four roles:
+//   warp 9     index warp: for each tile, resolves the 128 x L tap table
+//              (coords -> spiral -> row_of, i.e. idx() of Eq. 4) with every
+//              load of a phase in flight at once, into one of two tables, so
+//              the next tile's table is built while the current one is used;
+//   warps 0-3  producers: gather 128 rows x 64 bf16 of A through the table
+//              and the 64 x BN slice of W per k-block into a 128-byte-swizzled
+//              stage with 16-byte cp.async (zero-fill for absent taps and
+//              ragged edges), then publish the stage on its "full" mbarrier;
 //   warp 8     MMA issuer (one thread): 4 x tcgen05.mma (K = 16 each) per
 //              stage into a TMEM accumulator, tcgen05.commit frees the stage;
 //   warps 4-7  epilogue: tcgen05.ld the 128 x BN fp32 accumulator (warp w
@@ -41,7 +45,9 @@ constexpr int kAStageBytes = kBM * kBK * 2;
 constexpr int kProducerWarps = 4;
 constexpr int kEpilogueWarps = 4;
 constexpr int kMmaWarp = kProducerWarps + kEpilogueWarps;
-constexpr int kThreads = (kMmaWarp + 1) * 32;
+constexpr int kIndexWarp = kMmaWarp + 1;
+constexpr int kThreads = (kIndexWarp + 1) * 32;
+constexpr int kTabChunk = 8;  // spiral slots resolved per pass of the index warp
 
 template <int BN>
 struct Cfg {
@@ -54,10 +60,10 @@ struct Cfg {
     // N >> 3 at bits 17-22, M >> 4 at bits 24-28.
     static constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | (1u << 16) |
                                        ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(kBM >> 4) << 24);
-    static constexpr int kBarBytes = 8 * (2 * kStages + 5);
+    static constexpr int kBarBytes = 8 * (2 * kStages + 9);
     static size_t smem_bytes(int L) {
         return 1024 + (size_t)kStages * (kAStageBytes + kBStageBytes) + kBarBytes + 16 +
-               sizeof(int) * (size_t)kBM * L;
+               2 * sizeof(int) * (size_t)kBM * L;
     }
 };
 
@@ -82,13 +88,15 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const ConvArgs a) 
     uint8_t* const misc = base_ptr + (sBar - base) + C::kBarBytes;
     volatile uint32_t* const tmem_holder = reinterpret_cast<volatile uint32_t*>(misc);
     volatile int* const abort_flag = reinterpret_cast<volatile int*>(misc + 4);
-    int* const src_tab = reinterpret_cast<int*>(misc + 16);  // [kBM][L]
+    int* const tab_base = reinterpret_cast<int*>(misc + 16);  // [2][kBM][L]
 
     auto full_bar = [&](int s) { return sBar + 8u * s; };
     auto empty_bar = [&](int s) { return sBar + 8u * (C::kStages + s); };
     auto tfull_bar = [&](int i) { return sBar + 8u * (2 * C::kStages + i); };
     auto tempty_bar = [&](int i) { return sBar + 8u * (2 * C::kStages + 2 + i); };
     const uint32_t fin_bar = sBar + 8u * (2 * C::kStages + 4);
+    auto tabfull_bar = [&](int i) { return sBar + 8u * (2 * C::kStages + 5 + i); };
+    auto tabempty_bar = [&](int i) { return sBar + 8u * (2 * C::kStages + 7 + i); };
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
@@ -102,6 +110,10 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const ConvArgs a) 
             mbar_init(tempty_bar(i), kEpilogueWarps * 32);
         }
         mbar_init(fin_bar, 1);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(tabfull_bar(i), 32);
+            mbar_init(tabempty_bar(i), kProducerWarps * 32);
+        }
         *abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
     }
@@ -127,23 +139,17 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const ConvArgs a) 
         const __nv_bfloat16* __restrict__ W = static_cast<const __nv_bfloat16*>(a.W);
         const int t = threadIdx.x;  // 0..127
         const int q = t & 7;        // A: 16-byte chunk of the 128-byte row
-        // This warp gathers rows r with r % 16 in [4*warp, 4*warp+4); lane
-        // fills the source table of one of them, so the table is warp-private.
-        const int tab_row = 4 * warp + (lane & 3) + 16 * (lane >> 2);
         long long it = 0;
+        int lt = 0;
         bool ok = true;
-        for (long long w = blockIdx.x; w < work_total && ok; w += gridDim.x) {
-            const long long m0 = (w / n_tiles) * kBM;
+        for (long long w = blockIdx.x; w < work_total && ok; w += gridDim.x, ++lt) {
             const int n0 = (int)(w % n_tiles) * BN;
-            __syncwarp();
-            {
-                const long long n = m0 + tab_row;
-                int b = 0, v = 0;
-                const bool valid = n < rows && row_coord(a, n, b, v);
-                for (int l = 0; l < L; ++l)
-                    src_tab[tab_row * L + l] = valid ? (int)tap_row(a, n, b, v, l, rows) : -1;
+            const int buf = lt & 1;
+            if (!mbar_wait(tabfull_bar(buf), (uint32_t)((lt >> 1) & 1), abort_flag, a.status)) {
+                ok = false;
+                break;
             }
-            __syncwarp();
+            const uint32_t tab_s = smem_u32(tab_base) + (uint32_t)(buf * kBM * L) * 4u;
             int l = (q * 8) / C_in;  // slot and channel of this thread's chunk at k-block 0
             int c = q * 8 - l * C_in;
             for (int kb = 0; kb < num_kb; ++kb) {
@@ -155,12 +161,18 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const ConvArgs a) 
                 }
                 const uint32_t a_st = sA + s * kAStageBytes;
                 const bool kval = kb * kBK + q * 8 < K;
+                // All eight table entries of this stage first, then the copies.
+                int src[8];
 #pragma unroll
                 for (int i = 0; i < 8; ++i) {
                     const int r = (t >> 3) + 16 * i;
-                    const int src = kval ? src_tab[r * L + l] : -1;
-                    const __nv_bfloat16* gp = x + (src >= 0 ? (long long)src * C_in + c : 0);
-                    cp_async_16(a_st + r * 128 + ((q ^ (r & 7)) << 4), gp, src >= 0);
+                    src[i] = kval ? lds_s32(tab_s + (uint32_t)(r * L + l) * 4u) : -1;
+                }
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const int r = (t >> 3) + 16 * i;
+                    const __nv_bfloat16* gp = x + (src[i] >= 0 ? (long long)src[i] * C_in + c : 0);
+                    cp_async_16(a_st + r * 128 + ((q ^ (r & 7)) << 4), gp, src[i] >= 0);
                 }
                 const uint32_t b_st = sB + s * C::kBStageBytes;
                 constexpr int kCpr = BN / 8;  // 16-byte chunks per W row slice
@@ -188,6 +200,8 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const ConvArgs a) 
                     ++l;
                 }
             }
+            // Addresses of this tile's copies are issued: the table is free.
+            mbar_arrive(tabempty_bar(buf));
         }
         cp_async_wait_all();
         fence_proxy_async_smem();
@@ -238,6 +252,111 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const ConvArgs a) 
             mbar_wait(fin_bar, 0, &no_abort, a.status);
         }
         __syncwarp();
+    } else if (warp == kIndexWarp) {
+        // ------------------------------------------------------------ index warp
+        // Lane handles rows lane + 32*i (i < 4) of the tile. Phase 1 loads the
+        // coordinates, phase 2 all spiral entries of a chunk of slots, phase 3
+        // all row_of lookups of that chunk: three dependent round trips per
+        // tile instead of one per slot.
+        int lt = 0;
+        for (long long w = blockIdx.x; w < work_total; w += gridDim.x, ++lt) {
+            const int buf = lt & 1;
+            if (!mbar_wait(tabempty_bar(buf), (uint32_t)(((lt >> 1) & 1) ^ 1), abort_flag,
+                           a.status))
+                break;
+            const long long m0 = (w / n_tiles) * kBM;
+            const uint32_t tab_s = smem_u32(tab_base) + (uint32_t)(buf * kBM * L) * 4u;
+            // Loads are issued unconditionally from clamped, always-valid
+            // addresses and checked afterwards, so that every load of a
+            // phase is in flight at once.
+            int bb[4], vv[4];
+            bool ok[4];
+            unsigned err = 0;
+            const bool sparse = a.mode == kSparseDenseX || a.mode == kSparseCompactX;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const long long n = m0 + lane + 32 * i;
+                const bool in = n < rows;
+                const long long nn = in ? n : 0;
+                if (sparse) {
+                    bb[i] = __ldg(a.coords + 2 * nn);
+                    vv[i] = __ldg(a.coords + 2 * nn + 1);
+                } else if (a.mode == kDense) {
+                    bb[i] = (int)(nn / a.V);
+                    vv[i] = (int)(nn - (long long)bb[i] * a.V);
+                } else {
+                    bb[i] = 0;
+                    vv[i] = 0;
+                }
+            }
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const long long n = m0 + lane + 32 * i;
+                const bool in_range = bb[i] >= 0 && bb[i] < a.B && vv[i] >= 0 && vv[i] < a.V;
+                ok[i] = n < rows && in_range;
+                if (n < rows && !in_range) err |= kErrIndex;
+                if (!ok[i]) {
+                    bb[i] = 0;
+                    vv[i] = 0;
+                }
+            }
+            if (a.mode == kLinear) {
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+                    sts_s32(tab_s + (uint32_t)(lane + 32 * i) * 4u,
+                            ok[i] ? (int)(m0 + lane + 32 * i) : -1);
+            } else {
+                for (int l0 = 0; l0 < L; l0 += kTabChunk) {
+                    int u[4][kTabChunk];
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+#pragma unroll
+                        for (int d = 0; d < kTabChunk; ++d) {
+                            const int lc = l0 + d < L ? l0 + d : L - 1;
+                            u[i][d] = __ldg(a.spiral + (long long)vv[i] * L + lc);
+                        }
+                    int dr[4][kTabChunk];  // dense row b*V + u (< 2^31), or -1
+                    int j[4][kTabChunk];
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+#pragma unroll
+                        for (int d = 0; d < kTabChunk; ++d) {
+                            const int uu = u[i][d];
+                            const bool live = ok[i] && l0 + d < L;
+                            if (live && (uu < -1 || uu >= a.V)) err |= kErrIndex;
+                            const bool tap = live && uu >= 0 && uu < a.V;
+                            dr[i][d] = tap ? bb[i] * a.V + uu : -1;
+                        }
+                    if (sparse) {
+#pragma unroll
+                        for (int i = 0; i < 4; ++i)
+#pragma unroll
+                            for (int d = 0; d < kTabChunk; ++d)
+                                j[i][d] = __ldg(a.row_of + (dr[i][d] >= 0 ? dr[i][d] : 0));
+                    }
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+#pragma unroll
+                        for (int d = 0; d < kTabChunk; ++d) {
+                            if (l0 + d >= L) continue;
+                            int src = -1;
+                            if (dr[i][d] >= 0) {
+                                if (!sparse) {
+                                    src = dr[i][d];
+                                } else {
+                                    const int jj = j[i][d];
+                                    if (jj < -1 || jj >= rows) err |= kErrIndex;
+                                    if (jj >= 0 && jj < rows)
+                                        src = a.mode == kSparseDenseX ? dr[i][d] : jj;
+                                }
+                            }
+                            sts_s32(tab_s + (uint32_t)((lane + 32 * i) * L + l0 + d) * 4u, src);
+                        }
+                }
+            }
+            if (err) report(a.status, err);
+            mbar_arrive(tabfull_bar(buf));
+        }
     } else {
         // ------------------------------------------------------------ epilogue
         const int ew = warp - kProducerWarps;  // == warp % 4: TMEM lanes 32*ew..+32
@@ -259,29 +378,28 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const ConvArgs a) 
                                    r);
                 tmem_ld_wait();
                 const int col0 = n0 + cb * 32;
-                if (rvalid) {
-                    __nv_bfloat16* yp = y + row * C_out + col0;
+                // Bias of the chunk's 32 columns: one coalesced load, then
+                // broadcast by shuffles.
+                const int bcol = col0 + lane < C_out ? col0 + lane : C_out - 1;
+                const float bias_l = a.bias ? __ldg(a.bias + bcol) : 0.f;
+                __nv_bfloat16* yp = y + (rvalid ? row : 0) * C_out + col0;
 #pragma unroll
-                    for (int j8 = 0; j8 < 4; ++j8) {
-                        if (col0 + j8 * 8 < C_out) {
-                            uint32_t packed[4];
+                for (int j8 = 0; j8 < 4; ++j8) {
+                    uint32_t packed[4];
 #pragma unroll
-                            for (int h = 0; h < 4; ++h) {
-                                const int j = j8 * 8 + 2 * h;
-                                float z0 = __uint_as_float(r[j]);
-                                float z1 = __uint_as_float(r[j + 1]);
-                                if (a.bias) {
-                                    z0 += __ldg(a.bias + col0 + j);
-                                    z1 += __ldg(a.bias + col0 + j + 1);
-                                }
-                                const __nv_bfloat162 p =
-                                    __floats2bfloat162_rn(act_apply(z0, a.act), act_apply(z1, a.act));
-                                packed[h] = *reinterpret_cast<const uint32_t*>(&p);
-                            }
-                            *reinterpret_cast<uint4*>(yp + j8 * 8) =
-                                make_uint4(packed[0], packed[1], packed[2], packed[3]);
-                        }
+                    for (int h = 0; h < 4; ++h) {
+                        // every lane takes part in the shuffles
+                        const int j = j8 * 8 + 2 * h;
+                        const float z0 = __uint_as_float(r[j]) + __shfl_sync(0xffffffffu, bias_l, j);
+                        const float z1 =
+                            __uint_as_float(r[j + 1]) + __shfl_sync(0xffffffffu, bias_l, j + 1);
+                        const __nv_bfloat162 p =
+                            __floats2bfloat162_rn(act_apply(z0, a.act), act_apply(z1, a.act));
+                        packed[h] = *reinterpret_cast<const uint32_t*>(&p);
                     }
+                    if (rvalid && col0 + j8 * 8 < C_out)
+                        *reinterpret_cast<uint4*>(yp + j8 * 8) =
+                            make_uint4(packed[0], packed[1], packed[2], packed[3]);
                 }
             }
             tc_fence_before();

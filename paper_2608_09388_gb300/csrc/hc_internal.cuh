@@ -96,9 +96,10 @@ __device__ __forceinline__ long long active_rows(const ConvArgs& a) {
     return n;
 }
 
-// Output row n -> coordinate (b, v). Returns false (and reports) for an
-// out-of-range coordinate; linear rows have no coordinate (b = v = 0).
-__device__ __forceinline__ bool row_coord(const ConvArgs& a, long long n, int& b, int& v) {
+// Output row n -> coordinate (b, v). Returns false (setting kErrIndex in
+// `err`) for an out-of-range coordinate; linear rows have no coordinate.
+__device__ __forceinline__ bool row_coord(const ConvArgs& a, long long n, int& b, int& v,
+                                          unsigned& err) {
     if (a.mode == kDense) {
         b = (int)(n / a.V);
         v = (int)(n - (long long)b * a.V);
@@ -112,42 +113,66 @@ __device__ __forceinline__ bool row_coord(const ConvArgs& a, long long n, int& b
     b = __ldg(a.coords + 2 * n);
     v = __ldg(a.coords + 2 * n + 1);
     if (b < 0 || b >= a.B || v < 0 || v >= a.V) {
-        report(a.status, kErrIndex);
+        err |= kErrIndex;
         return false;
     }
     return true;
 }
 
-// Input row that feeds spiral slot l of output row n at (b, v), or -1 when
-// the tap is absent (no neighbour, or the neighbour is not an active row).
-// This is idx() of Eq. 4 for the sparse modes.
-__device__ __forceinline__ long long tap_row(const ConvArgs& a, long long n, int b, int v, int l,
-                                             long long n_rows) {
-    if (a.mode == kLinear) return n;
+// The helpers below never write memory: they return an error bit instead
+// (kErrIndex), which callers OR together and report once. A global atomic
+// between loads would stop the compiler from issuing the loads of many taps
+// back to back.
+
+// Spiral entry of slot l of vertex v (-1 = no neighbour). Out-of-range
+// entries read as -1 and set kErrIndex in `err`.
+__device__ __forceinline__ int load_spiral(const ConvArgs& a, int v, int l, unsigned& err) {
     int u = __ldg(a.spiral + (long long)v * a.L + l);
-    if (u == -1) return -1;
     if (u < -1 || u >= a.V) {
-        report(a.status, kErrIndex);
+        err |= kErrIndex;
         return -1;
     }
+    return u;
+}
+
+// Input row for neighbour vertex u of output row n at frame b, or -1 when the
+// tap is absent (no neighbour, or the neighbour is not an active row). This
+// is idx() of Eq. 4 for the sparse modes.
+__device__ __forceinline__ long long resolve_tap(const ConvArgs& a, long long n, int b, int u,
+                                                 long long n_rows, unsigned& err) {
+    if (a.mode == kLinear) return n;
+    if (u < 0) return -1;
     long long dense_row = (long long)b * a.V + u;
     if (a.mode == kDense) return dense_row;
     int j = __ldg(a.row_of + dense_row);
     if (j < 0) {
-        if (j != -1) report(a.status, kErrIndex);
+        if (j != -1) err |= kErrIndex;
         return -1;
     }
     if (j >= n_rows) {
-        report(a.status, kErrIndex);
+        err |= kErrIndex;
         return -1;
     }
     return a.mode == kSparseDenseX ? dense_row : (long long)j;
 }
 
+// Activation of Eq. 10. ELU(z) = z for z > 0, else exp(z) - 1, evaluated
+// with the fast exponential: the absolute error is a few 1e-7, far inside the
+// fp32 (1e-4 absolute) and bf16 (2e-2 relative) tolerances of this library.
 __device__ __forceinline__ float act_apply(float z, int act) {
-    if (act == HC_ACT_ELU) return z > 0.f ? z : expm1f(z);
+    if (act == HC_ACT_ELU) return z > 0.f ? z : __expf(z) - 1.0f;
     if (act == HC_ACT_RELU) return z > 0.f ? z : 0.f;
     return z;
+}
+
+// Explicit shared-memory accesses (32-bit shared addresses).
+__device__ __forceinline__ int lds_s32(uint32_t addr) {
+    int v;
+    asm volatile("ld.shared.b32 %0, [%1];\n" : "=r"(v) : "r"(addr));
+    return v;
+}
+__device__ __forceinline__ void sts_s32(uint32_t addr, int v) {
+    asm volatile("st.shared.b32 [%0], %1;\n" ::"r"(addr), "r"(v) : "memory");
 }
 
 __device__ __forceinline__ unsigned long long globaltimer_ns() {
