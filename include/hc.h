@@ -89,6 +89,35 @@ hc_status hc_mask_compact(const uint8_t* mask, int B, int V, int32_t* coords,
                           hc_stream_t stream);
 
 /*
+ * hc_mask_compact_static -- hc_mask_compact that allocates nothing. The paper
+ * has no counterpart; this entry point exists for callers of this library
+ * that cannot allocate device memory at the moment they compact a mask:
+ * code running while a stream is being captured into a CUDA graph (a
+ * cudaMalloc there breaks the capture), and processes that hand all device
+ * memory to their own pool up front and must not allocate behind its back.
+ *
+ * Same arguments, results and errors as hc_mask_compact (bit-identical
+ * outputs). Differences:
+ *  - Scratch: a fixed array of HC_STATIC_MAX_MASK_BYTES / 4096 int32 (16 KiB)
+ *    inside the library's device image, present on every GPU that loads the
+ *    library until the process exits. No cudaMalloc, cudaFree or allocating
+ *    library routine is called.
+ *  - Limit: B*V may not exceed HC_STATIC_MAX_MASK_BYTES; larger masks are
+ *    rejected with HC_ERR_UNSUPPORTED before anything is launched.
+ *  - Set-up: the first call on each device looks up the array's device
+ *    address (with that device current); make that first call before any
+ *    stream capture.
+ *  - Sharing: every call on a device uses the same array, which keeps the
+ *    previous call's contents (each call rewrites what it reads, so no
+ *    clearing is needed). Calls whose kernels overlap on the GPU (e.g. on
+ *    two streams without ordering between them) race on it.
+ */
+#define HC_STATIC_MAX_MASK_BYTES (4096 * 4096)
+hc_status hc_mask_compact_static(const uint8_t* mask, int B, int V, int32_t* coords,
+                                 int32_t* row_of, int32_t* batch_offsets, int32_t* count,
+                                 hc_stream_t stream);
+
+/*
  * hc_sparse_spiral_conv_fwd -- sparse convolution on the spiral
  * neighbourhood (Eqs. 4-5) with fused bias (Eq. 6) and activation (Eq. 10).
  *

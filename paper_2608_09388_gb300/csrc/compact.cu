@@ -12,6 +12,8 @@
 // Neither pass waits on another CTA, so there is no inter-CTA spin. The
 // mask is read with 16-byte loads; HBM traffic is 2 reads of the mask plus
 // the writes (8 B per active row, 4 B per row_of entry).
+#include <mutex>
+
 #include "hc_internal.cuh"
 
 namespace hc {
@@ -244,3 +246,107 @@ hc_status launch_compact(const DeviceCtx* ctx, const uint8_t* mask, int B, int V
 }
 
 }  // namespace hc
+
+// ---------------------------------------------------------------------------
+// hc_mask_compact_static: the same compaction for callers that cannot
+// allocate device memory. Its scratch (one int32 per 4096-byte mask tile) is
+// a fixed array in the library's device image instead of a cudaMalloc'd
+// workspace, so it serves masks of at most kStaticMaxTiles * 4096 bytes.
+// ---------------------------------------------------------------------------
+namespace hc {
+namespace {
+
+constexpr int kStaticMaxTiles = 4096;  // 16 KiB of scratch per device
+static_assert((long long)kStaticMaxTiles * kTile == HC_STATIC_MAX_MASK_BYTES,
+              "header limit and scratch size disagree");
+
+// Every GPU that loads the library holds this array until the process exits.
+// All calls on a device share it: it keeps the previous call's tile counts,
+// and two calls whose kernels overlap on the GPU would race on it.
+static __device__ __align__(256) int32_t g_static_tile_counts[kStaticMaxTiles];
+
+constexpr int kMaxStaticDevices = 64;
+int32_t* g_static_ptr[kMaxStaticDevices];
+std::mutex g_static_mutex;
+
+// Device address of the array for the current device. In host code the
+// array's name is only a host-side stand-in, so the address is looked up
+// once per device (with that device current) and cached.
+hc_status static_scratch(int32_t** out) {
+    int dev = -1;
+    hc_status st = check_cuda(cudaGetDevice(&dev), "cudaGetDevice");
+    if (st != HC_OK) return st;
+    if (dev < 0 || dev >= kMaxStaticDevices) {
+        set_error("device ordinal %d out of range", dev);
+        return HC_ERR_CUDA;
+    }
+    std::lock_guard<std::mutex> lock(g_static_mutex);
+    if (!g_static_ptr[dev]) {
+        void* p = nullptr;
+        st = check_cuda(cudaGetSymbolAddress(&p, g_static_tile_counts),
+                        "cudaGetSymbolAddress(static compaction scratch)");
+        if (st != HC_OK) return st;
+        g_static_ptr[dev] = static_cast<int32_t*>(p);
+    }
+    *out = g_static_ptr[dev];
+    return HC_OK;
+}
+
+// The count / (scan) / write passes into caller-chosen scratch. Every tile's
+// count is rewritten before it is read, so nothing has to be cleared first.
+hc_status launch_compact_into(const uint8_t* mask, int B, int V, int32_t* coords,
+                              int32_t* row_of, int32_t* offsets, int32_t* count,
+                              int32_t* tile_counts, cudaStream_t s) {
+    long long n = (long long)B * V;
+    if (n == 0) {
+        compact_empty_kernel<<<1, 256, 0, s>>>(B, offsets, count);
+        return check_cuda(cudaGetLastError(), "compact_empty_kernel");
+    }
+    int num_tiles = (int)((n + kTile - 1) / kTile);
+    compact_count_kernel<<<num_tiles, kThreads, 0, s>>>(mask, n, tile_counts);
+    hc_status st = check_cuda(cudaGetLastError(), "compact_count_kernel");
+    if (st != HC_OK) return st;
+    int prescanned = num_tiles > kMaxDirectTiles;
+    if (prescanned) {
+        compact_scan_kernel<<<1, 1024, 0, s>>>(tile_counts, num_tiles);
+        st = check_cuda(cudaGetLastError(), "compact_scan_kernel");
+        if (st != HC_OK) return st;
+    }
+    compact_write_kernel<<<num_tiles, kThreads, 0, s>>>(mask, n, B, V, tile_counts, num_tiles,
+                                                        prescanned, coords, row_of, offsets, count);
+    return check_cuda(cudaGetLastError(), "compact_write_kernel");
+}
+
+}  // namespace
+}  // namespace hc
+
+extern "C" hc_status hc_mask_compact_static(const uint8_t* mask, int B, int V, int32_t* coords,
+                                            int32_t* row_of, int32_t* batch_offsets,
+                                            int32_t* count, hc_stream_t stream) {
+    using namespace hc;
+    set_error("%s", "");
+    if (B < 0 || V < 0) {
+        set_error("hc_mask_compact_static: B=%d V=%d must be >= 0", B, V);
+        return HC_ERR_INVALID_ARG;
+    }
+    if (count == nullptr) {
+        set_error("hc_mask_compact_static: count is NULL");
+        return HC_ERR_INVALID_ARG;
+    }
+    const long long n = (long long)B * V;
+    if (n > 0 && (mask == nullptr || coords == nullptr)) {
+        set_error("hc_mask_compact_static: mask and coords are required");
+        return HC_ERR_INVALID_ARG;
+    }
+    if (n > HC_STATIC_MAX_MASK_BYTES) {
+        set_error("hc_mask_compact_static: B*V = %lld exceeds the fixed scratch limit of %d mask "
+                  "bytes; use hc_mask_compact",
+                  n, HC_STATIC_MAX_MASK_BYTES);
+        return HC_ERR_UNSUPPORTED;
+    }
+    int32_t* scratch = nullptr;
+    hc_status st = static_scratch(&scratch);
+    if (st != HC_OK) return st;
+    return launch_compact_into(mask, B, V, coords, row_of, batch_offsets, count, scratch,
+                               (cudaStream_t)stream);
+}

@@ -21,14 +21,15 @@ HC_F32, HC_BF16 = 0, 1
 HC_ACT_NONE, HC_ACT_ELU, HC_ACT_RELU = 0, 1, 2
 HC_LAYOUT_DENSE, HC_LAYOUT_COMPACT = 0, 1
 HC_MAX_SPIRAL = 32
+HC_STATIC_MAX_MASK_BYTES = 4096 * 4096
 
 STATUS_NAMES = {0: "HC_OK", 1: "HC_ERR_INVALID_ARG", 2: "HC_ERR_UNSUPPORTED",
                 3: "HC_ERR_CAPACITY", 4: "HC_ERR_INVALID_INDEX", 5: "HC_ERR_TIMEOUT",
                 6: "HC_ERR_CUDA"}
 
 # Exported symbols, as declared in include/hc.h.
-EXPORTS = ("hc_mask_compact", "hc_sparse_spiral_conv_fwd", "hc_sparse_linear_fwd",
-           "hc_scatter_dense", "hc_spiral_conv_fwd", "hc_get_device_status",
+EXPORTS = ("hc_mask_compact", "hc_mask_compact_static", "hc_sparse_spiral_conv_fwd",
+           "hc_sparse_linear_fwd", "hc_scatter_dense", "hc_spiral_conv_fwd", "hc_get_device_status",
            "hc_last_error_string", "hc_version")
 
 
@@ -55,6 +56,7 @@ def load_library(path: str | None = None):
         P, I = ctypes.c_void_p, ctypes.c_int
         sig = {
             "hc_mask_compact": [P, I, I, P, P, P, P, P],
+            "hc_mask_compact_static": [P, I, I, P, P, P, P, P],
             "hc_sparse_spiral_conv_fwd": [P, I, I, P, P, P, P, I, I, I, I, I, P, P, I, P, P],
             "hc_sparse_linear_fwd": [P, I, P, I, I, I, P, P, I, P, P],
             "hc_scatter_dense": [P, I, P, P, P, I, I, I, I, P, P],
@@ -110,6 +112,15 @@ def hc_mask_compact(mask, coords, row_of, batch_offsets, count, stream=None):
     _check(load_library().hc_mask_compact(_p(mask), B, V, _p(coords), _p(row_of),
                                           _p(batch_offsets), _p(count), _s(stream)),
            "hc_mask_compact")
+
+
+def hc_mask_compact_static(mask, coords, row_of, batch_offsets, count, stream=None):
+    """hc_mask_compact without any device allocation (fixed in-library
+    scratch; masks up to HC_STATIC_MAX_MASK_BYTES bytes)."""
+    B, V = mask.shape
+    _check(load_library().hc_mask_compact_static(_p(mask), B, V, _p(coords), _p(row_of),
+                                                 _p(batch_offsets), _p(count), _s(stream)),
+           "hc_mask_compact_static")
 
 
 def hc_sparse_spiral_conv_fwd(x, x_layout, coords, row_of, count, spiral, B, V, W, bias, act, y,
