@@ -10,6 +10,7 @@ Functions and the passages they follow:
 
 * ``mask_compact``         decomposition into coordinates C' (Eq. 2) and the
                            inverse map idx() (Eq. 4)
+* ``conv_rulebook``        the indexing matrix of Eq. 4 (tap -> input row)
 * ``sparse_spiral_conv``   sparse convolution on the spiral neighbourhood
                            (Eqs. 4-5), bias (Eq. 6) and activation (Eq. 10)
 * ``dense_spiral_conv``    the dense layer the sparse one replaces (Sec. 3.2)
@@ -78,6 +79,8 @@ def _load():
             lib.hco_sparse_linear.restype = None
             lib.hco_scatter_dense.argtypes = [P, I, P, I64, I64, I64, I, I, P]
             lib.hco_scatter_dense.restype = None
+            lib.hco_conv_rulebook.argtypes = [P, P, I64, P, I64, I, I, I64, P]
+            lib.hco_conv_rulebook.restype = None
             lib.hco_bf16_round.argtypes = [ctypes.c_double]
             lib.hco_bf16_round.restype = ctypes.c_uint16
             _lib = lib
@@ -117,6 +120,23 @@ def mask_compact(mask: np.ndarray):
     offsets = np.empty(B + 1, dtype=np.int32)
     n = _load().hco_mask_compact(_ptr(mask), B, V, _ptr(coords), _ptr(row_of), _ptr(offsets))
     return coords[:n].copy(), row_of, offsets, int(n)
+
+
+def conv_rulebook(coords, row_of, spiral, x_layout, stride=None):
+    """Eq. 4 mapping: int32 [L, stride] with entry (l, n) = the input row read
+    by slot l of output row n (dense row b*V+u, or compact row), -1 if absent.
+    Columns n >= N' are -1."""
+    coords = _c(coords, np.int32)
+    row_of = _c(row_of, np.int32)
+    spiral = _c(spiral, np.int32)
+    B, V = row_of.shape
+    L = spiral.shape[1]
+    n = coords.shape[0]
+    stride = B * V if stride is None else stride
+    rb = np.full((L, stride), -1, dtype=np.int32)
+    _load().hco_conv_rulebook(_ptr(coords), _ptr(row_of), n, _ptr(spiral), V, L, x_layout, stride,
+                              _ptr(rb))
+    return rb
 
 
 def _rows_arg(rows, n_default):

@@ -16,6 +16,7 @@
  * Functions (each cites the passage it follows):
  *   hco_mask_compact        decomposition into (C', S') coordinates, Eq. 2,
  *                           plus the inverse map idx() of Eq. 4
+ *   hco_conv_rulebook       the indexing matrix of Eq. 4 (tap -> input row)
  *   hco_sparse_spiral_conv  sparse convolution, Eqs. 4-5, with the spiral
  *                           neighbourhood of the POSA spiral blocks (Fig. 2)
  *                           and the activation of Eq. 10
@@ -127,6 +128,33 @@ int64_t hco_mask_compact(const uint8_t* mask, int64_t B, int64_t V,
     }
     offsets[B] = (int32_t)n;
     return n;
+}
+
+/* ------------------------------------------------------------- mapping */
+
+/* Eq. 4, materialised for the spiral neighbourhood: the indexing matrix that
+ * pairs every kernel tap of an output coordinate with the input row it reads.
+ * For output row n (coordinate (b, v) = C'[n]) and spiral slot l:
+ *     rulebook[l*stride + n] = idx(b, spiral[v][l])   if that tap is present,
+ *                            = -1                     otherwise,
+ * where the tap is present iff spiral[v][l] >= 0 and (b, spiral[v][l]) is an
+ * active row. idx() is the row of the input: b*V + u for a dense input, the
+ * compact position row_of[b, u] for a compact one. */
+void hco_conv_rulebook(const int32_t* coords, const int32_t* row_of, int64_t n_rows,
+                       const int32_t* spiral, int64_t V, int L, int x_layout, int64_t stride,
+                       int32_t* rulebook) {
+    for (int64_t n = 0; n < n_rows; ++n) {
+        int64_t b = coords[2 * n + 0], v = coords[2 * n + 1];
+        for (int l = 0; l < L; ++l) {
+            int64_t u = spiral[v * L + l];
+            int32_t e = -1;
+            if (u >= 0) {
+                int64_t j = row_of[b * V + u];
+                if (j >= 0) e = (int32_t)(x_layout == HCO_LAYOUT_DENSE ? b * V + u : j);
+            }
+            rulebook[(int64_t)l * stride + n] = e;
+        }
+    }
 }
 
 /* --------------------------------------------------- sparse spiral conv */

@@ -95,6 +95,11 @@ def check_golden_cases():
         if "y_rows" in case:
             for k, v in case["y_rows"].items():
                 np.testing.assert_array_equal(y_pre[int(k)], np.array(v, dtype=np.float64))
+        if "rulebook_compact" in case:
+            for lay, key in ((oracle.LAYOUT_COMPACT, "rulebook_compact"),
+                             (oracle.LAYOUT_DENSE, "rulebook_dense")):
+                rb = oracle.conv_rulebook(coords, row_of, sp, lay, stride=n)
+                np.testing.assert_array_equal(rb, case[key])
     d = g["dense_full_input"]
     sp = np.array(g["spiral_L3"], dtype=np.int32)
     y_pre, _ = oracle.dense_spiral_conv(np.array(d["x"], np.float32), sp,
@@ -128,6 +133,24 @@ def check_conv_vs_gather_matmul(seed=3, B=3, V=40, L=5, C_in=6, C_out=7, density
 
 def test_conv_vs_gather_matmul():
     check_conv_vs_gather_matmul()
+
+
+def test_rulebook_gather_matmul_equals_conv():
+    """Eq. 5 evaluated through the Eq. 4 rulebook with numpy (gather the rows
+    the rulebook names, zero for -1, one fp64 matmul) equals the loop conv,
+    for both input layouts."""
+    sp, m, x, W, b = inputs.random_case(21, 3, 70, 7, 5, 6, "f32", 0.4, neg_frac=0.15)
+    coords, row_of, offsets, n = oracle.mask_compact(m)
+    y_ref, _ = oracle.sparse_spiral_conv(x, oracle.LAYOUT_DENSE, coords, row_of, sp, W, b,
+                                         oracle.ACT_NONE)
+    xc = x[coords[:, 0], coords[:, 1]]
+    for lay, xs in ((oracle.LAYOUT_DENSE, x.reshape(-1, 5)), (oracle.LAYOUT_COMPACT, xc)):
+        rb = oracle.conv_rulebook(coords, row_of, sp, lay)
+        assert (rb[:, n:] == -1).all()
+        xz = np.concatenate([xs.astype(np.float64), np.zeros((1, 5))])
+        G = xz[np.where(rb[:, :n] >= 0, rb[:, :n], xs.shape[0])]  # [L, n, C_in]
+        G = G.transpose(1, 0, 2).reshape(n, -1)
+        np.testing.assert_allclose(G @ W.astype(np.float64) + b, y_ref, rtol=1e-12, atol=1e-12)
 
 
 def test_conv_L1_is_matmul():
@@ -331,6 +354,8 @@ MUTANTS = {
                          "for (int64_t b = B - 1; b >= 0; --b) {\n        offsets[b] = (int32_t)n;\n        for (int64_t v = 0; v < V; ++v) {"),
     "bf16 rounded through float32": ("double n = nearbyint(ldexp(x, -qexp));",
                                      "double n = nearbyint(ldexp((double)(float)x, -qexp));"),
+    "rulebook ignores activity": ("                if (j >= 0) e = (int32_t)(x_layout == HCO_LAYOUT_DENSE ? b * V + u : j);",
+                                  "                e = (int32_t)(x_layout == HCO_LAYOUT_DENSE ? b * V + u : j);"),
     "centre tap dropped": ("for (int l = 0; l < L; ++l) {\n            int64_t u = spiral[v * L + l];\n            if (u < 0) continue; /* no neighbour in this slot */",
                            "for (int l = 1; l < L; ++l) {\n            int64_t u = spiral[v * L + l];\n            if (u < 0) continue; /* no neighbour in this slot */"),
 }
@@ -353,7 +378,7 @@ def test_planted_mistake_is_caught(name, tmp_path, monkeypatch):
     good = oracle._load()
     lib = ctypes.CDLL(str(so))
     for fn in ("hco_mask_compact", "hco_sparse_spiral_conv", "hco_dense_spiral_conv",
-               "hco_sparse_linear", "hco_scatter_dense", "hco_bf16_round"):
+               "hco_sparse_linear", "hco_scatter_dense", "hco_bf16_round", "hco_conv_rulebook"):
         getattr(lib, fn).argtypes = getattr(good, fn).argtypes
         getattr(lib, fn).restype = getattr(good, fn).restype
     monkeypatch.setattr(oracle, "_lib", lib)
