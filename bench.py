@@ -4,9 +4,10 @@
 One step = one pass of the hot path over one batch of the 10475-vertex
 workload (B = 32 frames, spiral length L = 12, 64 -> 128 channels, bf16,
 clustered contact masks at ~5% density):
-    hc_mask_compact           mask -> coords, row_of, offsets, count
-    hc_sparse_spiral_conv_fwd gather + tcgen05 contraction + bias + ELU
-    hc_scatter_dense          compact rows -> dense [B, V, 128]
+    hc_mask_compact              mask -> coords, row_of, offsets, count (Eq. 2)
+    hc_conv_rulebook             tap -> input-row mapping (Eq. 4)
+    hc_sparse_conv_rulebook_fwd  gather + tcgen05 contraction + bias + ELU (Eq. 5)
+    hc_scatter_dense             compact rows -> dense [B, V, 128]
 Inputs are resident in HBM; every step reads its own input set (mask and
 features) from a rotation whose total size is more than twice the L2, so
 consecutive steps do not hit in L2. The timed steps are replayed from CUDA
@@ -185,6 +186,7 @@ def build_sets(torch, w, R, seed_base, dev):
         s.row_of = torch.empty((B, V), dtype=torch.int32, device=dev)
         s.offs = torch.empty((B + 1,), dtype=torch.int32, device=dev)
         s.count = torch.empty((1,), dtype=torch.int32, device=dev)
+        s.rb = torch.empty((w.L, B * V), dtype=torch.int32, device=dev)
         s.y = torch.empty((B * V, ly.C_out), dtype=torch.bfloat16, device=dev)
         s.out = torch.zeros((B, V, ly.C_out), dtype=torch.bfloat16, device=dev)
         sets.append(s)
@@ -211,7 +213,7 @@ def run_ours(args, rank, world, local_rank):
     w = inputs.make_workload(WORKLOAD)
     ly = w.layers[0]
     B, V, L = w.B, w.V, w.L
-    set_bytes = B * V * (1 + 2 * ly.C_in)
+    set_bytes = B * V * (1 + 2 * ly.C_in)  # mask + features read by a step
     R = max(4, math.ceil(2.5 * l2 / set_bytes))
     sets = build_sets(torch, w, R, inputs.SEEDS[WORKLOAD] + 1000 * rank, dev)
     spiral = torch.from_numpy(w.spiral).to(dev)
@@ -221,18 +223,19 @@ def run_ours(args, rank, world, local_rank):
 
     def step(s):
         hc.hc_mask_compact(s.mask, s.coords, s.row_of, s.offs, s.count, stream)
-        hc.hc_sparse_spiral_conv_fwd(s.x, hc.HC_LAYOUT_DENSE, s.coords, s.row_of, s.count, spiral,
-                                     B, V, Wt, bias, ly.act, s.y, stream)
+        hc.hc_conv_rulebook(s.coords, s.row_of, s.count, spiral, B, V, hc.HC_LAYOUT_DENSE, s.rb,
+                            stream)
+        hc.hc_sparse_conv_rulebook_fwd(s.x, s.rb, s.count, Wt, bias, ly.act, s.y, stream)
         hc.hc_scatter_dense(s.y, s.coords, s.row_of, s.count, B, V, 0, s.out, stream)
 
     def conv_only(s):
-        hc.hc_sparse_spiral_conv_fwd(s.x, hc.HC_LAYOUT_DENSE, s.coords, s.row_of, s.count, spiral,
-                                     B, V, Wt, bias, ly.act, s.y, stream)
+        hc.hc_sparse_conv_rulebook_fwd(s.x, s.rb, s.count, Wt, bias, ly.act, s.y, stream)
 
     def dense_only(s):
         hc.hc_spiral_conv_fwd(s.x, spiral, Wt, bias, ly.act, s.dense, stream)
 
-    kernels_per_step = 2 + (1 if (B * V + 4095) // 4096 > 1024 else 0) + 1 + 1
+    # compaction (2, or 3 with the pre-scan), rulebook, conv, scatter
+    kernels_per_step = 2 + (1 if (B * V + 4095) // 4096 > 1024 else 0) + 1 + 1 + 1
 
     # W warm-up steps, then one priming pass over every input set (both
     # eager, untimed; they also set up the library's per-stream workspace).
@@ -380,7 +383,8 @@ def run_ours(args, rank, world, local_rank):
             "active_rows_per_step": mean_rows,
             "rotation_sets": R,
             "launches_before_timed": (args.warmup + R) * kernels_per_step,
-            "step": "hc_mask_compact + hc_sparse_spiral_conv_fwd + hc_scatter_dense",
+            "step": "hc_mask_compact + hc_conv_rulebook + hc_sparse_conv_rulebook_fwd + "
+                    "hc_scatter_dense",
             "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
             "l2": f"{R} rotating input sets of {set_bytes / 2**20:.1f} MiB "
                   f"({R * set_bytes / 2**20:.0f} MiB > 2x L2 {l2 / 2**20:.0f} MiB)",
@@ -467,8 +471,9 @@ def measure_e2e(torch, hc, sets, w, spiral, Wt, bias, stream, dev, steps):
         mask_d.copy_(mh, non_blocking=True)
         x_d.copy_(xh, non_blocking=True)
         hc.hc_mask_compact(mask_d, s0.coords, s0.row_of, s0.offs, s0.count, stream)
-        hc.hc_sparse_spiral_conv_fwd(x_d, hc.HC_LAYOUT_DENSE, s0.coords, s0.row_of, s0.count,
-                                     spiral, B, V, Wt, bias, ly.act, s0.y, stream)
+        hc.hc_conv_rulebook(s0.coords, s0.row_of, s0.count, spiral, B, V, hc.HC_LAYOUT_DENSE,
+                            s0.rb, stream)
+        hc.hc_sparse_conv_rulebook_fwd(x_d, s0.rb, s0.count, Wt, bias, ly.act, s0.y, stream)
         hc.hc_scatter_dense(s0.y, s0.coords, s0.row_of, s0.count, B, V, 0, s0.out, stream)
         cnt_h.copy_(s0.count, non_blocking=True)
         stream.synchronize()
@@ -512,6 +517,7 @@ def run_sweep(torch, hc, dev, stream):
     row_of = torch.empty((B, V), dtype=torch.int32, device=dev)
     offs = torch.empty((B + 1,), dtype=torch.int32, device=dev)
     count = torch.empty((1,), dtype=torch.int32, device=dev)
+    rb = torch.empty((L, B * V), dtype=torch.int32, device=dev)
     pk = peaks()
 
     def timeit(fn, reps=20):
@@ -537,10 +543,11 @@ def run_sweep(torch, hc, dev, stream):
         mt = torch.from_numpy(m).to(dev)
         with torch.cuda.stream(stream):
             hc.hc_mask_compact(mt, coords, row_of, offs, count, stream)
+            hc.hc_conv_rulebook(coords, row_of, count, spiral, B, V, hc.HC_LAYOUT_DENSE, rb,
+                                stream)
         n = int(np.count_nonzero(m))
-        ms = timeit(lambda: hc.hc_sparse_spiral_conv_fwd(
-            x, hc.HC_LAYOUT_DENSE, coords, row_of, count, spiral, B, V, Wt, bias, ly.act, y,
-            stream))
+        ms = timeit(lambda: hc.hc_sparse_conv_rulebook_fwd(x, rb, count, Wt, bias, ly.act, y,
+                                                           stream))
         fl = 2.0 * L * ly.C_in * ly.C_out * n
         out.append({"density": d, "active_rows": n, "sparse_us": ms * 1e3,
                     "dense_us": dense_ms * 1e3, "speedup": dense_ms / ms,

@@ -148,6 +148,42 @@ hc_status hc_sparse_spiral_conv_fwd(const void* x, hc_layout x_layout, hc_dtype 
                                     hc_act act, void* y, hc_stream_t stream);
 
 /*
+ * hc_conv_rulebook -- the indexing matrix of the sparse convolution (Eq. 4),
+ * materialised: for every active row n < N' and spiral slot l < L,
+ *   rulebook[l*(B*V) + n] = the input row feeding that tap, or -1 when the
+ *   tap is absent (spiral[v*L+l] == -1, or the neighbour (b, u) is inactive).
+ * The input row is b*V + u for x_layout DENSE and row_of[b*V + u] for
+ * COMPACT. The coordinates do not change from layer to layer (Eq. 5), so one
+ * rulebook serves every conv layer run on the same mask.
+ *   coords, row_of, count   as written by hc_mask_compact
+ *   spiral    [V, L] int32, entries in [-1, V)
+ *   rulebook  [L, B*V] int32, slot-major, caller-owned; columns n >= N'
+ *             are not written.
+ * Out-of-range entries are reported (HC_ERR_INVALID_INDEX) and stored as -1.
+ */
+hc_status hc_conv_rulebook(const int32_t* coords, const int32_t* row_of, const int32_t* count,
+                           const int32_t* spiral, int B, int V, int L, hc_layout x_layout,
+                           int32_t* rulebook, hc_stream_t stream);
+
+/*
+ * hc_sparse_conv_rulebook_fwd -- the sparse convolution (Eq. 5) with fused
+ * bias (Eq. 6) and activation (Eq. 10), through a precomputed rulebook:
+ *   y[n, o] = act( bias[o] + sum_{l<L, r = rulebook[l*capacity+n] >= 0}
+ *                  sum_{c<C_in} x[r, c] * W[(l*C_in + c)*C_out + o] ),  n < N'
+ *   x         [x_rows, C_in] of dtype dt; rulebook entries must lie in
+ *             [-1, x_rows) (others are reported and skipped)
+ *   rulebook  [L, capacity] int32 as written by hc_conv_rulebook
+ *             (capacity = B*V there)
+ *   count     N' on the device, at most capacity (clamped, HC_ERR_CAPACITY)
+ *   W, bias, act, y as for hc_sparse_spiral_conv_fwd; y [capacity, C_out].
+ * Results equal hc_sparse_spiral_conv_fwd on the same inputs.
+ */
+hc_status hc_sparse_conv_rulebook_fwd(const void* x, hc_dtype dt, int x_rows,
+                                      const int32_t* rulebook, const int32_t* count, int capacity,
+                                      int L, int C_in, int C_out, const void* W, const float* bias,
+                                      hc_act act, void* y, hc_stream_t stream);
+
+/*
  * hc_sparse_linear_fwd -- linear layer on compact rows (Eq. 6), row-wise
  *   y[n, o] = act( bias[o] + sum_{c<C_in} x[n, c] * W[c*C_out + o] ),  n < N'
  * The coordinates are unchanged (C' = C).

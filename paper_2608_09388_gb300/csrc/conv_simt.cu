@@ -82,12 +82,15 @@ __global__ void __launch_bounds__(kThreads) conv_simt_kernel(const ConvArgs a) {
             const bool ok = in && in_range;
             if (!ok) b = v = 0;
             const bool linear = a.mode == kLinear;
+            const bool rb = a.mode == kRulebook;
             // Loads from clamped, always-valid addresses first; checks after.
             int u[HC_MAX_SPIRAL / 4];
 #pragma unroll
             for (int j = 0; j < HC_MAX_SPIRAL / 4; ++j) {
                 const int l = part + 4 * j < L ? part + 4 * j : L - 1;
-                u[j] = linear ? 0 : __ldg(a.spiral + (long long)v * L + l);
+                u[j] = linear ? 0
+                       : rb   ? __ldg(a.rulebook + (long long)l * a.capacity + nn)
+                              : __ldg(a.spiral + (long long)v * L + l);
             }
 #pragma unroll
             for (int j = 0; j < HC_MAX_SPIRAL / 4; ++j) {
@@ -96,6 +99,9 @@ __global__ void __launch_bounds__(kThreads) conv_simt_kernel(const ConvArgs a) {
                 int src = -1;
                 if (ok && linear) {
                     src = (int)n;
+                } else if (ok && rb) {
+                    if (u[j] < -1 || u[j] >= a.x_rows) err |= kErrIndex;
+                    else src = u[j];
                 } else if (ok) {
                     const int uu = u[j];
                     if (uu < -1 || uu >= a.V) err |= kErrIndex;

@@ -8,14 +8,18 @@
 // the bias of Eq. 6) and the activation of Eq. 10.
 //
 // One persistent CTA per SM, 320 threads in four roles:
-//   warp 9     index warp: for each tile, resolves the 128 x L tap table
+//   warp 9     index warp: for each tile, resolves the L x 128 tap table
 //              (coords -> spiral -> row_of, i.e. idx() of Eq. 4) with every
 //              load of a phase in flight at once, into one of two tables, so
 //              the next tile's table is built while the current one is used;
-//   warps 0-3  producers: gather 128 rows x 64 bf16 of A through the table
-//              and the 64 x BN slice of W per k-block into a 128-byte-swizzled
-//              stage with 16-byte cp.async (zero-fill for absent taps and
-//              ragged edges), then publish the stage on its "full" mbarrier;
+//   warps 0-3  producers: fill a stage with the 128 rows x 64 bf16 of A for
+//              one k-block and the 64 x BN slice of W. With C_in a multiple
+//              of 64 (a k-block never straddles two slots) one lane per warp
+//              issues TMA: tile::gather4 loads of four table rows at a time
+//              (absent taps use an out-of-range row, which TMA fills with
+//              zeros) and tiled loads of W, completing on the stage's "full"
+//              mbarrier by transaction count. Other channel counts use 16-byte
+//              cp.async per thread (zero-fill for absent taps);
 //   warp 8     MMA issuer (one thread): 4 x tcgen05.mma (K = 16 each) per
 //              stage into a TMEM accumulator, tcgen05.commit frees the stage;
 //   warps 4-7  epilogue: tcgen05.ld the 128 x BN fp32 accumulator (warp w
@@ -29,10 +33,18 @@
 //      block a [64 K-rows x 128 bytes] slab, K-row kr at kr*128 with chunk
 //      q stored at q ^ (kr % 8); 8-row groups 1024 bytes apart (SBO), the
 //      64-column blocks BK*128 bytes apart (LBO).
+// The TMA 128-byte swizzle writes exactly these layouts (stage buffers are
+// 1024-byte aligned).
 // Every mbarrier wait is bounded (hc::kWaitLimitNs); on timeout the CTA
 // records HC_ERR_TIMEOUT, unwinds, waits for its own copies and MMAs and
 // frees its TMEM.
+#include <cuda.h>
 #include <cuda_bf16.h>
+#include <cudaTypedefs.h>
+
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
 
 #include "hc_internal.cuh"
 
@@ -61,8 +73,12 @@ struct Cfg {
     static constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | (1u << 16) |
                                        ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(kBM >> 4) << 24);
     static constexpr int kBarBytes = 8 * (2 * kStages + 9);
+    // barriers, then 16 bytes (TMEM address, abort flag), then the two tap
+    // tables at a 128-byte boundary (the TMA producer reads them 16 bytes at
+    // a time).
+    static constexpr int kTabOffset = (kBarBytes + 16 + 127) / 128 * 128;
     static size_t smem_bytes(int L) {
-        return 1024 + (size_t)kStages * (kAStageBytes + kBStageBytes) + kBarBytes + 16 +
+        return 1024 + (size_t)kStages * (kAStageBytes + kBStageBytes) + kTabOffset +
                2 * sizeof(int) * (size_t)kBM * L;
     }
 };
@@ -75,9 +91,34 @@ __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr, uint32_t lbo
            ((uint64_t)(sbo >> 4) << 32) | (1ull << 46) | (2ull << 61);
 }
 
-template <int BN>
-__global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const ConvArgs a) {
+// Activation, bf16 rounding (RNE) and the 16-byte stores of one 32-column
+// chunk of one output row (r holds the fp32 sums with bias added).
+template <int ACT>
+__device__ __forceinline__ void epilogue_store(const uint32_t (&r)[32], __nv_bfloat16* y,
+                                               long long row, bool rvalid, int col0, int C_out) {
+    __nv_bfloat16* yp = y + (rvalid ? row : 0) * C_out + col0;
+#pragma unroll
+    for (int j8 = 0; j8 < 4; ++j8) {
+        uint32_t packed[4];
+#pragma unroll
+        for (int h = 0; h < 4; ++h) {
+            const int j = j8 * 8 + 2 * h;
+            const __nv_bfloat162 p = __floats2bfloat162_rn(act_fixed<ACT>(__uint_as_float(r[j])),
+                                                           act_fixed<ACT>(__uint_as_float(r[j + 1])));
+            packed[h] = *reinterpret_cast<const uint32_t*>(&p);
+        }
+        if (rvalid && col0 + j8 * 8 < C_out)
+            *reinterpret_cast<uint4*>(yp + j8 * 8) =
+                make_uint4(packed[0], packed[1], packed[2], packed[3]);
+    }
+}
+
+template <int BN, bool kTma>
+__global__ void __launch_bounds__(kThreads, 1)
+    conv_tc_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
+                   const __grid_constant__ CUtensorMap tmap_w) {
     using C = Cfg<BN>;
+    constexpr int kStageArrivals = kTma ? kProducerWarps : kProducerWarps * 32;
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;
@@ -88,7 +129,9 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const ConvArgs a) 
     uint8_t* const misc = base_ptr + (sBar - base) + C::kBarBytes;
     volatile uint32_t* const tmem_holder = reinterpret_cast<volatile uint32_t*>(misc);
     volatile int* const abort_flag = reinterpret_cast<volatile int*>(misc + 4);
-    int* const tab_base = reinterpret_cast<int*>(misc + 16);  // [2][kBM][L]
+    // Tap tables, [2][L][kBM] int32: entry (l, r) is the input row feeding
+    // slot l of tile row r, or -1.
+    const uint32_t tab0 = sBar + C::kTabOffset;
 
     auto full_bar = [&](int s) { return sBar + 8u * s; };
     auto empty_bar = [&](int s) { return sBar + 8u * (C::kStages + s); };
@@ -102,7 +145,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const ConvArgs a) 
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < C::kStages; ++s) {
-            mbar_init(full_bar(s), kProducerWarps * 32);
+            mbar_init(full_bar(s), kStageArrivals);
             mbar_init(empty_bar(s), 1);
         }
         for (int i = 0; i < 2; ++i) {
@@ -112,10 +155,14 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const ConvArgs a) 
         mbar_init(fin_bar, 1);
         for (int i = 0; i < 2; ++i) {
             mbar_init(tabfull_bar(i), 32);
-            mbar_init(tabempty_bar(i), kProducerWarps * 32);
+            mbar_init(tabempty_bar(i), kStageArrivals);
         }
         *abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
+    }
+    if (kTma && threadIdx.x == 32) {
+        prefetch_tensormap(&tmap_x);
+        prefetch_tensormap(&tmap_w);
     }
     if (warp == kMmaWarp) {
         tmem_alloc(smem_u32((const void*)tmem_holder), C::kTmemCols);
@@ -132,82 +179,154 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const ConvArgs a) 
     const long long work_total = m_tiles * n_tiles;
     const int num_kb = (a.K + kBK - 1) / kBK;
     const int L = a.L, C_in = a.C_in, C_out = a.C_out, K = a.K;
+    const uint32_t tab_bytes = (uint32_t)(kBM * L) * 4u;
 
     if (warp < kProducerWarps) {
         // ------------------------------------------------------------ producers
-        const __nv_bfloat16* __restrict__ x = static_cast<const __nv_bfloat16*>(a.x);
-        const __nv_bfloat16* __restrict__ W = static_cast<const __nv_bfloat16*>(a.W);
-        const int t = threadIdx.x;  // 0..127
-        const int q = t & 7;        // A: 16-byte chunk of the 128-byte row
-        long long it = 0;
-        int lt = 0;
-        bool ok = true;
-        for (long long w = blockIdx.x; w < work_total && ok; w += gridDim.x, ++lt) {
-            const int n0 = (int)(w % n_tiles) * BN;
-            const int buf = lt & 1;
-            if (!mbar_wait(tabfull_bar(buf), (uint32_t)((lt >> 1) & 1), abort_flag, a.status)) {
-                ok = false;
-                break;
+        if constexpr (kTma) {
+            // Warp w gathers tile rows [32w, 32w+32) of A with eight gather4
+            // loads issued by lanes 0-7 (one each: a TMA issue takes an
+            // issuing thread a few hundred cycles, so spreading the loads
+            // over lanes multiplies the issue rate); lanes 8 and 9 of warp 0
+            // load the W slice. Lane 0 keeps the pipeline bookkeeping.
+            {
+                const int height = (int)a.x_rows;  // rows of the x tensor map
+                const uint32_t my_bytes =
+                    8u * 512u + (warp == 0 ? (uint32_t)(BN / 64) * (kBK * 128u) : 0u);
+                long long it = 0;
+                int lt = 0;
+                bool ok = true;
+                for (long long w = blockIdx.x; w < work_total && ok; w += gridDim.x, ++lt) {
+                    const int n0 = (int)(w % n_tiles) * BN;
+                    const int buf = lt & 1;
+                    // Every lane waits (so every lane acquires the table); the
+                    // warp then agrees on the outcome and stays converged.
+                    ok = __all_sync(0xffffffffu, mbar_wait(tabfull_bar(buf),
+                                                           (uint32_t)((lt >> 1) & 1), abort_flag,
+                                                           a.status));
+                    if (!ok) break;
+                    const uint32_t tab_s = tab0 + (uint32_t)buf * tab_bytes;
+                    int l = 0, c = 0;  // slot and channel offset of k-block kb
+                    for (int kb = 0; kb < num_kb; ++kb) {
+                        const int s = (int)(it % C::kStages);
+                        const uint32_t ph = (uint32_t)((it / C::kStages) & 1);
+                        ok = __all_sync(0xffffffffu,
+                                        mbar_wait(empty_bar(s), ph ^ 1u, abort_flag, a.status));
+                        if (!ok) break;
+                        if (lane == 0) mbar_arrive_expect_tx(full_bar(s), my_bytes);
+                        __syncwarp();
+                        const uint32_t a_st = sA + s * kAStageBytes;
+                        if (lane < 8) {
+                            const int r0 = 32 * warp + 4 * lane;
+                            int4 src = lds_v4(tab_s + (uint32_t)(l * kBM + r0) * 4u);
+                            src.x = src.x < 0 ? height : src.x;
+                            src.y = src.y < 0 ? height : src.y;
+                            src.z = src.z < 0 ? height : src.z;
+                            src.w = src.w < 0 ? height : src.w;
+                            tma_gather4(a_st + (uint32_t)r0 * 128u, &tmap_x, c, src.x, src.y,
+                                        src.z, src.w, full_bar(s));
+                        } else if (warp == 0 && lane < 8 + BN / 64) {
+                            const int nb = lane - 8;
+                            tma_load_2d(sB + s * C::kBStageBytes + nb * (kBK * 128), &tmap_w,
+                                        n0 + nb * 64, kb * kBK, full_bar(s));
+                        }
+                        ++it;
+                        c += kBK;
+                        if (c >= C_in) {
+                            c = 0;
+                            ++l;
+                        }
+                    }
+                    __syncwarp();
+                    if (ok && lane == 0) mbar_arrive(tabempty_bar(buf));
+                }
+                __syncwarp();
+                if (!ok && lane == 0) {
+                    // Let the copies already issued land before the CTA exits.
+                    int no_abort = 0;
+                    for (long long j = it > C::kStages ? it - C::kStages : 0; j < it; ++j)
+                        mbar_wait(full_bar((int)(j % C::kStages)), (uint32_t)((j / C::kStages) & 1),
+                                  &no_abort, a.status);
+                }
             }
-            const uint32_t tab_s = smem_u32(tab_base) + (uint32_t)(buf * kBM * L) * 4u;
-            int l = (q * 8) / C_in;  // slot and channel of this thread's chunk at k-block 0
-            int c = q * 8 - l * C_in;
-            for (int kb = 0; kb < num_kb; ++kb) {
-                const int s = (int)(it % C::kStages);
-                const uint32_t ph = (uint32_t)((it / C::kStages) & 1);
-                if (!mbar_wait(empty_bar(s), ph ^ 1u, abort_flag, a.status)) {
+            __syncwarp();
+        } else {
+            const __nv_bfloat16* __restrict__ x = static_cast<const __nv_bfloat16*>(a.x);
+            const __nv_bfloat16* __restrict__ W = static_cast<const __nv_bfloat16*>(a.W);
+            const int t = threadIdx.x;  // 0..127
+            const int q = t & 7;        // A: 16-byte chunk of the 128-byte row
+            long long it = 0;
+            int lt = 0;
+            bool ok = true;
+            for (long long w = blockIdx.x; w < work_total && ok; w += gridDim.x, ++lt) {
+                const int n0 = (int)(w % n_tiles) * BN;
+                const int buf = lt & 1;
+                if (!mbar_wait(tabfull_bar(buf), (uint32_t)((lt >> 1) & 1), abort_flag,
+                               a.status)) {
                     ok = false;
                     break;
                 }
-                const uint32_t a_st = sA + s * kAStageBytes;
-                const bool kval = kb * kBK + q * 8 < K;
-                // All eight table entries of this stage first, then the copies.
-                int src[8];
+                const uint32_t tab_s = tab0 + (uint32_t)buf * tab_bytes;
+                int l = (q * 8) / C_in;  // slot and channel of this thread's chunk at k-block 0
+                int c = q * 8 - l * C_in;
+                for (int kb = 0; kb < num_kb; ++kb) {
+                    const int s = (int)(it % C::kStages);
+                    const uint32_t ph = (uint32_t)((it / C::kStages) & 1);
+                    if (!mbar_wait(empty_bar(s), ph ^ 1u, abort_flag, a.status)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t a_st = sA + s * kAStageBytes;
+                    const bool kval = kb * kBK + q * 8 < K;
+                    // All eight table entries of this stage first, then the copies.
+                    int src[8];
 #pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    const int r = (t >> 3) + 16 * i;
-                    src[i] = kval ? lds_s32(tab_s + (uint32_t)(r * L + l) * 4u) : -1;
-                }
+                    for (int i = 0; i < 8; ++i) {
+                        const int r = (t >> 3) + 16 * i;
+                        src[i] = kval ? lds_s32(tab_s + (uint32_t)(l * kBM + r) * 4u) : -1;
+                    }
 #pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    const int r = (t >> 3) + 16 * i;
-                    const __nv_bfloat16* gp = x + (src[i] >= 0 ? (long long)src[i] * C_in + c : 0);
-                    cp_async_16(a_st + r * 128 + ((q ^ (r & 7)) << 4), gp, src[i] >= 0);
-                }
-                const uint32_t b_st = sB + s * C::kBStageBytes;
-                constexpr int kCpr = BN / 8;  // 16-byte chunks per W row slice
+                    for (int i = 0; i < 8; ++i) {
+                        const int r = (t >> 3) + 16 * i;
+                        const __nv_bfloat16* gp =
+                            x + (src[i] >= 0 ? (long long)src[i] * C_in + c : 0);
+                        cp_async_16(a_st + r * 128 + ((q ^ (r & 7)) << 4), gp, src[i] >= 0);
+                    }
+                    const uint32_t b_st = sB + s * C::kBStageBytes;
+                    constexpr int kCpr = BN / 8;  // 16-byte chunks per W row slice
 #pragma unroll
-                for (int i = 0; i < (kBK * kCpr) / 128; ++i) {
-                    const int e = t + 128 * i;
-                    const int kr = e / kCpr, nq = e % kCpr;
-                    const int kk = kb * kBK + kr, col = n0 + nq * 8;
-                    const bool valid = kk < K && col < C_out;
-                    const __nv_bfloat16* gp = W + (valid ? (long long)kk * C_out + col : 0);
-                    cp_async_16(b_st + (nq >> 3) * (kBK * 128) + kr * 128 +
-                                    (((nq & 7) ^ (kr & 7)) << 4),
-                                gp, valid);
+                    for (int i = 0; i < (kBK * kCpr) / 128; ++i) {
+                        const int e = t + 128 * i;
+                        const int kr = e / kCpr, nq = e % kCpr;
+                        const int kk = kb * kBK + kr, col = n0 + nq * 8;
+                        const bool valid = kk < K && col < C_out;
+                        const __nv_bfloat16* gp = W + (valid ? (long long)kk * C_out + col : 0);
+                        cp_async_16(b_st + (nq >> 3) * (kBK * 128) + kr * 128 +
+                                        (((nq & 7) ^ (kr & 7)) << 4),
+                                    gp, valid);
+                    }
+                    cp_async_commit();
+                    if (it >= C::kLag) {
+                        cp_async_wait<C::kLag>();
+                        fence_proxy_async_smem();
+                        mbar_arrive(full_bar((int)((it - C::kLag) % C::kStages)));
+                    }
+                    ++it;
+                    c += kBK;
+                    while (c >= C_in) {
+                        c -= C_in;
+                        ++l;
+                    }
                 }
-                cp_async_commit();
-                if (it >= C::kLag) {
-                    cp_async_wait<C::kLag>();
-                    fence_proxy_async_smem();
-                    mbar_arrive(full_bar((int)((it - C::kLag) % C::kStages)));
-                }
-                ++it;
-                c += kBK;
-                while (c >= C_in) {
-                    c -= C_in;
-                    ++l;
-                }
+                // Addresses of this tile's copies are issued: the table is free.
+                if (ok) mbar_arrive(tabempty_bar(buf));
             }
-            // Addresses of this tile's copies are issued: the table is free.
-            mbar_arrive(tabempty_bar(buf));
+            cp_async_wait_all();
+            fence_proxy_async_smem();
+            if (ok)
+                for (long long j = it > C::kLag ? it - C::kLag : 0; j < it; ++j)
+                    mbar_arrive(full_bar((int)(j % C::kStages)));
         }
-        cp_async_wait_all();
-        fence_proxy_async_smem();
-        if (ok)
-            for (long long j = it > C::kLag ? it - C::kLag : 0; j < it; ++j)
-                mbar_arrive(full_bar((int)(j % C::kStages)));
     } else if (warp == kMmaWarp) {
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0) {
@@ -231,7 +350,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const ConvArgs a) 
                         break;
                     }
                     tc_fence_after();
-                    fence_proxy_async_smem();
+                    if (!kTma) fence_proxy_async_smem();
                     const uint32_t a_st = sA + s * kAStageBytes;
                     const uint32_t b_st = sB + s * C::kBStageBytes;
 #pragma unroll
@@ -256,8 +375,9 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const ConvArgs a) 
         // ------------------------------------------------------------ index warp
         // Lane handles rows lane + 32*i (i < 4) of the tile. Phase 1 loads the
         // coordinates, phase 2 all spiral entries of a chunk of slots, phase 3
-        // all row_of lookups of that chunk: three dependent round trips per
-        // tile instead of one per slot.
+        // all row_of lookups of that chunk. Loads are issued from clamped,
+        // always-valid addresses and checked afterwards, so that every load
+        // of a phase is in flight at once.
         int lt = 0;
         for (long long w = blockIdx.x; w < work_total; w += gridDim.x, ++lt) {
             const int buf = lt & 1;
@@ -265,19 +385,47 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const ConvArgs a) 
                            a.status))
                 break;
             const long long m0 = (w / n_tiles) * kBM;
-            const uint32_t tab_s = smem_u32(tab_base) + (uint32_t)(buf * kBM * L) * 4u;
-            // Loads are issued unconditionally from clamped, always-valid
-            // addresses and checked afterwards, so that every load of a
-            // phase is in flight at once.
+            const uint32_t tab_s = tab0 + (uint32_t)buf * tab_bytes;
+            unsigned err = 0;
+            if (a.mode == kRulebook) {
+                // Precomputed mapping: one coalesced pass over the tile's
+                // rulebook columns, entries checked against the input's rows.
+                constexpr int kRbChunk = 12;
+                for (int l0 = 0; l0 < L; l0 += kRbChunk) {
+                    int e[4][kRbChunk];
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+#pragma unroll
+                        for (int d = 0; d < kRbChunk; ++d) {
+                            const long long n = m0 + lane + 32 * i;
+                            const int lc = l0 + d < L ? l0 + d : L - 1;
+                            e[i][d] = __ldg(a.rulebook + (long long)lc * a.capacity + (n < rows ? n : 0));
+                        }
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+#pragma unroll
+                        for (int d = 0; d < kRbChunk; ++d) {
+                            if (l0 + d >= L) continue;
+                            const int ev = e[i][d];
+                            int src = -1;
+                            if (m0 + lane + 32 * i < rows) {
+                                if (ev < -1 || ev >= a.x_rows) err |= kErrIndex;
+                                else src = ev;
+                            }
+                            sts_s32(tab_s + (uint32_t)((l0 + d) * kBM + lane + 32 * i) * 4u, src);
+                        }
+                }
+                if (err) report(a.status, err);
+                mbar_arrive(tabfull_bar(buf));
+                continue;
+            }
             int bb[4], vv[4];
             bool ok[4];
-            unsigned err = 0;
             const bool sparse = a.mode == kSparseDenseX || a.mode == kSparseCompactX;
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
                 const long long n = m0 + lane + 32 * i;
-                const bool in = n < rows;
-                const long long nn = in ? n : 0;
+                const long long nn = n < rows ? n : 0;
                 if (sparse) {
                     bb[i] = __ldg(a.coords + 2 * nn);
                     vv[i] = __ldg(a.coords + 2 * nn + 1);
@@ -350,7 +498,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const ConvArgs a) 
                                         src = a.mode == kSparseDenseX ? dr[i][d] : jj;
                                 }
                             }
-                            sts_s32(tab_s + (uint32_t)((lane + 32 * i) * L + l0 + d) * 4u, src);
+                            sts_s32(tab_s + (uint32_t)((l0 + d) * kBM + lane + 32 * i) * 4u, src);
                         }
                 }
             }
@@ -379,28 +527,20 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const ConvArgs a) 
                 tmem_ld_wait();
                 const int col0 = n0 + cb * 32;
                 // Bias of the chunk's 32 columns: one coalesced load, then
-                // broadcast by shuffles.
+                // broadcast by shuffles (every lane takes part).
                 const int bcol = col0 + lane < C_out ? col0 + lane : C_out - 1;
                 const float bias_l = a.bias ? __ldg(a.bias + bcol) : 0.f;
-                __nv_bfloat16* yp = y + (rvalid ? row : 0) * C_out + col0;
 #pragma unroll
-                for (int j8 = 0; j8 < 4; ++j8) {
-                    uint32_t packed[4];
-#pragma unroll
-                    for (int h = 0; h < 4; ++h) {
-                        // every lane takes part in the shuffles
-                        const int j = j8 * 8 + 2 * h;
-                        const float z0 = __uint_as_float(r[j]) + __shfl_sync(0xffffffffu, bias_l, j);
-                        const float z1 =
-                            __uint_as_float(r[j + 1]) + __shfl_sync(0xffffffffu, bias_l, j + 1);
-                        const __nv_bfloat162 p =
-                            __floats2bfloat162_rn(act_apply(z0, a.act), act_apply(z1, a.act));
-                        packed[h] = *reinterpret_cast<const uint32_t*>(&p);
-                    }
-                    if (rvalid && col0 + j8 * 8 < C_out)
-                        *reinterpret_cast<uint4*>(yp + j8 * 8) =
-                            make_uint4(packed[0], packed[1], packed[2], packed[3]);
-                }
+                for (int j = 0; j < 32; ++j)
+                    r[j] = __float_as_uint(__uint_as_float(r[j]) +
+                                           __shfl_sync(0xffffffffu, bias_l, j));
+                // The activation is chosen once per chunk, not per element.
+                if (a.act == HC_ACT_ELU)
+                    epilogue_store<HC_ACT_ELU>(r, y, row, rvalid, col0, C_out);
+                else if (a.act == HC_ACT_RELU)
+                    epilogue_store<HC_ACT_RELU>(r, y, row, rvalid, col0, C_out);
+                else
+                    epilogue_store<HC_ACT_NONE>(r, y, row, rvalid, col0, C_out);
             }
             tc_fence_before();
             mbar_arrive(tempty_bar(acc));
@@ -414,23 +554,73 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const ConvArgs a) 
     }
 }
 
-template <int BN>
+// ---------------------------------------------------------------- host side
+
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    });
+    return fn;
+}
+
+// 2-D bf16 tensor map over a row-major [rows, cols] matrix with a 128-byte
+// swizzled box of box_cols x box_rows.
+hc_status encode_2d(CUtensorMap* m, const void* base, long long rows, long long cols, int box_cols,
+                    int box_rows) {
+    auto enc = tensor_map_encoder();
+    if (!enc) {
+        set_error("cuTensorMapEncodeTiled is unavailable");
+        return HC_ERR_CUDA;
+    }
+    cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
+    cuuint32_t box[2] = {(cuuint32_t)box_cols, (cuuint32_t)box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
+                     box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) {
+        set_error("cuTensorMapEncodeTiled failed (%d)", (int)r);
+        return HC_ERR_CUDA;
+    }
+    return HC_OK;
+}
+
+template <int BN, bool kTma>
 hc_status launch_bn(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s) {
     using C = Cfg<BN>;
     static bool attr_set[64] = {};
     if (!attr_set[ctx->device]) {
-        hc_status st = check_cuda(
-            cudaFuncSetAttribute(conv_tc_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)C::smem_bytes(HC_MAX_SPIRAL)),
-            "cudaFuncSetAttribute(conv_tc_kernel)");
+        hc_status st = check_cuda(cudaFuncSetAttribute(conv_tc_kernel<BN, kTma>,
+                                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                       (int)C::smem_bytes(HC_MAX_SPIRAL)),
+                                  "cudaFuncSetAttribute(conv_tc_kernel)");
         if (st != HC_OK) return st;
         attr_set[ctx->device] = true;
+    }
+    CUtensorMap tx, tw;
+    memset(&tx, 0, sizeof tx);
+    memset(&tw, 0, sizeof tw);
+    if (kTma) {
+        // x: [x_rows, C_in], boxes of one row x 64 channels (gather4);
+        // W: [K rows, C_out], boxes of 64 K-rows x 64 output channels.
+        hc_status st = encode_2d(&tx, a.x, a.x_rows, a.C_in, kBK, 1);
+        if (st != HC_OK) return st;
+        st = encode_2d(&tw, a.W, a.K, a.C_out, 64, kBK);
+        if (st != HC_OK) return st;
     }
     const long long n_tiles = (a.C_out + BN - 1) / BN;
     const long long cap_work = (a.capacity + kBM - 1) / kBM * n_tiles;
     long long grid = cap_work < ctx->num_sms ? cap_work : ctx->num_sms;
     if (grid < 1) grid = 1;
-    conv_tc_kernel<BN><<<(unsigned)grid, kThreads, C::smem_bytes(a.L), s>>>(a);
+    conv_tc_kernel<BN, kTma><<<(unsigned)grid, kThreads, C::smem_bytes(a.L), s>>>(a, tx, tw);
     return check_cuda(cudaGetLastError(), "conv_tc_kernel");
 }
 
@@ -443,8 +633,17 @@ bool conv_tc_supported(const ConvArgs& a, hc_dtype dt) {
 }
 
 hc_status launch_conv_tc(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s) {
-    if (a.C_out <= 64) return launch_bn<64>(ctx, a, s);
-    return launch_bn<128>(ctx, a, s);
+    // TMA gathers whole 64-channel blocks of one input row, so it needs C_in
+    // to be a multiple of 64; other channel counts gather with cp.async.
+    // HC_NO_TMA=1 selects the cp.async producer for every shape.
+    static int tma_off = -1;
+    if (tma_off < 0) {
+        const char* e = getenv("HC_NO_TMA");
+        tma_off = (e && e[0] == '1') ? 1 : 0;
+    }
+    const bool tma = !tma_off && a.C_in % kBK == 0;
+    if (a.C_out <= 64) return tma ? launch_bn<64, true>(ctx, a, s) : launch_bn<64, false>(ctx, a, s);
+    return tma ? launch_bn<128, true>(ctx, a, s) : launch_bn<128, false>(ctx, a, s);
 }
 
 }  // namespace hc

@@ -188,6 +188,7 @@ hc_status hc_sparse_spiral_conv_fwd(const void* x, hc_layout x_layout, hc_dtype 
     a.bias = bias;
     a.y = y;
     a.capacity = (long long)B * V;
+    a.x_rows = (long long)B * V;
     a.B = B;
     a.V = V;
     a.L = L;
@@ -218,6 +219,7 @@ hc_status hc_sparse_linear_fwd(const void* x, hc_dtype dt, const int32_t* count,
     a.bias = bias;
     a.y = y;
     a.capacity = capacity;
+    a.x_rows = capacity;
     a.B = 1;
     a.V = capacity;
     a.L = 1;
@@ -249,6 +251,7 @@ hc_status hc_spiral_conv_fwd(const void* x, hc_dtype dt, const int32_t* spiral, 
     a.bias = bias;
     a.y = y;
     a.capacity = (long long)B * V;
+    a.x_rows = (long long)B * V;
     a.B = B;
     a.V = V;
     a.L = L;
@@ -256,6 +259,62 @@ hc_status hc_spiral_conv_fwd(const void* x, hc_dtype dt, const int32_t* spiral, 
     a.C_out = C_out;
     a.K = L * C_in;
     a.mode = kDense;
+    a.act = act;
+    return dispatch_conv(ctx, a, dt, (cudaStream_t)stream);
+}
+
+hc_status hc_conv_rulebook(const int32_t* coords, const int32_t* row_of, const int32_t* count,
+                           const int32_t* spiral, int B, int V, int L, hc_layout x_layout,
+                           int32_t* rulebook, hc_stream_t stream) {
+    const char* fn = "hc_conv_rulebook";
+    t_last_error[0] = 0;
+    HC_REQUIRE(B >= 0 && V >= 0, "%s: B=%d V=%d must be >= 0", fn, B, V);
+    HC_REQUIRE((long long)B * V < (1ll << 31), "%s: B*V must be < 2^31", fn);
+    HC_REQUIRE(L >= 1, "%s: L=%d must be >= 1", fn, L);
+    if (L > HC_MAX_SPIRAL) {
+        set_error("%s: L=%d exceeds HC_MAX_SPIRAL=%d", fn, L, HC_MAX_SPIRAL);
+        return HC_ERR_UNSUPPORTED;
+    }
+    HC_REQUIRE(x_layout == HC_LAYOUT_DENSE || x_layout == HC_LAYOUT_COMPACT,
+               "%s: unknown layout %d", fn, (int)x_layout);
+    HC_REQUIRE(coords && row_of && count && spiral && rulebook,
+               "%s: coords, row_of, count, spiral and rulebook are required", fn);
+    if ((long long)B * V == 0) return HC_OK;
+    const DeviceCtx* ctx = device_ctx();
+    if (!ctx) return HC_ERR_CUDA;
+    return launch_rulebook(ctx, coords, row_of, count, spiral, B, V, L, (int)x_layout, rulebook,
+                           (cudaStream_t)stream);
+}
+
+hc_status hc_sparse_conv_rulebook_fwd(const void* x, hc_dtype dt, int x_rows,
+                                      const int32_t* rulebook, const int32_t* count, int capacity,
+                                      int L, int C_in, int C_out, const void* W, const float* bias,
+                                      hc_act act, void* y, hc_stream_t stream) {
+    const char* fn = "hc_sparse_conv_rulebook_fwd";
+    t_last_error[0] = 0;
+    hc_status st = check_conv_common(fn, dt, L, C_in, C_out, act, x, W, y);
+    if (st != HC_OK) return st;
+    HC_REQUIRE(x_rows >= 1 && capacity >= 0, "%s: x_rows=%d capacity=%d", fn, x_rows, capacity);
+    HC_REQUIRE(rulebook && count, "%s: rulebook and count are required", fn);
+    if (capacity == 0) return HC_OK;
+    const DeviceCtx* ctx = device_ctx();
+    if (!ctx) return HC_ERR_CUDA;
+    ConvArgs a{};
+    a.x = x;
+    a.count = count;
+    a.rulebook = rulebook;
+    a.W = W;
+    a.bias = bias;
+    a.y = y;
+    a.capacity = capacity;
+    a.x_rows = x_rows;
+    a.B = 1;
+    a.V = capacity;
+    a.L = L;
+    a.C_in = C_in;
+    a.C_out = C_out;
+    a.K = L * C_in;
+    a.mode = kRulebook;
     a.act = act;
     return dispatch_conv(ctx, a, dt, (cudaStream_t)stream);
 }

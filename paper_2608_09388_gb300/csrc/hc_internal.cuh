@@ -44,6 +44,7 @@ enum RowMode : int {
     kSparseCompactX = 1,  // rows = coords[0..count); input rows at row_of[b*V+u]
     kDense = 2,           // rows = all b*V+v; input rows at b*V+u
     kLinear = 3,          // rows = 0..count; input row = output row; L = 1
+    kRulebook = 4,        // rows = 0..count; input rows from a precomputed rulebook
 };
 
 struct ConvArgs {
@@ -57,6 +58,8 @@ struct ConvArgs {
     void* y;
     unsigned* status;
     long long capacity;  // upper bound on rows (B*V, or the linear capacity)
+    long long x_rows;    // rows of the input x (valid input row indices are < x_rows)
+    const int32_t* rulebook;  // kRulebook: [L, capacity] slot-major tap rows, -1 = absent
     int B, V, L, C_in, C_out, K;  // K = L*C_in
     int mode;
     int act;
@@ -69,6 +72,9 @@ hc_status launch_compact(const DeviceCtx* ctx, const uint8_t* mask, int B, int V
 hc_status launch_conv_simt(const DeviceCtx* ctx, const ConvArgs& a, hc_dtype dt, cudaStream_t s);
 hc_status launch_conv_tc(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s);
 bool conv_tc_supported(const ConvArgs& a, hc_dtype dt);
+hc_status launch_rulebook(const DeviceCtx* ctx, const int32_t* coords, const int32_t* row_of,
+                          const int32_t* count, const int32_t* spiral, int B, int V, int L,
+                          int x_layout, int32_t* rulebook, cudaStream_t s);
 hc_status launch_scatter(const DeviceCtx* ctx, const void* y, int elem_bytes, const int32_t* coords,
                          const int32_t* row_of, const int32_t* count, int B, int V, int C,
                          int zero_fill, void* out, cudaStream_t s);
@@ -105,7 +111,7 @@ __device__ __forceinline__ bool row_coord(const ConvArgs& a, long long n, int& b
         v = (int)(n - (long long)b * a.V);
         return true;
     }
-    if (a.mode == kLinear) {
+    if (a.mode == kLinear || a.mode == kRulebook) {
         b = 0;
         v = 0;
         return true;
@@ -156,12 +162,20 @@ __device__ __forceinline__ long long resolve_tap(const ConvArgs& a, long long n,
     return a.mode == kSparseDenseX ? dense_row : (long long)j;
 }
 
-// Activation of Eq. 10. ELU(z) = z for z > 0, else exp(z) - 1, evaluated
-// with the fast exponential: the absolute error is a few 1e-7, far inside the
-// fp32 (1e-4 absolute) and bf16 (2e-2 relative) tolerances of this library.
+// Activation of Eq. 10. ELU(z) = z for z > 0, else exp(z) - 1, written
+// without a branch as max(z, 0) + (exp(min(z, 0)) - 1): for z > 0 the second
+// term is exp(0) - 1 = 0 exactly. The fast exponential's absolute error is a
+// few 1e-7, far inside the fp32 (1e-4 absolute) and bf16 (2e-2 relative)
+// tolerances of this library.
+template <int ACT>
+__device__ __forceinline__ float act_fixed(float z) {
+    if (ACT == HC_ACT_ELU) return fmaxf(z, 0.f) + (__expf(fminf(z, 0.f)) - 1.0f);
+    if (ACT == HC_ACT_RELU) return fmaxf(z, 0.f);
+    return z;
+}
 __device__ __forceinline__ float act_apply(float z, int act) {
-    if (act == HC_ACT_ELU) return z > 0.f ? z : __expf(z) - 1.0f;
-    if (act == HC_ACT_RELU) return z > 0.f ? z : 0.f;
+    if (act == HC_ACT_ELU) return act_fixed<HC_ACT_ELU>(z);
+    if (act == HC_ACT_RELU) return act_fixed<HC_ACT_RELU>(z);
     return z;
 }
 
@@ -244,6 +258,43 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatil
             }
         }
     }
+}
+
+// ---- TMA (bulk tensor copies global -> shared, completion on an mbarrier)
+// Arrive on `bar` and add `bytes` to the transaction count its phase waits for.
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n" ::"r"(bar), "r"(bytes)
+                 : "memory");
+}
+// 2-D tiled load of the tensor map's box at (c0 = inner, c1 = outer).
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const void* tmap, int c0, int c1,
+                                            uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3}], [%4];\n" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(tmap)), "r"(c0), "r"(c1), "r"(bar)
+        : "memory");
+}
+// Four rows (r0..r3) of a box one row high, starting at column c0, written to
+// consecutive box rows in shared memory. Rows outside the tensor read zeros.
+__device__ __forceinline__ void tma_gather4(uint32_t dst, const void* tmap, int c0, int r0, int r1,
+                                            int r2, int r3, uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile::gather4.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3, %4, %5, %6}], [%7];\n" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(tmap)), "r"(c0), "r"(r0), "r"(r1), "r"(r2), "r"(r3),
+        "r"(bar)
+        : "memory");
+}
+__device__ __forceinline__ void prefetch_tensormap(const void* tmap) {
+    asm volatile("prefetch.tensormap [%0];\n" ::"l"(reinterpret_cast<uint64_t>(tmap)) : "memory");
+}
+__device__ __forceinline__ int4 lds_v4(uint32_t addr) {
+    int4 v;
+    asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];\n"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "r"(addr));
+    return v;
 }
 
 // ---- tcgen05 (5th-generation tensor cores, accumulators in TMEM)

@@ -1,0 +1,88 @@
+// The indexing matrix of the sparse convolution (Eq. 4) for the spiral
+// neighbourhood, materialised once per mask: for every active row n and
+// spiral slot l, the input row that feeds the tap, or -1 when the tap is
+// absent (no neighbour in that slot, or the neighbour is not an active row).
+// The coordinates do not change from layer to layer (Eq. 5 keeps the centre
+// coordinates), so one rulebook serves every conv layer of a network.
+//
+// Layout: [L, capacity] int32, slot-major (entry (l, n) at l*capacity + n),
+// so that a tile of consecutive rows reads each slot as one contiguous run.
+// One thread per active row; its coordinate, spiral entries and row_of
+// lookups are each issued together from clamped, always-valid addresses.
+#include "hc_internal.cuh"
+
+namespace hc {
+namespace {
+
+constexpr int kChunk = 8;
+
+__global__ void __launch_bounds__(256) rulebook_kernel(const int32_t* __restrict__ coords,
+                                                       const int32_t* __restrict__ row_of,
+                                                       const int32_t* __restrict__ count,
+                                                       const int32_t* __restrict__ spiral, int B,
+                                                       int V, int L, int x_layout,
+                                                       int32_t* __restrict__ rulebook,
+                                                       unsigned* status) {
+    const long long cap = (long long)B * V;
+    long long rows = *count;
+    unsigned err = 0;
+    if (rows < 0) {
+        err |= kErrIndex;
+        rows = 0;
+    }
+    if (rows > cap) {
+        err |= kErrCapacity;
+        rows = cap;
+    }
+    for (long long n = blockIdx.x * (long long)blockDim.x + threadIdx.x; n < rows;
+         n += (long long)gridDim.x * blockDim.x) {
+        int b = __ldg(coords + 2 * n), v = __ldg(coords + 2 * n + 1);
+        const bool ok = b >= 0 && b < B && v >= 0 && v < V;
+        if (!ok) {
+            err |= kErrIndex;
+            b = v = 0;
+        }
+        for (int l0 = 0; l0 < L; l0 += kChunk) {
+            int u[kChunk], dr[kChunk], j[kChunk];
+#pragma unroll
+            for (int d = 0; d < kChunk; ++d)
+                u[d] = __ldg(spiral + (long long)v * L + (l0 + d < L ? l0 + d : L - 1));
+#pragma unroll
+            for (int d = 0; d < kChunk; ++d) {
+                const bool live = ok && l0 + d < L;
+                if (live && (u[d] < -1 || u[d] >= V)) err |= kErrIndex;
+                dr[d] = (live && u[d] >= 0 && u[d] < V) ? b * V + u[d] : -1;
+            }
+#pragma unroll
+            for (int d = 0; d < kChunk; ++d) j[d] = __ldg(row_of + (dr[d] >= 0 ? dr[d] : 0));
+#pragma unroll
+            for (int d = 0; d < kChunk; ++d) {
+                if (l0 + d >= L) continue;
+                int e = -1;
+                if (dr[d] >= 0) {
+                    if (j[d] < -1 || j[d] >= rows) err |= kErrIndex;
+                    if (j[d] >= 0 && j[d] < rows) e = x_layout == HC_LAYOUT_DENSE ? dr[d] : j[d];
+                }
+                rulebook[(long long)(l0 + d) * cap + n] = e;
+            }
+        }
+    }
+    if (err) report(status, err);
+}
+
+}  // namespace
+
+hc_status launch_rulebook(const DeviceCtx* ctx, const int32_t* coords, const int32_t* row_of,
+                          const int32_t* count, const int32_t* spiral, int B, int V, int L,
+                          int x_layout, int32_t* rulebook, cudaStream_t s) {
+    const long long cap = (long long)B * V;
+    long long blocks = (cap + 255) / 256;
+    const long long lim = (long long)ctx->num_sms * 8;
+    if (blocks > lim) blocks = lim;
+    if (blocks < 1) blocks = 1;
+    rulebook_kernel<<<(unsigned)blocks, 256, 0, s>>>(coords, row_of, count, spiral, B, V, L,
+                                                      x_layout, rulebook, ctx->status);
+    return check_cuda(cudaGetLastError(), "rulebook_kernel");
+}
+
+}  // namespace hc

@@ -29,7 +29,8 @@ STATUS_NAMES = {0: "HC_OK", 1: "HC_ERR_INVALID_ARG", 2: "HC_ERR_UNSUPPORTED",
 
 # Exported symbols, as declared in include/hc.h.
 EXPORTS = ("hc_mask_compact", "hc_mask_compact_static", "hc_sparse_spiral_conv_fwd",
-           "hc_sparse_linear_fwd", "hc_scatter_dense", "hc_spiral_conv_fwd", "hc_get_device_status",
+           "hc_conv_rulebook", "hc_sparse_conv_rulebook_fwd", "hc_sparse_linear_fwd",
+           "hc_scatter_dense", "hc_spiral_conv_fwd", "hc_get_device_status",
            "hc_last_error_string", "hc_version")
 
 
@@ -58,6 +59,8 @@ def load_library(path: str | None = None):
             "hc_mask_compact": [P, I, I, P, P, P, P, P],
             "hc_mask_compact_static": [P, I, I, P, P, P, P, P],
             "hc_sparse_spiral_conv_fwd": [P, I, I, P, P, P, P, I, I, I, I, I, P, P, I, P, P],
+            "hc_conv_rulebook": [P, P, P, P, I, I, I, I, P, P],
+            "hc_sparse_conv_rulebook_fwd": [P, I, I, P, P, I, I, I, I, P, P, I, P, P],
             "hc_sparse_linear_fwd": [P, I, P, I, I, I, P, P, I, P, P],
             "hc_scatter_dense": [P, I, P, P, P, I, I, I, I, P, P],
             "hc_spiral_conv_fwd": [P, I, P, I, I, I, I, I, P, P, I, P, P],
@@ -133,6 +136,26 @@ def hc_sparse_spiral_conv_fwd(x, x_layout, coords, row_of, count, spiral, B, V, 
     _check(load_library().hc_sparse_spiral_conv_fwd(
         _p(x), x_layout, _dt(x), _p(coords), _p(row_of), _p(count), _p(spiral), B, V, L, C_in,
         C_out, _p(W), _p(bias), act, _p(y), _s(stream)), "hc_sparse_spiral_conv_fwd")
+
+
+def hc_conv_rulebook(coords, row_of, count, spiral, B, V, x_layout, rulebook, stream=None):
+    """Eq. 4 mapping: rulebook int32 [L, B*V] of input rows per (slot, active row)."""
+    L = spiral.shape[1]
+    _check(load_library().hc_conv_rulebook(_p(coords), _p(row_of), _p(count), _p(spiral), B, V, L,
+                                           x_layout, _p(rulebook), _s(stream)),
+           "hc_conv_rulebook")
+
+
+def hc_sparse_conv_rulebook_fwd(x, rulebook, count, W, bias, act, y, stream=None):
+    """Sparse conv through a rulebook [L, capacity]: x [x_rows, C_in] (or [B, V, C_in]),
+    W [L*C_in, C_out], y [capacity, C_out]."""
+    L, capacity = rulebook.shape
+    C_in = x.shape[-1]
+    x_rows = x.numel() // C_in
+    C_out = W.shape[1]
+    _check(load_library().hc_sparse_conv_rulebook_fwd(
+        _p(x), _dt(x), x_rows, _p(rulebook), _p(count), capacity, L, C_in, C_out, _p(W),
+        _p(bias), act, _p(y), _s(stream)), "hc_sparse_conv_rulebook_fwd")
 
 
 def hc_sparse_linear_fwd(x, count, W, bias, act, y, stream=None):

@@ -217,6 +217,106 @@ def test_deterministic_and_stream_ordered():
     np.testing.assert_array_equal(y1, y2)
 
 
+# ------------------------------------------------------------------ rulebook (Eq. 4 mapping)
+
+def gpu_rulebook(m, sp, layout):
+    B, V = m.shape
+    coords, row_of, offs, count = gpu_compact(m)
+    rb = torch.full((sp.shape[1], B * V), -7, dtype=torch.int32, device="cuda")
+    hc.hc_conv_rulebook(coords, row_of, count, to_torch(sp), B, V, layout, rb)
+    assert hc.hc_get_device_status() == hc.HC_OK
+    return rb, coords, row_of, count
+
+
+@pytest.mark.parametrize("layout", [hc.HC_LAYOUT_DENSE, hc.HC_LAYOUT_COMPACT])
+@pytest.mark.parametrize("shape", [(1, 40, 1), (3, 200, 9), (5, 300, 12), (2, 1000, 32), (1, 5, 5)])
+def test_rulebook_bit_exact(shape, layout):
+    B, V, L = shape
+    sp, m, x, W, b = inputs.random_case(B * 31 + V + L, B, V, L, 8, 8, "f32", 0.35, neg_frac=0.1)
+    rb, *_ = gpu_rulebook(m, sp, layout)
+    c, r, _, n = oracle.mask_compact(m)
+    ref = oracle.conv_rulebook(c, r, sp, layout)
+    np.testing.assert_array_equal(to_numpy(rb)[:, :n], ref[:, :n])
+
+
+RB_SHAPES = [
+    (3, 200, 9, 64, 64, 0.3, "bf16"),     # tensor cores, TMA gather
+    (2, 300, 12, 128, 128, 0.5, "bf16"),  # tensor cores, TMA gather, 2 k-blocks per slot
+    (4, 333, 7, 24, 40, 0.5, "bf16"),     # tensor cores, cp.async gather
+    (2, 300, 9, 45, 64, 0.3, "bf16"),     # CUDA cores (C_in not a multiple of 8)
+    (1, 655, 9, 16, 64, 0.1, "f32"),      # CUDA cores, fp32
+    (2, 257, 5, 64, 136, 0.9, "bf16"),    # two N tiles
+]
+
+
+@pytest.mark.parametrize("layout", [hc.HC_LAYOUT_DENSE, hc.HC_LAYOUT_COMPACT])
+@pytest.mark.parametrize("shape", RB_SHAPES)
+def test_conv_through_rulebook(shape, layout):
+    B, V, L, C_in, C_out, dens, dtype = shape
+    sp, m, x, W, b = inputs.random_case(B + V + L + C_in + C_out, B, V, L, C_in, C_out, dtype,
+                                        dens, neg_frac=0.1)
+    rb, coords, row_of, count = gpu_rulebook(m, sp, layout)
+    c, r, _, n = oracle.mask_compact(m)
+    xin = x if layout == hc.HC_LAYOUT_DENSE else np.ascontiguousarray(x[c[:, 0], c[:, 1]])
+    xt = to_torch(xin)
+    y = torch.full((B * V, C_out), float("nan"), dtype=xt.dtype, device="cuda")
+    hc.hc_sparse_conv_rulebook_fwd(xt, rb, count, to_torch(W), to_torch(b), hc.HC_ACT_ELU, y)
+    assert hc.hc_get_device_status() == hc.HC_OK
+    y_pre, _ = oracle.sparse_spiral_conv(xin, layout, c, r, sp, W, b, oracle.ACT_ELU)
+    check_close(to_numpy(y)[:n], y_pre, f"rulebook conv {shape} layout={layout}")
+
+
+def test_encoder_through_rulebooks():
+    """Stacked layers sharing one mask: one rulebook for the dense-input first
+    layer and one for the compact layers after it, reused by every layer."""
+    w = inputs.make_workload("encoder655_bf16")
+    m = w.masks[0]
+    B, V = m.shape
+    rb_d, coords, row_of, count = gpu_rulebook(m, w.spiral, hc.HC_LAYOUT_DENSE)
+    rb_c = torch.empty_like(rb_d)
+    hc.hc_conv_rulebook(coords, row_of, count, to_torch(w.spiral), B, V, hc.HC_LAYOUT_COMPACT, rb_c)
+    h = to_torch(w.x)
+    first = True
+    for ly in w.layers:
+        y = torch.empty((B * V, ly.C_out), dtype=torch.bfloat16, device="cuda")
+        if ly.kind == "conv":
+            hc.hc_sparse_conv_rulebook_fwd(h, rb_d if first else rb_c, count, to_torch(ly.W),
+                                           to_torch(ly.b), ly.act, y)
+        else:
+            hc.hc_sparse_linear_fwd(h, count, to_torch(ly.W), to_torch(ly.b), ly.act, y)
+        h, first = y, False
+    assert hc.hc_get_device_status() == hc.HC_OK
+    c, r, o, n, outs = oracle.encoder(w.x, m, w.spiral, w.layers, n_threads=NCPU)
+    check_close(to_numpy(h)[:n], outs[-1][0], "encoder through rulebooks")
+
+
+def test_rulebook_full_size_sampled():
+    w = inputs.make_workload("layer10475_bf16")
+    ly = w.layers[0]
+    B, V = w.B, w.V
+    rb, coords, row_of, count = gpu_rulebook(w.masks[0], w.spiral, hc.HC_LAYOUT_DENSE)
+    c, r, _, n = oracle.mask_compact(w.masks[0])
+    np.testing.assert_array_equal(to_numpy(rb)[:, :n], oracle.conv_rulebook(c, r, w.spiral, 0)[:, :n])
+    y = torch.empty((B * V, ly.C_out), dtype=torch.bfloat16, device="cuda")
+    hc.hc_sparse_conv_rulebook_fwd(to_torch(w.x), rb, count, to_torch(ly.W), to_torch(ly.b),
+                                   ly.act, y)
+    assert hc.hc_get_device_status() == hc.HC_OK
+    rows = sample_rows(n, 3000, seed=5)
+    y_pre, _ = oracle.sparse_spiral_conv(w.x, oracle.LAYOUT_DENSE, c, r, w.spiral, ly.W, ly.b,
+                                         ly.act, rows=rows, n_threads=NCPU)
+    check_close(to_numpy(y)[rows], y_pre, "rulebook conv, 10475-vertex layer")
+
+
+def test_rulebook_entry_out_of_range_is_reported():
+    sp, m, x, W, b = inputs.random_case(77, 2, 100, 5, 64, 64, "bf16", 1.0)
+    rb, coords, row_of, count = gpu_rulebook(m, sp, hc.HC_LAYOUT_DENSE)
+    rb[2, 5] = 200  # == x_rows: out of range
+    rb[1, 7] = -3
+    y = torch.empty((200, 64), dtype=torch.bfloat16, device="cuda")
+    hc.hc_sparse_conv_rulebook_fwd(to_torch(x), rb, count, to_torch(W), to_torch(b), 1, y)
+    assert hc.hc_get_device_status() == hc.HC_ERR_INVALID_INDEX
+
+
 # ------------------------------------------------------------------ dense conv
 
 @pytest.mark.parametrize("dtype", ["bf16", "f32"])
