@@ -175,13 +175,21 @@ hc_status hc_conv_rulebook(const int32_t* coords, const int32_t* row_of, const i
  *   rulebook  [L, capacity] int32 as written by hc_conv_rulebook
  *             (capacity = B*V there)
  *   count     N' on the device, at most capacity (clamped, HC_ERR_CAPACITY)
- *   W, bias, act, y as for hc_sparse_spiral_conv_fwd; y [capacity, C_out].
- * Results equal hc_sparse_spiral_conv_fwd on the same inputs.
+ *   W, bias, act as for hc_sparse_spiral_conv_fwd.
+ *   y         [capacity, C_out] compact output of dtype dt, or NULL.
+ *   out       [B, V, C_out] dense output of dtype dt, or NULL: when given, row
+ *             n is also written at coords[n] = (b, v), the scatter of
+ *             hc_scatter_dense fused into the epilogue (inactive rows of out
+ *             are not touched). Needs coords (as written by hc_mask_compact),
+ *             B >= 1 and V >= 1. At least one of y and out must be given.
+ * Results equal hc_sparse_spiral_conv_fwd (and hc_scatter_dense without
+ * zero fill) on the same inputs.
  */
 hc_status hc_sparse_conv_rulebook_fwd(const void* x, hc_dtype dt, int x_rows,
                                       const int32_t* rulebook, const int32_t* count, int capacity,
                                       int L, int C_in, int C_out, const void* W, const float* bias,
-                                      hc_act act, void* y, hc_stream_t stream);
+                                      hc_act act, void* y, const int32_t* coords, int B, int V,
+                                      void* out, hc_stream_t stream);
 
 /*
  * hc_sparse_linear_fwd -- linear layer on compact rows (Eq. 6), row-wise

@@ -70,6 +70,8 @@ __global__ void __launch_bounds__(kThreads) compact_count_kernel(const uint8_t* 
                                                                  long long n,
                                                                  int32_t* __restrict__ tile_counts) {
     __shared__ int red[kThreads / 32];
+    pdl_wait();
+    pdl_trigger();
     long long base = (long long)blockIdx.x * kTile + (long long)threadIdx.x * kItems;
     int c = __popc(load_flags(mask, n, base));
     int t = block_sum(c, red);
@@ -81,6 +83,8 @@ __global__ void __launch_bounds__(1024) compact_scan_kernel(int32_t* __restrict_
                                                             int num_tiles) {
     __shared__ int warp_tot[32];
     __shared__ int carry;
+    pdl_wait();
+    pdl_trigger();
     if (threadIdx.x == 0) carry = 0;
     __syncthreads();
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -123,6 +127,8 @@ __global__ void __launch_bounds__(kThreads)
     __shared__ int tile_base_s;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int tile = blockIdx.x;
+    pdl_wait();
+    pdl_trigger();
 
     // Rows before this tile.
     int tile_base;
@@ -213,6 +219,8 @@ __global__ void __launch_bounds__(kThreads)
 }
 
 __global__ void compact_empty_kernel(int B, int32_t* offsets, int32_t* count) {
+    pdl_wait();
+    pdl_trigger();
     for (int i = threadIdx.x; i <= B; i += blockDim.x)
         if (offsets) offsets[i] = 0;
     if (threadIdx.x == 0) *count = 0;
@@ -225,24 +233,24 @@ hc_status launch_compact(const DeviceCtx* ctx, const uint8_t* mask, int B, int V
     (void)ctx;
     long long n = (long long)B * V;
     if (n == 0) {
-        compact_empty_kernel<<<1, 256, 0, s>>>(B, offsets, count);
-        return check_cuda(cudaGetLastError(), "compact_empty_kernel");
+        return launch_pdl(compact_empty_kernel, dim3(1), dim3(256), 0, s, "compact_empty_kernel", B,
+                          offsets, count);
     }
     int num_tiles = (int)((n + kTile - 1) / kTile);
     int32_t* tile_counts = (int32_t*)stream_workspace(s, sizeof(int32_t) * (size_t)num_tiles);
     if (!tile_counts) return HC_ERR_CUDA;
-    compact_count_kernel<<<num_tiles, kThreads, 0, s>>>(mask, n, tile_counts);
-    hc_status st = check_cuda(cudaGetLastError(), "compact_count_kernel");
+    hc_status st = launch_pdl(compact_count_kernel, dim3(num_tiles), dim3(kThreads), 0, s,
+                              "compact_count_kernel", mask, n, tile_counts);
     if (st != HC_OK) return st;
     int prescanned = num_tiles > kMaxDirectTiles;
     if (prescanned) {
-        compact_scan_kernel<<<1, 1024, 0, s>>>(tile_counts, num_tiles);
-        st = check_cuda(cudaGetLastError(), "compact_scan_kernel");
+        st = launch_pdl(compact_scan_kernel, dim3(1), dim3(1024), 0, s, "compact_scan_kernel",
+                        tile_counts, num_tiles);
         if (st != HC_OK) return st;
     }
-    compact_write_kernel<<<num_tiles, kThreads, 0, s>>>(mask, n, B, V, tile_counts, num_tiles,
-                                                        prescanned, coords, row_of, offsets, count);
-    return check_cuda(cudaGetLastError(), "compact_write_kernel");
+    return launch_pdl(compact_write_kernel, dim3(num_tiles), dim3(kThreads), 0, s,
+                      "compact_write_kernel", mask, n, B, V, tile_counts, num_tiles, prescanned,
+                      coords, row_of, offsets, count);
 }
 
 }  // namespace hc
@@ -299,22 +307,22 @@ hc_status launch_compact_into(const uint8_t* mask, int B, int V, int32_t* coords
                               int32_t* tile_counts, cudaStream_t s) {
     long long n = (long long)B * V;
     if (n == 0) {
-        compact_empty_kernel<<<1, 256, 0, s>>>(B, offsets, count);
-        return check_cuda(cudaGetLastError(), "compact_empty_kernel");
+        return launch_pdl(compact_empty_kernel, dim3(1), dim3(256), 0, s, "compact_empty_kernel", B,
+                          offsets, count);
     }
     int num_tiles = (int)((n + kTile - 1) / kTile);
-    compact_count_kernel<<<num_tiles, kThreads, 0, s>>>(mask, n, tile_counts);
-    hc_status st = check_cuda(cudaGetLastError(), "compact_count_kernel");
+    hc_status st = launch_pdl(compact_count_kernel, dim3(num_tiles), dim3(kThreads), 0, s,
+                              "compact_count_kernel", mask, n, tile_counts);
     if (st != HC_OK) return st;
     int prescanned = num_tiles > kMaxDirectTiles;
     if (prescanned) {
-        compact_scan_kernel<<<1, 1024, 0, s>>>(tile_counts, num_tiles);
-        st = check_cuda(cudaGetLastError(), "compact_scan_kernel");
+        st = launch_pdl(compact_scan_kernel, dim3(1), dim3(1024), 0, s, "compact_scan_kernel",
+                        tile_counts, num_tiles);
         if (st != HC_OK) return st;
     }
-    compact_write_kernel<<<num_tiles, kThreads, 0, s>>>(mask, n, B, V, tile_counts, num_tiles,
-                                                        prescanned, coords, row_of, offsets, count);
-    return check_cuda(cudaGetLastError(), "compact_write_kernel");
+    return launch_pdl(compact_write_kernel, dim3(num_tiles), dim3(kThreads), 0, s,
+                      "compact_write_kernel", mask, n, B, V, tile_counts, num_tiles, prescanned,
+                      coords, row_of, offsets, count);
 }
 
 }  // namespace

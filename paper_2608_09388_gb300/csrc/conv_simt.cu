@@ -51,6 +51,8 @@ __global__ void __launch_bounds__(kThreads) conv_simt_kernel(const ConvArgs a) {
     const T* __restrict__ x = static_cast<const T*>(a.x);
     const T* __restrict__ W = static_cast<const T*>(a.W);
     T* __restrict__ y = static_cast<T*>(a.y);
+    pdl_wait();
+    pdl_trigger();
     const long long rows = active_rows(a);
     const long long m_tiles = (rows + kBM - 1) / kBM;
     const int n0 = blockIdx.y * kBN;
@@ -164,12 +166,22 @@ __global__ void __launch_bounds__(kThreads) conv_simt_kernel(const ConvArgs a) {
         for (int i = 0; i < 4; ++i) {
             const long long n = m0 + ty * 4 + i;
             if (n >= rows) continue;
+            T* dp = nullptr;  // fused scatter destination row, if any
+            if (a.out_dense) {
+                const int b = __ldg(a.out_coords + 2 * n), v = __ldg(a.out_coords + 2 * n + 1);
+                if (b >= 0 && b < a.out_B && v >= 0 && v < a.out_V)
+                    dp = static_cast<T*>(a.out_dense) + ((long long)b * a.out_V + v) * C_out;
+                else
+                    report(a.status, kErrIndex);
+            }
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
                 const int col = n0 + tx * 4 + j;
                 if (col >= C_out) continue;
                 const float z = acc[i][j] + (a.bias ? __ldg(a.bias + col) : 0.f);
-                y[n * C_out + col] = from_float<T>(act_apply(z, a.act));
+                const T val = from_float<T>(act_apply(z, a.act));
+                if (y) y[n * C_out + col] = val;
+                if (dp) dp[col] = val;
             }
         }
     }
@@ -184,10 +196,10 @@ hc_status launch_conv_simt(const DeviceCtx* ctx, const ConvArgs& a, hc_dtype dt,
     dim3 grid((unsigned)gx, (unsigned)((a.C_out + kBN - 1) / kBN));
     size_t smem = sizeof(int) * (size_t)kBM * a.L;
     if (dt == HC_F32)
-        conv_simt_kernel<float><<<grid, kThreads, smem, s>>>(a);
-    else
-        conv_simt_kernel<__nv_bfloat16><<<grid, kThreads, smem, s>>>(a);
-    return check_cuda(cudaGetLastError(), "conv_simt_kernel");
+        return launch_pdl(conv_simt_kernel<float>, grid, dim3(kThreads), smem, s,
+                          "conv_simt_kernel", a);
+    return launch_pdl(conv_simt_kernel<__nv_bfloat16>, grid, dim3(kThreads), smem, s,
+                      "conv_simt_kernel", a);
 }
 
 }  // namespace hc

@@ -64,7 +64,7 @@ constexpr int kTabChunk = 8;  // spiral slots resolved per pass of the index war
 template <int BN>
 struct Cfg {
     static constexpr int kBStageBytes = kBK * BN * 2;
-    static constexpr int kStages = BN == 64 ? 8 : 6;
+    static constexpr int kStages = BN == 64 ? 7 : 5;
     static constexpr int kLag = kStages - 1;  // cp.async groups a producer keeps in flight
     static constexpr int kTmemCols = 2 * BN;  // two accumulators
     // Instruction descriptor, kind::f16: D fp32 (bit 4), A bf16 (bits 7-9 = 1),
@@ -77,9 +77,12 @@ struct Cfg {
     // tables at a 128-byte boundary (the TMA producer reads them 16 bytes at
     // a time).
     static constexpr int kTabOffset = (kBarBytes + 16 + 127) / 128 * 128;
+    // After the tables: one 2 KB staging buffer per epilogue warp (32 rows x
+    // 64 bytes of bf16 output).
+    static constexpr int kEpiBytes = kEpilogueWarps * 32 * 64;
     static size_t smem_bytes(int L) {
         return 1024 + (size_t)kStages * (kAStageBytes + kBStageBytes) + kTabOffset +
-               2 * sizeof(int) * (size_t)kBM * L;
+               2 * sizeof(int) * (size_t)kBM * L + kEpiBytes;
     }
 };
 
@@ -91,12 +94,18 @@ __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr, uint32_t lbo
            ((uint64_t)(sbo >> 4) << 32) | (1ull << 46) | (2ull << 61);
 }
 
-// Activation, bf16 rounding (RNE) and the 16-byte stores of one 32-column
-// chunk of one output row (r holds the fp32 sums with bias added).
+// Epilogue of one 32-column chunk of a warp's 32 output rows: activation,
+// bf16 rounding (RNE), then the stores. Lane i holds row i's 32 fp32 sums
+// (bias added) in r. The rows go through a 2 KB shared buffer (16-byte
+// pieces XOR-swizzled by row so that neither the writes nor the reads have
+// bank conflicts) and leave it so that each store instruction writes eight
+// rows x 64 contiguous bytes, instead of 32 scattered 16-byte pieces. Each
+// row goes to its compact position (row_y, 0 = none) and to its dense
+// position of the fused scatter (row_d, 0 = none).
 template <int ACT>
-__device__ __forceinline__ void epilogue_store(const uint32_t (&r)[32], __nv_bfloat16* y,
-                                               long long row, bool rvalid, int col0, int C_out) {
-    __nv_bfloat16* yp = y + (rvalid ? row : 0) * C_out + col0;
+__device__ __forceinline__ void epilogue_chunk(const uint32_t (&r)[32], uint32_t stage, int lane,
+                                               long long row_y, long long row_d, int col0,
+                                               int C_out) {
 #pragma unroll
     for (int j8 = 0; j8 < 4; ++j8) {
         uint32_t packed[4];
@@ -107,10 +116,23 @@ __device__ __forceinline__ void epilogue_store(const uint32_t (&r)[32], __nv_bfl
                                                            act_fixed<ACT>(__uint_as_float(r[j + 1])));
             packed[h] = *reinterpret_cast<const uint32_t*>(&p);
         }
-        if (rvalid && col0 + j8 * 8 < C_out)
-            *reinterpret_cast<uint4*>(yp + j8 * 8) =
-                make_uint4(packed[0], packed[1], packed[2], packed[3]);
+        sts_v4(stage + (uint32_t)(lane * 64 + ((j8 ^ ((lane >> 1) & 3)) << 4)),
+               make_uint4(packed[0], packed[1], packed[2], packed[3]));
     }
+    __syncwarp();
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const int R = 8 * k + (lane >> 2), piece = lane & 3;
+        const uint4 v = lds_u4(stage + (uint32_t)(R * 64 + ((piece ^ ((R >> 1) & 3)) << 4)));
+        const long long yR = __shfl_sync(0xffffffffu, row_y, R);
+        const long long dR = __shfl_sync(0xffffffffu, row_d, R);
+        const int col = col0 + piece * 8;
+        if (col < C_out) {
+            if (yR) *reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(yR) + col) = v;
+            if (dR) *reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(dR) + col) = v;
+        }
+    }
+    __syncwarp();  // the buffer is reused by the next chunk
 }
 
 template <int BN, bool kTma>
@@ -132,6 +154,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // Tap tables, [2][L][kBM] int32: entry (l, r) is the input row feeding
     // slot l of tile row r, or -1.
     const uint32_t tab0 = sBar + C::kTabOffset;
+    const uint32_t epi0 = tab0 + 2u * (uint32_t)(kBM * a.L) * 4u;  // epilogue staging
 
     auto full_bar = [&](int s) { return sBar + 8u * s; };
     auto empty_bar = [&](int s) { return sBar + 8u * (C::kStages + s); };
@@ -172,6 +195,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem_base = *tmem_holder;
+    // The prologue above touched only on-chip state; global memory written
+    // by the previous grid is read from here on.
+    pdl_wait();
+    pdl_trigger();
 
     const long long rows = active_rows(a);
     const long long m_tiles = (rows + kBM - 1) / kBM;
@@ -519,6 +546,18 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_after();
             const long long row = m0 + ew * 32 + lane;
             const bool rvalid = row < rows;
+            // Row start addresses (0 = not written) of this lane's row.
+            const long long row_y = (rvalid && y) ? (long long)(y + row * C_out) : 0;
+            long long row_d = 0;
+            if (rvalid && a.out_dense) {
+                const int b = __ldg(a.out_coords + 2 * row), v = __ldg(a.out_coords + 2 * row + 1);
+                if (b >= 0 && b < a.out_B && v >= 0 && v < a.out_V)
+                    row_d = (long long)(static_cast<__nv_bfloat16*>(a.out_dense) +
+                                        ((long long)b * a.out_V + v) * C_out);
+                else
+                    report(a.status, kErrIndex);
+            }
+            const uint32_t stage = epi0 + (uint32_t)ew * 2048u;
 #pragma unroll 1
             for (int cb = 0; cb < BN / 32; ++cb) {
                 uint32_t r[32];
@@ -536,11 +575,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                                            __shfl_sync(0xffffffffu, bias_l, j));
                 // The activation is chosen once per chunk, not per element.
                 if (a.act == HC_ACT_ELU)
-                    epilogue_store<HC_ACT_ELU>(r, y, row, rvalid, col0, C_out);
+                    epilogue_chunk<HC_ACT_ELU>(r, stage, lane, row_y, row_d, col0, C_out);
                 else if (a.act == HC_ACT_RELU)
-                    epilogue_store<HC_ACT_RELU>(r, y, row, rvalid, col0, C_out);
+                    epilogue_chunk<HC_ACT_RELU>(r, stage, lane, row_y, row_d, col0, C_out);
                 else
-                    epilogue_store<HC_ACT_NONE>(r, y, row, rvalid, col0, C_out);
+                    epilogue_chunk<HC_ACT_NONE>(r, stage, lane, row_y, row_d, col0, C_out);
             }
             tc_fence_before();
             mbar_arrive(tempty_bar(acc));
@@ -620,14 +659,15 @@ hc_status launch_bn(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s) {
     const long long cap_work = (a.capacity + kBM - 1) / kBM * n_tiles;
     long long grid = cap_work < ctx->num_sms ? cap_work : ctx->num_sms;
     if (grid < 1) grid = 1;
-    conv_tc_kernel<BN, kTma><<<(unsigned)grid, kThreads, C::smem_bytes(a.L), s>>>(a, tx, tw);
-    return check_cuda(cudaGetLastError(), "conv_tc_kernel");
+    return launch_pdl(conv_tc_kernel<BN, kTma>, dim3((unsigned)grid), dim3(kThreads),
+                      C::smem_bytes(a.L), s, "conv_tc_kernel", a, tx, tw);
 }
 
 }  // namespace
 
 bool conv_tc_supported(const ConvArgs& a, hc_dtype dt) {
-    const uintptr_t al = (uintptr_t)a.x | (uintptr_t)a.W | (uintptr_t)a.y;
+    const uintptr_t al =
+        (uintptr_t)a.x | (uintptr_t)a.W | (uintptr_t)a.y | (uintptr_t)a.out_dense;
     return dt == HC_BF16 && a.C_in % 8 == 0 && a.C_out % 8 == 0 && al % 16 == 0 &&
            a.L <= HC_MAX_SPIRAL;
 }

@@ -289,13 +289,20 @@ hc_status hc_conv_rulebook(const int32_t* coords, const int32_t* row_of, const i
 hc_status hc_sparse_conv_rulebook_fwd(const void* x, hc_dtype dt, int x_rows,
                                       const int32_t* rulebook, const int32_t* count, int capacity,
                                       int L, int C_in, int C_out, const void* W, const float* bias,
-                                      hc_act act, void* y, hc_stream_t stream) {
+                                      hc_act act, void* y, const int32_t* coords, int B, int V,
+                                      void* out, hc_stream_t stream) {
     const char* fn = "hc_sparse_conv_rulebook_fwd";
     t_last_error[0] = 0;
-    hc_status st = check_conv_common(fn, dt, L, C_in, C_out, act, x, W, y);
+    HC_REQUIRE(y || out, "%s: at least one of y and out is required", fn);
+    hc_status st = check_conv_common(fn, dt, L, C_in, C_out, act, x, W, y ? y : out);
     if (st != HC_OK) return st;
     HC_REQUIRE(x_rows >= 1 && capacity >= 0, "%s: x_rows=%d capacity=%d", fn, x_rows, capacity);
     HC_REQUIRE(rulebook && count, "%s: rulebook and count are required", fn);
+    if (out) {
+        HC_REQUIRE(coords && B >= 1 && V >= 1, "%s: out needs coords, B >= 1 and V >= 1", fn);
+        HC_REQUIRE((long long)B * V < (1ll << 31), "%s: B*V must be < 2^31", fn);
+        HC_REQUIRE(!misaligned(out, dt == HC_F32 ? 4 : 2), "%s: misaligned out", fn);
+    }
     if (capacity == 0) return HC_OK;
     const DeviceCtx* ctx = device_ctx();
     if (!ctx) return HC_ERR_CUDA;
@@ -316,6 +323,10 @@ hc_status hc_sparse_conv_rulebook_fwd(const void* x, hc_dtype dt, int x_rows,
     a.K = L * C_in;
     a.mode = kRulebook;
     a.act = act;
+    a.out_dense = out;
+    a.out_coords = coords;
+    a.out_B = B;
+    a.out_V = V;
     return dispatch_conv(ctx, a, dt, (cudaStream_t)stream);
 }
 

@@ -60,6 +60,11 @@ struct ConvArgs {
     long long capacity;  // upper bound on rows (B*V, or the linear capacity)
     long long x_rows;    // rows of the input x (valid input row indices are < x_rows)
     const int32_t* rulebook;  // kRulebook: [L, capacity] slot-major tap rows, -1 = absent
+    // Optional fused scatter (Eq. 2 inverse): row n is also written to
+    // out_dense[(b*out_V + v)*C_out ...] with (b, v) = out_coords[n].
+    void* out_dense;
+    const int32_t* out_coords;
+    int out_B, out_V;
     int B, V, L, C_in, C_out, K;  // K = L*C_in
     int mode;
     int act;
@@ -79,8 +84,41 @@ hc_status launch_scatter(const DeviceCtx* ctx, const void* y, int elem_bytes, co
                          const int32_t* row_of, const int32_t* count, int B, int V, int C,
                          int zero_fill, void* out, cudaStream_t s);
 
+// ------------------------------------------------------------ launches
+// Every kernel of the library is launched with programmatic stream
+// serialisation: it may be scheduled while the previous kernel on the stream
+// is still finishing, runs its on-chip prologue, and waits (pdl_wait) for
+// the previous grid to complete before its first global-memory access.
+#if defined(__CUDACC__)
+template <typename... KArgs, typename... Args>
+hc_status launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                     cudaStream_t s, const char* what, Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return check_cuda(cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...), what);
+}
+#endif
+
 // ------------------------------------------------------------ device helpers
 #if defined(__CUDACC__)
+
+// Wait until the previous grid on the stream has completed and its writes are
+// visible (a no-op without a programmatic dependency), then allow the next
+// grid to be scheduled early.
+__device__ __forceinline__ void pdl_wait() {
+    asm volatile("griddepcontrol.wait;\n" ::: "memory");
+}
+__device__ __forceinline__ void pdl_trigger() {
+    asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
+}
 
 __device__ __forceinline__ void report(unsigned* status, unsigned bit) {
     atomicOr(status, bit);
@@ -288,6 +326,19 @@ __device__ __forceinline__ void tma_gather4(uint32_t dst, const void* tmap, int 
 }
 __device__ __forceinline__ void prefetch_tensormap(const void* tmap) {
     asm volatile("prefetch.tensormap [%0];\n" ::"l"(reinterpret_cast<uint64_t>(tmap)) : "memory");
+}
+__device__ __forceinline__ void sts_v4(uint32_t addr, uint4 v) {
+    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};\n" ::"r"(addr), "r"(v.x), "r"(v.y),
+                 "r"(v.z), "r"(v.w)
+                 : "memory");
+}
+__device__ __forceinline__ uint4 lds_u4(uint32_t addr) {
+    uint4 v;
+    asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];\n"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "r"(addr)
+                 : "memory");
+    return v;
 }
 __device__ __forceinline__ int4 lds_v4(uint32_t addr) {
     int4 v;

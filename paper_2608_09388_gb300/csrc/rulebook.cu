@@ -23,6 +23,8 @@ __global__ void __launch_bounds__(256) rulebook_kernel(const int32_t* __restrict
                                                        int V, int L, int x_layout,
                                                        int32_t* __restrict__ rulebook,
                                                        unsigned* status) {
+    pdl_wait();
+    pdl_trigger();
     const long long cap = (long long)B * V;
     long long rows = *count;
     unsigned err = 0;
@@ -80,9 +82,8 @@ hc_status launch_rulebook(const DeviceCtx* ctx, const int32_t* coords, const int
     const long long lim = (long long)ctx->num_sms * 8;
     if (blocks > lim) blocks = lim;
     if (blocks < 1) blocks = 1;
-    rulebook_kernel<<<(unsigned)blocks, 256, 0, s>>>(coords, row_of, count, spiral, B, V, L,
-                                                      x_layout, rulebook, ctx->status);
-    return check_cuda(cudaGetLastError(), "rulebook_kernel");
+    return launch_pdl(rulebook_kernel, dim3((unsigned)blocks), dim3(256), 0, s, "rulebook_kernel",
+                      coords, row_of, count, spiral, B, V, L, x_layout, rulebook, ctx->status);
 }
 
 }  // namespace hc

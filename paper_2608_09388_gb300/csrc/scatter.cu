@@ -43,6 +43,8 @@ template <typename U>
 __global__ void scatter_kernel(const U* __restrict__ y, const int32_t* __restrict__ coords,
                                const int32_t* __restrict__ count, int B, int V, int cpr,
                                U* __restrict__ out, unsigned* status) {
+    pdl_wait();
+    pdl_trigger();
     const long long rows = clamp_count(count, (long long)B * V, status);
     const long long total = rows * cpr;
     for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
@@ -62,6 +64,8 @@ template <typename U>
 __global__ void scatter_fill_kernel(const U* __restrict__ y, const int32_t* __restrict__ row_of,
                                     const int32_t* __restrict__ count, long long dense_rows,
                                     int cpr, U* __restrict__ out, unsigned* status) {
+    pdl_wait();
+    pdl_trigger();
     const long long rows = clamp_count(count, dense_rows, status);
     const long long total = dense_rows * cpr;
     for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
@@ -89,12 +93,11 @@ hc_status launch_typed(const DeviceCtx* ctx, const void* y, const int32_t* coord
     if (blocks > cap) blocks = cap;
     if (blocks < 1) blocks = 1;
     if (zero_fill)
-        scatter_fill_kernel<U><<<(unsigned)blocks, 256, 0, s>>>(
-            (const U*)y, row_of, count, dense_rows, cpr, (U*)out, ctx->status);
-    else
-        scatter_kernel<U><<<(unsigned)blocks, 256, 0, s>>>((const U*)y, coords, count, B, V, cpr,
-                                                          (U*)out, ctx->status);
-    return check_cuda(cudaGetLastError(), "scatter_kernel");
+        return launch_pdl(scatter_fill_kernel<U>, dim3((unsigned)blocks), dim3(256), 0, s,
+                          "scatter_fill_kernel", (const U*)y, row_of, count, dense_rows, cpr,
+                          (U*)out, ctx->status);
+    return launch_pdl(scatter_kernel<U>, dim3((unsigned)blocks), dim3(256), 0, s, "scatter_kernel",
+                      (const U*)y, coords, count, B, V, cpr, (U*)out, ctx->status);
 }
 
 }  // namespace

@@ -60,7 +60,8 @@ def load_library(path: str | None = None):
             "hc_mask_compact_static": [P, I, I, P, P, P, P, P],
             "hc_sparse_spiral_conv_fwd": [P, I, I, P, P, P, P, I, I, I, I, I, P, P, I, P, P],
             "hc_conv_rulebook": [P, P, P, P, I, I, I, I, P, P],
-            "hc_sparse_conv_rulebook_fwd": [P, I, I, P, P, I, I, I, I, P, P, I, P, P],
+            "hc_sparse_conv_rulebook_fwd": [P, I, I, P, P, I, I, I, I, P, P, I, P, P, I, I, P,
+                                            P],
             "hc_sparse_linear_fwd": [P, I, P, I, I, I, P, P, I, P, P],
             "hc_scatter_dense": [P, I, P, P, P, I, I, I, I, P, P],
             "hc_spiral_conv_fwd": [P, I, P, I, I, I, I, I, P, P, I, P, P],
@@ -146,16 +147,20 @@ def hc_conv_rulebook(coords, row_of, count, spiral, B, V, x_layout, rulebook, st
            "hc_conv_rulebook")
 
 
-def hc_sparse_conv_rulebook_fwd(x, rulebook, count, W, bias, act, y, stream=None):
+def hc_sparse_conv_rulebook_fwd(x, rulebook, count, W, bias, act, y, coords=None, out=None,
+                                stream=None):
     """Sparse conv through a rulebook [L, capacity]: x [x_rows, C_in] (or [B, V, C_in]),
-    W [L*C_in, C_out], y [capacity, C_out]."""
+    W [L*C_in, C_out], y [capacity, C_out] or None; out [B, V, C_out] (fused scatter at
+    coords) or None."""
     L, capacity = rulebook.shape
     C_in = x.shape[-1]
     x_rows = x.numel() // C_in
     C_out = W.shape[1]
+    B, V = (out.shape[0], out.shape[1]) if out is not None else (0, 0)
     _check(load_library().hc_sparse_conv_rulebook_fwd(
-        _p(x), _dt(x), x_rows, _p(rulebook), _p(count), capacity, L, C_in, C_out, _p(W),
-        _p(bias), act, _p(y), _s(stream)), "hc_sparse_conv_rulebook_fwd")
+        _p(x), _dt(x if y is None else y), x_rows, _p(rulebook), _p(count), capacity, L, C_in,
+        C_out, _p(W), _p(bias), act, _p(y), _p(coords), B, V, _p(out), _s(stream)),
+        "hc_sparse_conv_rulebook_fwd")
 
 
 def hc_sparse_linear_fwd(x, count, W, bias, act, y, stream=None):

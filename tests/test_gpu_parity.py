@@ -266,6 +266,35 @@ def test_conv_through_rulebook(shape, layout):
     check_close(to_numpy(y)[:n], y_pre, f"rulebook conv {shape} layout={layout}")
 
 
+@pytest.mark.parametrize("shape", [(3, 200, 9, 64, 128, "bf16"), (2, 300, 9, 24, 40, "bf16"),
+                                   (2, 300, 9, 45, 64, "bf16"), (1, 655, 9, 16, 64, "f32")])
+@pytest.mark.parametrize("with_compact", [True, False])
+def test_conv_through_rulebook_fused_scatter(shape, with_compact):
+    """The rulebook conv writing the dense [B, V, C_out] tensor directly (the
+    scatter fused into its epilogue): active rows hold the conv result, all
+    other rows keep their previous contents."""
+    B, V, L, C_in, C_out, dtype = shape
+    sp, m, x, W, b = inputs.random_case(B * 7 + V + C_in, B, V, L, C_in, C_out, dtype, 0.3, 0.1)
+    rb, coords, row_of, count = gpu_rulebook(m, sp, hc.HC_LAYOUT_DENSE)
+    c, r, _, n = oracle.mask_compact(m)
+    xt = to_torch(x)
+    prev = inputs.features(np.random.default_rng(3), (B, V, C_out), dtype)
+    out = to_torch(prev)
+    y = torch.full((B * V, C_out), float("nan"), dtype=xt.dtype, device="cuda") if with_compact \
+        else None
+    hc.hc_sparse_conv_rulebook_fwd(xt, rb, count, to_torch(W), to_torch(b), hc.HC_ACT_ELU, y,
+                                   coords=coords, out=out)
+    assert hc.hc_get_device_status() == hc.HC_OK
+    got = to_numpy(out)
+    y_pre, _ = oracle.sparse_spiral_conv(x, oracle.LAYOUT_DENSE, c, r, sp, W, b, oracle.ACT_ELU)
+    check_close(got[c[:, 0], c[:, 1]], y_pre, f"fused scatter {shape}")
+    inactive = np.ones((B, V), bool)
+    inactive[c[:, 0], c[:, 1]] = False
+    np.testing.assert_array_equal(got[inactive], prev[inactive])
+    if with_compact:
+        np.testing.assert_array_equal(to_numpy(y)[:n], got[c[:, 0], c[:, 1]])
+
+
 def test_encoder_through_rulebooks():
     """Stacked layers sharing one mask: one rulebook for the dense-input first
     layer and one for the compact layers after it, reused by every layer."""
