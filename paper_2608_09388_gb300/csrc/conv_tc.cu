@@ -13,13 +13,13 @@
 //              load of a phase in flight at once, into one of two tables, so
 //              the next tile's table is built while the current one is used;
 //   warps 0-3  producers: fill a stage with the 128 rows x 64 bf16 of A for
-//              one k-block and the 64 x BN slice of W. With C_in a multiple
-//              of 64 (a k-block never straddles two slots) one lane per warp
-//              issues TMA: tile::gather4 loads of four table rows at a time
-//              (absent taps use an out-of-range row, which TMA fills with
-//              zeros) and tiled loads of W, completing on the stage's "full"
-//              mbarrier by transaction count. Other channel counts use 16-byte
-//              cp.async per thread (zero-fill for absent taps);
+//              one k-block and the 64 x BN slice of W. The 128 threads gather
+//              A with 16-byte cp.async through the tap table (zero-fill for
+//              absent taps and for k past L*C_in) and signal completion on
+//              the stage's "full" mbarrier without blocking; thread 0 loads
+//              W with TMA tiled copies onto the same barrier (transaction
+//              count). Gather and weight loads thus use different engines.
+//              (A variant loads W with cp.async too, for comparison.);
 //   warp 8     MMA issuer (one thread): 4 x tcgen05.mma (K = 16 each) per
 //              stage into a TMEM accumulator, tcgen05.commit frees the stage;
 //   warps 4-7  epilogue: tcgen05.ld the 128 x BN fp32 accumulator (warp w
@@ -33,8 +33,8 @@
 //      block a [64 K-rows x 128 bytes] slab, K-row kr at kr*128 with chunk
 //      q stored at q ^ (kr % 8); 8-row groups 1024 bytes apart (SBO), the
 //      64-column blocks BK*128 bytes apart (LBO).
-// The TMA 128-byte swizzle writes exactly these layouts (stage buffers are
-// 1024-byte aligned).
+// The TMA 128-byte swizzle writes exactly the B layout (stage buffers are
+// 1024-byte aligned); the cp.async gather computes the A swizzle itself.
 // Every mbarrier wait is bounded (hc::kWaitLimitNs); on timeout the CTA
 // records HC_ERR_TIMEOUT, unwinds, waits for its own copies and MMAs and
 // frees its TMEM.
@@ -60,19 +60,24 @@ constexpr int kMmaWarp = kProducerWarps + kEpilogueWarps;
 constexpr int kIndexWarp = kMmaWarp + 1;
 constexpr int kThreads = (kIndexWarp + 1) * 32;
 constexpr int kTabChunk = 8;  // spiral slots resolved per pass of the index warp
+constexpr size_t kSmemLimit = 227 * 1024;  // opt-in dynamic shared memory per CTA
 
 template <int BN>
 struct Cfg {
+    static_assert(BN == 64 || BN == 128, "tile widths");
     static constexpr int kBStageBytes = kBK * BN * 2;
-    static constexpr int kStages = BN == 64 ? 7 : 5;
-    static constexpr int kLag = kStages - 1;  // cp.async groups a producer keeps in flight
+    // Pipeline depth: as many stages as fit next to the tap tables (which
+    // grow with L), between kMinStages and kMaxStages.
+    static constexpr int kMaxStages = BN == 64 ? 8 : 6;
+    static constexpr int kMinStages = BN == 64 ? 7 : 5;
+    static constexpr int kLag = kMinStages - 1;  // cp.async groups a producer keeps in flight
     static constexpr int kTmemCols = 2 * BN;  // two accumulators
     // Instruction descriptor, kind::f16: D fp32 (bit 4), A bf16 (bits 7-9 = 1),
     // B bf16 (bits 10-12 = 1), A K-major (bit 15 = 0), B MN-major (bit 16 = 1),
     // N >> 3 at bits 17-22, M >> 4 at bits 24-28.
     static constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | (1u << 16) |
                                        ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(kBM >> 4) << 24);
-    static constexpr int kBarBytes = 8 * (2 * kStages + 9);
+    static constexpr int kBarBytes = 8 * (2 * kMaxStages + 9);
     // barriers, then 16 bytes (TMEM address, abort flag), then the two tap
     // tables at a 128-byte boundary (the TMA producer reads them 16 bytes at
     // a time).
@@ -80,9 +85,14 @@ struct Cfg {
     // After the tables: one 2 KB staging buffer per epilogue warp (32 rows x
     // 64 bytes of bf16 output).
     static constexpr int kEpiBytes = kEpilogueWarps * 32 * 64;
-    static size_t smem_bytes(int L) {
-        return 1024 + (size_t)kStages * (kAStageBytes + kBStageBytes) + kTabOffset +
+    static size_t smem_bytes(int L, int stages) {
+        return 1024 + (size_t)stages * (kAStageBytes + kBStageBytes) + kTabOffset +
                2 * sizeof(int) * (size_t)kBM * L + kEpiBytes;
+    }
+    static int stages_for(int L) {
+        int st = kMaxStages;
+        while (st > kMinStages && smem_bytes(L, st) > kSmemLimit) --st;
+        return st;
     }
 };
 
@@ -140,14 +150,17 @@ __global__ void __launch_bounds__(kThreads, 1)
     conv_tc_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                    const __grid_constant__ CUtensorMap tmap_w) {
     using C = Cfg<BN>;
-    constexpr int kStageArrivals = kTma ? kProducerWarps : kProducerWarps * 32;
+    // "full": one cp.async completion arrival per producer thread, plus the
+    // expect-tx arrival of the weight TMA in the hybrid producer.
+    constexpr int kStageArrivals = kProducerWarps * 32 + (kTma ? 1 : 0);
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;
     uint8_t* const base_ptr = smem_raw + (base - raw);
     const uint32_t sA = base;
-    const uint32_t sB = sA + C::kStages * kAStageBytes;
-    const uint32_t sBar = sB + C::kStages * C::kBStageBytes;
+    const int nst = a.stages;
+    const uint32_t sB = sA + nst * kAStageBytes;
+    const uint32_t sBar = sB + nst * C::kBStageBytes;
     uint8_t* const misc = base_ptr + (sBar - base) + C::kBarBytes;
     volatile uint32_t* const tmem_holder = reinterpret_cast<volatile uint32_t*>(misc);
     volatile int* const abort_flag = reinterpret_cast<volatile int*>(misc + 4);
@@ -157,17 +170,17 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t epi0 = tab0 + 2u * (uint32_t)(kBM * a.L) * 4u;  // epilogue staging
 
     auto full_bar = [&](int s) { return sBar + 8u * s; };
-    auto empty_bar = [&](int s) { return sBar + 8u * (C::kStages + s); };
-    auto tfull_bar = [&](int i) { return sBar + 8u * (2 * C::kStages + i); };
-    auto tempty_bar = [&](int i) { return sBar + 8u * (2 * C::kStages + 2 + i); };
-    const uint32_t fin_bar = sBar + 8u * (2 * C::kStages + 4);
-    auto tabfull_bar = [&](int i) { return sBar + 8u * (2 * C::kStages + 5 + i); };
-    auto tabempty_bar = [&](int i) { return sBar + 8u * (2 * C::kStages + 7 + i); };
+    auto empty_bar = [&](int s) { return sBar + 8u * (C::kMaxStages + s); };
+    auto tfull_bar = [&](int i) { return sBar + 8u * (2 * C::kMaxStages + i); };
+    auto tempty_bar = [&](int i) { return sBar + 8u * (2 * C::kMaxStages + 2 + i); };
+    const uint32_t fin_bar = sBar + 8u * (2 * C::kMaxStages + 4);
+    auto tabfull_bar = [&](int i) { return sBar + 8u * (2 * C::kMaxStages + 5 + i); };
+    auto tabempty_bar = [&](int i) { return sBar + 8u * (2 * C::kMaxStages + 7 + i); };
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < C::kStages; ++s) {
+        for (int s = 0; s < nst; ++s) {
             mbar_init(full_bar(s), kStageArrivals);
             mbar_init(empty_bar(s), 1);
         }
@@ -178,15 +191,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_init(fin_bar, 1);
         for (int i = 0; i < 2; ++i) {
             mbar_init(tabfull_bar(i), 32);
-            mbar_init(tabempty_bar(i), kStageArrivals);
+            mbar_init(tabempty_bar(i), kProducerWarps * 32);
         }
         *abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
     }
-    if (kTma && threadIdx.x == 32) {
-        prefetch_tensormap(&tmap_x);
-        prefetch_tensormap(&tmap_w);
-    }
+    if (kTma && threadIdx.x == 32) prefetch_tensormap(&tmap_w);
     if (warp == kMmaWarp) {
         tmem_alloc(smem_u32((const void*)tmem_holder), C::kTmemCols);
         tmem_relinquish();
@@ -211,72 +221,81 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp < kProducerWarps) {
         // ------------------------------------------------------------ producers
         if constexpr (kTma) {
-            // Warp w gathers tile rows [32w, 32w+32) of A with eight gather4
-            // loads issued by lanes 0-7 (one each: a TMA issue takes an
-            // issuing thread a few hundred cycles, so spreading the loads
-            // over lanes multiplies the issue rate); lanes 8 and 9 of warp 0
-            // load the W slice. Lane 0 keeps the pipeline bookkeeping.
-            {
-                const int height = (int)a.x_rows;  // rows of the x tensor map
-                const uint32_t my_bytes =
-                    8u * 512u + (warp == 0 ? (uint32_t)(BN / 64) * (kBK * 128u) : 0u);
-                long long it = 0;
-                int lt = 0;
-                bool ok = true;
-                for (long long w = blockIdx.x; w < work_total && ok; w += gridDim.x, ++lt) {
-                    const int n0 = (int)(w % n_tiles) * BN;
-                    const int buf = lt & 1;
-                    // Every lane waits (so every lane acquires the table); the
-                    // warp then agrees on the outcome and stays converged.
-                    ok = __all_sync(0xffffffffu, mbar_wait(tabfull_bar(buf),
-                                                           (uint32_t)((lt >> 1) & 1), abort_flag,
-                                                           a.status));
-                    if (!ok) break;
-                    const uint32_t tab_s = tab0 + (uint32_t)buf * tab_bytes;
-                    int l = 0, c = 0;  // slot and channel offset of k-block kb
-                    for (int kb = 0; kb < num_kb; ++kb) {
-                        const int s = (int)(it % C::kStages);
-                        const uint32_t ph = (uint32_t)((it / C::kStages) & 1);
-                        ok = __all_sync(0xffffffffu,
-                                        mbar_wait(empty_bar(s), ph ^ 1u, abort_flag, a.status));
-                        if (!ok) break;
-                        if (lane == 0) mbar_arrive_expect_tx(full_bar(s), my_bytes);
-                        __syncwarp();
-                        const uint32_t a_st = sA + s * kAStageBytes;
-                        if (lane < 8) {
-                            const int r0 = 32 * warp + 4 * lane;
-                            int4 src = lds_v4(tab_s + (uint32_t)(l * kBM + r0) * 4u);
-                            src.x = src.x < 0 ? height : src.x;
-                            src.y = src.y < 0 ? height : src.y;
-                            src.z = src.z < 0 ? height : src.z;
-                            src.w = src.w < 0 ? height : src.w;
-                            tma_gather4(a_st + (uint32_t)r0 * 128u, &tmap_x, c, src.x, src.y,
-                                        src.z, src.w, full_bar(s));
-                        } else if (warp == 0 && lane < 8 + BN / 64) {
-                            const int nb = lane - 8;
+            // A is gathered by all 128 producer threads with 16-byte cp.async
+            // (row r of the stage at r*128 bytes, chunk q at q ^ (r % 8)),
+            // whose completion each thread signals on the stage's "full"
+            // barrier without blocking (cp.async.mbarrier.arrive.noinc);
+            // thread 0 loads the W slice with TMA tiled copies on the same
+            // barrier (transaction count). The two paths run on different
+            // engines (load/store unit and TMA), which measured ~1.8x the
+            // ingress of gathering the rows with TMA as well.
+            const __nv_bfloat16* __restrict__ x = static_cast<const __nv_bfloat16*>(a.x);
+            const int t = threadIdx.x;  // 0..127
+            const int q = t & 7;        // A: 16-byte chunk of the 128-byte row
+            constexpr uint32_t kWBytes = (uint32_t)(BN / 64) * (kBK * 128u);
+            long long it = 0;
+            int lt = 0;
+            bool ok = true;
+            for (long long w = blockIdx.x; w < work_total && ok; w += gridDim.x, ++lt) {
+                const int n0 = (int)(w % n_tiles) * BN;
+                const int buf = lt & 1;
+                if (!mbar_wait(tabfull_bar(buf), (uint32_t)((lt >> 1) & 1), abort_flag,
+                               a.status)) {
+                    ok = false;
+                    break;
+                }
+                const uint32_t tab_s = tab0 + (uint32_t)buf * tab_bytes;
+                int l = (q * 8) / C_in;  // slot and channel of this thread's chunk at k-block 0
+                int c = q * 8 - l * C_in;
+                for (int kb = 0; kb < num_kb; ++kb) {
+                    const int s = (int)(it % nst);
+                    const uint32_t ph = (uint32_t)((it / nst) & 1);
+                    if (!mbar_wait(empty_bar(s), ph ^ 1u, abort_flag, a.status)) {
+                        ok = false;
+                        break;
+                    }
+                    if (t == 0) {
+                        mbar_arrive_expect_tx(full_bar(s), kWBytes);
+#pragma unroll
+                        for (int nb = 0; nb < BN / 64; ++nb)
                             tma_load_2d(sB + s * C::kBStageBytes + nb * (kBK * 128), &tmap_w,
                                         n0 + nb * 64, kb * kBK, full_bar(s));
-                        }
-                        ++it;
-                        c += kBK;
-                        if (c >= C_in) {
-                            c = 0;
-                            ++l;
-                        }
                     }
-                    __syncwarp();
-                    if (ok && lane == 0) mbar_arrive(tabempty_bar(buf));
+                    const uint32_t a_st = sA + s * kAStageBytes;
+                    const bool kval = kb * kBK + q * 8 < K;
+                    // All eight table entries of this stage first, then the copies.
+                    int src[8];
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) {
+                        const int r = (t >> 3) + 16 * i;
+                        src[i] = kval ? lds_s32(tab_s + (uint32_t)(l * kBM + r) * 4u) : -1;
+                    }
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) {
+                        const int r = (t >> 3) + 16 * i;
+                        const __nv_bfloat16* gp =
+                            x + (src[i] >= 0 ? (long long)src[i] * C_in + c : 0);
+                        cp_async_16(a_st + r * 128 + ((q ^ (r & 7)) << 4), gp, src[i] >= 0);
+                    }
+                    cp_async_arrive_noinc(full_bar(s));
+                    ++it;
+                    c += kBK;
+                    while (c >= C_in) {
+                        c -= C_in;
+                        ++l;
+                    }
                 }
-                __syncwarp();
-                if (!ok && lane == 0) {
-                    // Let the copies already issued land before the CTA exits.
-                    int no_abort = 0;
-                    for (long long j = it > C::kStages ? it - C::kStages : 0; j < it; ++j)
-                        mbar_wait(full_bar((int)(j % C::kStages)), (uint32_t)((j / C::kStages) & 1),
-                                  &no_abort, a.status);
-                }
+                // Addresses of this tile's copies are issued: the table is free.
+                if (ok) mbar_arrive(tabempty_bar(buf));
             }
-            __syncwarp();
+            cp_async_wait_all();
+            if (!ok && t == 0) {
+                // Let the weight copies already issued land before the CTA exits.
+                int no_abort = 0;
+                for (long long j = it > nst ? it - nst : 0; j < it; ++j)
+                    mbar_wait(full_bar((int)(j % nst)), (uint32_t)((j / nst) & 1),
+                              &no_abort, a.status);
+            }
         } else {
             const __nv_bfloat16* __restrict__ x = static_cast<const __nv_bfloat16*>(a.x);
             const __nv_bfloat16* __restrict__ W = static_cast<const __nv_bfloat16*>(a.W);
@@ -297,8 +316,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 int l = (q * 8) / C_in;  // slot and channel of this thread's chunk at k-block 0
                 int c = q * 8 - l * C_in;
                 for (int kb = 0; kb < num_kb; ++kb) {
-                    const int s = (int)(it % C::kStages);
-                    const uint32_t ph = (uint32_t)((it / C::kStages) & 1);
+                    const int s = (int)(it % nst);
+                    const uint32_t ph = (uint32_t)((it / nst) & 1);
                     if (!mbar_wait(empty_bar(s), ph ^ 1u, abort_flag, a.status)) {
                         ok = false;
                         break;
@@ -336,7 +355,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (it >= C::kLag) {
                         cp_async_wait<C::kLag>();
                         fence_proxy_async_smem();
-                        mbar_arrive(full_bar((int)((it - C::kLag) % C::kStages)));
+                        mbar_arrive(full_bar((int)((it - C::kLag) % nst)));
                     }
                     ++it;
                     c += kBK;
@@ -352,7 +371,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             fence_proxy_async_smem();
             if (ok)
                 for (long long j = it > C::kLag ? it - C::kLag : 0; j < it; ++j)
-                    mbar_arrive(full_bar((int)(j % C::kStages)));
+                    mbar_arrive(full_bar((int)(j % nst)));
         }
     } else if (warp == kMmaWarp) {
         // ------------------------------------------------------------ MMA issuer
@@ -370,14 +389,16 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc_fence_after();
                 const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
                 for (int kb = 0; kb < num_kb; ++kb) {
-                    const int s = (int)(it % C::kStages);
-                    const uint32_t ph = (uint32_t)((it / C::kStages) & 1);
+                    const int s = (int)(it % nst);
+                    const uint32_t ph = (uint32_t)((it / nst) & 1);
                     if (!mbar_wait(full_bar(s), ph, abort_flag, a.status)) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
-                    if (!kTma) fence_proxy_async_smem();
+                    // The A operand was written by cp.async (generic proxy):
+                    // order it before the tensor core's async-proxy reads.
+                    fence_proxy_async_smem();
                     const uint32_t a_st = sA + s * kAStageBytes;
                     const uint32_t b_st = sB + s * C::kBStageBytes;
 #pragma unroll
@@ -639,7 +660,7 @@ hc_status launch_bn(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s) {
     if (!attr_set[ctx->device]) {
         hc_status st = check_cuda(cudaFuncSetAttribute(conv_tc_kernel<BN, kTma>,
                                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                       (int)C::smem_bytes(HC_MAX_SPIRAL)),
+                                                       (int)kSmemLimit),
                                   "cudaFuncSetAttribute(conv_tc_kernel)");
         if (st != HC_OK) return st;
         attr_set[ctx->device] = true;
@@ -648,19 +669,30 @@ hc_status launch_bn(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s) {
     memset(&tx, 0, sizeof tx);
     memset(&tw, 0, sizeof tw);
     if (kTma) {
-        // x: [x_rows, C_in], boxes of one row x 64 channels (gather4);
         // W: [K rows, C_out], boxes of 64 K-rows x 64 output channels.
-        hc_status st = encode_2d(&tx, a.x, a.x_rows, a.C_in, kBK, 1);
-        if (st != HC_OK) return st;
-        st = encode_2d(&tw, a.W, a.K, a.C_out, 64, kBK);
+        hc_status st = encode_2d(&tw, a.W, a.K, a.C_out, 64, kBK);
         if (st != HC_OK) return st;
     }
     const long long n_tiles = (a.C_out + BN - 1) / BN;
     const long long cap_work = (a.capacity + kBM - 1) / kBM * n_tiles;
     long long grid = cap_work < ctx->num_sms ? cap_work : ctx->num_sms;
     if (grid < 1) grid = 1;
+    ConvArgs ka = a;
+    ka.stages = C::stages_for(a.L);
+    // HC_TC_STAGES overrides the depth (clamped to what fits), for tuning.
+    static int env_stages = -1;
+    if (env_stages < 0) {
+        const char* e = getenv("HC_TC_STAGES");
+        env_stages = e ? atoi(e) : 0;
+    }
+    if (env_stages > 0) {
+        int st = env_stages < C::kMaxStages ? env_stages : C::kMaxStages;
+        if (st < C::kMinStages) st = C::kMinStages;
+        while (st > C::kMinStages && C::smem_bytes(a.L, st) > kSmemLimit) --st;
+        ka.stages = st;
+    }
     return launch_pdl(conv_tc_kernel<BN, kTma>, dim3((unsigned)grid), dim3(kThreads),
-                      C::smem_bytes(a.L), s, "conv_tc_kernel", a, tx, tw);
+                      C::smem_bytes(a.L, ka.stages), s, "conv_tc_kernel", ka, tx, tw);
 }
 
 }  // namespace
@@ -673,15 +705,14 @@ bool conv_tc_supported(const ConvArgs& a, hc_dtype dt) {
 }
 
 hc_status launch_conv_tc(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s) {
-    // TMA gathers whole 64-channel blocks of one input row, so it needs C_in
-    // to be a multiple of 64; other channel counts gather with cp.async.
-    // HC_NO_TMA=1 selects the cp.async producer for every shape.
+    // The weight slice comes by TMA; HC_NO_TMA=1 selects the all-cp.async
+    // producer instead (for comparison).
     static int tma_off = -1;
     if (tma_off < 0) {
         const char* e = getenv("HC_NO_TMA");
         tma_off = (e && e[0] == '1') ? 1 : 0;
     }
-    const bool tma = !tma_off && a.C_in % kBK == 0;
+    const bool tma = !tma_off;
     if (a.C_out <= 64) return tma ? launch_bn<64, true>(ctx, a, s) : launch_bn<64, false>(ctx, a, s);
     return tma ? launch_bn<128, true>(ctx, a, s) : launch_bn<128, false>(ctx, a, s);
 }

@@ -68,6 +68,7 @@ struct ConvArgs {
     int B, V, L, C_in, C_out, K;  // K = L*C_in
     int mode;
     int act;
+    int stages;  // pipeline depth chosen by the launcher (tensor-core kernel)
 };
 
 // Launchers (each in its own translation unit). All return HC_OK or an
@@ -242,6 +243,12 @@ __device__ __forceinline__ void cp_async_16(uint32_t dst, const void* src, bool 
     uint32_t n = valid ? 16u : 0u;
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(dst), "l"(src), "r"(n)
                  : "memory");
+}
+// Arrive on `bar` once every cp.async issued so far by this thread has
+// completed (the arrival is not counted in advance: the barrier's expected
+// count includes it).
+__device__ __forceinline__ void cp_async_arrive_noinc(uint32_t bar) {
+    asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];\n" ::"r"(bar) : "memory");
 }
 __device__ __forceinline__ void cp_async_commit() {
     asm volatile("cp.async.commit_group;\n" ::: "memory");
