@@ -153,6 +153,33 @@ class ClockSampler:
                 "power_w_max": max(power) if power else None, "reasons": sorted(reasons)}
 
 
+# ----------------------------------------------------------------- ranks
+
+def reduce_over_ranks(rows, ms, world, device):
+    """Whole-job figures of one timed region: the rows every rank processed,
+    summed, and the slowest rank's time (replicas run independent batches;
+    this is the only cross-rank exchange, two scalars, off the data path)."""
+    if world <= 1:
+        return rows, ms
+    import torch
+    t = torch.tensor([rows, ms], dtype=torch.float64, device=device)
+    r_sum = t.clone()
+    torch.distributed.all_reduce(r_sum, op=torch.distributed.ReduceOp.SUM)
+    r_max = t.clone()
+    torch.distributed.all_reduce(r_max, op=torch.distributed.ReduceOp.MAX)
+    return float(r_sum[0].item()), float(r_max[1].item())
+
+
+def any_rank(flag, world, device):
+    """True if the flag is set on any rank (all ranks get the same answer)."""
+    if world <= 1:
+        return bool(flag)
+    import torch
+    t = torch.tensor([1 if flag else 0], dtype=torch.int32, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return bool(int(t.item()))
+
+
 # ----------------------------------------------------------------- our arm
 
 class LayerSet:
@@ -294,13 +321,9 @@ def run_ours(args, rank, world, local_rank):
     t_start = time.perf_counter()
     while len(reps_ms) < 3 or time.perf_counter() - t_start < 1.0:
         reps_ms.append(timed_region())
-        if world > 1:
-            # every rank must agree on whether to run another repeat
-            flag = torch.tensor([1 if time.perf_counter() - t_start < 1.0 else 0],
-                                device=dev)
-            torch.distributed.all_reduce(flag, op=torch.distributed.ReduceOp.MAX)
-            if len(reps_ms) >= 3 and int(flag.item()) == 0:
-                break
+        if world > 1 and len(reps_ms) >= 3 and not any_rank(
+                time.perf_counter() - t_start < 1.0, world, dev):
+            break  # every rank agrees on the number of repeats
     clocks = sampler.stop()
     ms = statistics.median(reps_ms)
 
@@ -351,14 +374,7 @@ def run_ours(args, rank, world, local_rank):
         sweep = run_sweep(torch, hc, dev, stream)
 
     # Aggregate over ranks: rows summed, time = max over ranks.
-    tot_rows, max_ms = float(rows_timed), ms
-    if world > 1:
-        t = torch.tensor([tot_rows, ms], dtype=torch.float64, device=dev)
-        r_sum = t.clone()
-        torch.distributed.all_reduce(r_sum, op=torch.distributed.ReduceOp.SUM)
-        r_max = t.clone()
-        torch.distributed.all_reduce(r_max, op=torch.distributed.ReduceOp.MAX)
-        tot_rows, max_ms = float(r_sum[0].item()), float(r_max[1].item())
+    tot_rows, max_ms = reduce_over_ranks(float(rows_timed), ms, world, dev)
     if rank != 0:
         return None
 
