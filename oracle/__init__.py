@@ -15,6 +15,8 @@ Functions and the passages they follow:
                            (Eqs. 4-5), bias (Eq. 6) and activation (Eq. 10)
 * ``dense_spiral_conv``    the dense layer the sparse one replaces (Sec. 3.2)
 * ``sparse_linear``        linear layer on compact rows (Eq. 6)
+* ``sparse_group_norm``    group normalisation over each frame's active rows
+                           (Eqs. 7-9)
 * ``scatter_dense``        compact rows back to a dense tensor (inverse of Eq. 2)
 * ``encoder``              a stack of sparse layers: coordinates fixed once by
                            the mask (Eqs. 5, 6, 10 keep C'), each layer's output
@@ -79,6 +81,9 @@ def _load():
             lib.hco_sparse_linear.restype = None
             lib.hco_scatter_dense.argtypes = [P, I, P, I64, I64, I64, I, I, P]
             lib.hco_scatter_dense.restype = None
+            lib.hco_sparse_group_norm.argtypes = [P, I, P, I64, I, I, ctypes.c_double, P, P, I,
+                                                  P, P]
+            lib.hco_sparse_group_norm.restype = None
             lib.hco_conv_rulebook.argtypes = [P, P, I64, P, I64, I, I, I64, P]
             lib.hco_conv_rulebook.restype = None
             lib.hco_bf16_round.argtypes = [ctypes.c_double]
@@ -207,6 +212,25 @@ def sparse_linear(x, W, bias, act, rows=None, n_threads=1):
     y = np.empty((n, C_out), dtype=x.dtype)
     _load().hco_sparse_linear(_ptr(x), dt, _ptr(rows), n, C_in, C_out, _ptr(W), _ptr(bias), act,
                               _ptr(y_pre), _ptr(y), int(n_threads))
+    return y_pre, y
+
+
+def sparse_group_norm(x, offsets, G, eps=1e-5, gamma=None, beta=None, act=ACT_NONE):
+    """Eqs. 7-9 on compact rows x [N', C] with frame offsets [B+1]: returns
+    (y_pre fp64, y in the input dtype), both [N', C]; rows outside every
+    frame's range are left as NaN / zero."""
+    dt = _dtype_code(x)
+    x = np.ascontiguousarray(x)
+    offsets = _c(offsets, np.int32)
+    B = offsets.shape[0] - 1
+    C = x.shape[1]
+    assert C % G == 0
+    gamma = None if gamma is None else _c(gamma, np.float32)
+    beta = None if beta is None else _c(beta, np.float32)
+    y_pre = np.full(x.shape, np.nan, dtype=np.float64)
+    y = np.zeros_like(x)
+    _load().hco_sparse_group_norm(_ptr(x), dt, _ptr(offsets), B, C, G, float(eps), _ptr(gamma),
+                                  _ptr(beta), act, _ptr(y_pre), _ptr(y))
     return y_pre, y
 
 

@@ -23,6 +23,8 @@
  *   hco_dense_spiral_conv   the same layer on every vertex, no mask (the dense
  *                           operator the sparse one replaces, Sec. 3.2)
  *   hco_sparse_linear       linear layer on compact rows, Eq. 6
+ *   hco_sparse_group_norm   group normalisation over each frame's active rows,
+ *                           Eqs. 7-9 (G = 1: layer normalisation)
  *   hco_scatter_dense       inverse of the decomposition: compact rows back
  *                           into a dense [B, V, C] tensor
  *   hco_bf16_round          fp64 -> bf16 rounding (storage format)
@@ -261,6 +263,51 @@ void hco_sparse_linear(const void* x, int dtype, const int64_t* rows, int64_t n_
             double a = activate(acc + (bias ? (double)bias[o] : 0.0), act);
             if (y_pre) y_pre[i * C_out + o] = a;
             if (y) store_elem(y, dtype, i * C_out + o, a);
+        }
+    }
+}
+
+/* ---------------------------------------------------------- group norm */
+
+/* Eqs. 7-9: group normalisation over the active rows of each frame. Frame b
+ * owns the compact rows [offsets[b], offsets[b+1]) (the rows i with
+ * C'[i][0] = b); the C channels split into G groups of C/G consecutive
+ * channels. For every (b, g), with n = (rows of frame b) * (C/G) values:
+ *     mu     = (1/n) * sum of the group's values over the frame's rows   (Eq. 7)
+ *     sigma2 = (1/n) * sum of (value - mu)^2                             (Eq. 8)
+ *     out    = (value - mu) / sqrt(sigma2 + eps)                         (Eq. 9)
+ * then, per channel, out * gamma[c] + beta[c] when gamma/beta are given, and
+ * the activation of Eq. 10. Two passes in fp64. Frames without active rows
+ * produce nothing. */
+void hco_sparse_group_norm(const void* x, int dtype, const int32_t* offsets, int64_t B, int C,
+                           int G, double eps, const float* gamma, const float* beta, int act,
+                           double* y_pre, void* y) {
+    int cpg = C / G;
+    for (int64_t b = 0; b < B; ++b) {
+        int64_t r0 = offsets[b], r1 = offsets[b + 1];
+        if (r1 <= r0) continue;
+        for (int g = 0; g < G; ++g) {
+            double n = (double)(r1 - r0) * cpg;
+            double sum = 0.0;
+            for (int64_t i = r0; i < r1; ++i)
+                for (int c = g * cpg; c < (g + 1) * cpg; ++c) sum += load_elem(x, dtype, i * C + c);
+            double mu = sum / n;
+            double ss = 0.0;
+            for (int64_t i = r0; i < r1; ++i)
+                for (int c = g * cpg; c < (g + 1) * cpg; ++c) {
+                    double d = load_elem(x, dtype, i * C + c) - mu;
+                    ss += d * d;
+                }
+            double inv = 1.0 / sqrt(ss / n + eps);
+            for (int64_t i = r0; i < r1; ++i)
+                for (int c = g * cpg; c < (g + 1) * cpg; ++c) {
+                    double v = (load_elem(x, dtype, i * C + c) - mu) * inv;
+                    if (gamma) v *= (double)gamma[c];
+                    if (beta) v += (double)beta[c];
+                    v = activate(v, act);
+                    if (y_pre) y_pre[i * C + c] = v;
+                    if (y) store_elem(y, dtype, i * C + c, v);
+                }
         }
     }
 }

@@ -356,6 +356,10 @@ MUTANTS = {
                                      "double n = nearbyint(ldexp((double)(float)x, -qexp));"),
     "rulebook ignores activity": ("                if (j >= 0) e = (int32_t)(x_layout == HCO_LAYOUT_DENSE ? b * V + u : j);",
                                   "                e = (int32_t)(x_layout == HCO_LAYOUT_DENSE ? b * V + u : j);"),
+    "group norm variance around zero": ("                    double d = load_elem(x, dtype, i * C + c) - mu;",
+                                        "                    double d = load_elem(x, dtype, i * C + c);"),
+    "group norm counts rows only": ("            double n = (double)(r1 - r0) * cpg;",
+                                    "            double n = (double)(r1 - r0);"),
     "centre tap dropped": ("for (int l = 0; l < L; ++l) {\n            int64_t u = spiral[v * L + l];\n            if (u < 0) continue; /* no neighbour in this slot */",
                            "for (int l = 1; l < L; ++l) {\n            int64_t u = spiral[v * L + l];\n            if (u < 0) continue; /* no neighbour in this slot */"),
 }
@@ -378,11 +382,13 @@ def test_planted_mistake_is_caught(name, tmp_path, monkeypatch):
     good = oracle._load()
     lib = ctypes.CDLL(str(so))
     for fn in ("hco_mask_compact", "hco_sparse_spiral_conv", "hco_dense_spiral_conv",
-               "hco_sparse_linear", "hco_scatter_dense", "hco_bf16_round", "hco_conv_rulebook"):
+               "hco_sparse_linear", "hco_scatter_dense", "hco_bf16_round", "hco_conv_rulebook",
+               "hco_sparse_group_norm"):
         getattr(lib, fn).argtypes = getattr(good, fn).argtypes
         getattr(lib, fn).restype = getattr(good, fn).restype
     monkeypatch.setattr(oracle, "_lib", lib)
-    checks = [check_golden_cases, check_conv_vs_gather_matmul,
+    checks = [check_golden_cases, check_conv_vs_gather_matmul, check_group_norm_golden,
+              check_group_norm_vs_numpy,
               lambda: check_compact_vs_nonzero(inputs.uniform_mask(np.random.default_rng(1), 5, 20, 0.3)),
               check_bf16_round]
     caught = 0
@@ -392,3 +398,71 @@ def test_planted_mistake_is_caught(name, tmp_path, monkeypatch):
         except AssertionError:
             caught += 1
     assert caught >= 1, f"planted mistake '{name}' passed every pin"
+
+
+# ------------------------------------------------------------ group norm
+
+def check_group_norm_golden():
+    g = json.load(open(os.path.join(os.path.dirname(__file__), "golden", "group_norm.json")))
+    c0, c1, c2 = g["cases"]
+    y, _ = oracle.sparse_group_norm(np.array(c0["x"], np.float32), np.array(c0["offsets"]),
+                                    c0["G"], eps=0.0)
+    np.testing.assert_allclose(y, np.array(c0["y_over_sqrt_1_25"]) / math.sqrt(1.25), rtol=1e-14)
+    y, _ = oracle.sparse_group_norm(np.array(c1["x"], np.float32), np.array(c1["offsets"]),
+                                    c1["G"], eps=1.0)
+    np.testing.assert_allclose(y[:2], np.array(c1["y_frame0"]) / np.sqrt(1 + 1 / np.array([1, 100])),
+                               rtol=1e-14)
+    np.testing.assert_array_equal(y[2], [0.0, 0.0])
+    y, _ = oracle.sparse_group_norm(np.array(c2["x"], np.float32), np.array(c2["offsets"]),
+                                    c2["G"], eps=0.0)
+    np.testing.assert_allclose(y, np.array(c2["y"], np.float64), rtol=1e-14)
+
+
+def test_group_norm_golden():
+    check_group_norm_golden()
+
+
+def check_group_norm_vs_numpy(seed=31):
+    """Per frame and group, numpy's mean and (biased) variance of the gathered
+    group values give the same normalisation; gamma, beta and ELU follow."""
+    rng = np.random.default_rng(seed)
+    m = inputs.uniform_mask(rng, 5, 60, 0.3)
+    m[2] = 0  # an empty frame
+    coords, row_of, offsets, n = oracle.mask_compact(m)
+    C, G = 12, 3
+    x = (rng.standard_normal((n, C)) * 2 + 0.7).astype(np.float32)
+    gamma = rng.standard_normal(C).astype(np.float32)
+    beta = rng.standard_normal(C).astype(np.float32)
+    y, _ = oracle.sparse_group_norm(x, offsets, G, 1e-5, gamma, beta, oracle.ACT_ELU)
+    ref = np.empty((n, C))
+    xd = x.astype(np.float64)
+    for b in range(5):
+        r0, r1 = offsets[b], offsets[b + 1]
+        for g in range(G):
+            blk = xd[r0:r1, g * 4:(g + 1) * 4]
+            if blk.size == 0:
+                continue
+            z = (blk - blk.mean()) / np.sqrt(blk.var() + 1e-5)
+            z = z * gamma[g * 4:(g + 1) * 4] + beta[g * 4:(g + 1) * 4]
+            ref[r0:r1, g * 4:(g + 1) * 4] = np.where(z > 0, z, np.expm1(np.minimum(z, 0)))
+    np.testing.assert_allclose(y, ref, rtol=1e-12, atol=1e-12)
+
+
+def test_group_norm_vs_numpy():
+    check_group_norm_vs_numpy()
+
+
+def test_group_norm_is_layer_norm_at_g1_and_ignores_inactive_rows():
+    """G = 1 is layer normalisation over all channels of a frame's active rows;
+    inactive vertices (zeros in the dense masked tensor) do not enter the
+    statistics, unlike a dense group norm over all V rows."""
+    rng = np.random.default_rng(32)
+    m = inputs.uniform_mask(rng, 1, 50, 0.4)
+    coords, row_of, offsets, n = oracle.mask_compact(m)
+    x = (rng.standard_normal((n, 8)) + 3).astype(np.float32)
+    y, _ = oracle.sparse_group_norm(x, offsets, 1, 0.0)
+    assert abs(y.mean()) < 1e-12 and abs(y.var() - 1.0) < 1e-12
+    dense = np.zeros((50, 8))
+    dense[coords[:, 1]] = x
+    yd = (dense - dense.mean()) / dense.std()
+    assert not np.allclose(yd[coords[:, 1]], y)
