@@ -369,9 +369,10 @@ def run_ours(args, rank, world, local_rank):
 
     e2e = measure_e2e(torch, hc, sets, w, spiral, Wt, bias, stream, dev, args.e2e_steps)
 
-    sweep = None
+    sweep = gnorm = None
     if not args.no_extras and rank == 0:
         sweep = run_sweep(torch, hc, dev, stream)
+        gnorm = run_group_norm(torch, hc, sets, dev, stream)
 
     # Aggregate over ranks: rows summed, time = max over ranks.
     tot_rows, max_ms = reduce_over_ranks(float(rows_timed), ms, world, dev)
@@ -438,6 +439,8 @@ def run_ours(args, rank, world, local_rank):
     }
     if sweep is not None:
         line["sweep"] = sweep
+    if gnorm is not None:
+        line["group_norm"] = gnorm
     return line
 
 
@@ -574,6 +577,75 @@ def run_sweep(torch, hc, dev, stream):
     st = hc.hc_get_device_status(stream)
     if st != hc.HC_OK:
         raise RuntimeError(f"device status {hc.STATUS_NAMES.get(st)} in the sweep")
+    return out
+
+
+def run_group_norm(torch, hc, sets, dev, stream, G=8):
+    """Sparse group norm (Eqs. 7-9), G = 8, affine + ELU, on two inputs:
+    the bench layer's compact conv outputs (rotating over the input sets;
+    they sit in L2 as they would right after the conv) and a fully active
+    64 x 10475 x 128 bf16 activation (171 MB, larger than L2). Algorithmic
+    bytes: every active element read once and written once."""
+    pk = peaks()
+    C = sets[0].y.shape[1]
+    gamma = torch.linspace(0.5, 1.5, C, device=dev)
+    beta = torch.linspace(-0.1, 0.1, C, device=dev)
+    with torch.cuda.stream(stream):  # the e2e leg reuses set 0's compaction buffers
+        for s in sets:
+            hc.hc_mask_compact(s.mask, s.coords, s.row_of, s.offs, s.count, stream)
+    torch.cuda.synchronize(dev)
+    for s in sets:
+        assert int(s.count.item()) == s.rows
+        s.gn = torch.empty_like(s.y)
+
+    def timeit(fns, reps):
+        with torch.cuda.stream(stream):
+            for f in fns:
+                f()
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                for _ in range(reps):
+                    for f in fns:
+                        f()
+            g.replay()
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            g.replay()
+            b.record(stream)
+        torch.cuda.synchronize(dev)
+        return a.elapsed_time(b) / (reps * len(fns))
+
+    def gn(x, offs, y):
+        return lambda: hc.hc_sparse_group_norm_fwd(x, offs, G, 1e-5, gamma, beta, hc.HC_ACT_ELU,
+                                                   y, stream)
+
+    out = {"G": G, "act": "elu", "affine": True,
+           "kernels": "gn_stats_kernel + gn_apply_kernel (contiguous row ranges)"}
+    ms = timeit([gn(s.y[:s.rows], s.offs, s.gn[:s.rows]) for s in sets], 10)
+    rows = sum(s.rows for s in sets) / len(sets)
+    nbytes = 2 * rows * C * 2
+    out["layer_output"] = {"rows": rows, "C": C, "us": ms * 1e3,
+                           "gbs": nbytes / (ms * 1e-3) / 1e9,
+                           "hbm_frac": nbytes / (ms * 1e-3) / 1e9 / pk["hbm_gbs"],
+                           "note": "compact conv outputs of the bench layer, L2-resident"}
+    for s in sets:
+        del s.gn
+    Bl, Vl = 64, 10475
+    x = torch.randn((Bl * Vl, C), device=dev).to(torch.bfloat16)
+    y = torch.empty_like(x)
+    offs = (torch.arange(Bl + 1, device=dev, dtype=torch.int32) * Vl).contiguous()
+    ms = timeit([gn(x, offs, y)], 10)
+    nbytes = 2 * x.numel() * 2
+    gbs = nbytes / (ms * 1e-3) / 1e9
+    out["large"] = {"rows": Bl * Vl, "C": C, "bytes": nbytes, "us": ms * 1e3, "gbs": gbs,
+                    "hbm_frac": gbs / pk["hbm_gbs"],
+                    "peak": f"{pk['hbm_gbs']} GB/s ({pk['source']} copy)"}
+    st = hc.hc_get_device_status(stream)
+    if st != hc.HC_OK:
+        raise RuntimeError(f"device status {hc.STATUS_NAMES.get(st)} in group norm")
+    del x, y
+    torch.cuda.empty_cache()
     return out
 
 

@@ -204,6 +204,29 @@ hc_status hc_sparse_linear_fwd(const void* x, hc_dtype dt, const int32_t* count,
                                void* y, hc_stream_t stream);
 
 /*
+ * hc_sparse_group_norm_fwd -- group normalisation of compact rows (Eqs. 7-9),
+ * statistics taken over each frame's active rows only. Frame b owns the rows
+ * [batch_offsets[b], batch_offsets[b+1]) (as written by hc_mask_compact); the
+ * C channels form G groups of C/G consecutive channels. For every (b, g), over
+ * the n = rows(b) * C/G values of the group:
+ *   mu = sum / n,  var = sum((v - mu)^2) / n,  out = (v - mu) / sqrt(var + eps)
+ * then out * gamma[c] + beta[c] (each optional: NULL = 1 / 0) and the
+ * activation act (Eq. 10). G = 1 is layer normalisation.
+ *   x, y      [capacity, C] of dtype dt; y may be x (in place). Rows outside
+ *             every frame's range are not touched.
+ *   batch_offsets [B+1] int32 on the device, non-decreasing, within
+ *             [0, capacity]; otherwise HC_ERR_INVALID_INDEX is reported
+ *             (hc_get_device_status) and the output is unspecified, but no
+ *             access leaves x, y or the library's workspace.
+ * Statistics in fp32 by pairwise (count, mean, M2) merging; the variance is
+ * taken around the mean, never as E[x^2] - mean^2. Uses the library's
+ * per-stream workspace ((B + 3 * SMs) * G * 16 bytes at most).
+ */
+hc_status hc_sparse_group_norm_fwd(const void* x, hc_dtype dt, const int32_t* batch_offsets, int B,
+                                   int capacity, int C, int G, float eps, const float* gamma,
+                                   const float* beta, hc_act act, void* y, hc_stream_t stream);
+
+/*
  * hc_scatter_dense -- inverse of the decomposition (Eq. 2): compact rows back
  * into a dense [B, V, C] tensor.
  *   zero_fill == 0: out[coords[n]] = y[n] for n < N'; other rows untouched.

@@ -1,0 +1,591 @@
+// Sparse group normalisation (Eqs. 7-9): for every frame b and channel group
+// g, mean and variance over the frame's active rows [offsets[b], offsets[b+1])
+// and the group's C/G channels only, then (x - mean) / sqrt(var + eps),
+// optional per-channel affine, and the activation of Eq. 10 fused.
+//
+// Statistics. Values are read in chunks; per chunk its mean (shifted by the
+// chunk's first value) and centred sum of squares, merged into a running
+// (count, mean, M2) by the pairwise update of Chan, Golub and LeVeque, and
+// partial results merged the same way. The variance is never formed as
+// E[x^2] - mean^2, and a group of equal values gets exactly that mean and
+// M2 = 0, so it normalises to exactly 0. All in fp32: GB300's fp64 rate is
+// far too low for a bandwidth-bound kernel.
+//
+// Fast path (rows in 16-byte chunks, C/VEC a power of two <= 256, and either
+// VEC | C/G or C/G | VEC): the compact rows [offsets[0], offsets[B]) are cut
+// into gridDim.x equal contiguous ranges, one per CTA, independent of frame
+// boundaries. That balances the load whatever the frame sizes, and whole
+// rows are read with coalesced 16-byte loads; each thread owns one chunk
+// column, hence a fixed set of groups and fixed gamma/beta values.
+//   gn_stats_kernel: per frame segment of its range, a block merge per group
+//     and one partial (n, mean, M2) per (frame b, CTA c), written to slot
+//     b + c of the workspace. Frames are contiguous and in order, so the
+//     slots of frame b, b + [first CTA, last CTA], end before those of frame
+//     b + 1 begin: slots never collide and (B + gridDim.x) * G suffice.
+//   gn_apply_kernel: same ranges; per frame segment, merge the partials of
+//     the CTAs that hold the frame, normalise and store. Segments and rows
+//     are walked in reverse, so the most recently read rows, still in L2,
+//     are consumed first.
+// The general path (one CTA per (frame, group)) serves every other layout.
+// The output may alias the input in both paths. Deterministic, no atomics.
+#include <cuda_bf16.h>
+
+#include <cstdlib>
+
+#include "hc_internal.cuh"
+
+namespace hc {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kBatch = 4;
+constexpr int kMaxGroupsFast = 2048;
+
+// VEC consecutive elements as one raw chunk (16 bytes when VEC > 1).
+template <typename T, int VEC>
+struct Chunk;
+template <>
+struct Chunk<float, 1> {
+    using Raw = float;
+    static __device__ __forceinline__ Raw load(const float* p) { return *p; }
+    static __device__ __forceinline__ void unpack(Raw r, float* v) { v[0] = r; }
+    static __device__ __forceinline__ void store(float* p, const float* v) { *p = v[0]; }
+};
+template <>
+struct Chunk<float, 4> {
+    using Raw = float4;
+    static __device__ __forceinline__ Raw load(const float* p) {
+        return *reinterpret_cast<const float4*>(p);
+    }
+    static __device__ __forceinline__ void unpack(Raw r, float* v) {
+        v[0] = r.x, v[1] = r.y, v[2] = r.z, v[3] = r.w;
+    }
+    static __device__ __forceinline__ void store(float* p, const float* v) {
+        *reinterpret_cast<float4*>(p) = make_float4(v[0], v[1], v[2], v[3]);
+    }
+};
+template <>
+struct Chunk<__nv_bfloat16, 1> {
+    using Raw = __nv_bfloat16;
+    static __device__ __forceinline__ Raw load(const __nv_bfloat16* p) { return *p; }
+    static __device__ __forceinline__ void unpack(Raw r, float* v) { v[0] = __bfloat162float(r); }
+    static __device__ __forceinline__ void store(__nv_bfloat16* p, const float* v) {
+        *p = __float2bfloat16_rn(v[0]);
+    }
+};
+template <>
+struct Chunk<__nv_bfloat16, 8> {
+    using Raw = uint4;
+    static __device__ __forceinline__ Raw load(const __nv_bfloat16* p) {
+        return *reinterpret_cast<const uint4*>(p);
+    }
+    static __device__ __forceinline__ void unpack(Raw r, float* v) {
+        const uint32_t w[4] = {r.x, r.y, r.z, r.w};
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            v[2 * k] = __uint_as_float(w[k] << 16);
+            v[2 * k + 1] = __uint_as_float(w[k] & 0xffff0000u);
+        }
+    }
+    static __device__ __forceinline__ void store(__nv_bfloat16* p, const float* v) {
+        uint32_t w[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const __nv_bfloat162 h = __floats2bfloat162_rn(v[2 * k], v[2 * k + 1]);
+            w[k] = *reinterpret_cast<const uint32_t*>(&h);
+        }
+        *reinterpret_cast<uint4*>(p) = make_uint4(w[0], w[1], w[2], w[3]);
+    }
+};
+
+// Running (count, mean, M2), fp32. Counts are exact integers below 2^24.
+struct Stats {
+    float n = 0.f, mean = 0.f, m2 = 0.f;
+    template <int VEC>
+    __device__ __forceinline__ void add_chunk(const float* v) {
+        float s = 0.f;
+#pragma unroll
+        for (int k = 1; k < VEC; ++k) s += v[k] - v[0];
+        const float cm = v[0] + s * (1.f / VEC);
+        float q = 0.f;
+#pragma unroll
+        for (int k = 0; k < VEC; ++k) {
+            const float d = v[k] - cm;
+            q = fmaf(d, d, q);
+        }
+        const float nn = n + (float)VEC;
+        const float d = cm - mean;
+        const float r = (float)VEC / nn;
+        mean = fmaf(d, r, mean);
+        m2 += q + d * d * n * r;
+        n = nn;
+    }
+};
+
+// Pairwise merge of (nb, mb, qb) into (n, mean, m2).
+__device__ __forceinline__ void merge(float& n, float& mean, float& m2, float nb, float mb,
+                                      float qb) {
+    if (nb == 0.f) return;
+    const float nn = n + nb;
+    const float d = mb - mean;
+    const float r = nb / nn;
+    mean = fmaf(d, r, mean);
+    m2 += qb + d * d * n * r;
+    n = nn;
+}
+
+__device__ __forceinline__ void merge_xor(float& n, float& mean, float& m2, int o) {
+    const float nb = __shfl_xor_sync(0xffffffffu, n, o);
+    const float mb = __shfl_xor_sync(0xffffffffu, mean, o);
+    const float qb = __shfl_xor_sync(0xffffffffu, m2, o);
+    merge(n, mean, m2, nb, mb, qb);
+}
+
+// Merge over the whole block; every thread gets the result.
+__device__ __forceinline__ void block_merge(float& n, float& mean, float& m2, float* red) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) merge_xor(n, mean, m2, o);
+    if ((threadIdx.x & 31) == 0) {
+        red[3 * (threadIdx.x >> 5)] = n;
+        red[3 * (threadIdx.x >> 5) + 1] = mean;
+        red[3 * (threadIdx.x >> 5) + 2] = m2;
+    }
+    __syncthreads();
+    n = mean = m2 = 0.f;
+#pragma unroll
+    for (int w = 0; w < kThreads / 32; ++w)
+        merge(n, mean, m2, red[3 * w], red[3 * w + 1], red[3 * w + 2]);
+}
+
+// ---- fast path: contiguous row ranges ------------------------------------
+struct GnPart {
+    float n, mean, m2, pad;
+};
+
+// Row range of CTA c over [off0, end): R = ceil((end - off0) / grid).
+struct RangeMap {
+    long long off0, end, R;
+    __device__ __forceinline__ long long cta_of(long long row) const { return (row - off0) / R; }
+};
+
+// First frame b with offsets[b + 1] > row (the frame holding `row`).
+__device__ __forceinline__ int frame_of(const int32_t* offsets, int B, long long row) {
+    int lo = 0, hi = B;  // answer in [lo, hi]
+    while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if ((long long)__ldg(offsets + mid + 1) > row)
+            hi = mid;
+        else
+            lo = mid + 1;
+    }
+    return lo;
+}
+
+// Thread layout: cpr chunks per row; thread t owns chunk column t % cpr and
+// rows rg, rg + rpp, ... of a segment (rg = t / cpr, rpp = kThreads / cpr).
+// GPC groups per chunk when a group is narrower than a chunk, else 1 (the
+// chunk lies in group col / cpc, cpc = chunks per group).
+struct Layout {
+    int cpr, rpp, col, rg, cpc;
+};
+
+template <int VEC, int GPC>
+__device__ __forceinline__ Layout make_layout(int C, int G) {
+    Layout l;
+    l.cpr = C / VEC;
+    l.rpp = kThreads / l.cpr;
+    l.col = threadIdx.x % l.cpr;
+    l.rg = threadIdx.x / l.cpr;
+    l.cpc = GPC == 1 ? (C / G) / VEC : 1;
+    return l;
+}
+
+// This CTA's row range [lo, hi); false if there is nothing to do or the
+// frame table's span is unusable (reported).
+__device__ __forceinline__ bool range_setup(const int32_t* offsets, int B, long long capacity,
+                                            unsigned* status, RangeMap& m, long long& lo,
+                                            long long& hi) {
+    const long long o0 = __ldg(offsets), oB = __ldg(offsets + B);
+    if (o0 < 0 || oB < o0 || oB > capacity) {
+        if (threadIdx.x == 0 && blockIdx.x == 0) report(status, kErrIndex);
+        return false;
+    }
+    const long long total = oB - o0;
+    if (total == 0) return false;
+    m.off0 = o0;
+    m.end = oB;
+    m.R = (total + gridDim.x - 1) / gridDim.x;
+    lo = o0 + (long long)blockIdx.x * m.R;
+    hi = lo + m.R < oB ? lo + m.R : oB;
+    return lo < hi;
+}
+
+template <typename T, int VEC, int GPC>
+__global__ void __launch_bounds__(kThreads, 3)
+    gn_stats_kernel(const T* x, const int32_t* __restrict__ offsets, int B, int C, int G,
+                    long long capacity, GnPart* __restrict__ part, unsigned* status) {
+    using CK = Chunk<T, VEC>;
+    using Raw = typename CK::Raw;
+    constexpr int SUB = VEC / GPC;  // elements of one group inside a chunk (GPC > 1)
+    __shared__ float red[kThreads * GPC * 3];
+    pdl_wait();
+    pdl_trigger();
+    // frames must be in order (each CTA checks a share of the table)
+    for (long long i = (long long)blockIdx.x * kThreads + threadIdx.x; i < B;
+         i += (long long)gridDim.x * kThreads)
+        if (__ldg(offsets + i + 1) < __ldg(offsets + i)) report(status, kErrIndex);
+    RangeMap m;
+    long long lo, hi;
+    if (!range_setup(offsets, B, capacity, status, m, lo, hi)) return;
+    const Layout l = make_layout<VEC, GPC>(C, G);
+    // after the warp merge: row slots (warps, or thread rows) x cpr columns
+    const int nrs = l.cpr < 32 ? kThreads / 32 : kThreads / l.cpr;
+
+    for (int b = frame_of(offsets, B, lo); b < B; ++b) {
+        const long long f0 = __ldg(offsets + b), f1 = __ldg(offsets + b + 1);
+        if (f0 >= hi) break;
+        if (f1 < f0) continue;  // reported above
+        const long long s0 = f0 > lo ? f0 : lo, s1 = f1 < hi ? f1 : hi;
+        if (s0 >= s1) continue;
+        Stats st[GPC];
+        for (long long r = s0 + l.rg; r < s1; r += (long long)kBatch * l.rpp) {
+            Raw t[kBatch];
+#pragma unroll
+            for (int i = 0; i < kBatch; ++i)
+                if (r + (long long)i * l.rpp < s1)
+                    t[i] = CK::load(x + (r + (long long)i * l.rpp) * C + l.col * VEC);
+#pragma unroll
+            for (int i = 0; i < kBatch; ++i) {
+                if (r + (long long)i * l.rpp < s1) {
+                    float v[VEC];
+                    CK::unpack(t[i], v);
+#pragma unroll
+                    for (int s = 0; s < GPC; ++s) st[s].template add_chunk<SUB>(v + s * SUB);
+                }
+            }
+        }
+        // lanes holding the same column: merge across the warp
+#pragma unroll
+        for (int s = 0; s < GPC; ++s)
+            for (int o = l.cpr; o < 32; o <<= 1) merge_xor(st[s].n, st[s].mean, st[s].m2, o);
+        const int lane = threadIdx.x & 31;
+        if (l.cpr >= 32 || lane < l.cpr) {
+            const int slot = l.cpr < 32 ? (int)(threadIdx.x >> 5) : l.rg;
+#pragma unroll
+            for (int s = 0; s < GPC; ++s) {
+                float* e = red + 3 * ((slot * l.cpr + l.col) * GPC + s);
+                e[0] = st[s].n, e[1] = st[s].mean, e[2] = st[s].m2;
+            }
+        }
+        __syncthreads();
+        GnPart* out = part + (long long)(b + blockIdx.x) * G;
+        for (int g = threadIdx.x; g < G; g += kThreads) {
+            const int c0 = GPC == 1 ? g * l.cpc : g / GPC, nc = GPC == 1 ? l.cpc : 1;
+            const int s = GPC == 1 ? 0 : g % GPC;
+            float n = 0.f, mean = 0.f, m2 = 0.f;
+            for (int rs = 0; rs < nrs; ++rs)
+                for (int c = c0; c < c0 + nc; ++c) {
+                    const float* e = red + 3 * ((rs * l.cpr + c) * GPC + s);
+                    merge(n, mean, m2, e[0], e[1], e[2]);
+                }
+            out[g] = GnPart{n, mean, m2, 0.f};
+        }
+        __syncthreads();  // red[] is reused by the next segment
+    }
+}
+
+template <typename T, int VEC, int GPC>
+__global__ void __launch_bounds__(kThreads, 3)
+    gn_apply_kernel(const T* x, const int32_t* __restrict__ offsets, int B, int C, int G,
+                    long long capacity, const GnPart* __restrict__ part, float eps,
+                    const float* __restrict__ gamma, const float* __restrict__ beta, int act, T* y,
+                    unsigned* status) {
+    using CK = Chunk<T, VEC>;
+    using Raw = typename CK::Raw;
+    constexpr int SUB = VEC / GPC;
+    __shared__ float s_mu[kMaxGroupsFast], s_inv[kMaxGroupsFast];
+    pdl_wait();
+    pdl_trigger();
+    RangeMap m;
+    long long lo, hi;
+    if (!range_setup(offsets, B, capacity, status, m, lo, hi)) return;
+    const Layout l = make_layout<VEC, GPC>(C, G);
+    float ga[VEC], be[VEC];
+#pragma unroll
+    for (int k = 0; k < VEC; ++k) {
+        ga[k] = gamma ? __ldg(gamma + l.col * VEC + k) : 1.f;
+        be[k] = beta ? __ldg(beta + l.col * VEC + k) : 0.f;
+    }
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int b_first = frame_of(offsets, B, lo);
+    int b_last = frame_of(offsets, B, hi - 1);
+    if (b_last > B - 1) b_last = B - 1;
+
+    for (int b = b_last; b >= b_first; --b) {  // frames last to first
+        const long long f0 = __ldg(offsets + b), f1 = __ldg(offsets + b + 1);
+        if (f1 < f0) continue;  // reported by the statistics kernel
+        const long long s0 = f0 > lo ? f0 : lo, s1 = f1 < hi ? f1 : hi;
+        if (s0 >= s1) continue;
+        // partials of the CTAs that hold frame b: slots b + c, c in [c0, c1]
+        // (clamped to the table's span, so a malformed table cannot index
+        // outside the workspace)
+        const long long c0 = m.cta_of(f0 > m.off0 ? f0 : m.off0);
+        const long long c1 = m.cta_of((f1 < m.end ? f1 : m.end) - 1);
+        const GnPart* pb = part + (long long)b * G;
+        if (c1 - c0 < 8) {
+            for (int g = threadIdx.x; g < G; g += kThreads) {
+                float n = 0.f, mean = 0.f, m2 = 0.f;
+                for (long long c = c0; c <= c1; ++c) {
+                    const GnPart q = pb[c * G + g];
+                    merge(n, mean, m2, q.n, q.mean, q.m2);
+                }
+                s_mu[g] = mean;
+                s_inv[g] = 1.f / sqrtf(m2 / n + eps);
+            }
+        } else {
+            for (int g = warp; g < G; g += kThreads / 32) {
+                float n = 0.f, mean = 0.f, m2 = 0.f;
+                for (long long c = c0 + lane; c <= c1; c += 32) {
+                    const GnPart q = pb[c * G + g];
+                    merge(n, mean, m2, q.n, q.mean, q.m2);
+                }
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) merge_xor(n, mean, m2, o);
+                if (lane == 0) {
+                    s_mu[g] = mean;
+                    s_inv[g] = 1.f / sqrtf(m2 / n + eps);
+                }
+            }
+        }
+        __syncthreads();
+        float mu[GPC], inv[GPC];
+#pragma unroll
+        for (int s = 0; s < GPC; ++s) {
+            const int g = GPC == 1 ? l.col / l.cpc : l.col * GPC + s;
+            mu[s] = s_mu[g];
+            inv[s] = s_inv[g];
+        }
+        // rows of the segment, last to first
+        const long long last = (s1 - s0) - 1 - l.rg;  // this thread's highest row offset
+        for (long long r = last; r >= 0; r -= (long long)kBatch * l.rpp) {
+            Raw t[kBatch];
+#pragma unroll
+            for (int i = 0; i < kBatch; ++i)
+                if (r - (long long)i * l.rpp >= 0)
+                    t[i] = CK::load(x + (s0 + r - (long long)i * l.rpp) * C + l.col * VEC);
+#pragma unroll
+            for (int i = 0; i < kBatch; ++i) {
+                if (r - (long long)i * l.rpp >= 0) {
+                    float v[VEC];
+                    CK::unpack(t[i], v);
+#pragma unroll
+                    for (int k = 0; k < VEC; ++k) {
+                        const int s = k / SUB;
+                        const float z = fmaf((v[k] - mu[s]) * inv[s], ga[k], be[k]);
+                        v[k] = act_apply(z, act);
+                    }
+                    CK::store(y + (s0 + r - (long long)i * l.rpp) * C + l.col * VEC, v);
+                }
+            }
+        }
+        __syncthreads();  // s_mu / s_inv are rewritten for the next frame
+    }
+}
+
+// ---- general path: one CTA per (frame, group) ----------------------------
+// Any C, G and alignment. The group's part of a row is read in chunks of VEC
+// elements (16 bytes, or single elements); chunk e of the slice is at row
+// r0 + e / vpr, channel c0 + (e % vpr) * VEC. The first batch of every
+// thread stays in registers; pass 2 walks the other batches in reverse.
+struct SliceMap {
+    long long r0;
+    int C, c0, vpr, VEC;
+    bool narrow;  // 32-bit division suffices
+    __device__ __forceinline__ long long at(long long e, int& c) const {
+        long long q;
+        int rem;
+        if (narrow) {
+            const unsigned qe = (unsigned)e / (unsigned)vpr;
+            q = qe;
+            rem = (int)((unsigned)e - qe * (unsigned)vpr);
+        } else {
+            q = e / vpr;
+            rem = (int)(e - q * vpr);
+        }
+        c = c0 + rem * VEC;
+        return (r0 + q) * C + c;
+    }
+};
+
+template <typename T, int VEC>
+__global__ void __launch_bounds__(kThreads, 4)
+    group_norm_slice_kernel(const T* x, const int32_t* __restrict__ offsets, int C, int G,
+                            long long capacity, float eps, const float* __restrict__ gamma,
+                            const float* __restrict__ beta, int act, T* y, unsigned* status) {
+    using CK = Chunk<T, VEC>;
+    using Raw = typename CK::Raw;
+    constexpr long long kStride = (long long)kThreads * kBatch;
+    __shared__ float red[3 * (kThreads / 32)];
+    pdl_wait();
+    pdl_trigger();
+    const int b = blockIdx.x / G, g = blockIdx.x - b * G;
+    const long long r0 = __ldg(offsets + b), r1 = __ldg(offsets + b + 1);
+    if (r0 < 0 || r1 < r0 || r1 > capacity) {
+        if (threadIdx.x == 0) report(status, kErrIndex);
+        return;
+    }
+    const int cpg = C / G;
+    const SliceMap map{r0, C, g * cpg, cpg / VEC, VEC, (r1 - r0) * (cpg / VEC) < (1ll << 31)};
+    const long long nv = (r1 - r0) * map.vpr;
+    if (nv == 0) return;
+
+    // pass 1: statistics
+    Raw keep[kBatch];
+    Stats st;
+#pragma unroll
+    for (int i = 0; i < kBatch; ++i) {
+        const long long e = threadIdx.x + (long long)i * kThreads;
+        int c;
+        if (e < nv) keep[i] = CK::load(x + map.at(e, c));
+    }
+#pragma unroll
+    for (int i = 0; i < kBatch; ++i) {
+        if (threadIdx.x + (long long)i * kThreads < nv) {
+            float v[VEC];
+            CK::unpack(keep[i], v);
+            st.add_chunk<VEC>(v);
+        }
+    }
+    for (long long base = threadIdx.x + kStride; base < nv; base += kStride) {
+        Raw t[kBatch];
+#pragma unroll
+        for (int i = 0; i < kBatch; ++i) {
+            int c;
+            if (base + (long long)i * kThreads < nv)
+                t[i] = CK::load(x + map.at(base + i * kThreads, c));
+        }
+#pragma unroll
+        for (int i = 0; i < kBatch; ++i) {
+            if (base + (long long)i * kThreads < nv) {
+                float v[VEC];
+                CK::unpack(t[i], v);
+                st.add_chunk<VEC>(v);
+            }
+        }
+    }
+    float n = st.n, mean = st.mean, m2 = st.m2;
+    block_merge(n, mean, m2, red);
+    const float mu = mean;
+    const float inv = 1.f / sqrtf(m2 / n + eps);
+
+    // pass 2: normalise, affine, activation, store
+    auto finish = [&](Raw r, long long off, int c) {
+        float v[VEC];
+        CK::unpack(r, v);
+#pragma unroll
+        for (int k = 0; k < VEC; ++k) {
+            float z = (v[k] - mu) * inv;
+            if (gamma) z *= __ldg(gamma + c + k);
+            if (beta) z += __ldg(beta + c + k);
+            v[k] = act_apply(z, act);
+        }
+        CK::store(y + off, v);
+    };
+    for (long long j = (nv - 1) / kStride; j >= 1; --j) {
+        const long long base = threadIdx.x + j * kStride;
+        Raw t[kBatch];
+#pragma unroll
+        for (int i = 0; i < kBatch; ++i) {
+            int c;
+            if (base + (long long)i * kThreads < nv)
+                t[i] = CK::load(x + map.at(base + i * kThreads, c));
+        }
+#pragma unroll
+        for (int i = 0; i < kBatch; ++i) {
+            if (base + (long long)i * kThreads < nv) {
+                int c;
+                const long long off = map.at(base + i * kThreads, c);
+                finish(t[i], off, c);
+            }
+        }
+    }
+#pragma unroll
+    for (int i = 0; i < kBatch; ++i) {
+        const long long e = threadIdx.x + (long long)i * kThreads;
+        if (e < nv) {
+            int c;
+            const long long off = map.at(e, c);
+            finish(keep[i], off, c);
+        }
+    }
+}
+
+template <typename T, int VEC, int GPC>
+hc_status launch_fast(const DeviceCtx* ctx, const void* x, const int32_t* offsets, int B,
+                      long long capacity, int C, int G, float eps, const float* gamma,
+                      const float* beta, int act, void* y, cudaStream_t s) {
+    // ranges of at least ~64 rows; at most 3 CTAs per SM (the kernels' bound)
+    long long grid = (capacity + 63) / 64;
+    const long long cap = (long long)ctx->num_sms * 3;
+    if (grid > cap) grid = cap;
+    if (grid < 1) grid = 1;
+    GnPart* part = (GnPart*)stream_workspace(s, sizeof(GnPart) * (size_t)(B + grid) * G);
+    if (!part) return HC_ERR_CUDA;
+    hc_status st = launch_pdl(gn_stats_kernel<T, VEC, GPC>, dim3((unsigned)grid), dim3(kThreads),
+                              0, s, "gn_stats_kernel", (const T*)x, offsets, B, C, G, capacity,
+                              part, ctx->status);
+    if (st != HC_OK) return st;
+    return launch_pdl(gn_apply_kernel<T, VEC, GPC>, dim3((unsigned)grid), dim3(kThreads), 0, s,
+                      "gn_apply_kernel", (const T*)x, offsets, B, C, G, capacity,
+                      (const GnPart*)part, eps, gamma, beta, act, (T*)y, ctx->status);
+}
+
+template <typename T>
+hc_status launch_typed(const DeviceCtx* ctx, const void* x, const int32_t* offsets, int B,
+                       long long capacity, int C, int G, float eps, const float* gamma,
+                       const float* beta, int act, void* y, cudaStream_t s) {
+    constexpr int kVec = 16 / (int)sizeof(T);
+    const int cpg = C / G;
+    const uintptr_t al = (uintptr_t)x | (uintptr_t)y;
+    const bool aligned = C % kVec == 0 && al % 16 == 0;
+    const int cpr = C / kVec;
+    // HC_GN_SLICE forces the general path (for testing it on every layout)
+    const bool fast_rows = aligned && cpr >= 1 && cpr <= kThreads && (cpr & (cpr - 1)) == 0 &&
+                           G <= kMaxGroupsFast && getenv("HC_GN_SLICE") == nullptr;
+    if (fast_rows && cpg % kVec == 0)
+        return launch_fast<T, kVec, 1>(ctx, x, offsets, B, capacity, C, G, eps, gamma, beta, act,
+                                       y, s);
+    if (fast_rows && kVec % cpg == 0) {
+        if (kVec / cpg == 2)
+            return launch_fast<T, kVec, 2>(ctx, x, offsets, B, capacity, C, G, eps, gamma, beta,
+                                           act, y, s);
+        if (kVec / cpg == 4)
+            return launch_fast<T, kVec, 4>(ctx, x, offsets, B, capacity, C, G, eps, gamma, beta,
+                                           act, y, s);
+        if constexpr (kVec == 8)
+            return launch_fast<T, kVec, 8>(ctx, x, offsets, B, capacity, C, G, eps, gamma, beta,
+                                           act, y, s);
+    }
+    const dim3 grid((unsigned)((long long)B * G));
+    if (cpg % kVec == 0 && aligned)
+        return launch_pdl(group_norm_slice_kernel<T, kVec>, grid, dim3(kThreads), 0, s,
+                          "group_norm_slice_kernel", (const T*)x, offsets, C, G, capacity, eps,
+                          gamma, beta, act, (T*)y, ctx->status);
+    return launch_pdl(group_norm_slice_kernel<T, 1>, grid, dim3(kThreads), 0, s,
+                      "group_norm_slice_kernel", (const T*)x, offsets, C, G, capacity, eps, gamma,
+                      beta, act, (T*)y, ctx->status);
+}
+
+}  // namespace
+
+hc_status launch_group_norm(const DeviceCtx* ctx, const void* x, hc_dtype dt,
+                            const int32_t* offsets, int B, long long capacity, int C, int G,
+                            float eps, const float* gamma, const float* beta, int act, void* y,
+                            cudaStream_t s) {
+    if (dt == HC_F32)
+        return launch_typed<float>(ctx, x, offsets, B, capacity, C, G, eps, gamma, beta, act, y, s);
+    return launch_typed<__nv_bfloat16>(ctx, x, offsets, B, capacity, C, G, eps, gamma, beta, act,
+                                       y, s);
+}
+
+}  // namespace hc

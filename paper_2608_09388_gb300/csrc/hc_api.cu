@@ -330,6 +330,30 @@ hc_status hc_sparse_conv_rulebook_fwd(const void* x, hc_dtype dt, int x_rows,
     return dispatch_conv(ctx, a, dt, (cudaStream_t)stream);
 }
 
+hc_status hc_sparse_group_norm_fwd(const void* x, hc_dtype dt, const int32_t* batch_offsets, int B,
+                                   int capacity, int C, int G, float eps, const float* gamma,
+                                   const float* beta, hc_act act, void* y, hc_stream_t stream) {
+    const char* fn = "hc_sparse_group_norm_fwd";
+    t_last_error[0] = 0;
+    HC_REQUIRE(dt == HC_F32 || dt == HC_BF16, "%s: unknown dtype %d", fn, (int)dt);
+    HC_REQUIRE(act == HC_ACT_NONE || act == HC_ACT_ELU || act == HC_ACT_RELU,
+               "%s: unknown activation %d", fn, (int)act);
+    HC_REQUIRE(B >= 0 && capacity >= 0, "%s: B=%d capacity=%d must be >= 0", fn, B, capacity);
+    HC_REQUIRE(C >= 1 && G >= 1 && C % G == 0, "%s: C=%d must be a multiple of G=%d >= 1", fn, C,
+               G);
+    HC_REQUIRE((long long)B * G < (1ll << 31), "%s: B*G=%lld too large", fn, (long long)B * G);
+    HC_REQUIRE(eps >= 0.f, "%s: eps must be >= 0", fn);
+    HC_REQUIRE(batch_offsets != nullptr, "%s: batch_offsets is NULL", fn);
+    if (B == 0 || capacity == 0) return HC_OK;
+    HC_REQUIRE(x && y, "%s: x and y are required", fn);
+    const int eb = dt == HC_F32 ? 4 : 2;
+    HC_REQUIRE(!misaligned(x, eb) && !misaligned(y, eb), "%s: misaligned x/y", fn);
+    const DeviceCtx* ctx = device_ctx();
+    if (!ctx) return HC_ERR_CUDA;
+    return launch_group_norm(ctx, x, dt, batch_offsets, B, capacity, C, G, eps, gamma, beta,
+                             (int)act, y, (cudaStream_t)stream);
+}
+
 hc_status hc_scatter_dense(const void* y, hc_dtype dt, const int32_t* coords,
                            const int32_t* row_of, const int32_t* count, int B, int V, int C,
                            int zero_fill, void* out, hc_stream_t stream) {

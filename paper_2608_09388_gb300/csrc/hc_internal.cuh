@@ -81,6 +81,10 @@ bool conv_tc_supported(const ConvArgs& a, hc_dtype dt);
 hc_status launch_rulebook(const DeviceCtx* ctx, const int32_t* coords, const int32_t* row_of,
                           const int32_t* count, const int32_t* spiral, int B, int V, int L,
                           int x_layout, int32_t* rulebook, cudaStream_t s);
+hc_status launch_group_norm(const DeviceCtx* ctx, const void* x, hc_dtype dt,
+                            const int32_t* offsets, int B, long long capacity, int C, int G,
+                            float eps, const float* gamma, const float* beta, int act, void* y,
+                            cudaStream_t s);
 hc_status launch_scatter(const DeviceCtx* ctx, const void* y, int elem_bytes, const int32_t* coords,
                          const int32_t* row_of, const int32_t* count, int B, int V, int C,
                          int zero_fill, void* out, cudaStream_t s);

@@ -30,7 +30,7 @@ STATUS_NAMES = {0: "HC_OK", 1: "HC_ERR_INVALID_ARG", 2: "HC_ERR_UNSUPPORTED",
 # Exported symbols, as declared in include/hc.h.
 EXPORTS = ("hc_mask_compact", "hc_mask_compact_static", "hc_sparse_spiral_conv_fwd",
            "hc_conv_rulebook", "hc_sparse_conv_rulebook_fwd", "hc_sparse_linear_fwd",
-           "hc_scatter_dense", "hc_spiral_conv_fwd", "hc_get_device_status",
+           "hc_sparse_group_norm_fwd", "hc_scatter_dense", "hc_spiral_conv_fwd", "hc_get_device_status",
            "hc_last_error_string", "hc_version")
 
 
@@ -63,6 +63,7 @@ def load_library(path: str | None = None):
             "hc_sparse_conv_rulebook_fwd": [P, I, I, P, P, I, I, I, I, P, P, I, P, P, I, I, P,
                                             P],
             "hc_sparse_linear_fwd": [P, I, P, I, I, I, P, P, I, P, P],
+            "hc_sparse_group_norm_fwd": [P, I, P, I, I, I, I, ctypes.c_float, P, P, I, P, P],
             "hc_scatter_dense": [P, I, P, P, P, I, I, I, I, P, P],
             "hc_spiral_conv_fwd": [P, I, P, I, I, I, I, I, P, P, I, P, P],
             "hc_get_device_status": [P],
@@ -170,6 +171,16 @@ def hc_sparse_linear_fwd(x, count, W, bias, act, y, stream=None):
     _check(load_library().hc_sparse_linear_fwd(
         _p(x), _dt(x), _p(count), capacity, C_in, C_out, _p(W), _p(bias), act, _p(y),
         _s(stream)), "hc_sparse_linear_fwd")
+
+
+def hc_sparse_group_norm_fwd(x, batch_offsets, G, eps, gamma, beta, act, y, stream=None):
+    """Group norm of compact rows x [capacity, C], per frame (batch_offsets
+    [B+1]) and group of C/G channels; y may be x."""
+    capacity, C = x.shape
+    B = batch_offsets.shape[0] - 1
+    _check(load_library().hc_sparse_group_norm_fwd(
+        _p(x), _dt(x), _p(batch_offsets), B, capacity, C, G, float(eps), _p(gamma), _p(beta),
+        act, _p(y), _s(stream)), "hc_sparse_group_norm_fwd")
 
 
 def hc_scatter_dense(y, coords, row_of, count, B, V, zero_fill, out, stream=None):

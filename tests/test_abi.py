@@ -76,3 +76,21 @@ def test_missing_library_fails_loudly(tmp_path, monkeypatch):
     monkeypatch.setattr(hc, "_lib", None)
     with pytest.raises(RuntimeError, match="not built"):
         hc.load_library(str(tmp_path / "nope.so"))
+
+
+def test_group_norm_arguments_rejected_on_host(lib):
+    fake = ctypes.c_void_p(0x1000)
+    f = ctypes.c_float
+    gn = lib.hc_sparse_group_norm_fwd
+    bad = [
+        (fake, 0, fake, 2, 10, 10, 3, f(1e-5), None, None, 0, fake, None),  # C % G != 0
+        (fake, 0, fake, 2, 10, 8, 0, f(1e-5), None, None, 0, fake, None),   # G = 0
+        (fake, 0, fake, 2, 10, 8, 2, f(-1.0), None, None, 0, fake, None),   # eps < 0
+        (fake, 7, fake, 2, 10, 8, 2, f(1e-5), None, None, 0, fake, None),   # dtype
+        (fake, 0, fake, 2, 10, 8, 2, f(1e-5), None, None, 9, fake, None),   # activation
+        (fake, 0, None, 2, 10, 8, 2, f(1e-5), None, None, 0, fake, None),   # no offsets
+    ]
+    for args in bad:
+        assert gn(*args) == hc.HC_ERR_INVALID_ARG
+    # nothing to do: returns before any device call
+    assert gn(fake, 0, fake, 0, 10, 8, 2, f(1e-5), None, None, 0, fake, None) == hc.HC_OK

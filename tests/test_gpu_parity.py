@@ -403,6 +403,147 @@ def test_scatter_dense(C, zero_fill, dtype):
     np.testing.assert_array_equal(to_numpy(out), ref)
 
 
+# ------------------------------------------------------------------ group norm
+
+def _gn_case(rng, sizes, C, dtype, shift=3.0, slack=5):
+    """Compact rows for frames of the given row counts (plus `slack` rows
+    that belong to no frame), features N(shift, 1)."""
+    offs = np.concatenate([[0], np.cumsum(sizes)]).astype(np.int32)
+    cap = int(offs[-1]) + slack
+    x = rng.standard_normal((cap, C)).astype(np.float32) + np.float32(shift)
+    if dtype == "bf16":
+        x = inputs.to_bf16_bits(x)
+    return x, offs
+
+
+def run_group_norm(x, offs, G, gamma, beta, act, eps=1e-5, in_place=False):
+    xt = to_torch(x)
+    y = xt if in_place else torch.full_like(xt, float("nan"))
+    hc.hc_sparse_group_norm_fwd(xt, to_torch(offs), G, eps,
+                                None if gamma is None else to_torch(gamma),
+                                None if beta is None else to_torch(beta), act, y)
+    assert hc.hc_get_device_status() == hc.HC_OK
+    return to_numpy(y)
+
+
+def _as_f32(a):
+    return (a.astype(np.uint32) << 16).view(np.float32) if a.dtype == np.uint16 else a
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("C,G", [(8, 1), (64, 4), (64, 8), (128, 32), (128, 64), (128, 128),
+                                 (256, 16), (1024, 512), (42, 6), (48, 3)])
+@pytest.mark.parametrize("affine,act", [(False, 0), (True, 1), (True, 2)])
+def test_group_norm(C, G, affine, act, dtype):
+    """Frames of 0, 1, a few, a tile-ish and a large number of rows; rows
+    after the last frame stay untouched."""
+    rng = np.random.default_rng(C * 100 + G * 7 + act)
+    sizes = [0, 1, 3, 0, 130, 517, 2900, 64]
+    x, offs = _gn_case(rng, sizes, C, dtype)
+    gamma = (1.0 + 0.5 * rng.standard_normal(C)).astype(np.float32) if affine else None
+    beta = (0.3 * rng.standard_normal(C)).astype(np.float32) if affine else None
+    got = run_group_norm(x, offs, G, gamma, beta, act)
+    y_pre, _ = oracle.sparse_group_norm(x, offs, G, 1e-5, gamma, beta, act)
+    n = int(offs[-1])
+    check_close(got[:n], y_pre[:n], f"group norm C={C} G={G} {dtype}")
+    assert np.isnan(_as_f32(got[n:])).all()
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("C,G", [(64, 8), (128, 32), (2048, 8)])
+@pytest.mark.parametrize("path", ["rows", "slice"])
+def test_group_norm_paths_and_frame_shapes(C, G, path, dtype, monkeypatch):
+    """Both kernels (contiguous row ranges, and one CTA per frame and group)
+    on many tiny frames (a row range holds dozens of frame segments) and on
+    one frame spread over hundreds of row ranges (its partials are merged by
+    a warp)."""
+    if path == "slice":
+        monkeypatch.setenv("HC_GN_SLICE", "1")
+    rng = np.random.default_rng(C + G)
+    tiny = [int(v) for v in rng.integers(0, 6, size=300)]
+    big = [40000 if C <= 128 else 3000]
+    for sizes in (tiny, big, tiny[:40] + big + tiny[40:80]):
+        x, offs = _gn_case(rng, sizes, C, dtype, shift=-1.5)
+        gamma = (1.0 + 0.5 * rng.standard_normal(C)).astype(np.float32)
+        got = run_group_norm(x, offs, G, gamma, None, 2)
+        y_pre, _ = oracle.sparse_group_norm(x, offs, G, 1e-5, gamma, None, 2)
+        n = int(offs[-1])
+        check_close(got[:n], y_pre[:n], f"group norm {path} C={C} G={G} {dtype} B={len(sizes)}")
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_group_norm_in_place_and_misaligned(dtype):
+    rng = np.random.default_rng(5)
+    C, G = 64, 8
+    x, offs = _gn_case(rng, [300, 0, 1100, 7], C, dtype)
+    y_pre, _ = oracle.sparse_group_norm(x, offs, G, 1e-5, None, None, 1)
+    n = int(offs[-1])
+    check_close(run_group_norm(x, offs, G, None, None, 1, in_place=True)[:n], y_pre[:n],
+                "in place")
+    # a view starting one element in: the 16-byte paths are not taken
+    xt = to_torch(x)
+    buf = torch.empty(x.size + 1, dtype=xt.dtype, device="cuda")
+    xs = buf[1:].view(x.shape)
+    xs.copy_(xt)
+    ys = torch.full_like(xs, float("nan"))
+    hc.hc_sparse_group_norm_fwd(xs, to_torch(offs), G, 1e-5, None, None, 1, ys)
+    assert hc.hc_get_device_status() == hc.HC_OK
+    check_close(to_numpy(ys)[:n], y_pre[:n], "misaligned")
+
+
+@pytest.mark.parametrize("path", ["rows", "slice"])
+def test_group_norm_constant_group_and_eps(path, monkeypatch):
+    """A group of equal values normalises to exactly 0 (then + beta); eps
+    from 0 to large enters as 1/sqrt(var + eps)."""
+    if path == "slice":
+        monkeypatch.setenv("HC_GN_SLICE", "1")
+    C, G = 32, 4
+    offs = np.array([0, 200, 201], dtype=np.int32)
+    x = np.full((201, C), 100.25, dtype=np.float32)
+    beta = np.linspace(-1, 1, C).astype(np.float32)
+    got = run_group_norm(x, offs, G, None, beta, 0)
+    np.testing.assert_array_equal(got, np.broadcast_to(beta, got.shape))
+    rng = np.random.default_rng(9)
+    x, offs = _gn_case(rng, [50, 400], C, "f32", shift=-2.0, slack=0)
+    for eps in (0.0, 1e-5, 4.0):
+        y_pre, _ = oracle.sparse_group_norm(x, offs, G, eps, None, None, 0)
+        check_close(run_group_norm(x, offs, G, None, None, 0, eps=eps), y_pre, f"eps={eps}")
+
+
+def test_group_norm_on_compacted_layer_output():
+    """The normalisation an encoder applies after a conv: a full-size
+    compacted bf16 activation (32 clustered frames of the 10475-vertex
+    sphere, 128 channels, G = 8), frame ranges from hc_mask_compact."""
+    w = inputs.make_workload("layer10475_bf16")
+    coords, row_of, offs, count = gpu_compact(w.masks[0])
+    n = int(count.item())
+    rng = np.random.default_rng(77)
+    x = inputs.features(rng, (n, 128), "bf16")
+    gamma = (1.0 + 0.2 * rng.standard_normal(128)).astype(np.float32)
+    beta = (0.1 * rng.standard_normal(128)).astype(np.float32)
+    xt = to_torch(x)
+    y = torch.empty_like(xt)
+    hc.hc_sparse_group_norm_fwd(xt, offs, 8, 1e-5, to_torch(gamma), to_torch(beta),
+                                hc.HC_ACT_ELU, y)
+    assert hc.hc_get_device_status() == hc.HC_OK
+    y_pre, _ = oracle.sparse_group_norm(x, to_numpy(offs), 8, 1e-5, gamma, beta, oracle.ACT_ELU)
+    check_close(to_numpy(y), y_pre, "group norm full size")
+
+
+@pytest.mark.parametrize("path", ["rows", "slice"])
+def test_group_norm_bad_offsets_reported(path, monkeypatch):
+    if path == "slice":
+        monkeypatch.setenv("HC_GN_SLICE", "1")
+    x = torch.zeros((10, 16), dtype=torch.float32, device="cuda")
+    offs = torch.tensor([0, 4, 12], dtype=torch.int32, device="cuda")  # 12 > capacity
+    hc.hc_sparse_group_norm_fwd(x, offs, 4, 1e-5, None, None, 0, x)
+    assert hc.hc_get_device_status() == hc.HC_ERR_INVALID_INDEX
+    offs = torch.tensor([0, 5, 3], dtype=torch.int32, device="cuda")  # decreasing
+    hc.hc_sparse_group_norm_fwd(x, offs, 4, 1e-5, None, None, 0, x)
+    assert hc.hc_get_device_status() == hc.HC_ERR_INVALID_INDEX
+    assert hc.hc_get_device_status() == hc.HC_OK
+
+
 # ------------------------------------------------------------------ encoders
 
 def run_encoder_gpu(w):
