@@ -220,7 +220,7 @@ hc_status hc_sparse_linear_fwd(const void* x, hc_dtype dt, const int32_t* count,
  *             access leaves x, y or the library's workspace.
  * Statistics in fp32 by pairwise (count, mean, M2) merging; the variance is
  * taken around the mean, never as E[x^2] - mean^2. Uses the library's
- * per-stream workspace ((B + 3 * SMs) * G * 16 bytes at most).
+ * per-stream workspace ((B + 2 * SMs) * G * 16 bytes at most).
  */
 hc_status hc_sparse_group_norm_fwd(const void* x, hc_dtype dt, const int32_t* batch_offsets, int B,
                                    int capacity, int C, int G, float eps, const float* gamma,

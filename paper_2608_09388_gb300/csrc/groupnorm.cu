@@ -25,8 +25,14 @@
 //   gn_apply_kernel: same ranges; per frame segment, merge the partials of
 //     the CTAs that hold the frame, normalise and store. Segments and rows
 //     are walked in reverse, so the most recently read rows, still in L2,
-//     are consumed first.
-// The general path (one CTA per (frame, group)) serves every other layout.
+//     are consumed first, and its loads and stores carry an L2 evict-first
+//     policy (last use), which keeps the rest of the input in L2.
+// Frames are located by a kThreads-ary block search of the frame table and
+// read a window of kThreads frames at a time into shared memory; loads are
+// issued a batch ahead of the arithmetic.
+// The general path (one CTA per (frame, group)) serves every other layout,
+// and small frames (a group slice within its register cache), where one
+// launch beats the two latency-bound row-range launches.
 // The output may alias the input in both paths. Deterministic, no atomics.
 #include <cuda_bf16.h>
 
@@ -98,6 +104,33 @@ struct Chunk<__nv_bfloat16, 8> {
     }
 };
 
+// 16-byte accesses with an L2 evict-first policy (last use of a line).
+__device__ __forceinline__ uint64_t l2_evict_first_policy() {
+    uint64_t pol;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+    return pol;
+}
+__device__ __forceinline__ uint4 ld_ef(const void* p, uint64_t pol) {
+    uint4 v;
+    asm volatile("ld.global.L2::cache_hint.v4.u32 {%0, %1, %2, %3}, [%4], %5;"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(p), "l"(pol));
+    return v;
+}
+__device__ __forceinline__ void st_ef(void* p, uint4 v, uint64_t pol) {
+    asm volatile("st.global.L2::cache_hint.v4.u32 [%0], {%1, %2, %3, %4}, %5;" ::"l"(p), "r"(v.x),
+                 "r"(v.y), "r"(v.z), "r"(v.w), "l"(pol)
+                 : "memory");
+}
+template <typename Raw>
+__device__ __forceinline__ Raw as_raw(uint4 v) {
+    return *reinterpret_cast<const Raw*>(&v);
+}
+template <typename Raw>
+__device__ __forceinline__ uint4 as_u4(const Raw& v) {
+    return *reinterpret_cast<const uint4*>(&v);
+}
+
 // Running (count, mean, M2), fp32. Counts are exact integers below 2^24.
 struct Stats {
     float n = 0.f, mean = 0.f, m2 = 0.f;
@@ -115,7 +148,7 @@ struct Stats {
         }
         const float nn = n + (float)VEC;
         const float d = cm - mean;
-        const float r = (float)VEC / nn;
+        const float r = (float)VEC * __frcp_rn(nn);
         mean = fmaf(d, r, mean);
         m2 += q + d * d * n * r;
         n = nn;
@@ -128,7 +161,7 @@ __device__ __forceinline__ void merge(float& n, float& mean, float& m2, float nb
     if (nb == 0.f) return;
     const float nn = n + nb;
     const float d = mb - mean;
-    const float r = nb / nn;
+    const float r = nb * __frcp_rn(nn);
     mean = fmaf(d, r, mean);
     m2 += qb + d * d * n * r;
     n = nn;
@@ -168,17 +201,32 @@ struct RangeMap {
     __device__ __forceinline__ long long cta_of(long long row) const { return (row - off0) / R; }
 };
 
-// First frame b with offsets[b + 1] > row (the frame holding `row`).
-__device__ __forceinline__ int frame_of(const int32_t* offsets, int B, long long row) {
-    int lo = 0, hi = B;  // answer in [lo, hi]
-    while (lo < hi) {
-        const int mid = (lo + hi) >> 1;
-        if ((long long)__ldg(offsets + mid + 1) > row)
-            hi = mid;
-        else
-            lo = mid + 1;
+// First frame b in [0, B] with offsets[b + 1] > row (B if none): a
+// kThreads-ary search, every thread of the block taking part, so one round
+// trip to the table per factor of kThreads frames. A malformed (unsorted)
+// table yields some b in [0, B].
+__device__ __forceinline__ int find_frame(const int32_t* offsets, int B, long long row) {
+    long long wlo = 0, whi = B;
+    while (whi > wlo) {
+        const long long step = (whi - wlo + kThreads - 1) / kThreads;
+        const long long p = wlo + (long long)threadIdx.x * step;
+        const int before = p < whi && (long long)__ldg(offsets + p + 1) <= row;
+        const int k = __syncthreads_count(before);
+        if (step == 1) return (int)(wlo + k);
+        const long long nlo = k == 0 ? wlo : wlo + (long long)(k - 1) * step + 1;
+        const long long nhi = wlo + (long long)k * step < whi ? wlo + (long long)k * step : whi;
+        wlo = nlo;
+        whi = nhi;
     }
-    return lo;
+    __syncthreads();  // every exit path passes the same number of barriers
+    return (int)wlo;
+}
+
+// offsets[wb + j] for j in [0, n] into s_off (n <= kThreads).
+__device__ __forceinline__ void load_window(const int32_t* offsets, int wb, int n, int* s_off) {
+    __syncthreads();  // the previous window is no longer read
+    for (int j = threadIdx.x; j <= n; j += kThreads) s_off[j] = __ldg(offsets + wb + j);
+    __syncthreads();
 }
 
 // Thread layout: cpr chunks per row; thread t owns chunk column t % cpr and
@@ -221,13 +269,14 @@ __device__ __forceinline__ bool range_setup(const int32_t* offsets, int B, long 
 }
 
 template <typename T, int VEC, int GPC>
-__global__ void __launch_bounds__(kThreads, 3)
+__global__ void __launch_bounds__(kThreads, 2)
     gn_stats_kernel(const T* x, const int32_t* __restrict__ offsets, int B, int C, int G,
                     long long capacity, GnPart* __restrict__ part, unsigned* status) {
     using CK = Chunk<T, VEC>;
     using Raw = typename CK::Raw;
     constexpr int SUB = VEC / GPC;  // elements of one group inside a chunk (GPC > 1)
     __shared__ float red[kThreads * GPC * 3];
+    __shared__ int s_off[kThreads + 1];
     pdl_wait();
     pdl_trigger();
     // frames must be in order (each CTA checks a share of the table)
@@ -240,70 +289,94 @@ __global__ void __launch_bounds__(kThreads, 3)
     const Layout l = make_layout<VEC, GPC>(C, G);
     // after the warp merge: row slots (warps, or thread rows) x cpr columns
     const int nrs = l.cpr < 32 ? kThreads / 32 : kThreads / l.cpr;
+    const long long step = (long long)kBatch * l.rpp;
 
-    for (int b = frame_of(offsets, B, lo); b < B; ++b) {
-        const long long f0 = __ldg(offsets + b), f1 = __ldg(offsets + b + 1);
-        if (f0 >= hi) break;
-        if (f1 < f0) continue;  // reported above
-        const long long s0 = f0 > lo ? f0 : lo, s1 = f1 < hi ? f1 : hi;
-        if (s0 >= s1) continue;
+    auto segment = [&](int b, long long s0, long long s1) {
         Stats st[GPC];
-        for (long long r = s0 + l.rg; r < s1; r += (long long)kBatch * l.rpp) {
-            Raw t[kBatch];
+        Raw cur[kBatch];
 #pragma unroll
-            for (int i = 0; i < kBatch; ++i)
-                if (r + (long long)i * l.rpp < s1)
-                    t[i] = CK::load(x + (r + (long long)i * l.rpp) * C + l.col * VEC);
+        for (int i = 0; i < kBatch; ++i) {
+            const long long r = s0 + l.rg + (long long)i * l.rpp;
+            if (r < s1) cur[i] = CK::load(x + r * C + l.col * VEC);
+        }
+        for (long long r0 = s0 + l.rg; r0 < s1; r0 += step) {
+            Raw nxt[kBatch];  // next batch in flight while this one is reduced
 #pragma unroll
             for (int i = 0; i < kBatch; ++i) {
-                if (r + (long long)i * l.rpp < s1) {
-                    float v[VEC];
-                    CK::unpack(t[i], v);
+                const long long r = r0 + step + (long long)i * l.rpp;
+                if (r < s1) nxt[i] = CK::load(x + r * C + l.col * VEC);
+            }
 #pragma unroll
-                    for (int s = 0; s < GPC; ++s) st[s].template add_chunk<SUB>(v + s * SUB);
+            for (int i = 0; i < kBatch; ++i) {
+                if (r0 + (long long)i * l.rpp < s1) {
+                    float v[VEC];
+                    CK::unpack(cur[i], v);
+#pragma unroll
+                    for (int q = 0; q < GPC; ++q) st[q].template add_chunk<SUB>(v + q * SUB);
                 }
             }
+#pragma unroll
+            for (int i = 0; i < kBatch; ++i) cur[i] = nxt[i];
         }
         // lanes holding the same column: merge across the warp
 #pragma unroll
-        for (int s = 0; s < GPC; ++s)
-            for (int o = l.cpr; o < 32; o <<= 1) merge_xor(st[s].n, st[s].mean, st[s].m2, o);
+        for (int q = 0; q < GPC; ++q)
+            for (int o = l.cpr; o < 32; o <<= 1) merge_xor(st[q].n, st[q].mean, st[q].m2, o);
         const int lane = threadIdx.x & 31;
+        __syncthreads();  // red[] of the previous segment has been read
         if (l.cpr >= 32 || lane < l.cpr) {
             const int slot = l.cpr < 32 ? (int)(threadIdx.x >> 5) : l.rg;
 #pragma unroll
-            for (int s = 0; s < GPC; ++s) {
-                float* e = red + 3 * ((slot * l.cpr + l.col) * GPC + s);
-                e[0] = st[s].n, e[1] = st[s].mean, e[2] = st[s].m2;
+            for (int q = 0; q < GPC; ++q) {
+                float* e = red + 3 * ((slot * l.cpr + l.col) * GPC + q);
+                e[0] = st[q].n, e[1] = st[q].mean, e[2] = st[q].m2;
             }
         }
         __syncthreads();
         GnPart* out = part + (long long)(b + blockIdx.x) * G;
         for (int g = threadIdx.x; g < G; g += kThreads) {
             const int c0 = GPC == 1 ? g * l.cpc : g / GPC, nc = GPC == 1 ? l.cpc : 1;
-            const int s = GPC == 1 ? 0 : g % GPC;
+            const int q = GPC == 1 ? 0 : g % GPC;
             float n = 0.f, mean = 0.f, m2 = 0.f;
             for (int rs = 0; rs < nrs; ++rs)
                 for (int c = c0; c < c0 + nc; ++c) {
-                    const float* e = red + 3 * ((rs * l.cpr + c) * GPC + s);
+                    const float* e = red + 3 * ((rs * l.cpr + c) * GPC + q);
                     merge(n, mean, m2, e[0], e[1], e[2]);
                 }
             out[g] = GnPart{n, mean, m2, 0.f};
         }
-        __syncthreads();  // red[] is reused by the next segment
+    };
+
+    // frames overlapping [lo, hi), a window of kThreads frames at a time
+    for (int wb = find_frame(offsets, B, lo); wb < B; wb += kThreads) {
+        const int nw = B - wb < kThreads ? B - wb : kThreads;
+        load_window(offsets, wb, nw, s_off);
+        bool past = false;
+        for (int j = 0; j < nw; ++j) {
+            const long long f0 = s_off[j], f1 = s_off[j + 1];
+            if (f0 >= hi) {
+                past = true;
+                break;
+            }
+            const long long s0 = f0 > lo ? f0 : lo, s1 = f1 < hi ? f1 : hi;
+            if (s0 < s1) segment(wb + j, s0, s1);  // f1 < f0 is reported above
+        }
+        if (past || (long long)s_off[nw] >= hi) break;
     }
 }
 
 template <typename T, int VEC, int GPC>
-__global__ void __launch_bounds__(kThreads, 3)
+__global__ void __launch_bounds__(kThreads, 2)
     gn_apply_kernel(const T* x, const int32_t* __restrict__ offsets, int B, int C, int G,
                     long long capacity, const GnPart* __restrict__ part, float eps,
                     const float* __restrict__ gamma, const float* __restrict__ beta, int act, T* y,
                     unsigned* status) {
     using CK = Chunk<T, VEC>;
     using Raw = typename CK::Raw;
+    static_assert(sizeof(Raw) == 16, "the row-range path moves 16-byte chunks");
     constexpr int SUB = VEC / GPC;
     __shared__ float s_mu[kMaxGroupsFast], s_inv[kMaxGroupsFast];
+    __shared__ int s_off[kThreads + 1];
     pdl_wait();
     pdl_trigger();
     RangeMap m;
@@ -317,21 +390,17 @@ __global__ void __launch_bounds__(kThreads, 3)
         be[k] = beta ? __ldg(beta + l.col * VEC + k) : 0.f;
     }
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int b_first = frame_of(offsets, B, lo);
-    int b_last = frame_of(offsets, B, hi - 1);
-    if (b_last > B - 1) b_last = B - 1;
+    const long long step = (long long)kBatch * l.rpp;
+    const uint64_t pol = l2_evict_first_policy();
 
-    for (int b = b_last; b >= b_first; --b) {  // frames last to first
-        const long long f0 = __ldg(offsets + b), f1 = __ldg(offsets + b + 1);
-        if (f1 < f0) continue;  // reported by the statistics kernel
-        const long long s0 = f0 > lo ? f0 : lo, s1 = f1 < hi ? f1 : hi;
-        if (s0 >= s1) continue;
+    auto segment = [&](int b, long long f0, long long f1, long long s0, long long s1) {
         // partials of the CTAs that hold frame b: slots b + c, c in [c0, c1]
         // (clamped to the table's span, so a malformed table cannot index
         // outside the workspace)
         const long long c0 = m.cta_of(f0 > m.off0 ? f0 : m.off0);
         const long long c1 = m.cta_of((f1 < m.end ? f1 : m.end) - 1);
         const GnPart* pb = part + (long long)b * G;
+        __syncthreads();  // s_mu / s_inv of the previous segment have been read
         if (c1 - c0 < 8) {
             for (int g = threadIdx.x; g < G; g += kThreads) {
                 float n = 0.f, mean = 0.f, m2 = 0.f;
@@ -360,35 +429,65 @@ __global__ void __launch_bounds__(kThreads, 3)
         __syncthreads();
         float mu[GPC], inv[GPC];
 #pragma unroll
-        for (int s = 0; s < GPC; ++s) {
-            const int g = GPC == 1 ? l.col / l.cpc : l.col * GPC + s;
-            mu[s] = s_mu[g];
-            inv[s] = s_inv[g];
+        for (int q = 0; q < GPC; ++q) {
+            const int g = GPC == 1 ? l.col / l.cpc : l.col * GPC + q;
+            mu[q] = s_mu[g];
+            inv[q] = s_inv[g];
         }
-        // rows of the segment, last to first
-        const long long last = (s1 - s0) - 1 - l.rg;  // this thread's highest row offset
-        for (long long r = last; r >= 0; r -= (long long)kBatch * l.rpp) {
-            Raw t[kBatch];
+        // rows of the segment last to first (the statistics pass read them
+        // first to last, so the most recent ones are still in L2); every
+        // line is read and written here for the last time: evict first
+        auto row_at = [&](long long r) { return (s0 + r) * C + l.col * VEC; };
+        const long long top = (s1 - s0) - 1 - l.rg;  // this thread's highest row offset
+        Raw cur[kBatch];
 #pragma unroll
-            for (int i = 0; i < kBatch; ++i)
-                if (r - (long long)i * l.rpp >= 0)
-                    t[i] = CK::load(x + (s0 + r - (long long)i * l.rpp) * C + l.col * VEC);
+        for (int i = 0; i < kBatch; ++i)
+            if (top - (long long)i * l.rpp >= 0)
+                cur[i] = as_raw<Raw>(ld_ef(x + row_at(top - (long long)i * l.rpp), pol));
+        for (long long r0 = top; r0 >= 0; r0 -= step) {
+            Raw nxt[kBatch];
 #pragma unroll
             for (int i = 0; i < kBatch; ++i) {
-                if (r - (long long)i * l.rpp >= 0) {
+                const long long r = r0 - step - (long long)i * l.rpp;
+                if (r >= 0) nxt[i] = as_raw<Raw>(ld_ef(x + row_at(r), pol));
+            }
+#pragma unroll
+            for (int i = 0; i < kBatch; ++i) {
+                const long long r = r0 - (long long)i * l.rpp;
+                if (r >= 0) {
                     float v[VEC];
-                    CK::unpack(t[i], v);
+                    CK::unpack(cur[i], v);
 #pragma unroll
                     for (int k = 0; k < VEC; ++k) {
-                        const int s = k / SUB;
-                        const float z = fmaf((v[k] - mu[s]) * inv[s], ga[k], be[k]);
+                        const int q = k / SUB;
+                        const float z = fmaf((v[k] - mu[q]) * inv[q], ga[k], be[k]);
                         v[k] = act_apply(z, act);
                     }
-                    CK::store(y + (s0 + r - (long long)i * l.rpp) * C + l.col * VEC, v);
+                    T* dst = y + row_at(r);
+                    Raw packed;
+                    CK::store(reinterpret_cast<T*>(&packed), v);
+                    st_ef(dst, as_u4(packed), pol);
                 }
             }
+#pragma unroll
+            for (int i = 0; i < kBatch; ++i) cur[i] = nxt[i];
         }
-        __syncthreads();  // s_mu / s_inv are rewritten for the next frame
+    };
+
+    // frames overlapping [lo, hi); within a window of kThreads frames, last
+    // to first
+    for (int wb = find_frame(offsets, B, lo); wb < B; wb += kThreads) {
+        const int nw = B - wb < kThreads ? B - wb : kThreads;
+        load_window(offsets, wb, nw, s_off);
+        int nf = 0;  // frames of the window that start before hi
+        while (nf < nw && (long long)s_off[nf] < hi) ++nf;
+        for (int j = nf - 1; j >= 0; --j) {
+            const long long f0 = s_off[j], f1 = s_off[j + 1];
+            if (f1 < f0) continue;  // reported by the statistics kernel
+            const long long s0 = f0 > lo ? f0 : lo, s1 = f1 < hi ? f1 : hi;
+            if (s0 < s1) segment(wb + j, f0, f1, s0, s1);
+        }
+        if (nf < nw || (long long)s_off[nw] >= hi) break;
     }
 }
 
@@ -524,9 +623,9 @@ template <typename T, int VEC, int GPC>
 hc_status launch_fast(const DeviceCtx* ctx, const void* x, const int32_t* offsets, int B,
                       long long capacity, int C, int G, float eps, const float* gamma,
                       const float* beta, int act, void* y, cudaStream_t s) {
-    // ranges of at least ~64 rows; at most 3 CTAs per SM (the kernels' bound)
+    // ranges of at least ~64 rows; 2 CTAs per SM at most (the kernels' bound)
     long long grid = (capacity + 63) / 64;
-    const long long cap = (long long)ctx->num_sms * 3;
+    const long long cap = (long long)ctx->num_sms * 2;
     if (grid > cap) grid = cap;
     if (grid < 1) grid = 1;
     GnPart* part = (GnPart*)stream_workspace(s, sizeof(GnPart) * (size_t)(B + grid) * G);
@@ -549,9 +648,20 @@ hc_status launch_typed(const DeviceCtx* ctx, const void* x, const int32_t* offse
     const uintptr_t al = (uintptr_t)x | (uintptr_t)y;
     const bool aligned = C % kVec == 0 && al % 16 == 0;
     const int cpr = C / kVec;
-    // HC_GN_SLICE forces the general path (for testing it on every layout)
+    // Small frames: when the average frame's group slice fits the per-thread
+    // register cache of the per-(frame, group) kernel and there are enough
+    // (frame, group) blocks to fill the GPU, that single launch (one read,
+    // one write, no workspace) beats the two latency-bound row-range launches.
+    const long long avg_chunks = (capacity + B - 1) / B * (long long)(cpg / kVec);
+    const bool small_frames = cpg % kVec == 0 && aligned &&
+                              avg_chunks <= (long long)kThreads * kBatch &&
+                              (long long)B * G >= ctx->num_sms;
+    // HC_GN_SLICE forces the per-(frame, group) kernel, HC_GN_ROWS the
+    // row-range kernels where the layout allows (to test both on any shape)
+    const bool force_slice = getenv("HC_GN_SLICE") != nullptr;
+    const bool force_rows = getenv("HC_GN_ROWS") != nullptr;
     const bool fast_rows = aligned && cpr >= 1 && cpr <= kThreads && (cpr & (cpr - 1)) == 0 &&
-                           G <= kMaxGroupsFast && getenv("HC_GN_SLICE") == nullptr;
+                           G <= kMaxGroupsFast && !force_slice && (force_rows || !small_frames);
     if (fast_rows && cpg % kVec == 0)
         return launch_fast<T, kVec, 1>(ctx, x, offsets, B, capacity, C, G, eps, gamma, beta, act,
                                        y, s);

@@ -434,9 +434,13 @@ def _as_f32(a):
 @pytest.mark.parametrize("C,G", [(8, 1), (64, 4), (64, 8), (128, 32), (128, 64), (128, 128),
                                  (256, 16), (1024, 512), (42, 6), (48, 3)])
 @pytest.mark.parametrize("affine,act", [(False, 0), (True, 1), (True, 2)])
-def test_group_norm(C, G, affine, act, dtype):
+@pytest.mark.parametrize("path", ["auto", "rows"])
+def test_group_norm(C, G, affine, act, dtype, path, monkeypatch):
     """Frames of 0, 1, a few, a tile-ish and a large number of rows; rows
-    after the last frame stay untouched."""
+    after the last frame stay untouched. 'rows' forces the row-range kernels
+    wherever the layout allows them."""
+    if path == "rows":
+        monkeypatch.setenv("HC_GN_ROWS", "1")
     rng = np.random.default_rng(C * 100 + G * 7 + act)
     sizes = [0, 1, 3, 0, 130, 517, 2900, 64]
     x, offs = _gn_case(rng, sizes, C, dtype)
@@ -457,8 +461,7 @@ def test_group_norm_paths_and_frame_shapes(C, G, path, dtype, monkeypatch):
     on many tiny frames (a row range holds dozens of frame segments) and on
     one frame spread over hundreds of row ranges (its partials are merged by
     a warp)."""
-    if path == "slice":
-        monkeypatch.setenv("HC_GN_SLICE", "1")
+    monkeypatch.setenv("HC_GN_SLICE" if path == "slice" else "HC_GN_ROWS", "1")
     rng = np.random.default_rng(C + G)
     tiny = [int(v) for v in rng.integers(0, 6, size=300)]
     big = [40000 if C <= 128 else 3000]
@@ -495,8 +498,7 @@ def test_group_norm_in_place_and_misaligned(dtype):
 def test_group_norm_constant_group_and_eps(path, monkeypatch):
     """A group of equal values normalises to exactly 0 (then + beta); eps
     from 0 to large enters as 1/sqrt(var + eps)."""
-    if path == "slice":
-        monkeypatch.setenv("HC_GN_SLICE", "1")
+    monkeypatch.setenv("HC_GN_SLICE" if path == "slice" else "HC_GN_ROWS", "1")
     C, G = 32, 4
     offs = np.array([0, 200, 201], dtype=np.int32)
     x = np.full((201, C), 100.25, dtype=np.float32)
@@ -523,17 +525,23 @@ def test_group_norm_on_compacted_layer_output():
     beta = (0.1 * rng.standard_normal(128)).astype(np.float32)
     xt = to_torch(x)
     y = torch.empty_like(xt)
-    hc.hc_sparse_group_norm_fwd(xt, offs, 8, 1e-5, to_torch(gamma), to_torch(beta),
-                                hc.HC_ACT_ELU, y)
-    assert hc.hc_get_device_status() == hc.HC_OK
     y_pre, _ = oracle.sparse_group_norm(x, to_numpy(offs), 8, 1e-5, gamma, beta, oracle.ACT_ELU)
-    check_close(to_numpy(y), y_pre, "group norm full size")
+    for path in ("auto", "rows"):
+        if path == "rows":
+            os.environ["HC_GN_ROWS"] = "1"
+        try:
+            y.fill_(float("nan"))
+            hc.hc_sparse_group_norm_fwd(xt, offs, 8, 1e-5, to_torch(gamma), to_torch(beta),
+                                        hc.HC_ACT_ELU, y)
+            assert hc.hc_get_device_status() == hc.HC_OK
+        finally:
+            os.environ.pop("HC_GN_ROWS", None)
+        check_close(to_numpy(y), y_pre, f"group norm full size ({path})")
 
 
 @pytest.mark.parametrize("path", ["rows", "slice"])
 def test_group_norm_bad_offsets_reported(path, monkeypatch):
-    if path == "slice":
-        monkeypatch.setenv("HC_GN_SLICE", "1")
+    monkeypatch.setenv("HC_GN_SLICE" if path == "slice" else "HC_GN_ROWS", "1")
     x = torch.zeros((10, 16), dtype=torch.float32, device="cuda")
     offs = torch.tensor([0, 4, 12], dtype=torch.int32, device="cuda")  # 12 > capacity
     hc.hc_sparse_group_norm_fwd(x, offs, 4, 1e-5, None, None, 0, x)
