@@ -18,6 +18,11 @@ Functions and the passages they follow:
 * ``sparse_group_norm``    group normalisation over each frame's active rows
                            (Eqs. 7-9)
 * ``scatter_dense``        compact rows back to a dense tensor (inverse of Eq. 2)
+* ``mask_score``           the mask-score update of Eq. 3
+* ``select_topk``          the kappa highest-scoring masks kept at inference
+                           (Sec. 3.1, Sparse Mask Selection)
+* ``kappa_masks``          every kept mask applied to every sample (Eq. 1)
+* ``gather_rows``          the feature matrix S' of Eq. 2
 * ``encoder``              a stack of sparse layers: coordinates fixed once by
                            the mask (Eqs. 5, 6, 10 keep C'), each layer's output
                            stored in the layer dtype before the next reads it
@@ -86,6 +91,14 @@ def _load():
             lib.hco_sparse_group_norm.restype = None
             lib.hco_conv_rulebook.argtypes = [P, P, I64, P, I64, I, I, I64, P]
             lib.hco_conv_rulebook.restype = None
+            lib.hco_mask_score.argtypes = [P, I, I64, I64, I64, P, P, P, P, I]
+            lib.hco_mask_score.restype = None
+            lib.hco_select_topk.argtypes = [P, I64, I64, P]
+            lib.hco_select_topk.restype = None
+            lib.hco_kappa_masks.argtypes = [P, I64, P, I64, I64, P]
+            lib.hco_kappa_masks.restype = None
+            lib.hco_gather_rows.argtypes = [P, I, I64, I, P, I64, I64, P]
+            lib.hco_gather_rows.restype = None
             lib.hco_bf16_round.argtypes = [ctypes.c_double]
             lib.hco_bf16_round.restype = ctypes.c_uint16
             _lib = lib
@@ -273,3 +286,51 @@ def encoder(x_dense, mask, spiral, layers, n_threads=1):
         h = y
         layout = LAYOUT_COMPACT
     return coords, row_of, offsets, n, outs
+
+
+def mask_score(O, alpha, n_threads=1):
+    """Eq. 3 on per-mask outputs O [K, N, D] (float32 or bf16 bits) and
+    scores alpha [K]: returns (alpha_next fp64 [K], sim fp64 [K, K],
+    S fp64 [K, K] with S[i, k] = ||O_i^T O_k||_F^2)."""
+    O = np.ascontiguousarray(O)
+    dt = _dtype_code(O)
+    K, N, D = O.shape
+    a_in = _c(alpha, np.float64)
+    a_out = np.empty(K, dtype=np.float64)
+    sim = np.empty((K, K), dtype=np.float64)
+    S = np.empty((K, K), dtype=np.float64)
+    _load().hco_mask_score(_ptr(O), dt, K, N, D, _ptr(a_in), _ptr(a_out), _ptr(sim), _ptr(S),
+                           n_threads)
+    return a_out, sim, S
+
+
+def select_topk(alpha, kappa):
+    """Indices of the kappa highest fp32 scores, highest first, ties by index."""
+    alpha = _c(alpha, np.float32)
+    sel = np.empty(kappa, dtype=np.int32)
+    _load().hco_select_topk(_ptr(alpha), alpha.shape[0], kappa, _ptr(sel))
+    return sel
+
+
+def kappa_masks(masks, selected, B):
+    """[B * kappa, V] frame masks: frame b * kappa + j = masks[selected[j]]."""
+    masks = _c(masks, np.uint8)
+    selected = _c(selected, np.int32)
+    K, V = masks.shape
+    kappa = selected.shape[0]
+    out = np.empty((B * kappa, V), dtype=np.uint8)
+    _load().hco_kappa_masks(_ptr(masks), V, _ptr(selected), kappa, B, _ptr(out))
+    return out
+
+
+def gather_rows(x, coords, frames_per_sample=1):
+    """S' of Eq. 2: rows of the dense input x [B_in, V, C] at coords (f, v),
+    frame f reading sample f // frames_per_sample."""
+    x = np.ascontiguousarray(x)
+    coords = _c(coords, np.int32)
+    _, V, C = x.shape
+    n = coords.shape[0]
+    y = np.empty((n, C), dtype=x.dtype)
+    _load().hco_gather_rows(_ptr(x), x.dtype.itemsize, V, C, _ptr(coords), n,
+                            frames_per_sample, _ptr(y))
+    return y

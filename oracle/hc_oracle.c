@@ -27,12 +27,22 @@
  *                           Eqs. 7-9 (G = 1: layer normalisation)
  *   hco_scatter_dense       inverse of the decomposition: compact rows back
  *                           into a dense [B, V, C] tensor
+ *   hco_mask_score          the mask-score update of Eq. 3 (Gram matrices of
+ *                           the per-mask outputs, Frobenius norms)
+ *   hco_select_topk         the kappa masks with the highest score kept at
+ *                           inference (Sec. 3.1, "Sparse Mask Selection")
+ *   hco_kappa_masks         the kept masks applied to every sample: kappa
+ *                           frames per sample (Eq. 1 per kept mask)
+ *   hco_gather_rows         the feature matrix S' of Eq. 2: the input rows
+ *                           at the active coordinates
  *   hco_bf16_round          fp64 -> bf16 rounding (storage format)
  *
- * Parity status: compaction, conv, dense conv, linear and scatter are pinned
- * by tests against library routines (numpy.nonzero, numpy matmul), closed
- * forms, hand-worked cases and brute force (tests/test_oracle_pins.py). The
- * paper prints no numeric worked example for any operator.
+ * Parity status: compaction, conv, dense conv, linear, group norm, scatter,
+ * the mask score, top-kappa selection, kappa masks and the row gather are
+ * pinned by tests against library routines (numpy.nonzero, numpy matmul,
+ * numpy argsort), closed forms, invariances, hand-worked cases and brute
+ * force (tests/test_oracle_pins.py). The paper prints no numeric worked
+ * example for any operator.
  */
 #include <math.h>
 #include <stdint.h>
@@ -327,5 +337,102 @@ void hco_scatter_dense(const void* y, int elem_bytes, const int32_t* coords, int
     for (int64_t n = 0; n < count; ++n) {
         int64_t b = coords[2 * n + 0], v = coords[2 * n + 1];
         memcpy(dst + (b * V + v) * row_bytes, src + n * row_bytes, (size_t)row_bytes);
+    }
+}
+
+/* ---------------------------------------------------------- mask score */
+
+/* Eq. 3: with O_k the [N, D] output for mask k (row-major, masks stacked
+ * as [K, N, D]), and ||.||_F the Frobenius norm,
+ *     S[i][k]   = || O_i^T O_k ||_F^2            (D x D Gram of the pair)
+ *     sim[i][k] = S[i][k] / (|| O_k^T O_k ||_F || O_i^T O_i ||_F)
+ *               = S[i][k] / sqrt(S[i][i] * S[k][k])
+ *     alpha_out[k] = alpha_in[k] + 1/(K-1) * sum over i != k of (1 - sim[i][k])
+ * Every Gram entry is a plain fp64 sum over the N rows, squared and summed
+ * over the D x D entries. Readings where the equation is silent: a mask
+ * whose output is all zero has no defined similarity, and its terms count
+ * as 1 - 0 (it shares nothing); with K = 1 the sum is empty and alpha is
+ * unchanged. S and sim are [K, K] (either may be NULL). */
+void hco_mask_score(const void* O, int dtype, int64_t K, int64_t N, int64_t D,
+                    const double* alpha_in, double* alpha_out, double* sim_out, double* S_out,
+                    int n_threads) {
+    double* S = (double*)calloc((size_t)(K * K), sizeof(double));
+    int64_t n_pairs = K * (K + 1) / 2;
+    #pragma omp parallel for schedule(dynamic) num_threads(n_threads)
+    for (int64_t p = 0; p < n_pairs; ++p) {
+        /* pair p -> (i, k), i <= k */
+        int64_t i = 0, rem = p;
+        while (rem >= K - i) {
+            rem -= K - i;
+            ++i;
+        }
+        int64_t k = i + rem;
+        double acc = 0.0;
+        for (int64_t d = 0; d < D; ++d)
+            for (int64_t e = 0; e < D; ++e) {
+                double g = 0.0;
+                for (int64_t n = 0; n < N; ++n)
+                    g += load_elem(O, dtype, (i * N + n) * D + d) *
+                         load_elem(O, dtype, (k * N + n) * D + e);
+                acc += g * g;
+            }
+        S[i * K + k] = acc;
+        S[k * K + i] = acc;
+    }
+    for (int64_t k = 0; k < K; ++k) {
+        double sum = 0.0;
+        for (int64_t i = 0; i < K; ++i) {
+            double den = sqrt(S[i * K + i]) * sqrt(S[k * K + k]);
+            double sim = den > 0.0 ? S[i * K + k] / den : 0.0;
+            if (sim_out) sim_out[i * K + k] = sim;
+            if (i != k) sum += 1.0 - sim;
+        }
+        alpha_out[k] = K > 1 ? alpha_in[k] + sum / (double)(K - 1) : alpha_in[k];
+    }
+    if (S_out) memcpy(S_out, S, sizeof(double) * (size_t)(K * K));
+    free(S);
+}
+
+/* Sec. 3.1, Sparse Mask Selection: at inference only the kappa masks with
+ * the highest score are kept. Selected in order of decreasing score; equal
+ * scores are taken lowest index first. The scores are fp32 (as stored). */
+void hco_select_topk(const float* alpha, int64_t K, int64_t kappa, int32_t* selected) {
+    unsigned char* taken = (unsigned char*)calloc((size_t)K, 1);
+    for (int64_t j = 0; j < kappa; ++j) {
+        int64_t best = -1;
+        for (int64_t k = 0; k < K; ++k) {
+            if (taken[k]) continue;
+            if (best < 0 || alpha[k] > alpha[best]) best = k;
+        }
+        taken[best] = 1;
+        selected[j] = (int32_t)best;
+    }
+    free(taken);
+}
+
+/* Eq. 1 with every kept mask applied to every sample independently
+ * (Sec. 3.1): frame f = b * kappa + j is sample b under kept mask
+ * selected[j], so out[f][v] = masks[selected[j]][v]. masks is [K, V]. */
+void hco_kappa_masks(const uint8_t* masks, int64_t V, const int32_t* selected, int64_t kappa,
+                     int64_t B, uint8_t* out) {
+    for (int64_t b = 0; b < B; ++b)
+        for (int64_t j = 0; j < kappa; ++j)
+            memcpy(out + (b * kappa + j) * V, masks + (int64_t)selected[j] * V, (size_t)V);
+}
+
+/* Eq. 2, the feature matrix S': row n holds the input features at the n-th
+ * active coordinate (f, v). The input is the dense [B_in, V, C] tensor of
+ * samples; frame f reads sample f / frames_per_sample (frames_per_sample =
+ * kappa when every sample was masked by kappa kept masks, else 1). Rows are
+ * copied bit for bit. */
+void hco_gather_rows(const void* x, int elem_bytes, int64_t V, int C, const int32_t* coords,
+                     int64_t count, int64_t frames_per_sample, void* y) {
+    const unsigned char* src = (const unsigned char*)x;
+    unsigned char* dst = (unsigned char*)y;
+    int64_t row_bytes = (int64_t)C * elem_bytes;
+    for (int64_t n = 0; n < count; ++n) {
+        int64_t f = coords[2 * n + 0], v = coords[2 * n + 1];
+        memcpy(dst + n * row_bytes, src + ((f / frames_per_sample) * V + v) * row_bytes,
+               (size_t)row_bytes);
     }
 }

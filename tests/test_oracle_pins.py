@@ -360,6 +360,15 @@ MUTANTS = {
                                         "                    double d = load_elem(x, dtype, i * C + c);"),
     "group norm counts rows only": ("            double n = (double)(r1 - r0) * cpg;",
                                     "            double n = (double)(r1 - r0);"),
+    "mask score without the norms' square roots": ("            double den = sqrt(S[i * K + i]) * sqrt(S[k * K + k]);",
+                                                   "            double den = S[i * K + i] * S[k * K + k];"),
+    "mask score averaged over K": ("        alpha_out[k] = K > 1 ? alpha_in[k] + sum / (double)(K - 1) : alpha_in[k];",
+                                   "        alpha_out[k] = K > 1 ? alpha_in[k] + sum / (double)K : alpha_in[k];"),
+    "mask score Gram index": ("                         load_elem(O, dtype, (k * N + n) * D + e);",
+                              "                         load_elem(O, dtype, (k * N + n) * D + d);"),
+    "mask score numerator not squared": ("                acc += g * g;", "                acc += fabs(g);"),
+    "top-kappa ties by highest index": ("            if (best < 0 || alpha[k] > alpha[best]) best = k;",
+                                        "            if (best < 0 || alpha[k] >= alpha[best]) best = k;"),
     "centre tap dropped": ("for (int l = 0; l < L; ++l) {\n            int64_t u = spiral[v * L + l];\n            if (u < 0) continue; /* no neighbour in this slot */",
                            "for (int l = 1; l < L; ++l) {\n            int64_t u = spiral[v * L + l];\n            if (u < 0) continue; /* no neighbour in this slot */"),
 }
@@ -383,14 +392,16 @@ def test_planted_mistake_is_caught(name, tmp_path, monkeypatch):
     lib = ctypes.CDLL(str(so))
     for fn in ("hco_mask_compact", "hco_sparse_spiral_conv", "hco_dense_spiral_conv",
                "hco_sparse_linear", "hco_scatter_dense", "hco_bf16_round", "hco_conv_rulebook",
-               "hco_sparse_group_norm"):
+               "hco_sparse_group_norm", "hco_mask_score", "hco_select_topk", "hco_kappa_masks",
+               "hco_gather_rows"):
         getattr(lib, fn).argtypes = getattr(good, fn).argtypes
         getattr(lib, fn).restype = getattr(good, fn).restype
     monkeypatch.setattr(oracle, "_lib", lib)
     checks = [check_golden_cases, check_conv_vs_gather_matmul, check_group_norm_golden,
               check_group_norm_vs_numpy,
               lambda: check_compact_vs_nonzero(inputs.uniform_mask(np.random.default_rng(1), 5, 20, 0.3)),
-              check_bf16_round]
+              check_bf16_round, check_mask_score_golden, check_mask_score_vs_numpy,
+              check_mask_score_d1_is_squared_cosine, check_select_topk_vs_argsort]
     caught = 0
     for chk in checks:
         try:
@@ -466,3 +477,128 @@ def test_group_norm_is_layer_norm_at_g1_and_ignores_inactive_rows():
     dense[coords[:, 1]] = x
     yd = (dense - dense.mean()) / dense.std()
     assert not np.allclose(yd[coords[:, 1]], y)
+
+
+# ------------------------------------------------------------ mask score (Eq. 3)
+
+def check_mask_score_golden():
+    g = json.load(open(os.path.join(os.path.dirname(__file__), "golden", "mask_score.json")))
+    c0, c1, c2, c3 = g["cases"]
+    a, sim, _ = oracle.mask_score(np.array(c0["O"], np.float32), c0["alpha"])
+    np.testing.assert_allclose(a, c0["alpha_next"], rtol=0, atol=1e-15)
+    assert abs(sim[0, 1] - c0["sim01"]) < 1e-15
+    a, sim, _ = oracle.mask_score(np.array(c1["O"], np.float32), c1["alpha"])
+    r = 1 - 1 / math.sqrt(2)
+    np.testing.assert_allclose(a, [r / 2, r / 2, r], rtol=0, atol=1e-15)
+    np.testing.assert_allclose(sim, [[1, 1, 1 / math.sqrt(2)], [1, 1, 1 / math.sqrt(2)],
+                                     [1 / math.sqrt(2), 1 / math.sqrt(2), 1]], atol=1e-15)
+    a, _, _ = oracle.mask_score(np.array(c2["O"], np.float32), c2["alpha"])
+    np.testing.assert_array_equal(a, c2["alpha_next"])
+    a, _, _ = oracle.mask_score(np.array(c3["O"], np.float32), c3["alpha"])
+    np.testing.assert_array_equal(a, c3["alpha_next"])
+
+
+def test_mask_score_golden():
+    check_mask_score_golden()
+
+
+def check_mask_score_vs_numpy(seed=41, dtype="f32"):
+    """The Gram matrices from numpy's matmul (fp64), their squared Frobenius
+    norms and the update written out with numpy."""
+    rng = np.random.default_rng(seed)
+    K, N, D = 4, 97, 5
+    O = (rng.standard_normal((K, N, D)) + 0.3).astype(np.float32)
+    if dtype == "bf16":
+        O = inputs.to_bf16_bits(O)
+        Od = inputs.bf16_bits_to_f32(O).astype(np.float64)
+    else:
+        Od = O.astype(np.float64)
+    alpha = rng.standard_normal(K)
+    a, sim, S = oracle.mask_score(O, alpha, n_threads=2)
+    S_ref = np.array([[np.sum((Od[i].T @ Od[k]) ** 2) for k in range(K)] for i in range(K)])
+    np.testing.assert_allclose(S, S_ref, rtol=1e-12)
+    nrm = np.sqrt(np.diag(S_ref))
+    sim_ref = S_ref / np.outer(nrm, nrm)
+    a_ref = alpha + ((1 - sim_ref).sum(axis=0) - (1 - np.diag(sim_ref))) / (K - 1)
+    np.testing.assert_allclose(sim, sim_ref, rtol=1e-12)
+    np.testing.assert_allclose(a, a_ref, rtol=1e-12, atol=1e-12)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_mask_score_vs_numpy(dtype):
+    check_mask_score_vs_numpy(dtype=dtype)
+
+
+def check_mask_score_d1_is_squared_cosine(seed=42):
+    """D = 1: O_i^T O_k is the dot product of two vectors, so the similarity
+    is their squared cosine."""
+    rng = np.random.default_rng(seed)
+    v = rng.standard_normal((3, 40, 1)).astype(np.float32)
+    _, sim, _ = oracle.mask_score(v, np.zeros(3))
+    u = v[:, :, 0].astype(np.float64)
+    cos = (u @ u.T) / np.outer(np.linalg.norm(u, axis=1), np.linalg.norm(u, axis=1))
+    np.testing.assert_allclose(sim, cos ** 2, rtol=1e-12)
+
+
+def test_mask_score_d1_is_squared_cosine():
+    check_mask_score_d1_is_squared_cosine()
+
+
+def test_mask_score_invariances():
+    """The score compares feature distributions, not bases or scales: it is
+    unchanged by scaling a mask's output, by an orthogonal change of feature
+    basis per mask (Frobenius norms are invariant under both sides'
+    orthogonal factors), and by one permutation of the rows of all masks.
+    Identical outputs are fully similar (alpha unchanged); outputs on
+    disjoint rows share nothing (alpha + 1)."""
+    rng = np.random.default_rng(43)
+    K, N, D = 3, 60, 4
+    O = rng.standard_normal((K, N, D))
+    alpha = rng.standard_normal(K)
+    a0, _, _ = oracle.mask_score(O.astype(np.float32), alpha)
+    O2 = O.copy()
+    O2[1] *= -2.5
+    for k in range(K):
+        q, _ = np.linalg.qr(rng.standard_normal((D, D)))
+        O2[k] = O2[k] @ q
+    O2 = O2[:, rng.permutation(N)]
+    a1, _, _ = oracle.mask_score(O2.astype(np.float32), alpha)
+    np.testing.assert_allclose(a1, a0, rtol=1e-5, atol=1e-5)  # fp32 storage of the rotated data
+    same = np.repeat(O[:1], K, axis=0).astype(np.float32)
+    a2, _, _ = oracle.mask_score(same, alpha)
+    np.testing.assert_allclose(a2, alpha, atol=1e-12)
+    disj = np.zeros((K, N, D), np.float32)
+    for k in range(K):
+        disj[k, k * 20:(k + 1) * 20] = O[k, k * 20:(k + 1) * 20]
+    a3, _, _ = oracle.mask_score(disj, alpha)
+    np.testing.assert_allclose(a3, alpha + 1, atol=1e-12)
+
+
+def check_select_topk_vs_argsort(seed=44):
+    """Top-kappa against numpy's stable argsort of -alpha (ties by index)."""
+    rng = np.random.default_rng(seed)
+    for K, kappa in ((10, 3), (50, 10), (7, 7), (1, 1)):
+        alpha = rng.integers(-3, 4, size=K).astype(np.float32) * 0.5  # many ties
+        np.testing.assert_array_equal(oracle.select_topk(alpha, kappa),
+                                      np.argsort(-alpha, kind="stable")[:kappa])
+
+
+def test_select_topk_vs_argsort():
+    check_select_topk_vs_argsort()
+
+
+def test_kappa_masks_and_gather_rows_vs_numpy():
+    """Kept masks applied to every sample (frame b * kappa + j), and the rows
+    S' of Eq. 2 gathered from the samples, against numpy indexing."""
+    rng = np.random.default_rng(45)
+    K, V, B, kappa, C = 6, 40, 5, 3, 7
+    masks = inputs.uniform_mask(rng, K, V, 0.2)
+    sel = np.array([4, 0, 2], np.int32)
+    fm = oracle.kappa_masks(masks, sel, B)
+    np.testing.assert_array_equal(fm, np.tile(masks[sel], (B, 1)))
+    coords, _, _, n = oracle.mask_compact(fm)
+    x = rng.standard_normal((B, V, C)).astype(np.float32)
+    y = oracle.gather_rows(x, coords, kappa)
+    np.testing.assert_array_equal(y, x[coords[:, 0] // kappa, coords[:, 1]])
+    np.testing.assert_array_equal(oracle.gather_rows(x, oracle.mask_compact(masks[:B])[0]),
+                                  x[np.nonzero(masks[:B])])
