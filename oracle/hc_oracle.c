@@ -395,14 +395,21 @@ void hco_mask_score(const void* O, int dtype, int64_t K, int64_t N, int64_t D,
 
 /* Sec. 3.1, Sparse Mask Selection: at inference only the kappa masks with
  * the highest score are kept. Selected in order of decreasing score; equal
- * scores are taken lowest index first. The scores are fp32 (as stored). */
+ * scores are taken lowest index first. The scores are fp32 (as stored). The
+ * paper does not consider undefined scores: a NaN ranks below every number
+ * (NaNs among themselves by index). */
+static int score_above(float a, float b) {
+    if (isnan(a)) return 0;
+    return isnan(b) || a > b;
+}
+
 void hco_select_topk(const float* alpha, int64_t K, int64_t kappa, int32_t* selected) {
     unsigned char* taken = (unsigned char*)calloc((size_t)K, 1);
     for (int64_t j = 0; j < kappa; ++j) {
         int64_t best = -1;
         for (int64_t k = 0; k < K; ++k) {
             if (taken[k]) continue;
-            if (best < 0 || alpha[k] > alpha[best]) best = k;
+            if (best < 0 || score_above(alpha[k], alpha[best])) best = k;
         }
         taken[best] = 1;
         selected[j] = (int32_t)best;

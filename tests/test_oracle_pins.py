@@ -367,8 +367,7 @@ MUTANTS = {
     "mask score Gram index": ("                         load_elem(O, dtype, (k * N + n) * D + e);",
                               "                         load_elem(O, dtype, (k * N + n) * D + d);"),
     "mask score numerator not squared": ("                acc += g * g;", "                acc += fabs(g);"),
-    "top-kappa ties by highest index": ("            if (best < 0 || alpha[k] > alpha[best]) best = k;",
-                                        "            if (best < 0 || alpha[k] >= alpha[best]) best = k;"),
+    "top-kappa ties by highest index": ("    return isnan(b) || a > b;", "    return isnan(b) || a >= b;"),
     "centre tap dropped": ("for (int l = 0; l < L; ++l) {\n            int64_t u = spiral[v * L + l];\n            if (u < 0) continue; /* no neighbour in this slot */",
                            "for (int l = 1; l < L; ++l) {\n            int64_t u = spiral[v * L + l];\n            if (u < 0) continue; /* no neighbour in this slot */"),
 }
@@ -585,6 +584,15 @@ def check_select_topk_vs_argsort(seed=44):
 
 def test_select_topk_vs_argsort():
     check_select_topk_vs_argsort()
+
+
+def test_select_topk_nan_ranks_last():
+    """NaN scores rank below every number (numpy's argsort also puts NaN
+    last); among themselves by index."""
+    alpha = np.array([np.nan, 1.0, -np.inf, np.nan, 3.0, 1.0], np.float32)
+    np.testing.assert_array_equal(oracle.select_topk(alpha, 6), [4, 1, 5, 2, 0, 3])
+    np.testing.assert_array_equal(oracle.select_topk(alpha, 6),
+                                  np.argsort(-alpha, kind="stable"))
 
 
 def test_kappa_masks_and_gather_rows_vs_numpy():
