@@ -227,6 +227,62 @@ hc_status hc_sparse_group_norm_fwd(const void* x, hc_dtype dt, const int32_t* ba
                                    const float* beta, hc_act act, void* y, hc_stream_t stream);
 
 /*
+ * hc_mask_score_update -- the mask-score update of Eq. 3 (Sec. 3.1, Sparse
+ * Mask Selection). O holds the outputs of K masks, [K, N, D] row-major (mask
+ * k's N rows of D features). With S[i][k] = || O_i^T O_k ||_F^2:
+ *   sim[i][k]    = S[i][k] / (|| O_k^T O_k ||_F * || O_i^T O_i ||_F)
+ *   alpha_out[k] = alpha_in[k] + 1/(K-1) * sum over i != k of (1 - sim[i][k])
+ * Readings: a mask whose output is all zero has similarity 0 to every mask;
+ * with K = 1 alpha is copied unchanged.
+ *   O          [K, N, D] of dtype dt (bf16: tensor cores, fp32 accumulation;
+ *              fp32: CUDA cores, fp32 accumulation)
+ *   alpha_in, alpha_out  [K] fp32 on the device; may be the same buffer
+ *   sim        [K, K] fp32 or NULL
+ * K*D at most HC_MASK_SCORE_MAX_FEATURES (else HC_ERR_UNSUPPORTED). Uses the
+ * library's per-stream workspace: 64 KiB per work item (upper-triangle
+ * 128 x 128 tiles of the [K*D]^2 Gram matrix times row splits, about the
+ * SM count), plus N * K*D (rounded to 128) bf16 when D is not a multiple of 8.
+ */
+#define HC_MASK_SCORE_MAX_FEATURES 8192
+hc_status hc_mask_score_update(const void* O, hc_dtype dt, int K, int N, int D,
+                               const float* alpha_in, float* alpha_out, float* sim,
+                               hc_stream_t stream);
+
+/*
+ * hc_mask_select_topk -- the kappa masks kept at inference (Sec. 3.1, Sparse
+ * Mask Selection): indices of the kappa highest scores of alpha [K] (fp32,
+ * device), highest first; equal scores lowest index first; a NaN score ranks
+ * below every number. selected: [kappa] int32 on the device.
+ * K at most HC_TOPK_MAX_MASKS.
+ */
+#define HC_TOPK_MAX_MASKS 32768
+hc_status hc_mask_select_topk(const float* alpha, int K, int kappa, int32_t* selected,
+                              hc_stream_t stream);
+
+/*
+ * hc_kappa_masks -- every kept mask applied to every sample (Eq. 1 per kept
+ * mask, Sec. 3.1): out [B*kappa, V] with frame b*kappa + j equal to
+ * masks[selected[j]] ([K, V] uint8). The result feeds hc_mask_compact; a
+ * selected index outside [0, K) gives an all-zero frame and
+ * HC_ERR_INVALID_INDEX.
+ */
+hc_status hc_kappa_masks(const uint8_t* masks, int K, int V, const int32_t* selected, int kappa,
+                         int B, uint8_t* out, hc_stream_t stream);
+
+/*
+ * hc_gather_rows -- the feature matrix S' of Eq. 2: y[n] = x[f / fps, v] for
+ * the n-th active coordinate (f, v) = coords[n], n < *count, where x is the
+ * dense [B_in, V, C] input of dtype dt and fps = frames_per_sample (kappa
+ * after hc_kappa_masks, else 1). Rows are copied bit for bit; y is
+ * [capacity, C]. A coordinate outside the input is reported
+ * (HC_ERR_INVALID_INDEX) and its row left untouched; *count above capacity
+ * is clamped (HC_ERR_CAPACITY).
+ */
+hc_status hc_gather_rows(const void* x, hc_dtype dt, int B_in, int V, int C, const int32_t* coords,
+                         const int32_t* count, int capacity, int frames_per_sample, void* y,
+                         hc_stream_t stream);
+
+/*
  * hc_scatter_dense -- inverse of the decomposition (Eq. 2): compact rows back
  * into a dense [B, V, C] tensor.
  *   zero_fill == 0: out[coords[n]] = y[n] for n < N'; other rows untouched.

@@ -354,6 +354,74 @@ hc_status hc_sparse_group_norm_fwd(const void* x, hc_dtype dt, const int32_t* ba
                              (int)act, y, (cudaStream_t)stream);
 }
 
+hc_status hc_mask_score_update(const void* O, hc_dtype dt, int K, int N, int D,
+                               const float* alpha_in, float* alpha_out, float* sim,
+                               hc_stream_t stream) {
+    const char* fn = "hc_mask_score_update";
+    t_last_error[0] = 0;
+    HC_REQUIRE(dt == HC_F32 || dt == HC_BF16, "%s: unknown dtype %d", fn, (int)dt);
+    HC_REQUIRE(K >= 1 && D >= 1 && N >= 0, "%s: K=%d D=%d must be >= 1, N=%d >= 0", fn, K, D, N);
+    if ((long long)K * D > HC_MASK_SCORE_MAX_FEATURES) {
+        set_error("%s: K*D=%lld above the supported %d", fn, (long long)K * D,
+                  HC_MASK_SCORE_MAX_FEATURES);
+        return HC_ERR_UNSUPPORTED;
+    }
+    HC_REQUIRE(alpha_in && alpha_out, "%s: alpha_in and alpha_out are required", fn);
+    HC_REQUIRE(N == 0 || O != nullptr, "%s: O is NULL", fn);
+    HC_REQUIRE(!misaligned(O, dt == HC_F32 ? 4 : 2), "%s: misaligned O", fn);
+    const DeviceCtx* ctx = device_ctx();
+    if (!ctx) return HC_ERR_CUDA;
+    return launch_mask_score(ctx, O, dt, K, N, D, alpha_in, alpha_out, sim, (cudaStream_t)stream);
+}
+
+hc_status hc_mask_select_topk(const float* alpha, int K, int kappa, int32_t* selected,
+                              hc_stream_t stream) {
+    const char* fn = "hc_mask_select_topk";
+    t_last_error[0] = 0;
+    HC_REQUIRE(K >= 1 && K <= HC_TOPK_MAX_MASKS, "%s: K=%d must be in [1, %d]", fn, K,
+               HC_TOPK_MAX_MASKS);
+    HC_REQUIRE(kappa >= 0 && kappa <= K, "%s: kappa=%d must be in [0, K=%d]", fn, kappa, K);
+    HC_REQUIRE(alpha && selected, "%s: alpha and selected are required", fn);
+    if (kappa == 0) return HC_OK;
+    const DeviceCtx* ctx = device_ctx();
+    if (!ctx) return HC_ERR_CUDA;
+    return launch_topk(ctx, alpha, K, kappa, selected, (cudaStream_t)stream);
+}
+
+hc_status hc_kappa_masks(const uint8_t* masks, int K, int V, const int32_t* selected, int kappa,
+                         int B, uint8_t* out, hc_stream_t stream) {
+    const char* fn = "hc_kappa_masks";
+    t_last_error[0] = 0;
+    HC_REQUIRE(K >= 1 && V >= 0 && kappa >= 0 && B >= 0, "%s: K=%d V=%d kappa=%d B=%d", fn, K,
+               V, kappa, B);
+    HC_REQUIRE((long long)B * kappa * V < (1ll << 31), "%s: B*kappa*V must be < 2^31", fn);
+    if ((long long)B * kappa * V == 0) return HC_OK;
+    HC_REQUIRE(masks && selected && out, "%s: masks, selected and out are required", fn);
+    const DeviceCtx* ctx = device_ctx();
+    if (!ctx) return HC_ERR_CUDA;
+    return launch_kappa_masks(ctx, masks, K, V, selected, kappa, B, out, (cudaStream_t)stream);
+}
+
+hc_status hc_gather_rows(const void* x, hc_dtype dt, int B_in, int V, int C, const int32_t* coords,
+                         const int32_t* count, int capacity, int frames_per_sample, void* y,
+                         hc_stream_t stream) {
+    const char* fn = "hc_gather_rows";
+    t_last_error[0] = 0;
+    HC_REQUIRE(dt == HC_F32 || dt == HC_BF16, "%s: unknown dtype %d", fn, (int)dt);
+    HC_REQUIRE(B_in >= 0 && V >= 0 && C >= 1 && capacity >= 0 && frames_per_sample >= 1,
+               "%s: B_in=%d V=%d C=%d capacity=%d frames_per_sample=%d", fn, B_in, V, C, capacity,
+               frames_per_sample);
+    HC_REQUIRE(count != nullptr, "%s: count is NULL", fn);
+    if (capacity == 0) return HC_OK;
+    HC_REQUIRE(x && coords && y, "%s: x, coords and y are required", fn);
+    const int eb = dt == HC_F32 ? 4 : 2;
+    HC_REQUIRE(!misaligned(x, eb) && !misaligned(y, eb), "%s: misaligned x/y", fn);
+    const DeviceCtx* ctx = device_ctx();
+    if (!ctx) return HC_ERR_CUDA;
+    return launch_gather_rows(ctx, x, eb, B_in, V, C, coords, count, capacity, frames_per_sample,
+                              y, (cudaStream_t)stream);
+}
+
 hc_status hc_scatter_dense(const void* y, hc_dtype dt, const int32_t* coords,
                            const int32_t* row_of, const int32_t* count, int B, int V, int C,
                            int zero_fill, void* out, hc_stream_t stream) {

@@ -85,6 +85,17 @@ hc_status launch_group_norm(const DeviceCtx* ctx, const void* x, hc_dtype dt,
                             const int32_t* offsets, int B, long long capacity, int C, int G,
                             float eps, const float* gamma, const float* beta, int act, void* y,
                             cudaStream_t s);
+hc_status launch_mask_score(const DeviceCtx* ctx, const void* O, hc_dtype dt, int K, long long N,
+                            int D, const float* alpha_in, float* alpha_out, float* sim,
+                            cudaStream_t s);
+hc_status launch_topk(const DeviceCtx* ctx, const float* alpha, int K, int kappa, int32_t* selected,
+                      cudaStream_t s);
+hc_status launch_kappa_masks(const DeviceCtx* ctx, const uint8_t* masks, int K, int V,
+                             const int32_t* selected, int kappa, int B, uint8_t* out,
+                             cudaStream_t s);
+hc_status launch_gather_rows(const DeviceCtx* ctx, const void* x, int elem_bytes, int B_in, int V,
+                             int C, const int32_t* coords, const int32_t* count, int capacity,
+                             int frames_per_sample, void* y, cudaStream_t s);
 hc_status launch_scatter(const DeviceCtx* ctx, const void* y, int elem_bytes, const int32_t* coords,
                          const int32_t* row_of, const int32_t* count, int B, int V, int C,
                          int zero_fill, void* out, cudaStream_t s);

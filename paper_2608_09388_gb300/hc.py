@@ -30,7 +30,8 @@ STATUS_NAMES = {0: "HC_OK", 1: "HC_ERR_INVALID_ARG", 2: "HC_ERR_UNSUPPORTED",
 # Exported symbols, as declared in include/hc.h.
 EXPORTS = ("hc_mask_compact", "hc_mask_compact_static", "hc_sparse_spiral_conv_fwd",
            "hc_conv_rulebook", "hc_sparse_conv_rulebook_fwd", "hc_sparse_linear_fwd",
-           "hc_sparse_group_norm_fwd", "hc_scatter_dense", "hc_spiral_conv_fwd", "hc_get_device_status",
+           "hc_sparse_group_norm_fwd", "hc_mask_score_update", "hc_mask_select_topk",
+           "hc_kappa_masks", "hc_gather_rows", "hc_scatter_dense", "hc_spiral_conv_fwd", "hc_get_device_status",
            "hc_last_error_string", "hc_version")
 
 
@@ -64,6 +65,10 @@ def load_library(path: str | None = None):
                                             P],
             "hc_sparse_linear_fwd": [P, I, P, I, I, I, P, P, I, P, P],
             "hc_sparse_group_norm_fwd": [P, I, P, I, I, I, I, ctypes.c_float, P, P, I, P, P],
+            "hc_mask_score_update": [P, I, I, I, I, P, P, P, P],
+            "hc_mask_select_topk": [P, I, I, P, P],
+            "hc_kappa_masks": [P, I, I, P, I, I, P, P],
+            "hc_gather_rows": [P, I, I, I, I, P, P, I, I, P, P],
             "hc_scatter_dense": [P, I, P, P, P, I, I, I, I, P, P],
             "hc_spiral_conv_fwd": [P, I, P, I, I, I, I, I, P, P, I, P, P],
             "hc_get_device_status": [P],
@@ -181,6 +186,36 @@ def hc_sparse_group_norm_fwd(x, batch_offsets, G, eps, gamma, beta, act, y, stre
     _check(load_library().hc_sparse_group_norm_fwd(
         _p(x), _dt(x), _p(batch_offsets), B, capacity, C, G, float(eps), _p(gamma), _p(beta),
         act, _p(y), _s(stream)), "hc_sparse_group_norm_fwd")
+
+
+def hc_mask_score_update(O, alpha_in, alpha_out, sim=None, stream=None):
+    """Eq. 3 on mask outputs O [K, N, D]; alpha_in/alpha_out [K] fp32 (may
+    be the same tensor); sim [K, K] fp32 or None."""
+    K, N, D = O.shape
+    _check(load_library().hc_mask_score_update(
+        _p(O), _dt(O), K, N, D, _p(alpha_in), _p(alpha_out), _p(sim), _s(stream)),
+        "hc_mask_score_update")
+
+
+def hc_mask_select_topk(alpha, kappa, selected, stream=None):
+    """Indices of the kappa highest scores into selected [kappa] int32."""
+    _check(load_library().hc_mask_select_topk(_p(alpha), alpha.shape[0], kappa, _p(selected),
+                                              _s(stream)), "hc_mask_select_topk")
+
+
+def hc_kappa_masks(masks, selected, B, out, stream=None):
+    """out [B*kappa, V]: frame b*kappa + j = masks[selected[j]] (masks [K, V] uint8)."""
+    K, V = masks.shape
+    _check(load_library().hc_kappa_masks(_p(masks), K, V, _p(selected), selected.shape[0], B,
+                                         _p(out), _s(stream)), "hc_kappa_masks")
+
+
+def hc_gather_rows(x, coords, count, frames_per_sample, y, stream=None):
+    """S' of Eq. 2: y[n] = x[f // frames_per_sample, v] for coords[n] = (f, v)."""
+    B_in, V, C = x.shape
+    _check(load_library().hc_gather_rows(_p(x), _dt(x), B_in, V, C, _p(coords), _p(count),
+                                         y.shape[0], frames_per_sample, _p(y), _s(stream)),
+           "hc_gather_rows")
 
 
 def hc_scatter_dense(y, coords, row_of, count, B, V, zero_fill, out, stream=None):
