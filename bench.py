@@ -369,10 +369,11 @@ def run_ours(args, rank, world, local_rank):
 
     e2e = measure_e2e(torch, hc, sets, w, spiral, Wt, bias, stream, dev, args.e2e_steps)
 
-    sweep = gnorm = None
+    sweep = gnorm = mscore = None
     if not args.no_extras and rank == 0:
         sweep = run_sweep(torch, hc, dev, stream)
         gnorm = run_group_norm(torch, hc, sets, dev, stream)
+        mscore = run_mask_score(torch, hc, dev, stream)
 
     # Aggregate over ranks: rows summed, time = max over ranks.
     tot_rows, max_ms = reduce_over_ranks(float(rows_timed), ms, world, dev)
@@ -441,6 +442,8 @@ def run_ours(args, rank, world, local_rank):
         line["sweep"] = sweep
     if gnorm is not None:
         line["group_norm"] = gnorm
+    if mscore is not None:
+        line["mask_score"] = mscore
     return line
 
 
@@ -646,6 +649,52 @@ def run_group_norm(torch, hc, sets, dev, stream, G=8):
     if st != hc.HC_OK:
         raise RuntimeError(f"device status {hc.STATUS_NAMES.get(st)} in group norm")
     del x, y
+    torch.cuda.empty_cache()
+    return out
+
+
+def run_mask_score(torch, hc, dev, stream, K=10):
+    """Mask-score update (Eq. 3) for K = 10 masks, bf16 outputs, on the
+    4-layer encoder's output rows (64 frames x 655 vertices, 64 features)
+    and on a large layer's (32 frames x 10475 vertices, 128 features).
+    Algorithmic work: the symmetric Gram matrix of the [N, K*D] outputs,
+    N * KD * (KD + 1) flops (its upper triangle and diagonal)."""
+    pk = peaks()
+    out = {"K": K, "dtype": "bf16",
+           "kernels": "gram_tc_kernel (tcgen05 split-K Gram tiles) + pair_kernel + alpha_kernel"}
+    for name, N, D in (("encoder_outputs", 64 * 655, 64), ("large_layer", 32 * 10475, 128)):
+        g = torch.Generator(device=dev)
+        g.manual_seed(1234 + D)
+        O = torch.randn((K, N, D), generator=g, device=dev).to(torch.bfloat16)
+        a_in = torch.zeros(K, device=dev)
+        a_out = torch.empty(K, device=dev)
+        fn = lambda: hc.hc_mask_score_update(O, a_in, a_out, None, stream)  # noqa: E731
+        reps = 20 if N < 100000 else 5
+        with torch.cuda.stream(stream):
+            fn()
+            gr = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(gr, stream=stream):
+                for _ in range(reps):
+                    fn()
+            gr.replay()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            gr.replay()
+            e1.record(stream)
+        torch.cuda.synchronize(dev)
+        ms = e0.elapsed_time(e1) / reps
+        KD = K * D
+        flops = float(N) * KD * (KD + 1)
+        tf = flops / (ms * 1e-3) / 1e12
+        out[name] = {"N": N, "D": D, "us": ms * 1e3, "tflops": tf,
+                     "tensor_frac": tf / pk["bf16_tflops"],
+                     "input_bytes": O.numel() * 2,
+                     "peak": f"{pk['bf16_tflops']} TFLOP/s ({pk['source']} bf16 burst)"}
+        del O
+    st = hc.hc_get_device_status(stream)
+    if st != hc.HC_OK:
+        raise RuntimeError(f"device status {hc.STATUS_NAMES.get(st)} in the mask score")
     torch.cuda.empty_cache()
     return out
 

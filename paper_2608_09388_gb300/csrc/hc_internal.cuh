@@ -259,6 +259,12 @@ __device__ __forceinline__ void cp_async_16(uint32_t dst, const void* src, bool 
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(dst), "l"(src), "r"(n)
                  : "memory");
 }
+// 4 bytes, zero-filled when !valid (both addresses 4-byte aligned).
+__device__ __forceinline__ void cp_async_4(uint32_t dst, const void* src, bool valid) {
+    uint32_t n = valid ? 4u : 0u;
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"(dst), "l"(src), "r"(n)
+                 : "memory");
+}
 // Arrive on `bar` once every cp.async issued so far by this thread has
 // completed (the arrival is not counted in advance: the barrier's expected
 // count includes it).

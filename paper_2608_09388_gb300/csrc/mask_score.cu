@@ -8,21 +8,22 @@
 // k's features in columns k*D .. k*D + D - 1), G = O_all^T O_all and S[i][k]
 // is the sum of squares of G's (i, k) block. G is the only dense
 // contraction here (2 * N * (K*D)^2 flops, symmetric, so only its
-// upper-triangle 128 x 128 tiles are computed), and a squared block norm
-// needs the complete sum over N before squaring. So:
+// upper-triangle tiles are computed), and a squared block norm needs the
+// complete sum over N before squaring. So:
 //   1. gram: split-K partial tiles of G, one work item per (row split,
-//      upper tile), written to a workspace [item][128][128] fp32.
+//      upper tile), written to a workspace [item][tile][tile] fp32.
 //      bf16: tcgen05 (both operands MN-major from shared memory, fp32
 //      accumulators in TMEM); fp32: CUDA-core FFMA tiles.
-//   2. pairs: one block per pair i <= k sums the splits of every element of
-//      its D x D block (in a fixed order), squares and reduces: S[i][k].
-//   3. alpha: one block turns S into sim and the update.
+//   2. pairs: blocks per pair i <= k and chunk of its D x D block sum the
+//      splits of every entry (in a fixed order), square and reduce.
+//   3. alpha: a thread per mask adds the chunks into S, forms sim and the
+//      update (fp32; GB300's fp64 rate is far too low to be worth it here).
 // Deterministic: no atomics, every sum in a fixed order.
 //
-// bf16 operands are read straight from [K, N, D] with 16-byte cp.async when
-// D is a multiple of 8 (a 16-byte chunk never straddles two masks); other D
-// are first packed into a zero-padded [N, Mp] copy (Mp = K*D rounded up to
-// 128) in the workspace.
+// bf16 operands are read straight from [K, N, D] with cp.async: 16-byte
+// pieces when D is a multiple of 8, 4-byte pieces when D is even (a piece
+// never straddles two masks); odd D are first packed into a zero-padded
+// [N, Mp] copy (Mp = K*D rounded up to the tile) in the workspace.
 #include <cuda_bf16.h>
 
 #include "hc_internal.cuh"
@@ -30,30 +31,42 @@
 namespace hc {
 namespace {
 
-constexpr int kTile = 128;  // G tile edge (both operands: 128 feature columns)
-constexpr int kBK = 64;     // rows of O per pipeline stage (the contraction dim)
-constexpr int kStages = 6;
-constexpr int kOpBytes = kBK * kTile * 2;  // one operand tile of a stage (two 64-column atoms)
+constexpr int kBK = 64;  // rows of O per pipeline stage (the contraction dim)
+// tcgen05 path: TILE x TILE tiles of G (TILE = 128 or 256); per K16 step
+// TILE/128 MMAs of M=128 x N=TILE (the tile's row halves) into TILE/128
+// accumulators (128 or all 512 TMEM columns). A stage holds both operands'
+// TILE feature columns (TILE/64 64-column atoms each); 192 KB of stages, so
+// a 256 tile moves 64 KB per 8.4 MFLOP and a 128 tile 32 KB per 2.1 MFLOP.
+template <int TILE>
+struct TcCfg {
+    static constexpr int kHalves = TILE / 128;
+    static constexpr int kOpBytes = kBK * TILE * 2;
+    static constexpr int kStages = 196608 / (2 * kOpBytes);
+    static constexpr uint32_t kTmemCols = kHalves * TILE;
+    // kind::f16 instruction descriptor: D fp32 (bit 4), A and B bf16 (bits
+    // 7, 10), A and B MN-major (bits 15, 16), N >> 3 at 17, M >> 4 at 24.
+    static constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | (1u << 15) |
+                                       (1u << 16) | ((uint32_t)(TILE >> 3) << 17) |
+                                       ((uint32_t)(128 >> 4) << 24);
+};
 constexpr int kProducerWarps = 4, kEpilogueWarps = 4;
 constexpr int kMmaWarp = kProducerWarps + kEpilogueWarps;
 constexpr int kThreadsTc = (kMmaWarp + 1) * 32;
-constexpr int kPartElems = kTile * kTile;
-constexpr size_t kSmemTc = 1024 + (size_t)kStages * 2 * kOpBytes + 256;
-// kind::f16 instruction descriptor: D fp32 (bit 4), A and B bf16 (bits 7,
-// 10), A and B MN-major (bits 15, 16), N >> 3 at 17, M >> 4 at 24.
-constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | (1u << 15) | (1u << 16) |
-                            ((uint32_t)(kTile >> 3) << 17) | ((uint32_t)(kTile >> 4) << 24);
+constexpr size_t kSmemTc = 1024 + 196608 + 256;
+// CUDA-core path: 128 x 128 tiles.
+constexpr int kTileSimt = 128;
 
 struct GramArgs {
     const void* src;   // [Ksrc, N, Dsrc] (Ksrc = K, or 1 for the packed copy)
     long long N;       // rows
     int Dsrc;          // columns per source block
     int Mvalid;        // columns of O_all that exist (K*D); beyond: zeros
+    int tile;          // tile edge (256 tensor cores, 128 CUDA cores)
     int nt;            // tiles per edge of G
     int T;             // upper-triangle tiles
     int splits;
     long long rows_per_split;  // multiple of kBK
-    float* part;       // [splits * T][128][128]
+    float* part;       // [splits * T][tile][tile]
     unsigned* status;
 };
 
@@ -79,13 +92,24 @@ __device__ __forceinline__ uint64_t desc_sw128(uint32_t saddr, uint32_t lbo, uin
 
 // ---------------------------------------------------------------- bf16: tcgen05
 // Warps 0-3 load both operand tiles of a stage: thread t owns 16-byte chunk
-// column cc = t % 16 of the 128 feature columns (atom cc / 8, chunk cc % 8 in
-// the 128-byte row) and rows t / 16 + 8 i. In shared memory each operand is
-// two 64-column atoms of kBK rows x 128 bytes, chunks XOR-swizzled by row
-// (the layout a 128-byte-swizzled MN-major descriptor reads). Warp 8 issues
-// the MMAs; warps 4-7 move the finished accumulator to the workspace.
+// column t % (TILE/8) of the TILE feature columns (atom cc / 8, chunk cc % 8
+// in the 128-byte row) and rows t / (TILE/8) + (1024/TILE) i, so each row is
+// read whole. In shared memory each operand is TILE/64 64-column atoms of
+// kBK rows x 128 bytes, chunks XOR-swizzled by row (the layout a
+// 128-byte-swizzled MN-major descriptor reads). Warp 8 issues the MMAs;
+// warps 4-7 move the finished accumulators to the workspace.
+template <int TILE, bool kWide>  // 16-byte source pieces (D % 8 == 0), else 4-byte (D even)
 __global__ void __launch_bounds__(kThreadsTc, 1) gram_tc_kernel(const GramArgs a) {
+    using Cf = TcCfg<TILE>;
+    constexpr int kTileTc = TILE;
+    constexpr int kStages = Cf::kStages;
+    constexpr int kOpBytes = Cf::kOpBytes;
+    constexpr uint32_t kIdesc = Cf::kIdesc;
     constexpr uint32_t kArrivals = kProducerWarps * 32;
+    constexpr uint32_t kTmemCols = Cf::kTmemCols;
+    constexpr int kCpr = TILE / 8;                        // 16-byte chunks per row
+    constexpr int kRowsPerPass = kProducerWarps * 32 / kCpr;
+    constexpr int kAtom = kBK * 128;  // bytes of one 64-column atom
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;
@@ -112,7 +136,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) gram_tc_kernel(const GramArgs a
         asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
     }
     if (warp == kMmaWarp) {
-        tmem_alloc(smem_u32((const void*)tmem_holder), kTile);
+        tmem_alloc(smem_u32((const void*)tmem_holder), kTmemCols);
         tmem_relinquish();
     }
     tc_fence_before();
@@ -134,43 +158,55 @@ __global__ void __launch_bounds__(kThreadsTc, 1) gram_tc_kernel(const GramArgs a
 
     if (warp < kProducerWarps) {
         const __nv_bfloat16* __restrict__ src = static_cast<const __nv_bfloat16*>(a.src);
-        const int t = threadIdx.x;
-        const int cc = t & 15, atom = cc >> 3, q = cc & 7;
+        const int cc = threadIdx.x % kCpr, rg = threadIdx.x / kCpr;
+        const int atom = cc >> 3, q = cc & 7;
         // this thread's columns of each operand: source offset and validity
-        long long col_off[2];
-        bool col_ok[2];
+        // of each piece (one 8-column piece, or four 2-column pieces, which
+        // never straddle two masks when D is even)
+        constexpr int kPieces = kWide ? 1 : 4;
+        long long col_off[2][kPieces];
+        bool col_ok[2][kPieces];
 #pragma unroll
-        for (int op = 0; op < 2; ++op) {
-            const int m = (op == 0 ? tm : tn) * kTile + cc * 8;
-            col_ok[op] = m < a.Mvalid;
-            const int blk = col_ok[op] ? m / a.Dsrc : 0;
-            col_off[op] = col_ok[op] ? (long long)blk * a.N * a.Dsrc + (m - blk * a.Dsrc) : 0;
-        }
+        for (int op = 0; op < 2; ++op)
+#pragma unroll
+            for (int pc = 0; pc < kPieces; ++pc) {
+                const int m = (op == 0 ? tm : tn) * kTileTc + cc * 8 + pc * 2;
+                col_ok[op][pc] = m < a.Mvalid;
+                const int blk = col_ok[op][pc] ? m / a.Dsrc : 0;
+                col_off[op][pc] =
+                    col_ok[op][pc] ? (long long)blk * a.N * a.Dsrc + (m - blk * a.Dsrc) : 0;
+            }
         const int nops = diag ? 1 : 2;
-        bool ok = true;
         for (int kb = 0; kb < num_kb; ++kb) {
             const int s = kb % kStages;
             const uint32_t ph = (uint32_t)((kb / kStages) & 1);
-            if (!mbar_wait(empty_bar(s), ph ^ 1u, abort_flag, a.status)) {
-                ok = false;
-                break;
-            }
+            if (!mbar_wait(empty_bar(s), ph ^ 1u, abort_flag, a.status)) break;
             const long long n0 = r_begin + (long long)kb * kBK;
             for (int op = 0; op < nops; ++op) {
-                const uint32_t st = (op == 0 ? sA : sB) + s * kOpBytes + atom * (kBK * 128);
-#pragma unroll
-                for (int i = 0; i < kBK / 8; ++i) {
-                    const int r = (t >> 4) + 8 * i;
+                const uint32_t st = (op == 0 ? sA : sB) + s * kOpBytes + atom * kAtom;
+#pragma unroll 4
+                for (int i = 0; i < kBK / kRowsPerPass; ++i) {
+                    const int r = rg + kRowsPerPass * i;
                     const long long n = n0 + r;
-                    const bool valid = col_ok[op] && n < r_end;
-                    const __nv_bfloat16* gp = src + (valid ? col_off[op] + n * a.Dsrc : 0);
-                    cp_async_16(st + r * 128 + ((q ^ (r & 7)) << 4), gp, valid);
+                    const uint32_t dst = st + r * 128 + ((q ^ (r & 7)) << 4);
+                    if constexpr (kWide) {
+                        const bool valid = col_ok[op][0] && n < r_end;
+                        const __nv_bfloat16* gp = src + (valid ? col_off[op][0] + n * a.Dsrc : 0);
+                        cp_async_16(dst, gp, valid);
+                    } else {
+#pragma unroll
+                        for (int pc = 0; pc < 4; ++pc) {
+                            const bool valid = col_ok[op][pc] && n < r_end;
+                            const __nv_bfloat16* gp =
+                                src + (valid ? col_off[op][pc] + n * a.Dsrc : 0);
+                            cp_async_4(dst + pc * 4, gp, valid);
+                        }
+                    }
                 }
             }
             cp_async_arrive_noinc(full_bar(s));
         }
         cp_async_wait_all();
-        (void)ok;
     } else if (warp == kMmaWarp) {
         if (lane == 0) {
             bool ok = true;
@@ -188,9 +224,12 @@ __global__ void __launch_bounds__(kThreadsTc, 1) gram_tc_kernel(const GramArgs a
                 const uint32_t b_st = diag ? a_st : sB + s * kOpBytes;
 #pragma unroll
                 for (int k = 0; k < kBK / 16; ++k) {
-                    const uint64_t ad = desc_sw128(a_st + k * 16 * 128, kBK * 128, 1024);
-                    const uint64_t bd = desc_sw128(b_st + k * 16 * 128, kBK * 128, 1024);
-                    tc_mma_bf16(tmem_base, ad, bd, kIdesc, (kb | k) != 0 ? 1u : 0u);
+                    const uint64_t bd = desc_sw128(b_st + k * 16 * 128, kAtom, 1024);
+#pragma unroll
+                    for (int h = 0; h < Cf::kHalves; ++h) {
+                        const uint64_t ad = desc_sw128(a_st + h * 2 * kAtom + k * 16 * 128, kAtom, 1024);
+                        tc_mma_bf16(tmem_base + h * TILE, ad, bd, kIdesc, (kb | k) != 0 ? 1u : 0u);
+                    }
                 }
                 tc_commit(empty_bar(s));
             }
@@ -204,27 +243,31 @@ __global__ void __launch_bounds__(kThreadsTc, 1) gram_tc_kernel(const GramArgs a
         __syncwarp();
     } else {
         const int ew = warp - kProducerWarps;  // == warp % 4: TMEM lanes 32*ew..+32
-        const int row = ew * 32 + lane;
-        float* dst = a.part + (long long)item * kPartElems + (long long)row * kTile;
         if (mbar_wait(tfull_bar, 0, abort_flag, a.status)) {
             tc_fence_after();
 #pragma unroll 1
-            for (int cb = 0; cb < kTile / 32; ++cb) {
-                uint32_t r[32];
-                if (num_kb > 0) {
-                    tmem_ld_32x32b_x32(tmem_base + ((uint32_t)(ew * 32) << 16) + (uint32_t)(cb * 32),
-                                       r);
-                    tmem_ld_wait();
-                } else {
+            for (int h = 0; h < Cf::kHalves; ++h) {
+                const int row = h * 128 + ew * 32 + lane;
+                float* dst = a.part + (long long)item * kTileTc * kTileTc + (long long)row * kTileTc;
+#pragma unroll 1
+                for (int cb = 0; cb < kTileTc / 32; ++cb) {
+                    uint32_t r[32];
+                    if (num_kb > 0) {
+                        tmem_ld_32x32b_x32(tmem_base + ((uint32_t)(ew * 32) << 16) +
+                                               (uint32_t)(h * TILE + cb * 32),
+                                           r);
+                        tmem_ld_wait();
+                    } else {
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) r[j] = 0u;
+                        for (int j = 0; j < 32; ++j) r[j] = 0u;
+                    }
+                    float4* d4 = reinterpret_cast<float4*>(dst + cb * 32);
+#pragma unroll
+                    for (int j = 0; j < 8; ++j)
+                        d4[j] = make_float4(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]),
+                                            __uint_as_float(r[4 * j + 2]),
+                                            __uint_as_float(r[4 * j + 3]));
                 }
-                float4* d4 = reinterpret_cast<float4*>(dst + cb * 32);
-#pragma unroll
-                for (int j = 0; j < 8; ++j)
-                    d4[j] = make_float4(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]),
-                                        __uint_as_float(r[4 * j + 2]),
-                                        __uint_as_float(r[4 * j + 3]));
             }
             tc_fence_before();
         }
@@ -232,7 +275,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) gram_tc_kernel(const GramArgs a
     __syncthreads();
     if (warp == kMmaWarp) {
         tc_fence_after();
-        tmem_dealloc(tmem_base, kTile);
+        tmem_dealloc(tmem_base, kTmemCols);
     }
 }
 
@@ -242,8 +285,8 @@ constexpr int kSimtThreads = 256;
 constexpr int kSimtBK = 16;
 
 __global__ void __launch_bounds__(kSimtThreads) gram_simt_kernel(const GramArgs a) {
-    __shared__ float As[kSimtBK][kTile];
-    __shared__ float Bs[kSimtBK][kTile];
+    __shared__ float As[kSimtBK][kTileSimt];
+    __shared__ float Bs[kSimtBK][kTileSimt];
     pdl_wait();
     pdl_trigger();
     const float* __restrict__ src = static_cast<const float*>(a.src);
@@ -257,12 +300,12 @@ __global__ void __launch_bounds__(kSimtThreads) gram_simt_kernel(const GramArgs 
     if (r_end > a.N) r_end = a.N;
     const int t = threadIdx.x, ty = t >> 4, tx = t & 15;
     // columns this thread loads (fixed): mm = t % 128, rows t / 128 + 2 i
-    const int mm = t & (kTile - 1);
+    const int mm = t & (kTileSimt - 1);
     long long off[2];
     bool okc[2];
 #pragma unroll
     for (int op = 0; op < 2; ++op) {
-        const int m = (op == 0 ? tm : tn) * kTile + mm;
+        const int m = (op == 0 ? tm : tn) * kTileSimt + mm;
         okc[op] = m < a.Mvalid;
         const int blk = okc[op] ? m / a.Dsrc : 0;
         off[op] = okc[op] ? (long long)blk * a.N * a.Dsrc + (m - blk * a.Dsrc) : 0;
@@ -281,7 +324,7 @@ __global__ void __launch_bounds__(kSimtThreads) gram_simt_kernel(const GramArgs 
             if (!diag) Bs[r][mm] = (okc[1] && n < r_end) ? __ldg(src + off[1] + n * a.Dsrc) : 0.f;
         }
         __syncthreads();
-        const float(*Bp)[kTile] = diag ? As : Bs;
+        const float(*Bp)[kTileSimt] = diag ? As : Bs;
 #pragma unroll 4
         for (int k = 0; k < kSimtBK; ++k) {
             float av[8], bv[8];
@@ -296,10 +339,10 @@ __global__ void __launch_bounds__(kSimtThreads) gram_simt_kernel(const GramArgs 
         }
         __syncthreads();
     }
-    float* dst = a.part + (long long)item * kPartElems;
+    float* dst = a.part + (long long)item * kTileSimt * kTileSimt;
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
-        float4* d4 = reinterpret_cast<float4*>(dst + (ty * 8 + i) * kTile + tx * 8);
+        float4* d4 = reinterpret_cast<float4*>(dst + (ty * 8 + i) * kTileSimt + tx * 8);
         d4[0] = make_float4(acc[i][0], acc[i][1], acc[i][2], acc[i][3]);
         d4[1] = make_float4(acc[i][4], acc[i][5], acc[i][6], acc[i][7]);
     }
@@ -326,25 +369,43 @@ __global__ void pack_kernel(const __nv_bfloat16* __restrict__ O, long long N, in
 }
 
 // ---------------------------------------------------------------- pairs
-// Block p <-> pair (i, k), i <= k (row-major over the upper triangle of the
-// K x K matrix). S[i][k] = sum over the D x D block of (sum over splits)^2.
+// Block (p, c) <-> pair p = (i, k), i <= k (row-major over the upper
+// triangle of the K x K matrix, diagonal included), and chunk c of
+// kPairChunk entries of its D x D block: the sum over that chunk of
+// (sum over splits of G's entry)^2, written to P[p][c]. Fixed orders.
 constexpr int kPairThreads = 256;
+constexpr int kPairChunk = 1024;
 
-__global__ void __launch_bounds__(kPairThreads)
-    pair_kernel(const float* __restrict__ part, int K, int D, int nt, int T, int splits,
-                float* __restrict__ S) {
-    __shared__ double red[kPairThreads / 32];
-    pdl_wait();
-    pdl_trigger();
-    int i = 0, rem = blockIdx.x;
-    while (rem >= K - i) {
-        rem -= K - i;
+__device__ __forceinline__ int pair_of(int p, int K, int& k) {
+    int i = 0;
+    while (p >= K - i) {
+        p -= K - i;
         ++i;
     }
-    const int k = i + rem;
-    float acc = 0.f;
+    k = i + p;
+    return i;
+}
+__device__ __forceinline__ int pair_index(int i, int k, int K) {  // i <= k
+    return i * K - i * (i - 1) / 2 + (k - i);
+}
+
+__global__ void __launch_bounds__(kPairThreads)
+    pair_kernel(const float* __restrict__ part, int K, int D, int tile_shift, int nt, int T,
+                int splits, int nchunk, float* __restrict__ P) {
+    __shared__ float red[kPairThreads / 32];
+    pdl_wait();
+    pdl_trigger();
+    const int p = blockIdx.x / nchunk, chunk = blockIdx.x - p * nchunk;
+    int k;
+    const int i = pair_of(p, K, k);
     const int DD = D * D;
-    for (int idx = threadIdx.x; idx < DD; idx += kPairThreads) {
+    const int e0 = chunk * kPairChunk;
+    const int e1 = e0 + kPairChunk < DD ? e0 + kPairChunk : DD;
+    const int tmask = (1 << tile_shift) - 1;
+    const long long tile_elems = 1ll << (2 * tile_shift);
+    const long long split_stride = (long long)T * tile_elems;
+    float acc = 0.f;
+    for (int idx = e0 + threadIdx.x; idx < e1; idx += kPairThreads) {
         const int d = idx / D, e = idx - d * D;
         int m = i * D + d, m2 = k * D + e;
         if (m > m2) {  // below the diagonal: the symmetric entry of an upper tile
@@ -352,42 +413,51 @@ __global__ void __launch_bounds__(kPairThreads)
             m = m2;
             m2 = tmp;
         }
-        const int t = tile_index(m >> 7, m2 >> 7, nt);
-        const long long off = ((long long)(m & 127) << 7) + (m2 & 127);
+        const float* src = part + tile_index(m >> tile_shift, m2 >> tile_shift, nt) * tile_elems +
+                           ((long long)(m & tmask) << tile_shift) + (m2 & tmask);
         float g = 0.f;
-        for (int s = 0; s < splits; ++s) g += __ldg(part + ((long long)s * T + t) * kPartElems + off);
+#pragma unroll 8
+        for (int sp = 0; sp < splits; ++sp) g += __ldg(src + sp * split_stride);
         acc = fmaf(g, g, acc);
     }
-    double v = acc;
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = acc;
     __syncthreads();
     if (threadIdx.x == 0) {
-        double tot = 0.0;
+        float tot = 0.f;
+#pragma unroll
         for (int w = 0; w < kPairThreads / 32; ++w) tot += red[w];
-        S[i * K + k] = (float)tot;
-        S[k * K + i] = (float)tot;
+        P[blockIdx.x] = tot;
     }
 }
 
 // ---------------------------------------------------------------- alpha
-__global__ void alpha_kernel(const float* __restrict__ S, int K, const float* alpha_in,
+// Thread per mask k: S[i][k] = sum over chunks of P[pair(i, k)], the norms
+// ||O_i^T O_i||_F = sqrt(S[i][i]), then sim and the update (fp32).
+__device__ __forceinline__ float pair_sum(const float* P, int i, int k, int K, int nchunk) {
+    const int p = i <= k ? pair_index(i, k, K) : pair_index(k, i, K);
+    float s = 0.f;
+    for (int c = 0; c < nchunk; ++c) s += __ldg(P + (long long)p * nchunk + c);
+    return s;
+}
+
+__global__ void alpha_kernel(const float* __restrict__ P, int K, int nchunk, const float* alpha_in,
                              float* alpha_out, float* __restrict__ sim) {
     pdl_wait();
     pdl_trigger();
-    for (int k = threadIdx.x; k < K; k += blockDim.x) {
-        const double nk = sqrt((double)S[k * K + k]);
-        double sum = 0.0;
-        for (int i = 0; i < K; ++i) {
-            const double den = sqrt((double)S[i * K + i]) * nk;
-            const double s = den > 0.0 ? (double)S[i * K + k] / den : 0.0;
-            if (sim) sim[i * K + k] = (float)s;
-            if (i != k) sum += 1.0 - s;
-        }
-        const float a0 = alpha_in[k];
-        alpha_out[k] = K > 1 ? (float)((double)a0 + sum / (double)(K - 1)) : a0;
+    const int k = blockIdx.x * blockDim.x + threadIdx.x;
+    if (k >= K) return;
+    const float nk = sqrtf(pair_sum(P, k, k, K, nchunk));
+    float sum = 0.f;
+    for (int i = 0; i < K; ++i) {
+        const float den = sqrtf(pair_sum(P, i, i, K, nchunk)) * nk;
+        const float s = den > 0.f ? pair_sum(P, i, k, K, nchunk) / den : 0.f;
+        if (sim) sim[(long long)i * K + k] = s;
+        if (i != k) sum += 1.f - s;
     }
+    const float a0 = alpha_in[k];
+    alpha_out[k] = K > 1 ? a0 + sum / (float)(K - 1) : a0;
 }
 
 }  // namespace
@@ -395,23 +465,47 @@ __global__ void alpha_kernel(const float* __restrict__ S, int K, const float* al
 hc_status launch_mask_score(const DeviceCtx* ctx, const void* O, hc_dtype dt, int K, long long N,
                             int D, const float* alpha_in, float* alpha_out, float* sim,
                             cudaStream_t s) {
+    const bool tc = dt == HC_BF16;
+    // 256-wide tensor-core tiles halve the operand bytes per flop, which
+    // pays once G has enough tiles; small K*D keeps 128 tiles (fewer row
+    // splits, less split-K partial traffic).
+    const bool big = tc && (long long)K * D >= 1024;
+    const int tile = big ? 256 : 128;
+    const int tile_shift = big ? 8 : 7;
     const int KD = K * D;
-    const int Mp = (KD + kTile - 1) / kTile * kTile;
-    const int nt = Mp / kTile;
+    const int nt = (KD + tile - 1) / tile;
+    const int Mp = nt * tile;
     const int T = nt * (nt + 1) / 2;
-    int splits = ctx->num_sms / T;
-    if (splits < 1) splits = 1;
-    const long long max_splits = (N + kBK - 1) / kBK;
-    if (splits > max_splits) splits = (int)(max_splits > 0 ? max_splits : 1);
+    // Row splits: one CTA per SM (the kernel's shared memory), so pick the
+    // smallest split count whose waves of splits * T items are >= 95% full
+    // (else the fullest), with at least one 64-row block per split.
+    long long max_splits = (N + kBK - 1) / kBK;
+    const long long cap_splits = 8ll * ctx->num_sms / T + 1;
+    if (max_splits > cap_splits) max_splits = cap_splits;
+    if (max_splits < 1) max_splits = 1;
+    int splits = 1;
+    double best = 0.0;
+    for (int sp = 1; sp <= max_splits; ++sp) {
+        const long long items_sp = (long long)sp * T;
+        const long long waves = (items_sp + ctx->num_sms - 1) / ctx->num_sms;
+        const double eff = (double)items_sp / (double)(waves * ctx->num_sms);
+        if (eff > best + 1e-9) {
+            best = eff;
+            splits = sp;
+        }
+        if (eff >= 0.95) break;
+    }
     long long rps = (N + splits - 1) / splits;
     rps = (rps + kBK - 1) / kBK * kBK;
     if (rps < kBK) rps = kBK;
     const long long items = (long long)splits * T;
 
-    const bool tc = dt == HC_BF16;
-    const bool packed = tc && (D % 8 != 0 || (uintptr_t)O % 16 != 0);
-    const size_t part_bytes = sizeof(float) * (size_t)items * kPartElems;
-    const size_t s_bytes = sizeof(float) * (size_t)K * K;
+    const bool wide = D % 8 == 0 && (uintptr_t)O % 16 == 0;
+    const bool packed = tc && !wide && (D % 2 != 0 || (uintptr_t)O % 4 != 0);
+    const int n_pairs = K * (K + 1) / 2;
+    const int nchunk = (D * D + kPairChunk - 1) / kPairChunk;
+    const size_t part_bytes = sizeof(float) * (size_t)items * tile * tile;
+    const size_t s_bytes = sizeof(float) * (size_t)n_pairs * nchunk;
     const size_t pack_off = (part_bytes + s_bytes + 255) / 256 * 256;
     const size_t pack_bytes = packed ? sizeof(__nv_bfloat16) * (size_t)N * Mp : 0;
     uint8_t* ws = (uint8_t*)stream_workspace(s, pack_off + pack_bytes);
@@ -428,6 +522,7 @@ hc_status launch_mask_score(const DeviceCtx* ctx, const void* O, hc_dtype dt, in
         g.N = N;
         g.Dsrc = D;
         g.Mvalid = KD;
+        g.tile = tile;
         g.nt = nt;
         g.T = T;
         g.splits = splits;
@@ -449,26 +544,42 @@ hc_status launch_mask_score(const DeviceCtx* ctx, const void* O, hc_dtype dt, in
             }
             static bool attr_set[64] = {};
             if (!attr_set[ctx->device]) {
-                st = check_cuda(cudaFuncSetAttribute(gram_tc_kernel,
-                                                     cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                     (int)kSmemTc),
-                                "cudaFuncSetAttribute(gram_tc_kernel)");
-                if (st != HC_OK) return st;
+                const void* fns[4] = {(const void*)gram_tc_kernel<128, true>,
+                                      (const void*)gram_tc_kernel<128, false>,
+                                      (const void*)gram_tc_kernel<256, true>,
+                                      (const void*)gram_tc_kernel<256, false>};
+                for (const void* f : fns) {
+                    st = check_cuda(cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                         (int)kSmemTc),
+                                    "cudaFuncSetAttribute(gram_tc_kernel)");
+                    if (st != HC_OK) return st;
+                }
                 attr_set[ctx->device] = true;
             }
-            st = launch_pdl(gram_tc_kernel, dim3((unsigned)items), dim3(kThreadsTc), kSmemTc, s,
-                            "gram_tc_kernel", g);
+            const bool w16 = wide || packed;
+            const dim3 grid((unsigned)items), block(kThreadsTc);
+            if (big)
+                st = w16 ? launch_pdl(gram_tc_kernel<256, true>, grid, block, kSmemTc, s,
+                                      "gram_tc_kernel", g)
+                         : launch_pdl(gram_tc_kernel<256, false>, grid, block, kSmemTc, s,
+                                      "gram_tc_kernel", g);
+            else
+                st = w16 ? launch_pdl(gram_tc_kernel<128, true>, grid, block, kSmemTc, s,
+                                      "gram_tc_kernel", g)
+                         : launch_pdl(gram_tc_kernel<128, false>, grid, block, kSmemTc, s,
+                                      "gram_tc_kernel", g);
         } else {
             st = launch_pdl(gram_simt_kernel, dim3((unsigned)items), dim3(kSimtThreads), 0, s,
                             "gram_simt_kernel", g);
         }
         if (st != HC_OK) return st;
-        st = launch_pdl(pair_kernel, dim3((unsigned)(K * (K + 1) / 2)), dim3(kPairThreads), 0, s,
-                        "pair_kernel", (const float*)part, K, D, nt, T, splits, S);
+        st = launch_pdl(pair_kernel, dim3((unsigned)(n_pairs * nchunk)), dim3(kPairThreads), 0, s,
+                        "pair_kernel", (const float*)part, K, D, tile_shift, nt, T, splits, nchunk,
+                        S);
         if (st != HC_OK) return st;
     }
-    return launch_pdl(alpha_kernel, dim3(1), dim3(256), 0, s, "alpha_kernel", (const float*)S, K,
-                      alpha_in, alpha_out, sim);
+    return launch_pdl(alpha_kernel, dim3((unsigned)((K + 127) / 128)), dim3(128), 0, s,
+                      "alpha_kernel", (const float*)S, K, nchunk, alpha_in, alpha_out, sim);
 }
 
 }  // namespace hc

@@ -5,7 +5,7 @@ against the CPU oracle through the C-ABI.
 
 Tolerances: indices, masks and gathered rows are bit-exact. Scores: the
 Gram sums are fp32 (tensor-core accumulation for bf16 inputs, FFMA for
-fp32), S, sim and alpha are then formed in fp64 from fp32 sums, so |alpha -
+fp32) and S, sim and alpha are formed from them in fp32, so |alpha -
 alpha_oracle| and |sim - sim_oracle| <= 1e-4 (the fp32 bar)."""
 import os
 
@@ -53,10 +53,13 @@ def run_score(O_np, alpha_np, in_place=False):
 @pytest.mark.parametrize("dtype", ["bf16", "f32"])
 @pytest.mark.parametrize("K,N,D", [(2, 100, 8), (3, 1000, 64), (4, 777, 5), (5, 300, 1),
                                    (1, 50, 16), (6, 333, 130), (10, 4000, 42), (3, 64, 8),
-                                   (2, 1, 3), (40, 500, 16)])
+                                   (2, 1, 3), (40, 500, 16), (10, 3000, 128), (9, 700, 130),
+                                   (11, 500, 101)])
 def test_mask_score(K, N, D, dtype):
-    """Multi-tile Gram matrices (K*D > 128), ragged row counts, D not a
-    multiple of 8 (the packed path), D = 1, K = 1, one row."""
+    """Multi-tile Gram matrices (K*D > 128; K*D >= 1024 takes the 256-wide
+    tensor-core tiles), ragged row counts, D a multiple of 8 (16-byte
+    pieces), even (4-byte pieces) and odd (the packed copy), D = 1, K = 1,
+    one row."""
     rng = np.random.default_rng(K * 1000 + N + D)
     O = _outputs(rng, K, N, D, dtype)
     alpha = rng.standard_normal(K)
