@@ -23,6 +23,9 @@ Functions and the passages they follow:
                            (Sec. 3.1, Sparse Mask Selection)
 * ``kappa_masks``          every kept mask applied to every sample (Eq. 1)
 * ``gather_rows``          the feature matrix S' of Eq. 2
+* ``sparse_conv_bwd``      gradients of the sparse convolution with respect
+                           to input rows, weight and bias (chain rule on
+                           Eqs. 4-5, 6, 10, through the Eq. 4 mapping)
 * ``encoder``              a stack of sparse layers: coordinates fixed once by
                            the mask (Eqs. 5, 6, 10 keep C'), each layer's output
                            stored in the layer dtype before the next reads it
@@ -99,6 +102,9 @@ def _load():
             lib.hco_kappa_masks.restype = None
             lib.hco_gather_rows.argtypes = [P, I, I64, I, P, I64, I64, P]
             lib.hco_gather_rows.restype = None
+            lib.hco_sparse_conv_bwd.argtypes = [P, I, I64, P, I64, I64, I, I, I, P, P, P, I, P,
+                                                P, P]
+            lib.hco_sparse_conv_bwd.restype = None
             lib.hco_bf16_round.argtypes = [ctypes.c_double]
             lib.hco_bf16_round.restype = ctypes.c_uint16
             _lib = lib
@@ -334,3 +340,30 @@ def gather_rows(x, coords, frames_per_sample=1):
     _load().hco_gather_rows(_ptr(x), x.dtype.itemsize, V, C, _ptr(coords), n,
                             frames_per_sample, _ptr(y))
     return y
+
+
+def sparse_conv_bwd(x, rulebook, W, y, dy, act):
+    """Gradients of the sparse conv through the Eq. 4 mapping rulebook
+    [L, stride] (column n < len(dy) = output row n). x: input rows
+    [x_rows, C_in] (dense layout flattened to B*V rows, or compact); y: the
+    stored forward output [n_rows, C_out]; dy: upstream gradient, same shape;
+    all float32 or all bf16 bits. Returns (dx [x_rows, C_in], dW [L*C_in,
+    C_out], dbias [C_out]), fp64."""
+    x = np.ascontiguousarray(x)
+    dt = _dtype_code(x)
+    C_in = x.shape[-1]
+    x = x.reshape(-1, C_in)
+    rulebook = _c(rulebook, np.int32)
+    L, stride = rulebook.shape
+    W = _c(W, x.dtype)
+    C_out = W.shape[1]
+    y = _c(y, x.dtype)
+    dy = _c(dy, x.dtype)
+    n = dy.shape[0]
+    dx = np.empty((x.shape[0], C_in), dtype=np.float64)
+    dW = np.empty((L * C_in, C_out), dtype=np.float64)
+    db = np.empty(C_out, dtype=np.float64)
+    _load().hco_sparse_conv_bwd(_ptr(x), dt, x.shape[0], _ptr(rulebook), n, stride, L, C_in,
+                                C_out, _ptr(W), _ptr(y), _ptr(dy), act, _ptr(dx), _ptr(dW),
+                                _ptr(db))
+    return dx, dW, db

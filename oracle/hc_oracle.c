@@ -35,6 +35,9 @@
  *                           frames per sample (Eq. 1 per kept mask)
  *   hco_gather_rows         the feature matrix S' of Eq. 2: the input rows
  *                           at the active coordinates
+ *   hco_sparse_conv_bwd     gradients of the sparse convolution (Eqs. 4-5,
+ *                           6, 10) with respect to its input rows, weight
+ *                           and bias, through the Eq. 4 indexing matrix
  *   hco_bf16_round          fp64 -> bf16 rounding (storage format)
  *
  * Parity status: compaction, conv, dense conv, linear, group norm, scatter,
@@ -442,4 +445,61 @@ void hco_gather_rows(const void* x, int elem_bytes, int64_t V, int C, const int3
         memcpy(dst + n * row_bytes, src + ((f / frames_per_sample) * V + v) * row_bytes,
                (size_t)row_bytes);
     }
+}
+
+/* ------------------------------------------------------ sparse conv bwd */
+
+/* Gradients of the sparse spiral convolution (the paper gives the forward
+ * only; these follow from it by the chain rule). With the indexing matrix
+ * of Eq. 4, rulebook[l*stride + n] = the input row j read by tap l of
+ * output row n (or -1), the forward is
+ *     z[n][o] = bias[o] + sum_l sum_c x[j(n,l)][c] * W[l*C_in + c][o],
+ *     y = act(z)                                                (Eq. 10)
+ * and, for an upstream gradient dy = dL/dy over the n_rows output rows,
+ *     dz[n][o]   = dy[n][o] * act'(z[n][o])
+ *     dbias[o]   = sum_n dz[n][o]
+ *     dW[l*C_in + c][o] = sum_n x[j(n,l)][c] * dz[n][o]   (present taps only)
+ *     dx[j][c]   = sum over (n, l) with j(n,l) = j of sum_o dz[n][o] * W[l*C_in + c][o]
+ * act' is read off the stored output y: ELU (alpha = 1) has derivative 1
+ * for z > 0 and e^z = y + 1 otherwise; ReLU 1 for z > 0 else 0; none 1.
+ * dx ([x_rows, C_in]), dW ([L*C_in, C_out]) and dbias ([C_out]) are fp64
+ * and overwritten (rows of dx no tap reads are 0); any may be NULL. */
+static double act_grad_from_output(double y, int act) {
+    if (act == HCO_ACT_ELU) return y > 0.0 ? 1.0 : y + 1.0;
+    if (act == HCO_ACT_RELU) return y > 0.0 ? 1.0 : 0.0;
+    return 1.0;
+}
+
+void hco_sparse_conv_bwd(const void* x, int dtype, int64_t x_rows, const int32_t* rulebook,
+                         int64_t n_rows, int64_t stride, int L, int C_in, int C_out, const void* W,
+                         const void* y, const void* dy, int act, double* dx, double* dW,
+                         double* dbias) {
+    if (dx) memset(dx, 0, sizeof(double) * (size_t)(x_rows * C_in));
+    if (dW) memset(dW, 0, sizeof(double) * (size_t)((int64_t)L * C_in * C_out));
+    if (dbias) memset(dbias, 0, sizeof(double) * (size_t)C_out);
+    double* dz = (double*)malloc(sizeof(double) * (size_t)C_out);
+    for (int64_t n = 0; n < n_rows; ++n) {
+        for (int o = 0; o < C_out; ++o)
+            dz[o] = load_elem(dy, dtype, n * C_out + o) *
+                    act_grad_from_output(load_elem(y, dtype, n * C_out + o), act);
+        if (dbias)
+            for (int o = 0; o < C_out; ++o) dbias[o] += dz[o];
+        for (int l = 0; l < L; ++l) {
+            int64_t j = rulebook[(int64_t)l * stride + n];
+            if (j < 0) continue; /* absent tap: no term, no gradient */
+            for (int c = 0; c < C_in; ++c) {
+                int64_t k = (int64_t)l * C_in + c;
+                if (dW) {
+                    double xv = load_elem(x, dtype, j * C_in + c);
+                    for (int o = 0; o < C_out; ++o) dW[k * C_out + o] += xv * dz[o];
+                }
+                if (dx) {
+                    double g = 0.0;
+                    for (int o = 0; o < C_out; ++o) g += dz[o] * load_elem(W, dtype, k * C_out + o);
+                    dx[j * C_in + c] += g;
+                }
+            }
+        }
+    }
+    free(dz);
 }

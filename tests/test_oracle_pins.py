@@ -368,6 +368,15 @@ MUTANTS = {
                               "                         load_elem(O, dtype, (k * N + n) * D + d);"),
     "mask score numerator not squared": ("                acc += g * g;", "                acc += fabs(g);"),
     "top-kappa ties by highest index": ("    return isnan(b) || a > b;", "    return isnan(b) || a >= b;"),
+    "backward ELU derivative as exp(y)": ("    if (act == HCO_ACT_ELU) return y > 0.0 ? 1.0 : y + 1.0;",
+                                          "    if (act == HCO_ACT_ELU) return y > 0.0 ? 1.0 : exp(y);"),
+    "backward input gradient with a transposed weight": (
+        "                    for (int o = 0; o < C_out; ++o) g += dz[o] * load_elem(W, dtype, k * C_out + o);",
+        "                    for (int o = 0; o < C_out; ++o) g += dz[o] * load_elem(W, dtype, (int64_t)o * L * C_in + k);"),
+    "backward absent tap read as row 0": ("            if (j < 0) continue; /* absent tap: no term, no gradient */",
+                                          "            if (j < 0) j = 0;"),
+    "backward bias gradient skips the activation": ("            for (int o = 0; o < C_out; ++o) dbias[o] += dz[o];",
+                                                    "            for (int o = 0; o < C_out; ++o) dbias[o] += load_elem(dy, dtype, n * C_out + o);"),
     "centre tap dropped": ("for (int l = 0; l < L; ++l) {\n            int64_t u = spiral[v * L + l];\n            if (u < 0) continue; /* no neighbour in this slot */",
                            "for (int l = 1; l < L; ++l) {\n            int64_t u = spiral[v * L + l];\n            if (u < 0) continue; /* no neighbour in this slot */"),
 }
@@ -392,7 +401,7 @@ def test_planted_mistake_is_caught(name, tmp_path, monkeypatch):
     for fn in ("hco_mask_compact", "hco_sparse_spiral_conv", "hco_dense_spiral_conv",
                "hco_sparse_linear", "hco_scatter_dense", "hco_bf16_round", "hco_conv_rulebook",
                "hco_sparse_group_norm", "hco_mask_score", "hco_select_topk", "hco_kappa_masks",
-               "hco_gather_rows"):
+               "hco_gather_rows", "hco_sparse_conv_bwd"):
         getattr(lib, fn).argtypes = getattr(good, fn).argtypes
         getattr(lib, fn).restype = getattr(good, fn).restype
     monkeypatch.setattr(oracle, "_lib", lib)
@@ -400,7 +409,9 @@ def test_planted_mistake_is_caught(name, tmp_path, monkeypatch):
               check_group_norm_vs_numpy,
               lambda: check_compact_vs_nonzero(inputs.uniform_mask(np.random.default_rng(1), 5, 20, 0.3)),
               check_bf16_round, check_mask_score_golden, check_mask_score_vs_numpy,
-              check_mask_score_d1_is_squared_cosine, check_select_topk_vs_argsort]
+              check_mask_score_d1_is_squared_cosine, check_select_topk_vs_argsort,
+              check_bwd_finite_differences, check_bwd_linear_closed_form,
+              check_bwd_adjoint_identity]
     caught = 0
     for chk in checks:
         try:
@@ -610,3 +621,106 @@ def test_kappa_masks_and_gather_rows_vs_numpy():
     np.testing.assert_array_equal(y, x[coords[:, 0] // kappa, coords[:, 1]])
     np.testing.assert_array_equal(oracle.gather_rows(x, oracle.mask_compact(masks[:B])[0]),
                                   x[np.nonzero(masks[:B])])
+
+
+# ------------------------------------------------------------ backward (chain rule)
+
+def _bwd_case(seed, act, layout=oracle.LAYOUT_DENSE, B=2, V=30, L=5, C_in=3, C_out=4):
+    """A small conv with a fully seeded forward: values stay well inside
+    float32's exact range for dyadic steps of 2^-12."""
+    rng = np.random.default_rng(seed)
+    pts = inputs.sphere_points(rng, V)
+    sp = inputs.spiral_table(pts, L)
+    sp[3, 2] = -1  # a missing spiral slot
+    m = inputs.uniform_mask(rng, B, V, 0.6)
+    coords, row_of, _, n = oracle.mask_compact(m)
+    x_dense = rng.standard_normal((B, V, C_in)).astype(np.float32)
+    x = x_dense if layout == oracle.LAYOUT_DENSE else oracle.gather_rows(x_dense, coords)
+    W = (rng.standard_normal((L * C_in, C_out)) * 0.5).astype(np.float32)
+    b = rng.standard_normal(C_out).astype(np.float32)
+    g = rng.standard_normal((n, C_out)).astype(np.float32)  # upstream gradient
+    rb = oracle.conv_rulebook(coords, row_of, sp, layout, stride=n)
+    return dict(x=x, W=W, b=b, g=g, sp=sp, coords=coords, row_of=row_of, rb=rb, act=act,
+                layout=layout)
+
+
+def _loss(c, x=None, W=None, b=None):
+    y, _ = oracle.sparse_spiral_conv(c["x"] if x is None else x, c["layout"], c["coords"],
+                                     c["row_of"], c["sp"], c["W"] if W is None else W,
+                                     c["b"] if b is None else b, c["act"])
+    return float(np.sum(y * c["g"].astype(np.float64)))
+
+
+def check_bwd_finite_differences(seed=51, act=oracle.ACT_ELU, layout=oracle.LAYOUT_DENSE):
+    """Central differences of the fp64 forward loss sum(y * g) against the
+    backward, for sampled input, weight and bias entries. Steps are 2^-12,
+    exact in float32 for these magnitudes."""
+    c = _bwd_case(seed, act, layout)
+    _, y = oracle.sparse_spiral_conv(c["x"], c["layout"], c["coords"], c["row_of"], c["sp"],
+                                     c["W"], c["b"], act)
+    dx, dW, db = oracle.sparse_conv_bwd(c["x"], c["rb"], c["W"], y, c["g"], act)
+    h = 2.0 ** -12
+    rng = np.random.default_rng(seed + 1)
+    xf = c["x"].reshape(-1)
+    for idx in rng.choice(xf.size, 24, replace=False):
+        xp, xm = xf.copy(), xf.copy()
+        xp[idx] += h
+        xm[idx] -= h
+        fd = (_loss(c, x=xp.reshape(c["x"].shape)) - _loss(c, x=xm.reshape(c["x"].shape))) / (2 * h)
+        assert abs(fd - dx.reshape(-1)[idx]) <= 1e-5 * max(1.0, abs(fd)), ("dx", idx, fd)
+    Wf = c["W"].reshape(-1)
+    for idx in rng.choice(Wf.size, 24, replace=False):
+        wp, wm = Wf.copy(), Wf.copy()
+        wp[idx] += h
+        wm[idx] -= h
+        fd = (_loss(c, W=wp.reshape(c["W"].shape)) - _loss(c, W=wm.reshape(c["W"].shape))) / (2 * h)
+        assert abs(fd - dW.reshape(-1)[idx]) <= 1e-5 * max(1.0, abs(fd)), ("dW", idx, fd)
+    for o in range(c["b"].size):
+        bp, bm = c["b"].copy(), c["b"].copy()
+        bp[o] += h
+        bm[o] -= h
+        fd = (_loss(c, b=bp) - _loss(c, b=bm)) / (2 * h)
+        assert abs(fd - db[o]) <= 1e-5 * max(1.0, abs(fd)), ("db", o, fd)
+
+
+@pytest.mark.parametrize("act", [oracle.ACT_ELU, oracle.ACT_RELU, oracle.ACT_NONE])
+@pytest.mark.parametrize("layout", [oracle.LAYOUT_DENSE, oracle.LAYOUT_COMPACT])
+def test_bwd_finite_differences(act, layout):
+    check_bwd_finite_differences(act=act, layout=layout)
+
+
+def check_bwd_linear_closed_form(seed=52):
+    """L = 1 with the identity mapping is a linear layer: dW = x^T dz,
+    dx = dz W^T, dbias = column sums of dz (numpy matmul, fp64)."""
+    rng = np.random.default_rng(seed)
+    n, C_in, C_out = 37, 6, 5
+    x = rng.standard_normal((n, C_in)).astype(np.float32)
+    W = rng.standard_normal((C_in, C_out)).astype(np.float32)
+    y = rng.standard_normal((n, C_out)).astype(np.float32)
+    g = rng.standard_normal((n, C_out)).astype(np.float32)
+    rb = np.arange(n, dtype=np.int32)[None, :]
+    dx, dW, db = oracle.sparse_conv_bwd(x, rb, W, y, g, oracle.ACT_ELU)
+    dz = g.astype(np.float64) * np.where(y > 0, 1.0, y.astype(np.float64) + 1.0)
+    np.testing.assert_allclose(dW, x.astype(np.float64).T @ dz, rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(dx, dz @ W.astype(np.float64).T, rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(db, dz.sum(axis=0), rtol=1e-12, atol=1e-12)
+
+
+def test_bwd_linear_closed_form():
+    check_bwd_linear_closed_form()
+
+
+def check_bwd_adjoint_identity(seed=53):
+    """Without bias and activation the layer is bilinear in (x, W), so
+    <y, g> = <x, dx> = <W, dW> exactly (in fp64, up to rounding order)."""
+    c = _bwd_case(seed, oracle.ACT_NONE, B=3, V=60, L=7, C_in=4, C_out=6)
+    y, ys = oracle.sparse_spiral_conv(c["x"], c["layout"], c["coords"], c["row_of"], c["sp"],
+                                      c["W"], None, oracle.ACT_NONE)
+    dx, dW, _ = oracle.sparse_conv_bwd(c["x"], c["rb"], c["W"], ys, c["g"], oracle.ACT_NONE)
+    yg = float(np.sum(y * c["g"]))
+    assert abs(np.sum(c["x"].reshape(dx.shape).astype(np.float64) * dx) - yg) <= 1e-10 * abs(yg) + 1e-10
+    assert abs(np.sum(c["W"].astype(np.float64) * dW) - yg) <= 1e-10 * abs(yg) + 1e-10
+
+
+def test_bwd_adjoint_identity():
+    check_bwd_adjoint_identity()
