@@ -227,6 +227,53 @@ hc_status hc_sparse_group_norm_fwd(const void* x, hc_dtype dt, const int32_t* ba
                                    const float* beta, hc_act act, void* y, hc_stream_t stream);
 
 /*
+ * hc_conv_rulebook_transpose -- the Eq. 4 mapping read backwards, for the
+ * input gradient: for every input row j, the taps (n, l) with
+ * rulebook[l][n] == j, n < *count, as keys n*L + l in ascending order.
+ *   rulebook  [L, capacity] from hc_conv_rulebook (capacity = its stride)
+ *   row_ptr   [x_rows + 1] int32: row j's keys are taps[row_ptr[j] ..
+ *             row_ptr[j+1])
+ *   taps      [L * capacity] int32
+ * Entries outside [-1, x_rows) are skipped and reported
+ * (HC_ERR_INVALID_INDEX). Computed once per mask and reused by every layer.
+ * Uses the library's per-stream workspace (2 int32 per input row).
+ */
+hc_status hc_conv_rulebook_transpose(const int32_t* rulebook, const int32_t* count, int capacity,
+                                     int L, int x_rows, int32_t* row_ptr, int32_t* taps,
+                                     hc_stream_t stream);
+
+/*
+ * hc_sparse_conv_rulebook_bwd -- gradients of the sparse spiral convolution
+ * computed by hc_sparse_conv_rulebook_fwd. The paper gives the forward only
+ * (Eqs. 4-5, 6, 10); these follow from it by the chain rule:
+ *   dz[n][o]  = dy[n][o] * act'(y[n][o])   (ELU: 1 if y > 0 else y + 1;
+ *                                           ReLU: 1 if y > 0 else 0)
+ *   dbias[o]  = sum_n dz[n][o]
+ *   dW[l*C_in + c][o] = sum_n x[j(n,l)][c] * dz[n][o]
+ *   dx[j][c]  = sum over taps (n, l) reading row j of sum_o dz[n][o] W[l*C_in + c][o]
+ * over output rows n < *count, with j(n,l) = rulebook[l][n] (absent taps -1
+ * contribute nothing).
+ *   x        [x_rows, C_in] input rows the forward read (dense B*V rows or
+ *            compact), dtype dt; needed for dW
+ *   y, dy    [capacity, C_out] forward output and upstream gradient, dt
+ *   W        [L*C_in, C_out], dt; needed for dx
+ *   row_ptr, taps  from hc_conv_rulebook_transpose; needed for dx
+ *   dx       [x_rows, C_in], dt, every row written (0 where no tap reads
+ *            it), or NULL
+ *   dW       [L*C_in, C_out] fp32 or NULL;  dbias [C_out] fp32 or NULL
+ * bf16: dW on tensor cores (tcgen05, fp32 accumulation); dz and the
+ * per-tap products dz W^T are rounded to bf16 once before the input-gradient
+ * sums. fp32: CUDA cores throughout. Every sum runs in a fixed order
+ * (deterministic). Uses the library's per-stream workspace.
+ */
+hc_status hc_sparse_conv_rulebook_bwd(const void* x, hc_dtype dt, int x_rows,
+                                      const int32_t* rulebook, const int32_t* count, int capacity,
+                                      int L, int C_in, int C_out, const void* W, const void* y,
+                                      const void* dy, hc_act act, const int32_t* row_ptr,
+                                      const int32_t* taps, void* dx, float* dW, float* dbias,
+                                      hc_stream_t stream);
+
+/*
  * hc_mask_score_update -- the mask-score update of Eq. 3 (Sec. 3.1, Sparse
  * Mask Selection). O holds the outputs of K masks, [K, N, D] row-major (mask
  * k's N rows of D features). With S[i][k] = || O_i^T O_k ||_F^2:

@@ -94,6 +94,19 @@ static bool misaligned(const void* p, size_t a) {
     return ((uintptr_t)p) % a != 0;
 }
 
+// Conv kernels: tensor cores when supported (bf16, 16-byte aligned rows),
+// CUDA cores otherwise or when HC_FORCE_SIMT=1.
+hc_status dispatch_conv(const DeviceCtx* ctx, ConvArgs& a, hc_dtype dt, cudaStream_t s) {
+    static int force_simt = -1;
+    if (force_simt < 0) {
+        const char* e = getenv("HC_FORCE_SIMT");
+        force_simt = (e && e[0] == '1') ? 1 : 0;
+    }
+    a.status = ctx->status;
+    if (!force_simt && conv_tc_supported(a, dt)) return launch_conv_tc(ctx, a, s);
+    return launch_conv_simt(ctx, a, dt, s);
+}
+
 }  // namespace hc
 
 using namespace hc;
@@ -147,17 +160,6 @@ static hc_status check_conv_common(const char* fn, hc_dtype dt, int L, int C_in,
     HC_REQUIRE(!misaligned(x, eb) && !misaligned(W, eb) && !misaligned(y, eb),
                "%s: x, W, y must be aligned to the element size", fn);
     return HC_OK;
-}
-
-static hc_status dispatch_conv(const DeviceCtx* ctx, ConvArgs& a, hc_dtype dt, cudaStream_t s) {
-    static int force_simt = -1;
-    if (force_simt < 0) {
-        const char* e = getenv("HC_FORCE_SIMT");
-        force_simt = (e && e[0] == '1') ? 1 : 0;
-    }
-    a.status = ctx->status;
-    if (!force_simt && conv_tc_supported(a, dt)) return launch_conv_tc(ctx, a, s);
-    return launch_conv_simt(ctx, a, dt, s);
 }
 
 hc_status hc_sparse_spiral_conv_fwd(const void* x, hc_layout x_layout, hc_dtype dt,
@@ -352,6 +354,91 @@ hc_status hc_sparse_group_norm_fwd(const void* x, hc_dtype dt, const int32_t* ba
     if (!ctx) return HC_ERR_CUDA;
     return launch_group_norm(ctx, x, dt, batch_offsets, B, capacity, C, G, eps, gamma, beta,
                              (int)act, y, (cudaStream_t)stream);
+}
+
+hc_status hc_conv_rulebook_transpose(const int32_t* rulebook, const int32_t* count, int capacity,
+                                     int L, int x_rows, int32_t* row_ptr, int32_t* taps,
+                                     hc_stream_t stream) {
+    const char* fn = "hc_conv_rulebook_transpose";
+    t_last_error[0] = 0;
+    HC_REQUIRE(L >= 1 && L <= HC_MAX_SPIRAL, "%s: L=%d must be in [1, %d]", fn, L, HC_MAX_SPIRAL);
+    HC_REQUIRE(capacity >= 0 && x_rows >= 0, "%s: capacity=%d x_rows=%d must be >= 0", fn,
+               capacity, x_rows);
+    HC_REQUIRE((long long)capacity * L < (1ll << 31), "%s: capacity*L must be < 2^31", fn);
+    HC_REQUIRE(rulebook && count && row_ptr && (taps || capacity == 0),
+               "%s: rulebook, count, row_ptr and taps are required", fn);
+    const DeviceCtx* ctx = device_ctx();
+    if (!ctx) return HC_ERR_CUDA;
+    if (x_rows == 0)
+        return check_cuda(cudaMemsetAsync(row_ptr, 0, sizeof(int32_t), (cudaStream_t)stream),
+                          "cudaMemsetAsync(row_ptr)");
+    return launch_rulebook_transpose(ctx, rulebook, count, capacity, L, x_rows, row_ptr, taps,
+                                     (cudaStream_t)stream);
+}
+
+hc_status hc_sparse_conv_rulebook_bwd(const void* x, hc_dtype dt, int x_rows,
+                                      const int32_t* rulebook, const int32_t* count, int capacity,
+                                      int L, int C_in, int C_out, const void* W, const void* y,
+                                      const void* dy, hc_act act, const int32_t* row_ptr,
+                                      const int32_t* taps, void* dx, float* dW, float* dbias,
+                                      hc_stream_t stream) {
+    const char* fn = "hc_sparse_conv_rulebook_bwd";
+    t_last_error[0] = 0;
+    HC_REQUIRE(dt == HC_F32 || dt == HC_BF16, "%s: unknown dtype %d", fn, (int)dt);
+    HC_REQUIRE(act == HC_ACT_NONE || act == HC_ACT_ELU || act == HC_ACT_RELU,
+               "%s: unknown activation %d", fn, (int)act);
+    HC_REQUIRE(C_in >= 1 && C_out >= 1 && L >= 1, "%s: L=%d C_in=%d C_out=%d must be >= 1", fn, L,
+               C_in, C_out);
+    if (L > HC_MAX_SPIRAL) {
+        set_error("%s: L=%d exceeds HC_MAX_SPIRAL=%d", fn, L, HC_MAX_SPIRAL);
+        return HC_ERR_UNSUPPORTED;
+    }
+    HC_REQUIRE(capacity >= 0 && x_rows >= 0, "%s: capacity=%d x_rows=%d must be >= 0", fn,
+               capacity, x_rows);
+    HC_REQUIRE((long long)capacity * L < (1ll << 31) && (long long)L * C_in < (1ll << 31),
+               "%s: capacity*L and L*C_in must be < 2^31", fn);
+    HC_REQUIRE(rulebook && count && y && dy, "%s: rulebook, count, y and dy are required", fn);
+    HC_REQUIRE(!dW || x, "%s: x is required for dW", fn);
+    HC_REQUIRE(!dx || (W && row_ptr && taps), "%s: W, row_ptr and taps are required for dx", fn);
+    const size_t eb = dt == HC_F32 ? 4 : 2;
+    HC_REQUIRE(!misaligned(x, eb) && !misaligned(W, eb) && !misaligned(y, eb) &&
+                   !misaligned(dy, eb) && !misaligned(dx, eb),
+               "%s: x, W, y, dy, dx must be aligned to the element size", fn);
+    const DeviceCtx* ctx = device_ctx();
+    if (!ctx) return HC_ERR_CUDA;
+    cudaStream_t s = (cudaStream_t)stream;
+    if (capacity == 0) {  // no output rows: every gradient is zero
+        hc_status st = HC_OK;
+        if (dx && x_rows > 0)
+            st = check_cuda(cudaMemsetAsync(dx, 0, eb * (size_t)x_rows * C_in, s), "cudaMemsetAsync");
+        if (st == HC_OK && dW)
+            st = check_cuda(cudaMemsetAsync(dW, 0, sizeof(float) * (size_t)L * C_in * C_out, s),
+                            "cudaMemsetAsync");
+        if (st == HC_OK && dbias)
+            st = check_cuda(cudaMemsetAsync(dbias, 0, sizeof(float) * (size_t)C_out, s),
+                            "cudaMemsetAsync");
+        return st;
+    }
+    BwdArgs b{};
+    b.x = x;
+    b.dt = dt;
+    b.x_rows = x_rows;
+    b.rulebook = rulebook;
+    b.count = count;
+    b.capacity = capacity;
+    b.L = L;
+    b.C_in = C_in;
+    b.C_out = C_out;
+    b.W = W;
+    b.y = y;
+    b.dy = dy;
+    b.act = (int)act;
+    b.row_ptr = row_ptr;
+    b.taps = taps;
+    b.dx = x_rows > 0 ? dx : nullptr;
+    b.dW = dW;
+    b.dbias = dbias;
+    return launch_conv_bwd(ctx, b, s);
 }
 
 hc_status hc_mask_score_update(const void* O, hc_dtype dt, int K, int N, int D,

@@ -85,6 +85,30 @@ hc_status launch_group_norm(const DeviceCtx* ctx, const void* x, hc_dtype dt,
                             const int32_t* offsets, int B, long long capacity, int C, int G,
                             float eps, const float* gamma, const float* beta, int act, void* y,
                             cudaStream_t s);
+// Backward of the sparse conv through a rulebook (see bwd.cu).
+struct BwdArgs {
+    const void* x;
+    hc_dtype dt;
+    int x_rows;
+    const int32_t* rulebook;  // [L, capacity]
+    const int32_t* count;
+    int capacity;
+    int L, C_in, C_out;
+    const void* W;
+    const void* y;
+    const void* dy;
+    int act;
+    const int32_t* row_ptr;  // transposed mapping (needed for dx)
+    const int32_t* taps;
+    void* dx;
+    float* dW;
+    float* dbias;
+};
+hc_status dispatch_conv(const DeviceCtx* ctx, ConvArgs& a, hc_dtype dt, cudaStream_t s);
+hc_status launch_conv_bwd(const DeviceCtx* ctx, const BwdArgs& b, cudaStream_t s);
+hc_status launch_rulebook_transpose(const DeviceCtx* ctx, const int32_t* rb, const int32_t* count,
+                                    int capacity, int L, int x_rows, int32_t* ptr, int32_t* taps,
+                                    cudaStream_t s);
 hc_status launch_mask_score(const DeviceCtx* ctx, const void* O, hc_dtype dt, int K, long long N,
                             int D, const float* alpha_in, float* alpha_out, float* sim,
                             cudaStream_t s);

@@ -31,7 +31,8 @@ STATUS_NAMES = {0: "HC_OK", 1: "HC_ERR_INVALID_ARG", 2: "HC_ERR_UNSUPPORTED",
 EXPORTS = ("hc_mask_compact", "hc_mask_compact_static", "hc_sparse_spiral_conv_fwd",
            "hc_conv_rulebook", "hc_sparse_conv_rulebook_fwd", "hc_sparse_linear_fwd",
            "hc_sparse_group_norm_fwd", "hc_mask_score_update", "hc_mask_select_topk",
-           "hc_kappa_masks", "hc_gather_rows", "hc_scatter_dense", "hc_spiral_conv_fwd", "hc_get_device_status",
+           "hc_kappa_masks", "hc_gather_rows", "hc_conv_rulebook_transpose",
+           "hc_sparse_conv_rulebook_bwd", "hc_scatter_dense", "hc_spiral_conv_fwd", "hc_get_device_status",
            "hc_last_error_string", "hc_version")
 
 
@@ -66,6 +67,9 @@ def load_library(path: str | None = None):
             "hc_sparse_linear_fwd": [P, I, P, I, I, I, P, P, I, P, P],
             "hc_sparse_group_norm_fwd": [P, I, P, I, I, I, I, ctypes.c_float, P, P, I, P, P],
             "hc_mask_score_update": [P, I, I, I, I, P, P, P, P],
+            "hc_conv_rulebook_transpose": [P, P, I, I, I, P, P, P],
+            "hc_sparse_conv_rulebook_bwd": [P, I, I, P, P, I, I, I, I, P, P, P, I, P, P, P, P, P,
+                                            P],
             "hc_mask_select_topk": [P, I, I, P, P],
             "hc_kappa_masks": [P, I, I, P, I, I, P, P],
             "hc_gather_rows": [P, I, I, I, I, P, P, I, I, P, P],
@@ -186,6 +190,29 @@ def hc_sparse_group_norm_fwd(x, batch_offsets, G, eps, gamma, beta, act, y, stre
     _check(load_library().hc_sparse_group_norm_fwd(
         _p(x), _dt(x), _p(batch_offsets), B, capacity, C, G, float(eps), _p(gamma), _p(beta),
         act, _p(y), _s(stream)), "hc_sparse_group_norm_fwd")
+
+
+def hc_conv_rulebook_transpose(rulebook, count, x_rows, row_ptr, taps, stream=None):
+    """Taps reading each input row (keys n*L + l, ascending) from a rulebook [L, capacity]."""
+    L, capacity = rulebook.shape
+    _check(load_library().hc_conv_rulebook_transpose(_p(rulebook), _p(count), capacity, L, x_rows,
+                                                     _p(row_ptr), _p(taps), _s(stream)),
+           "hc_conv_rulebook_transpose")
+
+
+def hc_sparse_conv_rulebook_bwd(x, rulebook, count, W, y, dy, act, row_ptr=None, taps=None,
+                                dx=None, dW=None, dbias=None, stream=None):
+    """Gradients of the rulebook conv. x [x_rows, C_in] (or [B, V, C_in]);
+    y, dy [capacity, C_out]; dx like x (or None); dW [L*C_in, C_out] and
+    dbias [C_out] fp32 (or None)."""
+    L, capacity = rulebook.shape
+    C_in = x.shape[-1]
+    x_rows = x.numel() // C_in
+    C_out = W.shape[1]
+    _check(load_library().hc_sparse_conv_rulebook_bwd(
+        _p(x), _dt(x), x_rows, _p(rulebook), _p(count), capacity, L, C_in, C_out, _p(W), _p(y),
+        _p(dy), act, _p(row_ptr), _p(taps), _p(dx), _p(dW), _p(dbias), _s(stream)),
+        "hc_sparse_conv_rulebook_bwd")
 
 
 def hc_mask_score_update(O, alpha_in, alpha_out, sim=None, stream=None):
