@@ -369,11 +369,12 @@ def run_ours(args, rank, world, local_rank):
 
     e2e = measure_e2e(torch, hc, sets, w, spiral, Wt, bias, stream, dev, args.e2e_steps)
 
-    sweep = gnorm = mscore = None
+    sweep = gnorm = mscore = bwd = None
     if not args.no_extras and rank == 0:
         sweep = run_sweep(torch, hc, dev, stream)
         gnorm = run_group_norm(torch, hc, sets, dev, stream)
         mscore = run_mask_score(torch, hc, dev, stream)
+        bwd = run_backward(torch, hc, sets[1], w, spiral, Wt, dev, stream)
 
     # Aggregate over ranks: rows summed, time = max over ranks.
     tot_rows, max_ms = reduce_over_ranks(float(rows_timed), ms, world, dev)
@@ -444,6 +445,8 @@ def run_ours(args, rank, world, local_rank):
         line["group_norm"] = gnorm
     if mscore is not None:
         line["mask_score"] = mscore
+    if bwd is not None:
+        line["backward"] = bwd
     return line
 
 
@@ -697,6 +700,67 @@ def run_mask_score(torch, hc, dev, stream, K=10):
         raise RuntimeError(f"device status {hc.STATUS_NAMES.get(st)} in the mask score")
     torch.cuda.empty_cache()
     return out
+
+
+def run_backward(torch, hc, s, w, spiral, Wt, dev, stream):
+    """Backward of the bench layer (one input set: its mask, rulebook and
+    forward output), with an upstream gradient drawn on the device:
+    the transposed mapping (once per mask), then the full backward (input,
+    weight and bias gradients), and its weight-gradient and input-gradient
+    parts alone. Weight-gradient roofline: 2 * N' * L*C_in * C_out flops."""
+    pk = peaks()
+    ly = w.layers[0]
+    B, V, L = w.B, w.V, w.L
+    cap = B * V
+    K = L * ly.C_in
+    g = torch.Generator(device=dev)
+    g.manual_seed(4321)
+    dy = torch.randn((cap, ly.C_out), generator=g, device=dev).to(torch.bfloat16)
+    x = s.x.view(cap, ly.C_in)
+    row_ptr = torch.empty(cap + 1, dtype=torch.int32, device=dev)
+    taps = torch.empty(L * cap, dtype=torch.int32, device=dev)
+    dx = torch.empty_like(x)
+    dW = torch.empty((K, ly.C_out), device=dev)
+    db = torch.empty(ly.C_out, device=dev)
+
+    def transpose():
+        hc.hc_conv_rulebook_transpose(s.rb, s.count, cap, row_ptr, taps, stream)
+
+    def bwd(dx_, dW_, db_):
+        return lambda: hc.hc_sparse_conv_rulebook_bwd(x, s.rb, s.count, Wt, s.y, dy, ly.act,
+                                                      row_ptr, taps, dx_, dW_, db_, stream)
+
+    def timeit(fn, reps=20):
+        with torch.cuda.stream(stream):
+            fn()
+            gr = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(gr, stream=stream):
+                for _ in range(reps):
+                    fn()
+            gr.replay()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            gr.replay()
+            e1.record(stream)
+        torch.cuda.synchronize(dev)
+        return e0.elapsed_time(e1) / reps * 1e3
+
+    t_tr = timeit(transpose)
+    t_all = timeit(bwd(dx, dW, db))
+    t_w = timeit(bwd(None, dW, None))
+    t_x = timeit(bwd(dx, None, None))
+    st = hc.hc_get_device_status(stream)
+    if st != hc.HC_OK:
+        raise RuntimeError(f"device status {hc.STATUS_NAMES.get(st)} in the backward")
+    flops = 2.0 * s.rows * K * ly.C_out
+    tf = flops / (t_w * 1e-6) / 1e12
+    return {"workload": WORKLOAD, "active_rows": s.rows, "dtype": "bf16",
+            "transpose_us": t_tr, "bwd_us": t_all, "wgrad_part_us": t_w, "dgrad_part_us": t_x,
+            "wgrad_tflops": tf, "wgrad_tensor_frac": tf / pk["bf16_tflops"],
+            "kernels": "act_bwd + wgrad_tc_kernel (tcgen05 split-K) + wgrad_reduce; "
+                       "W^T + linear conv (dz W^T) + dgrad gather-sum",
+            "peak": f"{pk['bf16_tflops']} TFLOP/s ({pk['source']} bf16 burst)"}
 
 
 def cpu_baseline(w, budget_s=20.0):

@@ -16,7 +16,8 @@
 //                       materialised once), then every input row sums the P
 //                       slices of the taps that read it, in (n, l) order,
 //                       from the transposed mapping (rb_* kernels: counts,
-//                       exclusive scan, fill, per-row sort).
+//                       exclusive scan, fill, per-row sort), a warp per 32
+//                       rows where the channel chunks allow it.
 #include <cuda_bf16.h>
 
 #include "hc_internal.cuh"
@@ -61,9 +62,10 @@ __device__ __forceinline__ long long clamp_rows(const int32_t* count, long long 
 
 // ---------------------------------------------------------------- dz, dbias
 // Block (64, 4): thread (tx, ty) takes columns g*64 + tx of rows r0 + ty +
-// 4 i of the block's row range; the four row lanes' sums meet in shared
-// memory and the block writes one partial per column.
-constexpr int kActRowsPerBlock = 64;
+// 4 i of the block's row chunks (chunks blockIdx.x, + gridDim.x, ...); the
+// four row lanes' sums meet in shared memory and the block writes one
+// partial per column.
+constexpr int kActRowsPerBlock = 16;
 
 template <typename T>
 __global__ void __launch_bounds__(256)
@@ -75,22 +77,34 @@ __global__ void __launch_bounds__(256)
     pdl_trigger();
     const long long rows = clamp_rows(count, capacity, status);
     const int tx = threadIdx.x & 63, ty = threadIdx.x >> 6;
-    const long long r0 = (long long)blockIdx.x * kActRowsPerBlock;
-    long long r1 = r0 + kActRowsPerBlock;
-    if (r1 > rows) r1 = rows;
     for (int g0 = 0; g0 < C_out; g0 += 64) {
         const int o = g0 + tx;
         float sum = 0.f;
         if (o < C_out)
-            for (long long r = r0 + ty; r < r1; r += 4) {
-                const long long e = r * C_out + o;
-                const float yv = to_f(y[e]);
-                float d = 1.f;
-                if (act == HC_ACT_ELU) d = yv > 0.f ? 1.f : yv + 1.f;
-                else if (act == HC_ACT_RELU) d = yv > 0.f ? 1.f : 0.f;
-                const float v = to_f(dy[e]) * d;
-                dz[e] = from_f<T>(v);
-                sum += v;
+            for (long long r0 = (long long)blockIdx.x * kActRowsPerBlock; r0 < rows;
+                 r0 += (long long)gridDim.x * kActRowsPerBlock) {
+                const long long r1 = r0 + kActRowsPerBlock < rows ? r0 + kActRowsPerBlock : rows;
+                for (long long rb0 = r0 + ty; rb0 < r1; rb0 += 16) {
+                    // four rows' loads in flight, then their arithmetic
+                    float yv[4], gv[4];
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        const long long r = rb0 + 4 * i;
+                        yv[i] = r < r1 ? to_f(y[r * C_out + o]) : 0.f;
+                        gv[i] = r < r1 ? to_f(dy[r * C_out + o]) : 0.f;
+                    }
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        const long long r = rb0 + 4 * i;
+                        if (r >= r1) continue;
+                        float d = 1.f;
+                        if (act == HC_ACT_ELU) d = yv[i] > 0.f ? 1.f : yv[i] + 1.f;
+                        else if (act == HC_ACT_RELU) d = yv[i] > 0.f ? 1.f : 0.f;
+                        const float v = gv[i] * d;
+                        dz[r * C_out + o] = from_f<T>(v);
+                        sum += v;
+                    }
+                }
             }
         red[ty][tx] = sum;
         __syncthreads();
@@ -100,15 +114,25 @@ __global__ void __launch_bounds__(256)
     }
 }
 
+// dbias: block (32, 32) per 32 columns; row lane ty adds partials ty,
+// ty + 32, ... and the 32 lane sums are added in order.
 __global__ void dbias_kernel(const float* __restrict__ bpart, int nblocks, int C_out,
                              float* __restrict__ dbias) {
+    __shared__ float red[32][33];
     pdl_wait();
     pdl_trigger();
-    const int o = blockIdx.x * blockDim.x + threadIdx.x;
-    if (o >= C_out) return;
+    const int o = blockIdx.x * 32 + threadIdx.x;
     float s = 0.f;
-    for (int b = 0; b < nblocks; ++b) s += bpart[(long long)b * C_out + o];
-    dbias[o] = s;
+    if (o < C_out)
+        for (int b = threadIdx.y; b < nblocks; b += 32) s += bpart[(long long)b * C_out + o];
+    red[threadIdx.y][threadIdx.x] = s;
+    __syncthreads();
+    if (threadIdx.y == 0 && o < C_out) {
+        float t = 0.f;
+#pragma unroll 8
+        for (int i = 0; i < 32; ++i) t += red[i][threadIdx.x];
+        dbias[o] = t;
+    }
 }
 
 // W [K, C_out] -> W^T [C_out, K]
@@ -257,23 +281,49 @@ __global__ void rb_fill_kernel(const int32_t* __restrict__ rb, const int32_t* co
     }
 }
 
-// Within each row the fill order depends on timing: sort it (rows hold
-// about L entries; insertion sort).
+__device__ __forceinline__ void insertion_sort(int32_t* taps, int a, int b) {
+    for (int i = a + 1; i < b; ++i) {
+        const int key = taps[i];
+        int k = i - 1;
+        while (k >= a && taps[k] > key) {
+            taps[k + 1] = taps[k];
+            --k;
+        }
+        taps[k + 1] = key;
+    }
+}
+
+// Within each row the fill order depends on timing: sort it. Warp w takes
+// rows w, w + nwarps, ..., 32 at a time (row ranges in one load). A row of
+// up to 32 keys (about L) is sorted by rank: lane i holds key i and counts
+// the smaller keys by shuffles (keys are unique), then writes its key at
+// that rank. Longer rows are insertion-sorted in place by one lane.
 __global__ void rb_sort_kernel(const int32_t* __restrict__ ptr, int x_rows,
                                int32_t* __restrict__ taps) {
     pdl_wait();
     pdl_trigger();
-    for (long long j = blockIdx.x * (long long)blockDim.x + threadIdx.x; j < x_rows;
-         j += (long long)gridDim.x * blockDim.x) {
-        const int a = ptr[j], b = ptr[j + 1];
-        for (int i = a + 1; i < b; ++i) {
-            const int key = taps[i];
-            int k = i - 1;
-            while (k >= a && taps[k] > key) {
-                taps[k + 1] = taps[k];
-                --k;
+    const int lane = threadIdx.x & 31;
+    const long long nwarps = (long long)gridDim.x * (blockDim.x >> 5);
+    const long long w = (long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    for (long long q0 = 0; w + q0 * nwarps < x_rows; q0 += 32) {
+        const long long jl = w + (q0 + lane) * nwarps;
+        const bool have = jl < x_rows;
+        const int pa = have ? ptr[jl] : 0, pb = have ? ptr[jl + 1] : 0;
+        for (unsigned todo = __ballot_sync(0xffffffffu, have && pb - pa > 1); todo;
+             todo &= todo - 1) {
+            const int r = __ffs(todo) - 1;
+            const int a = __shfl_sync(0xffffffffu, pa, r), b = __shfl_sync(0xffffffffu, pb, r);
+            const int len = b - a;
+            if (len <= 32) {
+                const int key = lane < len ? taps[a + lane] : 0x7fffffff;
+                int rank = 0;
+#pragma unroll
+                for (int k = 0; k < 32; ++k) rank += __shfl_sync(0xffffffffu, key, k) < key;
+                if (lane < len) taps[a + rank] = key;
+            } else if (lane == 0) {
+                insertion_sort(taps, a, b);
             }
-            taps[k + 1] = key;
+            __syncwarp();
         }
     }
 }
@@ -306,17 +356,32 @@ __global__ void dgrad_kernel(const T* __restrict__ P, const int32_t* __restrict_
             if (c == 0) report(status, kErrIndex);
             b = a;
         }
-        for (int e = a; e < b; ++e) {
-            const int key = __ldg(taps + e);
-            if (key < 0 || (long long)key >= capacity * L) {
-                if (c == 0) report(status, kErrIndex);
-                continue;
-            }
-            const int n = key / L, l = key - n * L;
-            const U raw = *reinterpret_cast<const U*>(P + n * prow + (long long)l * C_in + c);
-            const T* v = reinterpret_cast<const T*>(&raw);
+        // a batch of keys, then all their P chunks in flight, then the sums
+        // (in key order)
+        constexpr int kBatchTaps = 4;
+        for (int e0 = a; e0 < b; e0 += kBatchTaps) {
+            int key[kBatchTaps];
 #pragma unroll
-            for (int k = 0; k < VEC; ++k) acc[k] += to_f(v[k]);
+            for (int i = 0; i < kBatchTaps; ++i) key[i] = e0 + i < b ? __ldg(taps + e0 + i) : -1;
+            U raw[kBatchTaps];
+#pragma unroll
+            for (int i = 0; i < kBatchTaps; ++i) {
+                if (e0 + i >= b) continue;
+                if (key[i] < 0 || (long long)key[i] >= capacity * L) {
+                    if (c == 0) report(status, kErrIndex);
+                    key[i] = -1;
+                    continue;
+                }
+                const int n = key[i] / L, l = key[i] - n * L;
+                raw[i] = *reinterpret_cast<const U*>(P + n * prow + (long long)l * C_in + c);
+            }
+#pragma unroll
+            for (int i = 0; i < kBatchTaps; ++i) {
+                if (e0 + i >= b || key[i] < 0) continue;
+                const T* v = reinterpret_cast<const T*>(&raw[i]);
+#pragma unroll
+                for (int k = 0; k < VEC; ++k) acc[k] += to_f(v[k]);
+            }
         }
         U out;
         T* ov = reinterpret_cast<T*>(&out);
@@ -347,9 +412,8 @@ struct WgradArgs {
     const void* dz;
     long long capacity;
     int x_rows, L, C_in, C_out, K;  // K = L * C_in
-    int m_tiles, n_tiles, T, splits;
-    long long rows_per_split;  // multiple of kBK
-    float* part;               // [splits * T][128][128]
+    int m_tiles, n_tiles, T, splits;  // rows split on the device, from *count
+    float* part;                      // [splits * T][128][128]
     unsigned* status;
 };
 
@@ -408,8 +472,10 @@ __global__ void __launch_bounds__(kThreadsTc, 1) wgrad_tc_kernel(const WgradArgs
     const int split = item / a.T;
     const int tile = item - split * a.T;
     const int tm = tile / a.n_tiles, tn = tile - tm * a.n_tiles;
-    const long long r_begin = (long long)split * a.rows_per_split;
-    long long r_end = r_begin + a.rows_per_split;
+    // the active rows (known on the device) split evenly, in kBK blocks
+    const long long rps = ((rows + a.splits - 1) / a.splits + kBK - 1) / kBK * kBK;
+    const long long r_begin = (long long)split * rps;
+    long long r_end = r_begin + rps;
     if (r_end > rows) r_end = rows;
     const int num_kb = r_end > r_begin ? (int)((r_end - r_begin + kBK - 1) / kBK) : 0;
 
@@ -540,8 +606,9 @@ __global__ void __launch_bounds__(256) wgrad_simt_kernel(const WgradArgs a) {
     const int split = item / a.T;
     const int tile = item - split * a.T;
     const int tm = tile / a.n_tiles, tn = tile - tm * a.n_tiles;
-    const long long r_begin = (long long)split * a.rows_per_split;
-    long long r_end = r_begin + a.rows_per_split;
+    const long long rps = ((rows + a.splits - 1) / a.splits + kBKs - 1) / kBKs * kBKs;
+    const long long r_begin = (long long)split * rps;
+    long long r_end = r_begin + rps;
     if (r_end > rows) r_end = rows;
     const int t = threadIdx.x, ty = t >> 4, tx = t & 15;
     const int mm = t & (kTile - 1);
@@ -617,6 +684,96 @@ __global__ void wgrad_reduce_kernel(const float* __restrict__ part, int K, int C
     }
 }
 
+// Rows whose 16-byte chunk count cpr divides 32: warp w takes rows w,
+// w + nwarps, ..., 32 at a time. Their row ranges come in one load (lane r
+// holds row r's); a ballot splits them into rows without taps, written as
+// zeros G rows per store, and rows with taps, for which lane
+// (g, c) = (lane / cpr, lane % cpr) sums chunk c of taps g, g + G, ...
+// (G = 32 / cpr groups, keys then P chunks loaded four at a time) and the
+// groups are added by a fixed shuffle tree.
+template <typename T>
+__global__ void __launch_bounds__(256)
+    dgrad_warp_kernel(const T* __restrict__ P, const int32_t* __restrict__ ptr,
+                      const int32_t* __restrict__ taps, int x_rows, int L, int C_in,
+                      long long capacity, T* __restrict__ dx, unsigned* status) {
+    constexpr int VEC = 16 / sizeof(T);
+    pdl_wait();
+    pdl_trigger();
+    const int lane = threadIdx.x & 31;
+    const int cpr = C_in / VEC, G = 32 / cpr;
+    const int g = lane / cpr, c = (lane - g * cpr) * VEC;
+    const long long prow = (long long)L * C_in;
+    const long long nwarps = (long long)gridDim.x * (blockDim.x >> 5);
+    const long long w = (long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    // rows w, w + nwarps, w + 2 nwarps, ...: clustered active rows spread
+    // over all warps instead of loading a few
+    for (long long q0 = 0; w + q0 * nwarps < x_rows; q0 += 32) {
+        const long long jl = w + (q0 + lane) * nwarps;
+        const bool have = jl < x_rows;
+        const int pa = have ? __ldg(ptr + jl) : 0;
+        const int pb = have ? __ldg(ptr + jl + 1) : 0;
+        const long long left = (x_rows - 1 - w) / nwarps + 1 - q0;  // rows left for this warp
+        const int nr = left < 32 ? (int)left : 32;
+        // rows without taps: zeros, G rows per store instruction
+        const unsigned busy = __ballot_sync(0xffffffffu, have && pb != pa);
+        for (int r0 = 0; r0 < nr; r0 += G) {
+            const int r = r0 + g;
+            if (r < nr && !((busy >> r) & 1u))
+                *reinterpret_cast<uint4*>(dx + (w + (q0 + r) * nwarps) * C_in + c) =
+                    make_uint4(0u, 0u, 0u, 0u);
+        }
+        // rows with taps
+        for (unsigned todo = busy; todo; todo &= todo - 1) {
+            const int r = __ffs(todo) - 1;
+            const long long j = w + (q0 + r) * nwarps;
+            int a = __shfl_sync(0xffffffffu, pa, r), b = __shfl_sync(0xffffffffu, pb, r);
+            if (a < 0 || b < a || (long long)b > capacity * L) {
+                if (lane == 0) report(status, kErrIndex);
+                b = a;
+            }
+            float acc[VEC];
+#pragma unroll
+            for (int k = 0; k < VEC; ++k) acc[k] = 0.f;
+            for (int e0 = a + g; e0 < b; e0 += 4 * G) {
+                int key[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const int e = e0 + i * G;
+                    key[i] = e < b ? __ldg(taps + e) : -1;
+                    if (e < b && (key[i] < 0 || (long long)key[i] >= capacity * L)) {
+                        report(status, kErrIndex);
+                        key[i] = -1;
+                    }
+                }
+                uint4 raw[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    if (key[i] < 0) continue;
+                    const int n = key[i] / L, l = key[i] - n * L;
+                    raw[i] = *reinterpret_cast<const uint4*>(P + n * prow + (long long)l * C_in + c);
+                }
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    if (key[i] < 0) continue;
+                    const T* v = reinterpret_cast<const T*>(&raw[i]);
+#pragma unroll
+                    for (int k = 0; k < VEC; ++k) acc[k] += to_f(v[k]);
+                }
+            }
+            for (int o = cpr; o < 32; o <<= 1)
+#pragma unroll
+                for (int k = 0; k < VEC; ++k) acc[k] += __shfl_xor_sync(0xffffffffu, acc[k], o);
+            if (g == 0) {
+                uint4 out;
+                T* ov = reinterpret_cast<T*>(&out);
+#pragma unroll
+                for (int k = 0; k < VEC; ++k) ov[k] = from_f<T>(acc[k]);
+                *reinterpret_cast<uint4*>(dx + j * C_in + c) = out;
+            }
+        }
+    }
+}
+
 template <typename T>
 hc_status launch_dgrad_typed(const DeviceCtx* ctx, const void* P, const int32_t* ptr,
                              const int32_t* taps, int x_rows, int L, int C_in, long long capacity,
@@ -625,6 +782,15 @@ hc_status launch_dgrad_typed(const DeviceCtx* ctx, const void* P, const int32_t*
     const int vec16 = 16 / (int)sizeof(T);
     const bool wide = C_in % vec16 == 0 && al % 16 == 0;
     const int vec = wide ? vec16 : 1;
+    const int cpr = C_in / vec16;
+    if (wide && cpr <= 32 && (32 % cpr) == 0) {
+        long long wblocks = ((long long)x_rows + 255) / 256;  // 8 warps x 32 rows per block
+        if (wblocks > (long long)ctx->num_sms * 8) wblocks = (long long)ctx->num_sms * 8;
+        if (wblocks < 1) wblocks = 1;
+        return launch_pdl(dgrad_warp_kernel<T>, dim3((unsigned)wblocks), dim3(256), 0, s,
+                          "dgrad_warp_kernel", (const T*)P, ptr, taps, x_rows, L, C_in, capacity,
+                          (T*)dx, ctx->status);
+    }
     long long blocks = ((long long)x_rows * (C_in / vec) + 255) / 256;
     const long long cap = (long long)ctx->num_sms * 8;
     if (blocks > cap) blocks = cap;
@@ -703,11 +869,10 @@ hc_status launch_conv_bwd(const DeviceCtx* ctx, const BwdArgs& b, cudaStream_t s
             if (eff >= 0.95) break;
         }
     }
-    long long rps = ((long long)b.capacity + splits - 1) / splits;
-    rps = (rps + kBK - 1) / kBK * kBK;
-    if (rps < kBK) rps = kBK;
     const long long items = (long long)splits * T;
-    const int act_blocks = (int)(((long long)b.capacity + kActRowsPerBlock - 1) / kActRowsPerBlock);
+    long long act_blocks_ll = ((long long)b.capacity + kActRowsPerBlock - 1) / kActRowsPerBlock;
+    if (act_blocks_ll > 8ll * ctx->num_sms) act_blocks_ll = 8ll * ctx->num_sms;
+    const int act_blocks = (int)(act_blocks_ll > 0 ? act_blocks_ll : 1);
 
     // workspace: dz | P | W^T | wgrad partials | dbias partials
     auto up = [](size_t v) { return (v + 255) / 256 * 256; };
@@ -736,7 +901,7 @@ hc_status launch_conv_bwd(const DeviceCtx* ctx, const BwdArgs& b, cudaStream_t s
                         (long long)b.capacity, b.C_out, b.act, (float*)dz, bpart, ctx->status);
     if (st != HC_OK) return st;
     if (b.dbias) {
-        st = launch_pdl(dbias_kernel, dim3((unsigned)((b.C_out + 127) / 128)), dim3(128), 0, s,
+        st = launch_pdl(dbias_kernel, dim3((unsigned)((b.C_out + 31) / 32)), dim3(32, 32), 0, s,
                         "dbias_kernel", (const float*)bpart, act_blocks, b.C_out, b.dbias);
         if (st != HC_OK) return st;
     }
@@ -757,7 +922,6 @@ hc_status launch_conv_bwd(const DeviceCtx* ctx, const BwdArgs& b, cudaStream_t s
         w.n_tiles = n_tiles;
         w.T = T;
         w.splits = splits;
-        w.rows_per_split = rps;
         w.part = part;
         w.status = ctx->status;
         const bool tc = bf && b.C_in % 8 == 0 && b.C_out % 8 == 0 && (uintptr_t)b.x % 16 == 0;

@@ -130,6 +130,29 @@ def test_rulebook_transpose_bit_exact():
                                   np.concatenate([sorted(v) for v in lists]).astype(np.int32))
 
 
+def test_rulebook_transpose_long_rows():
+    """A synthetic mapping whose entries land on 10 input rows (hundreds of
+    taps per row, past the 32 a warp sorts at once), with absent taps."""
+    rng = np.random.default_rng(3)
+    L, cap, n, x_rows = 6, 500, 431, 10
+    rb_np = rng.integers(-1, x_rows, size=(L, cap)).astype(np.int32)
+    rb = to_torch(rb_np)
+    count = torch.tensor([n], dtype=torch.int32, device="cuda")
+    row_ptr = torch.empty(x_rows + 1, dtype=torch.int32, device="cuda")
+    taps = torch.full((L * cap,), -7, dtype=torch.int32, device="cuda")
+    hc.hc_conv_rulebook_transpose(rb, count, x_rows, row_ptr, taps)
+    assert hc.hc_get_device_status() == hc.HC_OK
+    lists = [[] for _ in range(x_rows)]
+    for l in range(L):
+        for r in range(n):
+            if rb_np[l, r] >= 0:
+                lists[rb_np[l, r]].append(r * L + l)
+    ref_ptr = np.concatenate([[0], np.cumsum([len(v) for v in lists])])
+    np.testing.assert_array_equal(to_numpy(row_ptr), ref_ptr)
+    np.testing.assert_array_equal(to_numpy(taps)[:ref_ptr[-1]],
+                                  np.concatenate([sorted(v) for v in lists]).astype(np.int32))
+
+
 @pytest.mark.parametrize("dtype", ["bf16", "f32"])
 @pytest.mark.parametrize("layout", [oracle.LAYOUT_DENSE, oracle.LAYOUT_COMPACT])
 @pytest.mark.parametrize("shape", [(3, 200, 9, 16, 64), (2, 333, 12, 64, 128),
