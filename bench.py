@@ -51,7 +51,11 @@ def parse_args():
     p.add_argument("--steps", type=int, default=400)
     p.add_argument("--warmup", type=int, default=10)
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    p.add_argument("--no-extras", action="store_true", help="skip the density sweep")
+    p.add_argument("--no-extras", action="store_true",
+                   help="skip the side measurements (density sweep, group norm, mask score, "
+                        "backward)")
+    p.add_argument("--extra", choices=["all", "sweep", "group_norm", "mask_score", "backward"],
+                   default="all", help="run only this side measurement")
     p.add_argument("--clocks-csv", default=None, help="also write the raw clock samples here")
     p.add_argument("--e2e-steps", type=int, default=30)
     return p.parse_args()
@@ -371,10 +375,15 @@ def run_ours(args, rank, world, local_rank):
 
     sweep = gnorm = mscore = bwd = None
     if not args.no_extras and rank == 0:
-        sweep = run_sweep(torch, hc, dev, stream)
-        gnorm = run_group_norm(torch, hc, sets, dev, stream)
-        mscore = run_mask_score(torch, hc, dev, stream)
-        bwd = run_backward(torch, hc, sets[1], w, spiral, Wt, dev, stream)
+        want = lambda name: args.extra in ("all", name)  # noqa: E731
+        if want("sweep"):
+            sweep = run_sweep(torch, hc, dev, stream)
+        if want("group_norm"):
+            gnorm = run_group_norm(torch, hc, sets, dev, stream)
+        if want("mask_score"):
+            mscore = run_mask_score(torch, hc, dev, stream)
+        if want("backward"):
+            bwd = run_backward(torch, hc, sets[1], w, spiral, Wt, dev, stream)
 
     # Aggregate over ranks: rows summed, time = max over ranks.
     tot_rows, max_ms = reduce_over_ranks(float(rows_timed), ms, world, dev)

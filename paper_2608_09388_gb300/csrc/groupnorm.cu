@@ -648,13 +648,14 @@ hc_status launch_typed(const DeviceCtx* ctx, const void* x, const int32_t* offse
     const uintptr_t al = (uintptr_t)x | (uintptr_t)y;
     const bool aligned = C % kVec == 0 && al % 16 == 0;
     const int cpr = C / kVec;
-    // Small frames: when the average frame's group slice fits the per-thread
-    // register cache of the per-(frame, group) kernel and there are enough
-    // (frame, group) blocks to fill the GPU, that single launch (one read,
-    // one write, no workspace) beats the two latency-bound row-range launches.
+    // Small frames: when the average frame's group slice is within twice
+    // the per-thread register cache of the per-(frame, group) kernel (the
+    // rest re-read from L2) and there are enough (frame, group) blocks to
+    // fill the GPU, that single launch beats the two latency-bound row-range
+    // launches.
     const long long avg_chunks = (capacity + B - 1) / B * (long long)(cpg / kVec);
     const bool small_frames = cpg % kVec == 0 && aligned &&
-                              avg_chunks <= (long long)kThreads * kBatch &&
+                              avg_chunks <= 2ll * kThreads * kBatch &&
                               (long long)B * G >= ctx->num_sms;
     // HC_GN_SLICE forces the per-(frame, group) kernel, HC_GN_ROWS the
     // row-range kernels where the layout allows (to test both on any shape)
