@@ -210,6 +210,22 @@ __global__ void __launch_bounds__(kThreads, 1)
     pdl_wait();
     pdl_trigger();
 
+    // Rulebook mode: the index warp copies its first tile's entries into tap
+    // table 0 (cp.async, no registers held) before the row count arrives
+    // (rows clamped to the capacity, always valid memory), so the two L2
+    // round trips overlap instead of queueing.
+    const bool prefetched = warp == kIndexWarp && a.mode == kRulebook;
+    if (prefetched) {
+        const long long m0p = (blockIdx.x / ((a.C_out + BN - 1) / BN)) * (long long)kBM;
+        for (int d = 0; d < a.L; ++d)
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const long long n = m0p + lane + 32 * i;
+                cp_async_4(tab0 + (uint32_t)(d * kBM + lane + 32 * i) * 4u,
+                           a.rulebook + (long long)d * a.capacity + (n < a.capacity ? n : 0), true);
+            }
+    }
+
     const long long rows = active_rows(a);
     const long long m_tiles = (rows + kBM - 1) / kBM;
     const int n_tiles = (a.C_out + BN - 1) / BN;
@@ -217,6 +233,27 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int num_kb = (a.K + kBK - 1) / kBK;
     const int L = a.L, C_in = a.C_in, C_out = a.C_out, K = a.K;
     const uint32_t tab_bytes = (uint32_t)(kBM * L) * 4u;
+    if (prefetched) {
+        // the first tap table (buffer 0, not yet waited on by anyone): the
+        // copied entries checked against the input's rows and masked by the
+        // row count
+        cp_async_wait_all();
+        const long long m0 = (blockIdx.x / n_tiles) * (long long)kBM;
+        unsigned err = 0;
+        for (int d = 0; d < L; ++d)
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const uint32_t at = tab0 + (uint32_t)(d * kBM + lane + 32 * i) * 4u;
+                const int ev = lds_s32(at);
+                int src = -1;
+                if (m0 + lane + 32 * i < rows) {
+                    if (ev < -1 || ev >= a.x_rows) err |= kErrIndex;
+                    else src = ev;
+                }
+                sts_s32(at, src);
+            }
+        if (err) report(a.status, err);
+    }
 
     if (warp < kProducerWarps) {
         // ------------------------------------------------------------ producers
@@ -437,9 +474,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             unsigned err = 0;
             if (a.mode == kRulebook) {
                 // Precomputed mapping: one coalesced pass over the tile's
-                // rulebook columns, entries checked against the input's rows.
+                // rulebook columns, entries checked against the input's rows
+                // (the first tile's table was filled before the loop).
                 constexpr int kRbChunk = 12;
-                for (int l0 = 0; l0 < L; l0 += kRbChunk) {
+                for (int l0 = 0; l0 < L && lt > 0; l0 += kRbChunk) {
                     int e[4][kRbChunk];
 #pragma unroll
                     for (int i = 0; i < 4; ++i)
@@ -563,11 +601,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int n0 = (int)(w % n_tiles) * BN;
             const int acc = lt & 1;
             const uint32_t ph = (uint32_t)((lt >> 1) & 1);
-            if (!mbar_wait(tfull_bar(acc), ph, abort_flag, a.status)) break;
-            tc_fence_after();
+            // Everything that does not need the accumulator is loaded while
+            // the main loop runs: this lane's row addresses (0 = not
+            // written; the fused scatter's needs the row's coordinate) and
+            // the bias of each 32-column chunk (lane j holds column j's).
             const long long row = m0 + ew * 32 + lane;
             const bool rvalid = row < rows;
-            // Row start addresses (0 = not written) of this lane's row.
             const long long row_y = (rvalid && y) ? (long long)(y + row * C_out) : 0;
             long long row_d = 0;
             if (rvalid && a.out_dense) {
@@ -578,6 +617,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                 else
                     report(a.status, kErrIndex);
             }
+            float bias_c[BN / 32];
+#pragma unroll
+            for (int cb = 0; cb < BN / 32; ++cb) {
+                const int bcol = n0 + cb * 32 + lane < C_out ? n0 + cb * 32 + lane : C_out - 1;
+                bias_c[cb] = a.bias ? __ldg(a.bias + bcol) : 0.f;
+            }
+            if (!mbar_wait(tfull_bar(acc), ph, abort_flag, a.status)) break;
+            tc_fence_after();
             const uint32_t stage = epi0 + (uint32_t)ew * 2048u;
 #pragma unroll 1
             for (int cb = 0; cb < BN / 32; ++cb) {
@@ -586,10 +633,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                                    r);
                 tmem_ld_wait();
                 const int col0 = n0 + cb * 32;
-                // Bias of the chunk's 32 columns: one coalesced load, then
-                // broadcast by shuffles (every lane takes part).
-                const int bcol = col0 + lane < C_out ? col0 + lane : C_out - 1;
-                const float bias_l = a.bias ? __ldg(a.bias + bcol) : 0.f;
+                // Bias of the chunk's 32 columns (loaded above), broadcast by
+                // shuffles (every lane takes part).
+                float bias_l = bias_c[0];
+#pragma unroll
+                for (int k = 1; k < BN / 32; ++k)
+                    if (cb == k) bias_l = bias_c[k];
 #pragma unroll
                 for (int j = 0; j < 32; ++j)
                     r[j] = __float_as_uint(__uint_as_float(r[j]) +
