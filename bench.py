@@ -54,7 +54,8 @@ def parse_args():
     p.add_argument("--no-extras", action="store_true",
                    help="skip the side measurements (density sweep, group norm, mask score, "
                         "backward)")
-    p.add_argument("--extra", choices=["all", "sweep", "group_norm", "mask_score", "backward"],
+    p.add_argument("--extra", choices=["all", "sweep", "group_norm", "mask_score", "backward",
+                                       "kappa"],
                    default="all", help="run only this side measurement")
     p.add_argument("--clocks-csv", default=None, help="also write the raw clock samples here")
     p.add_argument("--e2e-steps", type=int, default=30)
@@ -373,7 +374,7 @@ def run_ours(args, rank, world, local_rank):
 
     e2e = measure_e2e(torch, hc, sets, w, spiral, Wt, bias, stream, dev, args.e2e_steps)
 
-    sweep = gnorm = mscore = bwd = None
+    sweep = gnorm = mscore = bwd = kap = None
     if not args.no_extras and rank == 0:
         want = lambda name: args.extra in ("all", name)  # noqa: E731
         if want("sweep"):
@@ -384,6 +385,8 @@ def run_ours(args, rank, world, local_rank):
             mscore = run_mask_score(torch, hc, dev, stream)
         if want("backward"):
             bwd = run_backward(torch, hc, sets[1], w, spiral, Wt, dev, stream)
+        if want("kappa"):
+            kap = run_kappa(torch, hc, dev, stream)
 
     # Aggregate over ranks: rows summed, time = max over ranks.
     tot_rows, max_ms = reduce_over_ranks(float(rows_timed), ms, world, dev)
@@ -456,6 +459,8 @@ def run_ours(args, rank, world, local_rank):
         line["mask_score"] = mscore
     if bwd is not None:
         line["backward"] = bwd
+    if kap is not None:
+        line["kappa_inference"] = kap
     return line
 
 
@@ -770,6 +775,92 @@ def run_backward(torch, hc, s, w, spiral, Wt, dev, stream):
             "kernels": "act_bwd + wgrad_tc_kernel (tcgen05 split-K) + wgrad_reduce; "
                        "W^T + linear conv (dz W^T) + dgrad gather-sum",
             "peak": f"{pk['bf16_tflops']} TFLOP/s ({pk['source']} bf16 burst)"}
+
+
+def run_kappa(torch, hc, dev, stream, K=10, kappa=3, density=0.1):
+    """Inference with kappa kept masks (Sec. 3.1; kappa = 3 of K = 10 as in
+    Sec. 4) on the 4-layer bf16 encoder (64 samples of the 655-vertex sphere,
+    16 -> 64 -> 64 -> 64 -> 64 + linear 64 -> 42): top-kappa by the mask
+    score, every kept mask on every sample (192 frames), compaction, the Eq. 4
+    mapping, the S' rows of Eq. 2 gathered from the samples, the four sparse
+    conv layers and the head, all on compact rows. Against the same encoder
+    run densely on every vertex of the 64 samples."""
+    from paper_2608_09388_gb300 import inputs
+    w = inputs.make_workload("encoder655_bf16")
+    B, V, L = w.B, w.V, w.L
+    F = B * kappa
+    rng = np.random.default_rng(inputs.SEEDS["encoder655_bf16"] + 77)
+    masks = torch.from_numpy(inputs.uniform_mask(rng, K, V, density)).to(dev)
+    alpha = torch.from_numpy(rng.standard_normal(K).astype(np.float32)).to(dev)
+    x = torch.from_numpy(w.x.view(np.int16)).view(torch.bfloat16).to(dev)
+    sp = torch.from_numpy(w.spiral).to(dev)
+    Ws = [torch.from_numpy(ly.W.view(np.int16)).view(torch.bfloat16).to(dev) for ly in w.layers]
+    bs = [torch.from_numpy(ly.b).to(dev) for ly in w.layers]
+    sel = torch.empty(kappa, dtype=torch.int32, device=dev)
+    fm = torch.empty((F, V), dtype=torch.uint8, device=dev)
+    coords = torch.empty((F * V, 2), dtype=torch.int32, device=dev)
+    row_of = torch.empty((F, V), dtype=torch.int32, device=dev)
+    offs = torch.empty(F + 1, dtype=torch.int32, device=dev)
+    count = torch.empty(1, dtype=torch.int32, device=dev)
+    rb = torch.empty((L, F * V), dtype=torch.int32, device=dev)
+    hs = [torch.empty((F * V, ly.C_in), dtype=torch.bfloat16, device=dev) for ly in w.layers]
+    out = torch.empty((F * V, w.layers[-1].C_out), dtype=torch.bfloat16, device=dev)
+    dense_h = [torch.empty((B, V, ly.C_out), dtype=torch.bfloat16, device=dev) for ly in w.layers]
+
+    def sparse():
+        hc.hc_mask_select_topk(alpha, kappa, sel, stream)
+        hc.hc_kappa_masks(masks, sel, B, fm, stream)
+        hc.hc_mask_compact(fm, coords, row_of, offs, count, stream)
+        hc.hc_conv_rulebook(coords, row_of, count, sp, F, V, hc.HC_LAYOUT_COMPACT, rb, stream)
+        hc.hc_gather_rows(x, coords, count, kappa, hs[0], stream)
+        for i, ly in enumerate(w.layers):
+            dst = hs[i + 1] if i + 1 < len(w.layers) else out
+            if ly.kind == "conv":
+                hc.hc_sparse_conv_rulebook_fwd(hs[i], rb, count, Ws[i], bs[i], ly.act, dst,
+                                               stream=stream)
+            else:
+                hc.hc_sparse_linear_fwd(hs[i], count, Ws[i], bs[i], ly.act, dst, stream)
+
+    def dense():
+        h = x
+        for i, ly in enumerate(w.layers):
+            if ly.kind == "conv":
+                hc.hc_spiral_conv_fwd(h, sp, Ws[i], bs[i], ly.act, dense_h[i], stream)
+            else:
+                hc.hc_sparse_linear_fwd(h.view(B * V, -1), full, Ws[i], bs[i], ly.act,
+                                        dense_h[i].view(B * V, -1), stream)
+            h = dense_h[i]
+
+    full = torch.tensor([B * V], dtype=torch.int32, device=dev)
+
+    def timeit(fn, reps=20):
+        with torch.cuda.stream(stream):
+            fn()
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                for _ in range(reps):
+                    fn()
+            g.replay()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            g.replay()
+            e1.record(stream)
+        torch.cuda.synchronize(dev)
+        return e0.elapsed_time(e1) / reps * 1e3
+
+    t_sparse = timeit(sparse)
+    t_dense = timeit(dense)
+    st = hc.hc_get_device_status(stream)
+    if st != hc.HC_OK:
+        raise RuntimeError(f"device status {hc.STATUS_NAMES.get(st)} in the kappa inference")
+    n = int(count.item())
+    return {"K": K, "kappa": kappa, "samples": B, "frames": F, "V": V, "mask_density": density,
+            "active_rows": n, "layers": "4 sparse spiral convs 16-64-64-64-64 + linear 64->42",
+            "us": t_sparse, "rows_per_s": n / (t_sparse * 1e-6),
+            "dense_encoder_us": t_dense, "speedup_vs_dense": t_dense / t_sparse,
+            "chain": "topk + kappa masks + compaction + Eq. 4 mapping + S' gather + 4 convs + "
+                     "linear head (compact rows throughout)"}
 
 
 def cpu_baseline(w, budget_s=20.0):
