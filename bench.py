@@ -380,7 +380,7 @@ def run_ours(args, rank, world, local_rank):
         if want("sweep"):
             sweep = run_sweep(torch, hc, dev, stream)
         if want("group_norm"):
-            gnorm = run_group_norm(torch, hc, sets, dev, stream)
+            gnorm = run_group_norm(torch, hc, sets, dev, stream, Wt, bias)
         if want("mask_score"):
             mscore = run_mask_score(torch, hc, dev, stream)
         if want("backward"):
@@ -600,12 +600,15 @@ def run_sweep(torch, hc, dev, stream):
     return out
 
 
-def run_group_norm(torch, hc, sets, dev, stream, G=8):
+def run_group_norm(torch, hc, sets, dev, stream, Wt, bias, G=8):
     """Sparse group norm (Eqs. 7-9), G = 8, affine + ELU, on two inputs:
     the bench layer's compact conv outputs (rotating over the input sets;
     they sit in L2 as they would right after the conv) and a fully active
     64 x 10475 x 128 bf16 activation (171 MB, larger than L2). Algorithmic
-    bytes: every active element read once and written once."""
+    bytes: every active element read once and written once. Then the whole
+    layer conv -> group norm -> ELU on the rotating sets: the convolution
+    alone (no activation), the two calls, and hc_sparse_conv_gn_fwd (group
+    statistics from the convolution's epilogue)."""
     pk = peaks()
     C = sets[0].y.shape[1]
     gamma = torch.linspace(0.5, 1.5, C, device=dev)
@@ -649,6 +652,27 @@ def run_group_norm(torch, hc, sets, dev, stream, G=8):
                            "hbm_frac": nbytes / (ms * 1e-3) / 1e9 / pk["hbm_gbs"],
                            "kernels": "group_norm_slice_kernel (one block per frame and group)",
                            "note": "compact conv outputs of the bench layer, L2-resident"}
+    def conv(s):
+        return lambda: hc.hc_sparse_conv_rulebook_fwd(s.x, s.rb, s.count, Wt, bias,
+                                                      hc.HC_ACT_NONE, s.gn, stream=stream)
+
+    def fused(s):
+        return lambda: hc.hc_sparse_conv_gn_fwd(s.x, s.rb, s.count, Wt, bias, s.coords, s.offs,
+                                                G, 1e-5, gamma, beta, hc.HC_ACT_ELU, s.gn,
+                                                stream)
+
+    layer = {"rows": rows, "C_out": C,
+             "note": "rotating input sets, inputs larger than L2 over a rotation"}
+    layer["conv_us"] = timeit([conv(s) for s in sets], 10) * 1e3
+    # conv then group norm in place: two calls, three launches
+    layer["two_calls_us"] = timeit([f for s in sets for f in (conv(s), gn(s.gn[:s.rows], s.offs,
+                                                                         s.gn[:s.rows]))],
+                                   10) * 2e3
+    layer["fused_us"] = timeit([fused(s) for s in sets], 10) * 1e3
+    layer["gn_added_us"] = {"two_calls": layer["two_calls_us"] - layer["conv_us"],
+                            "fused": layer["fused_us"] - layer["conv_us"]}
+    layer["kernels"] = "conv_tc_kernel (statistics in the epilogue) + gn_apply_kernel"
+    out["conv_layer"] = layer
     for s in sets:
         del s.gn
     Bl, Vl = 64, 10475

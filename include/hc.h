@@ -227,6 +227,36 @@ hc_status hc_sparse_group_norm_fwd(const void* x, hc_dtype dt, const int32_t* ba
                                    const float* beta, hc_act act, void* y, hc_stream_t stream);
 
 /*
+ * hc_sparse_conv_gn_fwd -- a convolution layer followed by group
+ * normalisation and the activation, the order of a block of the encoder
+ * (Eqs. 5-6, then Eqs. 7-9, then Eq. 10):
+ *   z = conv(x) + bias            as hc_sparse_conv_rulebook_fwd with act
+ *                                 NONE, stored in y (dtype dt)
+ *   y = act(GN(z) * gamma + beta) as hc_sparse_group_norm_fwd on y in place
+ * The group statistics are those of z as stored (bf16-rounded for bf16).
+ *   x, rulebook, count, capacity, L, C_in, C_out, W, bias as for
+ *             hc_sparse_conv_rulebook_fwd; y [capacity, C_out] of dtype dt
+ *   coords    [capacity, 2] int32 from hc_mask_compact (frame of row n is
+ *             coords[2n]), batch_offsets [B+1] from the same call: the frame
+ *             table must start at 0, end at *count and agree with coords
+ *             (HC_ERR_INVALID_INDEX otherwise, output unspecified)
+ *   G, eps, gamma, beta, act as for hc_sparse_group_norm_fwd (G divides C_out)
+ * bf16 with C_out/G a multiple of 8 dividing the tensor-core tile (64
+ * channels when C_out <= 64, else 128), C_out/8 a power of two: the
+ * tensor-core epilogue writes one partial (count, mean, M2) per (frame,
+ * 32-row block, group) and a single normalising pass reads them (two
+ * launches, y written once by each). Otherwise the two operations run one
+ * after the other. Uses the library's per-stream workspace
+ * ((B + capacity/32 + 1) * G * 16 bytes, or that of hc_sparse_group_norm_fwd).
+ */
+hc_status hc_sparse_conv_gn_fwd(const void* x, hc_dtype dt, int x_rows, const int32_t* rulebook,
+                                const int32_t* count, int capacity, int L, int C_in, int C_out,
+                                const void* W, const float* bias, const int32_t* coords,
+                                const int32_t* batch_offsets, int B, int G, float eps,
+                                const float* gamma, const float* beta, hc_act act, void* y,
+                                hc_stream_t stream);
+
+/*
  * hc_conv_rulebook_transpose -- the Eq. 4 mapping read backwards, for the
  * input gradient: for every input row j, the taps (n, l) with
  * rulebook[l][n] == j, n < *count, as keys n*L + l in ascending order.

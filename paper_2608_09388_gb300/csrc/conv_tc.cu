@@ -112,23 +112,25 @@ __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr, uint32_t lbo
 // rows x 64 contiguous bytes, instead of 32 scattered 16-byte pieces. Each
 // row goes to its compact position (row_y, 0 = none) and to its dense
 // position of the fused scatter (row_d, 0 = none).
+// Activation and bf16 rounding of a chunk: p[h] holds columns 2h (low
+// half) and 2h + 1 (high half).
 template <int ACT>
-__device__ __forceinline__ void epilogue_chunk(const uint32_t (&r)[32], uint32_t stage, int lane,
+__device__ __forceinline__ void epilogue_pack(const uint32_t (&r)[32], uint32_t (&p)[16]) {
+#pragma unroll
+    for (int h = 0; h < 16; ++h) {
+        const __nv_bfloat162 b = __floats2bfloat162_rn(act_fixed<ACT>(__uint_as_float(r[2 * h])),
+                                                       act_fixed<ACT>(__uint_as_float(r[2 * h + 1])));
+        p[h] = *reinterpret_cast<const uint32_t*>(&b);
+    }
+}
+
+__device__ __forceinline__ void epilogue_store(const uint32_t (&p)[16], uint32_t stage, int lane,
                                                long long row_y, long long row_d, int col0,
                                                int C_out) {
 #pragma unroll
-    for (int j8 = 0; j8 < 4; ++j8) {
-        uint32_t packed[4];
-#pragma unroll
-        for (int h = 0; h < 4; ++h) {
-            const int j = j8 * 8 + 2 * h;
-            const __nv_bfloat162 p = __floats2bfloat162_rn(act_fixed<ACT>(__uint_as_float(r[j])),
-                                                           act_fixed<ACT>(__uint_as_float(r[j + 1])));
-            packed[h] = *reinterpret_cast<const uint32_t*>(&p);
-        }
+    for (int j8 = 0; j8 < 4; ++j8)
         sts_v4(stage + (uint32_t)(lane * 64 + ((j8 ^ ((lane >> 1) & 3)) << 4)),
-               make_uint4(packed[0], packed[1], packed[2], packed[3]));
-    }
+               make_uint4(p[4 * j8], p[4 * j8 + 1], p[4 * j8 + 2], p[4 * j8 + 3]));
     __syncwarp();
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
@@ -143,6 +145,189 @@ __device__ __forceinline__ void epilogue_chunk(const uint32_t (&r)[32], uint32_t
         }
     }
     __syncwarp();  // the buffer is reused by the next chunk
+}
+
+template <int ACT>
+__device__ __forceinline__ void epilogue_chunk(const uint32_t (&r)[32], uint32_t stage, int lane,
+                                               long long row_y, long long row_d, int col0,
+                                               int C_out) {
+    uint32_t p[16];
+    epilogue_pack<ACT>(r, p);
+    epilogue_store(p, stage, lane, row_y, row_d, col0, C_out);
+}
+
+// Group-norm statistics of one warp's 32 rows (lane = row). Every lane
+// holds, per channel group, the mean and M2 of its CPG values of the group;
+// the warp writes one (count, mean, M2) per frame present to slot (frame +
+// block) of the partials, for NG groups g0 .. g0 + ng - 1 at once.
+
+// Column j of a packed chunk (bf16 pairs, column 2h in the low half of
+// p[h]) as fp32.
+__device__ __forceinline__ float bf_col(const uint32_t (&p)[16], int j) {
+    return __uint_as_float((j & 1) ? (p[j >> 1] & 0xffff0000u) : (p[j >> 1] << 16));
+}
+
+// Sum of N consecutive columns j0 .. (squared deviations from m when Sq) by
+// a pairwise tree: log2 N levels of independent additions. j0 is known at
+// compile time after unrolling (the values stay in registers).
+template <int N, bool Sq>
+__device__ __forceinline__ float tree_sum(const uint32_t (&p)[16], int j0, float m = 0.f) {
+    float t[N];
+#pragma unroll
+    for (int i = 0; i < N; ++i) {
+        const float x = bf_col(p, j0 + i);
+        t[i] = Sq ? (x - m) * (x - m) : x;
+    }
+#pragma unroll
+    for (int w = N / 2; w >= 1; w /= 2)
+#pragma unroll
+        for (int i = 0; i < w; ++i) t[i] += t[i + w];
+    return t[0];
+}
+
+// All 32 rows active and in frame fb (most blocks): the lanes hold equal
+// counts, so every butterfly level merges two halves of equal size n by the
+// pairwise update of Chan, Golub and LeVeque: mean = (mean_a + mean_b) / 2,
+// M2 = M2_a + M2_b + d^2 n / 2. Both partners of a level compute the same
+// values (the operations are symmetric in a and b).
+template <int NG>
+__device__ __forceinline__ void gn_flush_whole(const ConvArgs& a, long long block, int fb, int g0,
+                                               int ng, float n, float (&mean)[NG],
+                                               float (&m2)[NG], int lane) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+#pragma unroll
+        for (int q = 0; q < NG; ++q) {
+            const float mb = __shfl_xor_sync(0xffffffffu, mean[q], o);
+            const float qb = __shfl_xor_sync(0xffffffffu, m2[q], o);
+            const float d = mb - mean[q];
+            m2[q] = (m2[q] + qb) + d * d * (0.5f * n);
+            mean[q] = (mean[q] + mb) * 0.5f;
+        }
+        n *= 2.f;
+    }
+    if (lane == 0) {
+#pragma unroll
+        for (int q = 0; q < NG; ++q)
+            if (q < ng)
+                *reinterpret_cast<float4*>(a.gn_part + 4 * ((fb + block) * a.gn_G + g0 + q)) =
+                    make_float4(n, mean[q], m2[q], 0.f);
+    }
+}
+
+// Rows that straddle a frame boundary or the last active row (gn_b = the
+// lane's frame, -1 past the active rows): for each frame present, two
+// passes over its lanes (each with cpg values per group): the frame mean
+// from the sum of lane means, then M2 = sum over lanes of (lane M2 + cpg *
+// (lane mean - frame mean)^2), which is exact. Non-member lanes add 0.
+template <int NG>
+__device__ __forceinline__ void gn_flush_runs(const ConvArgs& a, long long block, int gn_b, int g0,
+                                              int ng, float cpg, const float (&mean)[NG],
+                                              const float (&m2)[NG], int lane) {
+    unsigned todo = __ballot_sync(0xffffffffu, gn_b >= 0);
+    while (todo) {
+        const int leader = __ffs(todo) - 1;
+        const int fb = __shfl_sync(0xffffffffu, gn_b, leader);
+        const bool mem = gn_b == fb;
+        const unsigned members = __ballot_sync(0xffffffffu, mem);
+        const float cnt = (float)__popc(members);
+        float fm[NG], fq[NG];
+#pragma unroll
+        for (int q = 0; q < NG; ++q) fm[q] = mem ? mean[q] : 0.f;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+            for (int q = 0; q < NG; ++q) fm[q] += __shfl_xor_sync(0xffffffffu, fm[q], o);
+#pragma unroll
+        for (int q = 0; q < NG; ++q) {
+            fm[q] = fm[q] / cnt;
+            const float d = mean[q] - fm[q];
+            fq[q] = mem ? fmaf(cpg * d, d, m2[q]) : 0.f;
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+            for (int q = 0; q < NG; ++q) fq[q] += __shfl_xor_sync(0xffffffffu, fq[q], o);
+        if (lane == leader) {
+#pragma unroll
+            for (int q = 0; q < NG; ++q)
+                if (q < ng)
+                    *reinterpret_cast<float4*>(a.gn_part + 4 * ((fb + block) * a.gn_G + g0 + q)) =
+                        make_float4(cnt * cpg, fm[q], fq[q], 0.f);
+        }
+        todo &= ~members;
+    }
+}
+
+// Statistics of one 32-column chunk (columns col0 .. col0 + 31) as stored
+// (v: the packed bf16 values) for groups of CPG <= 32 channels, which lie
+// inside the chunk and are flushed at once. whole: all 32 rows active and
+// in one frame.
+template <int CPG>
+__device__ __forceinline__ void gn_chunk(const ConvArgs& a, const uint32_t (&v)[16], int col0,
+                                         long long block, int gn_b, bool whole, int lane) {
+    // the chunk's 32 / CPG groups, two at a time (register pressure)
+    constexpr int NG = 32 / CPG, NB = NG < 2 ? NG : 2;
+    // C_out is a multiple of CPG: the groups in range are whole
+    const int ng = (a.C_out - col0) / CPG < NG ? (a.C_out - col0) / CPG : NG;
+#pragma unroll
+    for (int q0 = 0; q0 < NG; q0 += NB) {
+        if (q0 >= ng) break;
+        float mean[NB], m2[NB];
+#pragma unroll
+        for (int q = 0; q < NB; ++q) {
+            mean[q] = tree_sum<CPG, false>(v, (q0 + q) * CPG) * (1.f / CPG);
+            m2[q] = tree_sum<CPG, true>(v, (q0 + q) * CPG, mean[q]);
+        }
+        const int g0 = col0 / CPG + q0, nb = ng - q0 < NB ? ng - q0 : NB;
+        if (whole)
+            gn_flush_whole<NB>(a, block, gn_b, g0, nb, (float)CPG, mean, m2, lane);
+        else
+            gn_flush_runs<NB>(a, block, gn_b, g0, nb, (float)CPG, mean, m2, lane);
+    }
+}
+
+// The same for groups of cpg = 64 or 128 channels: merged over their chunks
+// in (run_mean, run_m2) and flushed by their last chunk.
+__device__ __forceinline__ void gn_chunk_wide(const ConvArgs& a, const uint32_t (&v)[16], int col0,
+                                              int cpg, long long block, int gn_b, bool whole,
+                                              int lane, float& run_mean, float& run_m2) {
+    const float mean = tree_sum<32, false>(v, 0) * (1.f / 32.f);
+    const float m2 = tree_sum<32, true>(v, 0, mean);
+    // chunk k (from 0) of the group joins 32 values to the 32 k before it:
+    // the pairwise update with n_a = 32 k, n_b = 32
+    const int k = (col0 & (cpg - 1)) >> 5;
+    if (k == 0) {
+        run_mean = mean, run_m2 = m2;
+    } else {
+        const float na = 32.f * k, rr = 1.f / (float)(k + 1), d = mean - run_mean;
+        run_mean = fmaf(d, rr, run_mean);
+        run_m2 += m2 + d * d * na * rr;
+    }
+    if (((col0 + 32) & (cpg - 1)) == 0) {
+        float m1[1] = {run_mean}, q1[1] = {run_m2};
+        const int g = col0 / cpg;
+        if (whole)
+            gn_flush_whole<1>(a, block, gn_b, g, 1, (float)cpg, m1, q1, lane);
+        else
+            gn_flush_runs<1>(a, block, gn_b, g, 1, (float)cpg, m1, q1, lane);
+    }
+}
+
+// The statistics of a chunk for the group width of the call (a power of two
+// from 8 to 128, checked by the launcher), from the values as stored (v:
+// packed bf16).
+__device__ __forceinline__ void gn_stats_chunk(const ConvArgs& a, const uint32_t (&v)[16],
+                                               int col0, long long block, int gn_b, bool whole,
+                                               int lane, float& run_mean, float& run_m2) {
+    switch (a.gn_cpg) {
+        case 8: gn_chunk<8>(a, v, col0, block, gn_b, whole, lane); break;
+        case 16: gn_chunk<16>(a, v, col0, block, gn_b, whole, lane); break;
+        case 32: gn_chunk<32>(a, v, col0, block, gn_b, whole, lane); break;
+        default:
+            gn_chunk_wide(a, v, col0, a.gn_cpg, block, gn_b, whole, lane, run_mean, run_m2);
+            break;
+    }
 }
 
 template <int BN, bool kTma>
@@ -623,6 +808,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int bcol = n0 + cb * 32 + lane < C_out ? n0 + cb * 32 + lane : C_out - 1;
                 bias_c[cb] = a.bias ? __ldg(a.bias + bcol) : 0.f;
             }
+            int gn_b = -1;  // frame of this lane's row, for the group-norm statistics
+            if (a.gn_part && rvalid) {
+                gn_b = __ldg(a.gn_coords + 2 * row);
+                if (gn_b < 0 || gn_b >= a.gn_B) {
+                    report(a.status, kErrIndex);
+                    gn_b = -1;
+                }
+            }
+            // all 32 rows of this warp active and in one frame
+            const int gn_b0 = __shfl_sync(0xffffffffu, gn_b, 0);
+            const bool gn_whole = __all_sync(0xffffffffu, gn_b >= 0 && gn_b == gn_b0);
+            float run_mean = 0.f, run_m2 = 0.f;
             if (!mbar_wait(tfull_bar(acc), ph, abort_flag, a.status)) break;
             tc_fence_after();
             const uint32_t stage = epi0 + (uint32_t)ew * 2048u;
@@ -643,8 +840,16 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int j = 0; j < 32; ++j)
                     r[j] = __float_as_uint(__uint_as_float(r[j]) +
                                            __shfl_sync(0xffffffffu, bias_l, j));
-                // The activation is chosen once per chunk, not per element.
-                if (a.act == HC_ACT_ELU)
+                if (a.gn_part) {
+                    // with statistics the activation is the identity (it
+                    // follows the normalisation)
+                    uint32_t p[16];
+                    epilogue_pack<HC_ACT_NONE>(r, p);
+                    if (col0 < C_out)
+                        gn_stats_chunk(a, p, col0, (m0 + ew * 32) / 32, gn_b, gn_whole, lane,
+                                       run_mean, run_m2);
+                    epilogue_store(p, stage, lane, row_y, row_d, col0, C_out);
+                } else if (a.act == HC_ACT_ELU)
                     epilogue_chunk<HC_ACT_ELU>(r, stage, lane, row_y, row_d, col0, C_out);
                 else if (a.act == HC_ACT_RELU)
                     epilogue_chunk<HC_ACT_RELU>(r, stage, lane, row_y, row_d, col0, C_out);
@@ -753,6 +958,10 @@ bool conv_tc_supported(const ConvArgs& a, hc_dtype dt) {
            a.L <= HC_MAX_SPIRAL;
 }
 
+int conv_tc_tile_n(const ConvArgs& a) {
+    return a.C_out <= 64 ? 64 : 128;
+}
+
 hc_status launch_conv_tc(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s) {
     // The weight slice comes by TMA; HC_NO_TMA=1 selects the all-cp.async
     // producer instead (for comparison).
@@ -762,7 +971,8 @@ hc_status launch_conv_tc(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s
         tma_off = (e && e[0] == '1') ? 1 : 0;
     }
     const bool tma = !tma_off;
-    if (a.C_out <= 64) return tma ? launch_bn<64, true>(ctx, a, s) : launch_bn<64, false>(ctx, a, s);
+    if (conv_tc_tile_n(a) == 64)
+        return tma ? launch_bn<64, true>(ctx, a, s) : launch_bn<64, false>(ctx, a, s);
     return tma ? launch_bn<128, true>(ctx, a, s) : launch_bn<128, false>(ctx, a, s);
 }
 

@@ -33,6 +33,10 @@
 // The general path (one CTA per (frame, group)) serves every other layout,
 // and small frames (a group slice within its register cache), where one
 // launch beats the two latency-bound row-range launches.
+// Partials from the convolution: the tensor-core convolution can write the
+// same (n, mean, M2) partials of its stored output itself, one per (frame b,
+// 32-row block c) in slot b + c (the slot argument above with ranges of 32
+// rows), so that gn_apply_kernel alone finishes the layer.
 // The output may alias the input in both paths. Deterministic, no atomics.
 #include <cuda_bf16.h>
 
@@ -370,7 +374,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     gn_apply_kernel(const T* x, const int32_t* __restrict__ offsets, int B, int C, int G,
                     long long capacity, const GnPart* __restrict__ part, float eps,
                     const float* __restrict__ gamma, const float* __restrict__ beta, int act, T* y,
-                    unsigned* status) {
+                    int part_rows, const int32_t* __restrict__ count, unsigned* status) {
     using CK = Chunk<T, VEC>;
     using Raw = typename CK::Raw;
     static_assert(sizeof(Raw) == 16, "the row-range path moves 16-byte chunks");
@@ -379,6 +383,19 @@ __global__ void __launch_bounds__(kThreads, 2)
     __shared__ int s_off[kThreads + 1];
     pdl_wait();
     pdl_trigger();
+    // part_rows > 0: the partials come per part_rows-row block of the rows
+    // [0, *count) that the convolution wrote; the frame table must cover
+    // exactly those rows, in order (checked here, as the statistics kernel
+    // does otherwise).
+    if (part_rows > 0) {
+        for (long long i = (long long)blockIdx.x * kThreads + threadIdx.x; i < B;
+             i += (long long)gridDim.x * kThreads)
+            if (__ldg(offsets + i + 1) < __ldg(offsets + i)) report(status, kErrIndex);
+        if (__ldg(offsets) != 0 || __ldg(offsets + B) != __ldg(count)) {
+            if (threadIdx.x == 0 && blockIdx.x == 0) report(status, kErrIndex);
+            return;
+        }
+    }
     RangeMap m;
     long long lo, hi;
     if (!range_setup(offsets, B, capacity, status, m, lo, hi)) return;
@@ -397,8 +414,9 @@ __global__ void __launch_bounds__(kThreads, 2)
         // partials of the CTAs that hold frame b: slots b + c, c in [c0, c1]
         // (clamped to the table's span, so a malformed table cannot index
         // outside the workspace)
-        const long long c0 = m.cta_of(f0 > m.off0 ? f0 : m.off0);
-        const long long c1 = m.cta_of((f1 < m.end ? f1 : m.end) - 1);
+        const long long p0 = f0 > m.off0 ? f0 : m.off0, p1 = (f1 < m.end ? f1 : m.end) - 1;
+        const long long c0 = part_rows > 0 ? p0 / part_rows : m.cta_of(p0);
+        const long long c1 = part_rows > 0 ? p1 / part_rows : m.cta_of(p1);
         const GnPart* pb = part + (long long)b * G;
         __syncthreads();  // s_mu / s_inv of the previous segment have been read
         if (c1 - c0 < 8) {
@@ -619,15 +637,19 @@ __global__ void __launch_bounds__(kThreads, 4)
     }
 }
 
-template <typename T, int VEC, int GPC>
-hc_status launch_fast(const DeviceCtx* ctx, const void* x, const int32_t* offsets, int B,
-                      long long capacity, int C, int G, float eps, const float* gamma,
-                      const float* beta, int act, void* y, cudaStream_t s) {
+long long fast_grid(const DeviceCtx* ctx, long long capacity) {
     // ranges of at least ~64 rows; 2 CTAs per SM at most (the kernels' bound)
     long long grid = (capacity + 63) / 64;
     const long long cap = (long long)ctx->num_sms * 2;
     if (grid > cap) grid = cap;
-    if (grid < 1) grid = 1;
+    return grid < 1 ? 1 : grid;
+}
+
+template <typename T, int VEC, int GPC>
+hc_status launch_fast(const DeviceCtx* ctx, const void* x, const int32_t* offsets, int B,
+                      long long capacity, int C, int G, float eps, const float* gamma,
+                      const float* beta, int act, void* y, cudaStream_t s) {
+    const long long grid = fast_grid(ctx, capacity);
     GnPart* part = (GnPart*)stream_workspace(s, sizeof(GnPart) * (size_t)(B + grid) * G);
     if (!part) return HC_ERR_CUDA;
     hc_status st = launch_pdl(gn_stats_kernel<T, VEC, GPC>, dim3((unsigned)grid), dim3(kThreads),
@@ -636,8 +658,10 @@ hc_status launch_fast(const DeviceCtx* ctx, const void* x, const int32_t* offset
     if (st != HC_OK) return st;
     return launch_pdl(gn_apply_kernel<T, VEC, GPC>, dim3((unsigned)grid), dim3(kThreads), 0, s,
                       "gn_apply_kernel", (const T*)x, offsets, B, C, G, capacity,
-                      (const GnPart*)part, eps, gamma, beta, act, (T*)y, ctx->status);
+                      (const GnPart*)part, eps, gamma, beta, act, (T*)y, 0,
+                      (const int32_t*)nullptr, ctx->status);
 }
+
 
 template <typename T>
 hc_status launch_typed(const DeviceCtx* ctx, const void* x, const int32_t* offsets, int B,
@@ -688,6 +712,23 @@ hc_status launch_typed(const DeviceCtx* ctx, const void* x, const int32_t* offse
 }
 
 }  // namespace
+
+bool group_norm_parts_supported(hc_dtype dt, int C, int G, const void* y) {
+    const int cpr = C / 8;
+    return dt == HC_BF16 && C % 8 == 0 && (C / G) % 8 == 0 && (uintptr_t)y % 16 == 0 &&
+           cpr >= 1 && cpr <= kThreads && (cpr & (cpr - 1)) == 0 && G <= kMaxGroupsFast;
+}
+
+hc_status launch_group_norm_apply(const DeviceCtx* ctx, void* y, const int32_t* offsets, int B,
+                                  long long capacity, int C, int G, const float* part,
+                                  int part_rows, const int32_t* count, float eps,
+                                  const float* gamma, const float* beta, int act, cudaStream_t s) {
+    using T = __nv_bfloat16;
+    return launch_pdl(gn_apply_kernel<T, 8, 1>, dim3((unsigned)fast_grid(ctx, capacity)),
+                      dim3(kThreads), 0, s, "gn_apply_kernel", (const T*)y, offsets, B, C, G,
+                      capacity, (const GnPart*)part, eps, gamma, beta, act, (T*)y, part_rows,
+                      count, ctx->status);
+}
 
 hc_status launch_group_norm(const DeviceCtx* ctx, const void* x, hc_dtype dt,
                             const int32_t* offsets, int B, long long capacity, int C, int G,

@@ -96,14 +96,18 @@ static bool misaligned(const void* p, size_t a) {
 
 // Conv kernels: tensor cores when supported (bf16, 16-byte aligned rows),
 // CUDA cores otherwise or when HC_FORCE_SIMT=1.
-hc_status dispatch_conv(const DeviceCtx* ctx, ConvArgs& a, hc_dtype dt, cudaStream_t s) {
+static bool use_conv_tc(const ConvArgs& a, hc_dtype dt) {
     static int force_simt = -1;
     if (force_simt < 0) {
         const char* e = getenv("HC_FORCE_SIMT");
         force_simt = (e && e[0] == '1') ? 1 : 0;
     }
+    return !force_simt && conv_tc_supported(a, dt);
+}
+
+hc_status dispatch_conv(const DeviceCtx* ctx, ConvArgs& a, hc_dtype dt, cudaStream_t s) {
     a.status = ctx->status;
-    if (!force_simt && conv_tc_supported(a, dt)) return launch_conv_tc(ctx, a, s);
+    if (use_conv_tc(a, dt)) return launch_conv_tc(ctx, a, s);
     return launch_conv_simt(ctx, a, dt, s);
 }
 
@@ -354,6 +358,70 @@ hc_status hc_sparse_group_norm_fwd(const void* x, hc_dtype dt, const int32_t* ba
     if (!ctx) return HC_ERR_CUDA;
     return launch_group_norm(ctx, x, dt, batch_offsets, B, capacity, C, G, eps, gamma, beta,
                              (int)act, y, (cudaStream_t)stream);
+}
+
+hc_status hc_sparse_conv_gn_fwd(const void* x, hc_dtype dt, int x_rows, const int32_t* rulebook,
+                                const int32_t* count, int capacity, int L, int C_in, int C_out,
+                                const void* W, const float* bias, const int32_t* coords,
+                                const int32_t* batch_offsets, int B, int G, float eps,
+                                const float* gamma, const float* beta, hc_act act, void* y,
+                                hc_stream_t stream) {
+    const char* fn = "hc_sparse_conv_gn_fwd";
+    t_last_error[0] = 0;
+    hc_status st = check_conv_common(fn, dt, L, C_in, C_out, act, x, W, y);
+    if (st != HC_OK) return st;
+    HC_REQUIRE(x_rows >= 1 && capacity >= 0, "%s: x_rows=%d capacity=%d", fn, x_rows, capacity);
+    HC_REQUIRE(rulebook && count && coords && batch_offsets,
+               "%s: rulebook, count, coords and batch_offsets are required", fn);
+    HC_REQUIRE(B >= 1 && G >= 1 && C_out % G == 0, "%s: B=%d >= 1 and C_out=%d a multiple of G=%d",
+               fn, B, C_out, G);
+    HC_REQUIRE((long long)B * G < (1ll << 31), "%s: B*G=%lld too large", fn, (long long)B * G);
+    HC_REQUIRE(eps >= 0.f, "%s: eps must be >= 0", fn);
+    if (capacity == 0) return HC_OK;
+    const DeviceCtx* ctx = device_ctx();
+    if (!ctx) return HC_ERR_CUDA;
+    cudaStream_t s = (cudaStream_t)stream;
+    ConvArgs a{};
+    a.x = x;
+    a.count = count;
+    a.rulebook = rulebook;
+    a.W = W;
+    a.bias = bias;
+    a.y = y;
+    a.capacity = capacity;
+    a.x_rows = x_rows;
+    a.B = 1;
+    a.V = capacity;
+    a.L = L;
+    a.C_in = C_in;
+    a.C_out = C_out;
+    a.K = L * C_in;
+    a.mode = kRulebook;
+    a.act = HC_ACT_NONE;  // the activation follows the normalisation
+    a.status = ctx->status;
+    const int cpg = C_out / G;
+    // channels per group a power of two from 8 to the tile's width
+    if (use_conv_tc(a, dt) && cpg >= 8 && (cpg & (cpg - 1)) == 0 && cpg <= conv_tc_tile_n(a) &&
+        group_norm_parts_supported(dt, C_out, G, y)) {
+        // statistics from the convolution's epilogue, one partial per
+        // (frame, 32-row block) in slot frame + block
+        const size_t slots = (size_t)B + ((size_t)capacity + 31) / 32;
+        float* part = (float*)stream_workspace(s, 16 * slots * (size_t)G);
+        if (!part) return HC_ERR_CUDA;
+        a.gn_part = part;
+        a.gn_coords = coords;
+        a.gn_G = G;
+        a.gn_B = B;
+        a.gn_cpg = cpg;
+        st = launch_conv_tc(ctx, a, s);
+        if (st != HC_OK) return st;
+        return launch_group_norm_apply(ctx, y, batch_offsets, B, capacity, C_out, G, part, 32,
+                                       count, eps, gamma, beta, (int)act, s);
+    }
+    st = dispatch_conv(ctx, a, dt, s);
+    if (st != HC_OK) return st;
+    return launch_group_norm(ctx, y, dt, batch_offsets, B, capacity, C_out, G, eps, gamma, beta,
+                             (int)act, y, s);
 }
 
 hc_status hc_conv_rulebook_transpose(const int32_t* rulebook, const int32_t* count, int capacity,

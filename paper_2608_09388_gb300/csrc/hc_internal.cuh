@@ -69,6 +69,15 @@ struct ConvArgs {
     int mode;
     int act;
     int stages;  // pipeline depth chosen by the launcher (tensor-core kernel)
+    // Optional group-norm statistics of the stored output (Eqs. 7-9,
+    // tensor-core kernel): every block c of 32 output rows writes, for each
+    // frame b among its rows (b = gn_coords[2n]) and each channel group g of
+    // gn_G, the (count, mean, M2) of its stored values to
+    // gn_part[4 * ((b + c) * gn_G + g)].
+    float* gn_part;
+    const int32_t* gn_coords;
+    int gn_G, gn_B;
+    int gn_cpg;  // channels per group, C_out / gn_G: 8, 16, 32, 64 or 128
 };
 
 // Launchers (each in its own translation unit). All return HC_OK or an
@@ -78,6 +87,7 @@ hc_status launch_compact(const DeviceCtx* ctx, const uint8_t* mask, int B, int V
 hc_status launch_conv_simt(const DeviceCtx* ctx, const ConvArgs& a, hc_dtype dt, cudaStream_t s);
 hc_status launch_conv_tc(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s);
 bool conv_tc_supported(const ConvArgs& a, hc_dtype dt);
+int conv_tc_tile_n(const ConvArgs& a);  // output channels per tensor-core tile
 hc_status launch_rulebook(const DeviceCtx* ctx, const int32_t* coords, const int32_t* row_of,
                           const int32_t* count, const int32_t* spiral, int B, int V, int L,
                           int x_layout, int32_t* rulebook, cudaStream_t s);
@@ -85,6 +95,14 @@ hc_status launch_group_norm(const DeviceCtx* ctx, const void* x, hc_dtype dt,
                             const int32_t* offsets, int B, long long capacity, int C, int G,
                             float eps, const float* gamma, const float* beta, int act, void* y,
                             cudaStream_t s);
+// The normalising pass alone, in place on bf16 y, from partials written per
+// part_rows-row block of the rows [0, *count) (the convolution's); the frame
+// table must start at 0 and end at *count.
+bool group_norm_parts_supported(hc_dtype dt, int C, int G, const void* y);
+hc_status launch_group_norm_apply(const DeviceCtx* ctx, void* y, const int32_t* offsets, int B,
+                                  long long capacity, int C, int G, const float* part,
+                                  int part_rows, const int32_t* count, float eps,
+                                  const float* gamma, const float* beta, int act, cudaStream_t s);
 // Backward of the sparse conv through a rulebook (see bwd.cu).
 struct BwdArgs {
     const void* x;

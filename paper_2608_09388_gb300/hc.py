@@ -30,7 +30,7 @@ STATUS_NAMES = {0: "HC_OK", 1: "HC_ERR_INVALID_ARG", 2: "HC_ERR_UNSUPPORTED",
 # Exported symbols, as declared in include/hc.h.
 EXPORTS = ("hc_mask_compact", "hc_mask_compact_static", "hc_sparse_spiral_conv_fwd",
            "hc_conv_rulebook", "hc_sparse_conv_rulebook_fwd", "hc_sparse_linear_fwd",
-           "hc_sparse_group_norm_fwd", "hc_mask_score_update", "hc_mask_select_topk",
+           "hc_sparse_group_norm_fwd", "hc_sparse_conv_gn_fwd", "hc_mask_score_update", "hc_mask_select_topk",
            "hc_kappa_masks", "hc_gather_rows", "hc_conv_rulebook_transpose",
            "hc_sparse_conv_rulebook_bwd", "hc_scatter_dense", "hc_spiral_conv_fwd", "hc_get_device_status",
            "hc_last_error_string", "hc_version")
@@ -66,6 +66,8 @@ def load_library(path: str | None = None):
                                             P],
             "hc_sparse_linear_fwd": [P, I, P, I, I, I, P, P, I, P, P],
             "hc_sparse_group_norm_fwd": [P, I, P, I, I, I, I, ctypes.c_float, P, P, I, P, P],
+            "hc_sparse_conv_gn_fwd": [P, I, I, P, P, I, I, I, I, P, P, P, P, I, I,
+                                      ctypes.c_float, P, P, I, P, P],
             "hc_mask_score_update": [P, I, I, I, I, P, P, P, P],
             "hc_conv_rulebook_transpose": [P, P, I, I, I, P, P, P],
             "hc_sparse_conv_rulebook_bwd": [P, I, I, P, P, I, I, I, I, P, P, P, I, P, P, P, P, P,
@@ -190,6 +192,22 @@ def hc_sparse_group_norm_fwd(x, batch_offsets, G, eps, gamma, beta, act, y, stre
     _check(load_library().hc_sparse_group_norm_fwd(
         _p(x), _dt(x), _p(batch_offsets), B, capacity, C, G, float(eps), _p(gamma), _p(beta),
         act, _p(y), _s(stream)), "hc_sparse_group_norm_fwd")
+
+
+def hc_sparse_conv_gn_fwd(x, rulebook, count, W, bias, coords, batch_offsets, G, eps, gamma,
+                          beta, act, y, stream=None):
+    """Sparse conv through a rulebook [L, capacity], then group norm per frame
+    (batch_offsets [B+1]) and group of C_out/G channels, then act: y
+    [capacity, C_out]."""
+    L, capacity = rulebook.shape
+    C_in = x.shape[-1]
+    x_rows = x.numel() // C_in
+    C_out = W.shape[1]
+    B = batch_offsets.shape[0] - 1
+    _check(load_library().hc_sparse_conv_gn_fwd(
+        _p(x), _dt(y), x_rows, _p(rulebook), _p(count), capacity, L, C_in, C_out, _p(W),
+        _p(bias), _p(coords), _p(batch_offsets), B, G, float(eps), _p(gamma), _p(beta), act,
+        _p(y), _s(stream)), "hc_sparse_conv_gn_fwd")
 
 
 def hc_conv_rulebook_transpose(rulebook, count, x_rows, row_ptr, taps, stream=None):

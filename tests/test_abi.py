@@ -94,3 +94,22 @@ def test_group_norm_arguments_rejected_on_host(lib):
         assert gn(*args) == hc.HC_ERR_INVALID_ARG
     # nothing to do: returns before any device call
     assert gn(fake, 0, fake, 0, 10, 8, 2, f(1e-5), None, None, 0, fake, None) == hc.HC_OK
+
+
+def test_conv_gn_arguments_rejected_on_host(lib):
+    fake = ctypes.c_void_p(0x1000)
+    f = ctypes.c_float
+    cg = lib.hc_sparse_conv_gn_fwd
+
+    def call(dt=1, x_rows=100, count=fake, capacity=100, L=9, C_in=16, C_out=64, coords=fake,
+             offs=fake, B=2, G=8, eps=1e-5, act=1):
+        return cg(fake, dt, x_rows, fake, count, capacity, L, C_in, C_out, fake, None, coords,
+                  offs, B, G, f(eps), None, None, act, fake, None)
+
+    for kw in (dict(G=7), dict(G=0), dict(B=0), dict(eps=-1.0), dict(dt=5), dict(act=9),
+               dict(coords=None), dict(offs=None), dict(count=None), dict(x_rows=0),
+               dict(capacity=-1), dict(C_out=0)):
+        assert call(**kw) == hc.HC_ERR_INVALID_ARG, kw
+    assert call(L=10 ** 4) == hc.HC_ERR_UNSUPPORTED
+    # nothing to do: returns before any device call
+    assert call(capacity=0) == hc.HC_OK
