@@ -241,13 +241,15 @@ hc_status hc_sparse_group_norm_fwd(const void* x, hc_dtype dt, const int32_t* ba
  *             table must start at 0, end at *count and agree with coords
  *             (HC_ERR_INVALID_INDEX otherwise, output unspecified)
  *   G, eps, gamma, beta, act as for hc_sparse_group_norm_fwd (G divides C_out)
- * bf16 with C_out/G a multiple of 8 dividing the tensor-core tile (64
+ * bf16 with C_out/G a power of two from 8 to the tensor-core tile (64
  * channels when C_out <= 64, else 128), C_out/8 a power of two: the
  * tensor-core epilogue writes one partial (count, mean, M2) per (frame,
- * 32-row block, group) and a single normalising pass reads them (two
+ * 32-row block inside the frame, group), and one per (row, group) for blocks
+ * shared by two frames, and a single normalising pass merges them (two
  * launches, y written once by each). Otherwise the two operations run one
  * after the other. Uses the library's per-stream workspace
- * ((B + capacity/32 + 1) * G * 16 bytes, or that of hc_sparse_group_norm_fwd).
+ * ((B + capacity/32 + 1) * G * 16 + capacity * G * 8 bytes, or that of
+ * hc_sparse_group_norm_fwd).
  */
 hc_status hc_sparse_conv_gn_fwd(const void* x, hc_dtype dt, int x_rows, const int32_t* rulebook,
                                 const int32_t* count, int capacity, int L, int C_in, int C_out,

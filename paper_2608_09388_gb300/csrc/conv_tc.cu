@@ -215,48 +215,15 @@ __device__ __forceinline__ void gn_flush_whole(const ConvArgs& a, long long bloc
     }
 }
 
-// Rows that straddle a frame boundary or the last active row (gn_b = the
-// lane's frame, -1 past the active rows): for each frame present, two
-// passes over its lanes (each with cpg values per group): the frame mean
-// from the sum of lane means, then M2 = sum over lanes of (lane M2 + cpg *
-// (lane mean - frame mean)^2), which is exact. Non-member lanes add 0.
-template <int NG>
-__device__ __forceinline__ void gn_flush_runs(const ConvArgs& a, long long block, int gn_b, int g0,
-                                              int ng, float cpg, const float (&mean)[NG],
-                                              const float (&m2)[NG], int lane) {
-    unsigned todo = __ballot_sync(0xffffffffu, gn_b >= 0);
-    while (todo) {
-        const int leader = __ffs(todo) - 1;
-        const int fb = __shfl_sync(0xffffffffu, gn_b, leader);
-        const bool mem = gn_b == fb;
-        const unsigned members = __ballot_sync(0xffffffffu, mem);
-        const float cnt = (float)__popc(members);
-        float fm[NG], fq[NG];
-#pragma unroll
-        for (int q = 0; q < NG; ++q) fm[q] = mem ? mean[q] : 0.f;
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1)
-#pragma unroll
-            for (int q = 0; q < NG; ++q) fm[q] += __shfl_xor_sync(0xffffffffu, fm[q], o);
-#pragma unroll
-        for (int q = 0; q < NG; ++q) {
-            fm[q] = fm[q] / cnt;
-            const float d = mean[q] - fm[q];
-            fq[q] = mem ? fmaf(cpg * d, d, m2[q]) : 0.f;
-        }
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1)
-#pragma unroll
-            for (int q = 0; q < NG; ++q) fq[q] += __shfl_xor_sync(0xffffffffu, fq[q], o);
-        if (lane == leader) {
-#pragma unroll
-            for (int q = 0; q < NG; ++q)
-                if (q < ng)
-                    *reinterpret_cast<float4*>(a.gn_part + 4 * ((fb + block) * a.gn_G + g0 + q)) =
-                        make_float4(cnt * cpg, fm[q], fq[q], 0.f);
-        }
-        todo &= ~members;
-    }
+// Rows of a block that straddles a frame boundary or the last active row
+// (gn_b = the lane's frame, -1 past the active rows): no merge across lanes;
+// every active row stores its own (mean, M2) of group g to the per-row
+// partials (row * G + g), and the normalising pass merges them with the
+// frame's whole blocks.
+__device__ __forceinline__ void gn_store_row(const ConvArgs& a, long long row, int gn_b, int g,
+                                             float mean, float m2) {
+    if (gn_b >= 0)
+        *reinterpret_cast<float2*>(a.gn_rows + 2 * (row * a.gn_G + g)) = make_float2(mean, m2);
 }
 
 // Statistics of one 32-column chunk (columns col0 .. col0 + 31) as stored
@@ -283,7 +250,9 @@ __device__ __forceinline__ void gn_chunk(const ConvArgs& a, const uint32_t (&v)[
         if (whole)
             gn_flush_whole<NB>(a, block, gn_b, g0, nb, (float)CPG, mean, m2, lane);
         else
-            gn_flush_runs<NB>(a, block, gn_b, g0, nb, (float)CPG, mean, m2, lane);
+#pragma unroll
+            for (int q = 0; q < NB; ++q)
+                if (q < nb) gn_store_row(a, block * 32 + lane, gn_b, g0 + q, mean[q], m2[q]);
     }
 }
 
@@ -310,7 +279,7 @@ __device__ __forceinline__ void gn_chunk_wide(const ConvArgs& a, const uint32_t 
         if (whole)
             gn_flush_whole<1>(a, block, gn_b, g, 1, (float)cpg, m1, q1, lane);
         else
-            gn_flush_runs<1>(a, block, gn_b, g, 1, (float)cpg, m1, q1, lane);
+            gn_store_row(a, block * 32 + lane, gn_b, g, run_mean, run_m2);
     }
 }
 

@@ -34,9 +34,11 @@
 // and small frames (a group slice within its register cache), where one
 // launch beats the two latency-bound row-range launches.
 // Partials from the convolution: the tensor-core convolution can write the
-// same (n, mean, M2) partials of its stored output itself, one per (frame b,
-// 32-row block c) in slot b + c (the slot argument above with ranges of 32
-// rows), so that gn_apply_kernel alone finishes the layer.
+// (n, mean, M2) partials of its stored output itself, one per (frame b,
+// 32-row block c lying inside the frame) in slot b + c (the slot argument
+// above with ranges of 32 rows), and one per row for the rows of blocks that
+// straddle a frame boundary, so that gn_apply_kernel alone finishes the
+// layer.
 // The output may alias the input in both paths. Deterministic, no atomics.
 #include <cuda_bf16.h>
 
@@ -50,6 +52,7 @@ namespace {
 constexpr int kThreads = 256;
 constexpr int kBatch = 4;
 constexpr int kMaxGroupsFast = 2048;
+constexpr int kMergeBatch = 4;  // partials a lane loads before merging them
 
 // VEC consecutive elements as one raw chunk (16 bytes when VEC > 1).
 template <typename T, int VEC>
@@ -254,10 +257,9 @@ __device__ __forceinline__ Layout make_layout(int C, int G) {
 
 // This CTA's row range [lo, hi); false if there is nothing to do or the
 // frame table's span is unusable (reported).
-__device__ __forceinline__ bool range_setup(const int32_t* offsets, int B, long long capacity,
-                                            unsigned* status, RangeMap& m, long long& lo,
-                                            long long& hi) {
-    const long long o0 = __ldg(offsets), oB = __ldg(offsets + B);
+__device__ __forceinline__ bool range_from(long long o0, long long oB, long long capacity,
+                                           unsigned* status, RangeMap& m, long long& lo,
+                                           long long& hi) {
     if (o0 < 0 || oB < o0 || oB > capacity) {
         if (threadIdx.x == 0 && blockIdx.x == 0) report(status, kErrIndex);
         return false;
@@ -270,6 +272,12 @@ __device__ __forceinline__ bool range_setup(const int32_t* offsets, int B, long 
     lo = o0 + (long long)blockIdx.x * m.R;
     hi = lo + m.R < oB ? lo + m.R : oB;
     return lo < hi;
+}
+
+__device__ __forceinline__ bool range_setup(const int32_t* offsets, int B, long long capacity,
+                                            unsigned* status, RangeMap& m, long long& lo,
+                                            long long& hi) {
+    return range_from(__ldg(offsets), __ldg(offsets + B), capacity, status, m, lo, hi);
 }
 
 template <typename T, int VEC, int GPC>
@@ -374,37 +382,63 @@ __global__ void __launch_bounds__(kThreads, 2)
     gn_apply_kernel(const T* x, const int32_t* __restrict__ offsets, int B, int C, int G,
                     long long capacity, const GnPart* __restrict__ part, float eps,
                     const float* __restrict__ gamma, const float* __restrict__ beta, int act, T* y,
-                    int part_rows, const int32_t* __restrict__ count, unsigned* status) {
+                    int part_rows, const float2* __restrict__ row_part,
+                    const int32_t* __restrict__ count, unsigned* status) {
     using CK = Chunk<T, VEC>;
     using Raw = typename CK::Raw;
     static_assert(sizeof(Raw) == 16, "the row-range path moves 16-byte chunks");
     constexpr int SUB = VEC / GPC;
     __shared__ float s_mu[kMaxGroupsFast], s_inv[kMaxGroupsFast];
     __shared__ int s_off[kThreads + 1];
-    pdl_wait();
+    // part_rows > 0: the partials come from the convolution (the kernel
+    // before this one) over the rows [0, *count): one per (frame b, block c
+    // of part_rows rows inside the frame) in slot b + c, one per row
+    // (row_part, C/G values each) for the frame's other rows. The frame table
+    // must cover exactly those rows, in order (checked here, as the
+    // statistics kernel does otherwise). The table, count, gamma and
+    // beta were written before that convolution started, so they are read
+    // before waiting for it: the set-up overlaps its last blocks.
+    __shared__ int s_count;
+    const bool early = part_rows > 0;
+    if (!early) pdl_wait();
     pdl_trigger();
-    // part_rows > 0: the partials come per part_rows-row block of the rows
-    // [0, *count) that the convolution wrote; the frame table must cover
-    // exactly those rows, in order (checked here, as the statistics kernel
-    // does otherwise).
-    if (part_rows > 0) {
-        for (long long i = (long long)blockIdx.x * kThreads + threadIdx.x; i < B;
-             i += (long long)gridDim.x * kThreads)
-            if (__ldg(offsets + i + 1) < __ldg(offsets + i)) report(status, kErrIndex);
-        if (__ldg(offsets) != 0 || __ldg(offsets + B) != __ldg(count)) {
-            if (threadIdx.x == 0 && blockIdx.x == 0) report(status, kErrIndex);
-            return;
-        }
-    }
-    RangeMap m;
-    long long lo, hi;
-    if (!range_setup(offsets, B, capacity, status, m, lo, hi)) return;
     const Layout l = make_layout<VEC, GPC>(C, G);
     float ga[VEC], be[VEC];
 #pragma unroll
     for (int k = 0; k < VEC; ++k) {
         ga[k] = gamma ? __ldg(gamma + l.col * VEC + k) : 1.f;
         be[k] = beta ? __ldg(beta + l.col * VEC + k) : 0.f;
+    }
+    // B <= kThreads: the whole frame table (and the row count) in one round
+    // trip; the checks and the row range then come from shared memory
+    const bool small = B <= kThreads;
+    if (small) {
+        for (int j = threadIdx.x; j <= B; j += kThreads) s_off[j] = __ldg(offsets + j);
+        if (threadIdx.x == 0) s_count = early ? __ldg(count) : 0;
+        __syncthreads();
+    }
+    if (early) {
+        if (small) {
+            if (threadIdx.x < B && s_off[threadIdx.x + 1] < s_off[threadIdx.x])
+                report(status, kErrIndex);
+        } else {
+            for (long long i = (long long)blockIdx.x * kThreads + threadIdx.x; i < B;
+                 i += (long long)gridDim.x * kThreads)
+                if (__ldg(offsets + i + 1) < __ldg(offsets + i)) report(status, kErrIndex);
+        }
+        const int o0 = small ? s_off[0] : __ldg(offsets), oB = small ? s_off[B] : __ldg(offsets + B);
+        const int n = small ? s_count : __ldg(count);
+        if (o0 != 0 || oB != n) {
+            if (threadIdx.x == 0 && blockIdx.x == 0) report(status, kErrIndex);
+            return;
+        }
+    }
+    RangeMap m;
+    long long lo, hi;
+    if (small) {
+        if (!range_from(s_off[0], s_off[B], capacity, status, m, lo, hi)) return;
+    } else if (!range_setup(offsets, B, capacity, status, m, lo, hi)) {
+        return;
     }
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const long long step = (long long)kBatch * l.rpp;
@@ -415,11 +449,58 @@ __global__ void __launch_bounds__(kThreads, 2)
         // (clamped to the table's span, so a malformed table cannot index
         // outside the workspace)
         const long long p0 = f0 > m.off0 ? f0 : m.off0, p1 = (f1 < m.end ? f1 : m.end) - 1;
-        const long long c0 = part_rows > 0 ? p0 / part_rows : m.cta_of(p0);
-        const long long c1 = part_rows > 0 ? p1 / part_rows : m.cta_of(p1);
+        const long long c0 = m.cta_of(p0), c1 = m.cta_of(p1);
         const GnPart* pb = part + (long long)b * G;
+        // rows of the segment last to first (the statistics pass read them
+        // first to last, so the most recent ones are still in L2); every
+        // line is read and written here for the last time: evict first. The
+        // first batch is issued before the partials are merged.
+        auto row_at = [&](long long r) { return (s0 + r) * C + l.col * VEC; };
+        const long long top = (s1 - s0) - 1 - l.rg;  // this thread's highest row offset
+        Raw cur[kBatch];
+#pragma unroll
+        for (int i = 0; i < kBatch; ++i)
+            if (top - (long long)i * l.rpp >= 0)
+                cur[i] = as_raw<Raw>(ld_ef(x + row_at(top - (long long)i * l.rpp), pol));
         __syncthreads();  // s_mu / s_inv of the previous segment have been read
-        if (c1 - c0 < 8) {
+        if (part_rows > 0) {
+            // whole blocks [w0, w1) of the frame's rows [p0, p1], and its
+            // other rows (at most 2 * part_rows - 2) [p0, h1) and [t0, p1]
+            const long long P = part_rows, w0 = (p0 + P - 1) / P, w1 = (p1 + 1) / P;
+            const bool any = w0 < w1;
+            const long long nw = any ? w1 - w0 : 0;
+            const long long h1 = any ? w0 * P : p1 + 1, t0 = any ? w1 * P : p1 + 1;
+            const long long nh = h1 - p0, items = nw + nh + (p1 + 1 - t0);
+            const float cpg = (float)(C / G);
+            for (int g = warp; g < G; g += kThreads / 32) {
+                float n = 0.f, mean = 0.f, m2 = 0.f;
+                // kMergeBatch items per lane loaded together, then merged
+                for (long long i0 = lane; i0 < items; i0 += 32 * kMergeBatch) {
+                    float4 q[kMergeBatch];
+#pragma unroll
+                    for (int k = 0; k < kMergeBatch; ++k) {
+                        const long long i = i0 + 32 * k;
+                        q[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+                        if (i < nw) {
+                            const GnPart p = pb[(w0 + i) * G + g];
+                            q[k] = make_float4(p.n, p.mean, p.m2, 0.f);
+                        } else if (i < items) {
+                            const long long r = i - nw < nh ? p0 + (i - nw) : t0 + (i - nw - nh);
+                            const float2 v = row_part[r * G + g];
+                            q[k] = make_float4(cpg, v.x, v.y, 0.f);
+                        }
+                    }
+#pragma unroll
+                    for (int k = 0; k < kMergeBatch; ++k) merge(n, mean, m2, q[k].x, q[k].y, q[k].z);
+                }
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) merge_xor(n, mean, m2, o);
+                if (lane == 0) {
+                    s_mu[g] = mean;
+                    s_inv[g] = 1.f / sqrtf(m2 / n + eps);
+                }
+            }
+        } else if (c1 - c0 < 8) {
             for (int g = threadIdx.x; g < G; g += kThreads) {
                 float n = 0.f, mean = 0.f, m2 = 0.f;
                 for (long long c = c0; c <= c1; ++c) {
@@ -452,16 +533,6 @@ __global__ void __launch_bounds__(kThreads, 2)
             mu[q] = s_mu[g];
             inv[q] = s_inv[g];
         }
-        // rows of the segment last to first (the statistics pass read them
-        // first to last, so the most recent ones are still in L2); every
-        // line is read and written here for the last time: evict first
-        auto row_at = [&](long long r) { return (s0 + r) * C + l.col * VEC; };
-        const long long top = (s1 - s0) - 1 - l.rg;  // this thread's highest row offset
-        Raw cur[kBatch];
-#pragma unroll
-        for (int i = 0; i < kBatch; ++i)
-            if (top - (long long)i * l.rpp >= 0)
-                cur[i] = as_raw<Raw>(ld_ef(x + row_at(top - (long long)i * l.rpp), pol));
         for (long long r0 = top; r0 >= 0; r0 -= step) {
             Raw nxt[kBatch];
 #pragma unroll
@@ -492,20 +563,33 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
     };
 
-    // frames overlapping [lo, hi); within a window of kThreads frames, last
-    // to first
-    for (int wb = find_frame(offsets, B, lo); wb < B; wb += kThreads) {
-        const int nw = B - wb < kThreads ? B - wb : kThreads;
-        load_window(offsets, wb, nw, s_off);
+    // frames overlapping [lo, hi) of a window (frames wb .. wb + nw - 1, so
+    // holding offsets[wb + j]), last to first; true when hi is reached
+    auto walk = [&](int wb, int nw, const int* so) {
         int nf = 0;  // frames of the window that start before hi
-        while (nf < nw && (long long)s_off[nf] < hi) ++nf;
+        while (nf < nw && (long long)so[nf] < hi) ++nf;
+        if (early) pdl_wait();  // x and the partials come from the convolution
         for (int j = nf - 1; j >= 0; --j) {
-            const long long f0 = s_off[j], f1 = s_off[j + 1];
+            const long long f0 = so[j], f1 = so[j + 1];
             if (f1 < f0) continue;  // reported by the statistics kernel
             const long long s0 = f0 > lo ? f0 : lo, s1 = f1 < hi ? f1 : hi;
             if (s0 < s1) segment(wb + j, f0, f1, s0, s1);
         }
-        if (nf < nw || (long long)s_off[nw] >= hi) break;
+        return nf < nw || (long long)so[nw] >= hi;
+    };
+    if (small) {
+        // the first frame of the range (the number of frames ending at or
+        // before lo), found in the table in shared memory
+        const int wb =
+            __syncthreads_count(threadIdx.x < B && (long long)s_off[threadIdx.x + 1] <= lo);
+        if (wb < B) walk(wb, B - wb, s_off + wb);
+        return;
+    }
+    // windows of kThreads frames
+    for (int wb = find_frame(offsets, B, lo); wb < B; wb += kThreads) {
+        const int nw = B - wb < kThreads ? B - wb : kThreads;
+        load_window(offsets, wb, nw, s_off);
+        if (walk(wb, nw, s_off)) break;
     }
 }
 
@@ -659,7 +743,7 @@ hc_status launch_fast(const DeviceCtx* ctx, const void* x, const int32_t* offset
     return launch_pdl(gn_apply_kernel<T, VEC, GPC>, dim3((unsigned)grid), dim3(kThreads), 0, s,
                       "gn_apply_kernel", (const T*)x, offsets, B, C, G, capacity,
                       (const GnPart*)part, eps, gamma, beta, act, (T*)y, 0,
-                      (const int32_t*)nullptr, ctx->status);
+                      (const float2*)nullptr, (const int32_t*)nullptr, ctx->status);
 }
 
 
@@ -721,13 +805,14 @@ bool group_norm_parts_supported(hc_dtype dt, int C, int G, const void* y) {
 
 hc_status launch_group_norm_apply(const DeviceCtx* ctx, void* y, const int32_t* offsets, int B,
                                   long long capacity, int C, int G, const float* part,
-                                  int part_rows, const int32_t* count, float eps,
-                                  const float* gamma, const float* beta, int act, cudaStream_t s) {
+                                  const float* rows, int part_rows, const int32_t* count,
+                                  float eps, const float* gamma, const float* beta, int act,
+                                  cudaStream_t s) {
     using T = __nv_bfloat16;
     return launch_pdl(gn_apply_kernel<T, 8, 1>, dim3((unsigned)fast_grid(ctx, capacity)),
                       dim3(kThreads), 0, s, "gn_apply_kernel", (const T*)y, offsets, B, C, G,
                       capacity, (const GnPart*)part, eps, gamma, beta, act, (T*)y, part_rows,
-                      count, ctx->status);
+                      (const float2*)rows, count, ctx->status);
 }
 
 hc_status launch_group_norm(const DeviceCtx* ctx, const void* x, hc_dtype dt,

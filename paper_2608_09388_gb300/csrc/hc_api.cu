@@ -403,20 +403,25 @@ hc_status hc_sparse_conv_gn_fwd(const void* x, hc_dtype dt, int x_rows, const in
     // channels per group a power of two from 8 to the tile's width
     if (use_conv_tc(a, dt) && cpg >= 8 && (cpg & (cpg - 1)) == 0 && cpg <= conv_tc_tile_n(a) &&
         group_norm_parts_supported(dt, C_out, G, y)) {
-        // statistics from the convolution's epilogue, one partial per
-        // (frame, 32-row block) in slot frame + block
+        // statistics from the convolution's epilogue: one partial per
+        // (frame, 32-row block inside it) in slot frame + block, one per row
+        // of the blocks that straddle a frame boundary
         const size_t slots = (size_t)B + ((size_t)capacity + 31) / 32;
-        float* part = (float*)stream_workspace(s, 16 * slots * (size_t)G);
-        if (!part) return HC_ERR_CUDA;
+        const size_t part_bytes = 16 * slots * (size_t)G;
+        char* ws = (char*)stream_workspace(s, part_bytes + 8 * (size_t)capacity * (size_t)G);
+        if (!ws) return HC_ERR_CUDA;
+        float* part = (float*)ws;
+        float* rows = (float*)(ws + part_bytes);
         a.gn_part = part;
+        a.gn_rows = rows;
         a.gn_coords = coords;
         a.gn_G = G;
         a.gn_B = B;
         a.gn_cpg = cpg;
         st = launch_conv_tc(ctx, a, s);
         if (st != HC_OK) return st;
-        return launch_group_norm_apply(ctx, y, batch_offsets, B, capacity, C_out, G, part, 32,
-                                       count, eps, gamma, beta, (int)act, s);
+        return launch_group_norm_apply(ctx, y, batch_offsets, B, capacity, C_out, G, part, rows,
+                                       32, count, eps, gamma, beta, (int)act, s);
     }
     st = dispatch_conv(ctx, a, dt, s);
     if (st != HC_OK) return st;

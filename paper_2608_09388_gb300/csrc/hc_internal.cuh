@@ -74,7 +74,11 @@ struct ConvArgs {
     // frame b among its rows (b = gn_coords[2n]) and each channel group g of
     // gn_G, the (count, mean, M2) of its stored values to
     // gn_part[4 * ((b + c) * gn_G + g)].
+    // Blocks whose rows are not all active and in one frame write, instead,
+    // every active row's (mean, M2) of each group (gn_C / gn_G values) to
+    // gn_rows[2 * (row * gn_G + g)].
     float* gn_part;
+    float* gn_rows;
     const int32_t* gn_coords;
     int gn_G, gn_B;
     int gn_cpg;  // channels per group, C_out / gn_G: 8, 16, 32, 64 or 128
@@ -95,14 +99,16 @@ hc_status launch_group_norm(const DeviceCtx* ctx, const void* x, hc_dtype dt,
                             const int32_t* offsets, int B, long long capacity, int C, int G,
                             float eps, const float* gamma, const float* beta, int act, void* y,
                             cudaStream_t s);
-// The normalising pass alone, in place on bf16 y, from partials written per
-// part_rows-row block of the rows [0, *count) (the convolution's); the frame
-// table must start at 0 and end at *count.
+// The normalising pass alone, in place on bf16 y, from the partials the
+// convolution wrote for the rows [0, *count): one per (frame, part_rows-row
+// block lying inside the frame, group) in part, and one per (row, group) in
+// rows for the other rows. The frame table must start at 0 and end at *count.
 bool group_norm_parts_supported(hc_dtype dt, int C, int G, const void* y);
 hc_status launch_group_norm_apply(const DeviceCtx* ctx, void* y, const int32_t* offsets, int B,
                                   long long capacity, int C, int G, const float* part,
-                                  int part_rows, const int32_t* count, float eps,
-                                  const float* gamma, const float* beta, int act, cudaStream_t s);
+                                  const float* rows, int part_rows, const int32_t* count,
+                                  float eps, const float* gamma, const float* beta, int act,
+                                  cudaStream_t s);
 // Backward of the sparse conv through a rulebook (see bwd.cu).
 struct BwdArgs {
     const void* x;

@@ -149,6 +149,21 @@ def test_conv_gn_many_tiny_frames(G):
     check_case(c, f"tiny frames G={G}")
 
 
+@pytest.mark.parametrize("G", [8, 2])
+def test_conv_gn_frames_at_block_edges(G):
+    """Frames of exactly 32 or 64 rows (every 32-row block inside one frame),
+    one row more or less (blocks shared by two frames), empty and single-row
+    frames: the block partials and the per-row partials of shared blocks."""
+    sizes = [64, 32, 33, 31, 0, 96, 1, 63, 65, 32]
+    B, V = len(sizes), 150
+    rng = np.random.default_rng(12)
+    m = np.zeros((B, V), np.uint8)
+    for b, k in enumerate(sizes):
+        m[b, rng.choice(V, size=k, replace=False)] = 1
+    c = _case(46, B, V, 9, 16, 128, G, "bf16", True, oracle.ACT_ELU, mask=m)
+    check_case(c, f"block edges G={G}")
+
+
 def test_conv_gn_large_frame_and_eps():
     """One frame spread over hundreds of 32-row blocks, eps from 0 to large."""
     B, V = 2, 12000
