@@ -127,6 +127,11 @@ __global__ void __launch_bounds__(kThreads)
     __shared__ int tile_base_s;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int tile = blockIdx.x;
+    // The mask is read before waiting on the count pass: that pass started
+    // only after everything before it on the stream had finished, so the
+    // mask is complete; its load overlaps the wait and the tile-count read.
+    long long base = (long long)tile * kTile + (long long)tid * kItems;
+    uint32_t flags = load_flags(mask, n, base);
     pdl_wait();
     pdl_trigger();
 
@@ -142,8 +147,6 @@ __global__ void __launch_bounds__(kThreads)
         tile_base = block_sum(part, red);
     }
 
-    long long base = (long long)tile * kTile + (long long)tid * kItems;
-    uint32_t flags = load_flags(mask, n, base);
     int c = __popc(flags);
 
     // Block-wide exclusive scan of c.
@@ -193,7 +196,9 @@ __global__ void __launch_bounds__(kThreads)
                 for (int k = 0; k < kItems / 4; ++k)
                     dst[k] = make_int4(ro[4 * k], ro[4 * k + 1], ro[4 * k + 2], ro[4 * k + 3]);
             } else {
-                for (int k = 0; k < kItems && base + k < n; ++k) row_of[base + k] = ro[k];
+#pragma unroll
+                for (int k = 0; k < kItems; ++k)
+                    if (base + k < n) row_of[base + k] = ro[k];
             }
         }
         // Frame offsets: offsets[b] = rows before position b*V, for every

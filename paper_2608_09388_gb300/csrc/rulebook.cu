@@ -8,15 +8,19 @@
 // Layout: [L, capacity] int32, slot-major (entry (l, n) at l*capacity + n),
 // so that a tile of consecutive rows reads each slot as one contiguous run.
 // One thread per active row; its coordinate, spiral entries and row_of
-// lookups are each issued together from clamped, always-valid addresses.
+// lookups are each issued together from clamped, always-valid addresses:
+// the first row's coordinate together with the row count, then up to
+// kChunk spiral slots, then their row_of entries (three round trips for
+// L <= kChunk); a thread with more rows fetches the next row's coordinate
+// during the current row's lookups.
 #include "hc_internal.cuh"
 
 namespace hc {
 namespace {
 
-constexpr int kChunk = 8;
+constexpr int kChunk = 16;
 
-__global__ void __launch_bounds__(256) rulebook_kernel(const int32_t* __restrict__ coords,
+__global__ void __launch_bounds__(256, 3) rulebook_kernel(const int32_t* __restrict__ coords,
                                                        const int32_t* __restrict__ row_of,
                                                        const int32_t* __restrict__ count,
                                                        const int32_t* __restrict__ spiral, int B,
@@ -26,6 +30,14 @@ __global__ void __launch_bounds__(256) rulebook_kernel(const int32_t* __restrict
     pdl_wait();
     pdl_trigger();
     const long long cap = (long long)B * V;
+    const long long n0 = blockIdx.x * (long long)blockDim.x + threadIdx.x;
+    // every n < capacity indexes coords: the first row's coordinate is
+    // fetched with the row count, before it is known to be active
+    int b0 = 0, v0 = 0;
+    if (n0 < cap) {
+        b0 = __ldg(coords + 2 * n0);
+        v0 = __ldg(coords + 2 * n0 + 1);
+    }
     long long rows = *count;
     unsigned err = 0;
     if (rows < 0) {
@@ -36,9 +48,14 @@ __global__ void __launch_bounds__(256) rulebook_kernel(const int32_t* __restrict
         err |= kErrCapacity;
         rows = cap;
     }
-    for (long long n = blockIdx.x * (long long)blockDim.x + threadIdx.x; n < rows;
-         n += (long long)gridDim.x * blockDim.x) {
-        int b = __ldg(coords + 2 * n), v = __ldg(coords + 2 * n + 1);
+    const long long stride = (long long)gridDim.x * blockDim.x;
+    for (long long n = n0; n < rows; n += stride) {
+        int b = b0, v = v0;
+        // the next row's coordinate, fetched while this row's lookups run
+        if (n + stride < rows) {
+            b0 = __ldg(coords + 2 * (n + stride));
+            v0 = __ldg(coords + 2 * (n + stride) + 1);
+        }
         const bool ok = b >= 0 && b < B && v >= 0 && v < V;
         if (!ok) {
             err |= kErrIndex;
@@ -79,6 +96,9 @@ hc_status launch_rulebook(const DeviceCtx* ctx, const int32_t* coords, const int
                           int x_layout, int32_t* rulebook, cudaStream_t s) {
     const long long cap = (long long)B * V;
     long long blocks = (cap + 255) / 256;
+    // up to 8 blocks per SM: beyond the resident ones (3 per SM) they cost
+    // the row count's round trip per wave when rows are few, but keep more
+    // lookups in flight when most rows are active
     const long long lim = (long long)ctx->num_sms * 8;
     if (blocks > lim) blocks = lim;
     if (blocks < 1) blocks = 1;

@@ -107,6 +107,55 @@ def test_compact_empty_sizes():
         assert int(count.item()) == 0 and (to_numpy(offs) == 0).all()
 
 
+def test_compact_repeated_sizes_and_streams():
+    """Calls of changing sizes back to back (more tiles, then fewer, then
+    more; the per-stream workspace grows and is reused) on the default
+    stream and on a second stream stay bit-exact."""
+    side = torch.cuda.Stream()
+    shapes = [(64, 10475), (3, 100), (1, 5000), (130, 10475), (2, 7), (64, 10475)]
+    for i, (B, V) in enumerate(shapes):
+        m = inputs.uniform_mask(np.random.default_rng(100 + i), B, V, 0.2)
+        assert_compact_equal(m, gpu_compact(m))
+        got = (torch.full((B * V, 2), -7, dtype=torch.int32, device="cuda"),
+               torch.full((B, V), -7, dtype=torch.int32, device="cuda"),
+               torch.full((B + 1,), -7, dtype=torch.int32, device="cuda"),
+               torch.full((1,), -7, dtype=torch.int32, device="cuda"))
+        mt = to_torch(m)
+        torch.cuda.synchronize()
+        with torch.cuda.stream(side):
+            hc.hc_mask_compact(mt, *got, side)
+        torch.cuda.synchronize()
+        assert_compact_equal(m, got)
+    assert hc.hc_get_device_status() == hc.HC_OK
+
+
+def test_compact_graph_replays():
+    """One compaction captured in a CUDA graph and replayed with new mask
+    contents each time (empty, dense and sparse masks): every replay
+    bit-exact."""
+    B, V = 32, 10475
+    stream = torch.cuda.Stream()
+    mask = torch.zeros((B, V), dtype=torch.uint8, device="cuda")
+    coords = torch.empty((B * V, 2), dtype=torch.int32, device="cuda")
+    row_of = torch.empty((B, V), dtype=torch.int32, device="cuda")
+    offs = torch.empty((B + 1,), dtype=torch.int32, device="cuda")
+    count = torch.empty((1,), dtype=torch.int32, device="cuda")
+    with torch.cuda.stream(stream):
+        hc.hc_mask_compact(mask, coords, row_of, offs, count, stream)  # sets up the state
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            hc.hc_mask_compact(mask, coords, row_of, offs, count, stream)
+    for i, d in enumerate((0.05, 0.0, 0.5, 1.0, 0.01)):
+        m = inputs.uniform_mask(np.random.default_rng(200 + i), B, V, d)
+        mask.copy_(torch.from_numpy(m))
+        torch.cuda.synchronize()
+        with torch.cuda.stream(stream):
+            g.replay()
+        torch.cuda.synchronize()
+        assert_compact_equal(m, (coords, row_of, offs, count))
+    assert hc.hc_get_device_status() == hc.HC_OK
+
+
 def test_compact_workload_masks():
     for name in ("layer655_f32", "encoder655_bf16", "motion655_bf16", "layer10475_bf16"):
         w = inputs.make_workload(name)
