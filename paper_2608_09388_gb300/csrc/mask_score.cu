@@ -371,10 +371,13 @@ __global__ void pack_kernel(const __nv_bfloat16* __restrict__ O, long long N, in
 // ---------------------------------------------------------------- pairs
 // Block (p, c) <-> pair p = (i, k), i <= k (row-major over the upper
 // triangle of the K x K matrix, diagonal included), and chunk c of
-// kPairChunk entries of its D x D block: the sum over that chunk of
-// (sum over splits of G's entry)^2, written to P[p][c]. Fixed orders.
+// kPairChunk entries of its D x D block, one entry per thread: the sum over
+// the chunk of (sum over splits of G's entry)^2, written to P[p][c]. A
+// thread issues its split loads kSplitBatch at a time (one round trip for
+// up to kSplitBatch splits). Fixed orders.
 constexpr int kPairThreads = 256;
-constexpr int kPairChunk = 1024;
+constexpr int kPairChunk = kPairThreads;
+constexpr int kSplitBatch = 16;
 
 __device__ __forceinline__ int pair_of(int p, int K, int& k) {
     int i = 0;
@@ -398,14 +401,9 @@ __global__ void __launch_bounds__(kPairThreads)
     const int p = blockIdx.x / nchunk, chunk = blockIdx.x - p * nchunk;
     int k;
     const int i = pair_of(p, K, k);
-    const int DD = D * D;
-    const int e0 = chunk * kPairChunk;
-    const int e1 = e0 + kPairChunk < DD ? e0 + kPairChunk : DD;
-    const int tmask = (1 << tile_shift) - 1;
-    const long long tile_elems = 1ll << (2 * tile_shift);
-    const long long split_stride = (long long)T * tile_elems;
+    const int idx = chunk * kPairChunk + threadIdx.x;
     float acc = 0.f;
-    for (int idx = e0 + threadIdx.x; idx < e1; idx += kPairThreads) {
+    if (idx < D * D) {
         const int d = idx / D, e = idx - d * D;
         int m = i * D + d, m2 = k * D + e;
         if (m > m2) {  // below the diagonal: the symmetric entry of an upper tile
@@ -413,12 +411,21 @@ __global__ void __launch_bounds__(kPairThreads)
             m = m2;
             m2 = tmp;
         }
+        const int tmask = (1 << tile_shift) - 1;
+        const long long tile_elems = 1ll << (2 * tile_shift);
+        const long long split_stride = (long long)T * tile_elems;
         const float* src = part + tile_index(m >> tile_shift, m2 >> tile_shift, nt) * tile_elems +
                            ((long long)(m & tmask) << tile_shift) + (m2 & tmask);
         float g = 0.f;
-#pragma unroll 8
-        for (int sp = 0; sp < splits; ++sp) g += __ldg(src + sp * split_stride);
-        acc = fmaf(g, g, acc);
+        for (int sp0 = 0; sp0 < splits; sp0 += kSplitBatch) {
+            float v[kSplitBatch];
+#pragma unroll
+            for (int j = 0; j < kSplitBatch; ++j)
+                v[j] = sp0 + j < splits ? __ldg(src + (sp0 + j) * split_stride) : 0.f;
+#pragma unroll
+            for (int j = 0; j < kSplitBatch; ++j) g += v[j];
+        }
+        acc = g * g;
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
@@ -440,6 +447,47 @@ __device__ __forceinline__ float pair_sum(const float* P, int i, int k, int K, i
     float s = 0.f;
     for (int c = 0; c < nchunk; ++c) s += __ldg(P + (long long)p * nchunk + c);
     return s;
+}
+
+// K <= kAlphaSmallK: one block; the pair sums S go to shared memory first,
+// every pair's chunks loaded at once (one round trip), then thread k forms
+// alpha_k from them (same arithmetic and order as alpha_kernel).
+constexpr int kAlphaSmallK = 64;
+constexpr int kAlphaThreads = 256;
+
+__global__ void __launch_bounds__(kAlphaThreads)
+    alpha_small_kernel(const float* __restrict__ P, int K, int nchunk, const float* alpha_in,
+                       float* alpha_out, float* __restrict__ sim) {
+    __shared__ float sS[kAlphaSmallK * (kAlphaSmallK + 1) / 2];
+    pdl_wait();
+    pdl_trigger();
+    const int n_pairs = K * (K + 1) / 2;
+    for (int p = threadIdx.x; p < n_pairs; p += kAlphaThreads) {
+        float s = 0.f;
+        for (int c0 = 0; c0 < nchunk; c0 += kSplitBatch) {
+            float v[kSplitBatch];
+#pragma unroll
+            for (int j = 0; j < kSplitBatch; ++j)
+                v[j] = c0 + j < nchunk ? __ldg(P + (long long)p * nchunk + c0 + j) : 0.f;
+#pragma unroll
+            for (int j = 0; j < kSplitBatch; ++j) s += v[j];
+        }
+        sS[p] = s;
+    }
+    __syncthreads();
+    const int k = threadIdx.x;
+    if (k >= K) return;
+    const float nk = sqrtf(sS[pair_index(k, k, K)]);
+    float sum = 0.f;
+    for (int i = 0; i < K; ++i) {
+        const float den = sqrtf(sS[pair_index(i, i, K)]) * nk;
+        const float sik = sS[i <= k ? pair_index(i, k, K) : pair_index(k, i, K)];
+        const float s = den > 0.f ? sik / den : 0.f;
+        if (sim) sim[(long long)i * K + k] = s;
+        if (i != k) sum += 1.f - s;
+    }
+    const float a0 = alpha_in[k];
+    alpha_out[k] = K > 1 ? a0 + sum / (float)(K - 1) : a0;
 }
 
 __global__ void alpha_kernel(const float* __restrict__ P, int K, int nchunk, const float* alpha_in,
@@ -578,6 +626,10 @@ hc_status launch_mask_score(const DeviceCtx* ctx, const void* O, hc_dtype dt, in
                         S);
         if (st != HC_OK) return st;
     }
+    if (K <= kAlphaSmallK)
+        return launch_pdl(alpha_small_kernel, dim3(1), dim3(kAlphaThreads), 0, s,
+                          "alpha_small_kernel", (const float*)S, K, nchunk, alpha_in, alpha_out,
+                          sim);
     return launch_pdl(alpha_kernel, dim3((unsigned)((K + 127) / 128)), dim3(128), 0, s,
                       "alpha_kernel", (const float*)S, K, nchunk, alpha_in, alpha_out, sim);
 }
