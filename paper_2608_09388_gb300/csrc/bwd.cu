@@ -343,7 +343,6 @@ __global__ void dgrad_kernel(const T* __restrict__ P, const int32_t* __restrict_
     pdl_trigger();
     const int cpr = C_in / VEC;
     const long long total = (long long)x_rows * cpr;
-    const long long prow = (long long)L * C_in;
     for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
          i += (long long)gridDim.x * blockDim.x) {
         const long long j = i / cpr;
@@ -372,8 +371,8 @@ __global__ void dgrad_kernel(const T* __restrict__ P, const int32_t* __restrict_
                     key[i] = -1;
                     continue;
                 }
-                const int n = key[i] / L, l = key[i] - n * L;
-                raw[i] = *reinterpret_cast<const U*>(P + n * prow + (long long)l * C_in + c);
+                // key n*L + l: P's row n, slot l starts at (n*L + l)*C_in
+                raw[i] = *reinterpret_cast<const U*>(P + (long long)key[i] * C_in + c);
             }
 #pragma unroll
             for (int i = 0; i < kBatchTaps; ++i) {
@@ -702,7 +701,6 @@ __global__ void __launch_bounds__(256)
     const int lane = threadIdx.x & 31;
     const int cpr = C_in / VEC, G = 32 / cpr;
     const int g = lane / cpr, c = (lane - g * cpr) * VEC;
-    const long long prow = (long long)L * C_in;
     const long long nwarps = (long long)gridDim.x * (blockDim.x >> 5);
     const long long w = (long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
     // rows w, w + nwarps, w + 2 nwarps, ...: clustered active rows spread
@@ -749,8 +747,8 @@ __global__ void __launch_bounds__(256)
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
                     if (key[i] < 0) continue;
-                    const int n = key[i] / L, l = key[i] - n * L;
-                    raw[i] = *reinterpret_cast<const uint4*>(P + n * prow + (long long)l * C_in + c);
+                    // key n*L + l: P's row n, slot l starts at (n*L + l)*C_in
+                    raw[i] = *reinterpret_cast<const uint4*>(P + (long long)key[i] * C_in + c);
                 }
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
