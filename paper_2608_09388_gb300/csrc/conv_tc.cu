@@ -425,6 +425,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int q = t & 7;        // A: 16-byte chunk of the 128-byte row
             constexpr uint32_t kWBytes = (uint32_t)(BN / 64) * (kBK * 128u);
             long long it = 0;
+            int st_s = 0;        // stage of iteration it (it % stages)
+            uint32_t st_ph = 0;  // its phase parity ((it / stages) & 1)
             int lt = 0;
             bool ok = true;
             for (long long w = blockIdx.x; w < work_total && ok; w += gridDim.x, ++lt) {
@@ -439,8 +441,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 int l = (q * 8) / C_in;  // slot and channel of this thread's chunk at k-block 0
                 int c = q * 8 - l * C_in;
                 for (int kb = 0; kb < num_kb; ++kb) {
-                    const int s = (int)(it % nst);
-                    const uint32_t ph = (uint32_t)((it / nst) & 1);
+                    const int s = st_s;
+                    const uint32_t ph = st_ph;
                     if (!mbar_wait(empty_bar(s), ph ^ 1u, abort_flag, a.status)) {
                         ok = false;
                         break;
@@ -470,6 +472,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                     cp_async_arrive_noinc(full_bar(s));
                     ++it;
+                    if (++st_s == nst) {
+                        st_s = 0;
+                        st_ph ^= 1u;
+                    }
                     c += kBK;
                     while (c >= C_in) {
                         c -= C_in;
@@ -493,6 +499,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int t = threadIdx.x;  // 0..127
             const int q = t & 7;        // A: 16-byte chunk of the 128-byte row
             long long it = 0;
+            int st_s = 0;        // stage of iteration it (it % stages)
+            uint32_t st_ph = 0;  // its phase parity ((it / stages) & 1)
             int lt = 0;
             bool ok = true;
             for (long long w = blockIdx.x; w < work_total && ok; w += gridDim.x, ++lt) {
@@ -507,8 +515,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 int l = (q * 8) / C_in;  // slot and channel of this thread's chunk at k-block 0
                 int c = q * 8 - l * C_in;
                 for (int kb = 0; kb < num_kb; ++kb) {
-                    const int s = (int)(it % nst);
-                    const uint32_t ph = (uint32_t)((it / nst) & 1);
+                    const int s = st_s;
+                    const uint32_t ph = st_ph;
                     if (!mbar_wait(empty_bar(s), ph ^ 1u, abort_flag, a.status)) {
                         ok = false;
                         break;
@@ -549,6 +557,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                         mbar_arrive(full_bar((int)((it - C::kLag) % nst)));
                     }
                     ++it;
+                    if (++st_s == nst) {
+                        st_s = 0;
+                        st_ph ^= 1u;
+                    }
                     c += kBK;
                     while (c >= C_in) {
                         c -= C_in;
@@ -568,6 +580,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0) {
             long long it = 0;
+            int st_s = 0;        // stage of iteration it (it % stages)
+            uint32_t st_ph = 0;  // its phase parity ((it / stages) & 1)
             int lt = 0;
             bool ok = true;
             for (long long w = blockIdx.x; w < work_total && ok; w += gridDim.x, ++lt) {
@@ -580,8 +594,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc_fence_after();
                 const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
                 for (int kb = 0; kb < num_kb; ++kb) {
-                    const int s = (int)(it % nst);
-                    const uint32_t ph = (uint32_t)((it / nst) & 1);
+                    const int s = st_s;
+                    const uint32_t ph = st_ph;
                     if (!mbar_wait(full_bar(s), ph, abort_flag, a.status)) {
                         ok = false;
                         break;
@@ -600,6 +614,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                     tc_commit(empty_bar(s));
                     ++it;
+                    if (++st_s == nst) {
+                        st_s = 0;
+                        st_ph ^= 1u;
+                    }
                 }
                 if (!ok) break;
                 tc_commit(tfull_bar(acc));
