@@ -345,8 +345,9 @@ __global__ void dgrad_kernel(const T* __restrict__ P, const int32_t* __restrict_
     const long long total = (long long)x_rows * cpr;
     for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
          i += (long long)gridDim.x * blockDim.x) {
-        const long long j = i / cpr;
-        const int c = (int)(i - j * cpr) * VEC;
+        int ci;
+        const long long j = div32(i, cpr, ci);
+        const int c = ci * VEC;
         float acc[VEC];
 #pragma unroll
         for (int k = 0; k < VEC; ++k) acc[k] = 0.f;
@@ -674,7 +675,8 @@ __global__ void wgrad_reduce_kernel(const float* __restrict__ part, int K, int C
     const long long total = (long long)K * C_out;
     for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
          e += (long long)gridDim.x * blockDim.x) {
-        const int m = (int)(e / C_out), o = (int)(e - (long long)m * C_out);
+        int o;
+        const int m = (int)div32(e, C_out, o);
         const int t = (m >> 7) * n_tiles + (o >> 7);
         const float* src = part + (long long)t * kPartElems + ((m & 127) << 7) + (o & 127);
         float s = 0.f;

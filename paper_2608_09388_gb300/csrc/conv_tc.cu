@@ -430,7 +430,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             int lt = 0;
             bool ok = true;
             for (long long w = blockIdx.x; w < work_total && ok; w += gridDim.x, ++lt) {
-                const int n0 = (int)(w % n_tiles) * BN;
+                const int n0 = ((int)w % n_tiles) * BN;  // w < 2^31
                 const int buf = lt & 1;
                 if (!mbar_wait(tabfull_bar(buf), (uint32_t)((lt >> 1) & 1), abort_flag,
                                a.status)) {
@@ -504,7 +504,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             int lt = 0;
             bool ok = true;
             for (long long w = blockIdx.x; w < work_total && ok; w += gridDim.x, ++lt) {
-                const int n0 = (int)(w % n_tiles) * BN;
+                const int n0 = ((int)w % n_tiles) * BN;  // w < 2^31
                 const int buf = lt & 1;
                 if (!mbar_wait(tabfull_bar(buf), (uint32_t)((lt >> 1) & 1), abort_flag,
                                a.status)) {
@@ -641,7 +641,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!mbar_wait(tabempty_bar(buf), (uint32_t)(((lt >> 1) & 1) ^ 1), abort_flag,
                            a.status))
                 break;
-            const long long m0 = (w / n_tiles) * kBM;
+            const long long m0 = (long long)((int)w / n_tiles) * kBM;
             const uint32_t tab_s = tab0 + (uint32_t)buf * tab_bytes;
             unsigned err = 0;
             if (a.mode == kRulebook) {
@@ -769,8 +769,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         __nv_bfloat16* __restrict__ y = static_cast<__nv_bfloat16*>(a.y);
         int lt = 0;
         for (long long w = blockIdx.x; w < work_total; w += gridDim.x, ++lt) {
-            const long long m0 = (w / n_tiles) * kBM;
-            const int n0 = (int)(w % n_tiles) * BN;
+            const long long m0 = (long long)((int)w / n_tiles) * kBM;
+            const int n0 = ((int)w % n_tiles) * BN;  // w < 2^31
             const int acc = lt & 1;
             const uint32_t ph = (uint32_t)((lt >> 1) & 1);
             // Everything that does not need the accumulator is loaded while
@@ -941,8 +941,10 @@ hc_status launch_bn(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s) {
 bool conv_tc_supported(const ConvArgs& a, hc_dtype dt) {
     const uintptr_t al =
         (uintptr_t)a.x | (uintptr_t)a.W | (uintptr_t)a.y | (uintptr_t)a.out_dense;
+    // tile indices are 32-bit in the kernel
+    const long long tiles = (a.capacity + kBM - 1) / kBM * ((a.C_out + 63) / 64);
     return dt == HC_BF16 && a.C_in % 8 == 0 && a.C_out % 8 == 0 && al % 16 == 0 &&
-           a.L <= HC_MAX_SPIRAL;
+           a.L <= HC_MAX_SPIRAL && tiles < (1ll << 31);
 }
 
 int conv_tc_tile_n(const ConvArgs& a) {

@@ -291,6 +291,19 @@ __device__ __forceinline__ void sts_s32(uint32_t addr, int v) {
     asm volatile("st.shared.b32 [%0], %1;\n" ::"r"(addr), "r"(v) : "memory");
 }
 
+// q = a / d and r = a - q * d for a >= 0, d > 0: 32-bit division when a
+// fits (a 64-bit division is a long subroutine), 64-bit otherwise.
+__device__ __forceinline__ long long div32(long long a, int d, int& r) {
+    if (a < (1ll << 31)) {
+        const unsigned q = (unsigned)a / (unsigned)d;
+        r = (int)((unsigned)a - q * (unsigned)d);
+        return q;
+    }
+    const long long q = a / d;
+    r = (int)(a - q * d);
+    return q;
+}
+
 __device__ __forceinline__ unsigned long long globaltimer_ns() {
     unsigned long long t;
     asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));

@@ -79,9 +79,10 @@ __global__ void kappa_masks_kernel(const uint8_t* __restrict__ masks, int K, int
     const long long total = B * kappa * (long long)V;
     for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
          e += (long long)gridDim.x * blockDim.x) {
-        const long long f = e / V;
-        const int v = (int)(e - f * V);
-        const int sel = __ldg(selected + (int)(f % kappa));
+        int v, j;
+        const long long f = div32(e, V, v);
+        div32(f, kappa, j);
+        const int sel = __ldg(selected + j);
         uint8_t m = 0;
         if (sel >= 0 && sel < K)
             m = masks[(long long)sel * V + v];
@@ -111,10 +112,10 @@ __global__ void gather_rows_kernel(const U* __restrict__ x, long long B_in, int 
     const long long total = rows * cpr;
     for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
          i += (long long)gridDim.x * blockDim.x) {
-        const long long n = i / cpr;
-        const int c = (int)(i - n * cpr);
+        int c;
+        const long long n = div32(i, cpr, c);
         const int f = __ldg(coords + 2 * n), v = __ldg(coords + 2 * n + 1);
-        const long long b = f >= 0 ? (long long)f / frames_per_sample : -1;
+        const long long b = f >= 0 ? f / frames_per_sample : -1;
         if (b < 0 || b >= B_in || v < 0 || v >= V) {
             if (c == 0) report(status, kErrIndex);
             continue;

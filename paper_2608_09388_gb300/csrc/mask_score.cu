@@ -357,8 +357,8 @@ __global__ void pack_kernel(const __nv_bfloat16* __restrict__ O, long long N, in
     const long long total = N * Mp;
     for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
          e += (long long)gridDim.x * blockDim.x) {
-        const long long n = e / Mp;
-        const int m = (int)(e - n * Mp);
+        int m;
+        const long long n = div32(e, Mp, m);
         __nv_bfloat16 v = __float2bfloat16_rn(0.f);
         if (m < KD) {
             const int k = m / D;

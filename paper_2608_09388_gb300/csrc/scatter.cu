@@ -49,8 +49,8 @@ __global__ void scatter_kernel(const U* __restrict__ y, const int32_t* __restric
     const long long total = rows * cpr;
     for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
          i += (long long)gridDim.x * blockDim.x) {
-        const long long n = i / cpr;
-        const int c = (int)(i - n * cpr);
+        int c;
+        const long long n = div32(i, cpr, c);
         const int b = __ldg(coords + 2 * n), v = __ldg(coords + 2 * n + 1);
         if (b < 0 || b >= B || v < 0 || v >= V) {
             report(status, kErrIndex);
@@ -70,8 +70,8 @@ __global__ void scatter_fill_kernel(const U* __restrict__ y, const int32_t* __re
     const long long total = dense_rows * cpr;
     for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
          i += (long long)gridDim.x * blockDim.x) {
-        const long long r = i / cpr;
-        const int c = (int)(i - r * cpr);
+        int c;
+        const long long r = div32(i, cpr, c);
         const int j = __ldg(row_of + r);
         U val = zero_chunk<U>();
         if (j >= 0 && j < rows)
