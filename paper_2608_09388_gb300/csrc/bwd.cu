@@ -164,7 +164,8 @@ __global__ void rb_count_kernel(const int32_t* __restrict__ rb, const int32_t* c
     const long long total = rows * L;
     for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
          e += (long long)gridDim.x * blockDim.x) {
-        const long long l = e / rows, n = e - l * rows;
+        int n;
+        const long long l = div32(e, (int)rows, n);  // rows <= capacity < 2^31
         const int j = __ldg(rb + l * capacity + n);
         if (j >= 0 && j < x_rows)
             atomicAdd(cnt + j, 1);
@@ -272,7 +273,8 @@ __global__ void rb_fill_kernel(const int32_t* __restrict__ rb, const int32_t* co
     const long long total = rows * L;
     for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
          e += (long long)gridDim.x * blockDim.x) {
-        const long long l = e / rows, n = e - l * rows;
+        int n;
+        const long long l = div32(e, (int)rows, n);  // rows <= capacity < 2^31
         const int j = __ldg(rb + l * capacity + n);
         if (j >= 0 && j < x_rows) {
             const int pos = atomicAdd(fill + j, 1);

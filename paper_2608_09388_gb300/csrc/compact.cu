@@ -171,8 +171,9 @@ __global__ void __launch_bounds__(kThreads)
 
     // coords and row_of for this thread's 16 positions.
     if (base < n) {
-        int b = (int)(base / V);
-        int v = (int)(base - (long long)b * V);
+        int v;
+        int b = (int)div32(base, V, v);  // base < B*V < 2^31
+        const int b_first = b, v_first = v;  // frame and vertex of base
         int r = row;
         int ro[kItems];
 #pragma unroll
@@ -205,8 +206,10 @@ __global__ void __launch_bounds__(kThreads)
         // frame boundary b*V that falls in [base, base+16).
         if (offsets) {
             long long end = base + kItems < n ? base + kItems : n;
-            long long b0 = (base + V - 1) / V;
-            for (long long bb = b0; bb * V < end; ++bb) {
+            // first frame boundary at or after base: the frame of base, plus
+            // one unless base starts that frame
+            long long bb = b_first + (v_first != 0 ? 1 : 0);
+            for (; bb * V < end; ++bb) {
                 int before = __popc(flags & ((1u << (int)(bb * V - base)) - 1u));
                 offsets[bb] = row + before;
             }
