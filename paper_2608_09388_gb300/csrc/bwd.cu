@@ -114,6 +114,72 @@ __global__ void __launch_bounds__(256)
     }
 }
 
+// Vectorised dz for rows of 16-byte chunks (cpr = C_out / VEC of them,
+// cpr dividing 256): a block takes kActVecItems / cpr consecutive rows
+// (ranges blockIdx.x, + gridDim.x, ...); thread t always holds chunk
+// t % cpr, so it sums its VEC columns over its rows in registers, and the
+// 256 / cpr row lanes of a column meet in shared memory in a fixed order.
+constexpr int kActVecItems = 1024;
+
+template <typename T>
+__global__ void __launch_bounds__(256)
+    act_bwd_vec_kernel(const T* __restrict__ y, const T* __restrict__ dy, const int32_t* count,
+                       long long capacity, int C_out, int act, T* __restrict__ dz,
+                       float* __restrict__ bpart, unsigned* status) {
+    constexpr int VEC = 16 / sizeof(T);
+    constexpr int kPer = kActVecItems / 256;
+    __shared__ float red[256 * VEC];
+    pdl_wait();
+    pdl_trigger();
+    const long long rows = clamp_rows(count, capacity, status);
+    const int t = threadIdx.x;
+    const int cpr = C_out / VEC, lanes = 256 / cpr;
+    const int c = t % cpr, rl = t / cpr;
+    const int R = kActVecItems / cpr;
+    float sum[VEC];
+#pragma unroll
+    for (int k = 0; k < VEC; ++k) sum[k] = 0.f;
+    for (long long r0 = (long long)blockIdx.x * R; r0 < rows; r0 += (long long)gridDim.x * R) {
+        uint4 yv[kPer], gv[kPer];
+#pragma unroll
+        for (int q = 0; q < kPer; ++q) {
+            const long long r = r0 + rl + (long long)q * lanes;
+            if (r < rows) {
+                yv[q] = *reinterpret_cast<const uint4*>(y + r * C_out + c * VEC);
+                gv[q] = *reinterpret_cast<const uint4*>(dy + r * C_out + c * VEC);
+            }
+        }
+#pragma unroll
+        for (int q = 0; q < kPer; ++q) {
+            const long long r = r0 + rl + (long long)q * lanes;
+            if (r >= rows) continue;
+            const T* yp = reinterpret_cast<const T*>(&yv[q]);
+            const T* gp = reinterpret_cast<const T*>(&gv[q]);
+            uint4 out;
+            T* op = reinterpret_cast<T*>(&out);
+#pragma unroll
+            for (int k = 0; k < VEC; ++k) {
+                const float yk = to_f(yp[k]);
+                float d = 1.f;
+                if (act == HC_ACT_ELU) d = yk > 0.f ? 1.f : yk + 1.f;
+                else if (act == HC_ACT_RELU) d = yk > 0.f ? 1.f : 0.f;
+                const float v = to_f(gp[k]) * d;
+                op[k] = from_f<T>(v);
+                sum[k] += v;
+            }
+            *reinterpret_cast<uint4*>(dz + r * C_out + c * VEC) = out;
+        }
+    }
+#pragma unroll
+    for (int k = 0; k < VEC; ++k) red[rl * C_out + c * VEC + k] = sum[k];
+    __syncthreads();
+    for (int o = t; o < C_out; o += 256) {
+        float s = 0.f;
+        for (int j = 0; j < lanes; ++j) s += red[j * C_out + o];
+        bpart[(long long)blockIdx.x * C_out + o] = s;
+    }
+}
+
 // dbias: block (32, 32) per 32 columns; row lane ty adds partials ty,
 // ty + 32, ... and the 32 lane sums are added in order.
 __global__ void dbias_kernel(const float* __restrict__ bpart, int nblocks, int C_out,
@@ -124,6 +190,7 @@ __global__ void dbias_kernel(const float* __restrict__ bpart, int nblocks, int C
     const int o = blockIdx.x * 32 + threadIdx.x;
     float s = 0.f;
     if (o < C_out)
+#pragma unroll 4
         for (int b = threadIdx.y; b < nblocks; b += 32) s += bpart[(long long)b * C_out + o];
     red[threadIdx.y][threadIdx.x] = s;
     __syncthreads();
@@ -687,92 +754,108 @@ __global__ void wgrad_reduce_kernel(const float* __restrict__ part, int K, int C
     }
 }
 
-// Rows whose 16-byte chunk count cpr divides 32: warp w takes rows w,
-// w + nwarps, ..., 32 at a time. Their row ranges come in one load (lane r
-// holds row r's); a ballot splits them into rows without taps, written as
-// zeros G rows per store, and rows with taps, for which lane
-// (g, c) = (lane / cpr, lane % cpr) sums chunk c of taps g, g + G, ...
-// (G = 32 / cpr groups, keys then P chunks loaded four at a time) and the
-// groups are added by a fixed shuffle tree.
+// Block-range gather-sum for rows of 16-byte chunks (cpr = C_in / VEC of
+// them). A block takes R consecutive input rows r0 .. r0 + R - 1 (ranges
+// blockIdx.x, + gridDim.x, ...). Their taps are one contiguous slice
+// taps[ptr[r0] .. ptr[r0 + R]) of the transposed mapping, copied to shared
+// memory in one coalesced pass (read from global memory instead when it does
+// not fit or the table is malformed there). The block then writes zero
+// chunks for the rows without taps and sums, for every (row with taps,
+// chunk) item, the P chunks of the row's taps in ascending key order, eight
+// loads in flight per thread. Every load of a round trip is issued by all
+// threads at once: row ranges, keys, then P.
+constexpr int kDgThreads = 256;
+constexpr int kDgMaxRows = 1024;
+constexpr int kDgKeys = 8192;
+
 template <typename T>
-__global__ void __launch_bounds__(256)
-    dgrad_warp_kernel(const T* __restrict__ P, const int32_t* __restrict__ ptr,
-                      const int32_t* __restrict__ taps, int x_rows, int L, int C_in,
-                      long long capacity, T* __restrict__ dx, unsigned* status) {
+__global__ void __launch_bounds__(kDgThreads, 4)
+    dgrad_range_kernel(const T* __restrict__ P, const int32_t* __restrict__ ptr,
+                       const int32_t* __restrict__ taps, int x_rows, int R, int C_in,
+                       long long capL, T* __restrict__ dx, unsigned* status) {
     constexpr int VEC = 16 / sizeof(T);
+    __shared__ int32_t s_ptr[kDgMaxRows + 1];
+    __shared__ uint16_t s_busy[kDgMaxRows];
+    __shared__ uint8_t s_on[kDgMaxRows];
+    __shared__ int32_t s_keys[kDgKeys];
+    __shared__ int s_nb;
     pdl_wait();
     pdl_trigger();
-    const int lane = threadIdx.x & 31;
-    const int cpr = C_in / VEC, G = 32 / cpr;
-    const int g = lane / cpr, c = (lane - g * cpr) * VEC;
-    const long long nwarps = (long long)gridDim.x * (blockDim.x >> 5);
-    const long long w = (long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-    // rows w, w + nwarps, w + 2 nwarps, ...: clustered active rows spread
-    // over all warps instead of loading a few
-    for (long long q0 = 0; w + q0 * nwarps < x_rows; q0 += 32) {
-        const long long jl = w + (q0 + lane) * nwarps;
-        const bool have = jl < x_rows;
-        const int pa = have ? __ldg(ptr + jl) : 0;
-        const int pb = have ? __ldg(ptr + jl + 1) : 0;
-        const long long left = (x_rows - 1 - w) / nwarps + 1 - q0;  // rows left for this warp
-        const int nr = left < 32 ? (int)left : 32;
-        // rows without taps: zeros, G rows per store instruction
-        const unsigned busy = __ballot_sync(0xffffffffu, have && pb != pa);
-        for (int r0 = 0; r0 < nr; r0 += G) {
-            const int r = r0 + g;
-            if (r < nr && !((busy >> r) & 1u))
-                *reinterpret_cast<uint4*>(dx + (w + (q0 + r) * nwarps) * C_in + c) =
-                    make_uint4(0u, 0u, 0u, 0u);
+    const int t = threadIdx.x, lane = t & 31;
+    const int cpr = C_in / VEC;
+    for (long long r0 = (long long)blockIdx.x * R; r0 < x_rows; r0 += (long long)gridDim.x * R) {
+        const int n = x_rows - r0 < R ? (int)(x_rows - r0) : R;
+        for (int i = t; i <= n; i += kDgThreads) s_ptr[i] = __ldg(ptr + r0 + i);
+        if (t == 0) s_nb = 0;
+        __syncthreads();
+        const int base = s_ptr[0], top = s_ptr[n];
+        const bool in_smem = base >= 0 && top >= base && top - base <= kDgKeys && top <= capL;
+        // the key slice, while the rows with taps are listed
+        if (in_smem)
+            for (int i = t; i < top - base; i += kDgThreads) s_keys[i] = __ldg(taps + base + i);
+        for (int i0 = 0; i0 < n; i0 += kDgThreads) {
+            const int i = i0 + t;
+            bool on = false;
+            if (i < n) {
+                const int a = s_ptr[i], b = s_ptr[i + 1];
+                const bool ok = a >= 0 && b >= a && b <= capL && (!in_smem || (a >= base && b <= top));
+                if (!ok) report(status, kErrIndex);
+                on = ok && b > a;
+                s_on[i] = on ? 1 : 0;
+            }
+            const unsigned bal = __ballot_sync(0xffffffffu, on);
+            int wbase = 0;
+            if (lane == 0 && bal) wbase = atomicAdd(&s_nb, __popc(bal));
+            wbase = __shfl_sync(0xffffffffu, wbase, 0);
+            if (on) s_busy[wbase + __popc(bal & ((1u << lane) - 1u))] = (uint16_t)i;
+        }
+        __syncthreads();
+        // rows without taps: zeros, consecutive chunks per thread
+        for (int f = t; f < n * cpr; f += kDgThreads) {
+            int c;
+            const int i = (int)div32(f, cpr, c);
+            if (!s_on[i])
+                *reinterpret_cast<uint4*>(dx + (r0 + i) * C_in + c * VEC) = make_uint4(0u, 0u, 0u, 0u);
         }
         // rows with taps
-        for (unsigned todo = busy; todo; todo &= todo - 1) {
-            const int r = __ffs(todo) - 1;
-            const long long j = w + (q0 + r) * nwarps;
-            int a = __shfl_sync(0xffffffffu, pa, r), b = __shfl_sync(0xffffffffu, pb, r);
-            if (a < 0 || b < a || (long long)b > capacity * L) {
-                if (lane == 0) report(status, kErrIndex);
-                b = a;
-            }
+        const int nb = s_nb;
+        const int32_t* kp = in_smem ? s_keys : taps;
+        const int koff = in_smem ? base : 0;
+        for (int f = t; f < nb * cpr; f += kDgThreads) {
+            int c;
+            const int bi = (int)div32(f, cpr, c);
+            const int i = s_busy[bi];
+            const int a = s_ptr[i] - koff, b = s_ptr[i + 1] - koff;
             float acc[VEC];
 #pragma unroll
             for (int k = 0; k < VEC; ++k) acc[k] = 0.f;
-            for (int e0 = a + g; e0 < b; e0 += 4 * G) {
-                int key[4];
+            for (int e0 = a; e0 < b; e0 += 8) {
+                uint4 raw[8];
+                bool use[8];
 #pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    const int e = e0 + i * G;
-                    key[i] = e < b ? __ldg(taps + e) : -1;
-                    if (e < b && (key[i] < 0 || (long long)key[i] >= capacity * L)) {
-                        report(status, kErrIndex);
-                        key[i] = -1;
-                    }
-                }
-                uint4 raw[4];
-#pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    if (key[i] < 0) continue;
+                for (int q = 0; q < 8; ++q) {
+                    const int key = e0 + q < b ? kp[e0 + q] : -1;
+                    use[q] = key >= 0 && (long long)key < capL;
+                    if (e0 + q < b && !use[q]) report(status, kErrIndex);
                     // key n*L + l: P's row n, slot l starts at (n*L + l)*C_in
-                    raw[i] = *reinterpret_cast<const uint4*>(P + (long long)key[i] * C_in + c);
+                    if (use[q])
+                        raw[q] = *reinterpret_cast<const uint4*>(P + (long long)key * C_in + c * VEC);
                 }
 #pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    if (key[i] < 0) continue;
-                    const T* v = reinterpret_cast<const T*>(&raw[i]);
+                for (int q = 0; q < 8; ++q) {
+                    if (!use[q]) continue;
+                    const T* v = reinterpret_cast<const T*>(&raw[q]);
 #pragma unroll
                     for (int k = 0; k < VEC; ++k) acc[k] += to_f(v[k]);
                 }
             }
-            for (int o = cpr; o < 32; o <<= 1)
+            uint4 out;
+            T* ov = reinterpret_cast<T*>(&out);
 #pragma unroll
-                for (int k = 0; k < VEC; ++k) acc[k] += __shfl_xor_sync(0xffffffffu, acc[k], o);
-            if (g == 0) {
-                uint4 out;
-                T* ov = reinterpret_cast<T*>(&out);
-#pragma unroll
-                for (int k = 0; k < VEC; ++k) ov[k] = from_f<T>(acc[k]);
-                *reinterpret_cast<uint4*>(dx + j * C_in + c) = out;
-            }
+            for (int k = 0; k < VEC; ++k) ov[k] = from_f<T>(acc[k]);
+            *reinterpret_cast<uint4*>(dx + (r0 + i) * C_in + c * VEC) = out;
         }
+        __syncthreads();  // the shared tables are reused by the next range
     }
 }
 
@@ -784,14 +867,19 @@ hc_status launch_dgrad_typed(const DeviceCtx* ctx, const void* P, const int32_t*
     const int vec16 = 16 / (int)sizeof(T);
     const bool wide = C_in % vec16 == 0 && al % 16 == 0;
     const int vec = wide ? vec16 : 1;
-    const int cpr = C_in / vec16;
-    if (wide && cpr <= 32 && (32 % cpr) == 0) {
-        long long wblocks = ((long long)x_rows + 255) / 256;  // 8 warps x 32 rows per block
-        if (wblocks > (long long)ctx->num_sms * 8) wblocks = (long long)ctx->num_sms * 8;
-        if (wblocks < 1) wblocks = 1;
-        return launch_pdl(dgrad_warp_kernel<T>, dim3((unsigned)wblocks), dim3(256), 0, s,
-                          "dgrad_warp_kernel", (const T*)P, ptr, taps, x_rows, L, C_in, capacity,
-                          (T*)dx, ctx->status);
+    if (wide && (long long)kDgMaxRows * (C_in / vec16) < (1ll << 31)) {
+        // ranges of R rows, about one per resident block (4 per SM)
+        const long long want = (long long)ctx->num_sms * 4;
+        long long R = ((long long)x_rows + want - 1) / want;
+        R = (R + 31) / 32 * 32;
+        if (R < 256) R = 256;
+        if (R > kDgMaxRows) R = kDgMaxRows;
+        long long blocks = ((long long)x_rows + R - 1) / R;
+        if (blocks > want) blocks = want;
+        if (blocks < 1) blocks = 1;
+        return launch_pdl(dgrad_range_kernel<T>, dim3((unsigned)blocks), dim3(kDgThreads), 0, s,
+                          "dgrad_range_kernel", (const T*)P, ptr, taps, x_rows, (int)R, C_in,
+                          capacity * L, (T*)dx, ctx->status);
     }
     long long blocks = ((long long)x_rows * (C_in / vec) + 255) / 256;
     const long long cap = (long long)ctx->num_sms * 8;
@@ -872,8 +960,14 @@ hc_status launch_conv_bwd(const DeviceCtx* ctx, const BwdArgs& b, cudaStream_t s
         }
     }
     const long long items = (long long)splits * T;
-    long long act_blocks_ll = ((long long)b.capacity + kActRowsPerBlock - 1) / kActRowsPerBlock;
-    if (act_blocks_ll > 8ll * ctx->num_sms) act_blocks_ll = 8ll * ctx->num_sms;
+    // dz: 16-byte chunks when a row is a whole number of them dividing 256
+    const int act_vec = 16 / eb, act_cpr = b.C_out / act_vec;
+    const bool act_wide = b.C_out % act_vec == 0 && 256 % act_cpr == 0 &&
+                          ((uintptr_t)b.y | (uintptr_t)b.dy) % 16 == 0;
+    const long long act_rows = act_wide ? kActVecItems / act_cpr : kActRowsPerBlock;
+    long long act_blocks_ll = ((long long)b.capacity + act_rows - 1) / act_rows;
+    const long long act_cap = (act_wide ? 4ll : 8ll) * ctx->num_sms;
+    if (act_blocks_ll > act_cap) act_blocks_ll = act_cap;
     const int act_blocks = (int)(act_blocks_ll > 0 ? act_blocks_ll : 1);
 
     // workspace: dz | P | W^T | wgrad partials | dbias partials
@@ -892,7 +986,16 @@ hc_status launch_conv_bwd(const DeviceCtx* ctx, const BwdArgs& b, cudaStream_t s
     float* bpart = (float*)(ws + dz_bytes + p_bytes + wt_bytes + part_bytes);
 
     hc_status st;
-    if (bf)
+    if (act_wide && bf)
+        st = launch_pdl(act_bwd_vec_kernel<__nv_bfloat16>, dim3((unsigned)act_blocks), dim3(256), 0,
+                        s, "act_bwd_vec_kernel", (const __nv_bfloat16*)b.y,
+                        (const __nv_bfloat16*)b.dy, b.count, (long long)b.capacity, b.C_out, b.act,
+                        (__nv_bfloat16*)dz, bpart, ctx->status);
+    else if (act_wide)
+        st = launch_pdl(act_bwd_vec_kernel<float>, dim3((unsigned)act_blocks), dim3(256), 0, s,
+                        "act_bwd_vec_kernel", (const float*)b.y, (const float*)b.dy, b.count,
+                        (long long)b.capacity, b.C_out, b.act, (float*)dz, bpart, ctx->status);
+    else if (bf)
         st = launch_pdl(act_bwd_kernel<__nv_bfloat16>, dim3((unsigned)act_blocks), dim3(256), 0, s,
                         "act_bwd_kernel", (const __nv_bfloat16*)b.y, (const __nv_bfloat16*)b.dy,
                         b.count, (long long)b.capacity, b.C_out, b.act, (__nv_bfloat16*)dz, bpart,

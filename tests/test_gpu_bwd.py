@@ -193,6 +193,22 @@ def test_backward_full_size_layer():
     check_against_oracle(c, run_bwd(c))
 
 
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_backward_many_taps_per_range(dtype):
+    """A synthetic mapping with ~48 taps per input row: the first 256-row
+    range holds more keys than the input gradient stages in shared memory
+    (8192), so it reads them from global memory; the tail range stages them."""
+    rng = np.random.default_rng(11)
+    L, n, x_rows, C_in, C_out = 24, 600, 300, 16, 32
+    rb = rng.integers(-1, x_rows, size=(L, n)).astype(np.int32)
+    x = inputs.features(rng, (x_rows, C_in), dtype)
+    W = inputs.weights(rng, L * C_in, C_out, dtype)
+    y = np.zeros((n, C_out), dtype=x.dtype)
+    dy = inputs.features(rng, (n, C_out), dtype)
+    c = dict(x=x, W=W, y=y, dy=dy, rb=rb, n=n, cap=n, act=oracle.ACT_NONE, dtype=dtype)
+    check_against_oracle(c, run_bwd(c, want=("dx",)), want=("dx",))
+
+
 def test_backward_bad_taps_reported():
     """A malformed transposed mapping is reported and its entries skipped."""
     c = _case(8, 2, 80, 5, 8, 16, "f32", oracle.LAYOUT_DENSE, oracle.ACT_NONE)
