@@ -110,8 +110,9 @@ __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr, uint32_t lbo
 // pieces XOR-swizzled by row so that neither the writes nor the reads have
 // bank conflicts) and leave it so that each store instruction writes eight
 // rows x 64 contiguous bytes, instead of 32 scattered 16-byte pieces. Each
-// row goes to its compact position (row_y, 0 = none) and to its dense
-// position of the fused scatter (row_d, 0 = none).
+// row goes to its compact position and to its dense position of the fused
+// scatter: lane i stores rows 8k + i/4 (k = 0..3), whose addresses it holds
+// in yk[k] and dk[k] (0 = not written).
 // Activation and bf16 rounding of a chunk: p[h] holds columns 2h (low
 // half) and 2h + 1 (high half).
 template <int ACT>
@@ -125,23 +126,27 @@ __device__ __forceinline__ void epilogue_pack(const uint32_t (&r)[32], uint32_t 
 }
 
 __device__ __forceinline__ void epilogue_store(const uint32_t (&p)[16], uint32_t stage, int lane,
-                                               long long row_y, long long row_d, int col0,
-                                               int C_out) {
+                                               const long long (&yk)[4], const long long (&dk)[4],
+                                               int col0, int C_out) {
 #pragma unroll
     for (int j8 = 0; j8 < 4; ++j8)
         sts_v4(stage + (uint32_t)(lane * 64 + ((j8 ^ ((lane >> 1) & 3)) << 4)),
                make_uint4(p[4 * j8], p[4 * j8 + 1], p[4 * j8 + 2], p[4 * j8 + 3]));
     __syncwarp();
+    // all four shared-memory reads first, then the stores (the reads do not
+    // wait behind the previous row group's stores)
+    uint4 v[4];
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
         const int R = 8 * k + (lane >> 2), piece = lane & 3;
-        const uint4 v = lds_u4(stage + (uint32_t)(R * 64 + ((piece ^ ((R >> 1) & 3)) << 4)));
-        const long long yR = __shfl_sync(0xffffffffu, row_y, R);
-        const long long dR = __shfl_sync(0xffffffffu, row_d, R);
-        const int col = col0 + piece * 8;
-        if (col < C_out) {
-            if (yR) *reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(yR) + col) = v;
-            if (dR) *reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(dR) + col) = v;
+        v[k] = lds_u4(stage + (uint32_t)(R * 64 + ((piece ^ ((R >> 1) & 3)) << 4)));
+    }
+    const int col = col0 + (lane & 3) * 8;
+    if (col < C_out) {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            if (yk[k]) *reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(yk[k]) + col) = v[k];
+            if (dk[k]) *reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(dk[k]) + col) = v[k];
         }
     }
     __syncwarp();  // the buffer is reused by the next chunk
@@ -149,11 +154,11 @@ __device__ __forceinline__ void epilogue_store(const uint32_t (&p)[16], uint32_t
 
 template <int ACT>
 __device__ __forceinline__ void epilogue_chunk(const uint32_t (&r)[32], uint32_t stage, int lane,
-                                               long long row_y, long long row_d, int col0,
-                                               int C_out) {
+                                               const long long (&yk)[4], const long long (&dk)[4],
+                                               int col0, int C_out) {
     uint32_t p[16];
     epilogue_pack<ACT>(r, p);
-    epilogue_store(p, stage, lane, row_y, row_d, col0, C_out);
+    epilogue_store(p, stage, lane, yk, dk, col0, C_out);
 }
 
 // Group-norm statistics of one warp's 32 rows (lane = row). Every lane
@@ -807,6 +812,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int gn_b0 = __shfl_sync(0xffffffffu, gn_b, 0);
             const bool gn_whole = __all_sync(0xffffffffu, gn_b >= 0 && gn_b == gn_b0);
             float run_mean = 0.f, run_m2 = 0.f;
+            // the addresses of the rows this lane stores in every chunk
+            long long yk[4], dk[4];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                yk[k] = __shfl_sync(0xffffffffu, row_y, 8 * k + (lane >> 2));
+                dk[k] = __shfl_sync(0xffffffffu, row_d, 8 * k + (lane >> 2));
+            }
             if (!mbar_wait(tfull_bar(acc), ph, abort_flag, a.status)) break;
             tc_fence_after();
             const uint32_t stage = epi0 + (uint32_t)ew * 2048u;
@@ -823,10 +835,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                 for (int k = 1; k < BN / 32; ++k)
                     if (cb == k) bias_l = bias_c[k];
+                if (a.bias)
 #pragma unroll
-                for (int j = 0; j < 32; ++j)
-                    r[j] = __float_as_uint(__uint_as_float(r[j]) +
-                                           __shfl_sync(0xffffffffu, bias_l, j));
+                    for (int j = 0; j < 32; ++j)
+                        r[j] = __float_as_uint(__uint_as_float(r[j]) +
+                                               __shfl_sync(0xffffffffu, bias_l, j));
                 if (a.gn_part) {
                     // with statistics the activation is the identity (it
                     // follows the normalisation)
@@ -835,13 +848,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (col0 < C_out)
                         gn_stats_chunk(a, p, col0, (m0 + ew * 32) / 32, gn_b, gn_whole, lane,
                                        run_mean, run_m2);
-                    epilogue_store(p, stage, lane, row_y, row_d, col0, C_out);
+                    epilogue_store(p, stage, lane, yk, dk, col0, C_out);
                 } else if (a.act == HC_ACT_ELU)
-                    epilogue_chunk<HC_ACT_ELU>(r, stage, lane, row_y, row_d, col0, C_out);
+                    epilogue_chunk<HC_ACT_ELU>(r, stage, lane, yk, dk, col0, C_out);
                 else if (a.act == HC_ACT_RELU)
-                    epilogue_chunk<HC_ACT_RELU>(r, stage, lane, row_y, row_d, col0, C_out);
+                    epilogue_chunk<HC_ACT_RELU>(r, stage, lane, yk, dk, col0, C_out);
                 else
-                    epilogue_chunk<HC_ACT_NONE>(r, stage, lane, row_y, row_d, col0, C_out);
+                    epilogue_chunk<HC_ACT_NONE>(r, stage, lane, yk, dk, col0, C_out);
             }
             tc_fence_before();
             mbar_arrive(tempty_bar(acc));
