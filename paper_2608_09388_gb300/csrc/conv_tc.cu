@@ -23,9 +23,11 @@
 //   warp 8     MMA issuer (one thread): 4 x tcgen05.mma (K = 16 each) per
 //              stage into a TMEM accumulator, tcgen05.commit frees the stage;
 //   warps 4-7  epilogue: tcgen05.ld the 128 x BN fp32 accumulator (warp w
-//              reads TMEM lanes 32*(w%4)..+32), add bias, activation, round
-//              to bf16 and store. Two accumulators (2*BN TMEM columns) let
-//              the epilogue of one tile overlap the main loop of the next.
+//              reads TMEM lanes 32*(w%4)..+32), activation, round to bf16
+//              and store; then tcgen05.st the bias of the tile after next
+//              into every row of the freed accumulator, onto which its MMAs
+//              accumulate. Two accumulators (2*BN TMEM columns) let the
+//              epilogue of one tile overlap the main loop of the next.
 // Shared-memory operand layouts (canonical tcgen05 forms, 128-byte swizzle):
 //   A: K-major, row r of the 128-row tile at r*128 bytes, 16-byte chunk q
 //      stored at chunk q ^ (r % 8); 8-row groups 1024 bytes apart (SBO).
@@ -106,7 +108,7 @@ __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr, uint32_t lbo
 
 // Epilogue of one 32-column chunk of a warp's 32 output rows: activation,
 // bf16 rounding (RNE), then the stores. Lane i holds row i's 32 fp32 sums
-// (bias added) in r. The rows go through a 2 KB shared buffer (16-byte
+// (bias included) in r. The rows go through a 2 KB shared buffer (16-byte
 // pieces XOR-swizzled by row so that neither the writes nor the reads have
 // bank conflicts) and leave it so that each store instruction writes eight
 // rows x 64 contiguous bytes, instead of 32 scattered 16-byte pieces. Each
@@ -589,10 +591,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint32_t st_ph = 0;  // its phase parity ((it / stages) & 1)
             int lt = 0;
             bool ok = true;
+            const bool has_bias = a.bias != nullptr;  // accumulators start at the bias
             for (long long w = blockIdx.x; w < work_total && ok; w += gridDim.x, ++lt) {
                 const int acc = lt & 1;
                 const uint32_t acc_ph = (uint32_t)((lt >> 1) & 1);
-                if (!mbar_wait(tempty_bar(acc), acc_ph ^ 1u, abort_flag, a.status)) {
+                // released by the epilogue once it holds the bias (or is free)
+                if (!mbar_wait(tempty_bar(acc), acc_ph, abort_flag, a.status)) {
                     ok = false;
                     break;
                 }
@@ -615,7 +619,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     for (int k = 0; k < kBK / 16; ++k) {
                         const uint64_t ad = smem_desc_sw128(a_st + k * 32, 16, 1024);
                         const uint64_t bd = smem_desc_sw128(b_st + k * 16 * 128, kBK * 128, 1024);
-                        tc_mma_bf16(d_tmem, ad, bd, C::kIdesc, (kb | k) != 0 ? 1u : 0u);
+                        tc_mma_bf16(d_tmem, ad, bd, C::kIdesc, (has_bias || (kb | k) != 0) ? 1u : 0u);
                     }
                     tc_commit(empty_bar(s));
                     ++it;
@@ -772,6 +776,31 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ------------------------------------------------------------ epilogue
         const int ew = warp - kProducerWarps;  // == warp % 4: TMEM lanes 32*ew..+32
         __nv_bfloat16* __restrict__ y = static_cast<__nv_bfloat16*>(a.y);
+        // Accumulator buffer acc is handed to the MMA warp holding the bias of
+        // tile w in every row (the MMAs then accumulate onto it), so the bias
+        // costs the epilogue nothing once the sums are ready.
+        auto release = [&](int acc, long long w) {
+            if (a.bias && w < work_total) {
+                const int n0 = ((int)w % n_tiles) * BN;
+#pragma unroll 1
+                for (int cb = 0; cb < BN / 32; ++cb) {
+                    uint32_t r[32];
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) {
+                        const int col = n0 + cb * 32 + j;
+                        r[j] = col < C_out ? __float_as_uint(__ldg(a.bias + col)) : 0u;
+                    }
+                    tmem_st_32x32b_x32(tmem_base + ((uint32_t)(ew * 32) << 16) +
+                                           (uint32_t)(acc * BN + cb * 32),
+                                       r);
+                }
+                tmem_st_wait();
+            }
+            tc_fence_before();
+            mbar_arrive(tempty_bar(acc));
+        };
+        release(0, blockIdx.x);
+        release(1, blockIdx.x + (long long)gridDim.x);
         int lt = 0;
         for (long long w = blockIdx.x; w < work_total; w += gridDim.x, ++lt) {
             const long long m0 = (long long)((int)w / n_tiles) * kBM;
@@ -780,8 +809,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t ph = (uint32_t)((lt >> 1) & 1);
             // Everything that does not need the accumulator is loaded while
             // the main loop runs: this lane's row addresses (0 = not
-            // written; the fused scatter's needs the row's coordinate) and
-            // the bias of each 32-column chunk (lane j holds column j's).
+            // written; the fused scatter's needs the row's coordinate).
             const long long row = m0 + ew * 32 + lane;
             const bool rvalid = row < rows;
             const long long row_y = (rvalid && y) ? (long long)(y + row * C_out) : 0;
@@ -793,12 +821,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                                         ((long long)b * a.out_V + v) * C_out);
                 else
                     report(a.status, kErrIndex);
-            }
-            float bias_c[BN / 32];
-#pragma unroll
-            for (int cb = 0; cb < BN / 32; ++cb) {
-                const int bcol = n0 + cb * 32 + lane < C_out ? n0 + cb * 32 + lane : C_out - 1;
-                bias_c[cb] = a.bias ? __ldg(a.bias + bcol) : 0.f;
             }
             int gn_b = -1;  // frame of this lane's row, for the group-norm statistics
             if (a.gn_part && rvalid) {
@@ -829,17 +851,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                                    r);
                 tmem_ld_wait();
                 const int col0 = n0 + cb * 32;
-                // Bias of the chunk's 32 columns (loaded above), broadcast by
-                // shuffles (every lane takes part).
-                float bias_l = bias_c[0];
-#pragma unroll
-                for (int k = 1; k < BN / 32; ++k)
-                    if (cb == k) bias_l = bias_c[k];
-                if (a.bias)
-#pragma unroll
-                    for (int j = 0; j < 32; ++j)
-                        r[j] = __float_as_uint(__uint_as_float(r[j]) +
-                                               __shfl_sync(0xffffffffu, bias_l, j));
                 if (a.gn_part) {
                     // with statistics the activation is the identity (it
                     // follows the normalisation)
@@ -856,8 +867,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 else
                     epilogue_chunk<HC_ACT_NONE>(r, stage, lane, yk, dk, col0, C_out);
             }
-            tc_fence_before();
-            mbar_arrive(tempty_bar(acc));
+            release(acc, w + 2 * (long long)gridDim.x);  // the tile after next
         }
     }
 
