@@ -4,8 +4,9 @@
 One step = one pass of the hot path over one batch of the 10475-vertex
 workload (B = 32 frames, spiral length L = 12, 64 -> 128 channels, bf16,
 clustered contact masks at ~5% density):
-    hc_mask_compact              mask -> coords, row_of, offsets, count (Eq. 2)
-    hc_conv_rulebook             tap -> input-row mapping (Eq. 4)
+    hc_mask_compact_rulebook     mask -> coords, row_of, offsets, count (Eq. 2) and
+                                 the tap -> input-row mapping (Eq. 4): a count pass,
+                                 then one fused pass per (frame, 1024 vertices)
     hc_sparse_conv_rulebook_fwd  gather + tcgen05 contraction + bias + ELU (Eq. 5),
                                  writing the compact rows and, fused into the same
                                  epilogue, their scatter into the dense [B, V, 128]
@@ -255,9 +256,8 @@ def run_ours(args, rank, world, local_rank):
     stream = torch.cuda.Stream(device=dev)
 
     def step(s):
-        hc.hc_mask_compact(s.mask, s.coords, s.row_of, s.offs, s.count, stream)
-        hc.hc_conv_rulebook(s.coords, s.row_of, s.count, spiral, B, V, hc.HC_LAYOUT_DENSE, s.rb,
-                            stream)
+        hc.hc_mask_compact_rulebook(s.mask, spiral, hc.HC_LAYOUT_DENSE, s.coords, s.row_of,
+                                    s.offs, s.count, s.rb, stream)
         hc.hc_sparse_conv_rulebook_fwd(s.x, s.rb, s.count, Wt, bias, ly.act, s.y,
                                        coords=s.coords, out=s.out, stream=stream)
 
@@ -268,8 +268,10 @@ def run_ours(args, rank, world, local_rank):
     def dense_only(s):
         hc.hc_spiral_conv_fwd(s.x, spiral, Wt, bias, ly.act, s.dense, stream)
 
-    # compaction (2, or 3 with the pre-scan), rulebook, conv with the fused scatter
-    kernels_per_step = 2 + (1 if (B * V + 4095) // 4096 > 1024 else 0) + 1 + 1
+    # count pass (+ the tile pre-scan past 1024 tiles), the fused compaction +
+    # mapping pass (or the write and mapping kernels past its limits), conv
+    fused = V <= 65535
+    kernels_per_step = 1 + (1 if (B * V + 4095) // 4096 > 1024 else 0) + (1 if fused else 2) + 1
 
     # W warm-up steps, then one priming pass over every input set (both
     # eager, untimed; they also set up the library's per-stream workspace).
@@ -416,8 +418,9 @@ def run_ours(args, rank, world, local_rank):
             "active_rows_per_step": mean_rows,
             "rotation_sets": R,
             "launches_before_timed": (args.warmup + R) * kernels_per_step,
-            "step": "hc_mask_compact + hc_conv_rulebook + hc_sparse_conv_rulebook_fwd "
-                    "(compact rows + scatter to dense [B,V,C_out] fused in its epilogue)",
+            "step": "hc_mask_compact_rulebook (count pass + fused compaction/Eq. 4 mapping) "
+                    "+ hc_sparse_conv_rulebook_fwd (compact rows + scatter to dense "
+                    "[B,V,C_out] fused in its epilogue)",
             "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
             "l2": f"{R} rotating input sets of {set_bytes / 2**20:.1f} MiB "
                   f"({R * set_bytes / 2**20:.0f} MiB > 2x L2 {l2 / 2**20:.0f} MiB)",
@@ -544,9 +547,8 @@ def measure_e2e(torch, hc, sets, w, spiral, Wt, bias, stream, dev, steps):
         if i >= nb:
             stream.wait_event(drained[b])  # step i - 2's rows have been read back
         with torch.cuda.stream(stream):
-            hc.hc_mask_compact(mask_d[b], o.coords, o.row_of, o.offs, o.count, stream)
-            hc.hc_conv_rulebook(o.coords, o.row_of, o.count, spiral, B, V, hc.HC_LAYOUT_DENSE,
-                                o.rb, stream)
+            hc.hc_mask_compact_rulebook(mask_d[b], spiral, hc.HC_LAYOUT_DENSE, o.coords,
+                                        o.row_of, o.offs, o.count, o.rb, stream)
             hc.hc_sparse_conv_rulebook_fwd(x_d[b], o.rb, o.count, Wt, bias, ly.act, o.y,
                                            coords=o.coords, out=o.out, stream=stream)
             cnt_h[b].copy_(o.count, non_blocking=True)
@@ -629,9 +631,8 @@ def run_sweep(torch, hc, dev, stream):
     for d, m in zip(w.densities, w.masks):
         mt = torch.from_numpy(m).to(dev)
         with torch.cuda.stream(stream):
-            hc.hc_mask_compact(mt, coords, row_of, offs, count, stream)
-            hc.hc_conv_rulebook(coords, row_of, count, spiral, B, V, hc.HC_LAYOUT_DENSE, rb,
-                                stream)
+            hc.hc_mask_compact_rulebook(mt, spiral, hc.HC_LAYOUT_DENSE, coords, row_of, offs,
+                                        count, rb, stream)
         n = int(np.count_nonzero(m))
         ms = timeit(lambda: hc.hc_sparse_conv_rulebook_fwd(x, rb, count, Wt, bias, ly.act, y,
                                                            stream=stream))
@@ -880,8 +881,8 @@ def run_kappa(torch, hc, dev, stream, K=10, kappa=3, density=0.1):
     def sparse():
         hc.hc_mask_select_topk(alpha, kappa, sel, stream)
         hc.hc_kappa_masks(masks, sel, B, fm, stream)
-        hc.hc_mask_compact(fm, coords, row_of, offs, count, stream)
-        hc.hc_conv_rulebook(coords, row_of, count, sp, F, V, hc.HC_LAYOUT_COMPACT, rb, stream)
+        hc.hc_mask_compact_rulebook(fm, sp, hc.HC_LAYOUT_COMPACT, coords, row_of, offs, count,
+                                    rb, stream)
         hc.hc_gather_rows(x, coords, count, kappa, hs[0], stream)
         for i, ly in enumerate(w.layers):
             dst = hs[i + 1] if i + 1 < len(w.layers) else out

@@ -166,6 +166,27 @@ hc_status hc_conv_rulebook(const int32_t* coords, const int32_t* row_of, const i
                            int32_t* rulebook, hc_stream_t stream);
 
 /*
+ * hc_mask_compact_rulebook -- hc_mask_compact followed by hc_conv_rulebook on
+ * its output (Eq. 2 and the Eq. 4 indexing matrix), in two kernels when
+ * V <= 65535: a count pass, then one pass per (frame, block of 1024
+ * vertices) that ranks the frame's mask bytes in shared memory and writes
+ * coords, row_of, batch_offsets, count and the rulebook columns of its
+ * active vertices, every tap lookup answered from shared memory. Larger
+ * frames run the two operations' own kernels. The results are identical to
+ * the two calls (bit-exact).
+ *   mask, B, V, coords, row_of, batch_offsets, count   as hc_mask_compact
+ *                                                      (row_of required)
+ *   spiral, L, x_layout, rulebook                      as hc_conv_rulebook
+ * Out-of-range spiral entries are reported (HC_ERR_INVALID_INDEX) and their
+ * taps stored as -1. Uses the library's per-stream workspace (one int32 per
+ * 4096 mask bytes).
+ */
+hc_status hc_mask_compact_rulebook(const uint8_t* mask, int B, int V, const int32_t* spiral, int L,
+                                   hc_layout x_layout, int32_t* coords, int32_t* row_of,
+                                   int32_t* batch_offsets, int32_t* count, int32_t* rulebook,
+                                   hc_stream_t stream);
+
+/*
  * hc_sparse_conv_rulebook_fwd -- the sparse convolution (Eq. 5) with fused
  * bias (Eq. 6) and activation (Eq. 10), through a precomputed rulebook:
  *   y[n, o] = act( bias[o] + sum_{l<L, r = rulebook[l*capacity+n] >= 0}

@@ -226,6 +226,206 @@ __global__ void __launch_bounds__(kThreads)
     }
 }
 
+// ---------------------------------------------------------------- compaction + Eq. 4 mapping
+// The write pass fused with the mapping (the rulebook of hc_conv_rulebook):
+// CTA (b, s) rebuilds frame b's activity and ranks in shared memory, per
+// 16-byte chunk of the mask bytes from the aligned byte below b*V: the
+// chunk's 16 activity flags and the frame's active rows before it, so that
+// the rank of vertex p (active rows of the frame before p) is the chunk's
+// count plus a popcount. It then writes row_of, coords and the rulebook
+// columns of the active vertices in its portion [s*kMapPortion,
+// (s+1)*kMapPortion); every tap lookup row_of[b, u] of Eq. 4 is a
+// shared-memory read. The mask, the ranks and the first spiral entries of
+// the portion's active vertices do not depend on the count pass and are
+// read before waiting on it; after the wait only the tile counts before the
+// frame are read (frame offset = those counts + the active bytes of the
+// frame's own 4096-byte tile before b*V, counted here). Shared memory stays
+// small (6 bytes per 16 vertices + 2 per portion vertex) so that the conv
+// that follows can start on the same SMs.
+constexpr int kMapThreads = 256;
+constexpr int kMapPortion = 1024;
+constexpr int kMapMaxV = 65535;
+constexpr int kMapMaxL = HC_MAX_SPIRAL;
+constexpr int kMapPre = 4;  // tap entries per thread read before the wait
+
+struct MapArgs {
+    const uint8_t* mask;
+    long long n;  // B * V
+    int B, V, L, x_layout, S, nch;
+    const int32_t* spiral;
+    const int32_t* tile_counts;
+    int num_tiles, prescanned;
+    int32_t* coords;
+    int32_t* row_of;
+    int32_t* offsets;
+    int32_t* count;
+    int32_t* rulebook;
+    unsigned* status;
+};
+
+size_t map_smem_bytes(int nch) {
+    return ((size_t)nch * 4 + (size_t)nch * 2 + 15) / 16 * 16 + sizeof(uint16_t) * kMapPortion;
+}
+
+// Exclusive block scan of v (kMapThreads threads); total in *tot.
+__device__ __forceinline__ int block_excl_scan(int v, int* red, int* tot) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+    }
+    __syncthreads();  // red[] is free
+    if (lane == 31) red[warp] = x;
+    __syncthreads();
+    int before = 0, all = 0;
+#pragma unroll
+    for (int w = 0; w < kMapThreads / 32; ++w) {
+        before += w < warp ? red[w] : 0;
+        all += red[w];
+    }
+    *tot = all;
+    return before + x - v;
+}
+
+__global__ void __launch_bounds__(kMapThreads) compact_map_kernel(const MapArgs a) {
+    extern __shared__ __align__(16) uint8_t map_smem[];
+    __shared__ int red[kMapThreads / 32];
+    const int V = a.V, L = a.L;
+    int32_t* s_rank = reinterpret_cast<int32_t*>(map_smem);           // [nch]
+    uint16_t* s_flag = reinterpret_cast<uint16_t*>(s_rank + a.nch);    // [nch]
+    uint16_t* act_v = reinterpret_cast<uint16_t*>(map_smem + ((size_t)a.nch * 6 + 15) / 16 * 16);
+    const int tid = threadIdx.x;
+    const int b = blockIdx.x / a.S, s = blockIdx.x - b * a.S;
+    const long long fb = (long long)b * V;  // the frame's first mask byte
+    const long long a0 = fb & ~15ll;
+    const int sh = (int)(fb - a0);  // vertex p is bit (p + sh) of the chunk list
+    const int nch = (int)((fb + V - a0 + 15) >> 4);
+
+    // active bytes of the frame's 4096-byte tile before fb (loaded with the
+    // frame's own chunks)
+    const int tb = (int)(fb / kTile);
+    uint32_t pf = 0;
+    {
+        const long long g = (long long)tb * kTile + 16ll * tid;
+        if (g < fb) {
+            pf = load_flags(a.mask, a.n, g);
+            const long long hi = fb - g;
+            if (hi < kItems) pf &= (1u << hi) - 1u;
+        }
+    }
+    // thread t takes chunks t*m .. t*m + m - 1: their flags, one block scan of
+    // the per-thread counts, then the chunks' ranks
+    const int m = (nch + kMapThreads - 1) / kMapThreads;
+    const int cb0 = tid * m;
+    int cnt = 0;
+#pragma unroll 4
+    for (int j = 0; j < m; ++j) {
+        const int c = cb0 + j;
+        if (c < nch) {
+            const long long g = a0 + 16ll * c;
+            uint32_t f = load_flags(a.mask, a.n, g);
+            const long long lo = fb - g, hi = fb + V - g;  // in-frame bytes lo .. hi-1
+            if (lo > 0) f &= 0xFFFFu << lo;
+            if (hi < kItems) f &= (1u << hi) - 1u;
+            s_flag[c] = (uint16_t)f;
+            cnt += __popc(f);
+        }
+    }
+    int fc;  // active rows of frame b
+    int r = block_excl_scan(cnt, red, &fc);
+    for (int j = 0; j < m; ++j) {
+        const int c = cb0 + j;
+        if (c < nch) {
+            s_rank[c] = r;
+            r += __popc((uint32_t)s_flag[c]);
+        }
+    }
+    const int part = block_sum(__popc(pf), red);  // synchronises: the chunk tables are complete
+    // rank of vertex p (active rows of the frame before it) and its activity
+    auto rank_of = [&](int p, bool& on) {
+        const int q = p + sh, c = q >> 4, k = q & 15;
+        const uint32_t f = s_flag[c];
+        on = (f >> k) & 1u;
+        return s_rank[c] + __popc(f & ((1u << k) - 1u));
+    };
+    const int v0 = s * kMapPortion, v1 = v0 + kMapPortion < V ? v0 + kMapPortion : V;
+    bool on;
+    const int R0 = rank_of(v0, on);  // v0 < V
+    const int R1 = v1 < V ? rank_of(v1, on) : fc;
+    const int nact = R1 - R0;
+    for (int p = v0 + tid; p < v1; p += kMapThreads) {
+        const int r = rank_of(p, on);
+        if (on) act_v[r - R0] = (uint16_t)(p - v0);
+    }
+    __syncthreads();
+    // the first tap entries of this thread (item i: slot l = i / nact,
+    // active vertex k = i % nact of the portion)
+    const int items = nact * L;
+    int u_pre[kMapPre];
+#pragma unroll
+    for (int q = 0; q < kMapPre; ++q) {
+        const int i = tid + q * kMapThreads;
+        u_pre[q] = -1;
+        if (i < items) {
+            int k;
+            const int l = (int)div32(i, nact, k);
+            u_pre[q] = __ldg(a.spiral + (long long)(v0 + act_v[k]) * L + l);
+        }
+    }
+
+    pdl_wait();  // the tile counts come from the count pass
+    pdl_trigger();
+    int before;
+    if (a.prescanned) {
+        before = a.tile_counts[tb];
+    } else {
+        int acc = 0;
+        for (int t = tid; t < tb; t += kMapThreads) acc += a.tile_counts[t];
+        before = block_sum(acc, red);
+    }
+    const int off = before + part;  // rows before frame b
+    if (tid == 0 && s == 0) {
+        if (a.offsets) a.offsets[b] = off;
+        if (b == a.B - 1) {
+            *a.count = off + fc;
+            if (a.offsets) a.offsets[a.B] = off + fc;
+        }
+    }
+    const long long n0 = (long long)off + R0;  // first row of the portion
+    unsigned err = 0;
+    for (int i = tid; i < items; i += kMapThreads) {
+        int k;
+        const int l = (int)div32(i, nact, k);
+        const int q = (i - tid) / kMapThreads;
+        int u = -1;
+#pragma unroll
+        for (int j = 0; j < kMapPre; ++j)
+            if (q == j) u = u_pre[j];
+        if (q >= kMapPre) u = __ldg(a.spiral + (long long)(v0 + act_v[k]) * L + l);
+        int e = -1;
+        if (u < -1 || u >= V) {
+            err |= kErrIndex;
+        } else if (u >= 0) {
+            bool hit;
+            const int r = rank_of(u, hit);
+            if (hit) e = a.x_layout == HC_LAYOUT_DENSE ? (int)(fb + u) : off + r;
+        }
+        a.rulebook[(long long)l * a.n + n0 + k] = e;
+    }
+    if (a.row_of)
+        for (int p = v0 + tid; p < v1; p += kMapThreads) {
+            const int r = rank_of(p, on);
+            a.row_of[fb + p] = on ? off + r : -1;
+        }
+    for (int k = tid; k < nact; k += kMapThreads) {
+        a.coords[2 * (n0 + k)] = b;
+        a.coords[2 * (n0 + k) + 1] = v0 + act_v[k];
+    }
+    if (err) report(a.status, err);
+}
+
 __global__ void compact_empty_kernel(int B, int32_t* offsets, int32_t* count) {
     pdl_wait();
     pdl_trigger();
@@ -235,6 +435,55 @@ __global__ void compact_empty_kernel(int B, int32_t* offsets, int32_t* count) {
 }
 
 }  // namespace
+
+bool compact_map_supported(int B, int V, int L) {
+    return B >= 1 && V >= 1 && V <= kMapMaxV && L >= 1 && L <= kMapMaxL &&
+           map_smem_bytes(V / 16 + 2) <= 48 * 1024;
+}
+
+// Count pass (and the tile pre-scan when there are many tiles), then the
+// fused write + mapping pass.
+hc_status launch_compact_map(const DeviceCtx* ctx, const uint8_t* mask, int B, int V,
+                             const int32_t* spiral, int L, int x_layout, int32_t* coords,
+                             int32_t* row_of, int32_t* offsets, int32_t* count, int32_t* rulebook,
+                             cudaStream_t s) {
+    const long long n = (long long)B * V;
+    const int num_tiles = (int)((n + kTile - 1) / kTile);
+    int32_t* tile_counts = (int32_t*)stream_workspace(s, sizeof(int32_t) * (size_t)num_tiles);
+    if (!tile_counts) return HC_ERR_CUDA;
+    hc_status st = launch_pdl(compact_count_kernel, dim3(num_tiles), dim3(kThreads), 0, s,
+                              "compact_count_kernel", mask, n, tile_counts);
+    if (st != HC_OK) return st;
+    const int prescanned = num_tiles > kMaxDirectTiles;
+    if (prescanned) {
+        st = launch_pdl(compact_scan_kernel, dim3(1), dim3(1024), 0, s, "compact_scan_kernel",
+                        tile_counts, num_tiles);
+        if (st != HC_OK) return st;
+    }
+    const int nch = V / 16 + 2;  // 16-byte chunks covering a frame, any alignment
+    const size_t smem = map_smem_bytes(nch);
+    MapArgs a{};
+    a.nch = nch;
+    a.mask = mask;
+    a.n = n;
+    a.B = B;
+    a.V = V;
+    a.L = L;
+    a.x_layout = x_layout;
+    a.S = (V + kMapPortion - 1) / kMapPortion;
+    a.spiral = spiral;
+    a.tile_counts = tile_counts;
+    a.num_tiles = num_tiles;
+    a.prescanned = prescanned;
+    a.coords = coords;
+    a.row_of = row_of;
+    a.offsets = offsets;
+    a.count = count;
+    a.rulebook = rulebook;
+    a.status = ctx->status;
+    return launch_pdl(compact_map_kernel, dim3((unsigned)((long long)B * a.S)), dim3(kMapThreads),
+                      smem, s, "compact_map_kernel", a);
+}
 
 hc_status launch_compact(const DeviceCtx* ctx, const uint8_t* mask, int B, int V, int32_t* coords,
                          int32_t* row_of, int32_t* offsets, int32_t* count, cudaStream_t s) {

@@ -292,6 +292,35 @@ hc_status hc_conv_rulebook(const int32_t* coords, const int32_t* row_of, const i
                            (cudaStream_t)stream);
 }
 
+hc_status hc_mask_compact_rulebook(const uint8_t* mask, int B, int V, const int32_t* spiral, int L,
+                                   hc_layout x_layout, int32_t* coords, int32_t* row_of,
+                                   int32_t* batch_offsets, int32_t* count, int32_t* rulebook,
+                                   hc_stream_t stream) {
+    const char* fn = "hc_mask_compact_rulebook";
+    t_last_error[0] = 0;
+    HC_REQUIRE(B >= 0 && V >= 0, "%s: B=%d V=%d must be >= 0", fn, B, V);
+    HC_REQUIRE((long long)B * V < (1ll << 31), "%s: B*V must be < 2^31", fn);
+    HC_REQUIRE(L >= 1, "%s: L=%d must be >= 1", fn, L);
+    if (L > HC_MAX_SPIRAL) {
+        set_error("%s: L=%d exceeds HC_MAX_SPIRAL=%d", fn, L, HC_MAX_SPIRAL);
+        return HC_ERR_UNSUPPORTED;
+    }
+    HC_REQUIRE(x_layout == HC_LAYOUT_DENSE || x_layout == HC_LAYOUT_COMPACT,
+               "%s: unknown layout %d", fn, (int)x_layout);
+    HC_REQUIRE(count != nullptr, "%s: count is NULL", fn);
+    HC_REQUIRE((long long)B * V == 0 || (mask && spiral && coords && row_of && rulebook),
+               "%s: mask, spiral, coords, row_of and rulebook are required", fn);
+    const DeviceCtx* ctx = device_ctx();
+    if (!ctx) return HC_ERR_CUDA;
+    const cudaStream_t s = (cudaStream_t)stream;
+    if ((long long)B * V > 0 && compact_map_supported(B, V, L))
+        return launch_compact_map(ctx, mask, B, V, spiral, L, (int)x_layout, coords, row_of,
+                                  batch_offsets, count, rulebook, s);
+    hc_status st = launch_compact(ctx, mask, B, V, coords, row_of, batch_offsets, count, s);
+    if (st != HC_OK || (long long)B * V == 0) return st;
+    return launch_rulebook(ctx, coords, row_of, count, spiral, B, V, L, (int)x_layout, rulebook, s);
+}
+
 hc_status hc_sparse_conv_rulebook_fwd(const void* x, hc_dtype dt, int x_rows,
                                       const int32_t* rulebook, const int32_t* count, int capacity,
                                       int L, int C_in, int C_out, const void* W, const float* bias,

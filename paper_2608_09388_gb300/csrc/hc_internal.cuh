@@ -92,6 +92,12 @@ hc_status launch_conv_simt(const DeviceCtx* ctx, const ConvArgs& a, hc_dtype dt,
 hc_status launch_conv_tc(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s);
 bool conv_tc_supported(const ConvArgs& a, hc_dtype dt);
 int conv_tc_tile_n(const ConvArgs& a);  // output channels per tensor-core tile
+// Compaction fused with the Eq. 4 mapping (frames of at most 65535 vertices).
+bool compact_map_supported(int B, int V, int L);
+hc_status launch_compact_map(const DeviceCtx* ctx, const uint8_t* mask, int B, int V,
+                             const int32_t* spiral, int L, int x_layout, int32_t* coords,
+                             int32_t* row_of, int32_t* offsets, int32_t* count, int32_t* rulebook,
+                             cudaStream_t s);
 hc_status launch_rulebook(const DeviceCtx* ctx, const int32_t* coords, const int32_t* row_of,
                           const int32_t* count, const int32_t* spiral, int B, int V, int L,
                           int x_layout, int32_t* rulebook, cudaStream_t s);

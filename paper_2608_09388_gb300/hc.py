@@ -29,7 +29,7 @@ STATUS_NAMES = {0: "HC_OK", 1: "HC_ERR_INVALID_ARG", 2: "HC_ERR_UNSUPPORTED",
 
 # Exported symbols, as declared in include/hc.h.
 EXPORTS = ("hc_mask_compact", "hc_mask_compact_static", "hc_sparse_spiral_conv_fwd",
-           "hc_conv_rulebook", "hc_sparse_conv_rulebook_fwd", "hc_sparse_linear_fwd",
+           "hc_conv_rulebook", "hc_mask_compact_rulebook", "hc_sparse_conv_rulebook_fwd", "hc_sparse_linear_fwd",
            "hc_sparse_group_norm_fwd", "hc_sparse_conv_gn_fwd", "hc_mask_score_update", "hc_mask_select_topk",
            "hc_kappa_masks", "hc_gather_rows", "hc_conv_rulebook_transpose",
            "hc_sparse_conv_rulebook_bwd", "hc_scatter_dense", "hc_spiral_conv_fwd", "hc_get_device_status",
@@ -62,6 +62,7 @@ def load_library(path: str | None = None):
             "hc_mask_compact_static": [P, I, I, P, P, P, P, P],
             "hc_sparse_spiral_conv_fwd": [P, I, I, P, P, P, P, I, I, I, I, I, P, P, I, P, P],
             "hc_conv_rulebook": [P, P, P, P, I, I, I, I, P, P],
+            "hc_mask_compact_rulebook": [P, I, I, P, I, I, P, P, P, P, P, P],
             "hc_sparse_conv_rulebook_fwd": [P, I, I, P, P, I, I, I, I, P, P, I, P, P, I, I, P,
                                             P],
             "hc_sparse_linear_fwd": [P, I, P, I, I, I, P, P, I, P, P],
@@ -157,6 +158,17 @@ def hc_conv_rulebook(coords, row_of, count, spiral, B, V, x_layout, rulebook, st
     _check(load_library().hc_conv_rulebook(_p(coords), _p(row_of), _p(count), _p(spiral), B, V, L,
                                            x_layout, _p(rulebook), _s(stream)),
            "hc_conv_rulebook")
+
+
+def hc_mask_compact_rulebook(mask, spiral, x_layout, coords, row_of, batch_offsets, count,
+                             rulebook, stream=None):
+    """hc_mask_compact then hc_conv_rulebook in one call (fused kernels where
+    the frame fits): mask uint8 [B, V], spiral int32 [V, L]."""
+    B, V = mask.shape
+    L = spiral.shape[1]
+    _check(load_library().hc_mask_compact_rulebook(
+        _p(mask), B, V, _p(spiral), L, x_layout, _p(coords), _p(row_of), _p(batch_offsets),
+        _p(count), _p(rulebook), _s(stream)), "hc_mask_compact_rulebook")
 
 
 def hc_sparse_conv_rulebook_fwd(x, rulebook, count, W, bias, act, y, coords=None, out=None,

@@ -113,3 +113,18 @@ def test_conv_gn_arguments_rejected_on_host(lib):
     assert call(L=10 ** 4) == hc.HC_ERR_UNSUPPORTED
     # nothing to do: returns before any device call
     assert call(capacity=0) == hc.HC_OK
+
+
+def test_compact_rulebook_arguments_rejected_on_host(lib):
+    fake = ctypes.c_void_p(0x1000)
+    f = lib.hc_mask_compact_rulebook
+
+    def call(mask=fake, B=2, V=100, spiral=fake, L=9, layout=0, coords=fake, row_of=fake,
+             count=fake, rb=fake):
+        return f(mask, B, V, spiral, L, layout, coords, row_of, None, count, rb, None)
+
+    for kw in (dict(B=-1), dict(V=-3), dict(L=0), dict(layout=5), dict(count=None),
+               dict(mask=None), dict(spiral=None), dict(coords=None), dict(row_of=None),
+               dict(rb=None), dict(B=1 << 16, V=1 << 15)):
+        assert call(**kw) == hc.HC_ERR_INVALID_ARG, kw
+    assert call(L=33) == hc.HC_ERR_UNSUPPORTED
