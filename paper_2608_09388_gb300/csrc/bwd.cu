@@ -7,7 +7,8 @@
 //   dx[j][c]  = sum over taps (n, l) reading j of (dz[n] W_l^T)[c]
 // Kernels (every sum in a fixed order, no floating-point atomics):
 //   act_bwd_kernel      dz (stored in the layer dtype) and per-block column
-//                       sums of dz in fp32; dbias_kernel adds the blocks.
+//                       sums of dz in fp32 (act_bwd_vec_kernel: 16-byte
+//                       chunks); dbias_kernel adds the blocks.
 //   wgrad (tcgen05)     split-K [L*C_in] x [C_out] tiles: A = the gathered
 //                       input rows (cp.async through the rulebook), B = dz,
 //                       both MN-major, fp32 accumulators in TMEM; fp32 on
@@ -16,8 +17,9 @@
 //                       materialised once), then every input row sums the P
 //                       slices of the taps that read it, in (n, l) order,
 //                       from the transposed mapping (rb_* kernels: counts,
-//                       exclusive scan, fill, per-row sort), a warp per 32
-//                       rows where the channel chunks allow it.
+//                       exclusive scan, fill, per-row sort): a block per
+//                       range of rows, their keys staged in shared memory,
+//                       where rows are whole 16-byte chunks.
 #include <cuda_bf16.h>
 
 #include "hc_internal.cuh"
