@@ -492,14 +492,17 @@ def time_torch_dense(torch, sets, w, Wt, bias, stream, dev):
 
 
 def measure_e2e(torch, hc, sets, w, spiral, Wt, bias, stream, dev, steps):
-    """Same metric through the C-ABI with host buffers: every step copies its
-    mask and features from pinned host memory, runs the hot path, and reads
-    back the count, the coordinates and the compact output rows. Steps are
-    pipelined over two buffer sets, as a serving loop would run them: the
-    host-to-device copy of step i+1 (on its own stream) overlaps the compute
-    of step i and the read-back of step i-1 (on a third stream). Every step
-    still moves all of its inputs and results; the host learns each step's
-    row count before reading its rows."""
+    """Same metric through the C-ABI with host inputs: every step copies its
+    mask from pinned host memory, compacts it and builds the Eq. 4 mapping
+    (compact layout), gathers the active rows of its dense features straight
+    from the pinned host buffer (hc_gather_rows reading host memory: only the
+    active rows cross the host link), runs the conv on those compact rows
+    (with the fused scatter), and reads back the count, the coordinates and
+    the compact output rows. Steps are pipelined over two buffer sets, as a
+    serving loop would run them: the mask copy of step i+1 (on its own
+    stream) overlaps the compute of step i and the read-back of step i-1 (on
+    a third stream). Every step moves the inputs it uses and all of its
+    results; the host learns each step's row count before reading its rows."""
     ly = w.layers[0]
     B, V = w.B, w.V
     host = []
@@ -507,7 +510,6 @@ def measure_e2e(torch, hc, sets, w, spiral, Wt, bias, stream, dev, steps):
         host.append((s.mask.cpu().pin_memory(), s.x.cpu().pin_memory()))
     nb = 2
     mask_d = [torch.empty_like(sets[0].mask) for _ in range(nb)]
-    x_d = [torch.empty_like(sets[0].x) for _ in range(nb)]
     outs = []  # device outputs of buffer b (the input sets' own buffers stay as they are)
     for _ in range(nb):
         o = LayerSet()
@@ -516,6 +518,7 @@ def measure_e2e(torch, hc, sets, w, spiral, Wt, bias, stream, dev, steps):
         o.offs = torch.empty((B + 1,), dtype=torch.int32, device=dev)
         o.count = torch.empty((1,), dtype=torch.int32, device=dev)
         o.rb = torch.empty((w.L, B * V), dtype=torch.int32, device=dev)
+        o.xc = torch.empty((B * V, ly.C_in), dtype=torch.bfloat16, device=dev)
         o.y = torch.empty((B * V, ly.C_out), dtype=torch.bfloat16, device=dev)
         o.out = torch.zeros((B, V, ly.C_out), dtype=torch.bfloat16, device=dev)
         outs.append(o)
@@ -541,19 +544,19 @@ def measure_e2e(torch, hc, sets, w, spiral, Wt, bias, stream, dev, steps):
             copy_s.wait_event(computed[b])  # step i - 2 no longer reads buffer b
         with torch.cuda.stream(copy_s):
             mask_d[b].copy_(mh, non_blocking=True)
-            x_d[b].copy_(xh, non_blocking=True)
             copied[b].record(copy_s)
         stream.wait_event(copied[b])
         if i >= nb:
             stream.wait_event(drained[b])  # step i - 2's rows have been read back
         with torch.cuda.stream(stream):
-            hc.hc_mask_compact_rulebook(mask_d[b], spiral, hc.HC_LAYOUT_DENSE, o.coords,
+            hc.hc_mask_compact_rulebook(mask_d[b], spiral, hc.HC_LAYOUT_COMPACT, o.coords,
                                         o.row_of, o.offs, o.count, o.rb, stream)
-            hc.hc_sparse_conv_rulebook_fwd(x_d[b], o.rb, o.count, Wt, bias, ly.act, o.y,
+            hc.hc_gather_rows(xh, o.coords, o.count, 1, o.xc, stream)  # rows from host memory
+            hc.hc_sparse_conv_rulebook_fwd(o.xc, o.rb, o.count, Wt, bias, ly.act, o.y,
                                            coords=o.coords, out=o.out, stream=stream)
             cnt_h[b].copy_(o.count, non_blocking=True)
             computed[b].record(stream)
-        acc["h2d"] += mh.numel() + xh.numel() * 2
+        acc["h2d"] += mh.numel()
 
     def read_back(i):
         b = i % nb
@@ -565,6 +568,7 @@ def measure_e2e(torch, hc, sets, w, spiral, Wt, bias, stream, dev, steps):
             y_h[b][:n].copy_(o.y[:n], non_blocking=True)
             c_h[b][:n].copy_(o.coords[:n], non_blocking=True)
             drained[b].record(back_s)
+        acc["h2d"] += n * ly.C_in * 2  # the active feature rows read from host memory
         acc["d2h"] += 4 + n * 8 + n * ly.C_out * 2
         acc["rows"] += n
 
@@ -586,8 +590,10 @@ def measure_e2e(torch, hc, sets, w, spiral, Wt, bias, stream, dev, steps):
     return {"value": acc["rows"] / dt, "unit": "rows/s", "steps": steps,
             "h2d_bytes_per_step": acc["h2d"] // steps, "d2h_bytes_per_step": acc["d2h"] // steps,
             "ms_per_step": dt / steps * 1e3,
-            "path": "pinned host mask + features -> C-ABI calls -> count, coords, rows to host; "
-                    "two buffer sets, the copy of step i+1 overlapping step i"}
+            "path": "pinned host mask (copied) + pinned host features (active rows gathered "
+                    "by hc_gather_rows over the host link) -> hc_mask_compact_rulebook, "
+                    "hc_gather_rows, hc_sparse_conv_rulebook_fwd -> count, coords, rows to "
+                    "host; two buffer sets, step i+1's mask copy overlapping step i"}
 
 
 def run_sweep(torch, hc, dev, stream):

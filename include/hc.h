@@ -376,7 +376,11 @@ hc_status hc_kappa_masks(const uint8_t* masks, int K, int V, const int32_t* sele
  * after hc_kappa_masks, else 1). Rows are copied bit for bit; y is
  * [capacity, C]. A coordinate outside the input is reported
  * (HC_ERR_INVALID_INDEX) and its row left untouched; *count above capacity
- * is clamped (HC_ERR_CAPACITY).
+ * is clamped (HC_ERR_CAPACITY). x may be pinned host memory (cudaHostAlloc,
+ * the same pointer on the device under unified addressing): the kernel then
+ * reads only the active rows across the host link (zero-copy), which is how
+ * a dense host-side input becomes compact device rows without copying the
+ * whole tensor.
  */
 hc_status hc_gather_rows(const void* x, hc_dtype dt, int B_in, int V, int C, const int32_t* coords,
                          const int32_t* count, int capacity, int frames_per_sample, void* y,

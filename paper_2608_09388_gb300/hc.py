@@ -100,6 +100,16 @@ def _p(t):
     return ctypes.c_void_p(t.data_ptr())
 
 
+def _p_host_ok(t):
+    """A device tensor, or a pinned host tensor (read by the kernel over the
+    host link under unified addressing)."""
+    if t is not None and not t.is_cuda and t.is_pinned():
+        if not t.is_contiguous():
+            raise ValueError("libhc takes contiguous tensors")
+        return ctypes.c_void_p(t.data_ptr())
+    return _p(t)
+
+
 def _s(stream):
     import torch
     if stream is None:
@@ -268,9 +278,10 @@ def hc_kappa_masks(masks, selected, B, out, stream=None):
 
 
 def hc_gather_rows(x, coords, count, frames_per_sample, y, stream=None):
-    """S' of Eq. 2: y[n] = x[f // frames_per_sample, v] for coords[n] = (f, v)."""
+    """S' of Eq. 2: y[n] = x[f // frames_per_sample, v] for coords[n] = (f, v).
+    x may be a pinned host tensor: only the active rows cross the host link."""
     B_in, V, C = x.shape
-    _check(load_library().hc_gather_rows(_p(x), _dt(x), B_in, V, C, _p(coords), _p(count),
+    _check(load_library().hc_gather_rows(_p_host_ok(x), _dt(x), B_in, V, C, _p(coords), _p(count),
                                          y.shape[0], frames_per_sample, _p(y), _s(stream)),
            "hc_gather_rows")
 

@@ -162,6 +162,28 @@ def test_gather_rows(C, fps, dtype):
     assert not to_numpy(y)[0].any()
 
 
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_gather_rows_from_pinned_host_memory(dtype):
+    """x in pinned host memory (read over the host link): the same rows, bit
+    for bit, as from device memory."""
+    rng = np.random.default_rng(17)
+    B, V, C = 4, 2000, 64
+    masks = inputs.uniform_mask(rng, B, V, 0.05)
+    x = inputs.features(rng, (B, V, C), dtype)
+    c_ref, _, _, n = oracle.mask_compact(masks)
+    coords = torch.full((B * V, 2), -1, dtype=torch.int32, device="cuda")
+    coords[:n] = to_torch(c_ref)
+    count = torch.tensor([n], dtype=torch.int32, device="cuda")
+    xt = to_torch(x)
+    xh = xt.cpu().pin_memory()
+    y = torch.zeros((B * V, C), dtype=xt.dtype, device="cuda")
+    hc.hc_gather_rows(xh, coords, count, 1, y)
+    assert hc.hc_get_device_status() == hc.HC_OK
+    np.testing.assert_array_equal(to_numpy(y)[:n], oracle.gather_rows(x, c_ref, 1))
+    with pytest.raises(ValueError):  # pageable host memory is refused by the binding
+        hc.hc_gather_rows(xt.cpu(), coords, count, 1, y)
+
+
 def test_kappa_inference_chain():
     """alpha -> top-3 -> kappa masks for every sample -> compaction -> S'
     -> sparse spiral conv on the compact rows, against the same chain on
