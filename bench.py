@@ -498,11 +498,12 @@ def measure_e2e(torch, hc, sets, w, spiral, Wt, bias, stream, dev, steps):
     from the pinned host buffer (hc_gather_rows reading host memory: only the
     active rows cross the host link), runs the conv on those compact rows
     (with the fused scatter), and reads back the count, the coordinates and
-    the compact output rows. Steps are pipelined over two buffer sets, as a
-    serving loop would run them: the mask copy of step i+1 (on its own
-    stream) overlaps the compute of step i and the read-back of step i-1 (on
-    a third stream). Every step moves the inputs it uses and all of its
-    results; the host learns each step's row count before reading its rows."""
+    the compact output rows. A step's device work (mask copy, the three
+    library calls, the count's read-back) is one CUDA graph per input set.
+    Steps are pipelined over two buffer sets, as a serving loop would run
+    them: the rows' read-back of step i-1 (on a second stream) overlaps step
+    i. Every step moves the inputs it uses and all of its results; the host
+    learns each step's row count before reading its rows."""
     ly = w.layers[0]
     B, V = w.B, w.V
     host = []
@@ -525,38 +526,50 @@ def measure_e2e(torch, hc, sets, w, spiral, Wt, bias, stream, dev, steps):
     cnt_h = [torch.empty((1,), dtype=torch.int32).pin_memory() for _ in range(nb)]
     y_h = [torch.empty((B * V, ly.C_out), dtype=torch.bfloat16).pin_memory() for _ in range(nb)]
     c_h = [torch.empty((B * V, 2), dtype=torch.int32).pin_memory() for _ in range(nb)]
-    copy_s = torch.cuda.Stream(device=dev)
     back_s = torch.cuda.Stream(device=dev)
 
     def event():
         return torch.cuda.Event()
 
-    copied = [event() for _ in range(nb)]
     computed = [event() for _ in range(nb)]
     drained = [event() for _ in range(nb)]
     acc = {"h2d": 0, "d2h": 0, "rows": 0}
 
+    def device_part(j):
+        b = j % nb
+        mh, xh = host[j]
+        o = outs[b]
+        mask_d[b].copy_(mh, non_blocking=True)
+        hc.hc_mask_compact_rulebook(mask_d[b], spiral, hc.HC_LAYOUT_COMPACT, o.coords,
+                                    o.row_of, o.offs, o.count, o.rb, stream)
+        hc.hc_gather_rows(xh, o.coords, o.count, 1, o.xc, stream)  # rows from host memory
+        hc.hc_sparse_conv_rulebook_fwd(o.xc, o.rb, o.count, Wt, bias, ly.act, o.y,
+                                       coords=o.coords, out=o.out, stream=stream)
+        cnt_h[b].copy_(o.count, non_blocking=True)
+
+    # one CUDA graph per input set (set j always uses buffer j % nb): the mask
+    # copy, the three library calls and the count's read-back
+    assert len(host) % nb == 0
+    with torch.cuda.stream(stream):
+        for j in range(len(host)):
+            device_part(j)
+    torch.cuda.synchronize(dev)
+    graphs = []
+    for j in range(len(host)):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            device_part(j)
+        graphs.append(g)
+
     def launch(i):
         b = i % nb
-        mh, xh = host[i % len(host)]
-        o = outs[b]
-        if i >= nb:
-            copy_s.wait_event(computed[b])  # step i - 2 no longer reads buffer b
-        with torch.cuda.stream(copy_s):
-            mask_d[b].copy_(mh, non_blocking=True)
-            copied[b].record(copy_s)
-        stream.wait_event(copied[b])
+        j = i % len(host)
         if i >= nb:
             stream.wait_event(drained[b])  # step i - 2's rows have been read back
         with torch.cuda.stream(stream):
-            hc.hc_mask_compact_rulebook(mask_d[b], spiral, hc.HC_LAYOUT_COMPACT, o.coords,
-                                        o.row_of, o.offs, o.count, o.rb, stream)
-            hc.hc_gather_rows(xh, o.coords, o.count, 1, o.xc, stream)  # rows from host memory
-            hc.hc_sparse_conv_rulebook_fwd(o.xc, o.rb, o.count, Wt, bias, ly.act, o.y,
-                                           coords=o.coords, out=o.out, stream=stream)
-            cnt_h[b].copy_(o.count, non_blocking=True)
+            graphs[j].replay()
             computed[b].record(stream)
-        acc["h2d"] += mh.numel()
+        acc["h2d"] += host[j][0].numel()
 
     def read_back(i):
         b = i % nb
@@ -587,13 +600,23 @@ def measure_e2e(torch, hc, sets, w, spiral, Wt, bias, stream, dev, steps):
     t0 = time.perf_counter()
     run(steps)
     dt = time.perf_counter() - t0
+    # the last step's rows as read back, against the same input set's rows
+    # from the device-resident step timed above (dense layout, same kernels)
+    last, b = steps - 1, (steps - 1) % nb
+    s_ref = sets[last % len(host)]
+    n = int(cnt_h[b][0])
+    same = (n == s_ref.rows and
+            torch.equal(y_h[b][:n], s_ref.y[:n].cpu()) and
+            torch.equal(c_h[b][:n], s_ref.coords[:n].cpu()))
     return {"value": acc["rows"] / dt, "unit": "rows/s", "steps": steps,
+            "rows_match_device_step": bool(same),
             "h2d_bytes_per_step": acc["h2d"] // steps, "d2h_bytes_per_step": acc["d2h"] // steps,
             "ms_per_step": dt / steps * 1e3,
             "path": "pinned host mask (copied) + pinned host features (active rows gathered "
                     "by hc_gather_rows over the host link) -> hc_mask_compact_rulebook, "
                     "hc_gather_rows, hc_sparse_conv_rulebook_fwd -> count, coords, rows to "
-                    "host; two buffer sets, step i+1's mask copy overlapping step i"}
+                    "host; one CUDA graph per step's device work, two buffer sets, step i-1's "
+                    "read-back overlapping step i"}
 
 
 def run_sweep(torch, hc, dev, stream):
