@@ -128,3 +128,30 @@ def test_compact_rulebook_arguments_rejected_on_host(lib):
                dict(rb=None), dict(B=1 << 16, V=1 << 15)):
         assert call(**kw) == hc.HC_ERR_INVALID_ARG, kw
     assert call(L=33) == hc.HC_ERR_UNSUPPORTED
+
+
+def test_gather_rows_arguments_rejected_on_host(lib):
+    fake = ctypes.c_void_p(0x1000)
+    g = lib.hc_gather_rows
+
+    def call(x=fake, dt=1, B_in=2, V=100, C=64, coords=fake, count=fake, cap=200, fps=1, y=fake):
+        return g(x, dt, B_in, V, C, coords, count, cap, fps, y, None)
+
+    for kw in (dict(dt=9), dict(B_in=-1), dict(C=0), dict(fps=0), dict(cap=-1), dict(count=None),
+               dict(x=None), dict(coords=None), dict(y=None), dict(x=ctypes.c_void_p(0x1001))):
+        assert call(**kw) == hc.HC_ERR_INVALID_ARG, kw
+    assert call(cap=0) == hc.HC_OK  # nothing to gather: no device call
+
+
+def test_binding_refuses_pageable_host_tensors(lib):
+    """Host memory is accepted only pinned, and only as hc_gather_rows' input;
+    a pageable tensor is refused before any library call."""
+    torch = pytest.importorskip("torch")
+    x = torch.zeros((2, 10, 8), dtype=torch.float32)
+    coords = torch.zeros((20, 2), dtype=torch.int32)
+    count = torch.zeros((1,), dtype=torch.int32)
+    y = torch.zeros((20, 8), dtype=torch.float32)
+    with pytest.raises(ValueError):
+        hc.hc_gather_rows(x, coords, count, 1, y)
+    with pytest.raises(ValueError):
+        hc.hc_sparse_linear_fwd(y, count, torch.zeros((8, 8)), None, hc.HC_ACT_NONE, y)
