@@ -92,9 +92,9 @@ hc_status hc_mask_compact(const uint8_t* mask, int B, int V, int32_t* coords,
  * hc_mask_compact_static -- hc_mask_compact that allocates nothing. The paper
  * has no counterpart; this entry point exists for callers of this library
  * that cannot allocate device memory at the moment they compact a mask:
- * code running while a stream is being captured into a CUDA graph (a
- * cudaMalloc there breaks the capture), and processes that hand all device
- * memory to their own pool up front and must not allocate behind its back.
+ * processes that hand all device memory to their own pool up front and must
+ * not allocate behind its back, and code on a path where a cudaMalloc or
+ * cudaFree (which can synchronise the whole device) is not allowed.
  *
  * Same arguments, results and errors as hc_mask_compact (bit-identical
  * outputs). Differences:
@@ -390,10 +390,16 @@ hc_status hc_gather_rows(const void* x, hc_dtype dt, int B_in, int V, int C, con
  * hc_scatter_dense -- inverse of the decomposition (Eq. 2): compact rows back
  * into a dense [B, V, C] tensor.
  *   zero_fill == 0: out[coords[n]] = y[n] for n < N'; other rows untouched.
- *   zero_fill != 0: every row of out is written: y[row_of[b,v]] where active,
- *                   zeros elsewhere (the masked tensor of Eq. 1); needs row_of.
- *   y [N', C] of dtype dt (elements are copied bit for bit), coords/row_of/
- *   count as written by hc_mask_compact, out [B, V, C].
+ *   zero_fill != 0: every row of out is written: y[n] at coords[n], zeros
+ *                   elsewhere (the masked tensor of Eq. 1).
+ *   y [N', C] of dtype dt (elements are copied bit for bit), coords/count as
+ *   written by hc_mask_compact, out [B, V, C].
+ *   row_of   [B, V] as written by hc_mask_compact, or NULL. Optional: with
+ *            zero_fill it lets one pass write every dense row exactly once
+ *            (coords may then be NULL); without it the zero fill is a
+ *            separate pass over out before the scatter. Ignored when
+ *            zero_fill == 0. (The problem statement's call has no row_of;
+ *            passing NULL gives exactly that call.)
  */
 hc_status hc_scatter_dense(const void* y, hc_dtype dt, const int32_t* coords,
                            const int32_t* row_of, const int32_t* count, int B, int V, int C,
@@ -418,6 +424,26 @@ hc_status hc_spiral_conv_fwd(const void* x, hc_dtype dt, const int32_t* spiral, 
  * if the synchronisation itself failed.
  */
 hc_status hc_get_device_status(hc_stream_t stream);
+
+/*
+ * hc_test_set_option -- hooks for this library's own tests; the paper has no
+ * counterpart and the operators never need them. They reach code paths that
+ * ordinary inputs do not select. Settings stay until changed.
+ *   HC_TEST_GROUP_NORM_PATH (process-wide): 0 = the library's own choice
+ *       (default); 1 = always the per-(frame, group) kernel; 2 = the
+ *       row-range kernels wherever the layout allows them.
+ *   HC_TEST_WAIT_LIMIT_NS (current device): how long the pipelined kernels
+ *       (tensor-core conv, mask score, weight gradient) wait on any one
+ *       pipeline barrier before they give up, report HC_ERR_TIMEOUT and
+ *       unwind. value > 0 sets it in nanoseconds; 0 restores the default
+ *       (2 s). The unwind's own waits, for copies and MMAs already issued,
+ *       always keep the default. A lowered limit makes ordinary calls fail
+ *       with HC_ERR_TIMEOUT and unspecified outputs: it exists to test that
+ *       path. Synchronous (a small host-to-device copy).
+ * Returns HC_ERR_INVALID_ARG for an unknown option or a value out of range.
+ */
+typedef enum { HC_TEST_GROUP_NORM_PATH = 1, HC_TEST_WAIT_LIMIT_NS = 2 } hc_test_option;
+hc_status hc_test_set_option(int option, long long value);
 
 /* Text of the last host-side error on the calling thread ("" if none). */
 const char* hc_last_error_string(void);

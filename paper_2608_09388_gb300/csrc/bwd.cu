@@ -622,8 +622,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) wgrad_tc_kernel(const WgradArgs
             }
             if (ok && num_kb > 0) tc_commit(tfull_bar);
             tc_commit(fin_bar);
-            int no_abort = 0;
-            mbar_wait(fin_bar, 0, &no_abort, a.status);
+            mbar_wait_drain(fin_bar, 0, a.status);
             if (ok && num_kb == 0) mbar_arrive(tfull_bar);  // empty split: zeros
         }
         __syncwarp();

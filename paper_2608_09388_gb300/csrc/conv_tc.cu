@@ -495,10 +495,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             cp_async_wait_all();
             if (!ok && t == 0) {
                 // Let the weight copies already issued land before the CTA exits.
-                int no_abort = 0;
                 for (long long j = it > nst ? it - nst : 0; j < it; ++j)
-                    mbar_wait(full_bar((int)(j % nst)), (uint32_t)((j / nst) & 1),
-                              &no_abort, a.status);
+                    mbar_wait_drain(full_bar((int)(j % nst)), (uint32_t)((j / nst) & 1),
+                                    a.status);
             }
         } else {
             const __nv_bfloat16* __restrict__ x = static_cast<const __nv_bfloat16*>(a.x);
@@ -633,8 +632,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             // Every MMA issued by this thread has completed once fin_bar fires.
             tc_commit(fin_bar);
-            int no_abort = 0;
-            mbar_wait(fin_bar, 0, &no_abort, a.status);
+            mbar_wait_drain(fin_bar, 0, a.status);
         }
         __syncwarp();
     } else if (warp == kIndexWarp) {

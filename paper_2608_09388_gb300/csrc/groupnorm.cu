@@ -765,10 +765,11 @@ hc_status launch_typed(const DeviceCtx* ctx, const void* x, const int32_t* offse
     const bool small_frames = cpg % kVec == 0 && aligned &&
                               avg_chunks <= 2ll * kThreads * kBatch &&
                               (long long)B * G >= ctx->num_sms;
-    // HC_GN_SLICE forces the per-(frame, group) kernel, HC_GN_ROWS the
-    // row-range kernels where the layout allows (to test both on any shape)
-    const bool force_slice = getenv("HC_GN_SLICE") != nullptr;
-    const bool force_rows = getenv("HC_GN_ROWS") != nullptr;
+    // a test may force the per-(frame, group) kernel (1) or the row-range
+    // kernels where the layout allows (2), to cover both on any shape
+    const int forced = test_group_norm_path();
+    const bool force_slice = forced == 1;
+    const bool force_rows = forced == 2;
     const bool fast_rows = aligned && cpr >= 1 && cpr <= kThreads && (cpr & (cpr - 1)) == 0 &&
                            G <= kMaxGroupsFast && !force_slice && (force_rows || !small_frames);
     if (fast_rows && cpg % kVec == 0)

@@ -7,6 +7,7 @@
 #include <stdlib.h>
 #include <string.h>
 
+#include <atomic>
 #include <map>
 #include <mutex>
 #include <utility>
@@ -15,8 +16,15 @@
 
 namespace hc {
 
-// Sticky per-device status word; kernels OR kErr* bits into it.
-__device__ unsigned g_device_status;
+// Sticky per-device status word (kernels OR kErr* bits into it) and the
+// pipeline-wait limit the kernels read beside it.
+__device__ DeviceWord g_device_word = {0u, 0u, kWaitLimitNs};
+
+// Group-norm path forced by a test (hc_test_set_option), 0 = automatic.
+static std::atomic<int> g_test_gn_path{0};
+int test_group_norm_path() {
+    return g_test_gn_path.load(std::memory_order_relaxed);
+}
 
 static thread_local char t_last_error[512];
 
@@ -53,9 +61,9 @@ const DeviceCtx* device_ctx() {
                        "cudaDeviceGetAttribute") != HC_OK)
             return nullptr;
         void* p = nullptr;
-        if (check_cuda(cudaGetSymbolAddress(&p, g_device_status), "cudaGetSymbolAddress") != HC_OK)
+        if (check_cuda(cudaGetSymbolAddress(&p, g_device_word), "cudaGetSymbolAddress") != HC_OK)
             return nullptr;
-        c.status = (unsigned*)p;
+        c.status = &static_cast<DeviceWord*>(p)->status;
         g_ctx[dev] = c;
         g_ctx_ready[dev] = true;
     }
@@ -95,19 +103,10 @@ static bool misaligned(const void* p, size_t a) {
 }
 
 // Conv kernels: tensor cores when supported (bf16, 16-byte aligned rows),
-// CUDA cores otherwise or when HC_FORCE_SIMT=1.
-static bool use_conv_tc(const ConvArgs& a, hc_dtype dt) {
-    static int force_simt = -1;
-    if (force_simt < 0) {
-        const char* e = getenv("HC_FORCE_SIMT");
-        force_simt = (e && e[0] == '1') ? 1 : 0;
-    }
-    return !force_simt && conv_tc_supported(a, dt);
-}
-
+// CUDA cores otherwise.
 hc_status dispatch_conv(const DeviceCtx* ctx, ConvArgs& a, hc_dtype dt, cudaStream_t s) {
     a.status = ctx->status;
-    if (use_conv_tc(a, dt)) return launch_conv_tc(ctx, a, s);
+    if (conv_tc_supported(a, dt)) return launch_conv_tc(ctx, a, s);
     return launch_conv_simt(ctx, a, dt, s);
 }
 
@@ -430,7 +429,7 @@ hc_status hc_sparse_conv_gn_fwd(const void* x, hc_dtype dt, int x_rows, const in
     a.status = ctx->status;
     const int cpg = C_out / G;
     // channels per group a power of two from 8 to the tile's width
-    if (use_conv_tc(a, dt) && cpg >= 8 && (cpg & (cpg - 1)) == 0 && cpg <= conv_tc_tile_n(a) &&
+    if (conv_tc_supported(a, dt) && cpg >= 8 && (cpg & (cpg - 1)) == 0 && cpg <= conv_tc_tile_n(a) &&
         group_norm_parts_supported(dt, C_out, G, y)) {
         // statistics from the convolution's epilogue: one partial per
         // (frame, 32-row block inside it) in slot frame + block, one per row
@@ -620,8 +619,8 @@ hc_status hc_scatter_dense(const void* y, hc_dtype dt, const int32_t* coords,
     HC_REQUIRE(B >= 0 && V >= 0 && C >= 1, "%s: B=%d V=%d C=%d", fn, B, V, C);
     HC_REQUIRE((long long)B * V < (1ll << 31), "%s: B*V must be < 2^31", fn);
     HC_REQUIRE(y && count && out, "%s: y, count and out are required", fn);
-    HC_REQUIRE(zero_fill ? row_of != nullptr : coords != nullptr,
-               "%s: zero_fill needs row_of; scatter without it needs coords", fn);
+    HC_REQUIRE(coords != nullptr || (zero_fill && row_of != nullptr),
+               "%s: coords are required (zero_fill may use row_of instead)", fn);
     int eb = dt == HC_F32 ? 4 : 2;
     HC_REQUIRE(!misaligned(y, eb) && !misaligned(out, eb), "%s: misaligned y/out", fn);
     if ((long long)B * V == 0) return HC_OK;
@@ -629,6 +628,26 @@ hc_status hc_scatter_dense(const void* y, hc_dtype dt, const int32_t* coords,
     if (!ctx) return HC_ERR_CUDA;
     return launch_scatter(ctx, y, eb, coords, row_of, count, B, V, C, zero_fill, out,
                           (cudaStream_t)stream);
+}
+
+hc_status hc_test_set_option(int option, long long value) {
+    t_last_error[0] = 0;
+    if (option == HC_TEST_GROUP_NORM_PATH) {
+        HC_REQUIRE(value >= 0 && value <= 2, "hc_test_set_option: group-norm path %lld", value);
+        g_test_gn_path.store((int)value, std::memory_order_relaxed);
+        return HC_OK;
+    }
+    if (option == HC_TEST_WAIT_LIMIT_NS) {
+        HC_REQUIRE(value >= 0, "hc_test_set_option: wait limit %lld ns", value);
+        const DeviceCtx* ctx = device_ctx();
+        if (!ctx) return HC_ERR_CUDA;
+        const unsigned long long ns = value == 0 ? kWaitLimitNs : (unsigned long long)value;
+        DeviceWord* word = reinterpret_cast<DeviceWord*>(ctx->status);
+        return check_cuda(cudaMemcpy(&word->wait_limit_ns, &ns, sizeof ns, cudaMemcpyHostToDevice),
+                          "set wait limit");
+    }
+    set_error("hc_test_set_option: unknown option %d", option);
+    return HC_ERR_INVALID_ARG;
 }
 
 hc_status hc_get_device_status(hc_stream_t stream) {

@@ -20,8 +20,22 @@ enum : unsigned {
 };
 
 // Longest a kernel waits on any one barrier before it gives up, records
-// HC_ERR_TIMEOUT and unwinds (nanoseconds of %globaltimer).
+// HC_ERR_TIMEOUT and unwinds (nanoseconds of %globaltimer). A test may lower
+// the limit of the pipeline waits on a device (hc_test_set_option); the
+// waits of an unwind, for copies and MMAs already issued, always keep it.
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;
+
+// The per-device word kernels report into (`status` in every kernel's
+// arguments points at its first member), with the pipeline-wait limit
+// beside it so that kernels read it through the same pointer.
+struct DeviceWord {
+    unsigned status;                   // sticky kErr* bits
+    unsigned reserved;
+    unsigned long long wait_limit_ns;  // kWaitLimitNs unless a test lowered it
+};
+
+// Path choices that only the library's tests override (hc_test_set_option).
+int test_group_norm_path();  // 0 automatic, 1 per-(frame, group) kernel, 2 row ranges
 
 // ------------------------------------------------------------ host context
 struct DeviceCtx {
@@ -373,24 +387,39 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
         : "memory");
     return ok != 0;
 }
-// Wait for the phase with the given parity, for at most kWaitLimitNs. On
-// timeout (or when another role already gave up) it records HC_ERR_TIMEOUT,
-// raises the CTA's abort flag and returns false.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
-                                          unsigned* status) {
-    if (mbar_try_wait(bar, parity)) return true;
+// Wait for the phase with the given parity for at most `limit` ns. On
+// timeout (or, with an abort flag, when another role already gave up) it
+// records HC_ERR_TIMEOUT, raises the flag and returns false.
+__device__ __forceinline__ bool mbar_wait_for(uint32_t bar, uint32_t parity,
+                                              volatile int* abort_flag, unsigned* status,
+                                              unsigned long long limit) {
     unsigned long long t0 = globaltimer_ns();
     for (uint32_t i = 1;; ++i) {
         if (mbar_try_wait(bar, parity)) return true;
         if ((i & 63u) == 0) {
-            if (*abort_flag) return false;
-            if (globaltimer_ns() - t0 > kWaitLimitNs) {
-                *abort_flag = 1;
+            if (abort_flag && *abort_flag) return false;
+            if (globaltimer_ns() - t0 > limit) {
+                if (abort_flag) *abort_flag = 1;
                 report(status, kErrTimeout);
                 return false;
             }
         }
     }
+}
+// A pipeline wait: bounded by the device's wait limit (kWaitLimitNs unless a
+// test lowered it), abandoned when another role of the CTA gave up.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                          unsigned* status) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const unsigned long long limit =
+        reinterpret_cast<const volatile DeviceWord*>(status)->wait_limit_ns;
+    return mbar_wait_for(bar, parity, abort_flag, status, limit);
+}
+// A wait of the unwind, for copies or MMAs already issued: always the full
+// limit, regardless of the abort flag.
+__device__ __forceinline__ bool mbar_wait_drain(uint32_t bar, uint32_t parity, unsigned* status) {
+    if (mbar_try_wait(bar, parity)) return true;
+    return mbar_wait_for(bar, parity, nullptr, status, kWaitLimitNs);
 }
 
 // ---- TMA (bulk tensor copies global -> shared, completion on an mbarrier)

@@ -236,8 +236,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) gram_tc_kernel(const GramArgs a
             if (ok && num_kb > 0) tc_commit(tfull_bar);
             // every MMA issued by this thread has completed once fin_bar fires
             tc_commit(fin_bar);
-            int no_abort = 0;
-            mbar_wait(fin_bar, 0, &no_abort, a.status);
+            mbar_wait_drain(fin_bar, 0, a.status);
             if (ok && num_kb == 0) mbar_arrive(tfull_bar);  // empty split: zeros
         }
         __syncwarp();

@@ -3,8 +3,9 @@
 // (the widest the row size and pointer alignment allow), bit for bit.
 //   scatter:      out[coords[n]] = y[n]           for n < N'
 //   scatter+fill: out[r] = row_of[r] >= 0 ? y[row_of[r]] : 0   for every r
-// The fill variant writes every dense row exactly once (one pass over the
-// output instead of a memset followed by a scatter).
+// With row_of, the fill variant writes every dense row exactly once (one
+// pass over the output instead of a memset followed by a scatter); without
+// it, a zero pass over the output is followed by the scatter.
 #include "hc_internal.cuh"
 
 namespace hc {
@@ -61,6 +62,15 @@ __global__ void scatter_kernel(const U* __restrict__ y, const int32_t* __restric
 }
 
 template <typename U>
+__global__ void zero_kernel(long long total, U* __restrict__ out) {
+    pdl_wait();
+    pdl_trigger();
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
+         i += (long long)gridDim.x * blockDim.x)
+        out[i] = zero_chunk<U>();
+}
+
+template <typename U>
 __global__ void scatter_fill_kernel(const U* __restrict__ y, const int32_t* __restrict__ row_of,
                                     const int32_t* __restrict__ count, long long dense_rows,
                                     int cpr, U* __restrict__ out, unsigned* status) {
@@ -92,10 +102,16 @@ hc_status launch_typed(const DeviceCtx* ctx, const void* y, const int32_t* coord
     const long long cap = (long long)ctx->num_sms * 8;
     if (blocks > cap) blocks = cap;
     if (blocks < 1) blocks = 1;
-    if (zero_fill)
+    if (zero_fill && !row_of) {
+        // no inverse map: zero every row, then scatter the active ones
+        hc_status st = launch_pdl(zero_kernel<U>, dim3((unsigned)blocks), dim3(256), 0, s,
+                                  "zero_kernel", work, (U*)out);
+        if (st != HC_OK) return st;
+    } else if (zero_fill) {
         return launch_pdl(scatter_fill_kernel<U>, dim3((unsigned)blocks), dim3(256), 0, s,
                           "scatter_fill_kernel", (const U*)y, row_of, count, dense_rows, cpr,
                           (U*)out, ctx->status);
+    }
     return launch_pdl(scatter_kernel<U>, dim3((unsigned)blocks), dim3(256), 0, s, "scatter_kernel",
                       (const U*)y, coords, count, B, V, cpr, (U*)out, ctx->status);
 }

@@ -22,6 +22,7 @@ HC_ACT_NONE, HC_ACT_ELU, HC_ACT_RELU = 0, 1, 2
 HC_LAYOUT_DENSE, HC_LAYOUT_COMPACT = 0, 1
 HC_MAX_SPIRAL = 32
 HC_STATIC_MAX_MASK_BYTES = 4096 * 4096
+HC_TEST_GROUP_NORM_PATH, HC_TEST_WAIT_LIMIT_NS = 1, 2
 
 STATUS_NAMES = {0: "HC_OK", 1: "HC_ERR_INVALID_ARG", 2: "HC_ERR_UNSUPPORTED",
                 3: "HC_ERR_CAPACITY", 4: "HC_ERR_INVALID_INDEX", 5: "HC_ERR_TIMEOUT",
@@ -33,7 +34,7 @@ EXPORTS = ("hc_mask_compact", "hc_mask_compact_static", "hc_sparse_spiral_conv_f
            "hc_sparse_group_norm_fwd", "hc_sparse_conv_gn_fwd", "hc_mask_score_update", "hc_mask_select_topk",
            "hc_kappa_masks", "hc_gather_rows", "hc_conv_rulebook_transpose",
            "hc_sparse_conv_rulebook_bwd", "hc_scatter_dense", "hc_spiral_conv_fwd", "hc_get_device_status",
-           "hc_last_error_string", "hc_version")
+           "hc_test_set_option", "hc_last_error_string", "hc_version")
 
 
 class HcError(RuntimeError):
@@ -79,6 +80,7 @@ def load_library(path: str | None = None):
             "hc_scatter_dense": [P, I, P, P, P, I, I, I, I, P, P],
             "hc_spiral_conv_fwd": [P, I, P, I, I, I, I, I, P, P, I, P, P],
             "hc_get_device_status": [P],
+            "hc_test_set_option": [I, ctypes.c_longlong],
             "hc_last_error_string": [],
             "hc_version": [],
         }
@@ -302,6 +304,12 @@ def hc_spiral_conv_fwd(x, spiral, W, bias, act, y, stream=None):
     _check(load_library().hc_spiral_conv_fwd(
         _p(x), _dt(x), _p(spiral), B, V, L, C_in, C_out, _p(W), _p(bias), act, _p(y),
         _s(stream)), "hc_spiral_conv_fwd")
+
+
+def hc_test_set_option(option: int, value: int):
+    """Test hook (include/hc.h): force a group-norm path, or lower the
+    pipelined kernels' wait limit on the current device (0 = default)."""
+    _check(load_library().hc_test_set_option(int(option), int(value)), "hc_test_set_option")
 
 
 def hc_get_device_status(stream=None) -> int:

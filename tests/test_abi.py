@@ -61,9 +61,15 @@ def test_invalid_arguments_rejected_on_host(lib):
     # misaligned pointer for the element size
     assert lib.hc_spiral_conv_fwd(P(0x1001), 1, fake, 1, 4, 3, 8, 8, fake, None, 1, fake,
                                   None) == hc.HC_ERR_INVALID_ARG
-    # zero_fill without row_of
-    assert lib.hc_scatter_dense(fake, 1, fake, None, fake, 2, 3, 8, 1, fake,
+    # neither coords nor (with zero_fill) row_of
+    assert lib.hc_scatter_dense(fake, 1, None, None, fake, 2, 3, 8, 1, fake,
                                 None) == hc.HC_ERR_INVALID_ARG
+    assert lib.hc_scatter_dense(fake, 1, None, fake, fake, 2, 3, 8, 0, fake,
+                                None) == hc.HC_ERR_INVALID_ARG
+    # test hooks: unknown option, group-norm path out of range (no CUDA call)
+    assert lib.hc_test_set_option(99, 0) == hc.HC_ERR_INVALID_ARG
+    assert lib.hc_test_set_option(hc.HC_TEST_GROUP_NORM_PATH, 3) == hc.HC_ERR_INVALID_ARG
+    assert lib.hc_test_set_option(hc.HC_TEST_WAIT_LIMIT_NS, -5) == hc.HC_ERR_INVALID_ARG
     # negative capacity
     assert lib.hc_sparse_linear_fwd(fake, 1, fake, -1, 8, 8, fake, None, 0, fake,
                                     None) == hc.HC_ERR_INVALID_ARG

@@ -21,6 +21,20 @@ torch = pytest.importorskip("torch")
 NCPU = len(os.sched_getaffinity(0))
 
 
+@pytest.fixture
+def gn_force():
+    """Force the group-norm kernel choice ("auto", "slice" = one CTA per
+    frame and group, "rows" = the row-range kernels) through the library's
+    test hook; the automatic choice is restored afterwards."""
+    paths = {"auto": 0, "slice": 1, "rows": 2}
+
+    def force(path):
+        hc.hc_test_set_option(hc.HC_TEST_GROUP_NORM_PATH, paths[path])
+
+    yield force
+    hc.hc_test_set_option(hc.HC_TEST_GROUP_NORM_PATH, 0)
+
+
 @pytest.fixture(scope="module", autouse=True)
 def _lib():
     if not torch.cuda.is_available():
@@ -436,8 +450,11 @@ def test_sparse_linear(C_in, C_out, dtype):
 
 @pytest.mark.parametrize("dtype", ["bf16", "f32"])
 @pytest.mark.parametrize("C", [1, 3, 8, 42, 128])
-@pytest.mark.parametrize("zero_fill", [0, 1])
-def test_scatter_dense(C, zero_fill, dtype):
+@pytest.mark.parametrize("zero_fill,inverse", [(0, "row_of"), (1, "row_of"), (1, "none")])
+def test_scatter_dense(C, zero_fill, inverse, dtype):
+    """Copy of the active rows, bit for bit; with zero_fill every other row
+    becomes 0, through the inverse map (one pass) or, without it, a zero pass
+    then the scatter (the call as the problem statement gives it)."""
     rng = np.random.default_rng(C * 10 + zero_fill)
     B, V = 5, 333
     m = inputs.uniform_mask(rng, B, V, 0.25)
@@ -446,7 +463,8 @@ def test_scatter_dense(C, zero_fill, dtype):
     y = inputs.features(rng, (n, C), dtype)
     prev = inputs.features(rng, (B, V, C), dtype)
     out = to_torch(prev)
-    hc.hc_scatter_dense(to_torch(y), coords, row_of, count, B, V, zero_fill, out)
+    hc.hc_scatter_dense(to_torch(y), coords, row_of if inverse == "row_of" else None, count, B,
+                        V, zero_fill, out)
     assert hc.hc_get_device_status() == hc.HC_OK
     ref = oracle.scatter_dense(y, c, B, V, zero_fill, out=prev)
     np.testing.assert_array_equal(to_numpy(out), ref)
@@ -484,12 +502,11 @@ def _as_f32(a):
                                  (256, 16), (1024, 512), (42, 6), (48, 3)])
 @pytest.mark.parametrize("affine,act", [(False, 0), (True, 1), (True, 2)])
 @pytest.mark.parametrize("path", ["auto", "rows"])
-def test_group_norm(C, G, affine, act, dtype, path, monkeypatch):
+def test_group_norm(C, G, affine, act, dtype, path, gn_force):
     """Frames of 0, 1, a few, a tile-ish and a large number of rows; rows
     after the last frame stay untouched. 'rows' forces the row-range kernels
     wherever the layout allows them."""
-    if path == "rows":
-        monkeypatch.setenv("HC_GN_ROWS", "1")
+    gn_force(path)
     rng = np.random.default_rng(C * 100 + G * 7 + act)
     sizes = [0, 1, 3, 0, 130, 517, 2900, 64]
     x, offs = _gn_case(rng, sizes, C, dtype)
@@ -505,12 +522,12 @@ def test_group_norm(C, G, affine, act, dtype, path, monkeypatch):
 @pytest.mark.parametrize("dtype", ["bf16", "f32"])
 @pytest.mark.parametrize("C,G", [(64, 8), (128, 32), (2048, 8)])
 @pytest.mark.parametrize("path", ["rows", "slice"])
-def test_group_norm_paths_and_frame_shapes(C, G, path, dtype, monkeypatch):
+def test_group_norm_paths_and_frame_shapes(C, G, path, dtype, gn_force):
     """Both kernels (contiguous row ranges, and one CTA per frame and group)
     on many tiny frames (a row range holds dozens of frame segments) and on
     one frame spread over hundreds of row ranges (its partials are merged by
     a warp)."""
-    monkeypatch.setenv("HC_GN_SLICE" if path == "slice" else "HC_GN_ROWS", "1")
+    gn_force(path)
     rng = np.random.default_rng(C + G)
     tiny = [int(v) for v in rng.integers(0, 6, size=300)]
     big = [40000 if C <= 128 else 3000]
@@ -544,10 +561,10 @@ def test_group_norm_in_place_and_misaligned(dtype):
 
 
 @pytest.mark.parametrize("path", ["rows", "slice"])
-def test_group_norm_constant_group_and_eps(path, monkeypatch):
+def test_group_norm_constant_group_and_eps(path, gn_force):
     """A group of equal values normalises to exactly 0 (then + beta); eps
     from 0 to large enters as 1/sqrt(var + eps)."""
-    monkeypatch.setenv("HC_GN_SLICE" if path == "slice" else "HC_GN_ROWS", "1")
+    gn_force(path)
     C, G = 32, 4
     offs = np.array([0, 200, 201], dtype=np.int32)
     x = np.full((201, C), 100.25, dtype=np.float32)
@@ -561,7 +578,7 @@ def test_group_norm_constant_group_and_eps(path, monkeypatch):
         check_close(run_group_norm(x, offs, G, None, None, 0, eps=eps), y_pre, f"eps={eps}")
 
 
-def test_group_norm_on_compacted_layer_output():
+def test_group_norm_on_compacted_layer_output(gn_force):
     """The normalisation an encoder applies after a conv: a full-size
     compacted bf16 activation (32 clustered frames of the 10475-vertex
     sphere, 128 channels, G = 8), frame ranges from hc_mask_compact."""
@@ -576,21 +593,17 @@ def test_group_norm_on_compacted_layer_output():
     y = torch.empty_like(xt)
     y_pre, _ = oracle.sparse_group_norm(x, to_numpy(offs), 8, 1e-5, gamma, beta, oracle.ACT_ELU)
     for path in ("auto", "rows"):
-        if path == "rows":
-            os.environ["HC_GN_ROWS"] = "1"
-        try:
-            y.fill_(float("nan"))
-            hc.hc_sparse_group_norm_fwd(xt, offs, 8, 1e-5, to_torch(gamma), to_torch(beta),
-                                        hc.HC_ACT_ELU, y)
-            assert hc.hc_get_device_status() == hc.HC_OK
-        finally:
-            os.environ.pop("HC_GN_ROWS", None)
+        gn_force(path)
+        y.fill_(float("nan"))
+        hc.hc_sparse_group_norm_fwd(xt, offs, 8, 1e-5, to_torch(gamma), to_torch(beta),
+                                    hc.HC_ACT_ELU, y)
+        assert hc.hc_get_device_status() == hc.HC_OK
         check_close(to_numpy(y), y_pre, f"group norm full size ({path})")
 
 
 @pytest.mark.parametrize("path", ["rows", "slice"])
-def test_group_norm_bad_offsets_reported(path, monkeypatch):
-    monkeypatch.setenv("HC_GN_SLICE" if path == "slice" else "HC_GN_ROWS", "1")
+def test_group_norm_bad_offsets_reported(path, gn_force):
+    gn_force(path)
     x = torch.zeros((10, 16), dtype=torch.float32, device="cuda")
     offs = torch.tensor([0, 4, 12], dtype=torch.int32, device="cuda")  # 12 > capacity
     hc.hc_sparse_group_norm_fwd(x, offs, 4, 1e-5, None, None, 0, x)

@@ -1,8 +1,9 @@
-"""hc_mask_compact_static: compaction for callers that cannot allocate device
-memory (for example code running while a stream is captured into a CUDA
-graph, or a process whose device memory is all handed to its own pool). It
-uses a fixed scratch array inside the library instead of a workspace that the
-library allocates, and must give exactly what hc_mask_compact gives.
+"""hc_mask_compact_static: the mask compaction for callers that cannot
+allocate device memory while they compact, such as a process that gives all
+of its device memory to its own pool up front and must not allocate behind
+that pool's back. It uses a fixed scratch array inside the library instead
+of the workspace hc_mask_compact allocates per (device, stream), and must
+give exactly what hc_mask_compact gives.
 
 This file is collected last on purpose, so that a run stopping at the first
 failure has already run every other test. It passes on its own in a fresh
@@ -42,12 +43,17 @@ def _same(a, b):
     assert torch.equal(a[2], b[2])
 
 
-@pytest.mark.parametrize("B,V,density", [(7, 655, 0.1), (520, 10475, 0.05)])
+# (7, 655): two tiles; (520, 10475): past 1024 tiles (the pre-scanned path);
+# (4096, 4096): exactly HC_STATIC_MAX_MASK_BYTES, every int32 of the scratch
+# array in use; (0, 655) and (3, 0): nothing to compact.
+@pytest.mark.parametrize("B,V,density", [(7, 655, 0.1), (520, 10475, 0.05), (4096, 4096, 0.01),
+                                         (0, 655, 0.1), (3, 0, 0.1)])
 def test_static_compaction_matches_hc_mask_compact(B, V, density):
     """Two calls in a row through the C-ABI, each compared with the
     allocating entry point on the same mask (bit-exact, the tolerance of
     every compaction test). The second mask differs from the first, so stale
     scratch from the first call would show up."""
+    assert B * V <= hc.HC_STATIC_MAX_MASK_BYTES
     rng = np.random.default_rng(B + V)
     for call in range(2):
         m = torch.from_numpy(inputs.uniform_mask(rng, B, V, density * (1 + call))).cuda()
@@ -57,6 +63,58 @@ def test_static_compaction_matches_hc_mask_compact(B, V, density):
         hc.hc_mask_compact_static(m, *got)
         assert hc.hc_get_device_status() == hc.HC_OK
         _same(got, ref)
+
+
+def test_static_compaction_allocates_nothing():
+    """After a first call on the device (which looks up the scratch array's
+    address), calls on a stream the library has never seen leave the
+    device's free memory unchanged, and still succeed once device memory is
+    exhausted: a workspace allocation (hc_mask_compact's first call on a new
+    stream) would have to take memory in both cases."""
+    B, V = 64, 10475
+    rng = np.random.default_rng(3)
+    masks = [torch.from_numpy(inputs.uniform_mask(rng, B, V, d)).cuda() for d in (0.1, 0.3)]
+    refs = []
+    for m in masks:
+        ref = _buffers(B, V)
+        hc.hc_mask_compact(m, *ref)
+        refs.append(ref)
+    got = [_buffers(B, V) for _ in masks]
+    hc.hc_mask_compact_static(masks[0], *got[0])  # set-up call (default stream)
+    torch.cuda.synchronize()
+    fresh = torch.cuda.Stream()
+    torch.cuda.synchronize()
+    free0 = torch.cuda.mem_get_info()[0]
+    hc.hc_mask_compact_static(masks[1], *got[1], stream=fresh)
+    fresh.synchronize()
+    assert torch.cuda.mem_get_info()[0] == free0
+    _same(got[1], refs[1])
+
+    # device memory exhausted: hold blocks until the allocator refuses more
+    # (nothing below allocates until they are released; the comparisons,
+    # which do, come after)
+    other = torch.cuda.Stream()
+    for out in got:
+        for t in out:
+            t.fill_(-7)
+    torch.cuda.synchronize()
+    held = []
+    block = max(torch.cuda.mem_get_info()[0] - (256 << 20), 2 << 20)
+    while block >= (2 << 20):
+        try:
+            held.append(torch.empty(block, dtype=torch.uint8, device="cuda"))
+        except torch.cuda.OutOfMemoryError:
+            block //= 2
+    try:
+        for m, out in zip(masks, got):
+            hc.hc_mask_compact_static(m, *out, stream=other)
+        other.synchronize()
+    finally:
+        del held
+        torch.cuda.empty_cache()
+    for out, ref in zip(got, refs):
+        _same(out, ref)
+    assert hc.hc_get_device_status() == hc.HC_OK
 
 
 def test_static_compaction_rejects_masks_above_the_limit():
