@@ -7,19 +7,20 @@
 // (zeros for absent taps, Eq. 4); the layer computes A * W + bias (Eq. 5 with
 // the bias of Eq. 6) and the activation of Eq. 10.
 //
-// One persistent CTA per SM, 320 threads in four roles:
+// One persistent CTA per SM, 352 threads in five roles:
 //   warp 9     index warp: for each tile, resolves the L x 128 tap table
 //              (coords -> spiral -> row_of, i.e. idx() of Eq. 4) with every
 //              load of a phase in flight at once, into one of two tables, so
 //              the next tile's table is built while the current one is used;
 //   warps 0-3  producers: fill a stage with the 128 rows x 64 bf16 of A for
-//              one k-block and the 64 x BN slice of W. The 128 threads gather
-//              A with 16-byte cp.async through the tap table (zero-fill for
-//              absent taps and for k past L*C_in) and signal completion on
-//              the stage's "full" mbarrier without blocking; thread 0 loads
-//              W with TMA tiled copies onto the same barrier (transaction
-//              count). Gather and weight loads thus use different engines.
-//              (A variant loads W with cp.async too, for comparison.);
+//              one k-block. The 128 threads gather A with 16-byte cp.async
+//              through the tap table (zero-fill for absent taps and for k past
+//              L*C_in) and signal completion on the stage's "full" mbarrier
+//              without blocking;
+//   warp 10    weight loader (one thread): the 64 x BN slice of W of each
+//              stage by TMA tiled copies onto the same barrier (transaction
+//              count). Gather and weight loads thus use different engines,
+//              and the gather warps never wait on a TMA issue;
 //   warp 8     MMA issuer (one thread): 4 x tcgen05.mma (K = 16 each) per
 //              stage into a TMEM accumulator, tcgen05.commit frees the stage;
 //   warps 4-7  epilogue: tcgen05.ld the 128 x BN fp32 accumulator (warp w
@@ -44,7 +45,6 @@
 #include <cuda_bf16.h>
 #include <cudaTypedefs.h>
 
-#include <cstdlib>
 #include <cstring>
 #include <mutex>
 
@@ -60,7 +60,8 @@ constexpr int kProducerWarps = 4;
 constexpr int kEpilogueWarps = 4;
 constexpr int kMmaWarp = kProducerWarps + kEpilogueWarps;
 constexpr int kIndexWarp = kMmaWarp + 1;
-constexpr int kThreads = (kIndexWarp + 1) * 32;
+constexpr int kWeightWarp = kIndexWarp + 1;
+constexpr int kThreads = (kWeightWarp + 1) * 32;
 constexpr int kTabChunk = 8;  // spiral slots resolved per pass of the index warp
 constexpr size_t kSmemLimit = 227 * 1024;  // opt-in dynamic shared memory per CTA
 
@@ -72,7 +73,6 @@ struct Cfg {
     // grow with L), between kMinStages and kMaxStages.
     static constexpr int kMaxStages = BN == 64 ? 8 : 6;
     static constexpr int kMinStages = BN == 64 ? 7 : 5;
-    static constexpr int kLag = kMinStages - 1;  // cp.async groups a producer keeps in flight
     static constexpr int kTmemCols = 2 * BN;  // two accumulators
     // Instruction descriptor, kind::f16: D fp32 (bit 4), A bf16 (bits 7-9 = 1),
     // B bf16 (bits 10-12 = 1), A K-major (bit 15 = 0), B MN-major (bit 16 = 1),
@@ -306,14 +306,13 @@ __device__ __forceinline__ void gn_stats_chunk(const ConvArgs& a, const uint32_t
     }
 }
 
-template <int BN, bool kTma>
+template <int BN>
 __global__ void __launch_bounds__(kThreads, 1)
-    conv_tc_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
-                   const __grid_constant__ CUtensorMap tmap_w) {
+    conv_tc_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_w) {
     using C = Cfg<BN>;
     // "full": one cp.async completion arrival per producer thread, plus the
-    // expect-tx arrival of the weight TMA in the hybrid producer.
-    constexpr int kStageArrivals = kProducerWarps * 32 + (kTma ? 1 : 0);
+    // expect-tx arrival of the weight loader.
+    constexpr int kStageArrivals = kProducerWarps * 32 + 1;
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;
@@ -357,7 +356,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         *abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
     }
-    if (kTma && threadIdx.x == 32) prefetch_tensormap(&tmap_w);
+    if (warp == kWeightWarp && lane == 0) prefetch_tensormap(&tmap_w);
     if (warp == kMmaWarp) {
         tmem_alloc(smem_u32((const void*)tmem_holder), C::kTmemCols);
         tmem_relinquish();
@@ -418,170 +417,106 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     if (warp < kProducerWarps) {
         // ------------------------------------------------------------ producers
-        if constexpr (kTma) {
-            // A is gathered by all 128 producer threads with 16-byte cp.async
-            // (row r of the stage at r*128 bytes, chunk q at q ^ (r % 8)),
-            // whose completion each thread signals on the stage's "full"
-            // barrier without blocking (cp.async.mbarrier.arrive.noinc);
-            // thread 0 loads the W slice with TMA tiled copies on the same
-            // barrier (transaction count). The two paths run on different
-            // engines (load/store unit and TMA), which measured ~1.8x the
-            // ingress of gathering the rows with TMA as well.
-            const __nv_bfloat16* __restrict__ x = static_cast<const __nv_bfloat16*>(a.x);
-            const int t = threadIdx.x;  // 0..127
-            const int q = t & 7;        // A: 16-byte chunk of the 128-byte row
-            constexpr uint32_t kWBytes = (uint32_t)(BN / 64) * (kBK * 128u);
-            long long it = 0;
-            int st_s = 0;        // stage of iteration it (it % stages)
-            uint32_t st_ph = 0;  // its phase parity ((it / stages) & 1)
-            int lt = 0;
-            bool ok = true;
-            for (long long w = blockIdx.x; w < work_total && ok; w += gridDim.x, ++lt) {
-                const int n0 = ((int)w % n_tiles) * BN;  // w < 2^31
-                const int buf = lt & 1;
-                if (!mbar_wait(tabfull_bar(buf), (uint32_t)((lt >> 1) & 1), abort_flag,
-                               a.status)) {
+        // A is gathered by all 128 producer threads with 16-byte cp.async
+        // (row r of the stage at r*128 bytes, chunk q at q ^ (r % 8)), whose
+        // completion each thread signals on the stage's "full" barrier
+        // without blocking (cp.async.mbarrier.arrive.noinc).
+        const __nv_bfloat16* __restrict__ x = static_cast<const __nv_bfloat16*>(a.x);
+        const int t = threadIdx.x;  // 0..127
+        const int q = t & 7;        // 16-byte chunk of the 128-byte row
+        int st_s = 0;        // stage of the current iteration (it % stages)
+        uint32_t st_ph = 0;  // its phase parity ((it / stages) & 1)
+        int lt = 0;
+        bool ok = true;
+        for (long long w = blockIdx.x; w < work_total && ok; w += gridDim.x, ++lt) {
+            const int buf = lt & 1;
+            if (!mbar_wait(tabfull_bar(buf), (uint32_t)((lt >> 1) & 1), abort_flag, a.status)) {
+                ok = false;
+                break;
+            }
+            const uint32_t tab_s = tab0 + (uint32_t)buf * tab_bytes;
+            int l = (q * 8) / C_in;  // slot and channel of this thread's chunk at k-block 0
+            int c = q * 8 - l * C_in;
+            for (int kb = 0; kb < num_kb; ++kb) {
+                const int s = st_s;
+                const uint32_t ph = st_ph;
+                if (!mbar_wait(empty_bar(s), ph ^ 1u, abort_flag, a.status)) {
                     ok = false;
                     break;
                 }
-                const uint32_t tab_s = tab0 + (uint32_t)buf * tab_bytes;
-                int l = (q * 8) / C_in;  // slot and channel of this thread's chunk at k-block 0
-                int c = q * 8 - l * C_in;
+                const uint32_t a_st = sA + s * kAStageBytes;
+                const bool kval = kb * kBK + q * 8 < K;
+                // All eight table entries of this stage first, then the copies.
+                int src[8];
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const int r = (t >> 3) + 16 * i;
+                    src[i] = kval ? lds_s32(tab_s + (uint32_t)(l * kBM + r) * 4u) : -1;
+                }
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const int r = (t >> 3) + 16 * i;
+                    const __nv_bfloat16* gp = x + (src[i] >= 0 ? (long long)src[i] * C_in + c : 0);
+                    cp_async_16(a_st + r * 128 + ((q ^ (r & 7)) << 4), gp, src[i] >= 0);
+                }
+                cp_async_arrive_noinc(full_bar(s));
+                if (++st_s == nst) {
+                    st_s = 0;
+                    st_ph ^= 1u;
+                }
+                c += kBK;
+                while (c >= C_in) {
+                    c -= C_in;
+                    ++l;
+                }
+            }
+            // Addresses of this tile's copies are issued: the table is free.
+            if (ok) mbar_arrive(tabempty_bar(buf));
+        }
+        cp_async_wait_all();
+    } else if (warp == kWeightWarp) {
+        // ------------------------------------------------------------ weight loader
+        if (lane == 0) {
+            constexpr uint32_t kWBytes = (uint32_t)(BN / 64) * (kBK * 128u);
+            long long it = 0;
+            int st_s = 0;
+            uint32_t st_ph = 0;
+            bool ok = true;
+            for (long long w = blockIdx.x; w < work_total && ok; w += gridDim.x) {
+                const int n0 = ((int)w % n_tiles) * BN;  // w < 2^31
                 for (int kb = 0; kb < num_kb; ++kb) {
                     const int s = st_s;
-                    const uint32_t ph = st_ph;
-                    if (!mbar_wait(empty_bar(s), ph ^ 1u, abort_flag, a.status)) {
+                    if (!mbar_wait(empty_bar(s), st_ph ^ 1u, abort_flag, a.status)) {
                         ok = false;
                         break;
                     }
-                    if (t == 0) {
-                        mbar_arrive_expect_tx(full_bar(s), kWBytes);
+                    mbar_arrive_expect_tx(full_bar(s), kWBytes);
+                    if (a.w3d) {
+                        // both 64-column blocks of the slice in one copy
+                        tma_load_3d(sB + s * C::kBStageBytes, &tmap_w, 0, kb * kBK, n0 / 64,
+                                    full_bar(s));
+                    } else {
 #pragma unroll
                         for (int nb = 0; nb < BN / 64; ++nb)
                             tma_load_2d(sB + s * C::kBStageBytes + nb * (kBK * 128), &tmap_w,
                                         n0 + nb * 64, kb * kBK, full_bar(s));
                     }
-                    const uint32_t a_st = sA + s * kAStageBytes;
-                    const bool kval = kb * kBK + q * 8 < K;
-                    // All eight table entries of this stage first, then the copies.
-                    int src[8];
-#pragma unroll
-                    for (int i = 0; i < 8; ++i) {
-                        const int r = (t >> 3) + 16 * i;
-                        src[i] = kval ? lds_s32(tab_s + (uint32_t)(l * kBM + r) * 4u) : -1;
-                    }
-#pragma unroll
-                    for (int i = 0; i < 8; ++i) {
-                        const int r = (t >> 3) + 16 * i;
-                        const __nv_bfloat16* gp =
-                            x + (src[i] >= 0 ? (long long)src[i] * C_in + c : 0);
-                        cp_async_16(a_st + r * 128 + ((q ^ (r & 7)) << 4), gp, src[i] >= 0);
-                    }
-                    cp_async_arrive_noinc(full_bar(s));
                     ++it;
                     if (++st_s == nst) {
                         st_s = 0;
                         st_ph ^= 1u;
                     }
-                    c += kBK;
-                    while (c >= C_in) {
-                        c -= C_in;
-                        ++l;
-                    }
                 }
-                // Addresses of this tile's copies are issued: the table is free.
-                if (ok) mbar_arrive(tabempty_bar(buf));
             }
-            cp_async_wait_all();
-            if (!ok && t == 0) {
-                // Let the weight copies already issued land before the CTA exits.
+            if (!ok) {
+                // Let the weight copies already issued land before the CTA
+                // exits (bounded: the full barriers also count the gather
+                // threads' arrivals, which an unwinding producer may not make).
                 for (long long j = it > nst ? it - nst : 0; j < it; ++j)
-                    mbar_wait_drain(full_bar((int)(j % nst)), (uint32_t)((j / nst) & 1),
-                                    a.status);
+                    mbar_wait_drain(full_bar((int)(j % nst)), (uint32_t)((j / nst) & 1), a.status);
             }
-        } else {
-            const __nv_bfloat16* __restrict__ x = static_cast<const __nv_bfloat16*>(a.x);
-            const __nv_bfloat16* __restrict__ W = static_cast<const __nv_bfloat16*>(a.W);
-            const int t = threadIdx.x;  // 0..127
-            const int q = t & 7;        // A: 16-byte chunk of the 128-byte row
-            long long it = 0;
-            int st_s = 0;        // stage of iteration it (it % stages)
-            uint32_t st_ph = 0;  // its phase parity ((it / stages) & 1)
-            int lt = 0;
-            bool ok = true;
-            for (long long w = blockIdx.x; w < work_total && ok; w += gridDim.x, ++lt) {
-                const int n0 = ((int)w % n_tiles) * BN;  // w < 2^31
-                const int buf = lt & 1;
-                if (!mbar_wait(tabfull_bar(buf), (uint32_t)((lt >> 1) & 1), abort_flag,
-                               a.status)) {
-                    ok = false;
-                    break;
-                }
-                const uint32_t tab_s = tab0 + (uint32_t)buf * tab_bytes;
-                int l = (q * 8) / C_in;  // slot and channel of this thread's chunk at k-block 0
-                int c = q * 8 - l * C_in;
-                for (int kb = 0; kb < num_kb; ++kb) {
-                    const int s = st_s;
-                    const uint32_t ph = st_ph;
-                    if (!mbar_wait(empty_bar(s), ph ^ 1u, abort_flag, a.status)) {
-                        ok = false;
-                        break;
-                    }
-                    const uint32_t a_st = sA + s * kAStageBytes;
-                    const bool kval = kb * kBK + q * 8 < K;
-                    // All eight table entries of this stage first, then the copies.
-                    int src[8];
-#pragma unroll
-                    for (int i = 0; i < 8; ++i) {
-                        const int r = (t >> 3) + 16 * i;
-                        src[i] = kval ? lds_s32(tab_s + (uint32_t)(l * kBM + r) * 4u) : -1;
-                    }
-#pragma unroll
-                    for (int i = 0; i < 8; ++i) {
-                        const int r = (t >> 3) + 16 * i;
-                        const __nv_bfloat16* gp =
-                            x + (src[i] >= 0 ? (long long)src[i] * C_in + c : 0);
-                        cp_async_16(a_st + r * 128 + ((q ^ (r & 7)) << 4), gp, src[i] >= 0);
-                    }
-                    const uint32_t b_st = sB + s * C::kBStageBytes;
-                    constexpr int kCpr = BN / 8;  // 16-byte chunks per W row slice
-#pragma unroll
-                    for (int i = 0; i < (kBK * kCpr) / 128; ++i) {
-                        const int e = t + 128 * i;
-                        const int kr = e / kCpr, nq = e % kCpr;
-                        const int kk = kb * kBK + kr, col = n0 + nq * 8;
-                        const bool valid = kk < K && col < C_out;
-                        const __nv_bfloat16* gp = W + (valid ? (long long)kk * C_out + col : 0);
-                        cp_async_16(b_st + (nq >> 3) * (kBK * 128) + kr * 128 +
-                                        (((nq & 7) ^ (kr & 7)) << 4),
-                                    gp, valid);
-                    }
-                    cp_async_commit();
-                    if (it >= C::kLag) {
-                        cp_async_wait<C::kLag>();
-                        fence_proxy_async_smem();
-                        mbar_arrive(full_bar((int)((it - C::kLag) % nst)));
-                    }
-                    ++it;
-                    if (++st_s == nst) {
-                        st_s = 0;
-                        st_ph ^= 1u;
-                    }
-                    c += kBK;
-                    while (c >= C_in) {
-                        c -= C_in;
-                        ++l;
-                    }
-                }
-                // Addresses of this tile's copies are issued: the table is free.
-                if (ok) mbar_arrive(tabempty_bar(buf));
-            }
-            cp_async_wait_all();
-            fence_proxy_async_smem();
-            if (ok)
-                for (long long j = it > C::kLag ? it - C::kLag : 0; j < it; ++j)
-                    mbar_arrive(full_bar((int)(j % nst)));
         }
+        __syncwarp();
     } else if (warp == kMmaWarp) {
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0) {
@@ -915,46 +850,62 @@ hc_status encode_2d(CUtensorMap* m, const void* base, long long rows, long long 
     return HC_OK;
 }
 
-template <int BN, bool kTma>
+// The weight matrix [K, C_out] (C_out a multiple of 64) as the 3-D tensor
+// [C_out / 64][K][64] with 128-byte swizzled boxes of 64 x box_k x box_blocks.
+hc_status encode_w3d(CUtensorMap* m, const void* base, long long K, long long C_out, int box_k,
+                     int box_blocks) {
+    auto enc = tensor_map_encoder();
+    if (!enc) {
+        set_error("cuTensorMapEncodeTiled is unavailable");
+        return HC_ERR_CUDA;
+    }
+    cuuint64_t dims[3] = {64, (cuuint64_t)K, (cuuint64_t)(C_out / 64)};
+    cuuint64_t strides[2] = {(cuuint64_t)C_out * 2, 128};
+    cuuint32_t box[3] = {64, (cuuint32_t)box_k, (cuuint32_t)box_blocks};
+    cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides,
+                     box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) {
+        set_error("cuTensorMapEncodeTiled (3-D weight view) failed (%d)", (int)r);
+        return HC_ERR_CUDA;
+    }
+    return HC_OK;
+}
+
+template <int BN>
 hc_status launch_bn(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s) {
     using C = Cfg<BN>;
     static bool attr_set[64] = {};
     if (!attr_set[ctx->device]) {
-        hc_status st = check_cuda(cudaFuncSetAttribute(conv_tc_kernel<BN, kTma>,
+        hc_status st = check_cuda(cudaFuncSetAttribute(conv_tc_kernel<BN>,
                                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                        (int)kSmemLimit),
                                   "cudaFuncSetAttribute(conv_tc_kernel)");
         if (st != HC_OK) return st;
         attr_set[ctx->device] = true;
     }
-    CUtensorMap tx, tw;
-    memset(&tx, 0, sizeof tx);
+    CUtensorMap tw;
     memset(&tw, 0, sizeof tw);
-    if (kTma) {
-        // W: [K rows, C_out], boxes of 64 K-rows x 64 output channels.
-        hc_status st = encode_2d(&tw, a.W, a.K, a.C_out, 64, kBK);
-        if (st != HC_OK) return st;
-    }
+    ConvArgs ka = a;
+    // W: [K rows, C_out]. With C_out a multiple of 64, the 3-D view
+    // [C_out / 64][K][64] (the 64-column blocks 128 bytes apart) takes a
+    // tile's BN columns of a k-block in one box of 64 x 64 x BN/64; otherwise
+    // 2-D boxes of 64 K-rows x 64 output channels, one per block.
+    hc_status st;
+    ka.w3d = a.C_out % 64 == 0;
+    if (ka.w3d)
+        st = encode_w3d(&tw, a.W, a.K, a.C_out, kBK, BN / 64);
+    else
+        st = encode_2d(&tw, a.W, a.K, a.C_out, 64, kBK);
+    if (st != HC_OK) return st;
     const long long n_tiles = (a.C_out + BN - 1) / BN;
     const long long cap_work = (a.capacity + kBM - 1) / kBM * n_tiles;
     long long grid = cap_work < ctx->num_sms ? cap_work : ctx->num_sms;
     if (grid < 1) grid = 1;
-    ConvArgs ka = a;
     ka.stages = C::stages_for(a.L);
-    // HC_TC_STAGES overrides the depth (clamped to what fits), for tuning.
-    static int env_stages = -1;
-    if (env_stages < 0) {
-        const char* e = getenv("HC_TC_STAGES");
-        env_stages = e ? atoi(e) : 0;
-    }
-    if (env_stages > 0) {
-        int st = env_stages < C::kMaxStages ? env_stages : C::kMaxStages;
-        if (st < C::kMinStages) st = C::kMinStages;
-        while (st > C::kMinStages && C::smem_bytes(a.L, st) > kSmemLimit) --st;
-        ka.stages = st;
-    }
-    return launch_pdl(conv_tc_kernel<BN, kTma>, dim3((unsigned)grid), dim3(kThreads),
-                      C::smem_bytes(a.L, ka.stages), s, "conv_tc_kernel", ka, tx, tw);
+    return launch_pdl(conv_tc_kernel<BN>, dim3((unsigned)grid), dim3(kThreads),
+                      C::smem_bytes(a.L, ka.stages), s, "conv_tc_kernel", ka, tw);
 }
 
 }  // namespace
@@ -973,17 +924,8 @@ int conv_tc_tile_n(const ConvArgs& a) {
 }
 
 hc_status launch_conv_tc(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s) {
-    // The weight slice comes by TMA; HC_NO_TMA=1 selects the all-cp.async
-    // producer instead (for comparison).
-    static int tma_off = -1;
-    if (tma_off < 0) {
-        const char* e = getenv("HC_NO_TMA");
-        tma_off = (e && e[0] == '1') ? 1 : 0;
-    }
-    const bool tma = !tma_off;
-    if (conv_tc_tile_n(a) == 64)
-        return tma ? launch_bn<64, true>(ctx, a, s) : launch_bn<64, false>(ctx, a, s);
-    return tma ? launch_bn<128, true>(ctx, a, s) : launch_bn<128, false>(ctx, a, s);
+    if (conv_tc_tile_n(a) == 64) return launch_bn<64>(ctx, a, s);
+    return launch_bn<128>(ctx, a, s);
 }
 
 }  // namespace hc

@@ -83,6 +83,7 @@ struct ConvArgs {
     int mode;
     int act;
     int stages;  // pipeline depth chosen by the launcher (tensor-core kernel)
+    int w3d;     // tensor-core kernel: W's tensor map is the 3-D view (one box per stage)
     // Optional group-norm statistics of the stored output (Eqs. 7-9,
     // tensor-core kernel): every block c of 32 output rows writes, for each
     // frame b among its rows (b = gn_coords[2n]) and each channel group g of
@@ -437,6 +438,15 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const void* tmap, int 
         "l"(reinterpret_cast<uint64_t>(tmap)), "r"(c0), "r"(c1), "r"(bar)
         : "memory");
 }
+// 3-D tiled load of the tensor map's box at (c0, c1, c2), innermost first.
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const void* tmap, int c0, int c1, int c2,
+                                            uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3, %4}], [%5];\n" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(tmap)), "r"(c0), "r"(c1), "r"(c2), "r"(bar)
+        : "memory");
+}
 // Four rows (r0..r3) of a box one row high, starting at column c0, written to
 // consecutive box rows in shared memory. Rows outside the tensor read zeros.
 __device__ __forceinline__ void tma_gather4(uint32_t dst, const void* tmap, int c0, int r0, int r1,
@@ -450,6 +460,24 @@ __device__ __forceinline__ void tma_gather4(uint32_t dst, const void* tmap, int 
 }
 __device__ __forceinline__ void prefetch_tensormap(const void* tmap) {
     asm volatile("prefetch.tensormap [%0];\n" ::"l"(reinterpret_cast<uint64_t>(tmap)) : "memory");
+}
+// ---- bulk copies shared -> global (TMA engine), tracked per thread in
+// bulk async-groups
+__device__ __forceinline__ void bulk_store(void* gdst, uint32_t ssrc, uint32_t bytes) {
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;\n" ::"l"(gdst),
+                 "r"(ssrc), "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit() {
+    asm volatile("cp.async.bulk.commit_group;\n" ::: "memory");
+}
+// Every bulk copy of this thread has finished reading shared memory.
+__device__ __forceinline__ void bulk_wait_read_all() {
+    asm volatile("cp.async.bulk.wait_group.read 0;\n" ::: "memory");
+}
+// Every bulk copy of this thread has completed.
+__device__ __forceinline__ void bulk_wait_all() {
+    asm volatile("cp.async.bulk.wait_group 0;\n" ::: "memory");
 }
 __device__ __forceinline__ void sts_v4(uint32_t addr, uint4 v) {
     asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};\n" ::"r"(addr), "r"(v.x), "r"(v.y),
@@ -498,6 +526,17 @@ __device__ __forceinline__ void tc_mma_bf16(uint32_t d_tmem, uint64_t a_desc, ui
         "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
         " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
         "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+// The same, accumulating onto D, with the rows (TMEM lanes) whose bit is set
+// in the 128-bit `disable` (word i, bit r: lane 32 i + r) left unchanged.
+__device__ __forceinline__ void tc_mma_bf16_masked(uint32_t d_tmem, uint64_t a_desc,
+                                                   uint64_t b_desc, uint32_t idesc, uint4 disable) {
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, 1, 0;\n"
+        " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, {%4, %5, %6, %7}, p;\n}\n" ::"r"(d_tmem),
+        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(disable.x), "r"(disable.y), "r"(disable.z),
+        "r"(disable.w)
         : "memory");
 }
 // Arrive once on `bar` when every tcgen05 op issued so far by this thread
