@@ -7,30 +7,43 @@
 // (zeros for absent taps, Eq. 4); the layer computes A * W + bias (Eq. 5 with
 // the bias of Eq. 6) and the activation of Eq. 10.
 //
-// One persistent CTA per SM, 352 threads in five roles:
-//   warp 9     index warp: for each tile, resolves the L x 128 tap table
-//              (coords -> spiral -> row_of, i.e. idx() of Eq. 4) with every
-//              load of a phase in flight at once, into one of two tables, so
-//              the next tile's table is built while the current one is used;
-//   warps 0-3  producers: fill a stage with the 128 rows x 64 bf16 of A for
-//              one k-block. The 128 threads gather A with 16-byte cp.async
-//              through the tap table (zero-fill for absent taps and for k past
-//              L*C_in) and signal completion on the stage's "full" mbarrier
-//              without blocking;
+// One persistent CTA per SM, 352 threads in five roles. A work item is tm
+// 128-row halves of output rows (tm = 2 when there are at least two items per
+// CTA, else 1, decided from the device row count) times BN output channels;
+// both halves are multiplied by the same W slice of every stage, which halves
+// the weight traffic and the per-stage overhead per MMA of large layers.
+//   warp 9     index warp: for each item, resolves the L x (tm*128) tap table
+//              (from the rulebook, or coords -> spiral -> row_of, i.e. idx()
+//              of Eq. 4) with every load of a phase in flight at once, into
+//              one of two tables, so the next item's table is built while the
+//              current one is used;
+//   warps 0-3  producers: fill a stage with the tm x 128 rows x 64 bf16 of A
+//              for one k-block. The 128 threads gather A with 16-byte cp.async
+//              through the tap table (zero-fill for absent taps and for k
+//              past L*C_in) and signal completion on the stage's "full"
+//              mbarrier without blocking;
 //   warp 10    weight loader (one thread): the 64 x BN slice of W of each
-//              stage by TMA tiled copies onto the same barrier (transaction
-//              count). Gather and weight loads thus use different engines,
-//              and the gather warps never wait on a TMA issue;
-//   warp 8     MMA issuer (one thread): 4 x tcgen05.mma (K = 16 each) per
-//              stage into a TMEM accumulator, tcgen05.commit frees the stage;
-//   warps 4-7  epilogue: tcgen05.ld the 128 x BN fp32 accumulator (warp w
-//              reads TMEM lanes 32*(w%4)..+32), activation, round to bf16
-//              and store; then tcgen05.st the bias of the tile after next
-//              into every row of the freed accumulator, onto which its MMAs
-//              accumulate. Two accumulators (2*BN TMEM columns) let the
-//              epilogue of one tile overlap the main loop of the next.
+//              stage by TMA (one 3-D box when C_out is a multiple of 64) onto
+//              the same barrier (transaction count). Gather and weight loads
+//              thus use different engines, and the gather warps never wait on
+//              a TMA issue (which held the whole ring back when a gather
+//              thread issued it);
+//   warp 8     MMA issuer (one thread): per stage 4 x tm tcgen05.mma
+//              (M = 128, N = BN, K = 16) into the item's TMEM accumulators,
+//              tcgen05.commit frees the stage;
+//   warps 4-7  epilogue: tcgen05.ld each half's 128 x BN fp32 accumulator
+//              (warp w reads TMEM lanes 32*(w%4)..+32), activation, round to
+//              bf16 and store; then tcgen05.st the bias of the item after
+//              next into every row of the freed accumulators, onto which its
+//              MMAs accumulate. Two accumulator sets (2*tm*BN TMEM columns)
+//              let the epilogue of one item overlap the main loop of the next.
+// Each role runs its whole loop in a copy compiled for its half count (the
+// count is known once the row count is read); a run-time half loop between
+// the MMAs and copies cost ~1 us per launch at the small layers.
+// The stage ring holds a.stages two-half stages; one-half items cut the same
+// bytes into more (up to kRing) stages of 16 KB of A plus the W slice.
 // Shared-memory operand layouts (canonical tcgen05 forms, 128-byte swizzle):
-//   A: K-major, row r of the 128-row tile at r*128 bytes, 16-byte chunk q
+//   A: K-major, per half row r at r*128 bytes, 16-byte chunk q
 //      stored at chunk q ^ (r % 8); 8-row groups 1024 bytes apart (SBO).
 //   B: MN-major (W is [K, C_out] row-major, C_out contiguous), per 64-column
 //      block a [64 K-rows x 128 bytes] slab, K-row kr at kr*128 with chunk
@@ -47,22 +60,26 @@
 
 #include <cstring>
 #include <mutex>
+#include <type_traits>
 
 #include "hc_internal.cuh"
 
 namespace hc {
 namespace {
 
-constexpr int kBM = 128;  // rows per tile = TMEM lanes
+constexpr int kBM = 128;  // rows per tile half = TMEM lanes
 constexpr int kBK = 64;   // bf16 per 128-byte smem row
-constexpr int kAStageBytes = kBM * kBK * 2;
+constexpr int kHalves = 2;  // 128-row halves per work item at most (both share each W stage)
+constexpr int kTabRows = kHalves * kBM;  // rows of a tap table
+constexpr int kAHalfBytes = kBM * kBK * 2;
+constexpr int kAStageBytes = kHalves * kAHalfBytes;
 constexpr int kProducerWarps = 4;
 constexpr int kEpilogueWarps = 4;
 constexpr int kMmaWarp = kProducerWarps + kEpilogueWarps;
 constexpr int kIndexWarp = kMmaWarp + 1;
 constexpr int kWeightWarp = kIndexWarp + 1;
 constexpr int kThreads = (kWeightWarp + 1) * 32;
-constexpr int kTabChunk = 8;  // spiral slots resolved per pass of the index warp
+constexpr int kTabChunk = 6;  // spiral slots resolved per pass of the index warp
 constexpr size_t kSmemLimit = 227 * 1024;  // opt-in dynamic shared memory per CTA
 
 template <int BN>
@@ -71,25 +88,28 @@ struct Cfg {
     static constexpr int kBStageBytes = kBK * BN * 2;
     // Pipeline depth: as many stages as fit next to the tap tables (which
     // grow with L), between kMinStages and kMaxStages.
-    static constexpr int kMaxStages = BN == 64 ? 8 : 6;
-    static constexpr int kMinStages = BN == 64 ? 7 : 5;
-    static constexpr int kTmemCols = 2 * BN;  // two accumulators
+    // (stages of two-half items; one-half items cut the same bytes into
+    // more, smaller stages, at most kRing)
+    static constexpr int kMaxStages = BN == 64 ? 5 : 4;
+    static constexpr int kMinStages = 2;
+    static constexpr int kRing = BN == 64 ? 8 : 6;
+    // two accumulator buffers, each one BN-column accumulator per half
+    static constexpr int kTmemCols = 2 * kHalves * BN;
     // Instruction descriptor, kind::f16: D fp32 (bit 4), A bf16 (bits 7-9 = 1),
     // B bf16 (bits 10-12 = 1), A K-major (bit 15 = 0), B MN-major (bit 16 = 1),
     // N >> 3 at bits 17-22, M >> 4 at bits 24-28.
     static constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | (1u << 16) |
                                        ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(kBM >> 4) << 24);
-    static constexpr int kBarBytes = 8 * (2 * kMaxStages + 9);
+    static constexpr int kBarBytes = 8 * (2 * kRing + 9);
     // barriers, then 16 bytes (TMEM address, abort flag), then the two tap
-    // tables at a 128-byte boundary (the TMA producer reads them 16 bytes at
-    // a time).
+    // tables ([L][kTabRows] int32 each) at a 128-byte boundary.
     static constexpr int kTabOffset = (kBarBytes + 16 + 127) / 128 * 128;
     // After the tables: one 2 KB staging buffer per epilogue warp (32 rows x
     // 64 bytes of bf16 output).
     static constexpr int kEpiBytes = kEpilogueWarps * 32 * 64;
     static size_t smem_bytes(int L, int stages) {
         return 1024 + (size_t)stages * (kAStageBytes + kBStageBytes) + kTabOffset +
-               2 * sizeof(int) * (size_t)kBM * L + kEpiBytes;
+               2 * sizeof(int) * (size_t)kTabRows * L + kEpiBytes;
     }
     static int stages_for(int L) {
         int st = kMaxStages;
@@ -317,30 +337,29 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t raw = smem_u32(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;
     uint8_t* const base_ptr = smem_raw + (base - raw);
-    const uint32_t sA = base;
-    const int nst = a.stages;
-    const uint32_t sB = sA + nst * kAStageBytes;
-    const uint32_t sBar = sB + nst * C::kBStageBytes;
+    const uint32_t sA = base;  // the stage ring (a.stages two-half stages)
+    const uint32_t ring_bytes = (uint32_t)a.stages * (kAStageBytes + C::kBStageBytes);
+    const uint32_t sBar = sA + ring_bytes;
     uint8_t* const misc = base_ptr + (sBar - base) + C::kBarBytes;
     volatile uint32_t* const tmem_holder = reinterpret_cast<volatile uint32_t*>(misc);
     volatile int* const abort_flag = reinterpret_cast<volatile int*>(misc + 4);
-    // Tap tables, [2][L][kBM] int32: entry (l, r) is the input row feeding
-    // slot l of tile row r, or -1.
+    // Tap tables, [2][L][kTabRows] int32: entry (l, r) is the input row
+    // feeding slot l of row r of the work item, or -1.
     const uint32_t tab0 = sBar + C::kTabOffset;
-    const uint32_t epi0 = tab0 + 2u * (uint32_t)(kBM * a.L) * 4u;  // epilogue staging
+    const uint32_t epi0 = tab0 + 2u * (uint32_t)(kTabRows * a.L) * 4u;  // epilogue staging
 
     auto full_bar = [&](int s) { return sBar + 8u * s; };
-    auto empty_bar = [&](int s) { return sBar + 8u * (C::kMaxStages + s); };
-    auto tfull_bar = [&](int i) { return sBar + 8u * (2 * C::kMaxStages + i); };
-    auto tempty_bar = [&](int i) { return sBar + 8u * (2 * C::kMaxStages + 2 + i); };
-    const uint32_t fin_bar = sBar + 8u * (2 * C::kMaxStages + 4);
-    auto tabfull_bar = [&](int i) { return sBar + 8u * (2 * C::kMaxStages + 5 + i); };
-    auto tabempty_bar = [&](int i) { return sBar + 8u * (2 * C::kMaxStages + 7 + i); };
+    auto empty_bar = [&](int s) { return sBar + 8u * (C::kRing + s); };
+    auto tfull_bar = [&](int i) { return sBar + 8u * (2 * C::kRing + i); };
+    auto tempty_bar = [&](int i) { return sBar + 8u * (2 * C::kRing + 2 + i); };
+    const uint32_t fin_bar = sBar + 8u * (2 * C::kRing + 4);
+    auto tabfull_bar = [&](int i) { return sBar + 8u * (2 * C::kRing + 5 + i); };
+    auto tabempty_bar = [&](int i) { return sBar + 8u * (2 * C::kRing + 7 + i); };
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < nst; ++s) {
+        for (int s = 0; s < C::kRing; ++s) {
             mbar_init(full_bar(s), kStageArrivals);
             mbar_init(empty_bar(s), 1);
         }
@@ -370,40 +389,58 @@ __global__ void __launch_bounds__(kThreads, 1)
     pdl_wait();
     pdl_trigger();
 
-    // Rulebook mode: the index warp copies its first tile's entries into tap
-    // table 0 (cp.async, no registers held) before the row count arrives
-    // (rows clamped to the capacity, always valid memory), so the two L2
-    // round trips overlap instead of queueing.
-    const bool prefetched = warp == kIndexWarp && a.mode == kRulebook;
-    if (prefetched) {
+    // Rulebook mode: the index warp copies the entries of its first 128-row
+    // tile into tap table 0 (cp.async, no registers held) before the row
+    // count arrives (rows clamped to the capacity, always valid memory), so
+    // the two L2 round trips overlap instead of queueing. The copy is used
+    // when the count gives one-half work items (few rows, where this latency
+    // matters); with two-half items the loop builds the table instead.
+    const bool prefetch = warp == kIndexWarp && a.mode == kRulebook;
+    if (prefetch) {
         const long long m0p = (blockIdx.x / ((a.C_out + BN - 1) / BN)) * (long long)kBM;
         for (int d = 0; d < a.L; ++d)
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
                 const long long n = m0p + lane + 32 * i;
-                cp_async_4(tab0 + (uint32_t)(d * kBM + lane + 32 * i) * 4u,
+                cp_async_4(tab0 + (uint32_t)(d * kTabRows + lane + 32 * i) * 4u,
                            a.rulebook + (long long)d * a.capacity + (n < a.capacity ? n : 0), true);
             }
     }
 
     const long long rows = active_rows(a);
-    const long long m_tiles = (rows + kBM - 1) / kBM;
     const int n_tiles = (a.C_out + BN - 1) / BN;
-    const long long work_total = m_tiles * n_tiles;
+    // Work item: tm 128-row halves sharing every W stage. Two halves (half
+    // the weight traffic and per-stage overhead per MMA) when that still
+    // gives every CTA two items; one otherwise (few rows: the launch is
+    // latency-bound, and larger items would only deepen the last wave).
+    const long long tiles128 = (rows + kBM - 1) / kBM;
+    const int tm = (tiles128 + 1) / 2 * n_tiles >= 2ll * gridDim.x ? 2 : 1;
+    const int item_rows = tm * kBM;
+    const long long m_items = (rows + item_rows - 1) / item_rows;
+    const long long work_total = m_items * n_tiles;
     const int num_kb = (a.K + kBK - 1) / kBK;
     const int L = a.L, C_in = a.C_in, C_out = a.C_out, K = a.K;
-    const uint32_t tab_bytes = (uint32_t)(kBM * L) * 4u;
+    const uint32_t tab_bytes = (uint32_t)(kTabRows * L) * 4u;
+    const bool prefetched = prefetch && tm == 1;
+    // Stage s: tm halves of A (16 KB each), then the W slice; as many stages
+    // as the ring holds (kRing at most). 16 KB multiples keep every operand
+    // 1024-byte aligned.
+    const uint32_t stage_bytes = (uint32_t)(tm * kAHalfBytes + C::kBStageBytes);
+    const int nst_fit = (int)(ring_bytes / stage_bytes);
+    const int nst = nst_fit < C::kRing ? nst_fit : C::kRing;
+    auto a_stage = [&](int st) { return sA + (uint32_t)st * stage_bytes; };
+    auto b_stage = [&](int st) { return sA + (uint32_t)st * stage_bytes + (uint32_t)(tm * kAHalfBytes); };
+    if (prefetch) cp_async_wait_all();
     if (prefetched) {
         // the first tap table (buffer 0, not yet waited on by anyone): the
         // copied entries checked against the input's rows and masked by the
         // row count
-        cp_async_wait_all();
         const long long m0 = (blockIdx.x / n_tiles) * (long long)kBM;
         unsigned err = 0;
         for (int d = 0; d < L; ++d)
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
-                const uint32_t at = tab0 + (uint32_t)(d * kBM + lane + 32 * i) * 4u;
+                const uint32_t at = tab0 + (uint32_t)(d * kTabRows + lane + 32 * i) * 4u;
                 const int ev = lds_s32(at);
                 int src = -1;
                 if (m0 + lane + 32 * i < rows) {
@@ -424,6 +461,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         const __nv_bfloat16* __restrict__ x = static_cast<const __nv_bfloat16*>(a.x);
         const int t = threadIdx.x;  // 0..127
         const int q = t & 7;        // 16-byte chunk of the 128-byte row
+        // The role's whole loop for a half count fixed at compile time (one
+        // copy of the loop is hot per launch).
+        auto producer = [&](auto tm_c) {
+        constexpr int TM = decltype(tm_c)::value;
         int st_s = 0;        // stage of the current iteration (it % stages)
         uint32_t st_ph = 0;  // its phase parity ((it / stages) & 1)
         int lt = 0;
@@ -444,20 +485,31 @@ __global__ void __launch_bounds__(kThreads, 1)
                     ok = false;
                     break;
                 }
-                const uint32_t a_st = sA + s * kAStageBytes;
                 const bool kval = kb * kBK + q * 8 < K;
-                // All eight table entries of this stage first, then the copies.
-                int src[8];
+                {
+                    // All table entries first, then the copies: half h's 128
+                    // rows at a_stage + h * 16 KB, its entries at table rows
+                    // h * 128 ..
+                    int src[TM][8];
 #pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    const int r = (t >> 3) + 16 * i;
-                    src[i] = kval ? lds_s32(tab_s + (uint32_t)(l * kBM + r) * 4u) : -1;
-                }
+                    for (int h = 0; h < TM; ++h)
 #pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    const int r = (t >> 3) + 16 * i;
-                    const __nv_bfloat16* gp = x + (src[i] >= 0 ? (long long)src[i] * C_in + c : 0);
-                    cp_async_16(a_st + r * 128 + ((q ^ (r & 7)) << 4), gp, src[i] >= 0);
+                        for (int i = 0; i < 8; ++i) {
+                            const int r = h * kBM + (t >> 3) + 16 * i;
+                            src[h][i] = kval ? lds_s32(tab_s + (uint32_t)(l * kTabRows + r) * 4u)
+                                             : -1;
+                        }
+#pragma unroll
+                    for (int h = 0; h < TM; ++h)
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) {
+                            const int r = (t >> 3) + 16 * i;
+                            const __nv_bfloat16* gp =
+                                x + (src[h][i] >= 0 ? (long long)src[h][i] * C_in + c : 0);
+                            cp_async_16(a_stage(s) + h * kAHalfBytes + r * 128 +
+                                            ((q ^ (r & 7)) << 4),
+                                        gp, src[h][i] >= 0);
+                        }
                 }
                 cp_async_arrive_noinc(full_bar(s));
                 if (++st_s == nst) {
@@ -474,6 +526,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (ok) mbar_arrive(tabempty_bar(buf));
         }
         cp_async_wait_all();
+        };
+        if (tm == 2)
+            producer(std::integral_constant<int, 2>{});
+        else
+            producer(std::integral_constant<int, 1>{});
     } else if (warp == kWeightWarp) {
         // ------------------------------------------------------------ weight loader
         if (lane == 0) {
@@ -493,12 +550,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                     mbar_arrive_expect_tx(full_bar(s), kWBytes);
                     if (a.w3d) {
                         // both 64-column blocks of the slice in one copy
-                        tma_load_3d(sB + s * C::kBStageBytes, &tmap_w, 0, kb * kBK, n0 / 64,
+                        tma_load_3d(b_stage(s), &tmap_w, 0, kb * kBK, n0 / 64,
                                     full_bar(s));
                     } else {
 #pragma unroll
                         for (int nb = 0; nb < BN / 64; ++nb)
-                            tma_load_2d(sB + s * C::kBStageBytes + nb * (kBK * 128), &tmap_w,
+                            tma_load_2d(b_stage(s) + nb * (kBK * 128), &tmap_w,
                                         n0 + nb * 64, kb * kBK, full_bar(s));
                     }
                     ++it;
@@ -519,7 +576,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
     } else if (warp == kMmaWarp) {
         // ------------------------------------------------------------ MMA issuer
-        if (lane == 0) {
+        // the role's whole loop for a half count fixed at compile time
+        auto mma = [&](auto tm_c) {
+            constexpr int TM = decltype(tm_c)::value;
             long long it = 0;
             int st_s = 0;        // stage of iteration it (it % stages)
             uint32_t st_ph = 0;  // its phase parity ((it / stages) & 1)
@@ -535,7 +594,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     break;
                 }
                 tc_fence_after();
-                const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
+                // accumulator of half h: columns (acc * TM + h) * BN
+                const uint32_t d_tmem = tmem_base + (uint32_t)(acc * TM * BN);
                 for (int kb = 0; kb < num_kb; ++kb) {
                     const int s = st_s;
                     const uint32_t ph = st_ph;
@@ -547,13 +607,22 @@ __global__ void __launch_bounds__(kThreads, 1)
                     // The A operand was written by cp.async (generic proxy):
                     // order it before the tensor core's async-proxy reads.
                     fence_proxy_async_smem();
-                    const uint32_t a_st = sA + s * kAStageBytes;
-                    const uint32_t b_st = sB + s * C::kBStageBytes;
+                    const uint32_t a_st = a_stage(s);
+                    const uint32_t b_st = b_stage(s);
+                    {
 #pragma unroll
-                    for (int k = 0; k < kBK / 16; ++k) {
-                        const uint64_t ad = smem_desc_sw128(a_st + k * 32, 16, 1024);
-                        const uint64_t bd = smem_desc_sw128(b_st + k * 16 * 128, kBK * 128, 1024);
-                        tc_mma_bf16(d_tmem, ad, bd, C::kIdesc, (has_bias || (kb | k) != 0) ? 1u : 0u);
+                        for (int k = 0; k < kBK / 16; ++k) {
+                            const uint64_t bd =
+                                smem_desc_sw128(b_st + k * 16 * 128, kBK * 128, 1024);
+                            const uint32_t acc_in = (has_bias || (kb | k) != 0) ? 1u : 0u;
+#pragma unroll
+                            for (int h = 0; h < TM; ++h) {
+                                const uint64_t ad =
+                                    smem_desc_sw128(a_st + h * kAHalfBytes + k * 32, 16, 1024);
+                                tc_mma_bf16(d_tmem + (uint32_t)(h * BN), ad, bd, C::kIdesc,
+                                            acc_in);
+                            }
+                        }
                     }
                     tc_commit(empty_bar(s));
                     ++it;
@@ -568,6 +637,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             // Every MMA issued by this thread has completed once fin_bar fires.
             tc_commit(fin_bar);
             mbar_wait_drain(fin_bar, 0, a.status);
+        };
+        if (lane == 0) {
+            if (tm == 2)
+                mma(std::integral_constant<int, 2>{});
+            else
+                mma(std::integral_constant<int, 1>{});
         }
         __syncwarp();
     } else if (warp == kIndexWarp) {
@@ -583,15 +658,18 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!mbar_wait(tabempty_bar(buf), (uint32_t)(((lt >> 1) & 1) ^ 1), abort_flag,
                            a.status))
                 break;
-            const long long m0 = (long long)((int)w / n_tiles) * kBM;
-            const uint32_t tab_s = tab0 + (uint32_t)buf * tab_bytes;
+            const long long m_item = (long long)((int)w / n_tiles) * item_rows;
             unsigned err = 0;
+            for (int h = 0; h < tm; ++h) {
+            // half h: rows m0 .. m0 + 127, table entries (l, r) at tab_s + (l * kTabRows + r) * 4
+            const long long m0 = m_item + h * kBM;
+            const uint32_t tab_s = tab0 + (uint32_t)buf * tab_bytes + (uint32_t)(h * kBM) * 4u;
             if (a.mode == kRulebook) {
                 // Precomputed mapping: one coalesced pass over the tile's
                 // rulebook columns, entries checked against the input's rows
-                // (the first tile's table was filled before the loop).
+                // (the first tile's table may have been filled before the loop).
                 constexpr int kRbChunk = 12;
-                for (int l0 = 0; l0 < L && lt > 0; l0 += kRbChunk) {
+                for (int l0 = 0; l0 < L && !(lt == 0 && prefetched); l0 += kRbChunk) {
                     int e[4][kRbChunk];
 #pragma unroll
                     for (int i = 0; i < 4; ++i)
@@ -612,11 +690,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 if (ev < -1 || ev >= a.x_rows) err |= kErrIndex;
                                 else src = ev;
                             }
-                            sts_s32(tab_s + (uint32_t)((l0 + d) * kBM + lane + 32 * i) * 4u, src);
+                            sts_s32(tab_s + (uint32_t)((l0 + d) * kTabRows + lane + 32 * i) * 4u, src);
                         }
                 }
-                if (err) report(a.status, err);
-                mbar_arrive(tabfull_bar(buf));
                 continue;
             }
             int bb[4], vv[4];
@@ -698,10 +774,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                                         src = a.mode == kSparseDenseX ? dr[i][d] : jj;
                                 }
                             }
-                            sts_s32(tab_s + (uint32_t)((l0 + d) * kBM + lane + 32 * i) * 4u, src);
+                            sts_s32(tab_s + (uint32_t)((l0 + d) * kTabRows + lane + 32 * i) * 4u, src);
                         }
                 }
             }
+            }  // halves
             if (err) report(a.status, err);
             mbar_arrive(tabfull_bar(buf));
         }
@@ -709,6 +786,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ------------------------------------------------------------ epilogue
         const int ew = warp - kProducerWarps;  // == warp % 4: TMEM lanes 32*ew..+32
         __nv_bfloat16* __restrict__ y = static_cast<__nv_bfloat16*>(a.y);
+        // the role's whole loop for a half count fixed at compile time
+        auto epilogue = [&](auto tm_c) {
+        constexpr int TM = decltype(tm_c)::value;
         // Accumulator buffer acc is handed to the MMA warp holding the bias of
         // tile w in every row (the MMAs then accumulate onto it), so the bias
         // costs the epilogue nothing once the sums are ready.
@@ -723,9 +803,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                         const int col = n0 + cb * 32 + j;
                         r[j] = col < C_out ? __float_as_uint(__ldg(a.bias + col)) : 0u;
                     }
-                    tmem_st_32x32b_x32(tmem_base + ((uint32_t)(ew * 32) << 16) +
-                                           (uint32_t)(acc * BN + cb * 32),
-                                       r);
+                    for (int h = 0; h < TM; ++h)
+                        tmem_st_32x32b_x32(tmem_base + ((uint32_t)(ew * 32) << 16) +
+                                               (uint32_t)((acc * TM + h) * BN + cb * 32),
+                                           r);
                 }
                 tmem_st_wait();
             }
@@ -735,11 +816,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         release(0, blockIdx.x);
         release(1, blockIdx.x + (long long)gridDim.x);
         int lt = 0;
-        for (long long w = blockIdx.x; w < work_total; w += gridDim.x, ++lt) {
-            const long long m0 = (long long)((int)w / n_tiles) * kBM;
+        bool live = true;
+        for (long long w = blockIdx.x; w < work_total && live; w += gridDim.x, ++lt) {
+            const long long m_item = (long long)((int)w / n_tiles) * item_rows;
             const int n0 = ((int)w % n_tiles) * BN;  // w < 2^31
             const int acc = lt & 1;
             const uint32_t ph = (uint32_t)((lt >> 1) & 1);
+            for (int h = 0; h < TM; ++h) {
+            const long long m0 = m_item + h * kBM;
             // Everything that does not need the accumulator is loaded while
             // the main loop runs: this lane's row addresses (0 = not
             // written; the fused scatter's needs the row's coordinate).
@@ -774,13 +858,19 @@ __global__ void __launch_bounds__(kThreads, 1)
                 yk[k] = __shfl_sync(0xffffffffu, row_y, 8 * k + (lane >> 2));
                 dk[k] = __shfl_sync(0xffffffffu, row_d, 8 * k + (lane >> 2));
             }
-            if (!mbar_wait(tfull_bar(acc), ph, abort_flag, a.status)) break;
-            tc_fence_after();
+            if (h == 0) {
+                if (!mbar_wait(tfull_bar(acc), ph, abort_flag, a.status)) {
+                    live = false;
+                    break;
+                }
+                tc_fence_after();
+            }
             const uint32_t stage = epi0 + (uint32_t)ew * 2048u;
+            const uint32_t acc_col = (uint32_t)((acc * TM + h) * BN);
 #pragma unroll 1
             for (int cb = 0; cb < BN / 32; ++cb) {
                 uint32_t r[32];
-                tmem_ld_32x32b_x32(tmem_base + ((uint32_t)(ew * 32) << 16) + (uint32_t)(acc * BN + cb * 32),
+                tmem_ld_32x32b_x32(tmem_base + ((uint32_t)(ew * 32) << 16) + acc_col + (uint32_t)(cb * 32),
                                    r);
                 tmem_ld_wait();
                 const int col0 = n0 + cb * 32;
@@ -800,10 +890,16 @@ __global__ void __launch_bounds__(kThreads, 1)
                 else
                     epilogue_chunk<HC_ACT_NONE>(r, stage, lane, yk, dk, col0, C_out);
             }
-            release(acc, w + 2 * (long long)gridDim.x);  // the tile after next
+            }  // halves
+            if (!live) break;
+            release(acc, w + 2 * (long long)gridDim.x);  // the item after next
         }
+        };
+        if (tm == 2)
+            epilogue(std::integral_constant<int, 2>{});
+        else
+            epilogue(std::integral_constant<int, 1>{});
     }
-
     __syncthreads();
     if (warp == kMmaWarp) {
         tc_fence_after();

@@ -394,16 +394,16 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
 __device__ __forceinline__ bool mbar_wait_for(uint32_t bar, uint32_t parity,
                                               volatile int* abort_flag, unsigned* status,
                                               unsigned long long limit) {
-    unsigned long long t0 = globaltimer_ns();
-    for (uint32_t i = 1;; ++i) {
+    // try_wait itself may suspend the thread for a while, so the clock and
+    // the abort flag are read after every unsuccessful try
+    const unsigned long long t0 = globaltimer_ns();
+    for (;;) {
         if (mbar_try_wait(bar, parity)) return true;
-        if ((i & 63u) == 0) {
-            if (abort_flag && *abort_flag) return false;
-            if (globaltimer_ns() - t0 > limit) {
-                if (abort_flag) *abort_flag = 1;
-                report(status, kErrTimeout);
-                return false;
-            }
+        if (abort_flag && *abort_flag) return false;
+        if (globaltimer_ns() - t0 > limit) {
+            if (abort_flag) *abort_flag = 1;
+            report(status, kErrTimeout);
+            return false;
         }
     }
 }
