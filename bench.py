@@ -56,10 +56,12 @@ def parse_args():
                    help="skip the side measurements (density sweep, group norm, mask score, "
                         "backward)")
     p.add_argument("--extra", choices=["all", "sweep", "group_norm", "mask_score", "backward",
-                                       "kappa"],
+                                       "kappa", "configs", "stages"],
                    default="all", help="run only this side measurement")
     p.add_argument("--clocks-csv", default=None, help="also write the raw clock samples here")
     p.add_argument("--e2e-steps", type=int, default=30)
+    p.add_argument("--no-e2e", action="store_true",
+                   help="skip the end-to-end measurement (for targeted profiler captures)")
     return p.parse_args()
 
 
@@ -374,15 +376,56 @@ def run_ours(args, rank, world, local_rank):
         del s.dense
     torch.cuda.empty_cache()
 
-    e2e = measure_e2e(torch, hc, sets, w, spiral, Wt, bias, stream, dev, args.e2e_steps)
-    # whole-job end-to-end figure: rows of all ranks over the slowest rank's time
-    e2e_rows, e2e_ms = reduce_over_ranks(float(e2e.pop("rows")), e2e.pop("seconds") * 1e3, world,
-                                         dev)
-    e2e["value"] = e2e_rows / (e2e_ms * 1e-3)
-    e2e["ms_per_step"] = e2e_ms / e2e["steps"]
-    e2e["ranks"] = world
+    e2e = None
+    if not args.no_e2e:
+        e2e = measure_e2e(torch, hc, sets, w, spiral, Wt, bias, stream, dev, args.e2e_steps)
+        # whole-job end-to-end figure: rows of all ranks over the slowest rank's time
+        e2e_rows, e2e_ms = reduce_over_ranks(float(e2e.pop("rows")), e2e.pop("seconds") * 1e3,
+                                             world, dev)
+        e2e["value"] = e2e_rows / (e2e_ms * 1e-3)
+        e2e["ms_per_step"] = e2e_ms / e2e["steps"]
+        e2e["ranks"] = world
 
-    sweep = gnorm = mscore = bwd = kap = None
+    # Compaction alone (count pass + fused compaction and Eq. 4 mapping, and
+    # the plain compaction without the mapping) over the same rotation; the
+    # step is compaction + conv.
+    def compact_map(s):
+        hc.hc_mask_compact_rulebook(s.mask, spiral, hc.HC_LAYOUT_DENSE, s.coords, s.row_of,
+                                    s.offs, s.count, s.rb, stream)
+
+    def compact_only(s):
+        hc.hc_mask_compact(s.mask, s.coords, s.row_of, s.offs, s.count, stream)
+
+    comp_us = {}
+    for tag, fn in (("compact_map_us", compact_map), ("compact_us", compact_only)):
+        g_c = capture(fn, range(R))
+        with torch.cuda.stream(stream):
+            g_c.replay()
+            q0 = torch.cuda.Event(enable_timing=True)
+            q1 = torch.cuda.Event(enable_timing=True)
+            q0.record(stream)
+            for _ in range(reps):
+                g_c.replay()
+            q1.record(stream)
+        torch.cuda.synchronize(dev)
+        comp_us[tag] = q0.elapsed_time(q1) / (reps * R) * 1e3
+    # bytes a compaction must move: the mask (1 B per vertex), row_of (4 B per
+    # vertex), the coordinates (8 B per active row), the frame offsets
+    comp_bytes = B * V * (1 + 4) + 8 * mean_rows + 4 * (B + 1)
+    # with the mapping: + the slot-major rulebook entries of the active rows
+    map_bytes = comp_bytes + 4 * L * mean_rows
+    compaction = {
+        "compact_us": comp_us["compact_us"],
+        "compact_gbs": comp_bytes / (comp_us["compact_us"] * 1e-6) / 1e9,
+        "compact_map_us": comp_us["compact_map_us"],
+        "compact_map_gbs": map_bytes / (comp_us["compact_map_us"] * 1e-6) / 1e9,
+        "conv_us": conv_ms * 1e3,
+        "step_us": ms / K * 1e3,
+        "peak_gbs": pk["hbm_gbs"],
+        "note": "latency-bound: ~1.7 MB per call; the fraction of HBM bandwidth is not its bound",
+    }
+
+    sweep = gnorm = mscore = bwd = kap = cfgs = stg = None
     if not args.no_extras and rank == 0:
         want = lambda name: args.extra in ("all", name)  # noqa: E731
         if want("sweep"):
@@ -395,6 +438,10 @@ def run_ours(args, rank, world, local_rank):
             bwd = run_backward(torch, hc, sets[1], w, spiral, Wt, dev, stream)
         if want("kappa"):
             kap = run_kappa(torch, hc, dev, stream)
+        if want("configs"):
+            cfgs = run_configs(torch, hc, dev, stream)
+        if want("stages"):
+            stg = run_stages(torch, hc, sets[0], w, dev, stream)
 
     # Aggregate over ranks: rows summed, time = max over ranks.
     tot_rows, max_ms = reduce_over_ranks(float(rows_timed), ms, world, dev)
@@ -470,6 +517,11 @@ def run_ours(args, rank, world, local_rank):
         line["backward"] = bwd
     if kap is not None:
         line["kappa_inference"] = kap
+    if cfgs is not None:
+        line["configs"] = cfgs
+    if stg is not None:
+        line["stages"] = stg
+    line["compaction"] = compaction
     return line
 
 
@@ -970,6 +1022,171 @@ def run_kappa(torch, hc, dev, stream, K=10, kappa=3, density=0.1):
                      "linear head (compact rows throughout)"}
 
 
+def run_stages(torch, hc, s, w, dev, stream):
+    """The HBM-bound stages of the path on one input set of the bench layer,
+    each timed alone (CUDA-graph replays): the S' row gather (Eq. 2) from the
+    dense features, the scatter of the conv's compact rows back to the dense
+    tensor (Eq. 2 inverse) without and with the zero fill, and the
+    compaction (in the "compaction" block). Achieved GB/s = the bytes each
+    must move / time, against the measured HBM copy bandwidth."""
+    B, V = w.B, w.V
+    C_in = w.layers[0].C_in
+    C_out = w.layers[0].C_out
+    n = s.rows
+    pk = peaks()
+    rows_x = torch.empty((B * V, C_in), dtype=torch.bfloat16, device=dev)
+    dense = torch.empty((B, V, C_out), dtype=torch.bfloat16, device=dev)
+    with torch.cuda.stream(stream):
+        hc.hc_mask_compact(s.mask, s.coords, s.row_of, s.offs, s.count, stream)
+    cases = {
+        "gather_rows": (lambda: hc.hc_gather_rows(s.x, s.coords, s.count, 1, rows_x, stream),
+                        n * (2 * C_in * 2 + 8)),
+        "scatter": (lambda: hc.hc_scatter_dense(s.y, s.coords, None, s.count, B, V, 0, dense,
+                                                stream),
+                    n * (2 * C_out * 2 + 8)),
+        "scatter_zero_fill": (lambda: hc.hc_scatter_dense(s.y, s.coords, s.row_of, s.count, B, V,
+                                                          1, dense, stream),
+                              B * V * (C_out * 2 + 4) + n * C_out * 2),
+    }
+    out = {"workload": WORKLOAD, "active_rows": n, "peak_gbs": pk["hbm_gbs"]}
+    for name, (fn, nbytes) in cases.items():
+        us = _graph_time_us(torch, fn, stream, dev)
+        out[name] = {"us": us, "bytes": nbytes, "gbs": nbytes / (us * 1e-6) / 1e9,
+                     "hbm_frac": nbytes / (us * 1e-6) / 1e9 / pk["hbm_gbs"]}
+    st = hc.hc_get_device_status(stream)
+    if st != hc.HC_OK:
+        raise RuntimeError(f"device status {hc.STATUS_NAMES.get(st)} in the stage timings")
+    return out
+
+
+def _graph_time_us(torch, fn, stream, dev, reps=20):
+    """Mean time of fn over `reps` calls replayed from one CUDA graph (after
+    an eager call and one replay), CUDA events on the stream."""
+    with torch.cuda.stream(stream):
+        fn()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for _ in range(reps):
+                fn()
+        g.replay()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        g.replay()
+        e1.record(stream)
+    torch.cuda.synchronize(dev)
+    return e0.elapsed_time(e1) / reps * 1e3
+
+
+def _oracle_rows_per_s(w, threads, budget_s):
+    """The oracle's whole stack (compaction, every layer on the compact rows)
+    on the first k frames of the workload, k chosen so that the run takes
+    about budget_s; returns (active rows per second, frames, rows)."""
+    import oracle
+
+    def run(k):
+        t0 = time.perf_counter()
+        _, _, _, n, _ = oracle.encoder(w.x[:k], w.masks[0][:k], w.spiral, w.layers,
+                                       n_threads=threads)
+        return time.perf_counter() - t0, n
+
+    t1, n1 = run(1)
+    k = max(1, min(w.B, int(budget_s / max(t1, 1e-4))))
+    t, n = (t1, n1) if k == 1 else run(k)
+    return n / t, k, n
+
+
+def run_configs(torch, hc, dev, stream, cpu_budget_s=3.0):
+    """The other workloads of the scope (655-vertex mesh): the single fp32
+    layer, the 4-layer bf16 encoder + 64 -> 42 head, and the 256-frame motion
+    encoder + 64 -> 1 head. Each runs as the paper's network would: compact
+    once (compaction + Eq. 4 mapping in the compact layout), gather S'
+    (Eq. 2), every layer on the compact rows, one CUDA graph; against the
+    same network run densely on every vertex, and against the oracle on 1
+    thread and on every host core (bounded frame samples)."""
+    from paper_2608_09388_gb300 import inputs
+    pk = peaks()
+    props = torch.cuda.get_device_properties(dev)
+    # fp32 FFMA peak: SMs x 128 lanes x 2 flops at the maximum SM clock
+    ffma_tflops = props.multi_processor_count * 128 * 2 * 2.07e9 / 1e12
+    cores = len(os.sched_getaffinity(0))
+    res = {}
+    for name in ("layer655_f32", "encoder655_bf16", "motion655_bf16"):
+        w = inputs.make_workload(name)
+        B, V, L = w.B, w.V, w.L
+
+        def T(a):
+            if a.dtype == np.uint16:
+                return torch.from_numpy(a.view(np.int16)).view(torch.bfloat16).to(dev)
+            return torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+
+        dt = torch.float32 if w.dtype == "f32" else torch.bfloat16
+        mask, x, sp = T(w.masks[0]), T(w.x), T(w.spiral)
+        Ws = [T(ly.W) for ly in w.layers]
+        bs = [T(ly.b) for ly in w.layers]
+        coords = torch.empty((B * V, 2), dtype=torch.int32, device=dev)
+        row_of = torch.empty((B, V), dtype=torch.int32, device=dev)
+        offs = torch.empty(B + 1, dtype=torch.int32, device=dev)
+        count = torch.empty(1, dtype=torch.int32, device=dev)
+        rb = torch.empty((L, B * V), dtype=torch.int32, device=dev)
+        hs = [torch.empty((B * V, ly.C_in), dtype=dt, device=dev) for ly in w.layers]
+        out = torch.empty((B * V, w.layers[-1].C_out), dtype=dt, device=dev)
+        dense_h = [torch.empty((B, V, ly.C_out), dtype=dt, device=dev) for ly in w.layers]
+        full = torch.tensor([B * V], dtype=torch.int32, device=dev)
+
+        def sparse():
+            hc.hc_mask_compact_rulebook(mask, sp, hc.HC_LAYOUT_COMPACT, coords, row_of, offs,
+                                        count, rb, stream)
+            hc.hc_gather_rows(x, coords, count, 1, hs[0], stream)
+            for i, ly in enumerate(w.layers):
+                dst = hs[i + 1] if i + 1 < len(w.layers) else out
+                if ly.kind == "conv":
+                    hc.hc_sparse_conv_rulebook_fwd(hs[i], rb, count, Ws[i], bs[i], ly.act, dst,
+                                                   stream=stream)
+                else:
+                    hc.hc_sparse_linear_fwd(hs[i], count, Ws[i], bs[i], ly.act, dst, stream)
+
+        def dense():
+            h = x
+            for i, ly in enumerate(w.layers):
+                if ly.kind == "conv":
+                    hc.hc_spiral_conv_fwd(h, sp, Ws[i], bs[i], ly.act, dense_h[i], stream)
+                else:
+                    hc.hc_sparse_linear_fwd(h.view(B * V, -1), full, Ws[i], bs[i], ly.act,
+                                            dense_h[i].view(B * V, -1), stream)
+                h = dense_h[i]
+
+        t_sparse = _graph_time_us(torch, sparse, stream, dev)
+        t_dense = _graph_time_us(torch, dense, stream, dev)
+        st = hc.hc_get_device_status(stream)
+        if st != hc.HC_OK:
+            raise RuntimeError(f"device status {hc.STATUS_NAMES.get(st)} in {name}")
+        n = int(count.item())
+        flops = sum(2.0 * (L if ly.kind == "conv" else 1) * ly.C_in * ly.C_out * n
+                    for ly in w.layers)
+        peak = pk["bf16_tflops"] if w.dtype == "bf16" else ffma_tflops
+        achieved = flops / (t_sparse * 1e-6) / 1e12
+        o1, k1, n1 = _oracle_rows_per_s(w, 1, cpu_budget_s)
+        on, kn, nn = _oracle_rows_per_s(w, cores, cpu_budget_s)
+        res[name] = {
+            "B": B, "V": V, "L": L, "dtype": w.dtype, "active_rows": n,
+            "layers": " -> ".join([str(w.layers[0].C_in)] + [str(ly.C_out) for ly in w.layers]),
+            "us": t_sparse, "rows_per_s": n / (t_sparse * 1e-6),
+            "gflops": flops / (t_sparse * 1e-6) / 1e9,
+            "roofline": {"bound": "tensor" if w.dtype == "bf16" else "alu", "achieved": achieved,
+                         "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
+                         "peak_source": "measured bf16 burst" if w.dtype == "bf16" else
+                         "FFMA: SMs x 128 x 2 x 2.07 GHz",
+                         "note": "latency-bound: a few thousand rows per launch"},
+            "dense_us": t_dense, "speedup_vs_dense": t_dense / t_sparse,
+            "oracle_1_thread": {"rows_per_s": o1, "frames": k1, "rows": n1, "cores": 1},
+            "oracle_all_cores": {"rows_per_s": on, "frames": kn, "rows": nn, "cores": cores},
+            "chain": "compaction + Eq. 4 mapping + S' gather + every layer on compact rows "
+                     "(one CUDA graph)",
+        }
+    return res
+
+
 def cpu_baseline(w, budget_s=20.0):
     """The CPU oracle as it stands on this host's cores: compaction, sparse
     conv and scatter of batch 0 of the workload (all of its active rows when
@@ -995,9 +1212,25 @@ def cpu_baseline(w, budget_s=20.0):
     oracle.scatter_dense(y, coords[:k], w.B, w.V, False)
     t_scatter = time.perf_counter() - t0
     secs = t_compact * k / max(n, 1) + t_conv + t_scatter
+    # the same on one thread, on a prefix of the rows sized to ~budget_s / 4
+    t0 = time.perf_counter()
+    oracle.sparse_spiral_conv(w.x, oracle.LAYOUT_DENSE, coords, row_of, w.spiral, ly.W, ly.b,
+                              ly.act, rows=probe[:64], n_threads=1)
+    per_row1 = (time.perf_counter() - t0) / max(1, min(64, len(probe)))
+    k1 = max(64, min(n, int(budget_s / 4 / max(per_row1, 1e-7))))
+    rows1 = np.arange(k1, dtype=np.int64)
+    t0 = time.perf_counter()
+    _, y1 = oracle.sparse_spiral_conv(w.x, oracle.LAYOUT_DENSE, coords, row_of, w.spiral, ly.W,
+                                      ly.b, ly.act, rows=rows1, n_threads=1)
+    t_conv1 = time.perf_counter() - t0
+    t0 = time.perf_counter()
+    oracle.scatter_dense(y1, coords[:k1], w.B, w.V, False)
+    secs1 = t_compact * k1 / max(n, 1) + t_conv1 + time.perf_counter() - t0
     return {"value": k / secs, "unit": "rows/s", "cores": cores, "kind": "oracle",
             "sample": f"batch 0 of {WORKLOAD}: compaction, sparse conv and scatter of "
-                      f"{k} of its {n} active rows (fp64 C oracle, OpenMP over rows)"}
+                      f"{k} of its {n} active rows (fp64 C oracle, OpenMP over rows)",
+            "single_thread": {"value": k1 / secs1, "unit": "rows/s", "cores": 1,
+                              "sample": f"the first {k1} active rows of batch 0"}}
 
 
 # ----------------------------------------------------------------- reference arm

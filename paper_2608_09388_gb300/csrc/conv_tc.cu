@@ -60,7 +60,6 @@
 
 #include <cstring>
 #include <mutex>
-#include <type_traits>
 
 #include "hc_internal.cuh"
 
@@ -69,10 +68,7 @@ namespace {
 
 constexpr int kBM = 128;  // rows per tile half = TMEM lanes
 constexpr int kBK = 64;   // bf16 per 128-byte smem row
-constexpr int kHalves = 2;  // 128-row halves per work item at most (both share each W stage)
-constexpr int kTabRows = kHalves * kBM;  // rows of a tap table
-constexpr int kAHalfBytes = kBM * kBK * 2;
-constexpr int kAStageBytes = kHalves * kAHalfBytes;
+constexpr int kAHalfBytes = kBM * kBK * 2;  // A of one 128-row half for one k-block
 constexpr int kProducerWarps = 4;
 constexpr int kEpilogueWarps = 4;
 constexpr int kMmaWarp = kProducerWarps + kEpilogueWarps;
@@ -82,25 +78,27 @@ constexpr int kThreads = (kWeightWarp + 1) * 32;
 constexpr int kTabChunk = 6;  // spiral slots resolved per pass of the index warp
 constexpr size_t kSmemLimit = 227 * 1024;  // opt-in dynamic shared memory per CTA
 
-template <int BN>
+// BN output channels per tile; TM 128-row halves per work item, all sharing
+// every W stage.
+template <int BN, int TM>
 struct Cfg {
     static_assert(BN == 64 || BN == 128, "tile widths");
+    static_assert(TM == 1 || TM == 2, "halves per item");
+    static constexpr int kTabRows = TM * kBM;  // rows of a tap table
+    static constexpr int kAStageBytes = TM * kAHalfBytes;
     static constexpr int kBStageBytes = kBK * BN * 2;
     // Pipeline depth: as many stages as fit next to the tap tables (which
     // grow with L), between kMinStages and kMaxStages.
-    // (stages of two-half items; one-half items cut the same bytes into
-    // more, smaller stages, at most kRing)
-    static constexpr int kMaxStages = BN == 64 ? 5 : 4;
+    static constexpr int kMaxStages = TM == 2 ? (BN == 64 ? 5 : 4) : (BN == 64 ? 8 : 6);
     static constexpr int kMinStages = 2;
-    static constexpr int kRing = BN == 64 ? 8 : 6;
-    // two accumulator buffers, each one BN-column accumulator per half
-    static constexpr int kTmemCols = 2 * kHalves * BN;
+    // two accumulator sets, each one BN-column accumulator per half
+    static constexpr int kTmemCols = 2 * TM * BN;
     // Instruction descriptor, kind::f16: D fp32 (bit 4), A bf16 (bits 7-9 = 1),
     // B bf16 (bits 10-12 = 1), A K-major (bit 15 = 0), B MN-major (bit 16 = 1),
     // N >> 3 at bits 17-22, M >> 4 at bits 24-28.
     static constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | (1u << 16) |
                                        ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(kBM >> 4) << 24);
-    static constexpr int kBarBytes = 8 * (2 * kRing + 9);
+    static constexpr int kBarBytes = 8 * (2 * kMaxStages + 9);
     // barriers, then 16 bytes (TMEM address, abort flag), then the two tap
     // tables ([L][kTabRows] int32 each) at a 128-byte boundary.
     static constexpr int kTabOffset = (kBarBytes + 16 + 127) / 128 * 128;
@@ -326,10 +324,11 @@ __device__ __forceinline__ void gn_stats_chunk(const ConvArgs& a, const uint32_t
     }
 }
 
-template <int BN>
+template <int BN, int TM>
 __global__ void __launch_bounds__(kThreads, 1)
     conv_tc_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_w) {
-    using C = Cfg<BN>;
+    using C = Cfg<BN, TM>;
+    constexpr int kTabRows = C::kTabRows;
     // "full": one cp.async completion arrival per producer thread, plus the
     // expect-tx arrival of the weight loader.
     constexpr int kStageArrivals = kProducerWarps * 32 + 1;
@@ -338,8 +337,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t base = (raw + 1023u) & ~1023u;
     uint8_t* const base_ptr = smem_raw + (base - raw);
     const uint32_t sA = base;  // the stage ring (a.stages two-half stages)
-    const uint32_t ring_bytes = (uint32_t)a.stages * (kAStageBytes + C::kBStageBytes);
-    const uint32_t sBar = sA + ring_bytes;
+    const int nst = a.stages;
+    constexpr uint32_t kStageBytes = C::kAStageBytes + C::kBStageBytes;
+    // stage st: TM halves of A (16 KB each), then the W slice (1024-byte aligned)
+    auto a_stage = [&](int st) { return sA + (uint32_t)st * kStageBytes; };
+    auto b_stage = [&](int st) { return sA + (uint32_t)st * kStageBytes + (uint32_t)C::kAStageBytes; };
+    const uint32_t sBar = sA + (uint32_t)nst * kStageBytes;
     uint8_t* const misc = base_ptr + (sBar - base) + C::kBarBytes;
     volatile uint32_t* const tmem_holder = reinterpret_cast<volatile uint32_t*>(misc);
     volatile int* const abort_flag = reinterpret_cast<volatile int*>(misc + 4);
@@ -349,17 +352,17 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t epi0 = tab0 + 2u * (uint32_t)(kTabRows * a.L) * 4u;  // epilogue staging
 
     auto full_bar = [&](int s) { return sBar + 8u * s; };
-    auto empty_bar = [&](int s) { return sBar + 8u * (C::kRing + s); };
-    auto tfull_bar = [&](int i) { return sBar + 8u * (2 * C::kRing + i); };
-    auto tempty_bar = [&](int i) { return sBar + 8u * (2 * C::kRing + 2 + i); };
-    const uint32_t fin_bar = sBar + 8u * (2 * C::kRing + 4);
-    auto tabfull_bar = [&](int i) { return sBar + 8u * (2 * C::kRing + 5 + i); };
-    auto tabempty_bar = [&](int i) { return sBar + 8u * (2 * C::kRing + 7 + i); };
+    auto empty_bar = [&](int s) { return sBar + 8u * (C::kMaxStages + s); };
+    auto tfull_bar = [&](int i) { return sBar + 8u * (2 * C::kMaxStages + i); };
+    auto tempty_bar = [&](int i) { return sBar + 8u * (2 * C::kMaxStages + 2 + i); };
+    const uint32_t fin_bar = sBar + 8u * (2 * C::kMaxStages + 4);
+    auto tabfull_bar = [&](int i) { return sBar + 8u * (2 * C::kMaxStages + 5 + i); };
+    auto tabempty_bar = [&](int i) { return sBar + 8u * (2 * C::kMaxStages + 7 + i); };
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < C::kRing; ++s) {
+        for (int s = 0; s < C::kMaxStages; ++s) {
             mbar_init(full_bar(s), kStageArrivals);
             mbar_init(empty_bar(s), 1);
         }
@@ -389,13 +392,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     pdl_wait();
     pdl_trigger();
 
-    // Rulebook mode: the index warp copies the entries of its first 128-row
-    // tile into tap table 0 (cp.async, no registers held) before the row
+    // Rulebook mode (one-half items): the index warp copies its first tile's
+    // entries into tap table 0 (cp.async, no registers held) before the row
     // count arrives (rows clamped to the capacity, always valid memory), so
-    // the two L2 round trips overlap instead of queueing. The copy is used
-    // when the count gives one-half work items (few rows, where this latency
-    // matters); with two-half items the loop builds the table instead.
-    const bool prefetch = warp == kIndexWarp && a.mode == kRulebook;
+    // the two L2 round trips overlap instead of queueing.
+    const bool prefetch = TM == 1 && warp == kIndexWarp && a.mode == kRulebook;
     if (prefetch) {
         const long long m0p = (blockIdx.x / ((a.C_out + BN - 1) / BN)) * (long long)kBM;
         for (int d = 0; d < a.L; ++d)
@@ -409,29 +410,15 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     const long long rows = active_rows(a);
     const int n_tiles = (a.C_out + BN - 1) / BN;
-    // Work item: tm 128-row halves sharing every W stage. Two halves (half
-    // the weight traffic and per-stage overhead per MMA) when that still
-    // gives every CTA two items; one otherwise (few rows: the launch is
-    // latency-bound, and larger items would only deepen the last wave).
-    const long long tiles128 = (rows + kBM - 1) / kBM;
-    const int tm = (tiles128 + 1) / 2 * n_tiles >= 2ll * gridDim.x ? 2 : 1;
-    const int item_rows = tm * kBM;
+    constexpr int item_rows = TM * kBM;
     const long long m_items = (rows + item_rows - 1) / item_rows;
     const long long work_total = m_items * n_tiles;
     const int num_kb = (a.K + kBK - 1) / kBK;
     const int L = a.L, C_in = a.C_in, C_out = a.C_out, K = a.K;
     const uint32_t tab_bytes = (uint32_t)(kTabRows * L) * 4u;
-    const bool prefetched = prefetch && tm == 1;
-    // Stage s: tm halves of A (16 KB each), then the W slice; as many stages
-    // as the ring holds (kRing at most). 16 KB multiples keep every operand
-    // 1024-byte aligned.
-    const uint32_t stage_bytes = (uint32_t)(tm * kAHalfBytes + C::kBStageBytes);
-    const int nst_fit = (int)(ring_bytes / stage_bytes);
-    const int nst = nst_fit < C::kRing ? nst_fit : C::kRing;
-    auto a_stage = [&](int st) { return sA + (uint32_t)st * stage_bytes; };
-    auto b_stage = [&](int st) { return sA + (uint32_t)st * stage_bytes + (uint32_t)(tm * kAHalfBytes); };
-    if (prefetch) cp_async_wait_all();
+    const bool prefetched = prefetch;
     if (prefetched) {
+        cp_async_wait_all();
         // the first tap table (buffer 0, not yet waited on by anyone): the
         // copied entries checked against the input's rows and masked by the
         // row count
@@ -461,10 +448,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         const __nv_bfloat16* __restrict__ x = static_cast<const __nv_bfloat16*>(a.x);
         const int t = threadIdx.x;  // 0..127
         const int q = t & 7;        // 16-byte chunk of the 128-byte row
-        // The role's whole loop for a half count fixed at compile time (one
-        // copy of the loop is hot per launch).
-        auto producer = [&](auto tm_c) {
-        constexpr int TM = decltype(tm_c)::value;
         int st_s = 0;        // stage of the current iteration (it % stages)
         uint32_t st_ph = 0;  // its phase parity ((it / stages) & 1)
         int lt = 0;
@@ -526,11 +509,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (ok) mbar_arrive(tabempty_bar(buf));
         }
         cp_async_wait_all();
-        };
-        if (tm == 2)
-            producer(std::integral_constant<int, 2>{});
-        else
-            producer(std::integral_constant<int, 1>{});
     } else if (warp == kWeightWarp) {
         // ------------------------------------------------------------ weight loader
         if (lane == 0) {
@@ -576,9 +554,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
     } else if (warp == kMmaWarp) {
         // ------------------------------------------------------------ MMA issuer
-        // the role's whole loop for a half count fixed at compile time
-        auto mma = [&](auto tm_c) {
-            constexpr int TM = decltype(tm_c)::value;
+        if (lane == 0) {
             long long it = 0;
             int st_s = 0;        // stage of iteration it (it % stages)
             uint32_t st_ph = 0;  // its phase parity ((it / stages) & 1)
@@ -637,12 +613,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             // Every MMA issued by this thread has completed once fin_bar fires.
             tc_commit(fin_bar);
             mbar_wait_drain(fin_bar, 0, a.status);
-        };
-        if (lane == 0) {
-            if (tm == 2)
-                mma(std::integral_constant<int, 2>{});
-            else
-                mma(std::integral_constant<int, 1>{});
         }
         __syncwarp();
     } else if (warp == kIndexWarp) {
@@ -660,7 +630,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 break;
             const long long m_item = (long long)((int)w / n_tiles) * item_rows;
             unsigned err = 0;
-            for (int h = 0; h < tm; ++h) {
+            for (int h = 0; h < TM; ++h) {
             // half h: rows m0 .. m0 + 127, table entries (l, r) at tab_s + (l * kTabRows + r) * 4
             const long long m0 = m_item + h * kBM;
             const uint32_t tab_s = tab0 + (uint32_t)buf * tab_bytes + (uint32_t)(h * kBM) * 4u;
@@ -786,9 +756,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ------------------------------------------------------------ epilogue
         const int ew = warp - kProducerWarps;  // == warp % 4: TMEM lanes 32*ew..+32
         __nv_bfloat16* __restrict__ y = static_cast<__nv_bfloat16*>(a.y);
-        // the role's whole loop for a half count fixed at compile time
-        auto epilogue = [&](auto tm_c) {
-        constexpr int TM = decltype(tm_c)::value;
+        {
         // Accumulator buffer acc is handed to the MMA warp holding the bias of
         // tile w in every row (the MMAs then accumulate onto it), so the bias
         // costs the epilogue nothing once the sums are ready.
@@ -894,11 +862,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!live) break;
             release(acc, w + 2 * (long long)gridDim.x);  // the item after next
         }
-        };
-        if (tm == 2)
-            epilogue(std::integral_constant<int, 2>{});
-        else
-            epilogue(std::integral_constant<int, 1>{});
+        }
     }
     __syncthreads();
     if (warp == kMmaWarp) {
@@ -969,12 +933,12 @@ hc_status encode_w3d(CUtensorMap* m, const void* base, long long K, long long C_
     return HC_OK;
 }
 
-template <int BN>
+template <int BN, int TM>
 hc_status launch_bn(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s) {
-    using C = Cfg<BN>;
+    using C = Cfg<BN, TM>;
     static bool attr_set[64] = {};
     if (!attr_set[ctx->device]) {
-        hc_status st = check_cuda(cudaFuncSetAttribute(conv_tc_kernel<BN>,
+        hc_status st = check_cuda(cudaFuncSetAttribute(conv_tc_kernel<BN, TM>,
                                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                        (int)kSmemLimit),
                                   "cudaFuncSetAttribute(conv_tc_kernel)");
@@ -996,11 +960,11 @@ hc_status launch_bn(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s) {
         st = encode_2d(&tw, a.W, a.K, a.C_out, 64, kBK);
     if (st != HC_OK) return st;
     const long long n_tiles = (a.C_out + BN - 1) / BN;
-    const long long cap_work = (a.capacity + kBM - 1) / kBM * n_tiles;
+    const long long cap_work = (a.capacity + TM * kBM - 1) / (TM * kBM) * n_tiles;
     long long grid = cap_work < ctx->num_sms ? cap_work : ctx->num_sms;
     if (grid < 1) grid = 1;
     ka.stages = C::stages_for(a.L);
-    return launch_pdl(conv_tc_kernel<BN>, dim3((unsigned)grid), dim3(kThreads),
+    return launch_pdl(conv_tc_kernel<BN, TM>, dim3((unsigned)grid), dim3(kThreads),
                       C::smem_bytes(a.L, ka.stages), s, "conv_tc_kernel", ka, tw);
 }
 
@@ -1020,8 +984,17 @@ int conv_tc_tile_n(const ConvArgs& a) {
 }
 
 hc_status launch_conv_tc(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s) {
-    if (conv_tc_tile_n(a) == 64) return launch_bn<64>(ctx, a, s);
-    return launch_bn<128>(ctx, a, s);
+    // Two-half items when the row count is known on the host (the dense
+    // layer) and fills every SM with at least two of them: they halve the
+    // weight traffic and per-stage overhead per MMA. The sparse calls' row
+    // count lives on the device, and the two-half code paths compiled into
+    // the same kernel cost the small layers ~1 us (instruction fetch), so
+    // they run one-half items.
+    const long long n_tiles = (a.C_out + 127) / 128;
+    const bool two = a.mode == kDense && (a.capacity + 2 * kBM - 1) / (2 * kBM) * n_tiles >=
+                                             2ll * ctx->num_sms;
+    if (conv_tc_tile_n(a) == 64) return launch_bn<64, 1>(ctx, a, s);
+    return two ? launch_bn<128, 2>(ctx, a, s) : launch_bn<128, 1>(ctx, a, s);
 }
 
 }  // namespace hc
