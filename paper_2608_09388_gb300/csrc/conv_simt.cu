@@ -5,10 +5,15 @@
 // multiple of 8, e.g. a 45-channel input or a 42- or 1-wide output head).
 //
 // Each CTA owns a 64-row x 64-column output tile and walks K = L*C_in in
-// steps of 16: the A tile is gathered through the per-tile table of source
-// rows (idx() of Eq. 4: -1 when the tap is absent), the W tile is read
-// directly, and each thread accumulates a 4x4 block. The grid is persistent
-// over row tiles because the row count N' is only known on the device.
+// chunks of KC (128 when K <= 256, else 64): the A chunk is gathered through the per-tile table of source
+// rows (idx() of Eq. 4: -1 when the tap is absent) and the W chunk read
+// directly, every load of a chunk issued before any is used (one dependent
+// round trip per KC of K rather than per 16: the small layers this kernel
+// serves are latency-bound; deeper layers take the smaller chunk, whose
+// registers and shared memory let more CTAs share an SM); each thread then
+// accumulates a 4x4 block. The
+// grid is persistent over row tiles because the row count N' is only known on
+// the device.
 #include <cuda_bf16.h>
 
 #include "hc_internal.cuh"
@@ -18,8 +23,14 @@ namespace {
 
 constexpr int kBM = 64;
 constexpr int kBN = 64;
-constexpr int kBK = 16;
 constexpr int kThreads = 256;
+constexpr int kAPitch = kBM + 4;  // floats per As row (16-byte aligned rows)
+
+// Shared memory of a chunk depth: As [KC][kAPitch] and Bs [KC][kBN] floats.
+template <int KC>
+constexpr size_t chunk_smem_bytes() {
+    return sizeof(float) * (size_t)(KC * kAPitch + KC * kBN);
+}
 
 template <typename T>
 __device__ __forceinline__ float to_float(T v);
@@ -42,11 +53,19 @@ __device__ __forceinline__ __nv_bfloat16 from_float<__nv_bfloat16>(float v) {
     return __float2bfloat16_rn(v);
 }
 
-template <typename T>
+template <typename T, int kKC>
 __global__ void __launch_bounds__(kThreads) conv_simt_kernel(const ConvArgs a) {
-    __shared__ __align__(16) float As[kBK][kBM + 4];
-    __shared__ __align__(16) float Bs[kBK][kBN];
-    extern __shared__ int src_tab[];  // [kBM][L]
+    constexpr int kAsFloats = kKC * kAPitch;
+    constexpr int kBsFloats = kKC * kBN;
+    // per thread per chunk: A rows tid/kKC + (256/kKC) i, B k-rows tid/64 + 4i
+    constexpr int kAPer = kBM * kKC / kThreads;
+    constexpr int kBPer = kKC * kBN / kThreads;
+    constexpr int kAStep = kThreads / kKC;
+    // dynamic: As [kKC][kAPitch] float, Bs [kKC][kBN] float, src_tab [kBM][L] int
+    extern __shared__ __align__(16) float smem_f[];
+    float* const As = smem_f;
+    float* const Bs = smem_f + kAsFloats;
+    int* const src_tab = reinterpret_cast<int*>(smem_f + kAsFloats + kBsFloats);
 
     const T* __restrict__ x = static_cast<const T*>(a.x);
     const T* __restrict__ W = static_cast<const T*>(a.W);
@@ -130,28 +149,39 @@ __global__ void __launch_bounds__(kThreads) conv_simt_kernel(const ConvArgs a) {
 #pragma unroll
             for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
 
-        for (int k0 = 0; k0 < K; k0 += kBK) {
-            for (int e = tid; e < kBM * kBK; e += kThreads) {
-                const int r = e / kBK, kk = e - r * kBK;
-                const int k = k0 + kk;
-                float val = 0.f;
-                if (k < K) {
-                    const int l = k / C_in, c = k - l * C_in;
-                    const int s = src_tab[r * L + l];
-                    if (s >= 0) val = to_float(x[(long long)s * C_in + c]);
-                }
-                As[kk][r] = val;
-            }
-            for (int e = tid; e < kBK * kBN; e += kThreads) {
-                const int kk = e / kBN, o = e - kk * kBN;
-                const int k = k0 + kk, col = n0 + o;
-                Bs[kk][o] = (k < K && col < C_out) ? to_float(W[(long long)k * C_out + col]) : 0.f;
-            }
-            __syncthreads();
+        // this thread's A column of every chunk (k = k0 + ka) and B column o
+        const int ka = tid & (kKC - 1), ra = tid / kKC;
+        const int ob = tid & (kBN - 1), kbr = tid >> 6;
+        for (int k0 = 0; k0 < K; k0 += kKC) {
+            const int k = k0 + ka;
+            const bool kin = k < K;
+            const int l = kin ? k / C_in : 0, c = kin ? k - l * C_in : 0;
+            float av_[kAPer], bv_[kBPer];
+            // every load of the chunk first ...
 #pragma unroll
-            for (int kk = 0; kk < kBK; ++kk) {
-                const float4 av = *reinterpret_cast<const float4*>(&As[kk][ty * 4]);
-                const float4 bv = *reinterpret_cast<const float4*>(&Bs[kk][tx * 4]);
+            for (int i = 0; i < kAPer; ++i) {
+                const int r = ra + kAStep * i;
+                const int s = kin ? src_tab[r * L + l] : -1;
+                av_[i] = s >= 0 ? to_float(x[(long long)s * C_in + c]) : 0.f;
+            }
+#pragma unroll
+            for (int i = 0; i < kBPer; ++i) {
+                const int kk = kbr + 4 * i, col = n0 + ob;
+                bv_[i] = (k0 + kk < K && col < C_out)
+                             ? to_float(W[(long long)(k0 + kk) * C_out + col])
+                             : 0.f;
+            }
+            // ... then the stores to shared memory
+#pragma unroll
+            for (int i = 0; i < kAPer; ++i) As[ka * kAPitch + ra + kAStep * i] = av_[i];
+#pragma unroll
+            for (int i = 0; i < kBPer; ++i) Bs[(kbr + 4 * i) * kBN + ob] = bv_[i];
+            __syncthreads();
+            const int kn = K - k0 < kKC ? K - k0 : kKC;
+#pragma unroll 16
+            for (int kk = 0; kk < kn; ++kk) {
+                const float4 av = *reinterpret_cast<const float4*>(&As[kk * kAPitch + ty * 4]);
+                const float4 bv = *reinterpret_cast<const float4*>(&Bs[kk * kBN + tx * 4]);
                 const float ar[4] = {av.x, av.y, av.z, av.w};
                 const float br[4] = {bv.x, bv.y, bv.z, bv.w};
 #pragma unroll
@@ -194,11 +224,37 @@ hc_status launch_conv_simt(const DeviceCtx* ctx, const ConvArgs& a, hc_dtype dt,
     long long gx = cap_tiles < (long long)ctx->num_sms * 8 ? cap_tiles : (long long)ctx->num_sms * 8;
     if (gx < 1) gx = 1;
     dim3 grid((unsigned)gx, (unsigned)((a.C_out + kBN - 1) / kBN));
-    size_t smem = sizeof(int) * (size_t)kBM * a.L;
-    if (dt == HC_F32)
-        return launch_pdl(conv_simt_kernel<float>, grid, dim3(kThreads), smem, s,
+    const size_t tab = sizeof(int) * (size_t)kBM * a.L;
+    static bool attr_set[64] = {};
+    if (!attr_set[ctx->device]) {
+        hc_status st = HC_OK;
+        auto allow = [&](auto kernel, size_t bytes) {
+            if (st == HC_OK)
+                st = check_cuda(cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                     (int)bytes),
+                                "cudaFuncSetAttribute(conv_simt_kernel)");
+        };
+        const size_t tab_max = sizeof(int) * (size_t)kBM * HC_MAX_SPIRAL;
+        allow(conv_simt_kernel<float, 128>, chunk_smem_bytes<128>() + tab_max);
+        allow(conv_simt_kernel<__nv_bfloat16, 128>, chunk_smem_bytes<128>() + tab_max);
+        allow(conv_simt_kernel<float, 64>, chunk_smem_bytes<64>() + tab_max);
+        allow(conv_simt_kernel<__nv_bfloat16, 64>, chunk_smem_bytes<64>() + tab_max);
+        if (st != HC_OK) return st;
+        attr_set[ctx->device] = true;
+    }
+    if (a.K <= 256) {
+        const size_t smem = chunk_smem_bytes<128>() + tab;
+        if (dt == HC_F32)
+            return launch_pdl(conv_simt_kernel<float, 128>, grid, dim3(kThreads), smem, s,
+                              "conv_simt_kernel", a);
+        return launch_pdl(conv_simt_kernel<__nv_bfloat16, 128>, grid, dim3(kThreads), smem, s,
                           "conv_simt_kernel", a);
-    return launch_pdl(conv_simt_kernel<__nv_bfloat16>, grid, dim3(kThreads), smem, s,
+    }
+    const size_t smem = chunk_smem_bytes<64>() + tab;
+    if (dt == HC_F32)
+        return launch_pdl(conv_simt_kernel<float, 64>, grid, dim3(kThreads), smem, s,
+                          "conv_simt_kernel", a);
+    return launch_pdl(conv_simt_kernel<__nv_bfloat16, 64>, grid, dim3(kThreads), smem, s,
                       "conv_simt_kernel", a);
 }
 

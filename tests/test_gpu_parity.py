@@ -407,6 +407,14 @@ def test_rulebook_entry_out_of_range_is_reported():
     y = torch.empty((200, 64), dtype=torch.bfloat16, device="cuda")
     hc.hc_sparse_conv_rulebook_fwd(to_torch(x), rb, count, to_torch(W), to_torch(b), 1, y)
     assert hc.hc_get_device_status() == hc.HC_ERR_INVALID_INDEX
+    # the bad entries contribute nothing: the same as absent taps
+    rb[2, 5] = -1
+    rb[1, 7] = -1
+    y_abs = torch.empty_like(y)
+    hc.hc_sparse_conv_rulebook_fwd(to_torch(x), rb, count, to_torch(W), to_torch(b), 1, y_abs)
+    assert hc.hc_get_device_status() == hc.HC_OK
+    n = int(count.item())
+    assert torch.equal(y[:n], y_abs[:n])
 
 
 # ------------------------------------------------------------------ dense conv
