@@ -681,11 +681,9 @@ def measure_e2e(torch, hc, sets, w, spiral, Wt, bias, stream, dev, steps):
 def run_sweep(torch, hc, dev, stream):
     """Mask-density sweep at V = 10475, L = 9, B = 64, 128 -> 128 channels:
     sparse conv (compaction and Eq. 4 mapping done beforehand) against the
-    dense layer, unordered and in the row order of hc_conv_rulebook_order
-    (timed apart: it is computed once per mask, like the mapping). The
-    tensor fractions count the MMA work issued (tensor_frac: the hardware
-    efficiency), the present taps' work (Eq. 5's sum), and for the unordered
-    call every tap of every row."""
+    dense layer. tensor_frac counts the work the kernel issues (every tap of
+    every active row, absent taps as zero rows: the dense-K formulation);
+    tensor_frac_present only the present taps' work (Eq. 5's sum)."""
     from paper_2608_09388_gb300 import inputs
     w = inputs.make_workload("sweep10475_bf16")
     ly = w.layers[0]
@@ -720,10 +718,6 @@ def run_sweep(torch, hc, dev, stream):
 
     yd = torch.empty((B, V, ly.C_out), dtype=torch.bfloat16, device=dev)
     dense_ms = timeit(lambda: hc.hc_spiral_conv_fwd(x, spiral, Wt, bias, ly.act, yd, stream), 5)
-    order = torch.empty((B * V,), dtype=torch.int32, device=dev)
-    taps = torch.empty(((B * V + 127) // 128,), dtype=torch.int32, device=dev)
-    srb = torch.empty_like(rb)
-    num_kb = (L * ly.C_in + 63) // 64
     out = []
     for d, m in zip(w.densities, w.masks):
         mt = torch.from_numpy(m).to(dev)
@@ -731,37 +725,18 @@ def run_sweep(torch, hc, dev, stream):
             hc.hc_mask_compact_rulebook(mt, spiral, hc.HC_LAYOUT_DENSE, coords, row_of, offs,
                                         count, rb, stream)
         n = int(np.count_nonzero(m))
-        ms_plain = timeit(lambda: hc.hc_sparse_conv_rulebook_fwd(x, rb, count, Wt, bias, ly.act,
-                                                                 y, stream=stream))
-        # the row order (once per mask, like the rulebook), then the conv in it
-        ms_order = timeit(lambda: hc.hc_conv_rulebook_order(rb, count, order, taps, srb, stream))
-        ms = timeit(lambda: hc.hc_sparse_conv_rulebook_ordered_fwd(x, rb, count, Wt, bias, ly.act,
-                                                                   y, order, taps, srb,
-                                                                   stream=stream))
-        # work: nominal (every tap of every row, the dense-K formulation),
-        # present (Eq. 5's present taps only), executed (the MMAs issued)
+        ms = timeit(lambda: hc.hc_sparse_conv_rulebook_fwd(x, rb, count, Wt, bias, ly.act, y,
+                                                           stream=stream))
         per_tap = 2.0 * ly.C_in * ly.C_out
         fl = per_tap * L * n
-        rb_np = rb[:, :n].cpu().numpy()
-        present = per_tap * float((rb_np >= 0).sum())
-        t_np = taps[:(n + 127) // 128].cpu().numpy().view(np.uint32)
-        kb_taps = [sum(1 << l for l in range((kb * 64) // ly.C_in,
-                                             min(L, (kb * 64 + 63) // ly.C_in + 1)))
-                   for kb in range(num_kb)]
-        kbs = sum(max(1, sum(1 for m_ in kb_taps if int(t) & m_)) for t in t_np)
-        executed = 2.0 * 128 * 64 * ly.C_out * kbs
+        present = per_tap * float((rb[:, :n] >= 0).sum().item())
         tf = lambda f, t: f / (t * 1e-3) / 1e12 / pk["bf16_tflops"]  # noqa: E731
         out.append({"density": d, "active_rows": n, "sparse_us": ms * 1e3,
-                    "order_us": ms_order * 1e3, "unordered_us": ms_plain * 1e3,
                     "dense_us": dense_ms * 1e3, "speedup": dense_ms / ms,
-                    "speedup_with_order": dense_ms / (ms + ms_order),
-                    "speedup_unordered": dense_ms / ms_plain,
                     "rows_per_s": n / (ms * 1e-3),
-                    "work_executed_of_nominal": executed / fl,
-                    "work_present_of_nominal": present / fl,
-                    "tensor_frac": tf(executed, ms),
-                    "tensor_frac_present": tf(present, ms),
-                    "tensor_frac_unordered": tf(fl, ms_plain)})
+                    "work_present_of_issued": present / fl,
+                    "tensor_frac": tf(fl, ms),
+                    "tensor_frac_present": tf(present, ms)})
     st = hc.hc_get_device_status(stream)
     if st != hc.HC_OK:
         raise RuntimeError(f"device status {hc.STATUS_NAMES.get(st)} in the sweep")

@@ -213,52 +213,6 @@ hc_status hc_sparse_conv_rulebook_fwd(const void* x, hc_dtype dt, int x_rows,
                                       void* out, hc_stream_t stream);
 
 /*
- * hc_conv_rulebook_order -- an execution order for the rulebook convolution
- * (a schedule: the paper has no counterpart and the results do not depend
- * on it). Eq. 5 sums only the taps whose rulebook entry is present; at low
- * mask density most are absent, but a tile of consecutive rows nearly always
- * has every tap present in some row. This pass sorts the active rows by their
- * presence pattern (key bit l set when rulebook[l*capacity + n] >= 0) so that
- * rows with the same taps share tiles, and records each 128-row tile's union.
- * It depends on the mask only: one call serves every conv layer of a network,
- * like the rulebook.
- *   rulebook   [L, capacity] int32 as written by hc_conv_rulebook /
- *              hc_mask_compact_rulebook; count = N' on the device.
- *   order      [capacity] int32: positions 0..N'-1 receive a permutation of
- *              the active rows, keys non-decreasing in their low min(L, 12)
- *              bits; rows of equal low bits come in an unspecified order (the
- *              conv's results do not depend on it).
- *   tile_taps  [ceil(capacity / 128)] uint32: entry t = the OR of the keys
- *              of order[128 t .. 128 t + 127] (positions below N').
- *   sorted_rulebook [L, capacity] int32, not the rulebook itself: column p
- *              (p < N') receives the rulebook column of row order[p].
- * Uses the per-stream workspace (4 * capacity bytes + 32 KiB at most).
- */
-hc_status hc_conv_rulebook_order(const int32_t* rulebook, const int32_t* count, int capacity, int L,
-                                 int32_t* order, uint32_t* tile_taps, int32_t* sorted_rulebook,
-                                 hc_stream_t stream);
-
-/*
- * hc_sparse_conv_rulebook_ordered_fwd -- hc_sparse_conv_rulebook_fwd in the
- * order written by hc_conv_rulebook_order: tile t computes the rows
- * order[128 t ..] (reading sorted_rulebook's columns 128 t ..) and multiplies
- * only the taps in tile_taps[t] (a tap absent from every row of a tile would
- * contribute zero to each of them). Same arguments and results as
- * hc_sparse_conv_rulebook_fwd on `rulebook` (outputs at each row's own
- * position n), plus order, tile_taps and sorted_rulebook from
- * hc_conv_rulebook_order on that rulebook and count. The order is taken on
- * the tensor-core path (bf16, C_in and C_out multiples of 8) when
- * L * C_in <= 4096; otherwise the call is hc_sparse_conv_rulebook_fwd.
- */
-hc_status hc_sparse_conv_rulebook_ordered_fwd(const void* x, hc_dtype dt, int x_rows,
-                                              const int32_t* rulebook, const int32_t* count,
-                                              int capacity, int L, int C_in, int C_out,
-                                              const void* W, const float* bias, hc_act act, void* y,
-                                              const int32_t* coords, int B, int V, void* out,
-                                              const int32_t* order, const uint32_t* tile_taps,
-                                              const int32_t* sorted_rulebook, hc_stream_t stream);
-
-/*
  * hc_sparse_linear_fwd -- linear layer on compact rows (Eq. 6), row-wise
  *   y[n, o] = act( bias[o] + sum_{c<C_in} x[n, c] * W[c*C_out + o] ),  n < N'
  * The coordinates are unchanged (C' = C).

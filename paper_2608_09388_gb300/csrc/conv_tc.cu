@@ -101,8 +101,7 @@ struct Cfg {
     static constexpr int kBarBytes = 8 * (2 * kMaxStages + 9);
     // barriers, then 16 bytes (TMEM address, abort flag), then the two tap
     // tables ([L][kTabRows] int32 each) at a 128-byte boundary.
-    // (the 16 bytes are followed by 64 words: the taps of each k-block)
-    static constexpr int kTabOffset = (kBarBytes + 16 + 256 + 127) / 128 * 128;
+    static constexpr int kTabOffset = (kBarBytes + 16 + 127) / 128 * 128;
     // After the tables: one 2 KB staging buffer per epilogue warp (32 rows x
     // 64 bytes of bf16 output).
     static constexpr int kEpiBytes = kEpilogueWarps * 32 * 64;
@@ -325,33 +324,10 @@ __device__ __forceinline__ void gn_stats_chunk(const ConvArgs& a, const uint32_t
     }
 }
 
-// The taps k-block kb covers (k = 64 kb .. 64 kb + 63, tap k / C_in).
-__device__ __forceinline__ uint32_t kblock_taps(int kb, int C_in, int L) {
-    const int lo = (kb * kBK) / C_in;
-    int hi = (kb * kBK + kBK - 1) / C_in;
-    if (hi > L - 1) hi = L - 1;
-    if (lo > hi) return 0u;
-    return (hi >= 31 ? 0xffffffffu : ((2u << hi) - 1u)) & ~((1u << lo) - 1u);
-}
-// The k-blocks a tile needs: bit kb set when one of the taps k-block kb
-// covers (kbtap[kb], shared memory) is in the tile's tap union; at least one
-// (an all-absent tile still gets its accumulator written).
-__device__ __forceinline__ unsigned long long needed_kblocks(uint32_t taps, int num_kb,
-                                                              const volatile uint32_t* kbtap) {
-    unsigned long long m = 0;
-    for (int kb = 0; kb < num_kb; ++kb)
-        if (taps & kbtap[kb]) m |= 1ull << kb;
-    return m ? m : 1ull;
-}
-
-// ORD: rows in the order of hc_conv_rulebook_order (a.order, a.tile_taps;
-// rulebook mode, one-half items, at most 64 k-blocks), each tile multiplying
-// only the k-blocks of its tap union.
-template <int BN, int TM, bool ORD>
+template <int BN, int TM>
 __global__ void __launch_bounds__(kThreads, 1)
     conv_tc_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_w) {
     using C = Cfg<BN, TM>;
-    static_assert(!ORD || TM == 1, "ordered rows use one-half items");
     constexpr int kTabRows = C::kTabRows;
     // "full": one cp.async completion arrival per producer thread, plus the
     // expect-tx arrival of the weight loader.
@@ -370,8 +346,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint8_t* const misc = base_ptr + (sBar - base) + C::kBarBytes;
     volatile uint32_t* const tmem_holder = reinterpret_cast<volatile uint32_t*>(misc);
     volatile int* const abort_flag = reinterpret_cast<volatile int*>(misc + 4);
-    // ordered rows: the taps of each k-block (at most 64 k-blocks)
-    volatile uint32_t* const kbtap = reinterpret_cast<volatile uint32_t*>(misc + 16);
     // Tap tables, [2][L][kTabRows] int32: entry (l, r) is the input row
     // feeding slot l of row r of the work item, or -1.
     const uint32_t tab0 = sBar + C::kTabOffset;
@@ -405,7 +379,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
     }
     if (warp == kWeightWarp && lane == 0) prefetch_tensormap(&tmap_w);
-    if (ORD && threadIdx.x < 64) kbtap[threadIdx.x] = kblock_taps(threadIdx.x, a.C_in, a.L);
     if (warp == kMmaWarp) {
         tmem_alloc(smem_u32((const void*)tmem_holder), C::kTmemCols);
         tmem_relinquish();
@@ -475,19 +448,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t tab_s = tab0 + (uint32_t)buf * tab_bytes;
             int l = (q * 8) / C_in;  // slot and channel of this thread's chunk at k-block 0
             int c = q * 8 - l * C_in;
-            unsigned long long kbm = ~0ull;  // k-blocks this tile multiplies
-            if constexpr (ORD) kbm = needed_kblocks(a.tile_taps[w / n_tiles], num_kb, kbtap);
             for (int kb = 0; kb < num_kb; ++kb) {
-                if constexpr (ORD) {
-                    if (!((kbm >> kb) & 1ull)) {
-                        c += kBK;
-                        while (c >= C_in) {
-                            c -= C_in;
-                            ++l;
-                        }
-                        continue;
-                    }
-                }
                 const int s = st_s;
                 const uint32_t ph = st_ph;
                 if (!mbar_wait(empty_bar(s), ph ^ 1u, abort_flag, a.status)) {
@@ -546,13 +507,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             bool ok = true;
             for (long long w = blockIdx.x; w < work_total && ok; w += gridDim.x) {
                 const int n0 = ((int)w % n_tiles) * BN;  // w < 2^31
-                unsigned long long kbm = ~0ull;
-                if constexpr (ORD)
-                    kbm = needed_kblocks(a.tile_taps[w / n_tiles], num_kb, kbtap);
                 for (int kb = 0; kb < num_kb; ++kb) {
-                    if constexpr (ORD) {
-                        if (!((kbm >> kb) & 1ull)) continue;
-                    }
                     const int s = st_s;
                     if (!mbar_wait(empty_bar(s), st_ph ^ 1u, abort_flag, a.status)) {
                         ok = false;
@@ -605,14 +560,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc_fence_after();
                 // accumulator of half h: columns (acc * TM + h) * BN
                 const uint32_t d_tmem = tmem_base + (uint32_t)(acc * TM * BN);
-                unsigned long long kbm = ~0ull;
-                if constexpr (ORD)
-                    kbm = needed_kblocks(a.tile_taps[w / n_tiles], num_kb, kbtap);
-                bool first = true;  // the tile's first MMA overwrites without a bias
                 for (int kb = 0; kb < num_kb; ++kb) {
-                    if constexpr (ORD) {
-                        if (!((kbm >> kb) & 1ull)) continue;
-                    }
                     const int s = st_s;
                     const uint32_t ph = st_ph;
                     if (!mbar_wait(full_bar(s), ph, abort_flag, a.status)) {
@@ -630,7 +578,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         for (int k = 0; k < kBK / 16; ++k) {
                             const uint64_t bd =
                                 smem_desc_sw128(b_st + k * 16 * 128, kBK * 128, 1024);
-                            const uint32_t acc_in = (has_bias || !first || k != 0) ? 1u : 0u;
+                            const uint32_t acc_in = (has_bias || (kb | k) != 0) ? 1u : 0u;
 #pragma unroll
                             for (int h = 0; h < TM; ++h) {
                                 const uint64_t ad =
@@ -641,7 +589,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                         }
                     }
                     tc_commit(empty_bar(s));
-                    first = false;
                     ++it;
                     if (++st_s == nst) {
                         st_s = 0;
@@ -679,8 +626,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                 // Precomputed mapping: one coalesced pass over the tile's
                 // rulebook columns, entries checked against the input's rows
                 // (the first tile's table may have been filled before the loop).
-                // (with ordered rows the rulebook is the sorted one: column p
-                // belongs to the row position p computes)
                 long long col[4];
                 bool live[4];
 #pragma unroll
@@ -857,15 +802,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             // Everything that does not need the accumulator is loaded while
             // the main loop runs: this lane's row addresses (0 = not
             // written; the fused scatter's needs the row's coordinate).
-            long long row = m0 + ew * 32 + lane;
-            bool rvalid = row < rows;
-            if constexpr (ORD) {
-                // position -> the row it computes
-                const int o = rvalid ? __ldg(a.order + row) : 0;
-                if (rvalid && (o < 0 || o >= rows)) report(a.status, kErrIndex);
-                rvalid = rvalid && o >= 0 && o < rows;
-                row = rvalid ? o : 0;
-            }
+            const long long row = m0 + ew * 32 + lane;
+            const bool rvalid = row < rows;
             const long long row_y = (rvalid && y) ? (long long)(y + row * C_out) : 0;
             long long row_d = 0;
             if (rvalid && a.out_dense) {
@@ -1002,12 +940,12 @@ hc_status encode_w3d(CUtensorMap* m, const void* base, long long K, long long C_
     return HC_OK;
 }
 
-template <int BN, int TM, bool ORD>
+template <int BN, int TM>
 hc_status launch_bn(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s) {
     using C = Cfg<BN, TM>;
     static bool attr_set[64] = {};
     if (!attr_set[ctx->device]) {
-        hc_status st = check_cuda(cudaFuncSetAttribute(conv_tc_kernel<BN, TM, ORD>,
+        hc_status st = check_cuda(cudaFuncSetAttribute(conv_tc_kernel<BN, TM>,
                                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                        (int)kSmemLimit),
                                   "cudaFuncSetAttribute(conv_tc_kernel)");
@@ -1033,7 +971,7 @@ hc_status launch_bn(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s) {
     long long grid = cap_work < ctx->num_sms ? cap_work : ctx->num_sms;
     if (grid < 1) grid = 1;
     ka.stages = C::stages_for(a.L);
-    return launch_pdl(conv_tc_kernel<BN, TM, ORD>, dim3((unsigned)grid), dim3(kThreads),
+    return launch_pdl(conv_tc_kernel<BN, TM>, dim3((unsigned)grid), dim3(kThreads),
                       C::smem_bytes(a.L, ka.stages), s, "conv_tc_kernel", ka, tw);
 }
 
@@ -1062,13 +1000,8 @@ hc_status launch_conv_tc(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s
     const long long n_tiles = (a.C_out + 127) / 128;
     const bool two = a.mode == kDense && (a.capacity + 2 * kBM - 1) / (2 * kBM) * n_tiles >=
                                              2ll * ctx->num_sms;
-    // rows in a given order (the caller checked: rulebook mode, at most 64
-    // k-blocks): tiles skip the k-blocks of taps none of their rows has
-    const bool ord = a.order != nullptr;
-    if (conv_tc_tile_n(a) == 64)
-        return ord ? launch_bn<64, 1, true>(ctx, a, s) : launch_bn<64, 1, false>(ctx, a, s);
-    if (ord) return launch_bn<128, 1, true>(ctx, a, s);
-    return two ? launch_bn<128, 2, false>(ctx, a, s) : launch_bn<128, 1, false>(ctx, a, s);
+    if (conv_tc_tile_n(a) == 64) return launch_bn<64, 1>(ctx, a, s);
+    return two ? launch_bn<128, 2>(ctx, a, s) : launch_bn<128, 1>(ctx, a, s);
 }
 
 }  // namespace hc

@@ -320,16 +320,13 @@ hc_status hc_mask_compact_rulebook(const uint8_t* mask, int B, int V, const int3
     return launch_rulebook(ctx, coords, row_of, count, spiral, B, V, L, (int)x_layout, rulebook, s);
 }
 
-}  // extern "C"
-
-// The rulebook conv, optionally in a row order (order and tile_taps both
-// given, or both NULL).
-static hc_status conv_rulebook(const char* fn, const void* x, hc_dtype dt, int x_rows,
-                               const int32_t* rulebook, const int32_t* count, int capacity, int L,
-                               int C_in, int C_out, const void* W, const float* bias, hc_act act,
-                               void* y, const int32_t* coords, int B, int V, void* out,
-                               const int32_t* order, const uint32_t* tile_taps,
-                               const int32_t* sorted_rb, cudaStream_t stream) {
+hc_status hc_sparse_conv_rulebook_fwd(const void* x, hc_dtype dt, int x_rows,
+                                      const int32_t* rulebook, const int32_t* count, int capacity,
+                                      int L, int C_in, int C_out, const void* W, const float* bias,
+                                      hc_act act, void* y, const int32_t* coords, int B, int V,
+                                      void* out, hc_stream_t stream) {
+    const char* fn = "hc_sparse_conv_rulebook_fwd";
+    t_last_error[0] = 0;
     HC_REQUIRE(y || out, "%s: at least one of y and out is required", fn);
     hc_status st = check_conv_common(fn, dt, L, C_in, C_out, act, x, W, y ? y : out);
     if (st != HC_OK) return st;
@@ -364,66 +361,7 @@ static hc_status conv_rulebook(const char* fn, const void* x, hc_dtype dt, int x
     a.out_coords = coords;
     a.out_B = B;
     a.out_V = V;
-    // The row order is taken by the tensor-core kernel when a tile's k-blocks
-    // fit its 64-bit k-block mask; otherwise rows run in order (the results
-    // are the same).
-    if (order && conv_tc_supported(a, dt) && (a.K + 63) / 64 <= 64) {
-        a.rulebook = sorted_rb;
-        a.order = order;
-        a.tile_taps = tile_taps;
-    }
-    return dispatch_conv(ctx, a, dt, stream);
-}
-
-extern "C" {
-
-hc_status hc_sparse_conv_rulebook_fwd(const void* x, hc_dtype dt, int x_rows,
-                                      const int32_t* rulebook, const int32_t* count, int capacity,
-                                      int L, int C_in, int C_out, const void* W, const float* bias,
-                                      hc_act act, void* y, const int32_t* coords, int B, int V,
-                                      void* out, hc_stream_t stream) {
-    t_last_error[0] = 0;
-    return conv_rulebook("hc_sparse_conv_rulebook_fwd", x, dt, x_rows, rulebook, count, capacity,
-                         L, C_in, C_out, W, bias, act, y, coords, B, V, out, nullptr, nullptr,
-                         nullptr, (cudaStream_t)stream);
-}
-
-hc_status hc_sparse_conv_rulebook_ordered_fwd(const void* x, hc_dtype dt, int x_rows,
-                                              const int32_t* rulebook, const int32_t* count,
-                                              int capacity, int L, int C_in, int C_out,
-                                              const void* W, const float* bias, hc_act act, void* y,
-                                              const int32_t* coords, int B, int V, void* out,
-                                              const int32_t* order, const uint32_t* tile_taps,
-                                              const int32_t* sorted_rulebook,
-                                              hc_stream_t stream) {
-    const char* fn = "hc_sparse_conv_rulebook_ordered_fwd";
-    t_last_error[0] = 0;
-    HC_REQUIRE(order && tile_taps && sorted_rulebook,
-               "%s: order, tile_taps and sorted_rulebook are required", fn);
-    return conv_rulebook(fn, x, dt, x_rows, rulebook, count, capacity, L, C_in, C_out, W, bias,
-                         act, y, coords, B, V, out, order, tile_taps, sorted_rulebook,
-                         (cudaStream_t)stream);
-}
-
-hc_status hc_conv_rulebook_order(const int32_t* rulebook, const int32_t* count, int capacity, int L,
-                                 int32_t* order, uint32_t* tile_taps, int32_t* sorted_rulebook,
-                                 hc_stream_t stream) {
-    const char* fn = "hc_conv_rulebook_order";
-    t_last_error[0] = 0;
-    HC_REQUIRE(capacity >= 0, "%s: capacity=%d must be >= 0", fn, capacity);
-    HC_REQUIRE(L >= 1, "%s: L=%d must be >= 1", fn, L);
-    if (L > HC_MAX_SPIRAL) {
-        set_error("%s: L=%d exceeds HC_MAX_SPIRAL=%d", fn, L, HC_MAX_SPIRAL);
-        return HC_ERR_UNSUPPORTED;
-    }
-    HC_REQUIRE(rulebook && count && order && tile_taps && sorted_rulebook,
-               "%s: rulebook, count, order, tile_taps and sorted_rulebook are required", fn);
-    HC_REQUIRE(sorted_rulebook != rulebook, "%s: sorted_rulebook must not be rulebook", fn);
-    if (capacity == 0) return HC_OK;
-    const DeviceCtx* ctx = device_ctx();
-    if (!ctx) return HC_ERR_CUDA;
-    return launch_rulebook_order(ctx, rulebook, count, capacity, L, order, tile_taps,
-                                 sorted_rulebook, (cudaStream_t)stream);
+    return dispatch_conv(ctx, a, dt, (cudaStream_t)stream);
 }
 
 hc_status hc_sparse_group_norm_fwd(const void* x, hc_dtype dt, const int32_t* batch_offsets, int B,

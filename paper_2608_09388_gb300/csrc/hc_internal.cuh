@@ -84,12 +84,6 @@ struct ConvArgs {
     int act;
     int stages;  // pipeline depth chosen by the launcher (tensor-core kernel)
     int w3d;     // tensor-core kernel: W's tensor map is the 3-D view (one box per stage)
-    // Optional row order (rulebook mode, tensor-core kernel): position p of
-    // the tiles computes row order[p] (the rulebook is then the sorted one,
-    // its column p being row order[p]'s), tile t only the taps set in
-    // tile_taps[t]; NULL = rows in order, every tap.
-    const int32_t* order;
-    const uint32_t* tile_taps;
     // Optional group-norm statistics of the stored output (Eqs. 7-9,
     // tensor-core kernel): every block c of 32 output rows writes, for each
     // frame b among its rows (b = gn_coords[2n]) and each channel group g of
@@ -119,12 +113,6 @@ hc_status launch_compact_map(const DeviceCtx* ctx, const uint8_t* mask, int B, i
                              const int32_t* spiral, int L, int x_layout, int32_t* coords,
                              int32_t* row_of, int32_t* offsets, int32_t* count, int32_t* rulebook,
                              cudaStream_t s);
-// Row order of the rulebook conv: active rows sorted by tap-presence pattern,
-// the tap union of every 128-row tile of the order, and the rulebook columns
-// in that order (see order.cu).
-hc_status launch_rulebook_order(const DeviceCtx* ctx, const int32_t* rulebook,
-                                const int32_t* count, long long capacity, int L, int32_t* order,
-                                uint32_t* tile_taps, int32_t* sorted_rb, cudaStream_t s);
 hc_status launch_rulebook(const DeviceCtx* ctx, const int32_t* coords, const int32_t* row_of,
                           const int32_t* count, const int32_t* spiral, int B, int V, int L,
                           int x_layout, int32_t* rulebook, cudaStream_t s);

@@ -66,18 +66,6 @@ def test_invalid_arguments_rejected_on_host(lib):
                                 None) == hc.HC_ERR_INVALID_ARG
     assert lib.hc_scatter_dense(fake, 1, None, fake, fake, 2, 3, 8, 0, fake,
                                 None) == hc.HC_ERR_INVALID_ARG
-    # row order of the rulebook conv: spiral too long, missing count
-    assert lib.hc_conv_rulebook_order(fake, fake, 10, 33, fake, fake, P(0x2000),
-                                      None) == hc.HC_ERR_UNSUPPORTED
-    assert lib.hc_conv_rulebook_order(fake, None, 10, 9, fake, fake, P(0x2000),
-                                      None) == hc.HC_ERR_INVALID_ARG
-    # the sorted rulebook may not be the rulebook itself
-    assert lib.hc_conv_rulebook_order(fake, fake, 10, 9, fake, fake, fake,
-                                      None) == hc.HC_ERR_INVALID_ARG
-    # the ordered conv needs the order, the tile unions and the sorted rulebook
-    assert lib.hc_sparse_conv_rulebook_ordered_fwd(fake, 1, 10, fake, fake, 10, 9, 16, 16, fake,
-                                                   None, 1, fake, None, 0, 0, None, None, fake,
-                                                   fake, None) == hc.HC_ERR_INVALID_ARG
     # test hooks: unknown option, group-norm path out of range (no CUDA call)
     assert lib.hc_test_set_option(99, 0) == hc.HC_ERR_INVALID_ARG
     assert lib.hc_test_set_option(hc.HC_TEST_GROUP_NORM_PATH, 3) == hc.HC_ERR_INVALID_ARG
