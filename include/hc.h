@@ -138,8 +138,12 @@ hc_status hc_mask_compact_static(const uint8_t* mask, int B, int V, int32_t* coo
  * 1 <= L <= HC_MAX_SPIRAL, C_in >= 1, C_out >= 1.
  * Out-of-range spiral/row_of/coords entries contribute nothing and set
  * HC_ERR_INVALID_INDEX; a count above B*V is clamped and sets HC_ERR_CAPACITY.
- * bf16 with C_in % 8 == 0, C_out % 8 == 0 and 16-byte aligned x, W, y runs
- * on the tensor cores (tcgen05); other shapes run on CUDA cores.
+ * bf16 with C_out % 8 == 0 and 16-byte aligned W, y runs on the tensor cores
+ * (tcgen05); other shapes run on CUDA cores. With C_in % 8 != 0 (x then
+ * needs only 2-byte alignment) x and W are first copied, with zero channels
+ * appended up to C_pad = the next multiple of 8, into the per-stream
+ * workspace (x_rows * C_pad * 2 + L * C_pad * C_out * 2 bytes; compact inputs
+ * copy their first N' rows only); the sums are unchanged.
  */
 hc_status hc_sparse_spiral_conv_fwd(const void* x, hc_layout x_layout, hc_dtype dt,
                                     const int32_t* coords, const int32_t* row_of,

@@ -878,6 +878,49 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 }
 
+// C_in not a multiple of 8: x [rows, C_in] and W [L*C_in, C_out] copied with
+// zero channels appended up to C_pad (a multiple of 8), so that every tap's
+// slice of a gathered row starts on a 16-byte boundary. 16-byte pieces of
+// the outputs, one per thread (grid-stride): first x's (rows past *count
+// skipped when count is given: compact inputs hold N' rows), then W's.
+__global__ void __launch_bounds__(256) channel_pad_kernel(
+    const uint16_t* __restrict__ x, long long x_rows, const int32_t* __restrict__ count, int C_in,
+    int C_pad, uint4* __restrict__ xp, const uint4* __restrict__ W, int L, int C_out,
+    uint4* __restrict__ Wp) {
+    pdl_wait();
+    pdl_trigger();
+    long long rows = x_rows;
+    if (count) {
+        const long long n = *count;
+        rows = n < 0 ? 0 : (n < x_rows ? n : x_rows);
+    }
+    const int xq = C_pad / 8;   // 16-byte pieces per padded row of x
+    const int wq = C_out / 8;   // 16-byte pieces per row of W
+    const long long nx = rows * xq;
+    const long long nw = (long long)L * C_pad * wq;
+    for (long long i = blockIdx.x * 256ll + threadIdx.x; i < nx + nw; i += gridDim.x * 256ll) {
+        if (i < nx) {
+            const long long r = i / xq;
+            const int c0 = (int)(i - r * xq) * 8;
+            const uint16_t* src = x + r * C_in + c0;
+            uint32_t v[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const uint32_t lo = c0 + 2 * e < C_in ? src[2 * e] : 0u;
+                const uint32_t hi = c0 + 2 * e + 1 < C_in ? src[2 * e + 1] : 0u;
+                v[e] = lo | (hi << 16);
+            }
+            xp[i] = make_uint4(v[0], v[1], v[2], v[3]);
+        } else {
+            const long long j = i - nx;
+            const long long rp = j / wq;  // padded row l * C_pad + c
+            const int l = (int)(rp / C_pad), c = (int)(rp - (long long)l * C_pad);
+            Wp[j] = c < C_in ? W[((long long)l * C_in + c) * wq + (j - rp * wq)]
+                             : make_uint4(0u, 0u, 0u, 0u);
+        }
+    }
+}
+
 // ---------------------------------------------------------------- host side
 
 PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
@@ -978,12 +1021,22 @@ hc_status launch_bn(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s) {
 }  // namespace
 
 bool conv_tc_supported(const ConvArgs& a, hc_dtype dt) {
-    const uintptr_t al =
-        (uintptr_t)a.x | (uintptr_t)a.W | (uintptr_t)a.y | (uintptr_t)a.out_dense;
+    // C_in not a multiple of 8 runs on channel-padded copies of x and W (x
+    // itself is read by 2-byte loads then)
+    const bool pad = a.C_in % 8 != 0;
+    const uintptr_t al = (pad ? 0 : (uintptr_t)a.x) | (uintptr_t)a.W | (uintptr_t)a.y |
+                         (uintptr_t)a.out_dense;
     // tile indices are 32-bit in the kernel
     const long long tiles = (a.capacity + kBM - 1) / kBM * ((a.C_out + 63) / 64);
-    return dt == HC_BF16 && a.C_in % 8 == 0 && a.C_out % 8 == 0 && al % 16 == 0 &&
+    return dt == HC_BF16 && a.C_out % 8 == 0 && al % 16 == 0 && (uintptr_t)a.x % 2 == 0 &&
            a.L <= HC_MAX_SPIRAL && tiles < (1ll << 31);
+}
+
+size_t conv_tc_pad_bytes(const ConvArgs& a) {
+    if (a.C_in % 8 == 0) return 0;
+    const size_t C_pad = (size_t)(a.C_in + 7) / 8 * 8;
+    const size_t xb = ((size_t)a.x_rows * C_pad * 2 + 255) / 256 * 256;
+    return xb + (size_t)a.L * C_pad * (size_t)a.C_out * 2;
 }
 
 int conv_tc_tile_n(const ConvArgs& a) {
@@ -991,6 +1044,38 @@ int conv_tc_tile_n(const ConvArgs& a) {
 }
 
 hc_status launch_conv_tc(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s) {
+    if (a.C_in % 8 != 0) {
+        // pad the channels (into the caller's workspace), then the same
+        // kernel on C_pad channels: the appended channels are zeros in x and
+        // rows of zeros in W, so every sum is unchanged
+        if (!a.pad_ws) {
+            set_error("conv_tc: C_in=%d needs the channel-padding workspace", a.C_in);
+            return HC_ERR_INVALID_ARG;
+        }
+        const int C_pad = (a.C_in + 7) / 8 * 8;
+        char* ws = static_cast<char*>(a.pad_ws);
+        const size_t xb = ((size_t)a.x_rows * C_pad * 2 + 255) / 256 * 256;
+        ConvArgs b = a;
+        b.x = ws;
+        b.W = ws + xb;
+        b.C_in = C_pad;
+        b.K = a.L * C_pad;
+        b.pad_ws = nullptr;
+        // compact inputs: only the first N' rows are read
+        const int32_t* rows_from = a.mode == kSparseCompactX ? a.count : nullptr;
+        const long long work = a.x_rows * (C_pad / 8) + (long long)a.L * C_pad * (a.C_out / 8);
+        long long grid = (work + 255) / 256;
+        const long long cap = 8ll * ctx->num_sms;
+        if (grid > cap) grid = cap;
+        if (grid < 1) grid = 1;
+        hc_status st = launch_pdl(channel_pad_kernel, dim3((unsigned)grid), dim3(256), 0, s,
+                                  "channel_pad_kernel", static_cast<const uint16_t*>(a.x),
+                                  a.x_rows, rows_from, a.C_in, C_pad, reinterpret_cast<uint4*>(ws),
+                                  static_cast<const uint4*>(a.W), a.L, a.C_out,
+                                  reinterpret_cast<uint4*>(ws + xb));
+        if (st != HC_OK) return st;
+        return launch_conv_tc(ctx, b, s);
+    }
     // Two-half items when the row count is known on the host (the dense
     // layer) and fills every SM with at least two of them: they halve the
     // weight traffic and per-stage overhead per MMA. The sparse calls' row

@@ -106,7 +106,13 @@ static bool misaligned(const void* p, size_t a) {
 // CUDA cores otherwise.
 hc_status dispatch_conv(const DeviceCtx* ctx, ConvArgs& a, hc_dtype dt, cudaStream_t s) {
     a.status = ctx->status;
-    if (conv_tc_supported(a, dt)) return launch_conv_tc(ctx, a, s);
+    if (conv_tc_supported(a, dt)) {
+        if (const size_t pb = conv_tc_pad_bytes(a)) {
+            a.pad_ws = stream_workspace(s, pb);
+            if (!a.pad_ws) return HC_ERR_CUDA;
+        }
+        return launch_conv_tc(ctx, a, s);
+    }
     return launch_conv_simt(ctx, a, dt, s);
 }
 
@@ -435,11 +441,14 @@ hc_status hc_sparse_conv_gn_fwd(const void* x, hc_dtype dt, int x_rows, const in
         // (frame, 32-row block inside it) in slot frame + block, one per row
         // of the blocks that straddle a frame boundary
         const size_t slots = (size_t)B + ((size_t)capacity + 31) / 32;
-        const size_t part_bytes = 16 * slots * (size_t)G;
-        char* ws = (char*)stream_workspace(s, part_bytes + 8 * (size_t)capacity * (size_t)G);
+        const size_t part_bytes = (16 * slots * (size_t)G + 255) / 256 * 256;
+        const size_t rows_bytes = (8 * (size_t)capacity * (size_t)G + 255) / 256 * 256;
+        const size_t pad_bytes = conv_tc_pad_bytes(a);
+        char* ws = (char*)stream_workspace(s, part_bytes + rows_bytes + pad_bytes);
         if (!ws) return HC_ERR_CUDA;
         float* part = (float*)ws;
         float* rows = (float*)(ws + part_bytes);
+        if (pad_bytes) a.pad_ws = ws + part_bytes + rows_bytes;
         a.gn_part = part;
         a.gn_rows = rows;
         a.gn_coords = coords;

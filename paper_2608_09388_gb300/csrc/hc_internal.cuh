@@ -97,6 +97,10 @@ struct ConvArgs {
     const int32_t* gn_coords;
     int gn_G, gn_B;
     int gn_cpg;  // channels per group, C_out / gn_G: 8, 16, 32, 64 or 128
+    // Tensor-core kernel with C_in not a multiple of 8: workspace of at
+    // least conv_tc_pad_bytes(a) bytes (256-byte aligned) for x and W with
+    // zero channels appended up to a multiple of 8.
+    void* pad_ws;
 };
 
 // Launchers (each in its own translation unit). All return HC_OK or an
@@ -107,6 +111,7 @@ hc_status launch_conv_simt(const DeviceCtx* ctx, const ConvArgs& a, hc_dtype dt,
 hc_status launch_conv_tc(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s);
 bool conv_tc_supported(const ConvArgs& a, hc_dtype dt);
 int conv_tc_tile_n(const ConvArgs& a);  // output channels per tensor-core tile
+size_t conv_tc_pad_bytes(const ConvArgs& a);  // 0 when C_in % 8 == 0
 // Compaction fused with the Eq. 4 mapping (frames of at most 65535 vertices).
 bool compact_map_supported(int B, int V, int L);
 hc_status launch_compact_map(const DeviceCtx* ctx, const uint8_t* mask, int B, int V,

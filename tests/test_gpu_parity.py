@@ -247,6 +247,55 @@ def test_sparse_conv_odd_channels_bf16(C_in, C_out):
     check_close(y[:n], y_pre, f"odd channels {C_in}->{C_out}")
 
 
+@pytest.mark.parametrize("entry", ["spiral_dense", "spiral_compact", "rulebook_scatter", "dense"])
+@pytest.mark.parametrize("L,C_in,C_out", [
+    (9, 45, 64),    # the motion encoder's first layer: chunks cross slots
+    (12, 13, 128),  # several slots per k-block
+    (32, 9, 64),    # K = 288: a ragged last k-block
+    (5, 100, 136),  # two output tiles, the second ragged
+])
+def test_tc_channels_not_multiple_of_8(entry, L, C_in, C_out):
+    """bf16 with C_in % 8 != 0 runs on the tensor cores with element-wise
+    gathers; several row tiles and a ragged tail, every entry point."""
+    B, V = 4, 1500
+    dens = 1.0 if entry == "dense" else 0.45
+    sp, m, x, W, b = inputs.random_case(L * 1000 + C_in * 10 + C_out, B, V, L, C_in, C_out,
+                                        "bf16", dens, neg_frac=0.1)
+    c, r, _, n = oracle.mask_compact(m)
+    assert n > 3 * 128
+    if entry == "dense":
+        yd = torch.full((B, V, C_out), float("nan"), dtype=torch.bfloat16, device="cuda")
+        hc.hc_spiral_conv_fwd(to_torch(x), to_torch(sp), to_torch(W), to_torch(b),
+                              hc.HC_ACT_ELU, yd)
+        assert hc.hc_get_device_status() == hc.HC_OK
+        y = to_numpy(yd).reshape(B * V, C_out)[c[:, 0] * V + c[:, 1]]
+        layout, xin = oracle.LAYOUT_DENSE, x
+    elif entry == "rulebook_scatter":
+        layout, xin = oracle.LAYOUT_DENSE, x
+        rb, coords, row_of, count = gpu_rulebook(m, sp, hc.HC_LAYOUT_DENSE)
+        prev = inputs.features(np.random.default_rng(9), (B, V, C_out), "bf16")
+        out = to_torch(prev)
+        yt = torch.full((B * V, C_out), float("nan"), dtype=torch.bfloat16, device="cuda")
+        hc.hc_sparse_conv_rulebook_fwd(to_torch(x), rb, count, to_torch(W), to_torch(b),
+                                       hc.HC_ACT_ELU, yt, coords=coords, out=out)
+        assert hc.hc_get_device_status() == hc.HC_OK
+        y = to_numpy(yt)[:n]
+        o = to_numpy(out)
+        np.testing.assert_array_equal(o[c[:, 0], c[:, 1]], y)
+        inactive = np.ones((B, V), bool)
+        inactive[c[:, 0], c[:, 1]] = False
+        np.testing.assert_array_equal(o[inactive], prev[inactive])
+    else:
+        layout = hc.HC_LAYOUT_DENSE if entry == "spiral_dense" else hc.HC_LAYOUT_COMPACT
+        xin = x if layout == hc.HC_LAYOUT_DENSE else np.ascontiguousarray(x[c[:, 0], c[:, 1]])
+        y, n_gpu = run_sparse_conv(xin, layout, m, sp, W, b, hc.HC_ACT_ELU)
+        assert n_gpu == n
+        y = y[:n]
+    y_pre, _ = oracle.sparse_spiral_conv(xin, layout, c, r, sp, W, b, oracle.ACT_ELU,
+                                         n_threads=NCPU)
+    check_close(y, y_pre, f"{entry} L={L} {C_in}->{C_out}")
+
+
 @pytest.mark.parametrize("act", [hc.HC_ACT_NONE, hc.HC_ACT_RELU])
 def test_sparse_conv_activations(act):
     sp, m, x, W, b = inputs.random_case(31, 2, 300, 9, 64, 64, "bf16", 0.4)
