@@ -290,6 +290,11 @@ def run_ours(args, rank, world, local_rank):
         assert int(s.count.item()) == s.rows, "active-row count differs from the mask"
 
     def capture(fn, idx):
+        # one eager call first: whatever workspace or per-stream state the
+        # call needs is allocated before the capture (no allocation inside)
+        with torch.cuda.stream(stream):
+            fn(sets[idx[0]])
+        torch.cuda.synchronize(dev)
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=stream):
             for i in idx:

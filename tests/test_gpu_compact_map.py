@@ -113,6 +113,34 @@ def test_workload_mask_and_many_tiles():
     check(big, w.spiral, hc.HC_LAYOUT_COMPACT, run_fused(big, w.spiral, hc.HC_LAYOUT_COMPACT))
 
 
+def test_many_frames_twice():
+    """Many frames (6000 frames of 1200 vertices: 12000 CTAs of the write
+    pass, more than the GPU holds at once; 16400 frames of 40 vertices),
+    each twice in a row on the same buffers."""
+    for B, V in ((6000, 1200), (16400, 40)):
+        rng = np.random.default_rng(B)
+        sp = rng.integers(0, V, size=(V, 5)).astype(np.int32)
+        sp[:, 0] = np.arange(V)
+        m = inputs.uniform_mask(rng, B, V, 0.07)
+        for _ in range(2):
+            check(m, sp, hc.HC_LAYOUT_COMPACT, run_fused(m, sp, hc.HC_LAYOUT_COMPACT))
+            assert hc.hc_get_device_status() == hc.HC_OK
+
+
+def test_streams_and_sizes_back_to_back():
+    """Calls of changing frame counts back to back on two streams (each
+    stream has its own workspace): every one bit-exact."""
+    side = torch.cuda.Stream()
+    for i, (B, V) in enumerate([(64, 655), (3, 10475), (200, 300), (1, 12), (64, 655)]):
+        sp, m = case(300 + i, B, V, 9, 0.3)
+        check(m, sp, hc.HC_LAYOUT_DENSE, run_fused(m, sp, hc.HC_LAYOUT_DENSE))
+        torch.cuda.synchronize()
+        with torch.cuda.stream(side):
+            got = run_fused(m, sp, hc.HC_LAYOUT_COMPACT)
+        check(m, sp, hc.HC_LAYOUT_COMPACT, got)
+    assert hc.hc_get_device_status() == hc.HC_OK
+
+
 @pytest.mark.parametrize("offset", [1, 5, 8])
 def test_misaligned_mask(offset):
     sp, m, *_ = inputs.random_case(offset, 9, 777, 9, 8, 8, "f32", 0.3, neg_frac=0.2)
