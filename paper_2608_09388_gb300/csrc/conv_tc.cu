@@ -7,16 +7,17 @@
 // (zeros for absent taps, Eq. 4); the layer computes A * W + bias (Eq. 5 with
 // the bias of Eq. 6) and the activation of Eq. 10.
 //
-// One persistent CTA per SM, 352 threads in five roles. A work item is tm
-// 128-row halves of output rows (tm = 2 when there are at least two items per
-// CTA, else 1, decided from the device row count) times BN output channels;
-// both halves are multiplied by the same W slice of every stage, which halves
-// the weight traffic and the per-stage overhead per MMA of large layers.
+// One persistent CTA per SM, 352 threads in five roles (384 with two-half
+// items). A work item is tm 128-row halves of output rows (tm = 2 for the
+// dense layer when it gives every SM at least two items, else 1) times BN
+// output channels; both halves are multiplied by the same W slice of every
+// stage, which halves the weight traffic and the per-stage overhead per MMA
+// of large layers.
 //   warp 9     index warp: for each item, resolves the L x (tm*128) tap table
 //              (from the rulebook, or coords -> spiral -> row_of, i.e. idx()
 //              of Eq. 4) with every load of a phase in flight at once, into
 //              one of two tables, so the next item's table is built while the
-//              current one is used;
+//              current one is used (two-half items: warp 11 builds half 1);
 //   warps 0-3  producers: fill a stage with the tm x 128 rows x 64 bf16 of A
 //              for one k-block. The 128 threads gather A with 16-byte cp.async
 //              through the tap table (zero-fill for absent taps and for k
@@ -74,7 +75,13 @@ constexpr int kEpilogueWarps = 4;
 constexpr int kMmaWarp = kProducerWarps + kEpilogueWarps;
 constexpr int kIndexWarp = kMmaWarp + 1;
 constexpr int kWeightWarp = kIndexWarp + 1;
-constexpr int kThreads = (kWeightWarp + 1) * 32;
+// Two-half items have a second index warp (half 1 of every tap table): one
+// warp resolving 2 x 128 rows x L slots per item fell behind the producers
+// (dense layer at L = 12: the table took ~12.7 us per item against 6.3 us of
+// gathers). One-half items launch without it.
+constexpr int kIndexWarp2 = kWeightWarp + 1;
+template <int TM>
+constexpr int kThreadsFor = (TM == 2 ? kIndexWarp2 + 1 : kWeightWarp + 1) * 32;
 constexpr int kTabChunk = 6;  // spiral slots resolved per pass of the index warp
 constexpr size_t kSmemLimit = 227 * 1024;  // opt-in dynamic shared memory per CTA
 
@@ -325,7 +332,7 @@ __device__ __forceinline__ void gn_stats_chunk(const ConvArgs& a, const uint32_t
 }
 
 template <int BN, int TM>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kThreadsFor<TM>, 1)
     conv_tc_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_w) {
     using C = Cfg<BN, TM>;
     constexpr int kTabRows = C::kTabRows;
@@ -372,7 +379,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         mbar_init(fin_bar, 1);
         for (int i = 0; i < 2; ++i) {
-            mbar_init(tabfull_bar(i), 32);
+            mbar_init(tabfull_bar(i), 32 * TM);  // the index warps' lanes
             mbar_init(tabempty_bar(i), kProducerWarps * 32);
         }
         *abort_flag = 0;
@@ -603,7 +610,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_wait_drain(fin_bar, 0, a.status);
         }
         __syncwarp();
-    } else if (warp == kIndexWarp) {
+    } else if (warp == kIndexWarp || (TM == 2 && warp == kIndexWarp2)) {
+        // two-half items: kIndexWarp builds half 0 of every table, kIndexWarp2 half 1
+        const int h_lo = warp == kIndexWarp ? 0 : 1;
+        const int h_hi = TM == 2 ? h_lo + 1 : 1;
         // ------------------------------------------------------------ index warp
         // Lane handles rows lane + 32*i (i < 4) of the tile. Phase 1 loads the
         // coordinates, phase 2 all spiral entries of a chunk of slots, phase 3
@@ -618,7 +628,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 break;
             const long long m_item = (long long)((int)w / n_tiles) * item_rows;
             unsigned err = 0;
-            for (int h = 0; h < TM; ++h) {
+            for (int h = h_lo; h < h_hi; ++h) {
             // half h: rows m0 .. m0 + 127, table entries (l, r) at tab_s + (l * kTabRows + r) * 4
             const long long m0 = m_item + h * kBM;
             const uint32_t tab_s = tab0 + (uint32_t)buf * tab_bytes + (uint32_t)(h * kBM) * 4u;
@@ -1014,7 +1024,7 @@ hc_status launch_bn(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s) {
     long long grid = cap_work < ctx->num_sms ? cap_work : ctx->num_sms;
     if (grid < 1) grid = 1;
     ka.stages = C::stages_for(a.L);
-    return launch_pdl(conv_tc_kernel<BN, TM>, dim3((unsigned)grid), dim3(kThreads),
+    return launch_pdl(conv_tc_kernel<BN, TM>, dim3((unsigned)grid), dim3(kThreadsFor<TM>),
                       C::smem_bytes(a.L, ka.stages), s, "conv_tc_kernel", ka, tw);
 }
 
