@@ -113,7 +113,9 @@ FUSED = [(3, 200, 9, 16, 64, 8),     # 8 channels per group, 4 groups per 32-col
          (3, 300, 9, 16, 128, 1),    # layer norm over 128 channels
          (4, 250, 9, 16, 64, 1),     # layer norm over the 64-channel tile
          (5, 200, 5, 8, 32, 4),      # C_out below the 64-channel tile
-         (3, 180, 7, 16, 256, 8)]    # two column tiles
+         (3, 180, 7, 16, 256, 8),    # two column tiles
+         (3, 200, 9, 45, 64, 8),     # C_in not a multiple of 8: channel-padded x and W
+         (2, 300, 9, 3, 128, 4)]     # C_in below 8
 # Two calls: fp32, or a group layout the epilogue does not take.
 UNFUSED = [(3, 200, 9, 16, 64, 16),  # 4 channels per group
            (3, 200, 9, 16, 48, 2),   # 24 per group

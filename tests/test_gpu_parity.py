@@ -253,6 +253,7 @@ def test_sparse_conv_odd_channels_bf16(C_in, C_out):
     (12, 13, 128),  # several slots per k-block
     (32, 9, 64),    # K = 288: a ragged last k-block
     (5, 100, 136),  # two output tiles, the second ragged
+    (9, 3, 64),     # C_in below 8: one 8-channel slot per tap
 ])
 def test_tc_channels_not_multiple_of_8(entry, L, C_in, C_out):
     """bf16 with C_in % 8 != 0 runs on the tensor cores with element-wise
