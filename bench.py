@@ -1116,7 +1116,13 @@ def run_configs(torch, hc, dev, stream, cpu_budget_s=3.0):
     once (compaction + Eq. 4 mapping in the compact layout), gather S'
     (Eq. 2), every layer on the compact rows, one CUDA graph; against the
     same network run densely on every vertex, and against the oracle on 1
-    thread and on every host core (bounded frame samples)."""
+    thread and on every host core (bounded frame samples).
+    Chains: "compact" (compaction + mapping in the compact layout, the S'
+    gather, every layer on compact rows) and "dense_layout" (the mapping in
+    the dense layout, every conv reading the previous layer's dense rows and
+    writing only its active rows back into a dense tensor by the fused
+    scatter, the per-vertex head as the rulebook conv on the centre slot:
+    no gather launch); the line reports the faster."""
     from paper_2608_09388_gb300 import inputs
     pk = peaks()
     props = torch.cuda.get_device_properties(dev)
@@ -1159,6 +1165,26 @@ def run_configs(torch, hc, dev, stream, cpu_budget_s=3.0):
                 else:
                     hc.hc_sparse_linear_fwd(hs[i], count, Ws[i], bs[i], ly.act, dst, stream)
 
+        # the dense-layout chain: inactive rows of the dense tensors are never
+        # read (their taps are absent in the rulebook)
+        rb_d = torch.empty((L, B * V), dtype=torch.int32, device=dev)
+        dense_a = [torch.empty((B, V, ly.C_out), dtype=dt, device=dev) for ly in w.layers]
+
+        def sparse_dense_layout():
+            hc.hc_mask_compact_rulebook(mask, sp, hc.HC_LAYOUT_DENSE, coords, row_of, offs,
+                                        count, rb_d, stream)
+            h = x
+            for i, ly in enumerate(w.layers):
+                last = i + 1 == len(w.layers)
+                taps = rb_d if ly.kind == "conv" else rb_d[0:1]  # centre slot: a 1x1 layer
+                if last:
+                    hc.hc_sparse_conv_rulebook_fwd(h, taps, count, Ws[i], bs[i], ly.act, out,
+                                                   stream=stream)
+                else:
+                    hc.hc_sparse_conv_rulebook_fwd(h, taps, count, Ws[i], bs[i], ly.act, None,
+                                                   coords=coords, out=dense_a[i], stream=stream)
+                h = dense_a[i]
+
         def dense():
             h = x
             for i, ly in enumerate(w.layers):
@@ -1169,7 +1195,11 @@ def run_configs(torch, hc, dev, stream, cpu_budget_s=3.0):
                                             dense_h[i].view(B * V, -1), stream)
                 h = dense_h[i]
 
-        t_sparse = _graph_time_us(torch, sparse, stream, dev)
+        t_compact = _graph_time_us(torch, sparse, stream, dev)
+        y_compact = out[:int(count.item())].clone()
+        t_dl = _graph_time_us(torch, sparse_dense_layout, stream, dev)
+        same = bool(torch.equal(out[:int(count.item())], y_compact))
+        t_sparse = min(t_compact, t_dl)
         t_dense = _graph_time_us(torch, dense, stream, dev)
         st = hc.hc_get_device_status(stream)
         if st != hc.HC_OK:
@@ -1194,8 +1224,9 @@ def run_configs(torch, hc, dev, stream, cpu_budget_s=3.0):
             "dense_us": t_dense, "speedup_vs_dense": t_dense / t_sparse,
             "oracle_1_thread": {"rows_per_s": o1, "frames": k1, "rows": n1, "cores": 1},
             "oracle_all_cores": {"rows_per_s": on, "frames": kn, "rows": nn, "cores": cores},
-            "chain": "compaction + Eq. 4 mapping + S' gather + every layer on compact rows "
-                     "(one CUDA graph)",
+            "chain": ("dense_layout" if t_dl < t_compact else "compact") + " (one CUDA graph)",
+            "chains_us": {"compact": t_compact, "dense_layout": t_dl},
+            "chains_same_output": same,
         }
     return res
 

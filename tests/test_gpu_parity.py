@@ -707,6 +707,41 @@ def test_encoder_end_to_end(name):
     check_close(got[:n], outs[-1][0], name)
 
 
+@pytest.mark.parametrize("name", ["layer655_f32", "encoder655_bf16", "motion655_bf16"])
+def test_dense_layout_chain_against_oracle(name):
+    """The configs' dense-layout chain: one dense-layout mapping, every conv
+    reading the previous layer's dense rows and writing only its active rows
+    into a dense tensor (fused scatter, no compact output), the per-vertex
+    head as the rulebook conv on the centre slot; the head's compact rows
+    against the oracle's stack, and the same bits as the compact chain."""
+    w = inputs.make_workload(name)
+    B, V = w.B, w.V
+    dt = torch.float32 if w.dtype == "f32" else torch.bfloat16
+    rb, coords, row_of, count = gpu_rulebook(w.masks[0], w.spiral, hc.HC_LAYOUT_DENSE)
+    h = to_torch(w.x)
+    for i, ly in enumerate(w.layers):
+        taps = rb if ly.kind == "conv" else rb[0:1]
+        if i + 1 == len(w.layers):
+            y = torch.full((B * V, ly.C_out), float("nan"), dtype=dt, device="cuda")
+            hc.hc_sparse_conv_rulebook_fwd(h, taps, count, to_torch(ly.W), to_torch(ly.b),
+                                           ly.act, y)
+            h = y
+        else:
+            d = torch.full((B, V, ly.C_out), float("nan"), dtype=dt, device="cuda")
+            hc.hc_sparse_conv_rulebook_fwd(h, taps, count, to_torch(ly.W), to_torch(ly.b),
+                                           ly.act, None, coords=coords, out=d)
+            h = d
+    assert hc.hc_get_device_status() == hc.HC_OK
+    n = int(count.item())
+    c, r, o, n_ref, outs = oracle.encoder(w.x, w.masks[0], w.spiral, w.layers, n_threads=NCPU)
+    assert n == n_ref
+    check_close(to_numpy(h)[:n], outs[-1][0], f"{name} dense-layout chain")
+    if len(w.layers) > 1:
+        got, n2 = run_encoder_gpu(w)
+        assert n2 == n
+        np.testing.assert_array_equal(to_numpy(h)[:n], got[:n])
+
+
 # ------------------------------------------------------------------ full size, sampled
 
 def test_layer10475_full_size_sampled():
