@@ -120,7 +120,8 @@ FUSED = [(3, 200, 9, 16, 64, 8),     # 8 channels per group, 4 groups per 32-col
 UNFUSED = [(3, 200, 9, 16, 64, 16),  # 4 channels per group
            (3, 200, 9, 16, 48, 2),   # 24 per group
            (2, 200, 9, 16, 256, 1),  # 256 per group, wider than a tile
-           (3, 200, 9, 16, 24, 3)]   # C_out/8 not a power of two
+           (3, 200, 9, 16, 24, 3),   # C_out/8 not a power of two
+           (3, 200, 9, 45, 48, 2)]   # padded channels, then the group norm's own workspace
 
 
 @pytest.mark.parametrize("shape", FUSED + UNFUSED)
