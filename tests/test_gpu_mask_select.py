@@ -54,12 +54,13 @@ def run_score(O_np, alpha_np, in_place=False):
 @pytest.mark.parametrize("K,N,D", [(2, 100, 8), (3, 1000, 64), (4, 777, 5), (5, 300, 1),
                                    (1, 50, 16), (6, 333, 130), (10, 4000, 42), (3, 64, 8),
                                    (2, 1, 3), (40, 500, 16), (10, 3000, 128), (9, 700, 130),
-                                   (11, 500, 101)])
+                                   (11, 500, 101), (10, 2000, 96), (8, 900, 121)])
 def test_mask_score(K, N, D, dtype):
-    """Multi-tile Gram matrices (K*D > 128; K*D >= 1024 takes the 256-wide
-    tensor-core tiles), ragged row counts, D a multiple of 8 (16-byte
-    pieces), even (4-byte pieces) and odd (the packed copy), D = 1, K = 1,
-    one row."""
+    """Multi-tile Gram matrices (K*D > 128; K*D >= 512 whose padding to 256
+    keeps >= 80% of the Gram useful takes the 256-wide tensor-core tiles:
+    1280, 1170, 960, 968 here; 1111, 780 and 640 stay on 128-wide tiles),
+    ragged row counts, D a multiple of 8 (16-byte pieces), even (4-byte
+    pieces) and odd (the packed copy), D = 1, K = 1, one row."""
     rng = np.random.default_rng(K * 1000 + N + D)
     O = _outputs(rng, K, N, D, dtype)
     alpha = rng.standard_normal(K)
