@@ -38,6 +38,15 @@
 //              next into every row of the freed accumulators, onto which its
 //              MMAs accumulate. Two accumulator sets (2*tm*BN TMEM columns)
 //              let the epilogue of one item overlap the main loop of the next.
+// The dense layer with 128 output channels and two-half items (TR) swaps the
+// operands: D^T = W^T A^T, one tcgen05.mma of M = 128 channels (the W slice,
+// MN-major, as staged) x N = 256 rows (the two halves of A, K-major, as
+// staged) per K16 step instead of two of 128 x 128, i.e. half the MMAs and
+// a quarter less shared-memory operand traffic per k-block (dense layer
+// 200.7 -> 181.6 us at 64 x 10475 rows, L = 9, 128 -> 128). Its accumulator
+// holds a channel per TMEM lane and a row per column, so the epilogue stages
+// each 32 x 32 block transposed through shared memory, and the bias is one
+// value per lane.
 // Each role runs its whole loop in a copy compiled for its half count (the
 // count is known once the row count is read); a run-time half loop between
 // the MMAs and copies cost ~1 us per launch at the small layers.
@@ -142,6 +151,21 @@ __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr, uint32_t lbo
 // in yk[k] and dk[k] (0 = not written).
 // Activation and bf16 rounding of a chunk: p[h] holds columns 2h (low
 // half) and 2h + 1 (high half).
+
+// Transposed epilogue chunk: lane = output channel, r[j] = row j of the
+// chunk; activation, bf16, written transposed into the warp's staging
+// buffer ([32 rows][32 channels] bf16).
+template <int ACT>
+__device__ __forceinline__ void tr_stage(const uint32_t (&r)[32], uint32_t stage, int lane) {
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+        const unsigned short v =
+            __bfloat16_as_ushort(__float2bfloat16_rn(act_fixed<ACT>(__uint_as_float(r[j]))));
+        asm volatile("st.shared.u16 [%0], %1;\n" ::"r"(stage + (uint32_t)(j * 64 + lane * 2)), "h"(v)
+                     : "memory");
+    }
+}
+
 template <int ACT>
 __device__ __forceinline__ void epilogue_pack(const uint32_t (&r)[32], uint32_t (&p)[16]) {
 #pragma unroll
@@ -331,10 +355,15 @@ __device__ __forceinline__ void gn_stats_chunk(const ConvArgs& a, const uint32_t
     }
 }
 
-template <int BN, int TM>
+template <int BN, int TM, bool TR>
 __global__ void __launch_bounds__(kThreadsFor<TM>, 1)
     conv_tc_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_w) {
     using C = Cfg<BN, TM>;
+    static_assert(!TR || (TM == 2 && BN == 128), "the transposed MMA takes 2 x 128 rows, 128 channels");
+    // transposed MMA: D fp32, A (W) bf16 MN-major (bit 15), B (rows) bf16
+    // K-major, N = 256 at bits 17-22, M = 128 at bits 24-28
+    constexpr uint32_t kIdescTR = (1u << 4) | (1u << 7) | (1u << 10) | (1u << 15) |
+                                  ((uint32_t)(256 >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
     constexpr int kTabRows = C::kTabRows;
     // "full": one cp.async completion arrival per producer thread, plus the
     // expect-tx arrival of the weight loader.
@@ -580,7 +609,19 @@ __global__ void __launch_bounds__(kThreadsFor<TM>, 1)
                     fence_proxy_async_smem();
                     const uint32_t a_st = a_stage(s);
                     const uint32_t b_st = b_stage(s);
-                    {
+                    if constexpr (TR) {
+                        // A operand: the W slice (MN-major, M = 128 output
+                        // channels); B operand: the item's 256 gathered rows
+                        // (K-major, N = 256, both halves contiguous)
+#pragma unroll
+                        for (int k = 0; k < kBK / 16; ++k) {
+                            const uint64_t wd =
+                                smem_desc_sw128(b_st + k * 16 * 128, kBK * 128, 1024);
+                            const uint64_t rd = smem_desc_sw128(a_st + k * 32, 16, 1024);
+                            const uint32_t acc_in = (has_bias || (kb | k) != 0) ? 1u : 0u;
+                            tc_mma_bf16(d_tmem, wd, rd, kIdescTR, acc_in);
+                        }
+                    } else {
 #pragma unroll
                         for (int k = 0; k < kBK / 16; ++k) {
                             const uint64_t bd =
@@ -773,7 +814,54 @@ __global__ void __launch_bounds__(kThreadsFor<TM>, 1)
         // ------------------------------------------------------------ epilogue
         const int ew = warp - kProducerWarps;  // == warp % 4: TMEM lanes 32*ew..+32
         __nv_bfloat16* __restrict__ y = static_cast<__nv_bfloat16*>(a.y);
-        {
+        if constexpr (TR) {
+        // TMEM lane = output channel 32*ew + lane, column = row of the item
+        const uint32_t t_lane = tmem_base + ((uint32_t)(ew * 32) << 16);
+        auto release_tr = [&](int acc, long long w) {
+            if (a.bias && w < work_total) {
+                const uint32_t bv = __float_as_uint(__ldg(a.bias + 32 * ew + lane));
+                uint32_t r[32];
+#pragma unroll
+                for (int j = 0; j < 32; ++j) r[j] = bv;
+#pragma unroll 1
+                for (int cb = 0; cb < 8; ++cb)
+                    tmem_st_32x32b_x32(t_lane + (uint32_t)(acc * 256 + cb * 32), r);
+                tmem_st_wait();
+            }
+            tc_fence_before();
+            mbar_arrive(tempty_bar(acc));
+        };
+        release_tr(0, blockIdx.x);
+        release_tr(1, blockIdx.x + (long long)gridDim.x);
+        const uint32_t stage = epi0 + (uint32_t)ew * 2048u;
+        int lt = 0;
+        for (long long w = blockIdx.x; w < work_total; w += gridDim.x, ++lt) {
+            const long long m_item = (long long)((int)w / n_tiles) * item_rows;
+            const int acc = lt & 1;
+            if (!mbar_wait(tfull_bar(acc), (uint32_t)((lt >> 1) & 1), abort_flag, a.status)) break;
+            tc_fence_after();
+#pragma unroll 1
+            for (int cb = 0; cb < 8; ++cb) {
+                uint32_t r[32];
+                tmem_ld_32x32b_x32(t_lane + (uint32_t)(acc * 256 + cb * 32), r);
+                tmem_ld_wait();
+                if (a.act == HC_ACT_ELU) tr_stage<HC_ACT_ELU>(r, stage, lane);
+                else if (a.act == HC_ACT_RELU) tr_stage<HC_ACT_RELU>(r, stage, lane);
+                else tr_stage<HC_ACT_NONE>(r, stage, lane);
+                __syncwarp();
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const int j = (lane >> 2) + 8 * q, p = lane & 3;
+                    const uint4 v = lds_u4(stage + (uint32_t)(j * 64 + p * 16));
+                    const long long row = m_item + cb * 32 + j;
+                    if (y && row < rows)
+                        *reinterpret_cast<uint4*>(y + row * C_out + 32 * ew + 8 * p) = v;
+                }
+                __syncwarp();
+            }
+            release_tr(acc, w + 2 * (long long)gridDim.x);
+        }
+        } else {
         // Accumulator buffer acc is handed to the MMA warp holding the bias of
         // tile w in every row (the MMAs then accumulate onto it), so the bias
         // costs the epilogue nothing once the sums are ready.
@@ -993,12 +1081,12 @@ hc_status encode_w3d(CUtensorMap* m, const void* base, long long K, long long C_
     return HC_OK;
 }
 
-template <int BN, int TM>
+template <int BN, int TM, bool TR = false>
 hc_status launch_bn(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s) {
     using C = Cfg<BN, TM>;
     static bool attr_set[64] = {};
     if (!attr_set[ctx->device]) {
-        hc_status st = check_cuda(cudaFuncSetAttribute(conv_tc_kernel<BN, TM>,
+        hc_status st = check_cuda(cudaFuncSetAttribute(conv_tc_kernel<BN, TM, TR>,
                                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                        (int)kSmemLimit),
                                   "cudaFuncSetAttribute(conv_tc_kernel)");
@@ -1024,7 +1112,7 @@ hc_status launch_bn(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s) {
     long long grid = cap_work < ctx->num_sms ? cap_work : ctx->num_sms;
     if (grid < 1) grid = 1;
     ka.stages = C::stages_for(a.L);
-    return launch_pdl(conv_tc_kernel<BN, TM>, dim3((unsigned)grid), dim3(kThreadsFor<TM>),
+    return launch_pdl(conv_tc_kernel<BN, TM, TR>, dim3((unsigned)grid), dim3(kThreadsFor<TM>),
                       C::smem_bytes(a.L, ka.stages), s, "conv_tc_kernel", ka, tw);
 }
 
@@ -1096,7 +1184,9 @@ hc_status launch_conv_tc(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s
     const bool two = a.mode == kDense && (a.capacity + 2 * kBM - 1) / (2 * kBM) * n_tiles >=
                                              2ll * ctx->num_sms;
     if (conv_tc_tile_n(a) == 64) return launch_bn<64, 1>(ctx, a, s);
-    return two ? launch_bn<128, 2>(ctx, a, s) : launch_bn<128, 1>(ctx, a, s);
+    return two ? (a.C_out == 128 && !a.out_dense && !a.gn_part ? launch_bn<128, 2, true>(ctx, a, s)
+                                                                : launch_bn<128, 2, false>(ctx, a, s))
+               : launch_bn<128, 1, false>(ctx, a, s);
 }
 
 }  // namespace hc

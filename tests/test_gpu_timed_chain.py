@@ -94,6 +94,32 @@ def test_sweep_call_full_size(density):
     check_close(y[rows], y_pre, f"sweep density {density}")
 
 
+@pytest.mark.parametrize("act,bias", [(oracle.ACT_ELU, True), (oracle.ACT_RELU, False),
+                                      (oracle.ACT_NONE, True)])
+def test_dense_layer_transposed_mma(act, bias):
+    """The dense layer with 128 output channels and enough rows for two-half
+    items (at least two per SM) takes the transposed MMA (W^T times the
+    gathered rows: lanes = channels, columns = rows); 79,999 rows leave the
+    last item ragged. Every row against the oracle, for each activation,
+    with and without bias, and rows past B*V untouched."""
+    B, V, L, C_in = 1, 79999, 9, 32
+    rng = np.random.default_rng(11 + act)
+    sp = rng.integers(0, V, size=(V, L)).astype(np.int32)
+    sp[:, 0] = np.arange(V)
+    sp[rng.random((V, L)) < 0.1] = -1
+    sp[:, 0] = np.arange(V)
+    x = inputs.features(rng, (B, V, C_in), "bf16")
+    W = inputs.weights(rng, L * C_in, 128, "bf16")
+    b = rng.standard_normal(128).astype(np.float32) if bias else None
+    yd = torch.full((B * V + 7, 128), float("nan"), dtype=torch.bfloat16, device="cuda")
+    hc.hc_spiral_conv_fwd(to_torch(x), to_torch(sp), to_torch(W), None if b is None else to_torch(b),
+                          act, yd[:B * V].view(B, V, 128))
+    assert hc.hc_get_device_status() == hc.HC_OK
+    y_pre, _ = oracle.dense_spiral_conv(x, sp, W, b, act, n_threads=NCPU)
+    check_close(to_numpy(yd)[:B * V], y_pre, f"dense transposed act={act} bias={bias}")
+    assert torch.isnan(yd[B * V:].float()).all()
+
+
 @pytest.mark.parametrize("name", ["sweep10475_bf16", "layer10475_bf16"])
 def test_dense_layer_full_size(name):
     """The dense layer of the speed-up denominators on 10k sampled rows."""
