@@ -688,7 +688,10 @@ def run_sweep(torch, hc, dev, stream):
     sparse conv (compaction and Eq. 4 mapping done beforehand) against the
     dense layer. tensor_frac counts the work the kernel issues (every tap of
     every active row, absent taps as zero rows: the dense-K formulation);
-    tensor_frac_present only the present taps' work (Eq. 5's sum)."""
+    tensor_frac_present only the present taps' work (Eq. 5's sum). The
+    *_hinted fields time hc_sparse_conv_rulebook_fwd_hint with the mask's
+    row count (known here on the host, where the mask was made) as the
+    estimate: same results, the tiling chosen for that many rows."""
     from paper_2608_09388_gb300 import inputs
     w = inputs.make_workload("sweep10475_bf16")
     ly = w.layers[0]
@@ -732,6 +735,8 @@ def run_sweep(torch, hc, dev, stream):
         n = int(np.count_nonzero(m))
         ms = timeit(lambda: hc.hc_sparse_conv_rulebook_fwd(x, rb, count, Wt, bias, ly.act, y,
                                                            stream=stream))
+        ms_h = timeit(lambda: hc.hc_sparse_conv_rulebook_fwd_hint(x, rb, count, Wt, bias, ly.act,
+                                                                  y, n, stream=stream))
         per_tap = 2.0 * ly.C_in * ly.C_out
         fl = per_tap * L * n
         present = per_tap * float((rb[:, :n] >= 0).sum().item())
@@ -741,7 +746,9 @@ def run_sweep(torch, hc, dev, stream):
                     "rows_per_s": n / (ms * 1e-3),
                     "work_present_of_issued": present / fl,
                     "tensor_frac": tf(fl, ms),
-                    "tensor_frac_present": tf(present, ms)})
+                    "tensor_frac_present": tf(present, ms),
+                    "sparse_hinted_us": ms_h * 1e3, "speedup_hinted": dense_ms / ms_h,
+                    "tensor_frac_hinted": tf(fl, ms_h)})
     st = hc.hc_get_device_status(stream)
     if st != hc.HC_OK:
         raise RuntimeError(f"device status {hc.STATUS_NAMES.get(st)} in the sweep")

@@ -217,6 +217,27 @@ hc_status hc_sparse_conv_rulebook_fwd(const void* x, hc_dtype dt, int x_rows,
                                       void* out, hc_stream_t stream);
 
 /*
+ * hc_sparse_conv_rulebook_fwd_hint -- hc_sparse_conv_rulebook_fwd with the
+ * caller's host-side estimate of N' (rows_hint >= 0; 0 = unknown), which
+ * the call uses only to choose how the tensor cores tile the rows: N' lives
+ * on the device, and the tiling that is fastest for many rows (two 128-row
+ * halves per item sharing every weight stage, multiplied as one
+ * M = 128 channels x N = 256 rows product) is slower when there are too few
+ * items to fill the GPU. It is taken when rows_hint gives at least two such
+ * items per SM (about 78k rows on 152 SMs), for bf16, C_out = 128, and
+ * neither out nor group-norm statistics; otherwise the call is
+ * hc_sparse_conv_rulebook_fwd. The results are bit-identical either way, so
+ * any estimate (the previous batch's count, the mask's expected density) is
+ * safe: a wrong one only costs time. rows_hint < 0 is HC_ERR_INVALID_ARG.
+ */
+hc_status hc_sparse_conv_rulebook_fwd_hint(const void* x, hc_dtype dt, int x_rows,
+                                           const int32_t* rulebook, const int32_t* count,
+                                           int capacity, int L, int C_in, int C_out,
+                                           const void* W, const float* bias, hc_act act, void* y,
+                                           const int32_t* coords, int B, int V, void* out,
+                                           long long rows_hint, hc_stream_t stream);
+
+/*
  * hc_sparse_linear_fwd -- linear layer on compact rows (Eq. 6), row-wise
  *   y[n, o] = act( bias[o] + sum_{c<C_in} x[n, c] * W[c*C_out + o] ),  n < N'
  * The coordinates are unchanged (C' = C).

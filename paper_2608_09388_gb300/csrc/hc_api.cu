@@ -326,13 +326,13 @@ hc_status hc_mask_compact_rulebook(const uint8_t* mask, int B, int V, const int3
     return launch_rulebook(ctx, coords, row_of, count, spiral, B, V, L, (int)x_layout, rulebook, s);
 }
 
-hc_status hc_sparse_conv_rulebook_fwd(const void* x, hc_dtype dt, int x_rows,
-                                      const int32_t* rulebook, const int32_t* count, int capacity,
-                                      int L, int C_in, int C_out, const void* W, const float* bias,
-                                      hc_act act, void* y, const int32_t* coords, int B, int V,
-                                      void* out, hc_stream_t stream) {
-    const char* fn = "hc_sparse_conv_rulebook_fwd";
-    t_last_error[0] = 0;
+}  // extern "C"
+
+static hc_status conv_rulebook(const char* fn, const void* x, hc_dtype dt, int x_rows,
+                               const int32_t* rulebook, const int32_t* count, int capacity, int L,
+                               int C_in, int C_out, const void* W, const float* bias, hc_act act,
+                               void* y, const int32_t* coords, int B, int V, void* out,
+                               long long rows_hint, cudaStream_t stream) {
     HC_REQUIRE(y || out, "%s: at least one of y and out is required", fn);
     hc_status st = check_conv_common(fn, dt, L, C_in, C_out, act, x, W, y ? y : out);
     if (st != HC_OK) return st;
@@ -367,7 +367,34 @@ hc_status hc_sparse_conv_rulebook_fwd(const void* x, hc_dtype dt, int x_rows,
     a.out_coords = coords;
     a.out_B = B;
     a.out_V = V;
-    return dispatch_conv(ctx, a, dt, (cudaStream_t)stream);
+    a.rows_hint = rows_hint;
+    return dispatch_conv(ctx, a, dt, stream);
+}
+
+extern "C" {
+
+hc_status hc_sparse_conv_rulebook_fwd(const void* x, hc_dtype dt, int x_rows,
+                                      const int32_t* rulebook, const int32_t* count, int capacity,
+                                      int L, int C_in, int C_out, const void* W, const float* bias,
+                                      hc_act act, void* y, const int32_t* coords, int B, int V,
+                                      void* out, hc_stream_t stream) {
+    t_last_error[0] = 0;
+    return conv_rulebook("hc_sparse_conv_rulebook_fwd", x, dt, x_rows, rulebook, count, capacity,
+                         L, C_in, C_out, W, bias, act, y, coords, B, V, out, 0,
+                         (cudaStream_t)stream);
+}
+
+hc_status hc_sparse_conv_rulebook_fwd_hint(const void* x, hc_dtype dt, int x_rows,
+                                           const int32_t* rulebook, const int32_t* count,
+                                           int capacity, int L, int C_in, int C_out,
+                                           const void* W, const float* bias, hc_act act, void* y,
+                                           const int32_t* coords, int B, int V, void* out,
+                                           long long rows_hint, hc_stream_t stream) {
+    const char* fn = "hc_sparse_conv_rulebook_fwd_hint";
+    t_last_error[0] = 0;
+    HC_REQUIRE(rows_hint >= 0, "%s: rows_hint=%lld must be >= 0", fn, rows_hint);
+    return conv_rulebook(fn, x, dt, x_rows, rulebook, count, capacity, L, C_in, C_out, W, bias,
+                         act, y, coords, B, V, out, rows_hint, (cudaStream_t)stream);
 }
 
 hc_status hc_sparse_group_norm_fwd(const void* x, hc_dtype dt, const int32_t* batch_offsets, int B,

@@ -97,6 +97,9 @@ struct ConvArgs {
     const int32_t* gn_coords;
     int gn_G, gn_B;
     int gn_cpg;  // channels per group, C_out / gn_G: 8, 16, 32, 64 or 128
+    // Host-side estimate of the active row count (rulebook mode; 0 =
+    // unknown): it only chooses the tensor-core kernel's item shape.
+    long long rows_hint;
     // Tensor-core kernel with C_in not a multiple of 8: workspace of at
     // least conv_tc_pad_bytes(a) bytes (256-byte aligned) for x and W with
     // zero channels appended up to a multiple of 8.

@@ -30,7 +30,8 @@ STATUS_NAMES = {0: "HC_OK", 1: "HC_ERR_INVALID_ARG", 2: "HC_ERR_UNSUPPORTED",
 
 # Exported symbols, as declared in include/hc.h.
 EXPORTS = ("hc_mask_compact", "hc_mask_compact_static", "hc_sparse_spiral_conv_fwd",
-           "hc_conv_rulebook", "hc_mask_compact_rulebook", "hc_sparse_conv_rulebook_fwd", "hc_sparse_linear_fwd",
+           "hc_conv_rulebook", "hc_mask_compact_rulebook", "hc_sparse_conv_rulebook_fwd",
+           "hc_sparse_conv_rulebook_fwd_hint", "hc_sparse_linear_fwd",
            "hc_sparse_group_norm_fwd", "hc_sparse_conv_gn_fwd", "hc_mask_score_update", "hc_mask_select_topk",
            "hc_kappa_masks", "hc_gather_rows", "hc_conv_rulebook_transpose",
            "hc_sparse_conv_rulebook_bwd", "hc_scatter_dense", "hc_spiral_conv_fwd", "hc_get_device_status",
@@ -66,6 +67,8 @@ def load_library(path: str | None = None):
             "hc_mask_compact_rulebook": [P, I, I, P, I, I, P, P, P, P, P, P],
             "hc_sparse_conv_rulebook_fwd": [P, I, I, P, P, I, I, I, I, P, P, I, P, P, I, I, P,
                                             P],
+            "hc_sparse_conv_rulebook_fwd_hint": [P, I, I, P, P, I, I, I, I, P, P, I, P, P, I, I,
+                                                 P, ctypes.c_longlong, P],
             "hc_sparse_linear_fwd": [P, I, P, I, I, I, P, P, I, P, P],
             "hc_sparse_group_norm_fwd": [P, I, P, I, I, I, I, ctypes.c_float, P, P, I, P, P],
             "hc_sparse_conv_gn_fwd": [P, I, I, P, P, I, I, I, I, P, P, P, P, I, I,
@@ -197,6 +200,21 @@ def hc_sparse_conv_rulebook_fwd(x, rulebook, count, W, bias, act, y, coords=None
         _p(x), _dt(x if y is None else y), x_rows, _p(rulebook), _p(count), capacity, L, C_in,
         C_out, _p(W), _p(bias), act, _p(y), _p(coords), B, V, _p(out), _s(stream)),
         "hc_sparse_conv_rulebook_fwd")
+
+
+def hc_sparse_conv_rulebook_fwd_hint(x, rulebook, count, W, bias, act, y, rows_hint,
+                                     coords=None, out=None, stream=None):
+    """hc_sparse_conv_rulebook_fwd with a host-side estimate of N' (an int >= 0,
+    0 = unknown) that only chooses the tensor-core tiling; same results."""
+    L, capacity = rulebook.shape
+    C_in = x.shape[-1]
+    x_rows = x.numel() // C_in
+    C_out = W.shape[1]
+    B, V = (out.shape[0], out.shape[1]) if out is not None else (0, 0)
+    _check(load_library().hc_sparse_conv_rulebook_fwd_hint(
+        _p(x), _dt(x if y is None else y), x_rows, _p(rulebook), _p(count), capacity, L, C_in,
+        C_out, _p(W), _p(bias), act, _p(y), _p(coords), B, V, _p(out), int(rows_hint),
+        _s(stream)), "hc_sparse_conv_rulebook_fwd_hint")
 
 
 def hc_sparse_linear_fwd(x, count, W, bias, act, y, stream=None):

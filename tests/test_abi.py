@@ -58,6 +58,16 @@ def test_invalid_arguments_rejected_on_host(lib):
     # unknown activation
     assert lib.hc_spiral_conv_fwd(fake, 1, fake, 1, 4, 3, 8, 8, fake, None, 9, fake,
                                   None) == hc.HC_ERR_INVALID_ARG
+    # a negative row estimate
+    lib.hc_sparse_conv_rulebook_fwd_hint.argtypes = [P, ctypes.c_int, ctypes.c_int, P, P,
+                                                     ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                                                     ctypes.c_int, P, P, ctypes.c_int, P, P,
+                                                     ctypes.c_int, ctypes.c_int, P,
+                                                     ctypes.c_longlong, P]
+    assert lib.hc_sparse_conv_rulebook_fwd_hint(fake, 1, 10, fake, fake, 10, 9, 16, 128, fake,
+                                                None, 1, fake, None, 0, 0, None, -1,
+                                                None) == hc.HC_ERR_INVALID_ARG
+    assert "rows_hint" in hc.hc_last_error_string()
     # misaligned pointer for the element size
     assert lib.hc_spiral_conv_fwd(P(0x1001), 1, fake, 1, 4, 3, 8, 8, fake, None, 1, fake,
                                   None) == hc.HC_ERR_INVALID_ARG

@@ -53,6 +53,20 @@ def _chain(mask, x, spiral, W, bias, act, out_fill=None):
     return n, to_numpy(coords)[:n], to_numpy(y), None if out is None else to_numpy(out)
 
 
+def _rulebook(mask, spiral):
+    """Compaction + Eq. 4 mapping (dense layout): rulebook, coords, row_of, count."""
+    B, V = mask.shape
+    L = spiral.shape[1]
+    coords = torch.empty((B * V, 2), dtype=torch.int32, device="cuda")
+    row_of = torch.empty((B, V), dtype=torch.int32, device="cuda")
+    offs = torch.empty((B + 1,), dtype=torch.int32, device="cuda")
+    count = torch.empty((1,), dtype=torch.int32, device="cuda")
+    rb = torch.empty((L, B * V), dtype=torch.int32, device="cuda")
+    hc.hc_mask_compact_rulebook(to_torch(mask), to_torch(spiral), hc.HC_LAYOUT_DENSE, coords,
+                                row_of, offs, count, rb)
+    return rb, coords, row_of, count
+
+
 def test_bench_step_every_row():
     """The 10475-vertex layer (32 clustered frames, L = 12, 64 -> 128, ELU):
     every active row of the compact output and of the dense scatter against
@@ -118,6 +132,35 @@ def test_dense_layer_transposed_mma(act, bias):
     y_pre, _ = oracle.dense_spiral_conv(x, sp, W, b, act, n_threads=NCPU)
     check_close(to_numpy(yd)[:B * V], y_pre, f"dense transposed act={act} bias={bias}")
     assert torch.isnan(yd[B * V:].float()).all()
+
+
+@pytest.mark.parametrize("density", [0.01, 0.1, 0.5, 1.0])
+def test_row_hint_same_bits(density):
+    """hc_sparse_conv_rulebook_fwd_hint on the density sweep's layer: with the
+    exact count as the estimate (two-half transposed items from 10% up, the
+    one-half kernel at 1%), with a wrong one in each direction, and with
+    none, every row is bit-identical to hc_sparse_conv_rulebook_fwd; the
+    oracle on 3000 sampled rows; rows past N' untouched."""
+    w = inputs.make_workload("sweep10475_bf16")
+    ly = w.layers[0]
+    m = w.masks[list(w.densities).index(density)]
+    B, V = m.shape
+    rb, coords, row_of, count = _rulebook(m, w.spiral)
+    n = int(count.item())
+    xt, Wt, bt = to_torch(w.x), to_torch(ly.W), to_torch(ly.b)
+    ref = torch.full((B * V, 128), float("nan"), dtype=torch.bfloat16, device="cuda")
+    hc.hc_sparse_conv_rulebook_fwd(xt, rb, count, Wt, bt, ly.act, ref)
+    for hint in (n, 0, B * V, 1000):
+        y = torch.full((B * V, 128), float("nan"), dtype=torch.bfloat16, device="cuda")
+        hc.hc_sparse_conv_rulebook_fwd_hint(xt, rb, count, Wt, bt, ly.act, y, hint)
+        assert hc.hc_get_device_status() == hc.HC_OK
+        assert torch.equal(y[:n], ref[:n]), f"hint {hint}"
+        assert torch.isnan(y[n:].float()).all()
+    c, r, _, _ = oracle.mask_compact(m)
+    rows = sample_rows(n, 3000, seed=12)
+    y_pre, _ = oracle.sparse_spiral_conv(w.x, oracle.LAYOUT_DENSE, c, r, w.spiral, ly.W, ly.b,
+                                         ly.act, rows=rows, n_threads=NCPU)
+    check_close(to_numpy(ref)[rows], y_pre, f"hinted sweep {density}")
 
 
 @pytest.mark.parametrize("name", ["sweep10475_bf16", "layer10475_bf16"])
