@@ -223,8 +223,8 @@ hc_status hc_sparse_conv_rulebook_fwd(const void* x, hc_dtype dt, int x_rows,
  * on the device, and the tiling that is fastest for many rows (two 128-row
  * halves per item sharing every weight stage, multiplied as one
  * M = 128 channels x N = 256 rows product) is slower when there are too few
- * items to fill the GPU. It is taken when rows_hint gives at least two such
- * items per SM (about 78k rows on 152 SMs), for bf16, C_out = 128, and
+ * items to fill the GPU. It is taken when rows_hint gives at least one such
+ * item per SM (about 39k rows on 152 SMs), for bf16, C_out = 128, and
  * neither out nor group-norm statistics; otherwise the call is
  * hc_sparse_conv_rulebook_fwd. The results are bit-identical either way, so
  * any estimate (the previous batch's count, the mask's expected density) is

@@ -1183,13 +1183,14 @@ hc_status launch_conv_tc(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s
     const long long n_tiles = (a.C_out + 127) / 128;
     const bool two = a.mode == kDense && (a.capacity + 2 * kBM - 1) / (2 * kBM) * n_tiles >=
                                              2ll * ctx->num_sms;
-    // A sparse call whose caller expects enough rows for two two-half items
-    // per SM (rows_hint) runs them too, with the transposed product (128
-    // output channels, no fused scatter or statistics): 250 -> 179 us at
-    // 670k rows, 32 -> 28 us at 67k; at 6.8k rows (27 items) they were
-    // 11 -> 18 us, hence the threshold. The results are the same either way.
+    // A sparse call whose caller expects at least one two-half item per SM
+    // (rows_hint) runs them too, with the transposed product (128 output
+    // channels, no fused scatter or statistics): 250 -> 179 us at 670k rows,
+    // 32 -> 28 us at 67k rows (1.7 items per SM), the same at 33k (0.9 per
+    // SM), 11 -> 18 us at 6.8k (0.2 per SM). The results are the same either
+    // way.
     if (a.mode == kRulebook && a.C_out == 128 && !a.out_dense && !a.gn_part &&
-        a.C_in % 8 == 0 && (a.rows_hint + 2 * kBM - 1) / (2 * kBM) >= 2ll * ctx->num_sms)
+        a.C_in % 8 == 0 && (a.rows_hint + 2 * kBM - 1) / (2 * kBM) >= ctx->num_sms)
         return launch_bn<128, 2, true>(ctx, a, s);
     if (conv_tc_tile_n(a) == 64) return launch_bn<64, 1>(ctx, a, s);
     return two ? (a.C_out == 128 && !a.out_dense && !a.gn_part ? launch_bn<128, 2, true>(ctx, a, s)
