@@ -233,65 +233,10 @@ __device__ __forceinline__ long long active_rows(const ConvArgs& a) {
     return n;
 }
 
-// Output row n -> coordinate (b, v). Returns false (setting kErrIndex in
-// `err`) for an out-of-range coordinate; linear rows have no coordinate.
-__device__ __forceinline__ bool row_coord(const ConvArgs& a, long long n, int& b, int& v,
-                                          unsigned& err) {
-    if (a.mode == kDense) {
-        b = (int)(n / a.V);
-        v = (int)(n - (long long)b * a.V);
-        return true;
-    }
-    if (a.mode == kLinear || a.mode == kRulebook) {
-        b = 0;
-        v = 0;
-        return true;
-    }
-    b = __ldg(a.coords + 2 * n);
-    v = __ldg(a.coords + 2 * n + 1);
-    if (b < 0 || b >= a.B || v < 0 || v >= a.V) {
-        err |= kErrIndex;
-        return false;
-    }
-    return true;
-}
-
 // The helpers below never write memory: they return an error bit instead
 // (kErrIndex), which callers OR together and report once. A global atomic
 // between loads would stop the compiler from issuing the loads of many taps
 // back to back.
-
-// Spiral entry of slot l of vertex v (-1 = no neighbour). Out-of-range
-// entries read as -1 and set kErrIndex in `err`.
-__device__ __forceinline__ int load_spiral(const ConvArgs& a, int v, int l, unsigned& err) {
-    int u = __ldg(a.spiral + (long long)v * a.L + l);
-    if (u < -1 || u >= a.V) {
-        err |= kErrIndex;
-        return -1;
-    }
-    return u;
-}
-
-// Input row for neighbour vertex u of output row n at frame b, or -1 when the
-// tap is absent (no neighbour, or the neighbour is not an active row). This
-// is idx() of Eq. 4 for the sparse modes.
-__device__ __forceinline__ long long resolve_tap(const ConvArgs& a, long long n, int b, int u,
-                                                 long long n_rows, unsigned& err) {
-    if (a.mode == kLinear) return n;
-    if (u < 0) return -1;
-    long long dense_row = (long long)b * a.V + u;
-    if (a.mode == kDense) return dense_row;
-    int j = __ldg(a.row_of + dense_row);
-    if (j < 0) {
-        if (j != -1) err |= kErrIndex;
-        return -1;
-    }
-    if (j >= n_rows) {
-        err |= kErrIndex;
-        return -1;
-    }
-    return a.mode == kSparseDenseX ? dense_row : (long long)j;
-}
 
 // Activation of Eq. 10. ELU(z) = z for z > 0, else exp(z) - 1, written
 // without a branch as max(z, 0) + (exp(min(z, 0)) - 1): for z > 0 the second
@@ -360,13 +305,6 @@ __device__ __forceinline__ void cp_async_4(uint32_t dst, const void* src, bool v
 // count includes it).
 __device__ __forceinline__ void cp_async_arrive_noinc(uint32_t bar) {
     asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];\n" ::"r"(bar) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() {
-    asm volatile("cp.async.commit_group;\n" ::: "memory");
-}
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-    asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory");
 }
 __device__ __forceinline__ void cp_async_wait_all() {
     asm volatile("cp.async.wait_all;\n" ::: "memory");
@@ -455,37 +393,8 @@ __device__ __forceinline__ void tma_load_3d(uint32_t dst, const void* tmap, int 
         "l"(reinterpret_cast<uint64_t>(tmap)), "r"(c0), "r"(c1), "r"(c2), "r"(bar)
         : "memory");
 }
-// Four rows (r0..r3) of a box one row high, starting at column c0, written to
-// consecutive box rows in shared memory. Rows outside the tensor read zeros.
-__device__ __forceinline__ void tma_gather4(uint32_t dst, const void* tmap, int c0, int r0, int r1,
-                                            int r2, int r3, uint32_t bar) {
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.tile::gather4.mbarrier::complete_tx::bytes"
-        " [%0], [%1, {%2, %3, %4, %5, %6}], [%7];\n" ::"r"(dst),
-        "l"(reinterpret_cast<uint64_t>(tmap)), "r"(c0), "r"(r0), "r"(r1), "r"(r2), "r"(r3),
-        "r"(bar)
-        : "memory");
-}
 __device__ __forceinline__ void prefetch_tensormap(const void* tmap) {
     asm volatile("prefetch.tensormap [%0];\n" ::"l"(reinterpret_cast<uint64_t>(tmap)) : "memory");
-}
-// ---- bulk copies shared -> global (TMA engine), tracked per thread in
-// bulk async-groups
-__device__ __forceinline__ void bulk_store(void* gdst, uint32_t ssrc, uint32_t bytes) {
-    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;\n" ::"l"(gdst),
-                 "r"(ssrc), "r"(bytes)
-                 : "memory");
-}
-__device__ __forceinline__ void bulk_commit() {
-    asm volatile("cp.async.bulk.commit_group;\n" ::: "memory");
-}
-// Every bulk copy of this thread has finished reading shared memory.
-__device__ __forceinline__ void bulk_wait_read_all() {
-    asm volatile("cp.async.bulk.wait_group.read 0;\n" ::: "memory");
-}
-// Every bulk copy of this thread has completed.
-__device__ __forceinline__ void bulk_wait_all() {
-    asm volatile("cp.async.bulk.wait_group 0;\n" ::: "memory");
 }
 __device__ __forceinline__ void sts_v4(uint32_t addr, uint4 v) {
     asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};\n" ::"r"(addr), "r"(v.x), "r"(v.y),
@@ -498,13 +407,6 @@ __device__ __forceinline__ uint4 lds_u4(uint32_t addr) {
                  : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
                  : "r"(addr)
                  : "memory");
-    return v;
-}
-__device__ __forceinline__ int4 lds_v4(uint32_t addr) {
-    int4 v;
-    asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];\n"
-                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-                 : "r"(addr));
     return v;
 }
 
@@ -534,17 +436,6 @@ __device__ __forceinline__ void tc_mma_bf16(uint32_t d_tmem, uint64_t a_desc, ui
         "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
         " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
         "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
-        : "memory");
-}
-// The same, accumulating onto D, with the rows (TMEM lanes) whose bit is set
-// in the 128-bit `disable` (word i, bit r: lane 32 i + r) left unchanged.
-__device__ __forceinline__ void tc_mma_bf16_masked(uint32_t d_tmem, uint64_t a_desc,
-                                                   uint64_t b_desc, uint32_t idesc, uint4 disable) {
-    asm volatile(
-        "{\n .reg .pred p;\n setp.ne.b32 p, 1, 0;\n"
-        " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, {%4, %5, %6, %7}, p;\n}\n" ::"r"(d_tmem),
-        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(disable.x), "r"(disable.y), "r"(disable.z),
-        "r"(disable.w)
         : "memory");
 }
 // Arrive once on `bar` when every tcgen05 op issued so far by this thread
