@@ -163,6 +163,41 @@ def test_row_hint_same_bits(density):
     check_close(to_numpy(ref)[rows], y_pre, f"hinted sweep {density}")
 
 
+@pytest.mark.parametrize("L,C_in,act,bias,density", [
+    (9, 64, oracle.ACT_ELU, True, 0.4),
+    (9, 45, oracle.ACT_RELU, False, 0.4),   # channel-padded input, then the two-half items
+    (12, 128, oracle.ACT_NONE, True, 0.3),
+    (1, 16, oracle.ACT_ELU, True, 0.5),     # one slot: a single k-block
+    (5, 200, oracle.ACT_ELU, True, 0.2),    # K = 1000: a ragged last k-block
+    (9, 64, oracle.ACT_ELU, True, 0.0),     # no active rows
+])
+def test_row_hint_forces_two_half_items_on_small_calls(L, C_in, act, bias, density):
+    """A row estimate far above the real count makes small calls run the
+    two-half transposed items (few items, the last ragged): every row
+    against the oracle and bit-identical to the default call; rows past N'
+    untouched."""
+    sp, m, x, W, b = inputs.random_case(L * 100 + C_in + int(density * 10), 3, 1001, L, C_in,
+                                        128, "bf16", density, neg_frac=0.1)
+    if not bias:
+        b = None
+    B, V = m.shape
+    rb, coords, row_of, count = _rulebook(m, sp)
+    n = int(count.item())
+    xt, Wt, bt = to_torch(x), to_torch(W), None if b is None else to_torch(b)
+    ref = torch.full((B * V, 128), float("nan"), dtype=torch.bfloat16, device="cuda")
+    hc.hc_sparse_conv_rulebook_fwd(xt, rb, count, Wt, bt, act, ref)
+    y = torch.full((B * V, 128), float("nan"), dtype=torch.bfloat16, device="cuda")
+    hc.hc_sparse_conv_rulebook_fwd_hint(xt, rb, count, Wt, bt, act, y, 10 ** 7)
+    assert hc.hc_get_device_status() == hc.HC_OK
+    assert torch.equal(y[:n], ref[:n])
+    assert torch.isnan(y[n:].float()).all()
+    if n:
+        c, r, _, _ = oracle.mask_compact(m)
+        y_pre, _ = oracle.sparse_spiral_conv(x, oracle.LAYOUT_DENSE, c, r, sp, W, b, act,
+                                             n_threads=NCPU)
+        check_close(to_numpy(y)[:n], y_pre, f"hinted L={L} C_in={C_in}")
+
+
 @pytest.mark.parametrize("name", ["sweep10475_bf16", "layer10475_bf16"])
 def test_dense_layer_full_size(name):
     """The dense layer of the speed-up denominators on 10k sampled rows."""
