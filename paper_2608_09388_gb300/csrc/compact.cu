@@ -29,6 +29,21 @@ __device__ __forceinline__ uint32_t nonzero_bytes(uint32_t w) {
     return (((w & 0x7F7F7F7Fu) + 0x7F7F7F7Fu) | w) & 0x80808080u;
 }
 
+// The 16 nonzero-byte flags of a 16-byte piece of the mask.
+__device__ __forceinline__ uint32_t flags_of(uint4 q) {
+    const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+    uint32_t flags = 0;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const uint32_t m = nonzero_bytes(w[k]);
+        flags |= ((m >> 7) & 1u) << (4 * k + 0);
+        flags |= ((m >> 15) & 1u) << (4 * k + 1);
+        flags |= ((m >> 23) & 1u) << (4 * k + 2);
+        flags |= ((m >> 31) & 1u) << (4 * k + 3);
+    }
+    return flags;
+}
+
 // Loads this thread's 16 mask bytes (zeros past n) as a 16-bit flag set.
 __device__ __forceinline__ uint32_t load_flags(const uint8_t* mask, long long n, long long base) {
     uint32_t flags = 0;
@@ -320,17 +335,32 @@ __global__ void __launch_bounds__(kMapThreads) compact_map_kernel(const MapArgs 
     const int m = (nch + kMapThreads - 1) / kMapThreads;
     const int cb0 = tid * m;
     int cnt = 0;
-#pragma unroll 4
-    for (int j = 0; j < m; ++j) {
-        const int c = cb0 + j;
-        if (c < nch) {
+    // the chunks' loads in batches of kBatch, all in flight before any is used
+    constexpr int kBatch = 4;
+    const bool vec_ok = (reinterpret_cast<uintptr_t>(a.mask + a0) & 15u) == 0;
+    for (int j0 = 0; j0 < m; j0 += kBatch) {
+        uint4 q[kBatch];
+#pragma unroll
+        for (int jj = 0; jj < kBatch; ++jj) {
+            const int c = cb0 + j0 + jj;
             const long long g = a0 + 16ll * c;
-            uint32_t f = load_flags(a.mask, a.n, g);
-            const long long lo = fb - g, hi = fb + V - g;  // in-frame bytes lo .. hi-1
-            if (lo > 0) f &= 0xFFFFu << lo;
-            if (hi < kItems) f &= (1u << hi) - 1u;
-            s_flag[c] = (uint16_t)f;
-            cnt += __popc(f);
+            q[jj] = (j0 + jj < m && c < nch && vec_ok && g + kItems <= a.n)
+                        ? __ldg(reinterpret_cast<const uint4*>(a.mask + g))
+                        : make_uint4(0u, 0u, 0u, 0u);
+        }
+#pragma unroll
+        for (int jj = 0; jj < kBatch; ++jj) {
+            const int c = cb0 + j0 + jj;
+            if (j0 + jj < m && c < nch) {
+                const long long g = a0 + 16ll * c;
+                uint32_t f = (vec_ok && g + kItems <= a.n) ? flags_of(q[jj])
+                                                          : load_flags(a.mask, a.n, g);
+                const long long lo = fb - g, hi = fb + V - g;  // in-frame bytes lo .. hi-1
+                if (lo > 0) f &= 0xFFFFu << lo;
+                if (hi < kItems) f &= (1u << hi) - 1u;
+                s_flag[c] = (uint16_t)f;
+                cnt += __popc(f);
+            }
         }
     }
     int fc;  // active rows of frame b
