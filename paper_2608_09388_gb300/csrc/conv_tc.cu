@@ -355,9 +355,43 @@ __device__ __forceinline__ void gn_stats_chunk(const ConvArgs& a, const uint32_t
     }
 }
 
-template <int BN, int TM, bool TR>
-__global__ void __launch_bounds__(kThreadsFor<TM>, 1)
-    conv_tc_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_w) {
+// Where a kernel's barriers sit, as indices of 8-byte slots from the start of
+// its barrier block, where its tap tables start (bytes from that block) and
+// how many rows each table has room for. Compile-time, so that every
+// barrier and table address is the block's address plus an immediate.
+template <int kFull_, int kEmpty_, int kTfull_, int kTempty_, int kFin_, int kTabfull_,
+          int kTabempty_, int kTabOffset_, int kTabRoom_>
+struct BarSlots {
+    static constexpr int kFull = kFull_, kEmpty = kEmpty_, kTfull = kTfull_, kTempty = kTempty_,
+                         kFin = kFin_, kTabfull = kTabfull_, kTabempty = kTabempty_,
+                         kTabOffset = kTabOffset_, kTabRoom = kTabRoom_;
+};
+// conv_tc_kernel's block: full and empty per stage (kMaxStages each), the two
+// accumulator pairs, fin, the table pairs.
+template <class C>
+using RingSlots = BarSlots<0, C::kMaxStages, 2 * C::kMaxStages, 2 * C::kMaxStages + 2,
+                           2 * C::kMaxStages + 4, 2 * C::kMaxStages + 5, 2 * C::kMaxStages + 7,
+                           C::kTabOffset, C::kTabRows>;
+
+// Run-time part of a launch's shared memory and TMEM.
+struct ConvSmem {
+    uint32_t ring;             // stage s at ring + s * (A bytes + W bytes)
+    int nst;                   // stages in the ring
+    uint32_t bars;             // the barrier block
+    volatile int* abort_flag;  // set by the first role that gives up
+    uint32_t tmem_base;
+};
+
+// The five roles of a launch on TM-half items of BN channels (after the
+// prologue: barriers initialised, TMEM allocated, launch dependency
+// passed). The arguments come by value: read through a reference to the
+// kernel parameter, the layers ran up to 14% slower. `prefetched`: this thread (the index warp) has already copied
+// the first item's rulebook entries into tap table 0, completing
+// tabfull(0) through the copies.
+template <int BN, int TM, bool TR, class S>
+__device__ __forceinline__ void conv_roles(const ConvArgs a, const CUtensorMap& tmap_w,
+                                           const ConvSmem& sm, const long long rows,
+                                           const bool prefetched) {
     using C = Cfg<BN, TM>;
     static_assert(!TR || (TM == 2 && BN == 128), "the transposed MMA takes 2 x 128 rows, 128 channels");
     // transposed MMA: D fp32, A (W) bf16 MN-major (bit 15), B (rows) bf16
@@ -365,93 +399,31 @@ __global__ void __launch_bounds__(kThreadsFor<TM>, 1)
     constexpr uint32_t kIdescTR = (1u << 4) | (1u << 7) | (1u << 10) | (1u << 15) |
                                   ((uint32_t)(256 >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
     constexpr int kTabRows = C::kTabRows;
-    // "full": one cp.async completion arrival per producer thread, plus the
-    // expect-tx arrival of the weight loader.
-    constexpr int kStageArrivals = kProducerWarps * 32 + 1;
-    extern __shared__ uint8_t smem_raw[];
-    const uint32_t raw = smem_u32(smem_raw);
-    const uint32_t base = (raw + 1023u) & ~1023u;
-    uint8_t* const base_ptr = smem_raw + (base - raw);
-    const uint32_t sA = base;  // the stage ring (a.stages two-half stages)
-    const int nst = a.stages;
     constexpr uint32_t kStageBytes = C::kAStageBytes + C::kBStageBytes;
+    const int nst = sm.nst;
     // stage st: TM halves of A (16 KB each), then the W slice (1024-byte aligned)
-    auto a_stage = [&](int st) { return sA + (uint32_t)st * kStageBytes; };
-    auto b_stage = [&](int st) { return sA + (uint32_t)st * kStageBytes + (uint32_t)C::kAStageBytes; };
-    const uint32_t sBar = sA + (uint32_t)nst * kStageBytes;
-    uint8_t* const misc = base_ptr + (sBar - base) + C::kBarBytes;
-    volatile uint32_t* const tmem_holder = reinterpret_cast<volatile uint32_t*>(misc);
-    volatile int* const abort_flag = reinterpret_cast<volatile int*>(misc + 4);
-    // Tap tables, [2][L][kTabRows] int32: entry (l, r) is the input row
-    // feeding slot l of row r of the work item, or -1.
-    const uint32_t tab0 = sBar + C::kTabOffset;
-    const uint32_t epi0 = tab0 + 2u * (uint32_t)(kTabRows * a.L) * 4u;  // epilogue staging
-
-    auto full_bar = [&](int s) { return sBar + 8u * s; };
-    auto empty_bar = [&](int s) { return sBar + 8u * (C::kMaxStages + s); };
-    auto tfull_bar = [&](int i) { return sBar + 8u * (2 * C::kMaxStages + i); };
-    auto tempty_bar = [&](int i) { return sBar + 8u * (2 * C::kMaxStages + 2 + i); };
-    const uint32_t fin_bar = sBar + 8u * (2 * C::kMaxStages + 4);
-    auto tabfull_bar = [&](int i) { return sBar + 8u * (2 * C::kMaxStages + 5 + i); };
-    auto tabempty_bar = [&](int i) { return sBar + 8u * (2 * C::kMaxStages + 7 + i); };
-
+    auto a_stage = [&](int st) { return sm.ring + (uint32_t)st * kStageBytes; };
+    auto b_stage = [&](int st) {
+        return sm.ring + (uint32_t)st * kStageBytes + (uint32_t)C::kAStageBytes;
+    };
+    const uint32_t sBar = sm.bars;
+    auto full_bar = [&](int s) { return sBar + 8u * (S::kFull + s); };
+    auto empty_bar = [&](int s) { return sBar + 8u * (S::kEmpty + s); };
+    auto tfull_bar = [&](int i) { return sBar + 8u * (S::kTfull + i); };
+    auto tempty_bar = [&](int i) { return sBar + 8u * (S::kTempty + i); };
+    const uint32_t fin_bar = sBar + 8u * S::kFin;
+    auto tabfull_bar = [&](int i) { return sBar + 8u * (S::kTabfull + i); };
+    auto tabempty_bar = [&](int i) { return sBar + 8u * (S::kTabempty + i); };
+    volatile int* const abort_flag = sm.abort_flag;
+    const uint32_t tmem_base = sm.tmem_base;
+    // Tap tables, [2][L][TM * 128] int32 (room for [2][L][kTabRoom]): entry
+    // (l, r) is the input row feeding slot l of row r of the work item, or
+    // -1; then the epilogue staging.
+    static_assert(S::kTabRoom >= kTabRows, "tap table room");
+    const uint32_t tab0 = sBar + S::kTabOffset;
+    const uint32_t epi0 = tab0 + 2u * (uint32_t)(S::kTabRoom * a.L) * 4u;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-    if (threadIdx.x == 0) {
-        for (int s = 0; s < C::kMaxStages; ++s) {
-            mbar_init(full_bar(s), kStageArrivals);
-            mbar_init(empty_bar(s), 1);
-        }
-        for (int i = 0; i < 2; ++i) {
-            mbar_init(tfull_bar(i), 1);
-            mbar_init(tempty_bar(i), kEpilogueWarps * 32);
-        }
-        mbar_init(fin_bar, 1);
-        for (int i = 0; i < 2; ++i) {
-            mbar_init(tabfull_bar(i), 32 * TM);  // the index warps' lanes
-            mbar_init(tabempty_bar(i), kProducerWarps * 32);
-        }
-        *abort_flag = 0;
-        asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
-    }
-    if (warp == kWeightWarp && lane == 0) prefetch_tensormap(&tmap_w);
-    if (warp == kMmaWarp) {
-        tmem_alloc(smem_u32((const void*)tmem_holder), C::kTmemCols);
-        tmem_relinquish();
-    }
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    const uint32_t tmem_base = *tmem_holder;
-    // The prologue above touched only on-chip state; global memory written
-    // by the previous grid is read from here on.
-    pdl_wait();
-    pdl_trigger();
-
-    // Rulebook mode (one-half items): the index warp copies its first tile's
-    // entries into tap table 0 (cp.async, rows clamped to the capacity,
-    // always valid memory) before the row count arrives, so the two L2 round
-    // trips overlap, and the copies themselves complete the table's "full"
-    // barrier: the producers start on the entries as copied. They are not
-    // checked first (a pass over them before the hand-over cost ~0.7 us of
-    // the launch); the producers read zeros for any entry outside
-    // [0, x_rows) (entries of rows past the count are never checked, and
-    // those rows are never stored), and the index warp reports bad entries
-    // of active rows once the table is handed over.
-    const bool prefetch = TM == 1 && warp == kIndexWarp && a.mode == kRulebook;
-    if (prefetch) {
-        const long long m0p = (blockIdx.x / ((a.C_out + BN - 1) / BN)) * (long long)kBM;
-        for (int d = 0; d < a.L; ++d)
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const long long n = m0p + lane + 32 * i;
-                cp_async_4(tab0 + (uint32_t)(d * kTabRows + lane + 32 * i) * 4u,
-                           a.rulebook + (long long)d * a.capacity + (n < a.capacity ? n : 0), true);
-            }
-        cp_async_arrive_noinc(tabfull_bar(0));
-    }
-
-    const long long rows = active_rows(a);
     const int n_tiles = (a.C_out + BN - 1) / BN;
     constexpr int item_rows = TM * kBM;
     const long long m_items = (rows + item_rows - 1) / item_rows;
@@ -459,7 +431,6 @@ __global__ void __launch_bounds__(kThreadsFor<TM>, 1)
     const int num_kb = (a.K + kBK - 1) / kBK;
     const int L = a.L, C_in = a.C_in, C_out = a.C_out, K = a.K;
     const uint32_t tab_bytes = (uint32_t)(kTabRows * L) * 4u;
-    const bool prefetched = prefetch;
 
     if (warp < kProducerWarps) {
         // ------------------------------------------------------------ producers
@@ -810,7 +781,7 @@ __global__ void __launch_bounds__(kThreadsFor<TM>, 1)
             if (!(lt == 0 && prefetched)) mbar_arrive(tabfull_bar(buf));  // else the copies did
         }
         if (prefetched) cp_async_wait_all();  // a CTA without items
-    } else {
+    } else if (warp < kMmaWarp) {
         // ------------------------------------------------------------ epilogue
         const int ew = warp - kProducerWarps;  // == warp % 4: TMEM lanes 32*ew..+32
         __nv_bfloat16* __restrict__ y = static_cast<__nv_bfloat16*>(a.y);
@@ -969,10 +940,215 @@ __global__ void __launch_bounds__(kThreadsFor<TM>, 1)
         }
         }
     }
+}
+
+template <int BN, int TM, bool TR>
+__global__ void __launch_bounds__(kThreadsFor<TM>, 1)
+    conv_tc_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_w) {
+    using C = Cfg<BN, TM>;
+    constexpr int kTabRows = C::kTabRows;
+    // "full": one cp.async completion arrival per producer thread, plus the
+    // expect-tx arrival of the weight loader.
+    constexpr int kStageArrivals = kProducerWarps * 32 + 1;
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t raw = smem_u32(smem_raw);
+    const uint32_t base = (raw + 1023u) & ~1023u;
+    uint8_t* const base_ptr = smem_raw + (base - raw);
+    const uint32_t sA = base;  // the stage ring (a.stages two-half stages)
+    const int nst = a.stages;
+    constexpr uint32_t kStageBytes = C::kAStageBytes + C::kBStageBytes;
+    const uint32_t sBar = sA + (uint32_t)nst * kStageBytes;
+    uint8_t* const misc = base_ptr + (sBar - base) + C::kBarBytes;
+    volatile uint32_t* const tmem_holder = reinterpret_cast<volatile uint32_t*>(misc);
+    volatile int* const abort_flag = reinterpret_cast<volatile int*>(misc + 4);
+    const uint32_t tab0 = sBar + C::kTabOffset;  // tap table 0
+
+    auto full_bar = [&](int s) { return sBar + 8u * s; };
+    auto empty_bar = [&](int s) { return sBar + 8u * (C::kMaxStages + s); };
+    auto tfull_bar = [&](int i) { return sBar + 8u * (2 * C::kMaxStages + i); };
+    auto tempty_bar = [&](int i) { return sBar + 8u * (2 * C::kMaxStages + 2 + i); };
+    const uint32_t fin_bar = sBar + 8u * (2 * C::kMaxStages + 4);
+    auto tabfull_bar = [&](int i) { return sBar + 8u * (2 * C::kMaxStages + 5 + i); };
+    auto tabempty_bar = [&](int i) { return sBar + 8u * (2 * C::kMaxStages + 7 + i); };
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < C::kMaxStages; ++s) {
+            mbar_init(full_bar(s), kStageArrivals);
+            mbar_init(empty_bar(s), 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(tfull_bar(i), 1);
+            mbar_init(tempty_bar(i), kEpilogueWarps * 32);
+        }
+        mbar_init(fin_bar, 1);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(tabfull_bar(i), 32 * TM);  // the index warps' lanes
+            mbar_init(tabempty_bar(i), kProducerWarps * 32);
+        }
+        *abort_flag = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
+    }
+    if (warp == kWeightWarp && lane == 0) prefetch_tensormap(&tmap_w);
+    if (warp == kMmaWarp) {
+        tmem_alloc(smem_u32((const void*)tmem_holder), C::kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_holder;
+    // The prologue above touched only on-chip state; global memory written
+    // by the previous grid is read from here on.
+    pdl_wait();
+    pdl_trigger();
+
+    // Rulebook mode (one-half items): the index warp copies its first tile's
+    // entries into tap table 0 (cp.async, rows clamped to the capacity,
+    // always valid memory) before the row count arrives, so the two L2 round
+    // trips overlap, and the copies themselves complete the table's "full"
+    // barrier: the producers start on the entries as copied. They are not
+    // checked first (a pass over them before the hand-over cost ~0.7 us of
+    // the launch); the producers read zeros for any entry outside
+    // [0, x_rows) (entries of rows past the count are never checked, and
+    // those rows are never stored), and the index warp reports bad entries
+    // of active rows once the table is handed over.
+    const bool prefetch = TM == 1 && warp == kIndexWarp && a.mode == kRulebook;
+    if (prefetch) {
+        const long long m0p = (blockIdx.x / ((a.C_out + BN - 1) / BN)) * (long long)kBM;
+        for (int d = 0; d < a.L; ++d)
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const long long n = m0p + lane + 32 * i;
+                cp_async_4(tab0 + (uint32_t)(d * kTabRows + lane + 32 * i) * 4u,
+                           a.rulebook + (long long)d * a.capacity + (n < a.capacity ? n : 0), true);
+            }
+        cp_async_arrive_noinc(tabfull_bar(0));
+    }
+
+    const ConvSmem sm{sA, nst, sBar, abort_flag, tmem_base};
+    conv_roles<BN, TM, TR, RingSlots<C>>(a, tmap_w, sm, active_rows(a), prefetch);
     __syncthreads();
     if (warp == kMmaWarp) {
         tc_fence_after();
         tmem_dealloc(tmem_base, C::kTmemCols);
+    }
+}
+
+// Shared memory of the row-count-dispatched kernel below: a ring as long as
+// the larger of the one-half (32 KB) and two-half (48 KB) rings, one barrier
+// block (full / empty for up to six stages, the accumulator, fin and
+// table-empty barriers, and a table-full pair per half count), the tap
+// tables sized for two-half items, and the epilogue staging.
+struct AutoLayout {
+    static constexpr int kRing1 = 6, kRing2 = 4;  // most stages per half count
+    static constexpr int kFull = 0, kEmpty = 6, kTfull = 12, kTempty = 14, kFin = 16,
+                         kTabfull1 = 17, kTabempty = 19, kTabfull2 = 21, kBars = 23;
+    static constexpr int kTabOffset = (8 * kBars + 16 + 127) / 128 * 128;
+    static constexpr int kStage1 = Cfg<128, 1>::kAStageBytes + Cfg<128, 1>::kBStageBytes;
+    static constexpr int kStage2 = Cfg<128, 2>::kAStageBytes + Cfg<128, 2>::kBStageBytes;
+    __host__ __device__ static size_t ring_bytes(int st1, int st2) {
+        const size_t r1 = (size_t)st1 * kStage1, r2 = (size_t)st2 * kStage2;
+        return r1 > r2 ? r1 : r2;
+    }
+    static size_t fixed_bytes(int L) {
+        return 1024 + kTabOffset + 2 * sizeof(int) * (size_t)(2 * kBM) * L +
+               Cfg<128, 2>::kEpiBytes;
+    }
+    static size_t smem_bytes(int L, int st1, int st2) { return fixed_bytes(L) + ring_bytes(st1, st2); }
+    static void stages_for(int L, int& st1, int& st2) {
+        const size_t avail = kSmemLimit - fixed_bytes(L);
+        st1 = (int)(avail / kStage1 < (size_t)kRing1 ? avail / kStage1 : kRing1);
+        st2 = (int)(avail / kStage2 < (size_t)kRing2 ? avail / kStage2 : kRing2);
+    }
+};
+
+// 128-channel rulebook calls whose row count is on the device: every CTA
+// reads the count after the launch dependency and runs two-half transposed
+// items when each CTA gets at least one (rows >= 256 per CTA), one-half
+// items otherwise. Both role sets are compiled in and each branch is taken
+// whole, so neither pays for the other in its loops. The one-half roles'
+// first-table prefetch (issued before the count is known) completes its own
+// table-full pair; when the two-half roles run instead, the prefetching
+// warp waits for those copies before the tables are rebuilt, and their
+// arrival lands on barriers nothing waits on.
+__global__ void __launch_bounds__(kThreadsFor<2>, 1)
+    conv_tc_auto_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_w) {
+    using L_ = AutoLayout;
+    constexpr int kStageArrivals = kProducerWarps * 32 + 1;
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t raw = smem_u32(smem_raw);
+    const uint32_t base = (raw + 1023u) & ~1023u;
+    uint8_t* const base_ptr = smem_raw + (base - raw);
+    const uint32_t ring = (uint32_t)L_::ring_bytes(a.stages, a.stages_tr);
+    const uint32_t sBar = base + ring;
+    uint8_t* const misc = base_ptr + ring + 8 * L_::kBars;
+    volatile uint32_t* const tmem_holder = reinterpret_cast<volatile uint32_t*>(misc);
+    volatile int* const abort_flag = reinterpret_cast<volatile int*>(misc + 4);
+    const uint32_t tab0 = sBar + L_::kTabOffset;  // the one-half roles' table 0
+    auto bar = [&](int i) { return sBar + 8u * i; };
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < L_::kRing1; ++s) {
+            mbar_init(bar(L_::kFull + s), kStageArrivals);
+            mbar_init(bar(L_::kEmpty + s), 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(bar(L_::kTfull + i), 1);
+            mbar_init(bar(L_::kTempty + i), kEpilogueWarps * 32);
+            mbar_init(bar(L_::kTabfull1 + i), 32);  // one index warp
+            mbar_init(bar(L_::kTabempty + i), kProducerWarps * 32);
+            mbar_init(bar(L_::kTabfull2 + i), 64);  // two index warps
+        }
+        mbar_init(bar(L_::kFin), 1);
+        *abort_flag = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
+    }
+    if (warp == kWeightWarp && lane == 0) prefetch_tensormap(&tmap_w);
+    if (warp == kMmaWarp) {
+        tmem_alloc(smem_u32((const void*)tmem_holder), Cfg<128, 2>::kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_holder;
+    pdl_wait();
+    pdl_trigger();
+
+    // the one-half roles' first table, copied while the row count is read
+    // (as in conv_tc_kernel)
+    const bool prefetch = warp == kIndexWarp;
+    if (prefetch) {
+        const long long m0p = (long long)blockIdx.x * kBM;
+        for (int d = 0; d < a.L; ++d)
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const long long n = m0p + lane + 32 * i;
+                cp_async_4(tab0 + (uint32_t)(d * kBM + lane + 32 * i) * 4u,
+                           a.rulebook + (long long)d * a.capacity + (n < a.capacity ? n : 0), true);
+            }
+        cp_async_arrive_noinc(bar(L_::kTabfull1));
+    }
+    const long long rows = active_rows(a);
+    using S1 = BarSlots<L_::kFull, L_::kEmpty, L_::kTfull, L_::kTempty, L_::kFin, L_::kTabfull1,
+                        L_::kTabempty, L_::kTabOffset, 2 * kBM>;
+    using S2 = BarSlots<L_::kFull, L_::kEmpty, L_::kTfull, L_::kTempty, L_::kFin, L_::kTabfull2,
+                        L_::kTabempty, L_::kTabOffset, 2 * kBM>;
+    if ((rows + 2 * kBM - 1) / (2 * kBM) >= (long long)gridDim.x) {
+        if (prefetch) cp_async_wait_all();
+        conv_roles<128, 2, true, S2>(a, tmap_w, ConvSmem{base, a.stages_tr, sBar, abort_flag, tmem_base},
+                                     rows, false);
+    } else {
+        conv_roles<128, 1, false, S1>(a, tmap_w, ConvSmem{base, a.stages, sBar, abort_flag, tmem_base},
+                                      rows, prefetch);
+    }
+    __syncthreads();
+    if (warp == kMmaWarp) {
+        tc_fence_after();
+        tmem_dealloc(tmem_base, Cfg<128, 2>::kTmemCols);
     }
 }
 
@@ -1081,31 +1257,39 @@ hc_status encode_w3d(CUtensorMap* m, const void* base, long long K, long long C_
     return HC_OK;
 }
 
+// W: [K rows, C_out]. With C_out a multiple of 64, the 3-D view
+// [C_out / 64][K][64] (the 64-column blocks 128 bytes apart) takes a tile's
+// BN columns of a k-block in one box of 64 x 64 x BN/64; otherwise 2-D boxes
+// of 64 K-rows x 64 output channels, one per block.
+hc_status encode_weights(CUtensorMap* tw, ConvArgs& ka, int BN) {
+    memset(tw, 0, sizeof *tw);
+    ka.w3d = ka.C_out % 64 == 0;
+    if (ka.w3d) return encode_w3d(tw, ka.W, ka.K, ka.C_out, kBK, BN / 64);
+    return encode_2d(tw, ka.W, ka.K, ka.C_out, 64, kBK);
+}
+
+template <typename Kernel>
+hc_status set_smem_limit(const DeviceCtx* ctx, Kernel k, bool (&done)[64], const char* what) {
+    if (!done[ctx->device]) {
+        hc_status st = check_cuda(
+            cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemLimit),
+            what);
+        if (st != HC_OK) return st;
+        done[ctx->device] = true;
+    }
+    return HC_OK;
+}
+
 template <int BN, int TM, bool TR = false>
 hc_status launch_bn(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s) {
     using C = Cfg<BN, TM>;
     static bool attr_set[64] = {};
-    if (!attr_set[ctx->device]) {
-        hc_status st = check_cuda(cudaFuncSetAttribute(conv_tc_kernel<BN, TM, TR>,
-                                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                       (int)kSmemLimit),
+    hc_status st = set_smem_limit(ctx, conv_tc_kernel<BN, TM, TR>, attr_set,
                                   "cudaFuncSetAttribute(conv_tc_kernel)");
-        if (st != HC_OK) return st;
-        attr_set[ctx->device] = true;
-    }
+    if (st != HC_OK) return st;
     CUtensorMap tw;
-    memset(&tw, 0, sizeof tw);
     ConvArgs ka = a;
-    // W: [K rows, C_out]. With C_out a multiple of 64, the 3-D view
-    // [C_out / 64][K][64] (the 64-column blocks 128 bytes apart) takes a
-    // tile's BN columns of a k-block in one box of 64 x 64 x BN/64; otherwise
-    // 2-D boxes of 64 K-rows x 64 output channels, one per block.
-    hc_status st;
-    ka.w3d = a.C_out % 64 == 0;
-    if (ka.w3d)
-        st = encode_w3d(&tw, a.W, a.K, a.C_out, kBK, BN / 64);
-    else
-        st = encode_2d(&tw, a.W, a.K, a.C_out, 64, kBK);
+    st = encode_weights(&tw, ka, BN);
     if (st != HC_OK) return st;
     const long long n_tiles = (a.C_out + BN - 1) / BN;
     const long long cap_work = (a.capacity + TM * kBM - 1) / (TM * kBM) * n_tiles;
@@ -1114,6 +1298,26 @@ hc_status launch_bn(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s) {
     ka.stages = C::stages_for(a.L);
     return launch_pdl(conv_tc_kernel<BN, TM, TR>, dim3((unsigned)grid), dim3(kThreadsFor<TM>),
                       C::smem_bytes(a.L, ka.stages), s, "conv_tc_kernel", ka, tw);
+}
+
+// conv_tc_auto_kernel: one CTA per SM, or one per 128-row item of the
+// capacity when there are fewer.
+hc_status launch_auto(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s) {
+    static bool attr_set[64] = {};
+    hc_status st = set_smem_limit(ctx, conv_tc_auto_kernel, attr_set,
+                                  "cudaFuncSetAttribute(conv_tc_auto_kernel)");
+    if (st != HC_OK) return st;
+    CUtensorMap tw;
+    ConvArgs ka = a;
+    st = encode_weights(&tw, ka, 128);
+    if (st != HC_OK) return st;
+    const long long items = (a.capacity + kBM - 1) / kBM;
+    long long grid = items < ctx->num_sms ? items : ctx->num_sms;
+    if (grid < 1) grid = 1;
+    AutoLayout::stages_for(a.L, ka.stages, ka.stages_tr);
+    return launch_pdl(conv_tc_auto_kernel, dim3((unsigned)grid), dim3(kThreadsFor<2>),
+                      AutoLayout::smem_bytes(a.L, ka.stages, ka.stages_tr), s,
+                      "conv_tc_auto_kernel", ka, tw);
 }
 
 }  // namespace
@@ -1189,9 +1393,15 @@ hc_status launch_conv_tc(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s
     // 32 -> 28 us at 67k rows (1.7 items per SM), the same at 33k (0.9 per
     // SM), 11 -> 18 us at 6.8k (0.2 per SM). The results are the same either
     // way.
-    if (a.mode == kRulebook && a.C_out == 128 && !a.out_dense && !a.gn_part &&
-        a.C_in % 8 == 0 && (a.rows_hint + 2 * kBM - 1) / (2 * kBM) >= ctx->num_sms)
-        return launch_bn<128, 2, true>(ctx, a, s);
+    // Without an estimate (rows_hint 0), a call whose capacity could fill
+    // every SM with two-half items leaves the choice to the CTAs, which read
+    // the row count (conv_tc_auto_kernel).
+    if (a.mode == kRulebook && a.C_out == 128 && !a.out_dense && !a.gn_part && a.C_in % 8 == 0) {
+        if ((a.rows_hint + 2 * kBM - 1) / (2 * kBM) >= ctx->num_sms)
+            return launch_bn<128, 2, true>(ctx, a, s);
+        if (a.rows_hint == 0 && (a.capacity + 2 * kBM - 1) / (2 * kBM) >= ctx->num_sms)
+            return launch_auto(ctx, a, s);
+    }
     if (conv_tc_tile_n(a) == 64) return launch_bn<64, 1>(ctx, a, s);
     return two ? (a.C_out == 128 && !a.out_dense && !a.gn_part ? launch_bn<128, 2, true>(ctx, a, s)
                                                                 : launch_bn<128, 2, false>(ctx, a, s))

@@ -83,6 +83,7 @@ struct ConvArgs {
     int mode;
     int act;
     int stages;  // pipeline depth chosen by the launcher (tensor-core kernel)
+    int stages_tr;  // the row-count-dispatched kernel's depth for two-half items
     int w3d;     // tensor-core kernel: W's tensor map is the 3-D view (one box per stage)
     // Optional group-norm statistics of the stored output (Eqs. 7-9,
     // tensor-core kernel): every block c of 32 output rows writes, for each

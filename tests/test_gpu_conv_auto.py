@@ -1,0 +1,144 @@
+"""The row-count-dispatched tensor-core kernel (conv_tc_auto_kernel): a
+128-channel rulebook call without a row estimate, whose capacity could give
+every SM a two-half item, reads N' on the device and runs two-half
+transposed items when N' >= 256 x CTAs (one CTA per SM), one-half items
+below. Around that threshold, and at no rows, one row, a ragged last item
+and the full capacity: every row against the oracle (Eqs. 4-5 with the bias
+and ELU), bit-identical to the calls that force each item shape through a
+row estimate, rows past N' untouched; bad rulebook entries reported in both
+branches and contributing nothing."""
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2608_09388_gb300 import hc, inputs
+
+from _util import check_close, to_numpy, to_torch
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+NCPU = len(os.sched_getaffinity(0))
+B, V, L, C_IN = 4, 10475, 9, 64
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2608_09388_gb300 import build
+    build.build()
+    hc.load_library()
+    assert hc.hc_get_device_status() == hc.HC_OK
+
+
+@pytest.fixture(scope="module")
+def case():
+    """Random spiral (slot 0 the vertex itself, ~10% absent entries),
+    features, weights and bias of a 64 -> 128 ELU layer on 4 x 10475
+    vertices: a capacity of 41,900 rows, above 256 rows per SM."""
+    rng = np.random.default_rng(2024)
+    sp = rng.integers(0, V, size=(V, L)).astype(np.int32)
+    sp[rng.random((V, L)) < 0.1] = -1
+    sp[:, 0] = np.arange(V)
+    x = inputs.features(rng, (B, V, C_IN), "bf16")
+    W = inputs.weights(rng, L * C_IN, 128, "bf16")
+    b = rng.standard_normal(128).astype(np.float32)
+    order = rng.permutation(B * V)  # vertices made active, in this order
+    return sp, x, W, b, order
+
+
+def threshold():
+    return 256 * torch.cuda.get_device_properties(0).multi_processor_count
+
+
+def mask_with(order, n):
+    m = np.zeros(B * V, np.uint8)
+    m[order[:n]] = 1
+    return m.reshape(B, V)
+
+
+def rulebook(m, sp):
+    coords = torch.empty((B * V, 2), dtype=torch.int32, device="cuda")
+    row_of = torch.empty((B, V), dtype=torch.int32, device="cuda")
+    offs = torch.empty((B + 1,), dtype=torch.int32, device="cuda")
+    count = torch.empty((1,), dtype=torch.int32, device="cuda")
+    rb = torch.empty((L, B * V), dtype=torch.int32, device="cuda")
+    hc.hc_mask_compact_rulebook(to_torch(m), to_torch(sp), hc.HC_LAYOUT_DENSE, coords, row_of,
+                                offs, count, rb)
+    return rb, count
+
+
+def run(x, rb, count, W, b, hint=None):
+    y = torch.full((B * V, 128), float("nan"), dtype=torch.bfloat16, device="cuda")
+    if hint is None:
+        hc.hc_sparse_conv_rulebook_fwd(x, rb, count, W, b, hc.HC_ACT_ELU, y)
+    else:
+        hc.hc_sparse_conv_rulebook_fwd_hint(x, rb, count, W, b, hc.HC_ACT_ELU, y, hint)
+    return y
+
+
+@pytest.mark.parametrize("offset", [-1, 0, 1, 255, 256, 300])
+def test_both_branches_at_the_threshold(case, offset):
+    """N' = 256 x SMs + offset: one-half items just below, two-half
+    transposed items from the threshold up (exact, one row into a new item,
+    a full last item, a ragged one)."""
+    sp, x, W, b, order = case
+    n = threshold() + offset
+    assert n <= B * V
+    m = mask_with(order, n)
+    rb, count = rulebook(m, sp)
+    assert int(count.item()) == n
+    xt, Wt, bt = to_torch(x), to_torch(W), to_torch(b)
+    y = run(xt, rb, count, Wt, bt)
+    assert hc.hc_get_device_status() == hc.HC_OK
+    assert torch.isnan(y[n:].float()).all()
+    for hint in (1, B * V):  # forced one-half, forced two-half transposed
+        assert torch.equal(run(xt, rb, count, Wt, bt, hint)[:n], y[:n]), f"hint {hint}"
+    c, r, _, _ = oracle.mask_compact(m)
+    y_pre, _ = oracle.sparse_spiral_conv(x, oracle.LAYOUT_DENSE, c, r, sp, W, b, oracle.ACT_ELU,
+                                         n_threads=NCPU)
+    check_close(to_numpy(y)[:n], y_pre, f"auto N'={n}")
+
+
+@pytest.mark.parametrize("n", [0, 1, 5000, B * V])
+def test_small_and_full_counts(case, n):
+    """No rows, one row, a count far below the threshold (one-half items on
+    a few CTAs), every vertex active."""
+    sp, x, W, b, order = case
+    m = mask_with(order, n)
+    rb, count = rulebook(m, sp)
+    xt, Wt, bt = to_torch(x), to_torch(W), to_torch(b)
+    y = run(xt, rb, count, Wt, bt)
+    assert hc.hc_get_device_status() == hc.HC_OK
+    assert torch.isnan(y[n:].float()).all()
+    assert torch.equal(run(xt, rb, count, Wt, bt, 1)[:n], y[:n])
+    if n:
+        c, r, _, _ = oracle.mask_compact(m)
+        y_pre, _ = oracle.sparse_spiral_conv(x, oracle.LAYOUT_DENSE, c, r, sp, W, b,
+                                             oracle.ACT_ELU, n_threads=NCPU)
+        check_close(to_numpy(y)[:n], y_pre, f"auto N'={n}")
+
+
+@pytest.mark.parametrize("offset", [-1, 0])
+def test_bad_entries_reported_in_both_branches(case, offset):
+    """Out-of-range rulebook entries of active rows, in the first item of a
+    CTA (the one-half roles' prefetched table) and in a later one: the call
+    reports HC_ERR_INVALID_INDEX and its rows are those of the same rulebook
+    with the entries absent."""
+    sp, x, W, b, order = case
+    n = threshold() + offset
+    rb, count = rulebook(mask_with(order, n), sp)
+    xt, Wt, bt = to_torch(x), to_torch(W), to_torch(b)
+    bad = [(2, 5, B * V), (1, 7, -3), (4, n - 3, B * V + 11), (0, 200 * 128 + 9, -2)]
+    for l, col, v in bad:
+        rb[l, col] = v
+    y = run(xt, rb, count, Wt, bt)
+    assert hc.hc_get_device_status() == hc.HC_ERR_INVALID_INDEX
+    for l, col, _ in bad:
+        rb[l, col] = -1
+    y_abs = run(xt, rb, count, Wt, bt)
+    assert hc.hc_get_device_status() == hc.HC_OK
+    assert torch.equal(y[:n], y_abs[:n])
