@@ -62,6 +62,11 @@ def parse_args():
     p.add_argument("--e2e-steps", type=int, default=30)
     p.add_argument("--no-e2e", action="store_true",
                    help="skip the end-to-end measurement (for targeted profiler captures)")
+    p.add_argument("--case", default=None,
+                   help="profiler target instead of the bench: run one layer call of the "
+                        "density sweep's workload --steps times and print its CUDA-event "
+                        "times; 'sweep:D' the sparse conv at mask density D (compaction and "
+                        "mapping done before), 'sweep-dense' the dense layer")
     return p.parse_args()
 
 
@@ -1238,6 +1243,66 @@ def run_configs(torch, hc, dev, stream, cpu_budget_s=3.0):
     return res
 
 
+def run_case(args):
+    """One layer call of the density sweep's workload (V = 10475, L = 9,
+    B = 64, 128 -> 128), args.steps times in a row, each timed with CUDA
+    events: a small, fixed launch sequence for a profiler to capture."""
+    import torch
+
+    from paper_2608_09388_gb300 import build as hc_build
+    from paper_2608_09388_gb300 import hc, inputs
+    hc_build.build()
+    hc.load_library()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.Stream(device=dev)
+    w = inputs.make_workload("sweep10475_bf16")
+    ly = w.layers[0]
+    B, V, L = w.B, w.V, w.L
+    x = torch.from_numpy(w.x.view(np.int16)).view(torch.bfloat16).to(dev)
+    spiral = torch.from_numpy(w.spiral).to(dev)
+    Wt = torch.from_numpy(ly.W.view(np.int16)).view(torch.bfloat16).to(dev)
+    bias = torch.from_numpy(ly.b).to(dev)
+    if args.case == "sweep-dense":
+        yd = torch.empty((B, V, ly.C_out), dtype=torch.bfloat16, device=dev)
+        fn = lambda: hc.hc_spiral_conv_fwd(x, spiral, Wt, bias, ly.act, yd, stream)  # noqa: E731
+        rows = B * V
+    elif args.case.startswith("sweep:"):
+        d = float(args.case.split(":", 1)[1])
+        if d not in w.densities:
+            raise SystemExit(f"--case {args.case}: density not in {list(w.densities)}")
+        m = torch.from_numpy(w.masks[list(w.densities).index(d)]).to(dev)
+        coords = torch.empty((B * V, 2), dtype=torch.int32, device=dev)
+        row_of = torch.empty((B, V), dtype=torch.int32, device=dev)
+        offs = torch.empty((B + 1,), dtype=torch.int32, device=dev)
+        count = torch.empty((1,), dtype=torch.int32, device=dev)
+        rb = torch.empty((L, B * V), dtype=torch.int32, device=dev)
+        y = torch.empty((B * V, ly.C_out), dtype=torch.bfloat16, device=dev)
+        with torch.cuda.stream(stream):
+            hc.hc_mask_compact_rulebook(m, spiral, hc.HC_LAYOUT_DENSE, coords, row_of, offs, count,
+                                        rb, stream)
+        torch.cuda.synchronize(dev)
+        rows = int(count.item())
+        fn = lambda: hc.hc_sparse_conv_rulebook_fwd(x, rb, count, Wt, bias, ly.act, y,  # noqa: E731
+                                                    stream=stream)
+    else:
+        raise SystemExit(f"--case {args.case}: expected sweep:D or sweep-dense")
+    times = []
+    for _ in range(args.steps):
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            a.record(stream)
+            fn()
+            b.record(stream)
+        torch.cuda.synchronize(dev)
+        times.append(a.elapsed_time(b) * 1e3)
+    status = hc.hc_get_device_status()
+    print(json.dumps({"case": args.case, "rows": rows, "us": times, "status": status}), flush=True)
+    if status != hc.HC_OK:
+        raise SystemExit(1)
+
+
 def cpu_baseline(w, budget_s=20.0):
     """The CPU oracle as it stands on this host's cores: compaction, sparse
     conv and scatter of batch 0 of the workload (all of its active rows when
@@ -1341,6 +1406,9 @@ def main():
         line = run_reference(args, rank)
         if line is not None:
             print(json.dumps(line), flush=True)
+        return
+    if args.case:
+        run_case(args)
         return
     import torch
     if world > 1:
