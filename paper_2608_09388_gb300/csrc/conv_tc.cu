@@ -154,14 +154,28 @@ __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr, uint32_t lbo
 
 // Transposed epilogue chunk: lane = output channel, r[j] = row j of the
 // chunk; activation, bf16, written transposed into the warp's staging
-// buffer ([32 rows][32 channels] bf16).
+// buffer ([32 rows][32 channels] bf16). Rows j and j + 1 of the lane's
+// channel are rounded as one bf16 pair; neighbouring lanes swap pairs and
+// each builds one 32-bit word of two channels with a byte permute, the even
+// lane for row j, the odd lane for row j + 1. Each store then writes two
+// whole 64-byte rows (16-bit stores of two lanes into one word took two
+// shared-memory wavefronts each).
 template <int ACT>
 __device__ __forceinline__ void tr_stage(const uint32_t (&r)[32], uint32_t stage, int lane) {
+    const uint32_t odd = (uint32_t)lane & 1u;
+    // even lane: its row-j half, then the neighbour's; odd lane: the
+    // neighbour's row-(j+1) half, then its own
+    const uint32_t sel = odd ? 0x3276u : 0x5410u;
+    const uint32_t col = stage + (uint32_t)(lane & ~1) * 2u + odd * 64u;
 #pragma unroll
-    for (int j = 0; j < 32; ++j) {
-        const unsigned short v =
-            __bfloat16_as_ushort(__float2bfloat16_rn(act_fixed<ACT>(__uint_as_float(r[j]))));
-        asm volatile("st.shared.u16 [%0], %1;\n" ::"r"(stage + (uint32_t)(j * 64 + lane * 2)), "h"(v)
+    for (int j = 0; j < 32; j += 2) {
+        const __nv_bfloat162 b = __floats2bfloat162_rn(act_fixed<ACT>(__uint_as_float(r[j])),
+                                                       act_fixed<ACT>(__uint_as_float(r[j + 1])));
+        const uint32_t own = *reinterpret_cast<const uint32_t*>(&b);
+        const uint32_t nb = __shfl_xor_sync(0xffffffffu, own, 1);
+        uint32_t w;
+        asm("prmt.b32 %0, %1, %2, %3;\n" : "=r"(w) : "r"(own), "r"(nb), "r"(sel));
+        asm volatile("st.shared.b32 [%0], %1;\n" ::"r"(col + (uint32_t)(j * 64)), "r"(w)
                      : "memory");
     }
 }
