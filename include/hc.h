@@ -219,16 +219,20 @@ hc_status hc_sparse_conv_rulebook_fwd(const void* x, hc_dtype dt, int x_rows,
 /*
  * hc_sparse_conv_rulebook_fwd_hint -- hc_sparse_conv_rulebook_fwd with the
  * caller's host-side estimate of N' (rows_hint >= 0; 0 = unknown), which
- * the call uses only to choose how the tensor cores tile the rows: N' lives
- * on the device, and the tiling that is fastest for many rows (two 128-row
- * halves per item sharing every weight stage, multiplied as one
- * M = 128 channels x N = 256 rows product) is slower when there are too few
- * items to fill the GPU. It is taken when rows_hint gives at least one such
- * item per SM (about 39k rows on 152 SMs), for bf16, C_out = 128, and
- * neither out nor group-norm statistics; otherwise the call is
- * hc_sparse_conv_rulebook_fwd. The results are bit-identical either way, so
- * any estimate (the previous batch's count, the mask's expected density) is
- * safe: a wrong one only costs time. rows_hint < 0 is HC_ERR_INVALID_ARG.
+ * the call uses only to choose how the tensor cores tile the rows. The
+ * tiling that is fastest for many rows (two 128-row halves per item sharing
+ * every weight stage, multiplied as one M = 128 channels x N = 256 rows
+ * product) is slower when there are too few items to fill the GPU; it
+ * applies to bf16, C_out = 128, and neither out nor group-norm statistics.
+ * With rows_hint giving at least one such item per SM (about 39k rows on
+ * 152 SMs) the launch uses it directly; with a smaller nonzero estimate it
+ * uses one-half items; with none (0, and in hc_sparse_conv_rulebook_fwd)
+ * a call whose capacity could fill the SMs with such items launches a
+ * kernel that reads N' on the device and chooses (a little slower than a
+ * direct launch at small N': ~0.2 us). The results are bit-identical in
+ * every case, so any estimate (the previous batch's count, the mask's
+ * expected density) is safe: a wrong one only costs time. rows_hint < 0 is
+ * HC_ERR_INVALID_ARG.
  */
 hc_status hc_sparse_conv_rulebook_fwd_hint(const void* x, hc_dtype dt, int x_rows,
                                            const int32_t* rulebook, const int32_t* count,
