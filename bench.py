@@ -59,7 +59,7 @@ def parse_args():
                                        "kappa", "configs", "stages"],
                    default="all", help="run only this side measurement")
     p.add_argument("--clocks-csv", default=None, help="also write the raw clock samples here")
-    p.add_argument("--e2e-steps", type=int, default=30)
+    p.add_argument("--e2e-steps", type=int, default=200)
     p.add_argument("--no-e2e", action="store_true",
                    help="skip the end-to-end measurement (for targeted profiler captures)")
     p.add_argument("--case", default=None,
@@ -559,27 +559,32 @@ def time_torch_dense(torch, sets, w, Wt, bias, stream, dev):
     return t0.elapsed_time(t1) / len(sets)
 
 
+E2E_IN_FLIGHT = 8  # buffer sets (and streams) of the end-to-end loop
+
+
 def measure_e2e(torch, hc, sets, w, spiral, Wt, bias, stream, dev, steps):
-    """Same metric through the C-ABI with host inputs: every step copies its
-    mask from pinned host memory, compacts it and builds the Eq. 4 mapping
-    (compact layout), gathers the active rows of its dense features straight
-    from the pinned host buffer (hc_gather_rows reading host memory: only the
-    active rows cross the host link), runs the conv on those compact rows
-    (with the fused scatter), and reads back the count, the coordinates and
-    the compact output rows. A step's device work (mask copy, the three
-    library calls, the count's read-back) is one CUDA graph per input set.
-    Steps are pipelined over two buffer sets, as a serving loop would run
-    them: the rows' read-back of step i-1 (on a second stream) overlaps step
-    i. Every step moves the inputs it uses and all of its results; the host
-    learns each step's row count before reading its rows."""
+    """Same metric through the C-ABI with host inputs and outputs: every step
+    copies its mask from pinned host memory, compacts it and builds the Eq. 4
+    mapping (compact layout), gathers the active rows of its dense features
+    straight from the pinned host buffer (hc_gather_rows reading host memory:
+    only the active rows cross the host link), runs the conv on those compact
+    rows (with the fused scatter), and writes its results to pinned host
+    memory: the count (a copy), the coordinates and the compact output rows
+    (hc_gather_rows in row order, the copy sized by the count on the device,
+    so the host never waits for N' inside the loop). A step is one CUDA graph
+    per input set; steps rotate over E2E_IN_FLIGHT buffer sets, each with its
+    own stream (and so its own library workspace), as a serving loop with
+    that many requests in flight would run them. Every step moves the inputs it uses and
+    all of its results."""
     ly = w.layers[0]
     B, V = w.B, w.V
     host = []
     for s in sets:
         host.append((s.mask.cpu().pin_memory(), s.x.cpu().pin_memory()))
-    nb = 2
+    nb = E2E_IN_FLIGHT
+    streams = [stream] + [torch.cuda.Stream(device=dev) for _ in range(nb - 1)]
     mask_d = [torch.empty_like(sets[0].mask) for _ in range(nb)]
-    outs = []  # device outputs of buffer b (the input sets' own buffers stay as they are)
+    outs = []  # device buffers of buffer set b (the input sets' own buffers stay as they are)
     for _ in range(nb):
         o = LayerSet()
         o.coords = torch.empty((B * V, 2), dtype=torch.int32, device=dev)
@@ -594,83 +599,60 @@ def measure_e2e(torch, hc, sets, w, spiral, Wt, bias, stream, dev, steps):
     cnt_h = [torch.empty((1,), dtype=torch.int32).pin_memory() for _ in range(nb)]
     y_h = [torch.empty((B * V, ly.C_out), dtype=torch.bfloat16).pin_memory() for _ in range(nb)]
     c_h = [torch.empty((B * V, 2), dtype=torch.int32).pin_memory() for _ in range(nb)]
-    back_s = torch.cuda.Stream(device=dev)
 
-    def event():
-        return torch.cuda.Event()
-
-    computed = [event() for _ in range(nb)]
-    drained = [event() for _ in range(nb)]
-    acc = {"h2d": 0, "d2h": 0, "rows": 0}
-
-    def device_part(j):
+    def step(j):
         b = j % nb
         mh, xh = host[j]
         o = outs[b]
+        st = streams[b]
         mask_d[b].copy_(mh, non_blocking=True)
         hc.hc_mask_compact_rulebook(mask_d[b], spiral, hc.HC_LAYOUT_COMPACT, o.coords,
-                                    o.row_of, o.offs, o.count, o.rb, stream)
-        hc.hc_gather_rows(xh, o.coords, o.count, 1, o.xc, stream)  # rows from host memory
+                                    o.row_of, o.offs, o.count, o.rb, st)
+        hc.hc_gather_rows(xh, o.coords, o.count, 1, o.xc, st)  # rows from host memory
         hc.hc_sparse_conv_rulebook_fwd(o.xc, o.rb, o.count, Wt, bias, ly.act, o.y,
-                                       coords=o.coords, out=o.out, stream=stream)
+                                       coords=o.coords, out=o.out, stream=st)
         cnt_h[b].copy_(o.count, non_blocking=True)
+        # the first N' coordinates and rows, into pinned host memory
+        hc.hc_gather_rows(o.coords.view(torch.float32).view(1, B * V, 2), None, o.count, 1,
+                          c_h[b].view(torch.float32), st)
+        hc.hc_gather_rows(o.y.view(1, B * V, ly.C_out), None, o.count, 1, y_h[b], st)
 
-    # one CUDA graph per input set (set j always uses buffer j % nb): the mask
-    # copy, the three library calls and the count's read-back
+    # one CUDA graph per input set, captured on its buffer set's stream
     assert len(host) % nb == 0
-    with torch.cuda.stream(stream):
-        for j in range(len(host)):
-            device_part(j)
+    for j in range(len(host)):
+        with torch.cuda.stream(streams[j % nb]):
+            step(j)
     torch.cuda.synchronize(dev)
     graphs = []
     for j in range(len(host)):
         g = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g, stream=stream):
-            device_part(j)
+        with torch.cuda.graph(g, stream=streams[j % nb]):
+            step(j)
         graphs.append(g)
-
-    def launch(i):
-        b = i % nb
-        j = i % len(host)
-        if i >= nb:
-            stream.wait_event(drained[b])  # step i - 2's rows have been read back
-        with torch.cuda.stream(stream):
-            graphs[j].replay()
-            computed[b].record(stream)
-        acc["h2d"] += host[j][0].numel()
-
-    def read_back(i):
-        b = i % nb
-        o = outs[b]
-        computed[b].synchronize()  # the host needs the row count
-        n = int(cnt_h[b][0])
-        back_s.wait_event(computed[b])
-        with torch.cuda.stream(back_s):
-            y_h[b][:n].copy_(o.y[:n], non_blocking=True)
-            c_h[b][:n].copy_(o.coords[:n], non_blocking=True)
-            drained[b].record(back_s)
-        acc["h2d"] += n * ly.C_in * 2  # the active feature rows read from host memory
-        acc["d2h"] += 4 + n * 8 + n * ly.C_out * 2
-        acc["rows"] += n
+    acc = {"h2d": 0, "d2h": 0, "rows": 0}
 
     def run(k):
         for i in range(k):
-            launch(i)
-            if i >= 1:
-                read_back(i - 1)
-        read_back(k - 1)
+            j = i % len(host)
+            with torch.cuda.stream(streams[j % nb]):
+                graphs[j].replay()
+            n = sets[j].rows  # the count this input set's mask gives (checked below)
+            acc["h2d"] += host[j][0].numel() + n * ly.C_in * 2  # mask + active feature rows
+            acc["d2h"] += 4 + n * 8 + n * ly.C_out * 2
+            acc["rows"] += n
         torch.cuda.synchronize(dev)
 
-    run(4)  # warm-up (and the library's per-stream workspaces)
+    run(4)  # warm-up
     for key in acc:
         acc[key] = 0
     torch.cuda.synchronize(dev)
     t0 = time.perf_counter()
     run(steps)
     dt = time.perf_counter() - t0
-    # the last step's rows as read back, against the same input set's rows
-    # from the device-resident step timed above (dense layout, same kernels)
-    last, b = steps - 1, (steps - 1) % nb
+    # the last step's results as written to host memory, against the same
+    # input set's from the device-resident step timed above
+    last = steps - 1
+    b = (last % len(host)) % nb
     s_ref = sets[last % len(host)]
     n = int(cnt_h[b][0])
     same = (n == s_ref.rows and
@@ -683,9 +665,10 @@ def measure_e2e(torch, hc, sets, w, spiral, Wt, bias, stream, dev, steps):
             "ms_per_step": dt / steps * 1e3,
             "path": "pinned host mask (copied) + pinned host features (active rows gathered "
                     "by hc_gather_rows over the host link) -> hc_mask_compact_rulebook, "
-                    "hc_gather_rows, hc_sparse_conv_rulebook_fwd -> count, coords, rows to "
-                    "host; one CUDA graph per step's device work, two buffer sets, step i-1's "
-                    "read-back overlapping step i"}
+                    "hc_gather_rows, hc_sparse_conv_rulebook_fwd -> count (copied), coords "
+                    "and rows (hc_gather_rows in row order, sized on the device) into pinned "
+                    f"host memory; one CUDA graph per step, {nb} buffer sets on {nb} streams, "
+                    "no host wait inside the loop"}
 
 
 def run_sweep(torch, hc, dev, stream):

@@ -410,6 +410,12 @@ hc_status hc_kappa_masks(const uint8_t* masks, int K, int V, const int32_t* sele
  * reads only the active rows across the host link (zero-copy), which is how
  * a dense host-side input becomes compact device rows without copying the
  * whole tensor.
+ * coords may be NULL: y[n] = row n of x (x viewed as B_in * V rows of C;
+ * frames_per_sample unused) for n < *count, rows n >= B_in * V reported
+ * (HC_ERR_INVALID_INDEX) and left untouched: a copy of the first N' rows
+ * sized on the device. With y in pinned host memory this reads compact
+ * results back without the host learning N' first (no host wait between
+ * the producing call and the copy).
  */
 hc_status hc_gather_rows(const void* x, hc_dtype dt, int B_in, int V, int C, const int32_t* coords,
                          const int32_t* count, int capacity, int frames_per_sample, void* y,

@@ -637,7 +637,7 @@ hc_status hc_gather_rows(const void* x, hc_dtype dt, int B_in, int V, int C, con
                frames_per_sample);
     HC_REQUIRE(count != nullptr, "%s: count is NULL", fn);
     if (capacity == 0) return HC_OK;
-    HC_REQUIRE(x && coords && y, "%s: x, coords and y are required", fn);
+    HC_REQUIRE(x && y, "%s: x and y are required", fn);
     const int eb = dt == HC_F32 ? 4 : 2;
     HC_REQUIRE(!misaligned(x, eb) && !misaligned(y, eb), "%s: misaligned x/y", fn);
     const DeviceCtx* ctx = device_ctx();

@@ -6,7 +6,9 @@
 //                       f = b * kappa + j is sample b under mask selected[j]
 //   gather_rows_kernel  the feature matrix S' of Eq. 2: the input row of
 //                       every active coordinate (f, v), frame f reading
-//                       sample f / frames_per_sample
+//                       sample f / frames_per_sample; without coordinates,
+//                       the first N' rows in order (a copy sized on the
+//                       device)
 #include "hc_internal.cuh"
 
 namespace hc {
@@ -114,6 +116,15 @@ __global__ void gather_rows_kernel(const U* __restrict__ x, long long B_in, int 
          i += (long long)gridDim.x * blockDim.x) {
         int c;
         const long long n = div32(i, cpr, c);
+        if (!coords) {
+            // rows in order: x viewed as B_in * V rows
+            if (n >= B_in * V) {
+                if (c == 0) report(status, kErrIndex);
+                continue;
+            }
+            y[i] = x[i];
+            continue;
+        }
         const int f = __ldg(coords + 2 * n), v = __ldg(coords + 2 * n + 1);
         const long long b = f >= 0 ? f / frames_per_sample : -1;
         if (b < 0 || b >= B_in || v < 0 || v >= V) {

@@ -298,11 +298,12 @@ def hc_kappa_masks(masks, selected, B, out, stream=None):
 
 
 def hc_gather_rows(x, coords, count, frames_per_sample, y, stream=None):
-    """S' of Eq. 2: y[n] = x[f // frames_per_sample, v] for coords[n] = (f, v).
-    x may be a pinned host tensor: only the active rows cross the host link."""
+    """S' of Eq. 2: y[n] = x[f // frames_per_sample, v] for coords[n] = (f, v);
+    coords None: y[n] = x row n (x viewed as B_in * V rows), n < count. x or y
+    may be a pinned host tensor: only the rows copied cross the host link."""
     B_in, V, C = x.shape
     _check(load_library().hc_gather_rows(_p_host_ok(x), _dt(x), B_in, V, C, _p(coords), _p(count),
-                                         y.shape[0], frames_per_sample, _p(y), _s(stream)),
+                                         y.shape[0], frames_per_sample, _p_host_ok(y), _s(stream)),
            "hc_gather_rows")
 
 

@@ -154,14 +154,15 @@ def test_gather_rows_arguments_rejected_on_host(lib):
         return g(x, dt, B_in, V, C, coords, count, cap, fps, y, None)
 
     for kw in (dict(dt=9), dict(B_in=-1), dict(C=0), dict(fps=0), dict(cap=-1), dict(count=None),
-               dict(x=None), dict(coords=None), dict(y=None), dict(x=ctypes.c_void_p(0x1001))):
+               dict(x=None), dict(y=None), dict(x=ctypes.c_void_p(0x1001))):
         assert call(**kw) == hc.HC_ERR_INVALID_ARG, kw
     assert call(cap=0) == hc.HC_OK  # nothing to gather: no device call
+    assert call(cap=0, coords=None) == hc.HC_OK  # rows in order: coords are optional
 
 
 def test_binding_refuses_pageable_host_tensors(lib):
-    """Host memory is accepted only pinned, and only as hc_gather_rows' input;
-    a pageable tensor is refused before any library call."""
+    """Host memory is accepted only pinned, and only by hc_gather_rows (its
+    input and output); a pageable tensor is refused before any library call."""
     torch = pytest.importorskip("torch")
     x = torch.zeros((2, 10, 8), dtype=torch.float32)
     coords = torch.zeros((20, 2), dtype=torch.int32)

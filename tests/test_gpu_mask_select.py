@@ -185,6 +185,43 @@ def test_gather_rows_from_pinned_host_memory(dtype):
         hc.hc_gather_rows(xt.cpu(), coords, count, 1, y)
 
 
+@pytest.mark.parametrize("dtype,C", [("bf16", 128), ("f32", 2), ("bf16", 3)])
+def test_gather_rows_in_order_into_pinned_host_memory(dtype, C):
+    """coords NULL: the first N' rows of a device tensor copied in order into
+    pinned host memory, the count read on the device (16-, 4- and 2-byte
+    chunks); rows past N' untouched; N' above the capacity clamped
+    (HC_ERR_CAPACITY), N' above the input's rows reported
+    (HC_ERR_INVALID_INDEX) with those rows untouched."""
+    rng = np.random.default_rng(C)
+    cap = 5000
+    x = inputs.features(rng, (1, cap, C), dtype)
+    xt = to_torch(x)
+    for n in (0, 1, 3777, cap):
+        count = torch.tensor([n], dtype=torch.int32, device="cuda")
+        yh = torch.full((cap, C), 7, dtype=xt.dtype).pin_memory()
+        hc.hc_gather_rows(xt, None, count, 1, yh)
+        torch.cuda.synchronize()
+        assert hc.hc_get_device_status() == hc.HC_OK
+        assert torch.equal(yh[:n], xt[0, :n].cpu())
+        assert (yh[n:] == 7).all()
+    # capacity below N': clamped
+    count = torch.tensor([cap], dtype=torch.int32, device="cuda")
+    yh = torch.full((100, C), 7, dtype=xt.dtype).pin_memory()
+    hc.hc_gather_rows(xt, None, count, 1, yh)
+    torch.cuda.synchronize()
+    assert hc.hc_get_device_status() == hc.HC_ERR_CAPACITY
+    assert torch.equal(yh, xt[0, :100].cpu())
+    # input rows below N': the rows past the input reported and untouched
+    xs = xt[:, :1000].contiguous()
+    count = torch.tensor([1200], dtype=torch.int32, device="cuda")
+    yh = torch.full((cap, C), 7, dtype=xt.dtype).pin_memory()
+    hc.hc_gather_rows(xs, None, count, 1, yh)
+    torch.cuda.synchronize()
+    assert hc.hc_get_device_status() == hc.HC_ERR_INVALID_INDEX
+    assert torch.equal(yh[:1000], xs[0].cpu())
+    assert (yh[1000:] == 7).all()
+
+
 def test_kappa_inference_chain():
     """alpha -> top-3 -> kappa masks for every sample -> compaction -> S'
     -> sparse spiral conv on the compact rows, against the same chain on
