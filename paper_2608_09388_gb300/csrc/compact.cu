@@ -68,6 +68,7 @@ __device__ __forceinline__ uint32_t load_flags(const uint8_t* mask, long long n,
     return flags;
 }
 
+template <int NT>
 __device__ __forceinline__ int block_sum(int v, int* red) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
 #pragma unroll
@@ -77,7 +78,7 @@ __device__ __forceinline__ int block_sum(int v, int* red) {
     __syncthreads();
     int t = 0;
 #pragma unroll
-    for (int w = 0; w < kThreads / 32; ++w) t += red[w];
+    for (int w = 0; w < NT / 32; ++w) t += red[w];
     return t;
 }
 
@@ -89,7 +90,7 @@ __global__ void __launch_bounds__(kThreads) compact_count_kernel(const uint8_t* 
     pdl_trigger();
     long long base = (long long)blockIdx.x * kTile + (long long)threadIdx.x * kItems;
     int c = __popc(load_flags(mask, n, base));
-    int t = block_sum(c, red);
+    int t = block_sum<kThreads>(c, red);
     if (threadIdx.x == 0) tile_counts[blockIdx.x] = t;
 }
 
@@ -159,7 +160,7 @@ __global__ void __launch_bounds__(kThreads)
     } else {
         int part = 0;
         for (int t = tid; t < tile; t += kThreads) part += tile_counts[t];
-        tile_base = block_sum(part, red);
+        tile_base = block_sum<kThreads>(part, red);
     }
 
     int c = __popc(flags);
@@ -233,7 +234,7 @@ __global__ void __launch_bounds__(kThreads)
 
     // The last tile knows the total.
     if (tile == num_tiles - 1) {
-        int tot = block_sum(c, red);
+        int tot = block_sum<kThreads>(c, red);
         if (tid == 0) {
             *count = tile_base + tot;
             if (offsets) offsets[B] = tile_base + tot;
@@ -372,7 +373,7 @@ __global__ void __launch_bounds__(kMapThreads) compact_map_kernel(const MapArgs 
             r += __popc((uint32_t)s_flag[c]);
         }
     }
-    const int part = block_sum(__popc(pf), red);  // synchronises: the chunk tables are complete
+    const int part = block_sum<kMapThreads>(__popc(pf), red);  // synchronises: the chunk tables are complete
     // rank of vertex p (active rows of the frame before it) and its activity
     auto rank_of = [&](int p, bool& on) {
         const int q = p + sh, c = q >> 4, k = q & 15;
@@ -413,7 +414,7 @@ __global__ void __launch_bounds__(kMapThreads) compact_map_kernel(const MapArgs 
     } else {
         int acc = 0;
         for (int t = tid; t < tb; t += kMapThreads) acc += a.tile_counts[t];
-        before = block_sum(acc, red);
+        before = block_sum<kMapThreads>(acc, red);
     }
     const int off = before + part;  // rows before frame b
     if (tid == 0 && s == 0) {
