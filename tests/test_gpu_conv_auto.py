@@ -15,7 +15,7 @@ import pytest
 import oracle
 from paper_2608_09388_gb300 import hc, inputs
 
-from _util import check_close, to_numpy, to_torch
+from _util import check_close, sample_rows, to_numpy, to_torch
 
 pytestmark = pytest.mark.gpu
 
@@ -65,7 +65,7 @@ def rulebook(m, sp):
     row_of = torch.empty((B, V), dtype=torch.int32, device="cuda")
     offs = torch.empty((B + 1,), dtype=torch.int32, device="cuda")
     count = torch.empty((1,), dtype=torch.int32, device="cuda")
-    rb = torch.empty((L, B * V), dtype=torch.int32, device="cuda")
+    rb = torch.empty((sp.shape[1], B * V), dtype=torch.int32, device="cuda")
     hc.hc_mask_compact_rulebook(to_torch(m), to_torch(sp), hc.HC_LAYOUT_DENSE, coords, row_of,
                                 offs, count, rb)
     return rb, count
@@ -142,3 +142,41 @@ def test_bad_entries_reported_in_both_branches(case, offset):
     y_abs = run(xt, rb, count, Wt, bt)
     assert hc.hc_get_device_status() == hc.HC_OK
     assert torch.equal(y[:n], y_abs[:n])
+
+
+@pytest.mark.parametrize("L,C_in,act", [(1, 64, hc.HC_ACT_ELU), (12, 64, hc.HC_ACT_RELU),
+                                        (32, 64, hc.HC_ACT_NONE), (9, 45, hc.HC_ACT_ELU),
+                                        (5, 200, hc.HC_ACT_ELU)])
+@pytest.mark.parametrize("branch", ["one-half", "two-half"])
+def test_spiral_lengths_and_channels(L, C_in, act, branch):
+    """Other spiral lengths (one k-block per slot up to 32 slots: the rings'
+    stage counts change with the tables' size), 45 input channels (padded to
+    48 by the channel-padding pass, then this kernel), 200 (a ragged last
+    k-block), each activation, in both branches: sampled rows (all of the
+    first and last item) against the oracle, every row bit-identical to the
+    call forcing that item shape, rows past N' untouched."""
+    rng = np.random.default_rng(L * 1000 + C_in)
+    sp = rng.integers(0, V, size=(V, L)).astype(np.int32)
+    sp[rng.random((V, L)) < 0.1] = -1
+    sp[:, 0] = np.arange(V)
+    x = inputs.features(rng, (B, V, C_in), "bf16")
+    W = inputs.weights(rng, L * C_in, 128, "bf16")
+    b = rng.standard_normal(128).astype(np.float32)
+    n = threshold() + 123 if branch == "two-half" else 20000
+    m = mask_with(rng.permutation(B * V), n)
+    rb, count = rulebook(m, sp)
+    xt, Wt, bt = to_torch(x), to_torch(W), to_torch(b)
+    y = torch.full((B * V, 128), float("nan"), dtype=torch.bfloat16, device="cuda")
+    hc.hc_sparse_conv_rulebook_fwd(xt, rb, count, Wt, bt, act, y)
+    assert hc.hc_get_device_status() == hc.HC_OK
+    assert torch.isnan(y[n:].float()).all()
+    forced = torch.full_like(y, float("nan"))
+    hc.hc_sparse_conv_rulebook_fwd_hint(xt, rb, count, Wt, bt, act, forced,
+                                        B * V if branch == "two-half" else 1)
+    assert torch.equal(forced[:n], y[:n])
+    c, r, _, _ = oracle.mask_compact(m)
+    rows = np.unique(np.concatenate([np.arange(256), np.arange(n - 256, n),
+                                     sample_rows(n, 3000, seed=L)]))
+    y_pre, _ = oracle.sparse_spiral_conv(x, oracle.LAYOUT_DENSE, c, r, sp, W, b, act, rows=rows,
+                                         n_threads=NCPU)
+    check_close(to_numpy(y)[rows], y_pre, f"auto L={L} C_in={C_in} {branch}")
