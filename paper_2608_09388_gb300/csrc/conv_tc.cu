@@ -8,11 +8,14 @@
 // the bias of Eq. 6) and the activation of Eq. 10.
 //
 // One persistent CTA per SM, 352 threads in five roles (384 with two-half
-// items). A work item is tm 128-row halves of output rows (tm = 2 for the
-// dense layer when it gives every SM at least two items, else 1) times BN
-// output channels; both halves are multiplied by the same W slice of every
-// stage, which halves the weight traffic and the per-stage overhead per MMA
-// of large layers.
+// items). A work item is tm 128-row halves of output rows times BN output
+// channels; both halves are multiplied by the same W slice of every stage,
+// which halves the weight traffic and the per-stage overhead per MMA of
+// large layers. tm = 2 for the dense layer when it gives every SM at least
+// two items, and for a rulebook call whose host-side row estimate gives
+// every SM one; a rulebook call without an estimate but with the capacity
+// for that many goes to conv_tc_auto_kernel, which reads the row count on
+// the device and runs whichever role set it calls for; else tm = 1.
 //   warp 9     index warp: for each item, resolves the L x (tm*128) tap table
 //              (from the rulebook, or coords -> spiral -> row_of, i.e. idx()
 //              of Eq. 4) with every load of a phase in flight at once, into
@@ -47,9 +50,11 @@
 // holds a channel per TMEM lane and a row per column, so the epilogue stages
 // each 32 x 32 block transposed through shared memory, and the bias is one
 // value per lane.
-// Each role runs its whole loop in a copy compiled for its half count (the
-// count is known once the row count is read); a run-time half loop between
-// the MMAs and copies cost ~1 us per launch at the small layers.
+// The roles are one function template (conv_roles) instantiated per half
+// count and layout: each role runs its whole loop in a copy compiled for its
+// half count (a run-time half loop between the MMAs and copies cost ~1 us
+// per launch at the small layers), and conv_tc_auto_kernel holds the
+// one-half and the transposed two-half copies, one branch taken per launch.
 // The stage ring holds a.stages two-half stages; one-half items cut the same
 // bytes into more (up to kRing) stages of 16 KB of A plus the W slice.
 // Shared-memory operand layouts (canonical tcgen05 forms, 128-byte swizzle):
