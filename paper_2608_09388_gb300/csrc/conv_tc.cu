@@ -1083,11 +1083,12 @@ struct AutoLayout {
     }
 };
 
-// 128-channel rulebook calls whose row count is on the device: every CTA
-// reads the count after the launch dependency and runs two-half transposed
-// items when each CTA gets at least one (rows >= 256 per CTA), one-half
-// items otherwise. Both role sets are compiled in and each branch is taken
-// whole, so neither pays for the other in its loops. The one-half roles'
+// 128-channel sparse calls (rulebook, or taps resolved from coords, spiral
+// and row_of) whose row count is on the device: every CTA reads the count
+// after the launch dependency and runs two-half transposed items when each
+// CTA gets at least one (rows >= 256 per CTA), one-half items otherwise.
+// Both role sets are compiled in and each branch is taken whole, so neither
+// pays for the other in its loops. The one-half roles' rulebook-mode
 // first-table prefetch (issued before the count is known) completes its own
 // table-full pair; when the two-half roles run instead, the prefetching
 // warp waits for those copies before the tables are rebuilt, and their
@@ -1137,9 +1138,9 @@ __global__ void __launch_bounds__(kThreadsFor<2>, 1)
     pdl_wait();
     pdl_trigger();
 
-    // the one-half roles' first table, copied while the row count is read
-    // (as in conv_tc_kernel)
-    const bool prefetch = warp == kIndexWarp;
+    // rulebook mode: the one-half roles' first table, copied while the row
+    // count is read (as in conv_tc_kernel)
+    const bool prefetch = warp == kIndexWarp && a.mode == kRulebook;
     if (prefetch) {
         const long long m0p = (long long)blockIdx.x * kBM;
         for (int d = 0; d < a.L; ++d)
@@ -1412,11 +1413,14 @@ hc_status launch_conv_tc(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s
     // 32 -> 28 us at 67k rows (1.7 items per SM), the same at 33k (0.9 per
     // SM), 11 -> 18 us at 6.8k (0.2 per SM). The results are the same either
     // way.
-    // Without an estimate (rows_hint 0), a call whose capacity could fill
-    // every SM with two-half items leaves the choice to the CTAs, which read
-    // the row count (conv_tc_auto_kernel).
-    if (a.mode == kRulebook && a.C_out == 128 && !a.out_dense && !a.gn_part && a.C_in % 8 == 0) {
-        if ((a.rows_hint + 2 * kBM - 1) / (2 * kBM) >= ctx->num_sms)
+    // Without an estimate (rows_hint 0), a sparse call (rulebook or
+    // resolved taps) whose capacity could fill every SM with two-half items
+    // leaves the choice to the CTAs, which read the row count
+    // (conv_tc_auto_kernel).
+    const bool sparse = a.mode == kRulebook || a.mode == kSparseDenseX ||
+                        a.mode == kSparseCompactX;
+    if (sparse && a.C_out == 128 && !a.out_dense && !a.gn_part && a.C_in % 8 == 0) {
+        if (a.mode == kRulebook && (a.rows_hint + 2 * kBM - 1) / (2 * kBM) >= ctx->num_sms)
             return launch_bn<128, 2, true>(ctx, a, s);
         if (a.rows_hint == 0 && (a.capacity + 2 * kBM - 1) / (2 * kBM) >= ctx->num_sms)
             return launch_auto(ctx, a, s);

@@ -180,3 +180,45 @@ def test_spiral_lengths_and_channels(L, C_in, act, branch):
     y_pre, _ = oracle.sparse_spiral_conv(x, oracle.LAYOUT_DENSE, c, r, sp, W, b, act, rows=rows,
                                          n_threads=NCPU)
     check_close(to_numpy(y)[rows], y_pre, f"auto L={L} C_in={C_in} {branch}")
+
+
+@pytest.mark.parametrize("layout", [hc.HC_LAYOUT_DENSE, hc.HC_LAYOUT_COMPACT])
+@pytest.mark.parametrize("offset", [-1, 7, None])
+def test_resolved_taps_both_layouts(case, layout, offset):
+    """hc_sparse_spiral_conv_fwd (taps resolved from coords, spiral and
+    row_of inside the kernel) goes through the same dispatch: one-half items
+    below 256 rows per SM, two-half transposed items from there up to every
+    vertex active (offset None), dense and compact inputs; bit-identical to
+    the rulebook call on the same layout, sampled rows (all of the first and
+    last item) against the oracle, rows past N' untouched."""
+    sp, x, W, b, order = case
+    n = B * V if offset is None else threshold() + offset
+    m = mask_with(order, n)
+    coords = torch.empty((B * V, 2), dtype=torch.int32, device="cuda")
+    row_of = torch.empty((B, V), dtype=torch.int32, device="cuda")
+    offs = torch.empty((B + 1,), dtype=torch.int32, device="cuda")
+    count = torch.empty((1,), dtype=torch.int32, device="cuda")
+    rb = torch.empty((L, B * V), dtype=torch.int32, device="cuda")
+    hc.hc_mask_compact_rulebook(to_torch(m), to_torch(sp), layout, coords, row_of, offs, count, rb)
+    c, r, _, n_ref = oracle.mask_compact(m)
+    assert int(count.item()) == n == n_ref
+    if layout == hc.HC_LAYOUT_DENSE:
+        xin, x_np = to_torch(x), x
+    else:
+        x_np = np.zeros((B * V, C_IN), x.dtype)
+        x_np[:n] = x[c[:, 0], c[:, 1]]
+        xin = to_torch(x_np)
+    Wt, bt = to_torch(W), to_torch(b)
+    y = torch.full((B * V, 128), float("nan"), dtype=torch.bfloat16, device="cuda")
+    hc.hc_sparse_spiral_conv_fwd(xin, layout, coords, row_of, count, to_torch(sp), B, V, Wt, bt,
+                                 hc.HC_ACT_ELU, y)
+    assert hc.hc_get_device_status() == hc.HC_OK
+    assert torch.isnan(y[n:].float()).all()
+    ref = run(xin.view(-1, C_IN), rb, count, Wt, bt)
+    assert torch.equal(y[:n], ref[:n])
+    rows = np.unique(np.concatenate([np.arange(256), np.arange(n - 256, n),
+                                     sample_rows(n, 3000, seed=n)]))
+    lay = oracle.LAYOUT_DENSE if layout == hc.HC_LAYOUT_DENSE else oracle.LAYOUT_COMPACT
+    y_pre, _ = oracle.sparse_spiral_conv(x_np if layout == hc.HC_LAYOUT_COMPACT else x, lay, c, r,
+                                         sp, W, b, oracle.ACT_ELU, rows=rows, n_threads=NCPU)
+    check_close(to_numpy(y)[rows], y_pre, f"resolved taps layout={layout} N'={n}")
