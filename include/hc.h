@@ -143,7 +143,11 @@ hc_status hc_mask_compact_static(const uint8_t* mask, int B, int V, int32_t* coo
  * needs only 2-byte alignment) x and W are first copied, with zero channels
  * appended up to C_pad = the next multiple of 8, into the per-stream
  * workspace (x_rows * C_pad * 2 + L * C_pad * C_out * 2 bytes; compact inputs
- * copy their first N' rows only); the sums are unchanged.
+ * copy their first N' rows only); the sums are unchanged. With C_out = 128
+ * and B*V of at least 256 rows per SM, the kernel reads N' on the device and
+ * multiplies 256-row items (two 128-row halves sharing each weight stage) when
+ * every SM gets one, 128-row items otherwise; the results are the same bits
+ * either way.
  */
 hc_status hc_sparse_spiral_conv_fwd(const void* x, hc_layout x_layout, hc_dtype dt,
                                     const int32_t* coords, const int32_t* row_of,
