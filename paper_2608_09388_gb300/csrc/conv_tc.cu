@@ -1400,10 +1400,11 @@ hc_status launch_conv_tc(const DeviceCtx* ctx, const ConvArgs& a, cudaStream_t s
     }
     // Two-half items when the row count is known on the host (the dense
     // layer) and fills every SM with at least two of them: they halve the
-    // weight traffic and per-stage overhead per MMA. The sparse calls' row
-    // count lives on the device, and the two-half code paths compiled into
-    // the same kernel cost the small layers ~1 us (instruction fetch), so
-    // they run one-half items.
+    // weight traffic and per-stage overhead per MMA. A sparse call's row
+    // count lives on the device, and two-half code paths compiled into the
+    // loops of the one-half kernel cost the small layers ~1 us (instruction
+    // fetch); such calls take two-half items through a row estimate or
+    // conv_tc_auto_kernel (below), one-half items otherwise.
     const long long n_tiles = (a.C_out + 127) / 128;
     const bool two = a.mode == kDense && (a.capacity + 2 * kBM - 1) / (2 * kBM) * n_tiles >=
                                              2ll * ctx->num_sms;
