@@ -46,6 +46,9 @@ METRIC = "active vertex-rows/s & % roofline, sparse spiral-conv layer; speed-up 
 WORKLOAD = "layer10475_bf16"
 
 
+E2E_IN_FLIGHT = 8  # default requests in flight of the end-to-end loop
+
+
 def parse_args():
     p = argparse.ArgumentParser()
     p.add_argument("--gpus", type=int, default=1)
@@ -60,6 +63,8 @@ def parse_args():
                    default="all", help="run only this side measurement")
     p.add_argument("--clocks-csv", default=None, help="also write the raw clock samples here")
     p.add_argument("--e2e-steps", type=int, default=200)
+    p.add_argument("--e2e-in-flight", type=int, default=E2E_IN_FLIGHT,
+                   help="requests in flight in the end-to-end loop (buffer sets and streams)")
     p.add_argument("--no-e2e", action="store_true",
                    help="skip the end-to-end measurement (for targeted profiler captures)")
     p.add_argument("--case", default=None,
@@ -388,7 +393,8 @@ def run_ours(args, rank, world, local_rank):
 
     e2e = None
     if not args.no_e2e:
-        e2e = measure_e2e(torch, hc, sets, w, spiral, Wt, bias, stream, dev, args.e2e_steps)
+        e2e = measure_e2e(torch, hc, sets, w, spiral, Wt, bias, stream, dev, args.e2e_steps,
+                          args.e2e_in_flight)
         # whole-job end-to-end figure: rows of all ranks over the slowest rank's time
         e2e_rows, e2e_ms = reduce_over_ranks(float(e2e.pop("rows")), e2e.pop("seconds") * 1e3,
                                              world, dev)
@@ -559,10 +565,7 @@ def time_torch_dense(torch, sets, w, Wt, bias, stream, dev):
     return t0.elapsed_time(t1) / len(sets)
 
 
-E2E_IN_FLIGHT = 8  # buffer sets (and streams) of the end-to-end loop
-
-
-def measure_e2e(torch, hc, sets, w, spiral, Wt, bias, stream, dev, steps):
+def measure_e2e(torch, hc, sets, w, spiral, Wt, bias, stream, dev, steps, in_flight):
     """Same metric through the C-ABI with host inputs and outputs: every step
     copies its mask from pinned host memory, compacts it and builds the Eq. 4
     mapping (compact layout), gathers the active rows of its dense features
@@ -572,16 +575,17 @@ def measure_e2e(torch, hc, sets, w, spiral, Wt, bias, stream, dev, steps):
     memory: the count (a copy), the coordinates and the compact output rows
     (hc_gather_rows in row order, the copy sized by the count on the device,
     so the host never waits for N' inside the loop). A step is one CUDA graph
-    per input set; steps rotate over E2E_IN_FLIGHT buffer sets, each with its
-    own stream (and so its own library workspace), as a serving loop with
-    that many requests in flight would run them. Every step moves the inputs it uses and
-    all of its results."""
+    per buffer set: step i runs on buffer set i % in_flight, which always
+    takes input set (i % in_flight) % len(sets), each buffer set with its own
+    stream (and so its own library workspace), as a serving loop with that
+    many requests in flight would run them. Every step moves the inputs it
+    uses and all of its results."""
     ly = w.layers[0]
     B, V = w.B, w.V
     host = []
     for s in sets:
         host.append((s.mask.cpu().pin_memory(), s.x.cpu().pin_memory()))
-    nb = min(E2E_IN_FLIGHT, len(host))
+    nb = max(1, in_flight)
     streams = [stream] + [torch.cuda.Stream(device=dev) for _ in range(nb - 1)]
     mask_d = [torch.empty_like(sets[0].mask) for _ in range(nb)]
     outs = []  # device buffers of buffer set b (the input sets' own buffers stay as they are)
@@ -600,9 +604,8 @@ def measure_e2e(torch, hc, sets, w, spiral, Wt, bias, stream, dev, steps):
     y_h = [torch.empty((B * V, ly.C_out), dtype=torch.bfloat16).pin_memory() for _ in range(nb)]
     c_h = [torch.empty((B * V, 2), dtype=torch.int32).pin_memory() for _ in range(nb)]
 
-    def step(j):
-        b = j % nb
-        mh, xh = host[j]
+    def step(b):
+        mh, xh = host[b % len(host)]
         o = outs[b]
         st = streams[b]
         mask_d[b].copy_(mh, non_blocking=True)
@@ -617,26 +620,25 @@ def measure_e2e(torch, hc, sets, w, spiral, Wt, bias, stream, dev, steps):
                           c_h[b].view(torch.float32), st)
         hc.hc_gather_rows(o.y.view(1, B * V, ly.C_out), None, o.count, 1, y_h[b], st)
 
-    # one CUDA graph per input set, captured on its buffer set's stream (set
-    # j always uses buffer set j % nb; two consecutive steps that share one,
-    # when nb does not divide the number of sets, run in order on its stream)
-    for j in range(len(host)):
-        with torch.cuda.stream(streams[j % nb]):
-            step(j)
+    # one CUDA graph per buffer set, captured on its stream
+    for b in range(nb):
+        with torch.cuda.stream(streams[b]):
+            step(b)
     torch.cuda.synchronize(dev)
     graphs = []
-    for j in range(len(host)):
+    for b in range(nb):
         g = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g, stream=streams[j % nb]):
-            step(j)
+        with torch.cuda.graph(g, stream=streams[b]):
+            step(b)
         graphs.append(g)
     acc = {"h2d": 0, "d2h": 0, "rows": 0}
 
     def run(k):
         for i in range(k):
-            j = i % len(host)
-            with torch.cuda.stream(streams[j % nb]):
-                graphs[j].replay()
+            b = i % nb
+            with torch.cuda.stream(streams[b]):
+                graphs[b].replay()
+            j = b % len(host)
             n = sets[j].rows  # the count this input set's mask gives (checked below)
             acc["h2d"] += host[j][0].numel() + n * ly.C_in * 2  # mask + active feature rows
             acc["d2h"] += 4 + n * 8 + n * ly.C_out * 2
@@ -652,9 +654,8 @@ def measure_e2e(torch, hc, sets, w, spiral, Wt, bias, stream, dev, steps):
     dt = time.perf_counter() - t0
     # the last step's results as written to host memory, against the same
     # input set's from the device-resident step timed above
-    last = steps - 1
-    b = (last % len(host)) % nb
-    s_ref = sets[last % len(host)]
+    b = (steps - 1) % nb
+    s_ref = sets[b % len(host)]
     n = int(cnt_h[b][0])
     same = (n == s_ref.rows and
             torch.equal(y_h[b][:n], s_ref.y[:n].cpu()) and
