@@ -71,7 +71,8 @@ def parse_args():
                    help="profiler target instead of the bench: run one layer call of the "
                         "density sweep's workload --steps times and print its CUDA-event "
                         "times; 'sweep:D' the sparse conv at mask density D (compaction and "
-                        "mapping done before), 'sweep-dense' the dense layer")
+                        "mapping done before), 'sweep-dense' the dense layer, 'mask-score' "
+                        "the mask-score update on the encoder outputs (K = 10, 41,920 x 64)")
     return p.parse_args()
 
 
@@ -1229,9 +1230,10 @@ def run_configs(torch, hc, dev, stream, cpu_budget_s=3.0):
 
 
 def run_case(args):
-    """One layer call of the density sweep's workload (V = 10475, L = 9,
-    B = 64, 128 -> 128), args.steps times in a row, each timed with CUDA
-    events: a small, fixed launch sequence for a profiler to capture."""
+    """One call, args.steps times in a row, each timed with CUDA events: a
+    small, fixed launch sequence for a profiler to capture. A layer of the
+    density sweep's workload (V = 10475, L = 9, B = 64, 128 -> 128), or the
+    mask-score update on the encoder outputs."""
     import torch
 
     from paper_2608_09388_gb300 import build as hc_build
@@ -1248,7 +1250,15 @@ def run_case(args):
     spiral = torch.from_numpy(w.spiral).to(dev)
     Wt = torch.from_numpy(ly.W.view(np.int16)).view(torch.bfloat16).to(dev)
     bias = torch.from_numpy(ly.b).to(dev)
-    if args.case == "sweep-dense":
+    if args.case == "mask-score":
+        g = torch.Generator(device=dev)
+        g.manual_seed(1234 + 64)
+        O = torch.randn((10, 64 * 655, 64), generator=g, device=dev).to(torch.bfloat16)
+        a_in = torch.zeros(10, device=dev)
+        a_out = torch.empty(10, device=dev)
+        fn = lambda: hc.hc_mask_score_update(O, a_in, a_out, None, stream)  # noqa: E731
+        rows = 64 * 655
+    elif args.case == "sweep-dense":
         yd = torch.empty((B, V, ly.C_out), dtype=torch.bfloat16, device=dev)
         fn = lambda: hc.hc_spiral_conv_fwd(x, spiral, Wt, bias, ly.act, yd, stream)  # noqa: E731
         rows = B * V
@@ -1271,7 +1281,7 @@ def run_case(args):
         fn = lambda: hc.hc_sparse_conv_rulebook_fwd(x, rb, count, Wt, bias, ly.act, y,  # noqa: E731
                                                     stream=stream)
     else:
-        raise SystemExit(f"--case {args.case}: expected sweep:D or sweep-dense")
+        raise SystemExit(f"--case {args.case}: expected sweep:D, sweep-dense or mask-score")
     times = []
     for _ in range(args.steps):
         a = torch.cuda.Event(enable_timing=True)
