@@ -253,11 +253,14 @@ __global__ void __launch_bounds__(kThreads)
 // (s+1)*kMapPortion); every tap lookup row_of[b, u] of Eq. 4 is a
 // shared-memory read. The mask, the ranks and the first spiral entries of
 // the portion's active vertices do not depend on the count pass and are
-// read before waiting on it; after the wait only the tile counts before the
-// frame are read (frame offset = those counts + the active bytes of the
-// frame's own 4096-byte tile before b*V, counted here). Shared memory stays
-// small (6 bytes per 16 vertices + 2 per portion vertex) so that the conv
-// that follows can start on the same SMs.
+// read before waiting on it (the count pass lets this one start only after
+// its own wait, so whatever wrote the mask and the spiral table before it
+// has finished); after the wait only the tile counts before the frame are
+// read (frame offset = those counts + the active bytes of the frame's own
+// 4096-byte tile before b*V, counted here). Shared memory stays small (6
+// bytes per 16 vertices + 2 per portion vertex); it is the registers (a
+// CTA's 12k beside a conv CTA's 59k) that keep the conv that follows off an
+// SM until the SM's mapping CTAs have finished.
 constexpr int kMapThreads = 256;
 constexpr int kMapPortion = 1024;
 constexpr int kMapMaxV = 65535;
